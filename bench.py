@@ -1,0 +1,405 @@
+"""Benchmark of the acceptance-aware loss hot path on GB300.
+
+One step = one pass of the whole path over one synthetic batch of the V = 128256
+workload (N = 8192 windows = 4 sequences x 2048 positions, K = 7, bf16 logits,
+Zipf target, draft = target + N(0, 1)):
+  aal_loss_fwd     EAL + WTV forward, weights 0.5 / 0.5, T = 1   (reads draft + target)
+  aal_loss_bwd     gradient w.r.t. the draft logits              (reads both, writes bf16)
+  aal_accept_reward  simulated greedy-verification reward and group advantages
+                     (16 rollouts x 256 windows per group)       (reads both)
+The metric is algorithmic HBM bytes per second (2 + 3 + 2 logit passes of R = N K rows
+of V bf16 values per step) and logit rows per second.
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+Prints one JSON line (rank 0).  N > 1 runs under torchrun: each rank processes its own
+batch (windows are independent, no collective on the data path), weak scaling.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+WORKLOAD = "v128k"
+MODE_T, W_G, W_S = 1.0, 0.5, 0.5
+WPR, RPG = 256, 16           # reward: windows per rollout, rollouts per group
+KERNELS_PER_STEP = 5         # row stats + window combine, backward, reward rows + groups
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=60)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def measured_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def algo_bytes(N, K, V, elt=2):
+    R = N * K
+    row = V * elt
+    return dict(fwd=2 * R * row, bwd=3 * R * row, reward=2 * R * row)
+
+
+# ----------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=self.file, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.file.flush()
+        self.file.seek(0)
+        rows = [l.strip().split(", ") for l in self.file.read().splitlines() if l.strip()]
+        os.unlink(self.file.name)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            if len(r) < 9:
+                continue
+            try:
+                sm.append(float(r[1]))
+                mx.append(float(r[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, r[5:9]):
+                if v.strip() == "Active":
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+# ----------------------------------------------------------------------------- our arm
+
+def run_ours(args, ws_count, rank, local):
+    import paper_2609_24150_gb300 as aal
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream()
+    target, draft, _ = synth.make_logits(WORKLOAD, seed=rank, device=dev)
+    N, K, V = draft.shape
+    grad = torch.empty_like(draft)
+    prob = aal.loss_problem(draft, aal.AAL_BOTH, MODE_T, W_G, W_S)
+    ws = torch.empty(aal.aal_workspace_size(prob), dtype=torch.uint8, device=dev)
+    loss = torch.empty(1, dtype=torch.float32, device=dev)
+    rprob = aal.reward_problem(draft, aal.AAL_GREEDY, 1.0, 5.0, 0, rank * N, WPR, RPG)
+    rws = torch.empty(aal.aal_reward_workspace_size(rprob), dtype=torch.uint8, device=dev)
+    tau = torch.empty(N, dtype=torch.int32, device=dev)
+    nroll = N // WPR
+    rl = torch.empty(nroll, dtype=torch.float32, device=dev)
+    adv = torch.empty(nroll, dtype=torch.float32, device=dev)
+
+    def step(d, t):
+        aal.aal_loss_fwd(prob, d, t, None, ws, loss, None, stream)
+        aal.aal_loss_bwd(prob, d, t, None, ws, 1.0, grad, stream)
+        aal.aal_accept_reward(rprob, d, t, None, rws, tau, None, rl, adv, stream)
+
+    for _ in range(args.warmup):
+        step(draft, target)
+    torch.cuda.synchronize()
+    assert aal.aal_check_device_status(ws) == aal.AAL_OK
+
+    # timed region: per-call events on the launching stream
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    if ws_count > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for i in range(args.steps):
+        ev[i][0].record(stream)
+        aal.aal_loss_fwd(prob, draft, target, None, ws, loss, None, stream)
+        ev[i][1].record(stream)
+        aal.aal_loss_bwd(prob, draft, target, None, ws, 1.0, grad, stream)
+        ev[i][2].record(stream)
+        aal.aal_accept_reward(rprob, draft, target, None, rws, tau, None, rl, adv, stream)
+        ev[i][3].record(stream)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    if ws_count > 1:
+        torch.distributed.barrier()
+    clk = clocks.stop()
+    ms_total = t_start.elapsed_time(t_end)
+    if ws_count > 1:
+        tt = torch.tensor([ms_total], dtype=torch.float64, device=dev)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        ms_total = float(tt.item())
+    ms_step = ms_total / args.steps
+    per = {"fwd": 0.0, "bwd": 0.0, "reward": 0.0}
+    for i in range(args.steps):
+        per["fwd"] += ev[i][0].elapsed_time(ev[i][1])
+        per["bwd"] += ev[i][1].elapsed_time(ev[i][2])
+        per["reward"] += ev[i][2].elapsed_time(ev[i][3])
+    per = {k: v / args.steps for k, v in per.items()}
+    assert aal.aal_check_device_status(ws) == aal.AAL_OK
+    loss_val = float(loss.item())
+
+    b = algo_bytes(N, K, V)
+    step_bytes = sum(b.values())
+    R = N * K
+    value = step_bytes * ws_count / (ms_step * 1e-3) / 1e9
+    peak, peak_src = measured_peak()
+
+    # dominant kernel: the call with the largest share; its algorithmic bytes / its time
+    dom = max(per, key=per.get)
+    dom_kernel = {"fwd": "rowstats (aal_loss_fwd)", "bwd": "backward_kernel (aal_loss_bwd)",
+                  "reward": "reward_rows (aal_accept_reward)"}[dom]
+    achieved = b[dom] / (per[dom] * 1e-3) / 1e9
+    traffic = recorded_traffic(dom)
+
+    res = {
+        "metric": "fused EAL/WTV fwd+bwd + acceptance reward: algorithmic HBM GB/s at V=128256",
+        "value": round(value, 1),
+        "unit": "GB/s",
+        "n_gpus": ws_count,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_step, 4),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded Zipf target logits over a random vocabulary permutation, "
+                "draft = target + N(0,1)); no model weights",
+        "config": {"workload": f"{WORKLOAD}: N=8192 windows (B=4 x T=2048), K=7, V=128256 bf16; "
+                               "EAL+WTV 0.5/0.5 at T=1 fwd+bwd, greedy reward 16 rollouts x 256 windows",
+                   "N": N, "K": K, "V": V, "rows_per_step": R,
+                   "bytes_per_step": step_bytes, "l2": "inputs larger than L2 (14.7 GB per tensor)",
+                   "parallelism": f"replicas x{ws_count} (independent windows)"},
+        "rows_per_s": round(R * ws_count / (ms_step * 1e-3), 1),
+        "breakdown_ms": {k: round(v, 4) for k, v in per.items()},
+        "breakdown_gbs": {k: round(b[k] / (per[k] * 1e-3) / 1e9, 1) for k in per},
+        "fwd_bwd_gbs": round((b["fwd"] + b["bwd"]) / ((per["fwd"] + per["bwd"]) * 1e-3) / 1e9, 1),
+        "frac_of_peak": round(value / ws_count / peak, 4),
+        "loss": loss_val,
+        "gpu_launches": KERNELS_PER_STEP * args.steps,
+        "roofline": {"bound": "hbm", "kernel": dom_kernel, "achieved": round(achieved, 1),
+                     "peak": peak, "peak_source": peak_src, "unit": "GB/s",
+                     "frac": round(achieved / peak, 4), "traffic": traffic,
+                     "algorithmic_bytes": b[dom]},
+        "clocks": clk,
+    }
+
+    if rank == 0:
+        res["e2e"] = run_e2e(args, aal, prob, rprob, draft, target, grad, ws, loss, rws, tau, rl, adv,
+                             stream, step_bytes)
+    if rank == 0 and ws_count == 1 and not args.no_cpu_baseline:
+        res["cpu_baseline"] = cpu_baseline(draft, target, args.cpu_seconds)
+    return res
+
+
+def host_memory_bytes():
+    avail = None
+    try:
+        with open("/proc/meminfo") as f:
+            for line in f:
+                if line.startswith("MemAvailable:"):
+                    avail = int(line.split()[1]) * 1024
+    except OSError:
+        pass
+    for cg in ("/sys/fs/cgroup/memory.max", "/sys/fs/cgroup/memory/memory.limit_in_bytes"):
+        try:
+            with open(cg) as f:
+                v = f.read().strip()
+            if v.isdigit():
+                lim = int(v)
+                avail = lim if avail is None else min(avail, lim)
+        except OSError:
+            pass
+    return avail
+
+
+def run_e2e(args, aal, prob, rprob, draft, target, grad, ws, loss, rws, tau, rl, adv, stream, step_bytes):
+    """Same step through the public API with inputs in pinned host memory: H2D of both logit
+    tensors and D2H of the loss and advantages are inside the timed region every step."""
+    need = 2 * draft.numel() * draft.element_size()
+    avail = host_memory_bytes()
+    if avail is not None and need > avail // 3:
+        return {"value": None, "unit": "GB/s", "skipped": f"pinned inputs need {need / 1e9:.1f} GB, "
+                f"host has {avail / 1e9:.1f} GB available"}
+    d_h = torch.empty(draft.shape, dtype=draft.dtype, pin_memory=True)
+    t_h = torch.empty(target.shape, dtype=target.dtype, pin_memory=True)
+    d_h.copy_(draft)
+    t_h.copy_(target)
+    loss_h = torch.empty(1, dtype=torch.float32, pin_memory=True)
+    adv_h = torch.empty(adv.shape, dtype=torch.float32, pin_memory=True)
+    rl_h = torch.empty(rl.shape, dtype=torch.float32, pin_memory=True)
+
+    def e2e_step():
+        draft.copy_(d_h, non_blocking=True)
+        target.copy_(t_h, non_blocking=True)
+        aal.aal_loss_fwd(prob, draft, target, None, ws, loss, None, stream)
+        aal.aal_loss_bwd(prob, draft, target, None, ws, 1.0, grad, stream)
+        aal.aal_accept_reward(rprob, draft, target, None, rws, tau, None, rl, adv, stream)
+        loss_h.copy_(loss, non_blocking=True)
+        adv_h.copy_(adv, non_blocking=True)
+        rl_h.copy_(rl, non_blocking=True)
+
+    e2e_step()
+    torch.cuda.synchronize()
+    a = torch.cuda.Event(enable_timing=True)
+    z = torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(args.e2e_steps):
+        e2e_step()
+    z.record(stream)
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(z) / args.e2e_steps
+    del d_h, t_h
+    return {"value": round(step_bytes / (ms * 1e-3) / 1e9, 1), "unit": "GB/s", "ms_per_step": round(ms, 3),
+            "h2d_bytes_per_step": need, "d2h_bytes_per_step": 4 + 2 * 4 * adv.numel(),
+            "steps": args.e2e_steps}
+
+
+# ----------------------------------------------------------------------------- oracle timings
+
+def _oracle_step(target_h, draft_h, row_offset):
+    import oracle
+    oracle.loss_forward(target_h, draft_h, None, oracle.MODE_BOTH, MODE_T, W_G, W_S, n_windows_total=8192)
+    oracle.loss_backward(target_h, draft_h, None, oracle.MODE_BOTH, MODE_T, W_G, W_S, 1.0, n_windows_total=8192)
+    oracle.accept_reward(target_h, draft_h, None, 1, 1.0, 0, row_offset)
+
+
+def cpu_baseline(draft, target, seconds):
+    """The fp64 oracle on the host cores over a bounded sample of the same workload bytes."""
+    K, V = draft.shape[1], draft.shape[2]
+    per_window = 2 * K * V * 2 + 3 * K * V * 2 + 2 * K * V * 2
+    t0 = time.perf_counter()
+    _oracle_step(target[:1].cpu(), draft[:1].cpu(), 0)
+    one = time.perf_counter() - t0
+    n = int(max(1, min(draft.shape[0], seconds / max(one, 1e-3))))
+    t_h, d_h = target[:n].cpu(), draft[:n].cpu()
+    t0 = time.perf_counter()
+    _oracle_step(t_h, d_h, 0)
+    dt = time.perf_counter() - t0
+    return {"value": round(n * per_window / dt / 1e9, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+            "sample": f"first {n} of 8192 windows ({n * K} rows x V={V}) of the same bf16 batch, "
+                      f"{dt:.1f} s; numpy fp64 on one thread of {os.cpu_count()} host cores",
+            "rows_per_s": round(n * K / dt, 2)}
+
+
+def run_reference(args, ws_count, rank):
+    """--impl reference: the oracle, as it stands, timed on the host cores per step."""
+    if rank != 0:
+        return None
+    n = 16
+    target, draft, _ = synth.make_logits(WORKLOAD, seed=0, device="cpu", n_windows=n)
+    K, V = draft.shape[1], draft.shape[2]
+    per_window = n * (2 * K * V * 2 + 3 * K * V * 2 + 2 * K * V * 2)
+    for _ in range(args.warmup):
+        _oracle_step(target, draft, 0)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        _oracle_step(target, draft, 0)
+    dt = (time.perf_counter() - t0) / args.steps
+    value = per_window / dt / 1e9
+    return {"impl": "reference", "metric": "fused EAL/WTV fwd+bwd + acceptance reward: algorithmic HBM GB/s at V=128256",
+            "value": round(value, 4), "unit": "GB/s", "n_gpus": ws_count, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(dt * 1e3, 3), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": f"{WORKLOAD}: N=8192, K=7, V=128256 bf16 (each step: a {n}-window sample)"},
+            "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+                             "sample": f"{n} windows ({n * K} rows x V={V}) per step, numpy fp64, one thread"},
+            "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    args = parse()
+    ws_count, rank, local = dist_env()
+    if ws_count > 1:
+        backend = "nccl" if args.impl == "ours" else "gloo"
+        torch.distributed.init_process_group(backend)
+    if args.impl == "reference":
+        res = run_reference(args, ws_count, rank)
+    else:
+        res = run_ours(args, ws_count, rank, local)
+    if rank == 0 and res is not None:
+        print(json.dumps(res), flush=True)
+    if ws_count > 1:
+        torch.distributed.destroy_process_group()
+
+
+def recorded_traffic(which):
+    """DRAM bytes per launch from the committed ncu summary, if the kernel is unchanged since."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f).get(which)
+    except (OSError, ValueError):
+        return None
+    if not rec:
+        return None
+    src = os.path.join(ROOT, "paper_2609_24150_gb300", "csrc", rec["source"])
+    try:
+        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    except OSError:
+        return None
+    return rec["dram_bytes_per_launch"] if sha == rec["source_sha256_16"] else None
+
+
+if __name__ == "__main__":
+    main()

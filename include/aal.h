@@ -1,0 +1,176 @@
+/*
+ * aal.h -- acceptance-aware draft-training losses on one GB300 (sm_103a).
+ *
+ * C ABI of libaal.so.  It computes, over full-vocabulary draft and target logits:
+ *   - the expected-accepted-length loss under greedy verification (EAL) and the
+ *     window total-variation loss under sampling verification (WTV), forward and
+ *     backward with respect to the draft logits;
+ *   - the simulated acceptance length, debiased reward and group-normalised
+ *     advantage of the GRPO stage.
+ * Paper: "Acceptance-Aware Draft Model Training for Speculative Decoding",
+ * Sec. 2.3 (acceptance under greedy / sampling verification, Eqs. acc_greedy,
+ * acc_sample), Sec. 3.1 (speculative window, Eq. eal_generic), Sec. 3.2 (Eq.
+ * loss_eal), Sec. 3.3 (Eqs. rejection_rate, eal_tv, loss_tv), Sec. 3.4 (GRPO
+ * reward, Eqs. debiased_reward, advantage).
+ *
+ * Common conventions
+ *   Layout.  Logits are row-major [N windows][K depths][V vocabulary], rows
+ *     contiguous, element type fp32 or bf16; depth k of window n is position
+ *     t + k of the window that starts at t.  Base pointers must be 16-byte
+ *     aligned (any V is accepted; rows whose byte length is not a multiple of
+ *     16 take a slower path).
+ *   Memory.  Every pointer is a DEVICE pointer owned by the caller, except the
+ *     aal_problem / aal_reward_problem structs, which are host memory read
+ *     during the call only.  The library allocates nothing and keeps no state
+ *     between calls; the workspace carries the forward's results to the
+ *     backward.
+ *   Streams.  `stream` is a cudaStream_t (NULL = legacy default stream).  All
+ *     calls are asynchronous on it; outputs are valid once the stream reaches
+ *     the call.  Calls that share a workspace must be ordered on one stream.
+ *   Errors.  Arguments are checked before anything is launched; a failed check
+ *     returns AAL_ERR_INVALID_ARG / AAL_ERR_UNSUPPORTED / AAL_ERR_WORKSPACE and
+ *     launches nothing.  A launch failure returns AAL_ERR_CUDA.  Device-side
+ *     errors (a bounded wait that ran out) are recorded in the workspace and
+ *     reported by aal_check_device_status().  No call aborts the process.
+ *   Gradients.  The target is frozen (Sec. 3.2, 3.3); only the draft gets a
+ *     gradient.
+ */
+#ifndef AAL_H_
+#define AAL_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define AAL_API __attribute__((visibility("default")))
+#else
+#define AAL_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  AAL_OK = 0,
+  AAL_ERR_INVALID_ARG = 1,  /* a NULL, misaligned or out-of-range argument */
+  AAL_ERR_UNSUPPORTED = 2,  /* valid request this build does not handle (e.g. K > 8) */
+  AAL_ERR_WORKSPACE = 3,    /* workspace missing or smaller than aal_*_workspace_size() */
+  AAL_ERR_CUDA = 4,         /* a CUDA runtime call or kernel launch failed */
+  AAL_ERR_TIMEOUT = 5       /* a device-side bounded wait ran out (see aal_check_device_status) */
+} aal_status;
+
+typedef enum { AAL_F32 = 0, AAL_BF16 = 1 } aal_dtype;
+
+/* Which loss terms to compute.  GREEDY: L_EAL (Eq. loss_eal); SAMPLING: L_WTV
+ * (Eq. loss_tv); BOTH: w_greedy * L_EAL + w_sampling * L_WTV. */
+typedef enum { AAL_GREEDY = 1, AAL_SAMPLING = 2, AAL_BOTH = 3 } aal_mode;
+
+#define AAL_MAX_K 8
+
+/* One loss problem (host struct).
+ *   N, K, V      windows, window size gamma (1..AAL_MAX_K), vocabulary size (>= 1); N may be 0.
+ *   dtype        aal_dtype of draft, target and the gradient.
+ *   mode         aal_mode.
+ *   temperature  T of the sampling term (Sec. 2.3: p~ ~ exp(log p / T)); must be finite
+ *                and > 0 when mode includes SAMPLING.  The greedy acceptance
+ *                a = q(x*) (Eq. acc_greedy) always uses the unscaled draft, so T is
+ *                ignored (and may be 0) for mode GREEDY.
+ *   w_greedy, w_sampling  weights of the two terms (used by every mode; a term the mode
+ *                does not select is not computed).  Must be finite. */
+typedef struct {
+  int64_t N, K, V;
+  int32_t dtype;
+  int32_t mode;
+  float temperature;
+  float w_greedy;
+  float w_sampling;
+  int32_t reserved; /* must be 0 */
+} aal_problem;
+
+/* Bytes of device workspace a loss problem needs (host-only, launches nothing). */
+AAL_API aal_status aal_workspace_size(const aal_problem* prob, size_t* bytes);
+
+/* Forward of the loss (Sec. 3.2 Eq. loss_eal, Sec. 3.3 Eq. loss_tv):
+ *   L = -(1/|W|) sum_n [ w_g sum_{k=1}^{K_n} prod_{j<k} a^g_{n,j}
+ *                       + w_s sum_{k=1}^{K_n} prod_{j<k} a^s_{n,j} ]
+ * with a^g = q(x*) (Eq. acc_greedy, x* = target argmax, lowest index on ties) and
+ * a^s = sum_v min(p~, q~) = 1 - TV(p~, q~) (Eqs. acc_sample, rejection_rate).
+ *   draft, target  [N][K][V] logits of the draft (z_q) and the target (z_p).
+ *   mask           [N][K] uint8, nonzero = valid position, or NULL (all valid).  A
+ *                  window stops at its first invalid position (K_n = number of leading
+ *                  valid depths) and belongs to W iff K_n >= 1.  |W| = 0 gives L = 0.
+ *   workspace      device buffer of at least aal_workspace_size() bytes, 256-byte
+ *                  aligned; holds per-row statistics for aal_loss_bwd.
+ *   loss           device float[1]: L.
+ *   eal            device float[N][2] or NULL: per-window expected accepted lengths
+ *                  (greedy, sampling); 0 for a term not computed or a window not in W. */
+AAL_API aal_status aal_loss_fwd(const aal_problem* prob, const void* draft, const void* target,
+                        const uint8_t* mask, void* workspace, size_t workspace_bytes,
+                        float* loss, float* eal, void* stream);
+
+/* Backward of the loss: grad_draft = dloss * dL/dz_q, [N][K][V] in the problem's dtype.
+ * Must follow aal_loss_fwd on the same stream with the same problem, inputs, mask
+ * and workspace.  dloss is the upstream gradient of L (a host scalar).  Rows of
+ * positions outside every window's valid prefix get exact zeros.  The gradient of
+ * the sampling term uses the subgradient that follows p~ at ties p~_v = q~_v. */
+AAL_API aal_status aal_loss_bwd(const aal_problem* prob, const void* draft, const void* target,
+                        const uint8_t* mask, const void* workspace, size_t workspace_bytes,
+                        float dloss, void* grad_draft, void* stream);
+
+/* Simulated acceptance reward of the GRPO stage (Sec. 3.4).
+ *   N, K, V, dtype       as for the loss; K is the window size gamma (1..AAL_MAX_K).
+ *   mode                 AAL_GREEDY: draft token S_k = argmax z_q is accepted iff it
+ *                        equals x*_k = argmax z_p (simulated greedy verification).
+ *                        AAL_SAMPLING: S_k is accepted iff u < min(1, p~(S_k)/q~(S_k))
+ *                        (Sec. 2.3) with u = Philox4x32-10 uniform keyed by
+ *                        (seed; window row_offset + n, depth k).
+ *   temperature          T for AAL_SAMPLING (finite, > 0).
+ *   seed, row_offset     Philox key and the global index of window 0 (so a batch can be
+ *                        streamed in pieces with the same draws).
+ *   windows_per_rollout  consecutive windows forming one rollout (>= 1).
+ *   rollouts_per_group   consecutive rollouts forming one advantage group (>= 1);
+ *                        N must be a multiple of windows_per_rollout * rollouts_per_group.
+ *   adv_clip             C_A of Eq. advantage (> 0). */
+typedef struct {
+  int64_t N, K, V;
+  int32_t dtype;
+  int32_t mode;
+  float temperature;
+  float adv_clip;
+  uint64_t seed;
+  int64_t row_offset;
+  int64_t windows_per_rollout;
+  int64_t rollouts_per_group;
+} aal_reward_problem;
+
+AAL_API aal_status aal_reward_workspace_size(const aal_reward_problem* prob, size_t* bytes);
+
+/* tau^pi = sum_{k=1}^{K} prod_{j<=k} 1[S_j accepted] per window for the draft (and the
+ * reference draft), R = tau^theta - tau^ref (Eq. debiased_reward; R = tau^theta when
+ * ref_draft is NULL), rollout length = mean R over the rollout's windows, and
+ * advantage A = clip((x - mean_g)/(std_g + 1e-6), -C_A, C_A) over each group of
+ * rollouts with the population std (Eq. advantage).
+ *   draft, target, ref_draft  [N][K][V] logits; ref_draft may be NULL.
+ *   tau, tau_ref              device int32[N]; tau_ref may be NULL (ignored without ref).
+ *   rollout_len, advantage    device float[N / windows_per_rollout]. */
+AAL_API aal_status aal_accept_reward(const aal_reward_problem* prob, const void* draft,
+                             const void* target, const void* ref_draft, void* workspace,
+                             size_t workspace_bytes, int32_t* tau, int32_t* tau_ref,
+                             float* rollout_len, float* advantage, void* stream);
+
+/* Synchronises `stream`, reads the device status word of a loss or reward workspace,
+ * clears it, and returns AAL_OK or the recorded device error (AAL_ERR_TIMEOUT). */
+AAL_API aal_status aal_check_device_status(void* workspace, void* stream);
+
+/* Static description of a status code; never NULL. */
+AAL_API const char* aal_status_string(aal_status status);
+
+/* Version of the ABI described by this header (major * 10000 + minor * 100 + patch). */
+AAL_API int32_t aal_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* AAL_H_ */

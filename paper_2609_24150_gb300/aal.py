@@ -1,0 +1,210 @@
+"""ctypes binding of libaal.so: same names as the C ABI, argument marshalling only."""
+
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional
+
+import torch
+
+AAL_OK = 0
+AAL_ERR_INVALID_ARG = 1
+AAL_ERR_UNSUPPORTED = 2
+AAL_ERR_WORKSPACE = 3
+AAL_ERR_CUDA = 4
+AAL_ERR_TIMEOUT = 5
+
+AAL_F32 = 0
+AAL_BF16 = 1
+
+AAL_GREEDY = 1
+AAL_SAMPLING = 2
+AAL_BOTH = 3
+
+AAL_MAX_K = 8
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+
+
+def library_path() -> str:
+    return os.path.join(_HERE, "libaal.so")
+
+
+class AalProblem(ctypes.Structure):
+    """Mirror of ``aal_problem``."""
+    _fields_ = [("N", ctypes.c_int64), ("K", ctypes.c_int64), ("V", ctypes.c_int64),
+                ("dtype", ctypes.c_int32), ("mode", ctypes.c_int32),
+                ("temperature", ctypes.c_float), ("w_greedy", ctypes.c_float),
+                ("w_sampling", ctypes.c_float), ("reserved", ctypes.c_int32)]
+
+
+class AalRewardProblem(ctypes.Structure):
+    """Mirror of ``aal_reward_problem``."""
+    _fields_ = [("N", ctypes.c_int64), ("K", ctypes.c_int64), ("V", ctypes.c_int64),
+                ("dtype", ctypes.c_int32), ("mode", ctypes.c_int32),
+                ("temperature", ctypes.c_float), ("adv_clip", ctypes.c_float),
+                ("seed", ctypes.c_uint64), ("row_offset", ctypes.c_int64),
+                ("windows_per_rollout", ctypes.c_int64), ("rollouts_per_group", ctypes.c_int64)]
+
+
+class AalError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        self.code = code
+        super().__init__(f"{where}: {aal_status_string(code)}")
+
+
+_LIB = None
+
+
+def library() -> ctypes.CDLL:
+    """Load libaal.so once; raise ImportError if it has not been built."""
+    global _LIB
+    if _LIB is not None:
+        return _LIB
+    path = library_path()
+    if not os.path.exists(path):
+        raise ImportError(f"{path} is missing: build it with `python -m paper_2609_24150_gb300.build`")
+    lib = ctypes.CDLL(path)
+    vp, sz = ctypes.c_void_p, ctypes.c_size_t
+    P = ctypes.POINTER(AalProblem)
+    RP = ctypes.POINTER(AalRewardProblem)
+    lib.aal_workspace_size.argtypes = [P, ctypes.POINTER(sz)]
+    lib.aal_reward_workspace_size.argtypes = [RP, ctypes.POINTER(sz)]
+    lib.aal_loss_fwd.argtypes = [P, vp, vp, vp, vp, sz, vp, vp, vp]
+    lib.aal_loss_bwd.argtypes = [P, vp, vp, vp, vp, sz, ctypes.c_float, vp, vp]
+    lib.aal_accept_reward.argtypes = [RP, vp, vp, vp, vp, sz, vp, vp, vp, vp, vp]
+    lib.aal_check_device_status.argtypes = [vp, vp]
+    lib.aal_status_string.argtypes = [ctypes.c_int]
+    lib.aal_status_string.restype = ctypes.c_char_p
+    lib.aal_abi_version.argtypes = []
+    lib.aal_abi_version.restype = ctypes.c_int32
+    for f in ("aal_workspace_size", "aal_reward_workspace_size", "aal_loss_fwd", "aal_loss_bwd",
+              "aal_accept_reward", "aal_check_device_status"):
+        getattr(lib, f).restype = ctypes.c_int
+    _LIB = lib
+    return lib
+
+
+# -------------------------------------------------------------------------- marshalling
+
+_DTYPES = {torch.float32: AAL_F32, torch.bfloat16: AAL_BF16}
+
+
+def _ptr(x, what: str, dtype=None, numel=None) -> Optional[int]:
+    """Device address of a CUDA tensor (or a raw int address); None stays NULL."""
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    if not isinstance(x, torch.Tensor):
+        raise TypeError(f"{what}: expected a CUDA tensor or an address, got {type(x)}")
+    if not x.is_cuda:
+        raise ValueError(f"{what}: tensor must be on a CUDA device (libaal has no CPU path)")
+    if not x.is_contiguous():
+        raise ValueError(f"{what}: tensor must be contiguous")
+    if dtype is not None and x.dtype != dtype:
+        raise ValueError(f"{what}: expected {dtype}, got {x.dtype}")
+    if numel is not None and x.numel() < numel:
+        raise ValueError(f"{what}: needs at least {numel} elements, has {x.numel()}")
+    return x.data_ptr()
+
+
+def _nbytes(x) -> int:
+    return x.numel() * x.element_size() if isinstance(x, torch.Tensor) else 0
+
+
+def _stream(stream) -> Optional[int]:
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, torch.cuda.Stream):
+        return stream.cuda_stream
+    return int(stream)
+
+
+def _check(code: int, where: str):
+    if code != AAL_OK:
+        raise AalError(code, where)
+
+
+def loss_problem(draft: torch.Tensor, mode: int, temperature: float = 1.0, w_greedy: float = 1.0,
+                 w_sampling: float = 1.0) -> AalProblem:
+    """Problem struct for [N][K][V] logits."""
+    if draft.dim() != 3:
+        raise ValueError("logits must be [N][K][V]")
+    N, K, V = draft.shape
+    if draft.dtype not in _DTYPES:
+        raise ValueError(f"unsupported dtype {draft.dtype}")
+    return AalProblem(N, K, V, _DTYPES[draft.dtype], mode, temperature, w_greedy, w_sampling, 0)
+
+
+def reward_problem(draft: torch.Tensor, mode: int, temperature: float = 1.0, adv_clip: float = 5.0,
+                   seed: int = 0, row_offset: int = 0, windows_per_rollout: int = 1,
+                   rollouts_per_group: int = 1) -> AalRewardProblem:
+    if draft.dim() != 3:
+        raise ValueError("logits must be [N][K][V]")
+    N, K, V = draft.shape
+    return AalRewardProblem(N, K, V, _DTYPES[draft.dtype], mode, temperature, adv_clip, seed,
+                            row_offset, windows_per_rollout, rollouts_per_group)
+
+
+# -------------------------------------------------------------------------- the C ABI
+
+def aal_status_string(code: int) -> str:
+    return library().aal_status_string(int(code)).decode()
+
+
+def aal_abi_version() -> int:
+    return int(library().aal_abi_version())
+
+
+def aal_workspace_size(problem: AalProblem) -> int:
+    out = ctypes.c_size_t(0)
+    _check(library().aal_workspace_size(ctypes.byref(problem), ctypes.byref(out)), "aal_workspace_size")
+    return out.value
+
+
+def aal_reward_workspace_size(problem: AalRewardProblem) -> int:
+    out = ctypes.c_size_t(0)
+    _check(library().aal_reward_workspace_size(ctypes.byref(problem), ctypes.byref(out)),
+           "aal_reward_workspace_size")
+    return out.value
+
+
+def aal_loss_fwd(problem: AalProblem, draft, target, mask, workspace, loss, eal=None, stream=None):
+    """Forward of the EAL / WTV loss; writes loss[0] (and eal[N][2] when given)."""
+    N = problem.N
+    code = library().aal_loss_fwd(
+        ctypes.byref(problem), _ptr(draft, "draft"), _ptr(target, "target"),
+        _ptr(mask, "mask", torch.uint8, N * problem.K), _ptr(workspace, "workspace"),
+        _nbytes(workspace), _ptr(loss, "loss", torch.float32, 1),
+        _ptr(eal, "eal", torch.float32, 2 * N), _stream(stream))
+    _check(code, "aal_loss_fwd")
+
+
+def aal_loss_bwd(problem: AalProblem, draft, target, mask, workspace, dloss: float, grad, stream=None):
+    """Backward: grad = dloss * dL/d draft, in the draft's dtype."""
+    code = library().aal_loss_bwd(
+        ctypes.byref(problem), _ptr(draft, "draft"), _ptr(target, "target"),
+        _ptr(mask, "mask", torch.uint8), _ptr(workspace, "workspace"), _nbytes(workspace),
+        float(dloss), _ptr(grad, "grad"), _stream(stream))
+    _check(code, "aal_loss_bwd")
+
+
+def aal_accept_reward(problem: AalRewardProblem, draft, target, ref_draft, workspace, tau,
+                      tau_ref, rollout_len, advantage, stream=None):
+    """Simulated acceptance lengths, debiased rewards, rollout lengths and advantages."""
+    N = problem.N
+    nroll = N // max(1, problem.windows_per_rollout)
+    code = library().aal_accept_reward(
+        ctypes.byref(problem), _ptr(draft, "draft"), _ptr(target, "target"),
+        _ptr(ref_draft, "ref_draft"), _ptr(workspace, "workspace"), _nbytes(workspace),
+        _ptr(tau, "tau", torch.int32, N), _ptr(tau_ref, "tau_ref", torch.int32, N),
+        _ptr(rollout_len, "rollout_len", torch.float32, nroll),
+        _ptr(advantage, "advantage", torch.float32, nroll), _stream(stream))
+    _check(code, "aal_accept_reward")
+
+
+def aal_check_device_status(workspace, stream=None) -> int:
+    """Synchronise and return (and clear) the workspace's device status code."""
+    return int(library().aal_check_device_status(_ptr(workspace, "workspace"), _stream(stream)))

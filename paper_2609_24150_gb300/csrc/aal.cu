@@ -1,0 +1,230 @@
+// C ABI of libaal (include/aal.h): argument checks, workspace layout, launches.
+#include <math.h>
+#include <string.h>
+
+#include "aal_internal.cuh"
+
+using namespace aal;
+
+namespace {
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+aal_status check_shape(int64_t N, int64_t K, int64_t V, int32_t dtype) {
+  if (N < 0 || K < 1 || V < 1) return AAL_ERR_INVALID_ARG;
+  if (K > AAL_MAX_K) return AAL_ERR_UNSUPPORTED;
+  if (V > 0x7fffffff) return AAL_ERR_UNSUPPORTED;  // token ids are int32
+  if (dtype != AAL_F32 && dtype != AAL_BF16) return AAL_ERR_INVALID_ARG;
+  if (N > 0 && N > INT64_MAX / (K * V * 4)) return AAL_ERR_INVALID_ARG;  // element count overflow
+  return AAL_OK;
+}
+
+aal_status check_problem(const aal_problem* p) {
+  if (p == nullptr) return AAL_ERR_INVALID_ARG;
+  aal_status st = check_shape(p->N, p->K, p->V, p->dtype);
+  if (st != AAL_OK) return st;
+  if (p->mode != AAL_GREEDY && p->mode != AAL_SAMPLING && p->mode != AAL_BOTH) return AAL_ERR_INVALID_ARG;
+  if ((p->mode & AAL_SAMPLING) && !(isfinite(p->temperature) && p->temperature > 0.f)) return AAL_ERR_INVALID_ARG;
+  if (!isfinite(p->w_greedy) || !isfinite(p->w_sampling)) return AAL_ERR_INVALID_ARG;
+  if (p->reserved != 0) return AAL_ERR_INVALID_ARG;
+  return AAL_OK;
+}
+
+aal_status check_reward(const aal_reward_problem* p) {
+  if (p == nullptr) return AAL_ERR_INVALID_ARG;
+  aal_status st = check_shape(p->N, p->K, p->V, p->dtype);
+  if (st != AAL_OK) return st;
+  if (p->mode != AAL_GREEDY && p->mode != AAL_SAMPLING) return AAL_ERR_INVALID_ARG;
+  if (p->mode == AAL_SAMPLING && !(isfinite(p->temperature) && p->temperature > 0.f)) return AAL_ERR_INVALID_ARG;
+  if (p->windows_per_rollout < 1 || p->rollouts_per_group < 1) return AAL_ERR_INVALID_ARG;
+  if (p->windows_per_rollout > INT64_MAX / p->rollouts_per_group) return AAL_ERR_INVALID_ARG;
+  if (p->N % (p->windows_per_rollout * p->rollouts_per_group) != 0) return AAL_ERR_INVALID_ARG;
+  if (!(isfinite(p->adv_clip) && p->adv_clip > 0.f)) return AAL_ERR_INVALID_ARG;
+  if (p->row_offset < 0) return AAL_ERR_INVALID_ARG;
+  return AAL_OK;
+}
+
+aal_status cuda_status(cudaError_t e) { return e == cudaSuccess ? AAL_OK : AAL_ERR_CUDA; }
+
+}  // namespace
+
+extern "C" {
+
+int32_t aal_abi_version(void) { return 10000; }
+
+const char* aal_status_string(aal_status s) {
+  switch (s) {
+    case AAL_OK: return "AAL_OK";
+    case AAL_ERR_INVALID_ARG: return "AAL_ERR_INVALID_ARG: a NULL, misaligned or out-of-range argument";
+    case AAL_ERR_UNSUPPORTED: return "AAL_ERR_UNSUPPORTED: valid request this build does not handle";
+    case AAL_ERR_WORKSPACE: return "AAL_ERR_WORKSPACE: workspace missing or too small";
+    case AAL_ERR_CUDA: return "AAL_ERR_CUDA: a CUDA call or kernel launch failed";
+    case AAL_ERR_TIMEOUT: return "AAL_ERR_TIMEOUT: a device-side bounded wait ran out";
+  }
+  return "unknown aal_status";
+}
+
+aal_status aal_workspace_size(const aal_problem* prob, size_t* bytes) {
+  aal_status st = check_problem(prob);
+  if (st != AAL_OK) return st;
+  if (bytes == nullptr) return AAL_ERR_INVALID_ARG;
+  *bytes = loss_layout(prob->N, prob->K).total;
+  return AAL_OK;
+}
+
+aal_status aal_reward_workspace_size(const aal_reward_problem* prob, size_t* bytes) {
+  aal_status st = check_reward(prob);
+  if (st != AAL_OK) return st;
+  if (bytes == nullptr) return AAL_ERR_INVALID_ARG;
+  *bytes = reward_layout(prob->N, prob->K).total;
+  return AAL_OK;
+}
+
+aal_status aal_loss_fwd(const aal_problem* prob, const void* draft, const void* target,
+                        const uint8_t* mask, void* workspace, size_t workspace_bytes, float* loss,
+                        float* eal, void* stream) {
+  aal_status st = check_problem(prob);
+  if (st != AAL_OK) return st;
+  if (loss == nullptr || !aligned(loss, 4) || (eal != nullptr && !aligned(eal, 4))) return AAL_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (prob->N == 0) return cuda_status(cudaMemsetAsync(loss, 0, sizeof(float), s));
+  if (draft == nullptr || target == nullptr || !aligned(draft, 16) || !aligned(target, 16))
+    return AAL_ERR_INVALID_ARG;
+  const LossLayout L = loss_layout(prob->N, prob->K);
+  if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < L.total) return AAL_ERR_WORKSPACE;
+
+  const bool greedy = (prob->mode & AAL_GREEDY) != 0, sampling = (prob->mode & AAL_SAMPLING) != 0;
+  const bool bf16 = prob->dtype == AAL_BF16;
+  LossWs ws = loss_ws(workspace, L);
+  cudaError_t e = cudaMemsetAsync(ws.hdr, 0, sizeof(WsHeader), s);
+  if (e != cudaSuccess) return AAL_ERR_CUDA;
+
+  RowStatsArgs ra;
+  ra.zq = draft;
+  ra.zp = target;
+  ra.R = L.R;
+  ra.V = prob->V;
+  ra.sT = sampling ? kLog2e / prob->temperature : 0.f;
+  ra.need_p = sampling;
+  ra.need_q = sampling;
+  ra.need_q1 = greedy && !(sampling && prob->temperature == 1.0f);
+  ra.overlap = sampling;
+  ra.ws = ws;
+  int cluster = 1;
+  e = launch_rowstats(ra, bf16, s, &cluster);
+  if (e != cudaSuccess) return AAL_ERR_CUDA;
+
+  WindowArgs wa;
+  wa.mask = mask;
+  wa.N = prob->N;
+  wa.K = (int32_t)prob->K;
+  wa.cluster = cluster;
+  wa.greedy = greedy;
+  wa.sampling = sampling;
+  wa.w_greedy = prob->w_greedy;
+  wa.w_sampling = prob->w_sampling;
+  wa.loss = loss;
+  wa.eal = eal;
+  wa.ws = ws;
+  wa.nwblk = L.nwblk;
+  return cuda_status(launch_window(wa, s));
+}
+
+aal_status aal_loss_bwd(const aal_problem* prob, const void* draft, const void* target,
+                        const uint8_t* mask, const void* workspace, size_t workspace_bytes, float dloss,
+                        void* grad_draft, void* stream) {
+  (void)mask;  // the forward folded the mask into dE/da (zero outside each window's valid prefix)
+  aal_status st = check_problem(prob);
+  if (st != AAL_OK) return st;
+  if (!isfinite(dloss)) return AAL_ERR_INVALID_ARG;
+  if (prob->N == 0) return AAL_OK;
+  if (draft == nullptr || target == nullptr || grad_draft == nullptr || !aligned(draft, 16) ||
+      !aligned(target, 16) || !aligned(grad_draft, 16))
+    return AAL_ERR_INVALID_ARG;
+  const LossLayout L = loss_layout(prob->N, prob->K);
+  if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < L.total) return AAL_ERR_WORKSPACE;
+  const bool greedy = (prob->mode & AAL_GREEDY) != 0, sampling = (prob->mode & AAL_SAMPLING) != 0;
+
+  BackwardArgs ba;
+  ba.zq = draft;
+  ba.zp = target;
+  ba.grad = grad_draft;
+  ba.R = L.R;
+  ba.V = prob->V;
+  ba.K = (int32_t)prob->K;
+  ba.sT = sampling ? kLog2e / prob->temperature : 0.f;
+  ba.invT = sampling ? 1.0f / prob->temperature : 0.f;
+  ba.dloss = dloss;
+  ba.w_greedy = greedy ? prob->w_greedy : 0.f;
+  ba.w_sampling = sampling ? prob->w_sampling : 0.f;
+  ba.q1_is_qT = greedy && sampling && prob->temperature == 1.0f;
+  ba.ws = loss_ws(const_cast<void*>(workspace), L);
+  return cuda_status(launch_backward(ba, prob->dtype == AAL_BF16, static_cast<cudaStream_t>(stream)));
+}
+
+aal_status aal_accept_reward(const aal_reward_problem* prob, const void* draft, const void* target,
+                             const void* ref_draft, void* workspace, size_t workspace_bytes, int32_t* tau,
+                             int32_t* tau_ref, float* rollout_len, float* advantage, void* stream) {
+  aal_status st = check_reward(prob);
+  if (st != AAL_OK) return st;
+  if (prob->N == 0) return AAL_OK;
+  if (draft == nullptr || target == nullptr || !aligned(draft, 16) || !aligned(target, 16) ||
+      (ref_draft != nullptr && !aligned(ref_draft, 16)))
+    return AAL_ERR_INVALID_ARG;
+  if (tau == nullptr || rollout_len == nullptr || advantage == nullptr || !aligned(tau, 4) ||
+      !aligned(rollout_len, 4) || !aligned(advantage, 4) || (tau_ref != nullptr && !aligned(tau_ref, 4)))
+    return AAL_ERR_INVALID_ARG;
+  const RewardLayout L = reward_layout(prob->N, prob->K);
+  if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < L.total) return AAL_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  char* base = static_cast<char*>(workspace);
+  WsHeader* hdr = reinterpret_cast<WsHeader*>(base + L.hdr);
+  if (cudaMemsetAsync(hdr, 0, sizeof(WsHeader), s) != cudaSuccess) return AAL_ERR_CUDA;
+
+  const bool sampling = prob->mode == AAL_SAMPLING;
+  RewardRowArgs ra;
+  ra.zq = draft;
+  ra.zp = target;
+  ra.zr = ref_draft;
+  ra.R = L.R;
+  ra.V = prob->V;
+  ra.K = (int32_t)prob->K;
+  ra.sampling = sampling;
+  ra.sT = sampling ? kLog2e / prob->temperature : 0.f;
+  ra.seed = prob->seed;
+  ra.row_offset = prob->row_offset;
+  ra.acc = reinterpret_cast<uint8_t*>(base + L.acc);
+  ra.acc_ref = reinterpret_cast<uint8_t*>(base + L.acc_ref);
+  ra.hdr = hdr;
+  cudaError_t e = launch_reward_rows(ra, prob->dtype == AAL_BF16, s);
+  if (e != cudaSuccess) return AAL_ERR_CUDA;
+
+  RewardGroupArgs ga;
+  ga.acc = ra.acc;
+  ga.acc_ref = ref_draft != nullptr ? ra.acc_ref : nullptr;
+  ga.rbuf = reinterpret_cast<float*>(base + L.rbuf);
+  ga.N = prob->N;
+  ga.K = (int32_t)prob->K;
+  ga.wpr = prob->windows_per_rollout;
+  ga.rpg = prob->rollouts_per_group;
+  ga.adv_clip = prob->adv_clip;
+  ga.tau = tau;
+  ga.tau_ref = ref_draft != nullptr ? tau_ref : nullptr;
+  ga.rollout_len = rollout_len;
+  ga.advantage = advantage;
+  return cuda_status(launch_reward_groups(ga, s));
+}
+
+aal_status aal_check_device_status(void* workspace, void* stream) {
+  if (workspace == nullptr || !aligned(workspace, 256)) return AAL_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaStreamSynchronize(s) != cudaSuccess) return AAL_ERR_CUDA;
+  uint32_t word = 0;
+  WsHeader* hdr = static_cast<WsHeader*>(workspace);  // the header is at offset 0 of both layouts
+  if (cudaMemcpy(&word, &hdr->status, sizeof(word), cudaMemcpyDeviceToHost) != cudaSuccess) return AAL_ERR_CUDA;
+  if (word == 0) return AAL_OK;
+  if (cudaMemset(&hdr->status, 0, sizeof(word)) != cudaSuccess) return AAL_ERR_CUDA;
+  return word == kStatusTimeout ? AAL_ERR_TIMEOUT : AAL_ERR_CUDA;
+}
+
+}  // extern "C"

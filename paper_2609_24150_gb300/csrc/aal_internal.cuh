@@ -1,0 +1,322 @@
+// Internal declarations of libaal: device helpers, workspace layout, launchers.
+//
+// Everything here is private to the library; the public surface is include/aal.h.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/aal.h"
+
+namespace aal {
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr int kMaxCluster = 8;          // CTAs that may share one logit row
+constexpr uint32_t kStatusTimeout = 5;  // == AAL_ERR_TIMEOUT
+
+// ---------------------------------------------------------------------------
+// Workspace layout.  Offsets are in bytes from the (256-byte aligned) base and
+// are pure functions of the problem, so forward and backward agree on them.
+// ---------------------------------------------------------------------------
+struct WsHeader {
+  uint32_t status;        // device error word (0 = ok), set by bounded waits
+  uint32_t done_blocks;   // "last block finishes" counter of the window kernel
+  int32_t nvalid;         // |W|, written by the forward
+  int32_t cluster;        // CTAs per row used by the row-statistics kernel
+  float loss;             // copy of the loss
+  float pad[59];
+};
+static_assert(sizeof(WsHeader) == 256, "header is 256 bytes");
+
+struct LossLayout {
+  int64_t R = 0, N = 0, nwblk = 0;
+  size_t hdr = 0;
+  size_t Lp = 0, Lq = 0, Lq1 = 0;   // float[R] log2-domain log-sum-exp of z_p/T, z_q/T, z_q
+  size_t ag = 0, as = 0, qlt = 0;   // float[R] a^greedy, a^sample, sum_{lq<lp} q~
+  size_t dEg = 0, dEs = 0;          // float[R] dE_n / da_{n,j}
+  size_t xstar = 0;                 // int32[R] target argmax
+  size_t cpart = 0;                 // float2[R][kMaxCluster] per-CTA (overlap, Qlt) partials
+  size_t wpart = 0;                 // double[nwblk][4] window-kernel block partials
+  size_t total = 0;
+};
+
+__host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+constexpr int kWindowThreads = 256;
+
+inline LossLayout loss_layout(int64_t N, int64_t K) {
+  LossLayout L;
+  L.N = N;
+  L.R = N * K;
+  L.nwblk = (N + kWindowThreads - 1) / kWindowThreads;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    size_t o = off;
+    off = align_up(off + bytes, 256);
+    return o;
+  };
+  const size_t R = (size_t)L.R;
+  L.hdr = take(sizeof(WsHeader));
+  L.Lp = take(R * 4);
+  L.Lq = take(R * 4);
+  L.Lq1 = take(R * 4);
+  L.ag = take(R * 4);
+  L.as = take(R * 4);
+  L.qlt = take(R * 4);
+  L.dEg = take(R * 4);
+  L.dEs = take(R * 4);
+  L.xstar = take(R * 4);
+  L.cpart = take(R * kMaxCluster * 8);
+  L.wpart = take((size_t)(L.nwblk > 0 ? L.nwblk : 1) * 4 * 8);
+  L.total = off;
+  return L;
+}
+
+struct RewardLayout {
+  int64_t R = 0;
+  size_t hdr = 0, acc = 0, acc_ref = 0, rbuf = 0, total = 0;
+};
+
+inline RewardLayout reward_layout(int64_t N, int64_t K) {
+  RewardLayout L;
+  L.R = N * K;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    size_t o = off;
+    off = align_up(off + bytes, 256);
+    return o;
+  };
+  L.hdr = take(sizeof(WsHeader));
+  L.acc = take((size_t)L.R);
+  L.acc_ref = take((size_t)L.R);
+  L.rbuf = take((size_t)N * 4);
+  L.total = off;
+  return L;
+}
+
+// Pointers into a loss workspace.
+struct LossWs {
+  WsHeader* hdr;
+  float *Lp, *Lq, *Lq1, *ag, *as, *qlt, *dEg, *dEs;
+  int32_t* xstar;
+  float2* cpart;
+  double* wpart;
+};
+
+inline LossWs loss_ws(void* base, const LossLayout& L) {
+  char* b = static_cast<char*>(base);
+  LossWs w;
+  w.hdr = reinterpret_cast<WsHeader*>(b + L.hdr);
+  w.Lp = reinterpret_cast<float*>(b + L.Lp);
+  w.Lq = reinterpret_cast<float*>(b + L.Lq);
+  w.Lq1 = reinterpret_cast<float*>(b + L.Lq1);
+  w.ag = reinterpret_cast<float*>(b + L.ag);
+  w.as = reinterpret_cast<float*>(b + L.as);
+  w.qlt = reinterpret_cast<float*>(b + L.qlt);
+  w.dEg = reinterpret_cast<float*>(b + L.dEg);
+  w.dEs = reinterpret_cast<float*>(b + L.dEs);
+  w.xstar = reinterpret_cast<int32_t*>(b + L.xstar);
+  w.cpart = reinterpret_cast<float2*>(b + L.cpart);
+  w.wpart = reinterpret_cast<double*>(b + L.wpart);
+  return w;
+}
+
+// ---------------------------------------------------------------------------
+// Launch descriptions (host side fills, kernels read by value).
+// ---------------------------------------------------------------------------
+struct RowStatsArgs {
+  const void* zq;       // draft logits  [R][V]
+  const void* zp;       // target logits [R][V]
+  int64_t R, V;
+  float sT;             // log2(e) / T  (scale of the temperature softmaxes)
+  bool need_p;          // log-sum-exp of z_p / T   (sampling term)
+  bool need_q;          // log-sum-exp of z_q / T   (sampling term)
+  bool need_q1;         // log-sum-exp of z_q       (greedy term, when T != 1 or no sampling)
+  bool overlap;         // second phase: sum min(p~, q~) and Qlt (sampling term)
+  LossWs ws;
+};
+
+struct WindowArgs {
+  const uint8_t* mask;  // [N][K] or null
+  int64_t N;
+  int32_t K;
+  int32_t cluster;      // partials per row in ws.cpart
+  bool greedy, sampling;
+  float w_greedy, w_sampling;
+  float* loss;          // device float[1]
+  float* eal;           // device float[N][2] or null
+  LossWs ws;
+  int64_t nwblk;
+};
+
+struct BackwardArgs {
+  const void* zq;
+  const void* zp;
+  void* grad;
+  int64_t R, V;
+  int32_t K;
+  float sT, invT;
+  float dloss;
+  float w_greedy, w_sampling;  // 0 for a term the mode does not select
+  bool q1_is_qT;               // T == 1 with both terms: q = q~, one exponential per element
+  LossWs ws;
+};
+
+struct RewardRowArgs {
+  const void* zq;    // draft
+  const void* zp;    // target
+  const void* zr;    // reference draft or null
+  int64_t R, V;
+  int32_t K;
+  bool sampling;
+  float sT;
+  uint64_t seed;
+  int64_t row_offset;
+  uint8_t* acc;
+  uint8_t* acc_ref;
+  WsHeader* hdr;
+};
+
+struct RewardGroupArgs {
+  const uint8_t* acc;
+  const uint8_t* acc_ref;  // null without a reference draft
+  float* rbuf;             // [N] debiased rewards
+  int64_t N;
+  int32_t K;
+  int64_t wpr, rpg;
+  float adv_clip;
+  int32_t* tau;
+  int32_t* tau_ref;
+  float* rollout_len;
+  float* advantage;
+};
+
+// Launchers (return cudaGetLastError() of their launches).
+cudaError_t launch_rowstats(const RowStatsArgs& a, bool bf16, cudaStream_t s, int* cluster_used);
+cudaError_t launch_window(const WindowArgs& a, cudaStream_t s);
+cudaError_t launch_backward(const BackwardArgs& a, bool bf16, cudaStream_t s);
+cudaError_t launch_reward_rows(const RewardRowArgs& a, bool bf16, cudaStream_t s);
+cudaError_t launch_reward_groups(const RewardGroupArgs& a, cudaStream_t s);
+
+// ---------------------------------------------------------------------------
+// Device helpers.
+// ---------------------------------------------------------------------------
+#ifdef __CUDACC__
+
+// 2^x on the MUFU unit; denormal results flush to zero.
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+template <typename T>
+__device__ __forceinline__ float load_elem(const T* p);
+template <>
+__device__ __forceinline__ float load_elem<float>(const float* p) { return __ldg(p); }
+template <>
+__device__ __forceinline__ float load_elem<uint16_t>(const uint16_t* p) {
+  return __uint_as_float(((uint32_t)__ldg(p)) << 16);
+}
+
+// Streaming 16-byte load that should not linger in L1 (read once per pass).
+__device__ __forceinline__ uint4 ldg_stream(const uint4* p) {
+  uint4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+
+// Online log2-sum-exp state: M = running max of the scaled values, S = sum 2^(x - M).
+struct Lse {
+  float M, S;
+};
+__device__ __forceinline__ void lse_init(Lse& a) {
+  a.M = -INFINITY;
+  a.S = 0.f;
+}
+__device__ __forceinline__ void lse_push(Lse& a, float x) {
+  if (x > a.M) {
+    a.S = a.S * ex2(a.M - x) + 1.f;
+    a.M = x;
+  } else if (a.M != -INFINITY) {
+    a.S += ex2(x - a.M);
+  }
+}
+__device__ __forceinline__ Lse lse_merge(Lse a, Lse b) {
+  Lse r;
+  r.M = fmaxf(a.M, b.M);
+  if (r.M == -INFINITY) {
+    r.S = 0.f;
+  } else {
+    float sa = (a.M == -INFINITY) ? 0.f : a.S * ex2(a.M - r.M);
+    float sb = (b.M == -INFINITY) ? 0.f : b.S * ex2(b.M - r.M);
+    r.S = sa + sb;
+  }
+  return r;
+}
+// log2 of the normaliser: M + log2(S), accurate log (once per row).
+__device__ __forceinline__ float lse_log2(Lse a) { return a.M + log2f(a.S); }
+
+// Argmax with the lowest index on ties, carrying one extra value.
+struct Amax {
+  float v;
+  int32_t i;
+  float carry;
+};
+__device__ __forceinline__ void amax_init(Amax& a) {
+  a.v = -INFINITY;
+  a.i = 0x7fffffff;
+  a.carry = 0.f;
+}
+__device__ __forceinline__ Amax amax_merge(Amax a, Amax b) {
+  return (b.v > a.v || (b.v == a.v && b.i < a.i)) ? b : a;
+}
+
+__device__ __forceinline__ Lse shfl_lse(Lse a, int off) {
+  Lse b;
+  b.M = __shfl_xor_sync(0xffffffffu, a.M, off);
+  b.S = __shfl_xor_sync(0xffffffffu, a.S, off);
+  return b;
+}
+__device__ __forceinline__ Amax shfl_amax(Amax a, int off) {
+  Amax b;
+  b.v = __shfl_xor_sync(0xffffffffu, a.v, off);
+  b.i = __shfl_xor_sync(0xffffffffu, a.i, off);
+  b.carry = __shfl_xor_sync(0xffffffffu, a.carry, off);
+  return b;
+}
+
+// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11): ten rounds of two 32x32->64
+// multiplies with a Weyl-sequence key schedule.
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    if (r > 0) {
+      k0 += 0x9E3779B9u;
+      k1 += 0xBB67AE85u;
+    }
+    const uint32_t hi0 = __umulhi(0xD2511F53u, c.x), lo0 = 0xD2511F53u * c.x;
+    const uint32_t hi1 = __umulhi(0xCD9E8D57u, c.z), lo1 = 0xCD9E8D57u * c.z;
+    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+  }
+  return c;
+}
+
+// The sampling reward's uniform for (seed; window n; depth k): odd multiple of 2^-24 in (0,1).
+__device__ __forceinline__ float philox_uniform(uint64_t seed, uint64_t n, uint32_t k) {
+  uint4 c = make_uint4((uint32_t)n, (uint32_t)(n >> 32), k, 0u);
+  uint4 x = philox4x32_10(c, (uint32_t)seed, (uint32_t)(seed >> 32));
+  return (float)((x.x >> 9) * 2u + 1u) * 5.9604644775390625e-08f;  // * 2^-24
+}
+
+// Bounded wait support: every spin in this library gives up after this many polls.
+constexpr uint32_t kSpinLimit = 1u << 26;
+
+#endif  // __CUDACC__
+
+}  // namespace aal

@@ -1,0 +1,187 @@
+// Backward of the EAL / WTV losses with respect to the draft logits.
+//
+// For row r = (n, j) with g^g = -(dloss/|W|) w_g dE^g_n/da^g_{n,j} and
+// g^s = -(dloss/|W|) w_s dE^s_n/da^s_{n,j} (dE/da from the window kernel):
+//   dz_u = g^g a^g (delta_{u,x*} - q(u))                 greedy term, Eq. acc_greedy
+//        + g^s (1/T) q~(u) (c_u - Qlt),  c_u = [q~_u < p~_u]   sampling term, Eq. acc_sample
+// (the softmax Jacobian applied to d a / d q; at a tie q~_u = p~_u the min follows the
+// frozen p~, so c_u = 0).  q(u), q~(u) and c_u are recomputed from the logits and the
+// row's saved log-sum-exps; nothing of size V is materialised.  One pass: reads z_q
+// (and z_p when the sampling term is on), writes dz in the logits' dtype.
+#include "aal_internal.cuh"
+
+namespace aal {
+namespace {
+
+constexpr int kBwdThreads = 256;
+
+template <typename T>
+struct Io;
+
+template <>
+struct Io<float> {
+  static constexpr int E = 4;
+  __device__ static void unpack(const uint4& w, float* o) {
+    o[0] = __uint_as_float(w.x);
+    o[1] = __uint_as_float(w.y);
+    o[2] = __uint_as_float(w.z);
+    o[3] = __uint_as_float(w.w);
+  }
+  __device__ static uint4 pack(const float* d) {
+    return make_uint4(__float_as_uint(d[0]), __float_as_uint(d[1]), __float_as_uint(d[2]),
+                      __float_as_uint(d[3]));
+  }
+  __device__ static void store1(float* p, float d) { *p = d; }
+};
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+template <>
+struct Io<uint16_t> {
+  static constexpr int E = 8;
+  __device__ static void unpack(const uint4& w, float* o) {
+    o[0] = bf16_lo(w.x);
+    o[1] = bf16_hi(w.x);
+    o[2] = bf16_lo(w.y);
+    o[3] = bf16_hi(w.y);
+    o[4] = bf16_lo(w.z);
+    o[5] = bf16_hi(w.z);
+    o[6] = bf16_lo(w.w);
+    o[7] = bf16_hi(w.w);
+  }
+  __device__ static uint4 pack(const float* d) {
+    return make_uint4(pack_bf16x2(d[0], d[1]), pack_bf16x2(d[2], d[3]), pack_bf16x2(d[4], d[5]),
+                      pack_bf16x2(d[6], d[7]));
+  }
+  __device__ static void store1(uint16_t* p, float d) {
+    *p = (uint16_t)(pack_bf16x2(d, 0.f) & 0xffffu);
+  }
+};
+
+__device__ __forceinline__ void st_stream(uint4* p, const uint4& v) {
+  asm volatile("st.global.cs.v4.u32 [%0], {%1,%2,%3,%4};" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z),
+               "r"(v.w)
+               : "memory");
+}
+
+struct RowCoef {
+  float sT, Lq, Lp, Lq1;
+  float cpos, cneg;  // g^s/T (1 - Qlt) and -g^s/T Qlt
+  float Ag;          // g^g a^g
+  int32_t xs;
+};
+
+template <bool GREEDY, bool SAMPLING, bool Q1_IS_QT>
+__device__ __forceinline__ float grad_elem(const RowCoef& c, float q, float p, int64_t u) {
+  float d = 0.f, qt = 0.f;
+  if (SAMPLING) {
+    const float lq = fmaf(q, c.sT, -c.Lq);
+    const float lp = fmaf(p, c.sT, -c.Lp);
+    qt = ex2(lq);
+    d = qt * (lq < lp ? c.cpos : c.cneg);
+  }
+  if (GREEDY) {
+    const float q1 = Q1_IS_QT ? qt : ex2(fmaf(q, kLog2e, -c.Lq1));
+    d = fmaf(-c.Ag, q1, d);
+    if (u == c.xs) d += c.Ag;
+  }
+  return d;
+}
+
+template <typename T, bool VEC, bool GREEDY, bool SAMPLING, bool Q1_IS_QT>
+__global__ void __launch_bounds__(kBwdThreads) backward_kernel(BackwardArgs a) {
+  const int nvalid = a.ws.hdr->nvalid;
+  const float scale = nvalid > 0 ? -a.dloss / (float)nvalid : 0.f;
+  constexpr int E = Io<T>::E;
+  for (int64_t r = blockIdx.x; r < a.R; r += gridDim.x) {
+    const float gg = GREEDY ? scale * a.w_greedy * a.ws.dEg[r] : 0.f;
+    const float gs = SAMPLING ? scale * a.w_sampling * a.ws.dEs[r] : 0.f;
+    T* out = static_cast<T*>(a.grad) + r * a.V;
+    const T* zq = static_cast<const T*>(a.zq) + r * a.V;
+    const T* zp = static_cast<const T*>(a.zp) + r * a.V;
+    if (gg == 0.f && gs == 0.f) {
+      if (VEC) {
+        uint4* o4 = reinterpret_cast<uint4*>(out);
+        for (int64_t i = threadIdx.x; i < a.V / E; i += kBwdThreads) st_stream(o4 + i, make_uint4(0, 0, 0, 0));
+      } else {
+        for (int64_t v = threadIdx.x; v < a.V; v += kBwdThreads) Io<T>::store1(out + v, 0.f);
+      }
+      continue;
+    }
+    RowCoef c;
+    c.sT = a.sT;
+    c.Lq = SAMPLING ? a.ws.Lq[r] : 0.f;
+    c.Lp = SAMPLING ? a.ws.Lp[r] : 0.f;
+    c.Lq1 = GREEDY ? a.ws.Lq1[r] : 0.f;
+    const float qlt = SAMPLING ? a.ws.qlt[r] : 0.f;
+    const float Bs = gs * a.invT;
+    c.cpos = Bs * (1.f - qlt);
+    c.cneg = -Bs * qlt;
+    c.Ag = GREEDY ? gg * a.ws.ag[r] : 0.f;
+    c.xs = GREEDY ? a.ws.xstar[r] : -1;
+    if (VEC) {
+      const int64_t nv = a.V / E;
+      const uint4* q4 = reinterpret_cast<const uint4*>(zq);
+      const uint4* p4 = reinterpret_cast<const uint4*>(zp);
+      uint4* o4 = reinterpret_cast<uint4*>(out);
+      for (int64_t i = threadIdx.x; i < nv; i += kBwdThreads) {
+        float qv[E], pv[E], d[E];
+        Io<T>::unpack(ldg_stream(q4 + i), qv);
+        if (SAMPLING) Io<T>::unpack(ldg_stream(p4 + i), pv);
+#pragma unroll
+        for (int e = 0; e < E; ++e)
+          d[e] = grad_elem<GREEDY, SAMPLING, Q1_IS_QT>(c, qv[e], SAMPLING ? pv[e] : 0.f, i * E + e);
+        st_stream(o4 + i, Io<T>::pack(d));
+      }
+    } else {
+      for (int64_t v = threadIdx.x; v < a.V; v += kBwdThreads) {
+        const float q = load_elem<T>(zq + v);
+        const float p = SAMPLING ? load_elem<T>(zp + v) : 0.f;
+        Io<T>::store1(out + v, grad_elem<GREEDY, SAMPLING, Q1_IS_QT>(c, q, p, v));
+      }
+    }
+  }
+}
+
+template <typename T, bool VEC, bool G, bool S, bool Q>
+cudaError_t go(const BackwardArgs& a, cudaStream_t s) {
+  int dev = 0, sms = 0, per_sm = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, backward_kernel<T, VEC, G, S, Q>, kBwdThreads, 0);
+  if (per_sm < 1) per_sm = 1;
+  int64_t grid = (int64_t)sms * per_sm;
+  if (grid > a.R) grid = a.R;
+  if (grid < 1) return cudaSuccess;
+  backward_kernel<T, VEC, G, S, Q><<<(unsigned)grid, kBwdThreads, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+template <typename T, bool VEC>
+cudaError_t dispatch_mode(const BackwardArgs& a, cudaStream_t s) {
+  const bool G = a.w_greedy != 0.f, S = a.w_sampling != 0.f;
+  if (G && S) return a.q1_is_qT ? go<T, VEC, true, true, true>(a, s) : go<T, VEC, true, true, false>(a, s);
+  if (G) return go<T, VEC, true, false, false>(a, s);
+  if (S) return go<T, VEC, false, true, false>(a, s);
+  return go<T, VEC, false, false, false>(a, s);
+}
+
+template <typename T>
+cudaError_t dispatch(const BackwardArgs& a, cudaStream_t s) {
+  const bool vec = ((a.V * (int64_t)sizeof(T)) % 16 == 0) &&
+                   ((reinterpret_cast<uintptr_t>(a.zq) | reinterpret_cast<uintptr_t>(a.zp) |
+                     reinterpret_cast<uintptr_t>(a.grad)) % 16 == 0);
+  return vec ? dispatch_mode<T, true>(a, s) : dispatch_mode<T, false>(a, s);
+}
+
+}  // namespace
+
+cudaError_t launch_backward(const BackwardArgs& a, bool bf16, cudaStream_t s) {
+  return bf16 ? dispatch<uint16_t>(a, s) : dispatch<float>(a, s);
+}
+
+}  // namespace aal

@@ -1,0 +1,257 @@
+// Simulated acceptance reward of the GRPO stage (Sec. 3.4).
+//
+// Row kernel, per logit row r = (window n, depth k), one pass over V:
+//   S_k = argmax z_q (greedy draft trajectory), x*_k = argmax z_p, S^ref_k = argmax z_ref,
+//   lowest index on ties.  Greedy verification accepts iff S_k == x*_k.  Sampling
+//   verification accepts iff u < min(1, p~(S_k)/q~(S_k)) (Sec. 2.3), with
+//   u = Philox4x32-10(counter (n_lo, n_hi, k, 0), key seed) and n the global window
+//   index; it needs the log-sum-exps of z_p/T and z_q/T, streamed online.
+// Group kernel, per group of rollouts:
+//   tau = sum_{k=1}^{K} prod_{j<=k} accept_j (the leading run), R = tau - tau^ref
+//   (Eq. debiased_reward), rollout length = mean R over the rollout's windows,
+//   A = clip((x - mean)/(std + 1e-6), -C_A, C_A) with the population std (Eq. advantage).
+#include "aal_internal.cuh"
+
+namespace aal {
+namespace {
+
+constexpr int kRowThreads = 256;
+constexpr int kRowWarps = kRowThreads / 32;
+constexpr int kGroupThreads = 256;
+
+template <typename T>
+__device__ __forceinline__ void unpack_any(const uint4& w, float* o);
+template <>
+__device__ __forceinline__ void unpack_any<float>(const uint4& w, float* o) {
+  o[0] = __uint_as_float(w.x);
+  o[1] = __uint_as_float(w.y);
+  o[2] = __uint_as_float(w.z);
+  o[3] = __uint_as_float(w.w);
+}
+template <>
+__device__ __forceinline__ void unpack_any<uint16_t>(const uint4& w, float* o) {
+  o[0] = bf16_lo(w.x);
+  o[1] = bf16_hi(w.x);
+  o[2] = bf16_lo(w.y);
+  o[3] = bf16_hi(w.y);
+  o[4] = bf16_lo(w.z);
+  o[5] = bf16_hi(w.z);
+  o[6] = bf16_lo(w.w);
+  o[7] = bf16_hi(w.w);
+}
+
+struct RowState {
+  Amax q, p, r;  // draft (carry: z_p at its argmax), target, reference (carry: z_p)
+  Lse lp, lq, lr;
+};
+
+__device__ __forceinline__ RowState merge_state(const RowState& a, const RowState& b) {
+  RowState o;
+  o.q = amax_merge(a.q, b.q);
+  o.p = amax_merge(a.p, b.p);
+  o.r = amax_merge(a.r, b.r);
+  o.lp = lse_merge(a.lp, b.lp);
+  o.lq = lse_merge(a.lq, b.lq);
+  o.lr = lse_merge(a.lr, b.lr);
+  return o;
+}
+
+__device__ __forceinline__ RowState shfl_state(const RowState& a, int off) {
+  RowState o;
+  o.q = shfl_amax(a.q, off);
+  o.p = shfl_amax(a.p, off);
+  o.r = shfl_amax(a.r, off);
+  o.lp = shfl_lse(a.lp, off);
+  o.lq = shfl_lse(a.lq, off);
+  o.lr = shfl_lse(a.lr, off);
+  return o;
+}
+
+__device__ __forceinline__ void init_state(RowState& s) {
+  amax_init(s.q);
+  amax_init(s.p);
+  amax_init(s.r);
+  lse_init(s.lp);
+  lse_init(s.lq);
+  lse_init(s.lr);
+}
+
+template <typename T, bool VEC, bool SAMPLING, bool REF>
+__global__ void __launch_bounds__(kRowThreads) reward_rows(RewardRowArgs a) {
+  __shared__ RowState red[kRowWarps];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  for (int64_t r = blockIdx.x; r < a.R; r += gridDim.x) {
+    const T* zq = static_cast<const T*>(a.zq) + r * a.V;
+    const T* zp = static_cast<const T*>(a.zp) + r * a.V;
+    const T* zr = REF ? static_cast<const T*>(a.zr) + r * a.V : nullptr;
+    RowState st;
+    init_state(st);
+    auto visit = [&](int64_t v, float q, float p, float rr) {
+      if (q > st.q.v) {
+        st.q.v = q;
+        st.q.i = (int32_t)v;
+        st.q.carry = p;
+      }
+      if (p > st.p.v) {
+        st.p.v = p;
+        st.p.i = (int32_t)v;
+      }
+      if (REF && rr > st.r.v) {
+        st.r.v = rr;
+        st.r.i = (int32_t)v;
+        st.r.carry = p;
+      }
+      if (SAMPLING) {
+        lse_push(st.lp, p * a.sT);
+        lse_push(st.lq, q * a.sT);
+        if (REF) lse_push(st.lr, rr * a.sT);
+      }
+    };
+    if (VEC) {
+      constexpr int E = 16 / sizeof(T);
+      const int64_t nv = a.V / E;
+      for (int64_t i = threadIdx.x; i < nv; i += kRowThreads) {
+        float qv[E], pv[E], rv[E];
+        unpack_any<T>(ldg_stream(reinterpret_cast<const uint4*>(zq) + i), qv);
+        unpack_any<T>(ldg_stream(reinterpret_cast<const uint4*>(zp) + i), pv);
+        if (REF) unpack_any<T>(ldg_stream(reinterpret_cast<const uint4*>(zr) + i), rv);
+#pragma unroll
+        for (int e = 0; e < E; ++e) visit(i * E + e, qv[e], pv[e], REF ? rv[e] : 0.f);
+      }
+    } else {
+      for (int64_t v = threadIdx.x; v < a.V; v += kRowThreads)
+        visit(v, load_elem<T>(zq + v), load_elem<T>(zp + v), REF ? load_elem<T>(zr + v) : 0.f);
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) st = merge_state(st, shfl_state(st, off));
+    if (lane == 0) red[warp] = st;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      RowState t = red[0];
+      for (int w = 1; w < kRowWarps; ++w) t = merge_state(t, red[w]);
+      uint8_t acc, acc_ref = 0;
+      if (!SAMPLING) {
+        acc = (t.q.i == t.p.i) ? 1 : 0;
+        if (REF) acc_ref = (t.r.i == t.p.i) ? 1 : 0;
+      } else {
+        const int64_t n = r / a.K;
+        const uint32_t k = (uint32_t)(r - n * a.K);
+        const float u = philox_uniform(a.seed, (uint64_t)(a.row_offset + n), k);
+        const float Lp = lse_log2(t.lp), Lq = lse_log2(t.lq);
+        // log2 p~(S) - log2 q~(S)
+        const float d = fmaf(t.q.carry, a.sT, -Lp) - fmaf(t.q.v, a.sT, -Lq);
+        acc = (u < exp2f(fminf(d, 0.f))) ? 1 : 0;
+        if (REF) {
+          const float Lr = lse_log2(t.lr);
+          const float dr = fmaf(t.r.carry, a.sT, -Lp) - fmaf(t.r.v, a.sT, -Lr);
+          acc_ref = (u < exp2f(fminf(dr, 0.f))) ? 1 : 0;
+        }
+      }
+      a.acc[r] = acc;
+      if (REF) a.acc_ref[r] = acc_ref;
+    }
+    __syncthreads();
+  }
+}
+
+template <typename T, bool VEC, bool S, bool R>
+cudaError_t go(const RewardRowArgs& a, cudaStream_t s) {
+  int dev = 0, sms = 0, per_sm = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, reward_rows<T, VEC, S, R>, kRowThreads, 0);
+  if (per_sm < 1) per_sm = 1;
+  int64_t grid = (int64_t)sms * per_sm;
+  if (grid > a.R) grid = a.R;
+  if (grid < 1) return cudaSuccess;
+  reward_rows<T, VEC, S, R><<<(unsigned)grid, kRowThreads, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+template <typename T, bool VEC>
+cudaError_t dispatch_flags(const RewardRowArgs& a, cudaStream_t s) {
+  const bool ref = a.zr != nullptr;
+  if (a.sampling) return ref ? go<T, VEC, true, true>(a, s) : go<T, VEC, true, false>(a, s);
+  return ref ? go<T, VEC, false, true>(a, s) : go<T, VEC, false, false>(a, s);
+}
+
+template <typename T>
+cudaError_t dispatch(const RewardRowArgs& a, cudaStream_t s) {
+  const bool vec = ((a.V * (int64_t)sizeof(T)) % 16 == 0) &&
+                   ((reinterpret_cast<uintptr_t>(a.zq) | reinterpret_cast<uintptr_t>(a.zp) |
+                     reinterpret_cast<uintptr_t>(a.zr)) % 16 == 0);
+  return vec ? dispatch_flags<T, true>(a, s) : dispatch_flags<T, false>(a, s);
+}
+
+__device__ __forceinline__ double block_sum(double x, double* sm) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) x += __shfl_xor_sync(0xffffffffu, x, off);
+  __syncthreads();
+  if (lane == 0) sm[warp] = x;
+  __syncthreads();
+  double t = sm[0];
+  for (int w = 1; w < kGroupThreads / 32; ++w) t += sm[w];
+  return t;
+}
+
+// One CTA per advantage group.
+__global__ void __launch_bounds__(kGroupThreads) reward_groups(RewardGroupArgs a) {
+  __shared__ double sm[kGroupThreads / 32];
+  const int64_t g = blockIdx.x;
+  const int64_t w0 = g * a.rpg * a.wpr, nw = a.rpg * a.wpr;
+  const int K = a.K;
+  // per window: tau, tau_ref, R
+  for (int64_t i = threadIdx.x; i < nw; i += kGroupThreads) {
+    const int64_t n = w0 + i;
+    int tau = 0;
+    while (tau < K && a.acc[n * K + tau] != 0) ++tau;
+    int tr = 0;
+    if (a.acc_ref != nullptr)
+      while (tr < K && a.acc_ref[n * K + tr] != 0) ++tr;
+    a.tau[n] = tau;
+    if (a.tau_ref != nullptr) a.tau_ref[n] = tr;
+    a.rbuf[n] = (float)(tau - tr);
+  }
+  __syncthreads();
+  // rollout lengths: mean R over each rollout's windows (fixed-order block sums)
+  const volatile float* rb = a.rbuf;
+  for (int64_t ro = 0; ro < a.rpg; ++ro) {
+    double s = 0.0;
+    for (int64_t i = threadIdx.x; i < a.wpr; i += kGroupThreads) s += rb[w0 + ro * a.wpr + i];
+    s = block_sum(s, sm);
+    if (threadIdx.x == 0) a.rollout_len[g * a.rpg + ro] = (float)(s / (double)a.wpr);
+  }
+  __syncthreads();
+  // group mean and population std, then clipped standardised advantages
+  const volatile float* rl = a.rollout_len;
+  double s = 0.0;
+  for (int64_t i = threadIdx.x; i < a.rpg; i += kGroupThreads) s += rl[g * a.rpg + i];
+  const double mean = block_sum(s, sm) / (double)a.rpg;
+  double v = 0.0;
+  for (int64_t i = threadIdx.x; i < a.rpg; i += kGroupThreads) {
+    const double d = rl[g * a.rpg + i] - mean;
+    v += d * d;
+  }
+  const double sd = sqrt(block_sum(v, sm) / (double)a.rpg);
+  for (int64_t i = threadIdx.x; i < a.rpg; i += kGroupThreads) {
+    double A = (rl[g * a.rpg + i] - mean) / (sd + 1e-6);
+    A = fmin(fmax(A, -(double)a.adv_clip), (double)a.adv_clip);
+    a.advantage[g * a.rpg + i] = (float)A;
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_reward_rows(const RewardRowArgs& a, bool bf16, cudaStream_t s) {
+  return bf16 ? dispatch<uint16_t>(a, s) : dispatch<float>(a, s);
+}
+
+cudaError_t launch_reward_groups(const RewardGroupArgs& a, cudaStream_t s) {
+  const int64_t groups = a.N / (a.wpr * a.rpg);
+  if (groups < 1) return cudaSuccess;
+  reward_groups<<<(unsigned)groups, kGroupThreads, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace aal

@@ -1,0 +1,222 @@
+// Forward per-row statistics of the EAL / WTV losses.
+//
+// For every logit row r = (window n, depth j) this computes, from z_p (target)
+// and z_q (draft):
+//   Lp, Lq   log2-domain log-sum-exp of z_p/T and z_q/T (the temperature-scaled
+//            distributions of Sec. 2.3),
+//   Lq1      log2-domain log-sum-exp of z_q (the unscaled draft of Eq. acc_greedy),
+//   x*       argmax_v z_p (lowest index on ties) and a^greedy = q(x*) (Eq. acc_greedy),
+//   a^sample = sum_v min(p~_v, q~_v)   (Eq. acc_sample),
+//   Qlt      = sum_{v: q~_v < p~_v} q~_v, which the backward of a^sample needs.
+// a^sample needs both normalisers before it can be summed, so it is a second phase
+// over the row.  This file holds the generic kernel: one CTA per row, both
+// phases streamed from global memory (the second mostly from L2), any V and any
+// row alignment.
+#include "aal_internal.cuh"
+
+namespace aal {
+namespace {
+
+constexpr int kGenericThreads = 256;
+constexpr int kGenericWarps = kGenericThreads / 32;
+
+template <typename T>
+struct Vec {
+  static constexpr int E = 16 / sizeof(T);
+};
+
+template <typename T>
+__device__ __forceinline__ void unpack(const uint4& w, float* out);
+template <>
+__device__ __forceinline__ void unpack<float>(const uint4& w, float* out) {
+  out[0] = __uint_as_float(w.x);
+  out[1] = __uint_as_float(w.y);
+  out[2] = __uint_as_float(w.z);
+  out[3] = __uint_as_float(w.w);
+}
+template <>
+__device__ __forceinline__ void unpack<uint16_t>(const uint4& w, float* out) {
+  out[0] = bf16_lo(w.x);
+  out[1] = bf16_hi(w.x);
+  out[2] = bf16_lo(w.y);
+  out[3] = bf16_hi(w.y);
+  out[4] = bf16_lo(w.z);
+  out[5] = bf16_hi(w.z);
+  out[6] = bf16_lo(w.w);
+  out[7] = bf16_hi(w.w);
+}
+
+struct Phase1 {
+  Lse p, q, q1;
+  Amax am;
+};
+
+__device__ __forceinline__ Phase1 merge1(const Phase1& a, const Phase1& b) {
+  Phase1 r;
+  r.p = lse_merge(a.p, b.p);
+  r.q = lse_merge(a.q, b.q);
+  r.q1 = lse_merge(a.q1, b.q1);
+  r.am = amax_merge(a.am, b.am);
+  return r;
+}
+
+__device__ __forceinline__ Phase1 shfl1(const Phase1& a, int off) {
+  Phase1 b;
+  b.p = shfl_lse(a.p, off);
+  b.q = shfl_lse(a.q, off);
+  b.q1 = shfl_lse(a.q1, off);
+  b.am = shfl_amax(a.am, off);
+  return b;
+}
+
+template <typename T, bool VEC>
+__global__ void __launch_bounds__(kGenericThreads) rowstats_generic(RowStatsArgs a) {
+  __shared__ Phase1 red1[kGenericWarps];
+  __shared__ float2 red2[kGenericWarps];
+  __shared__ Phase1 row1;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+
+  for (int64_t r = blockIdx.x; r < a.R; r += gridDim.x) {
+    const T* zq = static_cast<const T*>(a.zq) + r * a.V;
+    const T* zp = static_cast<const T*>(a.zp) + r * a.V;
+
+    Phase1 acc;
+    lse_init(acc.p);
+    lse_init(acc.q);
+    lse_init(acc.q1);
+    amax_init(acc.am);
+    auto visit = [&](int64_t v, float p, float q) {
+      if (p > acc.am.v) {
+        acc.am.v = p;
+        acc.am.i = (int32_t)v;
+        acc.am.carry = q;
+      }
+      if (a.need_p) lse_push(acc.p, p * a.sT);
+      if (a.need_q) lse_push(acc.q, q * a.sT);
+      if (a.need_q1) lse_push(acc.q1, q * kLog2e);
+    };
+    constexpr int E = Vec<T>::E;
+    if (VEC) {
+      const int64_t nv = a.V / E;
+      const uint4* p4 = reinterpret_cast<const uint4*>(zp);
+      const uint4* q4 = reinterpret_cast<const uint4*>(zq);
+      for (int64_t i = threadIdx.x; i < nv; i += blockDim.x) {
+        float pv[E], qv[E];
+        unpack<T>(ldg_stream(p4 + i), pv);
+        unpack<T>(ldg_stream(q4 + i), qv);
+#pragma unroll
+        for (int e = 0; e < E; ++e) visit(i * E + e, pv[e], qv[e]);
+      }
+    } else {
+      for (int64_t v = threadIdx.x; v < a.V; v += blockDim.x)
+        visit(v, load_elem<T>(zp + v), load_elem<T>(zq + v));
+    }
+
+    // block reduction of phase 1 (fixed butterfly + fixed warp order: deterministic)
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) acc = merge1(acc, shfl1(acc, off));
+    if (lane == 0) red1[warp] = acc;
+    __syncthreads();
+    if (warp == 0) {
+      Phase1 x;
+      if (lane < kGenericWarps) {
+        x = red1[lane];
+      } else {
+        lse_init(x.p);
+        lse_init(x.q);
+        lse_init(x.q1);
+        amax_init(x.am);
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) x = merge1(x, shfl1(x, off));
+      if (lane == 0) row1 = x;
+    }
+    __syncthreads();
+    const Phase1 tot = row1;
+    const float Lp = a.need_p ? lse_log2(tot.p) : 0.f;
+    const float Lq = a.need_q ? lse_log2(tot.q) : 0.f;
+    const float Lq1 = a.need_q1 ? lse_log2(tot.q1) : Lq;
+
+    float s_min = 0.f, s_qlt = 0.f;
+    if (a.overlap) {
+      auto visit2 = [&](float p, float q) {
+        const float lp = fmaf(p, a.sT, -Lp);
+        const float lq = fmaf(q, a.sT, -Lq);
+        const float e = ex2(fminf(lp, lq));
+        s_min += e;
+        if (lq < lp) s_qlt += e;
+      };
+      if (VEC) {
+        const int64_t nv = a.V / E;
+        const uint4* p4 = reinterpret_cast<const uint4*>(zp);
+        const uint4* q4 = reinterpret_cast<const uint4*>(zq);
+        for (int64_t i = threadIdx.x; i < nv; i += blockDim.x) {
+          float pv[E], qv[E];
+          unpack<T>(ldg_stream(p4 + i), pv);
+          unpack<T>(ldg_stream(q4 + i), qv);
+#pragma unroll
+          for (int e = 0; e < E; ++e) visit2(pv[e], qv[e]);
+        }
+      } else {
+        for (int64_t v = threadIdx.x; v < a.V; v += blockDim.x)
+          visit2(load_elem<T>(zp + v), load_elem<T>(zq + v));
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) {
+        s_min += __shfl_xor_sync(0xffffffffu, s_min, off);
+        s_qlt += __shfl_xor_sync(0xffffffffu, s_qlt, off);
+      }
+      if (lane == 0) red2[warp] = make_float2(s_min, s_qlt);
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        float2 t = red2[0];
+        for (int w = 1; w < kGenericWarps; ++w) {
+          t.x += red2[w].x;
+          t.y += red2[w].y;
+        }
+        s_min = t.x;
+        s_qlt = t.y;
+      }
+    }
+    if (threadIdx.x == 0) {
+      a.ws.Lp[r] = Lp;
+      a.ws.Lq[r] = Lq;
+      a.ws.Lq1[r] = Lq1;
+      a.ws.xstar[r] = tot.am.i;
+      a.ws.ag[r] = exp2f(fmaf(tot.am.carry, kLog2e, -Lq1));
+      a.ws.cpart[r * kMaxCluster] = make_float2(s_min, s_qlt);
+    }
+    __syncthreads();  // red1/red2/row1 are reused by the next row
+  }
+}
+
+template <typename T>
+cudaError_t launch_generic(const RowStatsArgs& a, cudaStream_t s) {
+  const bool vec = ((a.V * (int64_t)sizeof(T)) % 16 == 0) &&
+                   ((reinterpret_cast<uintptr_t>(a.zq) | reinterpret_cast<uintptr_t>(a.zp)) % 16 == 0);
+  int dev = 0, sms = 0, per_sm = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (vec)
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rowstats_generic<T, true>, kGenericThreads, 0);
+  else
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rowstats_generic<T, false>, kGenericThreads, 0);
+  if (per_sm < 1) per_sm = 1;
+  int64_t grid = (int64_t)sms * per_sm;
+  if (grid > a.R) grid = a.R;
+  if (grid < 1) return cudaSuccess;
+  if (vec)
+    rowstats_generic<T, true><<<(unsigned)grid, kGenericThreads, 0, s>>>(a);
+  else
+    rowstats_generic<T, false><<<(unsigned)grid, kGenericThreads, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_rowstats(const RowStatsArgs& a, bool bf16, cudaStream_t s, int* cluster_used) {
+  *cluster_used = 1;
+  return bf16 ? launch_generic<uint16_t>(a, s) : launch_generic<float>(a, s);
+}
+
+}  // namespace aal

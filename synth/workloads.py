@@ -10,9 +10,10 @@ model families evaluated there, and the logit distributions (Gaussian, Zipf
 over a random permutation, heavy-tailed Gumbel, planted peaks, low-overlap rows)
 give the range of target/draft overlap that the losses see in training.
 
-Generation is chunked over windows with a fixed chunk size, so the first ``n``
-windows of a workload are the same bytes whether or not the rest is drawn.
-Values are drawn in fp32 and rounded once to the storage dtype.
+Generation is chunked over windows with a fixed chunk size (256 windows), so on
+a given device the first ``n`` windows, for ``n`` a multiple of the chunk size,
+are the same bytes whether or not the rest is drawn.  Values are drawn in fp32
+and rounded once to the storage dtype.
 """
 
 from __future__ import annotations
@@ -120,12 +121,11 @@ def make_logits(name: str, seed: int = 0, device="cpu", n_windows: Optional[int]
     valid) or ``None`` when the workload masks nothing.
     """
     w = WORKLOADS[name]
-    N = w.N if N is None else N
+    N_full = w.N if N is None else N
     K = w.K if K is None else K
     V = w.V if V is None else V
     dtype = w.dtype if dtype is None else dtype
-    if n_windows is not None:
-        N = min(N, n_windows)
+    N = N_full if n_windows is None else min(N_full, n_windows)
     g = _gen(device, seed)
     target = torch.empty((N, K, V), dtype=dtype, device=device)
     draft = torch.empty((N, K, V), dtype=dtype, device=device)
@@ -139,7 +139,8 @@ def make_logits(name: str, seed: int = 0, device="cpu", n_windows: Optional[int]
     mask = None
     if rate > 0.0:
         gm = _gen(device, seed + 7919)
-        mask = (torch.rand((N, K), generator=gm, device=device) >= rate).to(torch.uint8)
+        mask = (torch.rand((N_full, K), generator=gm, device=device) >= rate).to(torch.uint8)
+        mask = mask[:N].contiguous()
     return target, draft, mask
 
 

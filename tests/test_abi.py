@@ -1,0 +1,143 @@
+"""The C-ABI library loads, exports what include/aal.h declares, and rejects bad arguments
+on the host before launching anything (CPU only: no call here reaches the GPU)."""
+
+import ctypes
+import glob
+import os
+import re
+import subprocess
+
+import pytest
+import torch
+
+import paper_2609_24150_gb300 as aal
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared():
+    names = set()
+    for h in glob.glob(os.path.join(ROOT, "include", "*.h")):
+        text = open(h).read()
+        names |= set(re.findall(r"AAL_API\s+[\w\s\*]+?\b(aal_\w+)\s*\(", text))
+    return names
+
+
+def test_header_declares_the_entry_points():
+    names = _declared()
+    assert {"aal_loss_fwd", "aal_loss_bwd", "aal_accept_reward", "aal_workspace_size",
+            "aal_reward_workspace_size", "aal_check_device_status", "aal_status_string",
+            "aal_abi_version"} <= names
+
+
+def test_library_exports_every_declared_symbol():
+    lib = aal.library()
+    for name in _declared():
+        assert hasattr(lib, name), name
+    out = subprocess.run(["nm", "-D", "--defined-only", aal.library_path()], capture_output=True,
+                         text=True).stdout
+    exported = {l.split()[-1] for l in out.splitlines() if " T " in l}
+    assert {n for n in exported if n.startswith("aal_")} == _declared()
+
+
+def test_status_strings_and_version():
+    assert aal.aal_abi_version() == 10000
+    for code in range(6):
+        assert aal.aal_status_string(code).startswith("AAL_")
+    assert aal.aal_status_string(99) == "unknown aal_status"
+
+
+def _prob(**kw):
+    d = dict(N=4, K=3, V=100, dtype=aal.AAL_BF16, mode=aal.AAL_BOTH, temperature=1.0,
+             w_greedy=0.5, w_sampling=0.5, reserved=0)
+    d.update(kw)
+    return aal.AalProblem(**d)
+
+
+def _ws_size(p):
+    out = ctypes.c_size_t(0)
+    code = aal.library().aal_workspace_size(ctypes.byref(p), ctypes.byref(out))
+    return code, out.value
+
+
+def test_workspace_size_grows_with_rows():
+    c1, s1 = _ws_size(_prob(N=4))
+    c2, s2 = _ws_size(_prob(N=4096))
+    assert c1 == c2 == aal.AAL_OK and 0 < s1 < s2 and s1 % 256 == 0
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(K=0), aal.AAL_ERR_INVALID_ARG),
+    (dict(K=9), aal.AAL_ERR_UNSUPPORTED),
+    (dict(V=0), aal.AAL_ERR_INVALID_ARG),
+    (dict(N=-1), aal.AAL_ERR_INVALID_ARG),
+    (dict(dtype=7), aal.AAL_ERR_INVALID_ARG),
+    (dict(mode=0), aal.AAL_ERR_INVALID_ARG),
+    (dict(mode=4), aal.AAL_ERR_INVALID_ARG),
+    (dict(temperature=0.0), aal.AAL_ERR_INVALID_ARG),
+    (dict(temperature=-1.0), aal.AAL_ERR_INVALID_ARG),
+    (dict(temperature=float("nan")), aal.AAL_ERR_INVALID_ARG),
+    (dict(w_greedy=float("inf")), aal.AAL_ERR_INVALID_ARG),
+    (dict(reserved=1), aal.AAL_ERR_INVALID_ARG),
+    (dict(V=2**31), aal.AAL_ERR_UNSUPPORTED),
+    (dict(N=2**60, V=2**20), aal.AAL_ERR_INVALID_ARG),
+])
+def test_bad_problems_are_rejected(kw, code):
+    assert _ws_size(_prob(**kw))[0] == code
+
+
+def test_greedy_mode_accepts_zero_temperature():
+    assert _ws_size(_prob(mode=aal.AAL_GREEDY, temperature=0.0))[0] == aal.AAL_OK
+
+
+def test_null_and_misaligned_pointers_rejected_before_launch():
+    lib = aal.library()
+    p = _prob()
+    code, size = _ws_size(p)
+    fake_ws = 1 << 20                      # never dereferenced: rejected before any launch
+    fake = 1 << 24
+    # NULL problem
+    assert lib.aal_loss_fwd(None, fake, fake, None, fake_ws, size, fake, None, None) == aal.AAL_ERR_INVALID_ARG
+    # NULL / misaligned logits
+    assert lib.aal_loss_fwd(ctypes.byref(p), None, fake, None, fake_ws, size, fake, None, None) == aal.AAL_ERR_INVALID_ARG
+    assert lib.aal_loss_fwd(ctypes.byref(p), fake + 2, fake, None, fake_ws, size, fake, None, None) == aal.AAL_ERR_INVALID_ARG
+    # NULL loss
+    assert lib.aal_loss_fwd(ctypes.byref(p), fake, fake, None, fake_ws, size, None, None, None) == aal.AAL_ERR_INVALID_ARG
+    # workspace too small / misaligned / missing
+    assert lib.aal_loss_fwd(ctypes.byref(p), fake, fake, None, fake_ws, size - 1, fake, None, None) == aal.AAL_ERR_WORKSPACE
+    assert lib.aal_loss_fwd(ctypes.byref(p), fake, fake, None, fake_ws + 16, size, fake, None, None) == aal.AAL_ERR_WORKSPACE
+    assert lib.aal_loss_fwd(ctypes.byref(p), fake, fake, None, None, size, fake, None, None) == aal.AAL_ERR_WORKSPACE
+    # backward: NULL gradient, non-finite upstream gradient
+    assert lib.aal_loss_bwd(ctypes.byref(p), fake, fake, None, fake_ws, size, 1.0, None, None) == aal.AAL_ERR_INVALID_ARG
+    assert lib.aal_loss_bwd(ctypes.byref(p), fake, fake, None, fake_ws, size, float("nan"), fake, None) == aal.AAL_ERR_INVALID_ARG
+
+
+def _rprob(**kw):
+    d = dict(N=8, K=4, V=100, dtype=aal.AAL_BF16, mode=aal.AAL_GREEDY, temperature=1.0,
+             adv_clip=5.0, seed=0, row_offset=0, windows_per_rollout=2, rollouts_per_group=2)
+    d.update(kw)
+    return aal.AalRewardProblem(**d)
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(), aal.AAL_OK),
+    (dict(mode=aal.AAL_BOTH), aal.AAL_ERR_INVALID_ARG),
+    (dict(mode=aal.AAL_SAMPLING, temperature=0.0), aal.AAL_ERR_INVALID_ARG),
+    (dict(windows_per_rollout=3), aal.AAL_ERR_INVALID_ARG),     # 8 windows not a multiple of 6
+    (dict(rollouts_per_group=0), aal.AAL_ERR_INVALID_ARG),
+    (dict(adv_clip=0.0), aal.AAL_ERR_INVALID_ARG),
+    (dict(row_offset=-1), aal.AAL_ERR_INVALID_ARG),
+    (dict(K=9), aal.AAL_ERR_UNSUPPORTED),
+])
+def test_reward_problem_checks(kw, code):
+    out = ctypes.c_size_t(0)
+    p = _rprob(**kw)
+    assert aal.library().aal_reward_workspace_size(ctypes.byref(p), ctypes.byref(out)) == code
+
+
+def test_binding_refuses_cpu_tensors():
+    t = torch.zeros(2, 2, 8, dtype=torch.bfloat16)
+    p = aal.loss_problem(t, aal.AAL_BOTH)
+    with pytest.raises(ValueError, match="CUDA"):
+        aal.aal_loss_fwd(p, t, t, None, torch.zeros(1024, dtype=torch.uint8),
+                         torch.zeros(1), None)
