@@ -31,7 +31,10 @@ static_assert(sizeof(WsHeader) == 256, "header is 256 bytes");
 struct LossLayout {
   int64_t R = 0, N = 0, nwblk = 0;
   size_t hdr = 0;
-  size_t Lp = 0, Lq = 0, Lq1 = 0;   // float[R] log2-domain log-sum-exp of z_p/T, z_q/T, z_q
+  // float[R] each: the log2-domain normaliser of z_p/T, z_q/T and z_q, kept in two parts:
+  // M = max_v z_v s (s = log2(e)/T, rounded product) and Ls = log2 sum_v 2^(z_v s - M),
+  // so log2 p~_v = fma(z_v, s, -M) - Ls holds its precision for large logits.
+  size_t Mp = 0, Lsp = 0, Mq = 0, Lsq = 0, Mq1 = 0, Lsq1 = 0;
   size_t ag = 0, as = 0, qlt = 0;   // float[R] a^greedy, a^sample, sum_{lq<lp} q~
   size_t dEg = 0, dEs = 0;          // float[R] dE_n / da_{n,j}
   size_t xstar = 0;                 // int32[R] target argmax
@@ -57,9 +60,12 @@ inline LossLayout loss_layout(int64_t N, int64_t K) {
   };
   const size_t R = (size_t)L.R;
   L.hdr = take(sizeof(WsHeader));
-  L.Lp = take(R * 4);
-  L.Lq = take(R * 4);
-  L.Lq1 = take(R * 4);
+  L.Mp = take(R * 4);
+  L.Lsp = take(R * 4);
+  L.Mq = take(R * 4);
+  L.Lsq = take(R * 4);
+  L.Mq1 = take(R * 4);
+  L.Lsq1 = take(R * 4);
   L.ag = take(R * 4);
   L.as = take(R * 4);
   L.qlt = take(R * 4);
@@ -97,7 +103,7 @@ inline RewardLayout reward_layout(int64_t N, int64_t K) {
 // Pointers into a loss workspace.
 struct LossWs {
   WsHeader* hdr;
-  float *Lp, *Lq, *Lq1, *ag, *as, *qlt, *dEg, *dEs;
+  float *Mp, *Lsp, *Mq, *Lsq, *Mq1, *Lsq1, *ag, *as, *qlt, *dEg, *dEs;
   int32_t* xstar;
   float2* cpart;
   double* wpart;
@@ -107,9 +113,12 @@ inline LossWs loss_ws(void* base, const LossLayout& L) {
   char* b = static_cast<char*>(base);
   LossWs w;
   w.hdr = reinterpret_cast<WsHeader*>(b + L.hdr);
-  w.Lp = reinterpret_cast<float*>(b + L.Lp);
-  w.Lq = reinterpret_cast<float*>(b + L.Lq);
-  w.Lq1 = reinterpret_cast<float*>(b + L.Lq1);
+  w.Mp = reinterpret_cast<float*>(b + L.Mp);
+  w.Lsp = reinterpret_cast<float*>(b + L.Lsp);
+  w.Mq = reinterpret_cast<float*>(b + L.Mq);
+  w.Lsq = reinterpret_cast<float*>(b + L.Lsq);
+  w.Mq1 = reinterpret_cast<float*>(b + L.Mq1);
+  w.Lsq1 = reinterpret_cast<float*>(b + L.Lsq1);
   w.ag = reinterpret_cast<float*>(b + L.ag);
   w.as = reinterpret_cast<float*>(b + L.as);
   w.qlt = reinterpret_cast<float*>(b + L.qlt);
@@ -231,7 +240,10 @@ __device__ __forceinline__ uint4 ldg_stream(const uint4* p) {
   return v;
 }
 
-// Online log2-sum-exp state: M = running max of the scaled values, S = sum 2^(x - M).
+// Online log2-sum-exp state of the values z*s: M = running max of the rounded products
+// z*s, S = sum_v 2^(fma(z_v, s, -M)).  Every term, the max's included, is formed the same
+// way as the later evaluation fma(z, s, -M) - log2(S), so the max element's own rounding
+// cancels.
 struct Lse {
   float M, S;
 };
@@ -239,12 +251,13 @@ __device__ __forceinline__ void lse_init(Lse& a) {
   a.M = -INFINITY;
   a.S = 0.f;
 }
-__device__ __forceinline__ void lse_push(Lse& a, float x) {
+__device__ __forceinline__ void lse_push(Lse& a, float z, float s) {
+  const float x = __fmul_rn(z, s);
   if (x > a.M) {
-    a.S = a.S * ex2(a.M - x) + 1.f;
+    a.S = a.S * ex2(a.M - x) + ex2(fmaf(z, s, -x));
     a.M = x;
   } else if (a.M != -INFINITY) {
-    a.S += ex2(x - a.M);
+    a.S += ex2(fmaf(z, s, -a.M));
   }
 }
 __device__ __forceinline__ Lse lse_merge(Lse a, Lse b) {
@@ -259,8 +272,12 @@ __device__ __forceinline__ Lse lse_merge(Lse a, Lse b) {
   }
   return r;
 }
-// log2 of the normaliser: M + log2(S), accurate log (once per row).
-__device__ __forceinline__ float lse_log2(Lse a) { return a.M + log2f(a.S); }
+// log2(S) of the normaliser, accurate log (once per row); the normaliser is M + log2(S).
+__device__ __forceinline__ float lse_ls(Lse a) { return log2f(a.S); }
+// log2 of the scaled probability of logit z: fma(z, s, -M) - Ls.
+__device__ __forceinline__ float log2_prob(float z, float s, float M, float Ls) {
+  return fmaf(z, s, -M) - Ls;
+}
 
 // Argmax with the lowest index on ties, carrying one extra value.
 struct Amax {

@@ -69,7 +69,7 @@ __device__ __forceinline__ void st_stream(uint4* p, const uint4& v) {
 }
 
 struct RowCoef {
-  float sT, Lq, Lp, Lq1;
+  float sT, Mq, Lsq, Mp, Lsp, Mq1, Lsq1;
   float cpos, cneg;  // g^s/T (1 - Qlt) and -g^s/T Qlt
   float Ag;          // g^g a^g
   int32_t xs;
@@ -79,13 +79,13 @@ template <bool GREEDY, bool SAMPLING, bool Q1_IS_QT>
 __device__ __forceinline__ float grad_elem(const RowCoef& c, float q, float p, int64_t u) {
   float d = 0.f, qt = 0.f;
   if (SAMPLING) {
-    const float lq = fmaf(q, c.sT, -c.Lq);
-    const float lp = fmaf(p, c.sT, -c.Lp);
+    const float lq = log2_prob(q, c.sT, c.Mq, c.Lsq);
+    const float lp = log2_prob(p, c.sT, c.Mp, c.Lsp);
     qt = ex2(lq);
     d = qt * (lq < lp ? c.cpos : c.cneg);
   }
   if (GREEDY) {
-    const float q1 = Q1_IS_QT ? qt : ex2(fmaf(q, kLog2e, -c.Lq1));
+    const float q1 = Q1_IS_QT ? qt : ex2(log2_prob(q, kLog2e, c.Mq1, c.Lsq1));
     d = fmaf(-c.Ag, q1, d);
     if (u == c.xs) d += c.Ag;
   }
@@ -114,9 +114,12 @@ __global__ void __launch_bounds__(kBwdThreads) backward_kernel(BackwardArgs a) {
     }
     RowCoef c;
     c.sT = a.sT;
-    c.Lq = SAMPLING ? a.ws.Lq[r] : 0.f;
-    c.Lp = SAMPLING ? a.ws.Lp[r] : 0.f;
-    c.Lq1 = GREEDY ? a.ws.Lq1[r] : 0.f;
+    c.Mq = SAMPLING ? a.ws.Mq[r] : 0.f;
+    c.Lsq = SAMPLING ? a.ws.Lsq[r] : 0.f;
+    c.Mp = SAMPLING ? a.ws.Mp[r] : 0.f;
+    c.Lsp = SAMPLING ? a.ws.Lsp[r] : 0.f;
+    c.Mq1 = GREEDY ? a.ws.Mq1[r] : 0.f;
+    c.Lsq1 = GREEDY ? a.ws.Lsq1[r] : 0.f;
     const float qlt = SAMPLING ? a.ws.qlt[r] : 0.f;
     const float Bs = gs * a.invT;
     c.cpos = Bs * (1.f - qlt);

@@ -102,9 +102,9 @@ __global__ void __launch_bounds__(kRowThreads) reward_rows(RewardRowArgs a) {
         st.r.carry = p;
       }
       if (SAMPLING) {
-        lse_push(st.lp, p * a.sT);
-        lse_push(st.lq, q * a.sT);
-        if (REF) lse_push(st.lr, rr * a.sT);
+        lse_push(st.lp, p, a.sT);
+        lse_push(st.lq, q, a.sT);
+        if (REF) lse_push(st.lr, rr, a.sT);
       }
     };
     if (VEC) {
@@ -137,13 +137,13 @@ __global__ void __launch_bounds__(kRowThreads) reward_rows(RewardRowArgs a) {
         const int64_t n = r / a.K;
         const uint32_t k = (uint32_t)(r - n * a.K);
         const float u = philox_uniform(a.seed, (uint64_t)(a.row_offset + n), k);
-        const float Lp = lse_log2(t.lp), Lq = lse_log2(t.lq);
+        const float Lsp = lse_ls(t.lp), Lsq = lse_ls(t.lq);
         // log2 p~(S) - log2 q~(S)
-        const float d = fmaf(t.q.carry, a.sT, -Lp) - fmaf(t.q.v, a.sT, -Lq);
+        const float d = log2_prob(t.q.carry, a.sT, t.lp.M, Lsp) - log2_prob(t.q.v, a.sT, t.lq.M, Lsq);
         acc = (u < exp2f(fminf(d, 0.f))) ? 1 : 0;
         if (REF) {
-          const float Lr = lse_log2(t.lr);
-          const float dr = fmaf(t.r.carry, a.sT, -Lp) - fmaf(t.r.v, a.sT, -Lr);
+          const float Lsr = lse_ls(t.lr);
+          const float dr = log2_prob(t.r.carry, a.sT, t.lp.M, Lsp) - log2_prob(t.r.v, a.sT, t.lr.M, Lsr);
           acc_ref = (u < exp2f(fminf(dr, 0.f))) ? 1 : 0;
         }
       }

@@ -2,9 +2,9 @@
 //
 // For every logit row r = (window n, depth j) this computes, from z_p (target)
 // and z_q (draft):
-//   Lp, Lq   log2-domain log-sum-exp of z_p/T and z_q/T (the temperature-scaled
-//            distributions of Sec. 2.3),
-//   Lq1      log2-domain log-sum-exp of z_q (the unscaled draft of Eq. acc_greedy),
+//   (M, Ls)  the log2-domain normalisers of z_p/T and z_q/T (the temperature-scaled
+//            distributions of Sec. 2.3) and of z_q (the unscaled draft of Eq.
+//            acc_greedy): M = max_v z_v s, Ls = log2 sum_v 2^(z_v s - M),
 //   x*       argmax_v z_p (lowest index on ties) and a^greedy = q(x*) (Eq. acc_greedy),
 //   a^sample = sum_v min(p~_v, q~_v)   (Eq. acc_sample),
 //   Qlt      = sum_{v: q~_v < p~_v} q~_v, which the backward of a^sample needs.
@@ -91,9 +91,9 @@ __global__ void __launch_bounds__(kGenericThreads) rowstats_generic(RowStatsArgs
         acc.am.i = (int32_t)v;
         acc.am.carry = q;
       }
-      if (a.need_p) lse_push(acc.p, p * a.sT);
-      if (a.need_q) lse_push(acc.q, q * a.sT);
-      if (a.need_q1) lse_push(acc.q1, q * kLog2e);
+      if (a.need_p) lse_push(acc.p, p, a.sT);
+      if (a.need_q) lse_push(acc.q, q, a.sT);
+      if (a.need_q1) lse_push(acc.q1, q, kLog2e);
     };
     constexpr int E = Vec<T>::E;
     if (VEC) {
@@ -133,15 +133,15 @@ __global__ void __launch_bounds__(kGenericThreads) rowstats_generic(RowStatsArgs
     }
     __syncthreads();
     const Phase1 tot = row1;
-    const float Lp = a.need_p ? lse_log2(tot.p) : 0.f;
-    const float Lq = a.need_q ? lse_log2(tot.q) : 0.f;
-    const float Lq1 = a.need_q1 ? lse_log2(tot.q1) : Lq;
+    const float Mp = tot.p.M, Lsp = a.need_p ? lse_ls(tot.p) : 0.f;
+    const float Mq = tot.q.M, Lsq = a.need_q ? lse_ls(tot.q) : 0.f;
+    const float Mq1 = a.need_q1 ? tot.q1.M : Mq, Lsq1 = a.need_q1 ? lse_ls(tot.q1) : Lsq;
 
     float s_min = 0.f, s_qlt = 0.f;
     if (a.overlap) {
       auto visit2 = [&](float p, float q) {
-        const float lp = fmaf(p, a.sT, -Lp);
-        const float lq = fmaf(q, a.sT, -Lq);
+        const float lp = log2_prob(p, a.sT, Mp, Lsp);
+        const float lq = log2_prob(q, a.sT, Mq, Lsq);
         const float e = ex2(fminf(lp, lq));
         s_min += e;
         if (lq < lp) s_qlt += e;
@@ -179,11 +179,14 @@ __global__ void __launch_bounds__(kGenericThreads) rowstats_generic(RowStatsArgs
       }
     }
     if (threadIdx.x == 0) {
-      a.ws.Lp[r] = Lp;
-      a.ws.Lq[r] = Lq;
-      a.ws.Lq1[r] = Lq1;
+      a.ws.Mp[r] = Mp;
+      a.ws.Lsp[r] = Lsp;
+      a.ws.Mq[r] = Mq;
+      a.ws.Lsq[r] = Lsq;
+      a.ws.Mq1[r] = Mq1;
+      a.ws.Lsq1[r] = Lsq1;
       a.ws.xstar[r] = tot.am.i;
-      a.ws.ag[r] = exp2f(fmaf(tot.am.carry, kLog2e, -Lq1));
+      a.ws.ag[r] = exp2f(log2_prob(tot.am.carry, kLog2e, Mq1, Lsq1));
       a.ws.cpart[r * kMaxCluster] = make_float2(s_min, s_qlt);
     }
     __syncthreads();  // red1/red2/row1 are reused by the next row
