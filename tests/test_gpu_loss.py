@@ -181,11 +181,12 @@ def test_v128k_full_size_sampled_windows(v128k):
                windows=windows, n_windows_total=N)
     implied = loss_from_eal(run, aal.AAL_BOTH, 0.5, 0.5, N)
     assert abs(float(run.loss.item()) - implied) <= 1e-5 * abs(implied)
-    # every gradient row is finite and sums to ~0 (softmax shift invariance), at full size
+    # every gradient row is finite and sums to 0 (softmax shift invariance) up to the bf16
+    # rounding of its elements: |sum g^| <= 2^-9 sum |g| plus fp32 accumulation error
     for n0 in range(0, N, 512):
-        g = run.grad[n0:n0 + 512].float()
+        g = run.grad[n0:n0 + 512].double()
         assert torch.isfinite(g).all()
-        assert (g.sum(-1).abs() <= 1e-2 * g.abs().amax(-1) + 1e-6).all()
+        assert (g.sum(-1).abs() <= 2.0 ** -8 * g.abs().sum(-1) + 1e-9).all()
     del run
     torch.cuda.empty_cache()
 
