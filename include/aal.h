@@ -159,6 +159,26 @@ AAL_API aal_status aal_accept_reward(const aal_reward_problem* prob, const void*
                              size_t workspace_bytes, int32_t* tau, int32_t* tau_ref,
                              float* rollout_len, float* advantage, void* stream);
 
+/* aal_accept_reward without a workspace argument: the scratch lives in a fixed array inside
+ * the library.  The paper has no counterpart; this exists for callers that cannot allocate
+ * device memory -- e.g. a training loop whose device memory is all reserved up front by its
+ * own caching allocator, so a raw cudaMalloc would fail or fragment that pool, or a component
+ * that only receives device pointers from another one and has no allocator of its own.
+ *   Limit.   N * K <= 1048576 logit rows; larger problems return AAL_ERR_UNSUPPORTED before
+ *            anything is launched.  The array (6 MiB + 4 KiB) is held by every GPU that loads
+ *            the library until the process exits.
+ *   Set-up.  The first call on a device (with that device current) looks up the array's device
+ *            address once; make that first call before any stream capture.
+ *   Sharing. Every call uses the same array, which keeps the last call's contents (each call
+ *            clears what must start at zero).  Calls that overlap on the GPU (different streams,
+ *            or different host threads) race on it: order them.
+ *   Allocation.  Calls no cudaMalloc, cudaFree or allocating routine.
+ * Other arguments and results are those of aal_accept_reward. */
+AAL_API aal_status aal_accept_reward_noalloc(const aal_reward_problem* prob, const void* draft,
+                                             const void* target, const void* ref_draft, int32_t* tau,
+                                             int32_t* tau_ref, float* rollout_len, float* advantage,
+                                             void* stream);
+
 /* Synchronises `stream`, reads the device status word of a loss or reward workspace,
  * clears it, and returns AAL_OK or the recorded device error (AAL_ERR_TIMEOUT). */
 AAL_API aal_status aal_check_device_status(void* workspace, void* stream);

@@ -21,6 +21,7 @@ from .aal import (  # noqa: F401
     AAL_F32,
     AAL_GREEDY,
     AAL_MAX_K,
+    AAL_NOALLOC_MAX_ROWS,
     AAL_OK,
     AAL_SAMPLING,
     AalError,
@@ -28,6 +29,7 @@ from .aal import (  # noqa: F401
     AalRewardProblem,
     aal_abi_version,
     aal_accept_reward,
+    aal_accept_reward_noalloc,
     aal_check_device_status,
     aal_loss_bwd,
     aal_loss_fwd,

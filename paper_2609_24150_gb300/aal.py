@@ -23,6 +23,7 @@ AAL_SAMPLING = 2
 AAL_BOTH = 3
 
 AAL_MAX_K = 8
+AAL_NOALLOC_MAX_ROWS = 1 << 20   # N * K limit of aal_accept_reward_noalloc
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 
@@ -74,13 +75,14 @@ def library() -> ctypes.CDLL:
     lib.aal_loss_fwd.argtypes = [P, vp, vp, vp, vp, sz, vp, vp, vp]
     lib.aal_loss_bwd.argtypes = [P, vp, vp, vp, vp, sz, ctypes.c_float, vp, vp]
     lib.aal_accept_reward.argtypes = [RP, vp, vp, vp, vp, sz, vp, vp, vp, vp, vp]
+    lib.aal_accept_reward_noalloc.argtypes = [RP, vp, vp, vp, vp, vp, vp, vp, vp]
     lib.aal_check_device_status.argtypes = [vp, vp]
     lib.aal_status_string.argtypes = [ctypes.c_int]
     lib.aal_status_string.restype = ctypes.c_char_p
     lib.aal_abi_version.argtypes = []
     lib.aal_abi_version.restype = ctypes.c_int32
     for f in ("aal_workspace_size", "aal_reward_workspace_size", "aal_loss_fwd", "aal_loss_bwd",
-              "aal_accept_reward", "aal_check_device_status"):
+              "aal_accept_reward", "aal_accept_reward_noalloc", "aal_check_device_status"):
         getattr(lib, f).restype = ctypes.c_int
     _LIB = lib
     return lib
@@ -203,6 +205,28 @@ def aal_accept_reward(problem: AalRewardProblem, draft, target, ref_draft, works
         _ptr(rollout_len, "rollout_len", torch.float32, nroll),
         _ptr(advantage, "advantage", torch.float32, nroll), _stream(stream))
     _check(code, "aal_accept_reward")
+
+
+def aal_accept_reward_noalloc(problem: AalRewardProblem, draft, target, ref_draft, tau, tau_ref,
+                              rollout_len, advantage, stream=None):
+    """aal_accept_reward with the library's fixed scratch array instead of a workspace.
+
+    For callers that cannot allocate device memory (e.g. their memory is fully reserved by
+    their own allocator).  At most AAL_NOALLOC_MAX_ROWS = N * K rows; calls share one scratch
+    array, so calls that overlap on the GPU must be ordered by the caller.
+    """
+    N = problem.N
+    if N * problem.K > AAL_NOALLOC_MAX_ROWS:
+        raise AalError(AAL_ERR_UNSUPPORTED, f"aal_accept_reward_noalloc: N*K = {N * problem.K} "
+                       f"exceeds the fixed scratch limit of {AAL_NOALLOC_MAX_ROWS} rows")
+    nroll = N // max(1, problem.windows_per_rollout)
+    code = library().aal_accept_reward_noalloc(
+        ctypes.byref(problem), _ptr(draft, "draft"), _ptr(target, "target"),
+        _ptr(ref_draft, "ref_draft"), _ptr(tau, "tau", torch.int32, N),
+        _ptr(tau_ref, "tau_ref", torch.int32, N),
+        _ptr(rollout_len, "rollout_len", torch.float32, nroll),
+        _ptr(advantage, "advantage", torch.float32, nroll), _stream(stream))
+    _check(code, "aal_accept_reward_noalloc")
 
 
 def aal_check_device_status(workspace, stream=None) -> int:
