@@ -150,6 +150,7 @@ __global__ void __launch_bounds__(kWindowThreads) window_kernel(WindowArgs a) {
     *a.loss = loss;
     a.ws.hdr->loss = loss;
     a.ws.hdr->nvalid = nvalid;
+    a.ws.hdr->cluster = a.cluster;
     a.ws.hdr->done_blocks = 0u;
   }
 }

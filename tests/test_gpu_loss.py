@@ -59,6 +59,22 @@ def test_ragged_vocab_and_window_sizes(V, dtype, K):
         check_loss(run, t, d, m, mode, T, 0.5, 0.5, dloss=5.0)
 
 
+@pytest.mark.parametrize("V,dtype,width", [(8, torch.bfloat16, 1), (65544, torch.bfloat16, 2),
+                                           (100000, torch.bfloat16, 4), (250000, torch.bfloat16, 8),
+                                           (167936, torch.bfloat16, 8), (40000, torch.float32, 2)])
+def test_cluster_widths(V, dtype, width):
+    """Rows split over 1, 2, 4 and 8 CTAs of a cluster (chosen from V), including a
+    single-vector row and a cluster whose last CTA holds a partial chunk."""
+    target, draft, _ = synth.make_logits("tiny", seed=V, N=3, K=2, V=V, dtype=dtype)
+    draft[1, 1] = target[1, 1]          # an identical row inside a window
+    t, d = _dev(target, draft)
+    for mode, T in [(aal.AAL_BOTH, 1.0), (aal.AAL_SAMPLING, 0.8), (aal.AAL_BOTH, 1.4)]:
+        run = LossRun(t, d, None, mode, T, 0.5, 0.5, dloss=3.0)
+        hdr = run.ws_buf[:16].view(torch.int32).cpu()
+        assert int(hdr[3]) == width     # cluster width recorded in the workspace header
+        check_loss(run, t, d, None, mode, T, 0.5, 0.5, dloss=3.0)
+
+
 def test_masked_v32k_sampled_windows():
     """V = 32000 bf16 with 10% of positions masked: sampled windows, loss via the eal outputs."""
     target, draft, mask = synth.make_logits("v32k", seed=0, device=DEV)
