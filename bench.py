@@ -50,6 +50,9 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--windows", type=int, default=None,
+                    help="run the first WINDOWS windows of the workload (profiling captures)")
     return ap.parse_args()
 
 
@@ -136,8 +139,10 @@ def run_ours(args, ws_count, rank, local):
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
     stream = torch.cuda.current_stream()
-    target, draft, _ = synth.make_logits(WORKLOAD, seed=rank, device=dev)
+    target, draft, _ = synth.make_logits(WORKLOAD, seed=rank, device=dev, n_windows=args.windows)
     N, K, V = draft.shape
+    if N % (WPR * RPG) != 0:
+        raise SystemExit(f"--windows must be a multiple of {WPR * RPG}")
     grad = torch.empty_like(draft)
     prob = aal.loss_problem(draft, aal.AAL_BOTH, MODE_T, W_G, W_S)
     ws = torch.empty(aal.aal_workspace_size(prob), dtype=torch.uint8, device=dev)
@@ -244,7 +249,7 @@ def run_ours(args, ws_count, rank, local):
         "clocks": clk,
     }
 
-    if rank == 0:
+    if rank == 0 and not args.no_e2e:
         res["e2e"] = run_e2e(args, aal, prob, rprob, draft, target, grad, ws, loss, rws, tau, rl, adv,
                              stream, step_bytes)
     if rank == 0 and ws_count == 1 and not args.no_cpu_baseline:
