@@ -141,16 +141,19 @@ def run_ours(args, ws_count, rank, local):
     stream = torch.cuda.current_stream()
     target, draft, _ = synth.make_logits(WORKLOAD, seed=rank, device=dev, n_windows=args.windows)
     N, K, V = draft.shape
-    if N % (WPR * RPG) != 0:
-        raise SystemExit(f"--windows must be a multiple of {WPR * RPG}")
+    # reward grouping: 16 rollouts of 256 windows per group; a smaller batch keeps the 16
+    # rollouts per group and shortens the rollouts
+    wpr = WPR if N % (WPR * RPG) == 0 else N // RPG
+    if wpr < 1 or N % (wpr * RPG) != 0:
+        raise SystemExit(f"--windows must be a multiple of {RPG}")
     grad = torch.empty_like(draft)
     prob = aal.loss_problem(draft, aal.AAL_BOTH, MODE_T, W_G, W_S)
     ws = torch.empty(aal.aal_workspace_size(prob), dtype=torch.uint8, device=dev)
     loss = torch.empty(1, dtype=torch.float32, device=dev)
-    rprob = aal.reward_problem(draft, aal.AAL_GREEDY, 1.0, 5.0, 0, rank * N, WPR, RPG)
+    rprob = aal.reward_problem(draft, aal.AAL_GREEDY, 1.0, 5.0, 0, rank * N, wpr, RPG)
     rws = torch.empty(aal.aal_reward_workspace_size(rprob), dtype=torch.uint8, device=dev)
     tau = torch.empty(N, dtype=torch.int32, device=dev)
-    nroll = N // WPR
+    nroll = N // wpr
     rl = torch.empty(nroll, dtype=torch.float32, device=dev)
     adv = torch.empty(nroll, dtype=torch.float32, device=dev)
 
