@@ -70,22 +70,26 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t* b, uint32_t bytes) {
 __device__ __forceinline__ void mbar_arrive(uint64_t* b) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(s32(b)) : "memory");
 }
+// try_wait with a suspend-time hint: a thread whose phase has not completed sleeps in
+// hardware (up to kSuspendNs) instead of spinning, leaving the issue slots to the warps
+// that have work.
+constexpr uint32_t kSuspendNs = 20000;
 __device__ __forceinline__ bool mbar_test(uint64_t* b, uint32_t parity) {
   uint32_t ok;
   asm volatile(
-      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n selp.u32 %0, 1, 0, p;\n}"
       : "=r"(ok)
-      : "r"(s32(b)), "r"(parity)
+      : "r"(s32(b)), "r"(parity), "r"(kSuspendNs)
       : "memory");
   return ok != 0;
 }
 __device__ __forceinline__ bool mbar_test_cluster(uint64_t* b, uint32_t parity) {
   uint32_t ok;
   asm volatile(
-      "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n"
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n"
       " selp.u32 %0, 1, 0, p;\n}"
       : "=r"(ok)
-      : "r"(s32(b)), "r"(parity)
+      : "r"(s32(b)), "r"(parity), "r"(kSuspendNs)
       : "memory");
   return ok != 0;
 }
@@ -149,8 +153,7 @@ __device__ __forceinline__ uint64_t now_ns() {
 template <bool CLUSTER>
 __device__ __forceinline__ bool wait_phase(uint64_t* b, uint32_t parity, volatile int* abort_flag,
                                            uint64_t limit_ns, WsHeader* hdr) {
-  if (*abort_flag) return false;
-  if (CLUSTER ? mbar_test_cluster(b, parity) : mbar_test(b, parity)) return true;
+  if (CLUSTER ? mbar_test_cluster(b, parity) : mbar_test(b, parity)) return !*abort_flag;
   const uint64_t t0 = now_ns();
   for (uint32_t it = 0; it < kSpinLimit; ++it) {
     if (CLUSTER ? mbar_test_cluster(b, parity) : mbar_test(b, parity)) return true;
@@ -242,6 +245,106 @@ __device__ __forceinline__ void unpack8<float>(const uint4& w, float* o) {
   o[1] = __uint_as_float(w.y);
   o[2] = __uint_as_float(w.z);
   o[3] = __uint_as_float(w.w);
+}
+
+// ---- packed arithmetic (sm_100+): two fp32 lanes per instruction, exact IEEE rounding
+__device__ __forceinline__ float2 f2fma(float2 a, float2 b, float2 c) {
+  float2 d;
+  asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\tmov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+      "mov.b64 rc, {%6, %7};\n\tfma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+  return d;
+}
+__device__ __forceinline__ float2 f2add(float2 a, float2 b) {
+  float2 d;
+  asm("{\n\t.reg .b64 ra, rb, rd;\n\tmov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+      "add.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return d;
+}
+__device__ __forceinline__ uint32_t bmax2(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
+}
+__device__ __forceinline__ float set_lt(float a, float b) {  // 1.0f if a < b else 0.0f
+  float d;
+  asm("set.lt.f32.f32 %0, %1, %2;" : "=f"(d) : "f"(a), "f"(b));
+  return d;
+}
+// max of the 16 bf16 values in two 16-byte vectors (exact: max of bf16 values is a bf16 value)
+__device__ __forceinline__ float bmax16(const uint4& a, const uint4& b) {
+  const uint32_t m = bmax2(bmax2(bmax2(a.x, a.y), bmax2(a.z, a.w)), bmax2(bmax2(b.x, b.y), bmax2(b.z, b.w)));
+  return fmaxf(bf16_lo(m), bf16_hi(m));
+}
+__device__ __forceinline__ float2 bpair(uint32_t w) { return make_float2(bf16_lo(w), bf16_hi(w)); }
+
+// One tensor's 16 bf16 values folded into (M, S): max first, then 2^(z s - M) summed with
+// packed fma / add over two independent accumulators.
+__device__ __forceinline__ void lse16(float& M, float& S, const uint4& a, const uint4& b, float vmax, float s) {
+  const float xm = __fmul_rn(vmax, s);
+  if (xm > M) {
+    S *= ex2(M - xm);
+    M = xm;
+  }
+  if (M == -INFINITY) return;
+  const float2 s2 = make_float2(s, s), m2 = make_float2(-M, -M);
+  const uint32_t w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+  float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
+#pragma unroll
+  for (int k = 0; k < 8; k += 2) {
+    const float2 x0 = f2fma(bpair(w[k]), s2, m2);
+    const float2 x1 = f2fma(bpair(w[k + 1]), s2, m2);
+    acc0 = f2add(acc0, make_float2(ex2(x0.x), ex2(x0.y)));
+    acc1 = f2add(acc1, make_float2(ex2(x1.x), ex2(x1.y)));
+  }
+  const float2 t = f2add(acc0, acc1);
+  S += t.x + t.y;
+}
+
+// Phase 1 on a full bf16 chunk slice: 16 values of z_p and z_q per thread.
+template <bool NEED_Q1>
+__device__ __forceinline__ void phase1_bf16x16(Part& A, const uint4& p0, const uint4& p1, const uint4& q0,
+                                               const uint4& q1, int64_t idx0, int64_t idx1, float sT) {
+  const float pm = bmax16(p0, p1), qm = bmax16(q0, q1);
+  if (pm > A.av) {  // new argmax of z_p: its first occurrence (rare after the first chunks)
+    const uint32_t pw[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
+    const uint32_t qw[8] = {q0.x, q0.y, q0.z, q0.w, q1.x, q1.y, q1.z, q1.w};
+    int e = 0;
+    float carry = 0.f;
+#pragma unroll
+    for (int k = 15; k >= 0; --k) {
+      const float v = (k & 1) ? bf16_hi(pw[k >> 1]) : bf16_lo(pw[k >> 1]);
+      if (v == pm) {
+        e = k;
+        carry = (k & 1) ? bf16_hi(qw[k >> 1]) : bf16_lo(qw[k >> 1]);
+      }
+    }
+    A.av = pm;
+    A.ai = (int32_t)(e < 8 ? idx0 + e : idx1 + (e - 8));
+    A.ac = carry;
+  }
+  lse16(A.pM, A.pS, p0, p1, pm, sT);
+  lse16(A.qM, A.qS, q0, q1, qm, sT);
+  if (NEED_Q1) lse16(A.q1M, A.q1S, q0, q1, qm, kLog2e);
+}
+
+// Phase 2 on 8 bf16 values of each tensor: sum_v min(p~, q~) and sum_{q~ < p~} q~.
+__device__ __forceinline__ void phase2_bf16x8(float2& smin2, float2& sqlt2, const uint4& pw, const uint4& qw,
+                                              float2 s2, float2 negM, float2 negLs) {
+  const uint32_t pa[4] = {pw.x, pw.y, pw.z, pw.w};
+  const uint32_t qa[4] = {qw.x, qw.y, qw.z, qw.w};
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    // lanes (p, q) of element 2k and of element 2k+1
+    const float2 l0 = f2add(f2fma(make_float2(bf16_lo(pa[k]), bf16_lo(qa[k])), s2, negM), negLs);
+    const float2 l1 = f2add(f2fma(make_float2(bf16_hi(pa[k]), bf16_hi(qa[k])), s2, negM), negLs);
+    const float2 e = make_float2(ex2(fminf(l0.x, l0.y)), ex2(fminf(l1.x, l1.y)));
+    smin2 = f2add(smin2, e);
+    sqlt2 = f2fma(e, make_float2(set_lt(l0.y, l0.x), set_lt(l1.y, l1.x)), sqlt2);
+  }
 }
 
 template <typename T, bool NEED_Q1>
@@ -371,26 +474,38 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int nvec = (int)min((int64_t)CH, a.V - e0) / E;
         const uint4* P = reinterpret_cast<const uint4*>(ring + slot * kSlotBytes);
         const uint4* Q = reinterpret_cast<const uint4*>(ring + slot * kSlotBytes + kHalfSlot);
-        for (int i = t; i < nvec; i += kGroupThreads)
-          phase1_vec<T, NEED_Q1>(A, P[i], Q[i], e0 + (int64_t)i * E, a.sT);
+        if (sizeof(T) == 2 && nvec == 2 * kGroupThreads) {
+          const int i1 = t + kGroupThreads;
+          phase1_bf16x16<NEED_Q1>(A, P[t], P[i1], Q[t], Q[i1], e0 + (int64_t)t * E, e0 + (int64_t)i1 * E, a.sT);
+        } else {
+          for (int i = t; i < nvec; i += kGroupThreads)
+            phase1_vec<T, NEED_Q1>(A, P[i], Q[i], e0 + (int64_t)i * E, a.sT);
+        }
       }
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) A = part_merge(A, part_shfl(A, off));
       if (lane == 0) S.red1[j & 1][w] = A;
       named_barrier(kBarP1, kGroupThreads);
-      if (t == 0 && !*abort_flag) {
-        Part tot = S.red1[j & 1][0];
-        for (int k = 1; k < kP1Warps; ++k) tot = part_merge(tot, S.red1[j & 1][k]);
+      if (w == 0) {
+        // lanes 0..7 hold the warp partials; a fixed butterfly over them (the other lanes
+        // carry the identity) gives every lane the CTA partial
+        Part tot;
+        if (lane < kP1Warps) tot = S.red1[j & 1][lane];
+        else part_init(tot);
+#pragma unroll
+        for (int off = kP1Warps / 2; off > 0; off >>= 1) tot = part_merge(tot, part_shfl(tot, off));
+        tot = part_shfl(tot, 0 ^ lane);  // lane 0's value to every lane (butterfly: all equal)
         const int s = (int)(j % kXDepth);
-        if (wait_phase<true>(&S.xempty[s], ((j / kXDepth) & 1u) ^ 1u, abort_flag, limit_ns, hdr)) {
+        bool ok = false;
+        if (lane == 0) ok = wait_phase<true>(&S.xempty[s], ((j / kXDepth) & 1u) ^ 1u, abort_flag, limit_ns, hdr);
+        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+        if (ok && lane < C) {  // lane c writes this CTA's partial into peer c, then signals it
           const uint4* src = reinterpret_cast<const uint4*>(&tot);
-          for (int cr = 0; cr < C; ++cr) {
-            uint4* dst = reinterpret_cast<uint4*>(&S.xpart[s][rank]);
-            st_remote(dst + 0, (uint32_t)cr, src[0]);
-            st_remote(dst + 1, (uint32_t)cr, src[1]);
-            st_remote(dst + 2, (uint32_t)cr, src[2]);
-          }
-          for (int cr = 0; cr < C; ++cr) mbar_arrive_remote(&S.xfull[s], (uint32_t)cr);
+          uint4* dst = reinterpret_cast<uint4*>(&S.xpart[s][rank]);
+          st_remote(dst + 0, (uint32_t)lane, src[0]);
+          st_remote(dst + 1, (uint32_t)lane, src[1]);
+          st_remote(dst + 2, (uint32_t)lane, src[2]);
+          mbar_arrive_remote(&S.xfull[s], (uint32_t)lane);
         }
       }
       __syncwarp();
@@ -416,6 +531,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       const float Mp = tot.pM, Lsp = log2f(tot.pS);
       const float Mq = tot.qM, Lsq = log2f(tot.qS);
       float smin = 0.f, sqlt = 0.f;
+      float2 smin2 = make_float2(0.f, 0.f), sqlt2 = make_float2(0.f, 0.f);
+      const float2 s2 = make_float2(a.sT, a.sT), negM = make_float2(-Mp, -Mq), negLs = make_float2(-Lsp, -Lsq);
       for (int c = c0; c < c1; ++c, ++g) {
         const int slot = (int)(g % kSlots);
         if (wait_phase<false>(&S.full[slot], (g / kSlots) & 1u, abort_flag, limit_ns, hdr)) {
@@ -423,11 +540,21 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int nvec = (int)min((int64_t)CH, a.V - e0) / E;
           const uint4* P = reinterpret_cast<const uint4*>(ring + slot * kSlotBytes);
           const uint4* Q = reinterpret_cast<const uint4*>(ring + slot * kSlotBytes + kHalfSlot);
-          for (int i = t; i < nvec; i += kGroupThreads) phase2_vec<T>(smin, sqlt, P[i], Q[i], a.sT, Mp, Lsp, Mq, Lsq);
+          if (sizeof(T) == 2 && nvec == 2 * kGroupThreads) {
+            const int i1 = t + kGroupThreads;
+            const uint4 pa = P[t], pb = P[i1], qa = Q[t], qb = Q[i1];
+            phase2_bf16x8(smin2, sqlt2, pa, qa, s2, negM, negLs);
+            phase2_bf16x8(smin2, sqlt2, pb, qb, s2, negM, negLs);
+          } else {
+            for (int i = t; i < nvec; i += kGroupThreads)
+              phase2_vec<T>(smin, sqlt, P[i], Q[i], a.sT, Mp, Lsp, Mq, Lsq);
+          }
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&S.empty[slot]);
       }
+      smin += smin2.x + smin2.y;
+      sqlt += sqlt2.x + sqlt2.y;
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) {
         smin += __shfl_xor_sync(0xffffffffu, smin, off);
