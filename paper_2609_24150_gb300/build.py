@@ -45,9 +45,13 @@ def _compile(src: str, extra) -> str:
 
 
 def build(verbose: bool = False, ptxas_info: bool = False) -> str:
-    """Compile every CUDA source and link libaal.so; returns its path."""
+    """Compile every CUDA source and link libaal.so; returns its path.
+
+    Extra nvcc flags may be given in the AAL_NVCC_FLAGS environment variable.
+    """
     os.makedirs(BUILD, exist_ok=True)
     extra = ["-Xptxas", "-v"] if ptxas_info else []
+    extra += os.environ.get("AAL_NVCC_FLAGS", "").split()
     with cf.ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
         objs = list(ex.map(lambda s: _compile(s, extra), SOURCES))
     tmp = LIB + ".tmp"

@@ -30,10 +30,6 @@ namespace {
 constexpr int kSlots = 13;                       // ring slots per CTA
 constexpr int kSlotBytes = 16384;                // 8 KB of z_p + 8 KB of z_q
 constexpr int kHalfSlot = kSlotBytes / 2;
-constexpr int kP1Warps = 8;
-constexpr int kP2Warps = 8;
-constexpr int kGroupThreads = 32 * kP1Warps;     // == 32 * kP2Warps
-constexpr int kThreads = 32 * (1 + kP1Warps + kP2Warps);
 constexpr int kXDepth = 4;                       // depth of the partial-exchange ring
 constexpr int kSlack = 3;                        // slots a row leaves free for the next row
 constexpr int kBarP1 = 1, kBarP2a = 2, kBarP2b = 3;
@@ -52,8 +48,8 @@ struct Smem {
   uint64_t xfull[kXDepth];
   uint64_t xempty[kXDepth];
   Part xpart[kXDepth][kMaxCluster];
-  Part red1[2][kP1Warps];
-  float2 red2[2][kP2Warps];
+  Part red1[2][8];
+  float2 red2[2][8];
   int abort_flag;
 };
 
@@ -248,6 +244,12 @@ __device__ __forceinline__ void unpack8<float>(const uint4& w, float* o) {
 }
 
 // ---- packed arithmetic (sm_100+): two fp32 lanes per instruction, exact IEEE rounding
+#ifdef AAL_SCALAR_PAIRS
+__device__ __forceinline__ float2 f2fma(float2 a, float2 b, float2 c) {
+  return make_float2(fmaf(a.x, b.x, c.x), fmaf(a.y, b.y, c.y));
+}
+__device__ __forceinline__ float2 f2add(float2 a, float2 b) { return make_float2(a.x + b.x, a.y + b.y); }
+#else
 __device__ __forceinline__ float2 f2fma(float2 a, float2 b, float2 c) {
   float2 d;
   asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\tmov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
@@ -264,6 +266,7 @@ __device__ __forceinline__ float2 f2add(float2 a, float2 b) {
       : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
   return d;
 }
+#endif
 __device__ __forceinline__ uint32_t bmax2(uint32_t a, uint32_t b) {
   uint32_t d;
   asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
@@ -397,9 +400,30 @@ __device__ __forceinline__ void phase2_vec(float& smin, float& sqlt, const uint4
 
 // ---------------------------------------------------------------- the kernel
 
-template <typename T, bool NEED_Q1>
-__global__ void __launch_bounds__(kThreads, 1)
+#ifndef AAL_GROUP_WARPS
+#define AAL_GROUP_WARPS 8
+#endif
+constexpr int kGroupWarps = AAL_GROUP_WARPS;  // warps in each of the two consumer groups
+constexpr int kVecPerChunk = kHalfSlot / 16;   // 16-byte vectors per tensor per chunk
+
+// Ring position: slot index and phase parity advanced one chunk at a time.
+struct RingPos {
+  int slot = 0;
+  uint32_t phase = 0;
+  __device__ __forceinline__ void next() {
+    if (++slot == kSlots) {
+      slot = 0;
+      phase ^= 1u;
+    }
+  }
+};
+
+template <typename T, bool NEED_Q1, int G>
+__global__ void __launch_bounds__(32 * (1 + 2 * G), 1)
     rowstats_cluster(RowStatsArgs a, int C, int m, int nch, uint64_t limit_ns) {
+  constexpr int GT = 32 * G;                // threads per consumer group
+  constexpr int NV = kVecPerChunk / GT;     // vectors per thread per full chunk
+  static_assert(NV * GT == kVecPerChunk, "group must tile the chunk");
   extern __shared__ __align__(1024) unsigned char smem[];
   unsigned char* ring = smem;
   Smem& S = *reinterpret_cast<Smem*>(smem + kSlots * kSlotBytes);
@@ -412,13 +436,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   constexpr int ES = sizeof(T);
   constexpr int E = 16 / ES;           // elements per 16-byte vector
   constexpr int CH = kHalfSlot / ES;   // elements per chunk per tensor
+  const int V = (int)a.V;
   const int c0 = (int)rank * m;
   const int c1 = min(nch, c0 + m);
+  const int nfull = V / CH;            // chunks [0, nfull) are full
 
   if (threadIdx.x == 0) {
     for (int k = 0; k < kSlots; ++k) {
       mbar_init(&S.full[k], 1);
-      mbar_init(&S.empty[k], kP2Warps);
+      mbar_init(&S.empty[k], G);
     }
     for (int k = 0; k < kXDepth; ++k) {
       mbar_init(&S.xfull[k], (uint32_t)C);
@@ -433,68 +459,68 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------ producer
     if (lane == 0) {
       const uint64_t pol = evict_first_policy();
-      uint32_t g = 0;
-      for (int64_t r = cid; r < a.R; r += ncl) {
+      RingPos pos;
+      uint32_t issued = 0;
+      for (int64_t r = cid; r < a.R && !*abort_flag; r += ncl) {
         const char* prow = static_cast<const char*>(a.zp) + r * a.V * ES;
         const char* qrow = static_cast<const char*>(a.zq) + r * a.V * ES;
-        for (int c = c0; c < c1; ++c, ++g) {
-          if (*abort_flag) break;
-          const int slot = (int)(g % kSlots);
-          const uint32_t ph = (g / kSlots) & 1u;
-          if (!wait_phase<false>(&S.empty[slot], ph ^ 1u, abort_flag, limit_ns, hdr)) break;
-          const int64_t e0 = (int64_t)c * CH;
-          const int len = (int)min((int64_t)CH, a.V - e0);
-          const uint32_t bytes = (uint32_t)(len * ES);
-          mbar_expect_tx(&S.full[slot], 2u * bytes);
-          bulk_load(ring + slot * kSlotBytes, prow + e0 * ES, bytes, &S.full[slot], pol);
-          bulk_load(ring + slot * kSlotBytes + kHalfSlot, qrow + e0 * ES, bytes, &S.full[slot], pol);
+        for (int c = c0; c < c1; ++c) {
+          if (!wait_phase<false>(&S.empty[pos.slot], pos.phase ^ 1u, abort_flag, limit_ns, hdr)) break;
+          const int e0 = c * CH;
+          const uint32_t bytes = (uint32_t)(min(CH, V - e0) * ES);
+          mbar_expect_tx(&S.full[pos.slot], 2u * bytes);
+          bulk_load(ring + pos.slot * kSlotBytes, prow + (int64_t)e0 * ES, bytes, &S.full[pos.slot], pol);
+          bulk_load(ring + pos.slot * kSlotBytes + kHalfSlot, qrow + (int64_t)e0 * ES, bytes, &S.full[pos.slot], pol);
+          pos.next();
+          ++issued;
         }
-        if (*abort_flag) break;
       }
       // drain: every copy issued must have landed before the CTA may exit
-      const uint32_t first = g > (uint32_t)kSlots ? g - (uint32_t)kSlots : 0u;
-      for (uint32_t j = first; j < g; ++j) {
+      const uint32_t first = issued > (uint32_t)kSlots ? issued - (uint32_t)kSlots : 0u;
+      for (uint32_t j = first; j < issued; ++j) {
         const uint64_t t0 = now_ns();
         for (uint32_t it = 0; it < kSpinLimit && !mbar_test(&S.full[j % kSlots], (j / kSlots) & 1u); ++it)
           if (now_ns() - t0 > limit_ns) break;
       }
     }
-  } else if (warp <= kP1Warps) {
+  } else if (warp <= G) {
     // ------------------------------------------------------------ phase 1
     const int t = threadIdx.x - 32;
     const int w = t >> 5;
-    uint32_t g = 0, j = 0;
+    RingPos pos;
+    uint32_t j = 0;
     for (int64_t r = cid; r < a.R; r += ncl, ++j) {
       Part A;
       part_init(A);
-      for (int c = c0; c < c1; ++c, ++g) {
-        const int slot = (int)(g % kSlots);
-        if (!wait_phase<false>(&S.full[slot], (g / kSlots) & 1u, abort_flag, limit_ns, hdr)) continue;
-        const int64_t e0 = (int64_t)c * CH;
-        const int nvec = (int)min((int64_t)CH, a.V - e0) / E;
-        const uint4* P = reinterpret_cast<const uint4*>(ring + slot * kSlotBytes);
-        const uint4* Q = reinterpret_cast<const uint4*>(ring + slot * kSlotBytes + kHalfSlot);
-        if (sizeof(T) == 2 && nvec == 2 * kGroupThreads) {
-          const int i1 = t + kGroupThreads;
-          phase1_bf16x16<NEED_Q1>(A, P[t], P[i1], Q[t], Q[i1], e0 + (int64_t)t * E, e0 + (int64_t)i1 * E, a.sT);
+      for (int c = c0; c < c1; ++c, pos.next()) {
+        if (!wait_phase<false>(&S.full[pos.slot], pos.phase, abort_flag, limit_ns, hdr)) continue;
+        const int e0 = c * CH;
+        const uint4* P = reinterpret_cast<const uint4*>(ring + pos.slot * kSlotBytes);
+        const uint4* Q = reinterpret_cast<const uint4*>(ring + pos.slot * kSlotBytes + kHalfSlot);
+        if (sizeof(T) == 2 && c < nfull) {
+#pragma unroll
+          for (int v = 0; v < NV; v += 2) {
+            const int i0 = t + v * GT, i1 = i0 + GT;
+            phase1_bf16x16<NEED_Q1>(A, P[i0], P[i1], Q[i0], Q[i1], e0 + i0 * E, e0 + i1 * E, a.sT);
+          }
         } else {
-          for (int i = t; i < nvec; i += kGroupThreads)
-            phase1_vec<T, NEED_Q1>(A, P[i], Q[i], e0 + (int64_t)i * E, a.sT);
+          const int nvec = min(CH, V - e0) / E;
+          for (int i = t; i < nvec; i += GT) phase1_vec<T, NEED_Q1>(A, P[i], Q[i], e0 + i * E, a.sT);
         }
       }
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) A = part_merge(A, part_shfl(A, off));
       if (lane == 0) S.red1[j & 1][w] = A;
-      named_barrier(kBarP1, kGroupThreads);
+      named_barrier(kBarP1, GT);
       if (w == 0) {
-        // lanes 0..7 hold the warp partials; a fixed butterfly over them (the other lanes
-        // carry the identity) gives every lane the CTA partial
+        // lanes 0..G-1 hold the warp partials; a fixed butterfly over them (the other lanes
+        // carry the identity) leaves the CTA partial in lane 0
         Part tot;
-        if (lane < kP1Warps) tot = S.red1[j & 1][lane];
+        if (lane < G) tot = S.red1[j & 1][lane];
         else part_init(tot);
 #pragma unroll
-        for (int off = kP1Warps / 2; off > 0; off >>= 1) tot = part_merge(tot, part_shfl(tot, off));
-        tot = part_shfl(tot, 0 ^ lane);  // lane 0's value to every lane (butterfly: all equal)
+        for (int off = G / 2; off > 0; off >>= 1) tot = part_merge(tot, part_shfl(tot, off));
+        tot = part_shfl(tot, lane);  // lane 0's value to every lane
         const int s = (int)(j % kXDepth);
         bool ok = false;
         if (lane == 0) ok = wait_phase<true>(&S.xempty[s], ((j / kXDepth) & 1u) ^ 1u, abort_flag, limit_ns, hdr);
@@ -512,9 +538,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ------------------------------------------------------------ phase 2
-    const int t = threadIdx.x - 32 * (1 + kP1Warps);
+    const int t = threadIdx.x - 32 * (1 + G);
     const int w = t >> 5;
-    uint32_t g = 0, j = 0;
+    RingPos pos;
+    uint32_t j = 0;
     for (int64_t r = cid; r < a.R; r += ncl, ++j) {
       const int s = (int)(j % kXDepth);
       Part tot;
@@ -524,7 +551,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tot = S.xpart[s][0];
         for (int k = 1; k < C; ++k) tot = part_merge(tot, S.xpart[s][k]);
       }
-      named_barrier(kBarP2a, kGroupThreads);  // every phase-2 thread has read the exchange slot
+      named_barrier(kBarP2a, GT);  // every phase-2 thread has read the exchange slot
       if (t == 0 && ok && !*abort_flag)
         for (int cr = 0; cr < C; ++cr) mbar_arrive_remote(&S.xempty[s], (uint32_t)cr);
       __syncwarp();
@@ -533,25 +560,24 @@ __global__ void __launch_bounds__(kThreads, 1)
       float smin = 0.f, sqlt = 0.f;
       float2 smin2 = make_float2(0.f, 0.f), sqlt2 = make_float2(0.f, 0.f);
       const float2 s2 = make_float2(a.sT, a.sT), negM = make_float2(-Mp, -Mq), negLs = make_float2(-Lsp, -Lsq);
-      for (int c = c0; c < c1; ++c, ++g) {
-        const int slot = (int)(g % kSlots);
-        if (wait_phase<false>(&S.full[slot], (g / kSlots) & 1u, abort_flag, limit_ns, hdr)) {
-          const int64_t e0 = (int64_t)c * CH;
-          const int nvec = (int)min((int64_t)CH, a.V - e0) / E;
-          const uint4* P = reinterpret_cast<const uint4*>(ring + slot * kSlotBytes);
-          const uint4* Q = reinterpret_cast<const uint4*>(ring + slot * kSlotBytes + kHalfSlot);
-          if (sizeof(T) == 2 && nvec == 2 * kGroupThreads) {
-            const int i1 = t + kGroupThreads;
-            const uint4 pa = P[t], pb = P[i1], qa = Q[t], qb = Q[i1];
-            phase2_bf16x8(smin2, sqlt2, pa, qa, s2, negM, negLs);
-            phase2_bf16x8(smin2, sqlt2, pb, qb, s2, negM, negLs);
+      for (int c = c0; c < c1; ++c, pos.next()) {
+        if (wait_phase<false>(&S.full[pos.slot], pos.phase, abort_flag, limit_ns, hdr)) {
+          const int e0 = c * CH;
+          const uint4* P = reinterpret_cast<const uint4*>(ring + pos.slot * kSlotBytes);
+          const uint4* Q = reinterpret_cast<const uint4*>(ring + pos.slot * kSlotBytes + kHalfSlot);
+          if (sizeof(T) == 2 && c < nfull) {
+#pragma unroll
+            for (int v = 0; v < NV; ++v) {
+              const int i = t + v * GT;
+              phase2_bf16x8(smin2, sqlt2, P[i], Q[i], s2, negM, negLs);
+            }
           } else {
-            for (int i = t; i < nvec; i += kGroupThreads)
-              phase2_vec<T>(smin, sqlt, P[i], Q[i], a.sT, Mp, Lsp, Mq, Lsq);
+            const int nvec = min(CH, V - e0) / E;
+            for (int i = t; i < nvec; i += GT) phase2_vec<T>(smin, sqlt, P[i], Q[i], a.sT, Mp, Lsp, Mq, Lsq);
           }
         }
         __syncwarp();
-        if (lane == 0) mbar_arrive(&S.empty[slot]);
+        if (lane == 0) mbar_arrive(&S.empty[pos.slot]);
       }
       smin += smin2.x + smin2.y;
       sqlt += sqlt2.x + sqlt2.y;
@@ -561,10 +587,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         sqlt += __shfl_xor_sync(0xffffffffu, sqlt, off);
       }
       if (lane == 0) S.red2[j & 1][w] = make_float2(smin, sqlt);
-      named_barrier(kBarP2b, kGroupThreads);
+      named_barrier(kBarP2b, GT);
       if (t == 0 && !*abort_flag) {
         float2 x = S.red2[j & 1][0];
-        for (int k = 1; k < kP2Warps; ++k) {
+        for (int k = 1; k < G; ++k) {
           x.x += S.red2[j & 1][k].x;
           x.y += S.red2[j & 1][k].y;
         }
@@ -594,7 +620,7 @@ constexpr size_t kSmemBytes = (size_t)kSlots * kSlotBytes + sizeof(Smem);
 template <typename T, bool NEED_Q1>
 cudaError_t launch_T(const RowStatsArgs& a, cudaStream_t s, int C, int m, int nch, uint64_t limit_ns,
                      bool* launched) {
-  auto kern = rowstats_cluster<T, NEED_Q1>;
+  auto kern = rowstats_cluster<T, NEED_Q1, kGroupWarps>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
@@ -605,7 +631,7 @@ cudaError_t launch_T(const RowStatsArgs& a, cudaStream_t s, int C, int m, int nc
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  cfg.blockDim = dim3(kThreads);
+  cfg.blockDim = dim3(32 * (1 + 2 * kGroupWarps));
   cfg.dynamicSmemBytes = kSmemBytes;
   cfg.stream = s;
   cfg.gridDim = dim3((unsigned)C);
