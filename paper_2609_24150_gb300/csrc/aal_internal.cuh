@@ -202,6 +202,7 @@ struct RewardGroupArgs {
 
 // Launchers (return cudaGetLastError() of their launches).
 cudaError_t launch_rowstats(const RowStatsArgs& a, bool bf16, cudaStream_t s, int* cluster_used);
+cudaError_t launch_rowstats_stream(const RowStatsArgs& a, bool bf16, cudaStream_t s, uint64_t limit_ns);
 int rowstats_cluster_width(int64_t V, int elt, int* m_out, int* nch_out);
 cudaError_t launch_rowstats_cluster(const RowStatsArgs& a, bool bf16, cudaStream_t s, int C, int m, int nch,
                                     uint64_t limit_ns, bool* launched);

@@ -224,6 +224,12 @@ cudaError_t launch_rowstats(const RowStatsArgs& a, bool bf16, cudaStream_t s, in
   const int elt = bf16 ? 2 : 4;
   const bool aligned = ((a.V * elt) % 16 == 0) &&
                        ((reinterpret_cast<uintptr_t>(a.zq) | reinterpret_cast<uintptr_t>(a.zp)) % 16 == 0);
+#ifndef AAL_FWD_CLUSTER
+  if (a.overlap && aligned) {
+    *cluster_used = 1;
+    return launch_rowstats_stream(a, bf16, s, kWaitLimitNs);
+  }
+#else
   if (a.overlap && aligned) {
     int m = 0, nch = 0;
     const int C = rowstats_cluster_width(a.V, elt, &m, &nch);
@@ -236,6 +242,7 @@ cudaError_t launch_rowstats(const RowStatsArgs& a, bool bf16, cudaStream_t s, in
       }
     }
   }
+#endif
   *cluster_used = 1;
   return bf16 ? launch_generic<uint16_t>(a, s) : launch_generic<float>(a, s);
 }

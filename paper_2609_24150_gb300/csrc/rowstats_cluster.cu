@@ -31,7 +31,10 @@ constexpr int kSlots = 13;                       // ring slots per CTA
 constexpr int kSlotBytes = 16384;                // 8 KB of z_p + 8 KB of z_q
 constexpr int kHalfSlot = kSlotBytes / 2;
 constexpr int kXDepth = 4;                       // depth of the partial-exchange ring
-constexpr int kSlack = 3;                        // slots a row leaves free for the next row
+#ifndef AAL_RING_SLACK
+#define AAL_RING_SLACK 3
+#endif
+constexpr int kSlack = AAL_RING_SLACK;           // slots a row leaves free for the next row
 constexpr int kBarP1 = 1, kBarP2a = 2, kBarP2b = 3;
 
 // A CTA's phase-1 partial of one row (48 bytes: three 16-byte DSMEM stores).

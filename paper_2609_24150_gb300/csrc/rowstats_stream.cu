@@ -1,0 +1,464 @@
+// Forward per-row statistics, GB300 path: whole rows per CTA, streamed twice through a
+// shared-memory ring by the Tensor Memory Accelerator.
+//
+// Same outputs as the generic kernel in rowstats.cu: the normalisers (M, Ls) of z_p/T,
+// z_q/T and z_q, x* = argmax z_p with a^greedy = q(x*) (Eq. acc_greedy), and the sums
+// a^sample = sum_v min(p~_v, q~_v) (Eq. acc_sample) and Qlt = sum_{q~_v < p~_v} q~_v.
+// a^sample needs both normalisers first, so every row is visited twice:
+//
+//   * One producer thread per CTA walks its rows and, for each, issues the row's chunks
+//     twice into a FIFO ring of shared-memory slots with 1-D TMA bulk copies (completion
+//     counted in bytes on an mbarrier per slot).  The first pass comes from HBM and is kept
+//     in L2 (evict_last); the second pass, a row later at most, is served from L2 and is
+//     marked evict_first.  Slots are released as soon as a chunk has been consumed, so the
+//     copies run ahead of the arithmetic by the whole ring.
+//   * The consumer warps fold each first-pass chunk into online max / log-sum-exp / argmax
+//     state, reduce it across the CTA at the end of the row, then fold each second-pass
+//     chunk into the overlap sums.  The producer keeps streaming through that reduction.
+//
+// There is no cross-CTA communication, so all 152 SMs run one CTA each.  Every wait is
+// bounded (ptx::wait_phase); after a timeout every thread keeps walking the same loops
+// without waiting or computing, so all meet the same named barriers, the producer drains
+// its copies, and the kernel returns with AAL_ERR_TIMEOUT in the workspace status word.
+#include "ptx.cuh"
+
+namespace aal {
+namespace {
+
+using namespace ptx;
+
+constexpr int kSlots = 13;          // ring slots
+constexpr int kSlotBytes = 16384;   // 8 KB of z_p + 8 KB of z_q
+constexpr int kHalfSlot = kSlotBytes / 2;
+constexpr int kVecPerChunk = kHalfSlot / 16;
+#ifndef AAL_STREAM_WARPS
+#define AAL_STREAM_WARPS 8
+#endif
+constexpr int kWarps = AAL_STREAM_WARPS;  // consumer warps
+constexpr int kConsumers = 32 * kWarps;
+constexpr int kThreads = 32 + kConsumers;
+constexpr int kNV = kVecPerChunk / kConsumers;  // 16-byte vectors per thread per full chunk
+static_assert(kNV * kConsumers == kVecPerChunk, "consumers must tile a chunk");
+constexpr int kBarRow = 1, kBarSum = 2;
+
+// Phase-1 state of a thread, a warp or a row.
+struct RowPart {
+  float pM, pS, qM, qS, q1M, q1S;  // online log2-sum-exp states (M = max of z*s)
+  float av, ac;                    // running max of z_p and z_q at its first position
+  int32_t ai;                      // that position
+};
+
+struct Smem {
+  uint64_t full[kSlots];
+  uint64_t empty[kSlots];
+  RowPart red[kWarps];
+  float2 red2[2][kWarps];
+  int abort_flag;
+};
+
+__device__ __forceinline__ void part_init(RowPart& a) {
+  a.pM = a.qM = a.q1M = -INFINITY;
+  a.pS = a.qS = a.q1S = 0.f;
+  a.av = -INFINITY;
+  a.ac = 0.f;
+  a.ai = 0x7fffffff;
+}
+
+// Butterfly reductions over a warp: every lane ends with the same, order-fixed result.
+__device__ __forceinline__ void warp_lse(float& M, float& S) {
+  float m = M;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
+  float s = (M == -INFINITY) ? 0.f : S * ex2(M - m);
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+  M = m;
+  S = s;
+}
+__device__ __forceinline__ void warp_amax(float& v, int32_t& i, float& c) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    const float v2 = __shfl_xor_sync(0xffffffffu, v, off);
+    const int32_t i2 = __shfl_xor_sync(0xffffffffu, i, off);
+    const float c2 = __shfl_xor_sync(0xffffffffu, c, off);
+    if (v2 > v || (v2 == v && i2 < i)) {
+      v = v2;
+      i = i2;
+      c = c2;
+    }
+  }
+}
+template <bool NEED_Q1>
+__device__ __forceinline__ void warp_part(RowPart& a) {
+  warp_lse(a.pM, a.pS);
+  warp_lse(a.qM, a.qS);
+  if (NEED_Q1) warp_lse(a.q1M, a.q1S);
+  warp_amax(a.av, a.ai, a.ac);
+}
+
+// ---------------------------------------------------------------- per-chunk arithmetic
+
+// Fold n bf16 words (2n values) of one tensor into (M, S); vmax is their maximum.
+template <int NW>
+__device__ __forceinline__ void lse_words(float& M, float& S, const uint32_t* w, float vmax, float s) {
+  const float xm = __fmul_rn(vmax, s);
+  if (xm > M) {
+    S *= ex2(M - xm);  // M == -inf: ex2(-inf) = 0 and S is still 0
+    M = xm;
+  }
+  if (M == -INFINITY) return;
+  const float2 s2 = make_float2(s, s), m2 = make_float2(-M, -M);
+  float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
+#pragma unroll
+  for (int k = 0; k < NW; k += 2) {
+    const float2 x0 = f2fma(bpair(w[k]), s2, m2);
+    acc0 = f2add(acc0, make_float2(ex2(x0.x), ex2(x0.y)));
+    if (k + 1 < NW) {
+      const float2 x1 = f2fma(bpair(w[k + 1]), s2, m2);
+      acc1 = f2add(acc1, make_float2(ex2(x1.x), ex2(x1.y)));
+    }
+  }
+  const float2 t = f2add(acc0, acc1);
+  S += t.x + t.y;
+}
+
+// Phase 1 on NV 16-byte vectors of bf16 per tensor; vector v holds elements
+// idx0 + v * vstride + [0, 8).
+template <int NV, bool NEED_Q1>
+__device__ __forceinline__ void phase1_bf16(RowPart& A, const uint4* pv, const uint4* qv, int idx0, int vstride,
+                                            float sT) {
+  constexpr int NW = 4 * NV;
+  uint32_t pw[NW], qw[NW];
+#pragma unroll
+  for (int v = 0; v < NV; ++v) {
+    pw[4 * v + 0] = pv[v].x;
+    pw[4 * v + 1] = pv[v].y;
+    pw[4 * v + 2] = pv[v].z;
+    pw[4 * v + 3] = pv[v].w;
+    qw[4 * v + 0] = qv[v].x;
+    qw[4 * v + 1] = qv[v].y;
+    qw[4 * v + 2] = qv[v].z;
+    qw[4 * v + 3] = qv[v].w;
+  }
+  uint32_t pmw = pw[0], qmw = qw[0];
+#pragma unroll
+  for (int k = 1; k < NW; ++k) {
+    pmw = bmax2(pmw, pw[k]);
+    qmw = bmax2(qmw, qw[k]);
+  }
+  const float pm = fmaxf(bf16_lo(pmw), bf16_hi(pmw));
+  const float qm = fmaxf(bf16_lo(qmw), bf16_hi(qmw));
+  if (pm > A.av) {  // a new argmax of z_p: its first occurrence among these values
+    int e = 0;
+    float carry = 0.f;
+#pragma unroll
+    for (int k = 2 * NW - 1; k >= 0; --k) {
+      const float x = (k & 1) ? bf16_hi(pw[k >> 1]) : bf16_lo(pw[k >> 1]);
+      if (x == pm) {
+        e = k;
+        carry = (k & 1) ? bf16_hi(qw[k >> 1]) : bf16_lo(qw[k >> 1]);
+      }
+    }
+    A.av = pm;
+    A.ai = idx0 + (e >> 3) * vstride + (e & 7);
+    A.ac = carry;
+  }
+  lse_words<NW>(A.pM, A.pS, pw, pm, sT);
+  lse_words<NW>(A.qM, A.qS, qw, qm, sT);
+  if (NEED_Q1) lse_words<NW>(A.q1M, A.q1S, qw, qm, kLog2e);
+}
+
+// Phase 2 on one 16-byte vector of bf16 per tensor.
+__device__ __forceinline__ void phase2_bf16(float2& smin2, float2& sqlt2, const uint4& pw, const uint4& qw,
+                                            float2 s2, float2 negM, float2 negLs) {
+  const uint32_t pa[4] = {pw.x, pw.y, pw.z, pw.w};
+  const uint32_t qa[4] = {qw.x, qw.y, qw.z, qw.w};
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    // (p, q) lanes of elements 2k and 2k+1: log2 p~ and log2 q~
+    const float2 l0 = f2add(f2fma(make_float2(bf16_lo(pa[k]), bf16_lo(qa[k])), s2, negM), negLs);
+    const float2 l1 = f2add(f2fma(make_float2(bf16_hi(pa[k]), bf16_hi(qa[k])), s2, negM), negLs);
+    const float2 e = make_float2(ex2(fminf(l0.x, l0.y)), ex2(fminf(l1.x, l1.y)));
+    smin2 = f2add(smin2, e);
+    sqlt2 = f2fma(e, make_float2(set_lt(l0.y, l0.x), set_lt(l1.y, l1.x)), sqlt2);
+  }
+}
+
+// Scalar element paths (fp32 rows, and the partial last chunk of a bf16 row).
+template <typename T>
+__device__ __forceinline__ void unpack_vec(const uint4& w, float* o);
+template <>
+__device__ __forceinline__ void unpack_vec<uint16_t>(const uint4& w, float* o) {
+  o[0] = bf16_lo(w.x);
+  o[1] = bf16_hi(w.x);
+  o[2] = bf16_lo(w.y);
+  o[3] = bf16_hi(w.y);
+  o[4] = bf16_lo(w.z);
+  o[5] = bf16_hi(w.z);
+  o[6] = bf16_lo(w.w);
+  o[7] = bf16_hi(w.w);
+}
+template <>
+__device__ __forceinline__ void unpack_vec<float>(const uint4& w, float* o) {
+  o[0] = __uint_as_float(w.x);
+  o[1] = __uint_as_float(w.y);
+  o[2] = __uint_as_float(w.z);
+  o[3] = __uint_as_float(w.w);
+}
+
+template <int N>
+__device__ __forceinline__ void lse_vals(float& M, float& S, const float* v, float vmax, float s) {
+  const float xm = __fmul_rn(vmax, s);
+  if (xm > M) {
+    S *= ex2(M - xm);
+    M = xm;
+  }
+  if (M == -INFINITY) return;
+  float acc = 0.f;
+#pragma unroll
+  for (int e = 0; e < N; ++e) acc += ex2(fmaf(v[e], s, -M));
+  S += acc;
+}
+
+template <typename T, bool NEED_Q1>
+__device__ __forceinline__ void phase1_vec(RowPart& A, const uint4& pw, const uint4& qw, int idx0, float sT) {
+  constexpr int E = 16 / sizeof(T);
+  float pv[8], qv[8];
+  unpack_vec<T>(pw, pv);
+  unpack_vec<T>(qw, qv);
+  float pm = pv[0], qm = qv[0];
+#pragma unroll
+  for (int e = 1; e < E; ++e) {
+    pm = fmaxf(pm, pv[e]);
+    qm = fmaxf(qm, qv[e]);
+  }
+  if (pm > A.av) {
+    int e = 0;
+    float carry = qv[0];
+#pragma unroll
+    for (int k = E - 1; k >= 0; --k) {
+      if (pv[k] == pm) {
+        e = k;
+        carry = qv[k];
+      }
+    }
+    A.av = pm;
+    A.ai = idx0 + e;
+    A.ac = carry;
+  }
+  lse_vals<E>(A.pM, A.pS, pv, pm, sT);
+  lse_vals<E>(A.qM, A.qS, qv, qm, sT);
+  if (NEED_Q1) lse_vals<E>(A.q1M, A.q1S, qv, qm, kLog2e);
+}
+
+template <typename T>
+__device__ __forceinline__ void phase2_vec(float& smin, float& sqlt, const uint4& pw, const uint4& qw, float sT,
+                                           float Mp, float Lsp, float Mq, float Lsq) {
+  constexpr int E = 16 / sizeof(T);
+  float pv[8], qv[8];
+  unpack_vec<T>(pw, pv);
+  unpack_vec<T>(qw, qv);
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    const float lp = fmaf(pv[e], sT, -Mp) - Lsp;
+    const float lq = fmaf(qv[e], sT, -Mq) - Lsq;
+    const float t = ex2(fminf(lp, lq));
+    smin += t;
+    sqlt += (lq < lp) ? t : 0.f;
+  }
+}
+
+struct RingPos {
+  int slot = 0;
+  uint32_t phase = 0;
+  __device__ __forceinline__ void next() {
+    if (++slot == kSlots) {
+      slot = 0;
+      phase ^= 1u;
+    }
+  }
+};
+
+// ---------------------------------------------------------------- the kernel
+
+template <typename T, bool NEED_Q1>
+__global__ void __launch_bounds__(kThreads, 1) rowstats_stream(RowStatsArgs a, int nch, uint64_t limit_ns) {
+  extern __shared__ __align__(1024) unsigned char smem[];
+  unsigned char* ring = smem;
+  Smem& S = *reinterpret_cast<Smem*>(smem + kSlots * kSlotBytes);
+  volatile int* abort_flag = &S.abort_flag;
+  WsHeader* hdr = a.ws.hdr;
+  constexpr int ES = sizeof(T);
+  constexpr int E = 16 / ES;          // elements per 16-byte vector
+  constexpr int CH = kHalfSlot / ES;  // elements per chunk per tensor
+  const int V = (int)a.V;
+  const int nfull = V / CH;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int k = 0; k < kSlots; ++k) {
+      mbar_init(&S.full[k], 1);
+      mbar_init(&S.empty[k], kWarps);
+    }
+    S.abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+
+  if (warp == kWarps) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      const uint64_t keep = policy_evict_last(), drop = policy_evict_first();
+      RingPos pos;
+      uint32_t issued = 0;
+      for (int64_t r = blockIdx.x; r < a.R && !*abort_flag; r += gridDim.x) {
+        const char* prow = static_cast<const char*>(a.zp) + r * a.V * ES;
+        const char* qrow = static_cast<const char*>(a.zq) + r * a.V * ES;
+        for (int pass = 0; pass < 2 && !*abort_flag; ++pass) {
+          const uint64_t pol = pass == 0 ? keep : drop;
+          for (int c = 0; c < nch; ++c) {
+            if (!wait_phase(&S.empty[pos.slot], pos.phase ^ 1u, abort_flag, limit_ns, hdr)) break;
+            const int e0 = c * CH;
+            const uint32_t bytes = (uint32_t)(min(CH, V - e0) * ES);
+            mbar_expect_tx(&S.full[pos.slot], 2u * bytes);
+            bulk_load(ring + pos.slot * kSlotBytes, prow + (int64_t)e0 * ES, bytes, &S.full[pos.slot], pol);
+            bulk_load(ring + pos.slot * kSlotBytes + kHalfSlot, qrow + (int64_t)e0 * ES, bytes, &S.full[pos.slot], pol);
+            pos.next();
+            ++issued;
+          }
+        }
+      }
+      // drain: every copy issued must have landed before the CTA may exit
+      const uint32_t first = issued > (uint32_t)kSlots ? issued - (uint32_t)kSlots : 0u;
+      for (uint32_t j = first; j < issued; ++j) {
+        const uint64_t t0 = now_ns();
+        for (uint32_t it = 0; it < kSpinLimit && !mbar_try(&S.full[j % kSlots], (j / kSlots) & 1u, 100000); ++it)
+          if (now_ns() - t0 > limit_ns) break;
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ consumers
+    const int t = threadIdx.x;
+    RingPos pos;
+    uint32_t j = 0;
+    for (int64_t r = blockIdx.x; r < a.R; r += gridDim.x, ++j) {
+      // pass 1: online normalisers and argmax
+      RowPart A;
+      part_init(A);
+      for (int c = 0; c < nch; ++c, pos.next()) {
+        if (wait_phase(&S.full[pos.slot], pos.phase, abort_flag, limit_ns, hdr)) {
+          const int e0 = c * CH;
+          const uint4* P = reinterpret_cast<const uint4*>(ring + pos.slot * kSlotBytes);
+          const uint4* Q = reinterpret_cast<const uint4*>(ring + pos.slot * kSlotBytes + kHalfSlot);
+          if (sizeof(T) == 2 && c < nfull) {
+            uint4 pv[kNV], qv[kNV];
+#pragma unroll
+            for (int v = 0; v < kNV; ++v) {
+              pv[v] = P[t + v * kConsumers];
+              qv[v] = Q[t + v * kConsumers];
+            }
+            phase1_bf16<kNV, NEED_Q1>(A, pv, qv, e0 + t * E, kConsumers * E, a.sT);
+          } else {
+            const int nvec = min(CH, V - e0) / E;
+            for (int i = t; i < nvec; i += kConsumers) phase1_vec<T, NEED_Q1>(A, P[i], Q[i], e0 + i * E, a.sT);
+          }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&S.empty[pos.slot]);
+      }
+      warp_part<NEED_Q1>(A);
+      if (lane == 0) S.red[warp] = A;
+      named_barrier(kBarRow, kConsumers);
+      // every warp combines the warp partials itself (lanes >= kWarps carry the identity)
+      RowPart tot;
+      if (lane < kWarps) tot = S.red[lane];
+      else part_init(tot);
+      warp_part<NEED_Q1>(tot);
+      const float Mp = tot.pM, Lsp = log2f(tot.pS);
+      const float Mq = tot.qM, Lsq = log2f(tot.qS);
+
+      // pass 2: overlap sums
+      float smin = 0.f, sqlt = 0.f;
+      float2 smin2 = make_float2(0.f, 0.f), sqlt2 = make_float2(0.f, 0.f);
+      const float2 s2 = make_float2(a.sT, a.sT), negM = make_float2(-Mp, -Mq), negLs = make_float2(-Lsp, -Lsq);
+      for (int c = 0; c < nch; ++c, pos.next()) {
+        if (wait_phase(&S.full[pos.slot], pos.phase, abort_flag, limit_ns, hdr)) {
+          const int e0 = c * CH;
+          const uint4* P = reinterpret_cast<const uint4*>(ring + pos.slot * kSlotBytes);
+          const uint4* Q = reinterpret_cast<const uint4*>(ring + pos.slot * kSlotBytes + kHalfSlot);
+          if (sizeof(T) == 2 && c < nfull) {
+#pragma unroll
+            for (int v = 0; v < kNV; ++v) {
+              const int i = t + v * kConsumers;
+              phase2_bf16(smin2, sqlt2, P[i], Q[i], s2, negM, negLs);
+            }
+          } else {
+            const int nvec = min(CH, V - e0) / E;
+            for (int i = t; i < nvec; i += kConsumers) phase2_vec<T>(smin, sqlt, P[i], Q[i], a.sT, Mp, Lsp, Mq, Lsq);
+          }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&S.empty[pos.slot]);
+      }
+      smin += smin2.x + smin2.y;
+      sqlt += sqlt2.x + sqlt2.y;
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) {
+        smin += __shfl_xor_sync(0xffffffffu, smin, off);
+        sqlt += __shfl_xor_sync(0xffffffffu, sqlt, off);
+      }
+      if (lane == 0) S.red2[j & 1][warp] = make_float2(smin, sqlt);
+      named_barrier(kBarSum, kConsumers);
+      if (t == 0 && !*abort_flag) {
+        float2 x = S.red2[j & 1][0];
+        for (int k = 1; k < kWarps; ++k) {
+          x.x += S.red2[j & 1][k].x;
+          x.y += S.red2[j & 1][k].y;
+        }
+        const float Mq1 = NEED_Q1 ? tot.q1M : Mq;
+        const float Lsq1 = NEED_Q1 ? log2f(tot.q1S) : Lsq;
+        a.ws.cpart[r * kMaxCluster] = x;
+        a.ws.Mp[r] = Mp;
+        a.ws.Lsp[r] = Lsp;
+        a.ws.Mq[r] = Mq;
+        a.ws.Lsq[r] = Lsq;
+        a.ws.Mq1[r] = Mq1;
+        a.ws.Lsq1[r] = Lsq1;
+        a.ws.xstar[r] = tot.ai;
+        a.ws.ag[r] = exp2f(log2_prob(tot.ac, kLog2e, Mq1, Lsq1));
+      }
+      __syncwarp();
+    }
+  }
+  __syncwarp();
+  __syncthreads();
+}
+
+constexpr size_t kSmemBytes = (size_t)kSlots * kSlotBytes + sizeof(Smem);
+
+template <typename T, bool NEED_Q1>
+cudaError_t launch_T(const RowStatsArgs& a, cudaStream_t s, int nch, uint64_t limit_ns) {
+  auto kern = rowstats_stream<T, NEED_Q1>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+  if (e != cudaSuccess) return e;
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  int64_t grid = sms;
+  if (grid > a.R) grid = a.R;
+  if (grid < 1) return cudaSuccess;
+  kern<<<(unsigned)grid, kThreads, kSmemBytes, s>>>(a, nch, limit_ns);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_rowstats_stream(const RowStatsArgs& a, bool bf16, cudaStream_t s, uint64_t limit_ns) {
+  const int elt = bf16 ? 2 : 4;
+  const int64_t CH = kHalfSlot / elt;
+  const int nch = (int)((a.V + CH - 1) / CH);
+  if (bf16) return a.need_q1 ? launch_T<uint16_t, true>(a, s, nch, limit_ns) : launch_T<uint16_t, false>(a, s, nch, limit_ns);
+  return a.need_q1 ? launch_T<float, true>(a, s, nch, limit_ns) : launch_T<float, false>(a, s, nch, limit_ns);
+}
+
+}  // namespace aal
