@@ -168,19 +168,22 @@ __device__ __forceinline__ void phase1_bf16(RowPart& A, const uint4* pv, const u
   if (NEED_Q1) lse_words<NW>(A.q1M, A.q1S, qw, qm, kLog2e);
 }
 
-// Phase 2 on one 16-byte vector of bf16 per tensor.
+// Phase 2 on one 16-byte vector of bf16 per tensor.  Packed lanes pair the two elements
+// of one 32-bit word, so each unpacked pair already sits in a register pair.
+struct Norm2 {
+  float2 s, negMp, negLsp, negMq, negLsq;
+};
 __device__ __forceinline__ void phase2_bf16(float2& smin2, float2& sqlt2, const uint4& pw, const uint4& qw,
-                                            float2 s2, float2 negM, float2 negLs) {
+                                            const Norm2& n) {
   const uint32_t pa[4] = {pw.x, pw.y, pw.z, pw.w};
   const uint32_t qa[4] = {qw.x, qw.y, qw.z, qw.w};
 #pragma unroll
   for (int k = 0; k < 4; ++k) {
-    // (p, q) lanes of elements 2k and 2k+1: log2 p~ and log2 q~
-    const float2 l0 = f2add(f2fma(make_float2(bf16_lo(pa[k]), bf16_lo(qa[k])), s2, negM), negLs);
-    const float2 l1 = f2add(f2fma(make_float2(bf16_hi(pa[k]), bf16_hi(qa[k])), s2, negM), negLs);
-    const float2 e = make_float2(ex2(fminf(l0.x, l0.y)), ex2(fminf(l1.x, l1.y)));
+    const float2 lp = f2add(f2fma(bpair(pa[k]), n.s, n.negMp), n.negLsp);  // log2 p~ of 2 elements
+    const float2 lq = f2add(f2fma(bpair(qa[k]), n.s, n.negMq), n.negLsq);  // log2 q~ of the same
+    const float2 e = make_float2(ex2(fminf(lp.x, lq.x)), ex2(fminf(lp.y, lq.y)));
     smin2 = f2add(smin2, e);
-    sqlt2 = f2fma(e, make_float2(set_lt(l0.y, l0.x), set_lt(l1.y, l1.x)), sqlt2);
+    sqlt2 = f2fma(e, make_float2(set_lt(lq.x, lp.x), set_lt(lq.y, lp.y)), sqlt2);
   }
 }
 
@@ -380,7 +383,12 @@ __global__ void __launch_bounds__(kThreads, 1) rowstats_stream(RowStatsArgs a, i
       // pass 2: overlap sums
       float smin = 0.f, sqlt = 0.f;
       float2 smin2 = make_float2(0.f, 0.f), sqlt2 = make_float2(0.f, 0.f);
-      const float2 s2 = make_float2(a.sT, a.sT), negM = make_float2(-Mp, -Mq), negLs = make_float2(-Lsp, -Lsq);
+      Norm2 nrm;
+      nrm.s = make_float2(a.sT, a.sT);
+      nrm.negMp = make_float2(-Mp, -Mp);
+      nrm.negLsp = make_float2(-Lsp, -Lsp);
+      nrm.negMq = make_float2(-Mq, -Mq);
+      nrm.negLsq = make_float2(-Lsq, -Lsq);
       for (int c = 0; c < nch; ++c, pos.next()) {
         if (wait_phase(&S.full[pos.slot], pos.phase, abort_flag, limit_ns, hdr)) {
           const int e0 = c * CH;
@@ -390,7 +398,7 @@ __global__ void __launch_bounds__(kThreads, 1) rowstats_stream(RowStatsArgs a, i
 #pragma unroll
             for (int v = 0; v < kNV; ++v) {
               const int i = t + v * kConsumers;
-              phase2_bf16(smin2, sqlt2, P[i], Q[i], s2, negM, negLs);
+              phase2_bf16(smin2, sqlt2, P[i], Q[i], nrm);
             }
           } else {
             const int nvec = min(CH, V - e0) / E;

@@ -59,19 +59,17 @@ def test_ragged_vocab_and_window_sizes(V, dtype, K):
         check_loss(run, t, d, m, mode, T, 0.5, 0.5, dloss=5.0)
 
 
-@pytest.mark.parametrize("V,dtype,width", [(8, torch.bfloat16, 1), (65544, torch.bfloat16, 2),
-                                           (100000, torch.bfloat16, 4), (250000, torch.bfloat16, 8),
-                                           (167936, torch.bfloat16, 8), (40000, torch.float32, 2)])
-def test_cluster_widths(V, dtype, width):
-    """Rows split over 1, 2, 4 and 8 CTAs of a cluster (chosen from V), including a
-    single-vector row and a cluster whose last CTA holds a partial chunk."""
+@pytest.mark.parametrize("V,dtype", [(8, torch.bfloat16), (4096, torch.bfloat16), (4104, torch.bfloat16),
+                                     (65544, torch.bfloat16), (100000, torch.bfloat16),
+                                     (250000, torch.bfloat16), (40000, torch.float32)])
+def test_streamed_row_shapes(V, dtype):
+    """Rows of one vector, exactly one chunk, one chunk plus one vector, and many chunks with
+    a partial last chunk, through the TMA-streamed forward (row length a multiple of 16 B)."""
     target, draft, _ = synth.make_logits("tiny", seed=V, N=3, K=2, V=V, dtype=dtype)
     draft[1, 1] = target[1, 1]          # an identical row inside a window
     t, d = _dev(target, draft)
     for mode, T in [(aal.AAL_BOTH, 1.0), (aal.AAL_SAMPLING, 0.8), (aal.AAL_BOTH, 1.4)]:
         run = LossRun(t, d, None, mode, T, 0.5, 0.5, dloss=3.0)
-        hdr = run.ws_buf[:16].view(torch.int32).cpu()
-        assert int(hdr[3]) == width     # cluster width recorded in the workspace header
         check_loss(run, t, d, None, mode, T, 0.5, 0.5, dloss=3.0)
 
 
