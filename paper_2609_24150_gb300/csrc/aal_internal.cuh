@@ -203,9 +203,6 @@ struct RewardGroupArgs {
 // Launchers (return cudaGetLastError() of their launches).
 cudaError_t launch_rowstats(const RowStatsArgs& a, bool bf16, cudaStream_t s, int* cluster_used);
 cudaError_t launch_rowstats_stream(const RowStatsArgs& a, bool bf16, cudaStream_t s, uint64_t limit_ns);
-int rowstats_cluster_width(int64_t V, int elt, int* m_out, int* nch_out);
-cudaError_t launch_rowstats_cluster(const RowStatsArgs& a, bool bf16, cudaStream_t s, int C, int m, int nch,
-                                    uint64_t limit_ns, bool* launched);
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // bounded waits give up after 1 s
 cudaError_t launch_window(const WindowArgs& a, cudaStream_t s);
 cudaError_t launch_backward(const BackwardArgs& a, bool bf16, cudaStream_t s);

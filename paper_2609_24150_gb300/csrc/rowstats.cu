@@ -217,32 +217,17 @@ cudaError_t launch_generic(const RowStatsArgs& a, cudaStream_t s) {
 
 }  // namespace
 
-// The cluster kernel (rowstats_cluster.cu) serves rows whose byte length is a multiple
-// of 16 when the sampling term needs the second phase; everything else, and any device on
-// which the cluster shape cannot be made resident, takes the generic kernel.
+// The TMA-streamed kernel (rowstats_stream.cu) serves rows whose byte length is a
+// multiple of 16 when the sampling term needs the second pass; everything else takes the
+// generic kernel.
 cudaError_t launch_rowstats(const RowStatsArgs& a, bool bf16, cudaStream_t s, int* cluster_used) {
   const int elt = bf16 ? 2 : 4;
   const bool aligned = ((a.V * elt) % 16 == 0) &&
                        ((reinterpret_cast<uintptr_t>(a.zq) | reinterpret_cast<uintptr_t>(a.zp)) % 16 == 0);
-#ifndef AAL_FWD_CLUSTER
   if (a.overlap && aligned) {
     *cluster_used = 1;
     return launch_rowstats_stream(a, bf16, s, kWaitLimitNs);
   }
-#else
-  if (a.overlap && aligned) {
-    int m = 0, nch = 0;
-    const int C = rowstats_cluster_width(a.V, elt, &m, &nch);
-    if (C > 0) {
-      bool launched = false;
-      cudaError_t e = launch_rowstats_cluster(a, bf16, s, C, m, nch, kWaitLimitNs, &launched);
-      if (e != cudaSuccess || launched) {
-        *cluster_used = C;
-        return e;
-      }
-    }
-  }
-#endif
   *cluster_used = 1;
   return bf16 ? launch_generic<uint16_t>(a, s) : launch_generic<float>(a, s);
 }

@@ -27,12 +27,18 @@ namespace {
 
 using namespace ptx;
 
-constexpr int kSlots = 13;          // ring slots
-constexpr int kSlotBytes = 16384;   // 8 KB of z_p + 8 KB of z_q
+#ifndef AAL_STREAM_SLOTS
+#define AAL_STREAM_SLOTS 7
+#endif
+#ifndef AAL_STREAM_SLOT_KB
+#define AAL_STREAM_SLOT_KB 32
+#endif
+constexpr int kSlots = AAL_STREAM_SLOTS;               // ring slots
+constexpr int kSlotBytes = AAL_STREAM_SLOT_KB * 1024;  // half z_p, half z_q
 constexpr int kHalfSlot = kSlotBytes / 2;
 constexpr int kVecPerChunk = kHalfSlot / 16;
 #ifndef AAL_STREAM_WARPS
-#define AAL_STREAM_WARPS 8
+#define AAL_STREAM_WARPS 16
 #endif
 constexpr int kWarps = AAL_STREAM_WARPS;  // consumer warps
 constexpr int kConsumers = 32 * kWarps;
@@ -98,7 +104,9 @@ __device__ __forceinline__ void warp_part(RowPart& a) {
 
 // ---------------------------------------------------------------- per-chunk arithmetic
 
-// Fold n bf16 words (2n values) of one tensor into (M, S); vmax is their maximum.
+// Fold NW bf16 words (2 NW values) of one tensor into (M, S); vmax is their maximum.
+// Each value costs one fma (the bf16 operand is widened inside the instruction), one
+// ex2, and half a packed add.
 template <int NW>
 __device__ __forceinline__ void lse_words(float& M, float& S, const uint32_t* w, float vmax, float s) {
   const float xm = __fmul_rn(vmax, s);
@@ -107,16 +115,13 @@ __device__ __forceinline__ void lse_words(float& M, float& S, const uint32_t* w,
     M = xm;
   }
   if (M == -INFINITY) return;
-  const float2 s2 = make_float2(s, s), m2 = make_float2(-M, -M);
+  const float nM = -M;
   float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
 #pragma unroll
-  for (int k = 0; k < NW; k += 2) {
-    const float2 x0 = f2fma(bpair(w[k]), s2, m2);
-    acc0 = f2add(acc0, make_float2(ex2(x0.x), ex2(x0.y)));
-    if (k + 1 < NW) {
-      const float2 x1 = f2fma(bpair(w[k + 1]), s2, m2);
-      acc1 = f2add(acc1, make_float2(ex2(x1.x), ex2(x1.y)));
-    }
+  for (int k = 0; k < NW; ++k) {
+    const float2 e = make_float2(ex2(fmaf(bf16_lo(w[k]), s, nM)), ex2(fmaf(bf16_hi(w[k]), s, nM)));
+    if (k & 1) acc1 = f2add(acc1, e);
+    else acc0 = f2add(acc0, e);
   }
   const float2 t = f2add(acc0, acc1);
   S += t.x + t.y;
@@ -168,22 +173,19 @@ __device__ __forceinline__ void phase1_bf16(RowPart& A, const uint4* pv, const u
   if (NEED_Q1) lse_words<NW>(A.q1M, A.q1S, qw, qm, kLog2e);
 }
 
-// Phase 2 on one 16-byte vector of bf16 per tensor.  Packed lanes pair the two elements
-// of one 32-bit word, so each unpacked pair already sits in a register pair.
-struct Norm2 {
-  float2 s, negMp, negLsp, negMq, negLsq;
-};
+// Phase 2 on one 16-byte vector of bf16 per tensor, with the row normalisers folded into
+// one addend each (nLp = -(M_p + Ls_p)): log2 p~ = fma(z_p, s, nLp).
 __device__ __forceinline__ void phase2_bf16(float2& smin2, float2& sqlt2, const uint4& pw, const uint4& qw,
-                                            const Norm2& n) {
+                                            float s, float nLp, float nLq) {
   const uint32_t pa[4] = {pw.x, pw.y, pw.z, pw.w};
   const uint32_t qa[4] = {qw.x, qw.y, qw.z, qw.w};
 #pragma unroll
   for (int k = 0; k < 4; ++k) {
-    const float2 lp = f2add(f2fma(bpair(pa[k]), n.s, n.negMp), n.negLsp);  // log2 p~ of 2 elements
-    const float2 lq = f2add(f2fma(bpair(qa[k]), n.s, n.negMq), n.negLsq);  // log2 q~ of the same
-    const float2 e = make_float2(ex2(fminf(lp.x, lq.x)), ex2(fminf(lp.y, lq.y)));
+    const float lp0 = fmaf(bf16_lo(pa[k]), s, nLp), lp1 = fmaf(bf16_hi(pa[k]), s, nLp);
+    const float lq0 = fmaf(bf16_lo(qa[k]), s, nLq), lq1 = fmaf(bf16_hi(qa[k]), s, nLq);
+    const float2 e = make_float2(ex2(fminf(lp0, lq0)), ex2(fminf(lp1, lq1)));
     smin2 = f2add(smin2, e);
-    sqlt2 = f2fma(e, make_float2(set_lt(lq.x, lp.x), set_lt(lq.y, lp.y)), sqlt2);
+    sqlt2 = f2fma(e, make_float2(set_lt(lq0, lp0), set_lt(lq1, lp1)), sqlt2);
   }
 }
 
@@ -383,12 +385,8 @@ __global__ void __launch_bounds__(kThreads, 1) rowstats_stream(RowStatsArgs a, i
       // pass 2: overlap sums
       float smin = 0.f, sqlt = 0.f;
       float2 smin2 = make_float2(0.f, 0.f), sqlt2 = make_float2(0.f, 0.f);
-      Norm2 nrm;
-      nrm.s = make_float2(a.sT, a.sT);
-      nrm.negMp = make_float2(-Mp, -Mp);
-      nrm.negLsp = make_float2(-Lsp, -Lsp);
-      nrm.negMq = make_float2(-Mq, -Mq);
-      nrm.negLsq = make_float2(-Lsq, -Lsq);
+      // one-float normalisers for the overlap pass: |error| <= ulp(M + Ls) / 2 in log2 units
+      const float nLp = -(Mp + Lsp), nLq = -(Mq + Lsq);
       for (int c = 0; c < nch; ++c, pos.next()) {
         if (wait_phase(&S.full[pos.slot], pos.phase, abort_flag, limit_ns, hdr)) {
           const int e0 = c * CH;
@@ -398,7 +396,7 @@ __global__ void __launch_bounds__(kThreads, 1) rowstats_stream(RowStatsArgs a, i
 #pragma unroll
             for (int v = 0; v < kNV; ++v) {
               const int i = t + v * kConsumers;
-              phase2_bf16(smin2, sqlt2, P[i], Q[i], nrm);
+              phase2_bf16(smin2, sqlt2, P[i], Q[i], a.sT, nLp, nLq);
             }
           } else {
             const int nvec = min(CH, V - e0) / E;
