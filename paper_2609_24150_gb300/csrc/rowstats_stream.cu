@@ -47,11 +47,15 @@ constexpr int kNV = kVecPerChunk / kConsumers;  // 16-byte vectors per thread pe
 static_assert(kNV * kConsumers == kVecPerChunk, "consumers must tile a chunk");
 constexpr int kBarRow = 1, kBarSum = 2;
 
-// Phase-1 state of a thread, a warp or a row.
+// Phase-1 state of a thread, a warp or a row.  The target argmax is tracked per 16-byte
+// vector (8 contiguous elements): av is the largest z_p seen and ab the first element index
+// of the first vector that holds it.  Vectors are disjoint contiguous ranges, so the lowest
+// ab among equal av contains the first occurrence; the position inside that vector is
+// found in the second pass, by the one thread that streams the vector again.
 struct RowPart {
   float pM, pS, qM, qS, q1M, q1S;  // online log2-sum-exp states (M = max of z*s)
-  float av, ac;                    // running max of z_p and z_q at its first position
-  int32_t ai;                      // that position
+  float av;
+  int32_t ab;
 };
 
 struct Smem {
@@ -59,6 +63,8 @@ struct Smem {
   uint64_t empty[kSlots];
   RowPart red[kWarps];
   float2 red2[2][kWarps];
+  int32_t arg_index;  // x*, written by the thread that finds it in the second pass
+  float arg_carry;    // z_q at x*
   int abort_flag;
 };
 
@@ -66,8 +72,7 @@ __device__ __forceinline__ void part_init(RowPart& a) {
   a.pM = a.qM = a.q1M = -INFINITY;
   a.pS = a.qS = a.q1S = 0.f;
   a.av = -INFINITY;
-  a.ac = 0.f;
-  a.ai = 0x7fffffff;
+  a.ab = 0x7fffffff;
 }
 
 // Butterfly reductions over a warp: every lane ends with the same, order-fixed result.
@@ -81,16 +86,14 @@ __device__ __forceinline__ void warp_lse(float& M, float& S) {
   M = m;
   S = s;
 }
-__device__ __forceinline__ void warp_amax(float& v, int32_t& i, float& c) {
+__device__ __forceinline__ void warp_amax(float& v, int32_t& i) {
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
     const float v2 = __shfl_xor_sync(0xffffffffu, v, off);
     const int32_t i2 = __shfl_xor_sync(0xffffffffu, i, off);
-    const float c2 = __shfl_xor_sync(0xffffffffu, c, off);
     if (v2 > v || (v2 == v && i2 < i)) {
       v = v2;
       i = i2;
-      c = c2;
     }
   }
 }
@@ -99,7 +102,13 @@ __device__ __forceinline__ void warp_part(RowPart& a) {
   warp_lse(a.pM, a.pS);
   warp_lse(a.qM, a.qS);
   if (NEED_Q1) warp_lse(a.q1M, a.q1S);
-  warp_amax(a.av, a.ai, a.ac);
+  warp_amax(a.av, a.ab);
+}
+// A vector's maximum beats the running one: remember it and where its vector starts.
+__device__ __forceinline__ void amax_vec(RowPart& A, float vmax, int base) {
+  const bool take = vmax > A.av;
+  A.av = take ? vmax : A.av;
+  A.ab = take ? base : A.ab;
 }
 
 // ---------------------------------------------------------------- per-chunk arithmetic
@@ -116,6 +125,15 @@ __device__ __forceinline__ void lse_words(float& M, float& S, const uint32_t* w,
   }
   if (M == -INFINITY) return;
   const float nM = -M;
+#ifdef AAL_SCALAR_ACC
+  float acc0 = 0.f, acc1 = 0.f;
+#pragma unroll
+  for (int k = 0; k < NW; ++k) {
+    acc0 += ex2(fmaf(bf16_lo(w[k]), s, nM));
+    acc1 += ex2(fmaf(bf16_hi(w[k]), s, nM));
+  }
+  S += acc0 + acc1;
+#else
   float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
 #pragma unroll
   for (int k = 0; k < NW; ++k) {
@@ -125,6 +143,7 @@ __device__ __forceinline__ void lse_words(float& M, float& S, const uint32_t* w,
   }
   const float2 t = f2add(acc0, acc1);
   S += t.x + t.y;
+#endif
 }
 
 // Phase 1 on NV 16-byte vectors of bf16 per tensor; vector v holds elements
@@ -145,29 +164,18 @@ __device__ __forceinline__ void phase1_bf16(RowPart& A, const uint4* pv, const u
     qw[4 * v + 2] = qv[v].z;
     qw[4 * v + 3] = qv[v].w;
   }
-  uint32_t pmw = pw[0], qmw = qw[0];
+  float pm = -INFINITY;
 #pragma unroll
-  for (int k = 1; k < NW; ++k) {
-    pmw = bmax2(pmw, pw[k]);
-    qmw = bmax2(qmw, qw[k]);
+  for (int v = 0; v < NV; ++v) {  // per-vector maxima of z_p, in element order
+    const uint32_t m2 = bmax2(bmax2(pw[4 * v], pw[4 * v + 1]), bmax2(pw[4 * v + 2], pw[4 * v + 3]));
+    const float vm = fmaxf(bf16_lo(m2), bf16_hi(m2));
+    amax_vec(A, vm, idx0 + v * vstride);
+    pm = fmaxf(pm, vm);
   }
-  const float pm = fmaxf(bf16_lo(pmw), bf16_hi(pmw));
+  uint32_t qmw = qw[0];
+#pragma unroll
+  for (int k = 1; k < NW; ++k) qmw = bmax2(qmw, qw[k]);
   const float qm = fmaxf(bf16_lo(qmw), bf16_hi(qmw));
-  if (pm > A.av) {  // a new argmax of z_p: its first occurrence among these values
-    int e = 0;
-    float carry = 0.f;
-#pragma unroll
-    for (int k = 2 * NW - 1; k >= 0; --k) {
-      const float x = (k & 1) ? bf16_hi(pw[k >> 1]) : bf16_lo(pw[k >> 1]);
-      if (x == pm) {
-        e = k;
-        carry = (k & 1) ? bf16_hi(qw[k >> 1]) : bf16_lo(qw[k >> 1]);
-      }
-    }
-    A.av = pm;
-    A.ai = idx0 + (e >> 3) * vstride + (e & 7);
-    A.ac = carry;
-  }
   lse_words<NW>(A.pM, A.pS, pw, pm, sT);
   lse_words<NW>(A.qM, A.qS, qw, qm, sT);
   if (NEED_Q1) lse_words<NW>(A.q1M, A.q1S, qw, qm, kLog2e);
@@ -183,11 +191,24 @@ __device__ __forceinline__ void phase2_bf16(float2& smin2, float2& sqlt2, const 
   for (int k = 0; k < 4; ++k) {
     const float lp0 = fmaf(bf16_lo(pa[k]), s, nLp), lp1 = fmaf(bf16_hi(pa[k]), s, nLp);
     const float lq0 = fmaf(bf16_lo(qa[k]), s, nLq), lq1 = fmaf(bf16_hi(qa[k]), s, nLq);
+#ifdef AAL_SCALAR_ACC
+    const float e0 = ex2(fminf(lp0, lq0)), e1 = ex2(fminf(lp1, lq1));
+    smin2.x += e0;
+    smin2.y += e1;
+    sqlt2.x = fmaf(e0, set_lt(lq0, lp0), sqlt2.x);
+    sqlt2.y = fmaf(e1, set_lt(lq1, lp1), sqlt2.y);
+#else
     const float2 e = make_float2(ex2(fminf(lp0, lq0)), ex2(fminf(lp1, lq1)));
     smin2 = f2add(smin2, e);
     sqlt2 = f2fma(e, make_float2(set_lt(lq0, lp0), set_lt(lq1, lp1)), sqlt2);
+#endif
   }
 }
+
+// The first element of a 16-byte vector equal to `target` (the row's max of z_p), with
+// the z_q value at the same position.
+template <typename T>
+__device__ __forceinline__ void find_first(const uint4& pw, const uint4& qw, float target, int* at, float* carry);
 
 // Scalar element paths (fp32 rows, and the partial last chunk of a bf16 row).
 template <typename T>
@@ -209,6 +230,25 @@ __device__ __forceinline__ void unpack_vec<float>(const uint4& w, float* o) {
   o[1] = __uint_as_float(w.y);
   o[2] = __uint_as_float(w.z);
   o[3] = __uint_as_float(w.w);
+}
+
+template <typename T>
+__device__ __forceinline__ void find_first(const uint4& pw, const uint4& qw, float target, int* at, float* carry) {
+  constexpr int E = 16 / sizeof(T);
+  float pv[8], qv[8];
+  unpack_vec<T>(pw, pv);
+  unpack_vec<T>(qw, qv);
+  int e = 0;
+  float c = qv[0];
+#pragma unroll
+  for (int k = E - 1; k >= 0; --k) {
+    if (pv[k] == target) {
+      e = k;
+      c = qv[k];
+    }
+  }
+  *at = e;
+  *carry = c;
 }
 
 template <int N>
@@ -237,20 +277,7 @@ __device__ __forceinline__ void phase1_vec(RowPart& A, const uint4& pw, const ui
     pm = fmaxf(pm, pv[e]);
     qm = fmaxf(qm, qv[e]);
   }
-  if (pm > A.av) {
-    int e = 0;
-    float carry = qv[0];
-#pragma unroll
-    for (int k = E - 1; k >= 0; --k) {
-      if (pv[k] == pm) {
-        e = k;
-        carry = qv[k];
-      }
-    }
-    A.av = pm;
-    A.ai = idx0 + e;
-    A.ac = carry;
-  }
+  amax_vec(A, pm, idx0);
   lse_vals<E>(A.pM, A.pS, pv, pm, sT);
   lse_vals<E>(A.qM, A.qS, qv, qm, sT);
   if (NEED_Q1) lse_vals<E>(A.q1M, A.q1S, qv, qm, kLog2e);
@@ -306,6 +333,8 @@ __global__ void __launch_bounds__(kThreads, 1) rowstats_stream(RowStatsArgs a, i
       mbar_init(&S.empty[k], kWarps);
     }
     S.abort_flag = 0;
+    S.arg_index = 0x7fffffff;
+    S.arg_carry = 0.f;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   __syncthreads();
@@ -387,11 +416,22 @@ __global__ void __launch_bounds__(kThreads, 1) rowstats_stream(RowStatsArgs a, i
       float2 smin2 = make_float2(0.f, 0.f), sqlt2 = make_float2(0.f, 0.f);
       // one-float normalisers for the overlap pass: |error| <= ulp(M + Ls) / 2 in log2 units
       const float nLp = -(Mp + Lsp), nLq = -(Mq + Lsq);
+      // the vector that holds the first z_p maximum: chunk cstar, vector istar, thread tstar
+      const int cstar = tot.ab == 0x7fffffff ? -1 : tot.ab / CH;
+      const int istar = tot.ab == 0x7fffffff ? 0 : (tot.ab - cstar * CH) / E;
+      const int tstar = istar % kConsumers;
       for (int c = 0; c < nch; ++c, pos.next()) {
         if (wait_phase(&S.full[pos.slot], pos.phase, abort_flag, limit_ns, hdr)) {
           const int e0 = c * CH;
           const uint4* P = reinterpret_cast<const uint4*>(ring + pos.slot * kSlotBytes);
           const uint4* Q = reinterpret_cast<const uint4*>(ring + pos.slot * kSlotBytes + kHalfSlot);
+          if (c == cstar && t == tstar) {
+            int at;
+            float carry;
+            find_first<T>(P[istar], Q[istar], tot.av, &at, &carry);
+            S.arg_index = tot.ab + at;
+            S.arg_carry = carry;
+          }
           if (sizeof(T) == 2 && c < nfull) {
 #pragma unroll
             for (int v = 0; v < kNV; ++v) {
@@ -430,8 +470,10 @@ __global__ void __launch_bounds__(kThreads, 1) rowstats_stream(RowStatsArgs a, i
         a.ws.Lsq[r] = Lsq;
         a.ws.Mq1[r] = Mq1;
         a.ws.Lsq1[r] = Lsq1;
-        a.ws.xstar[r] = tot.ai;
-        a.ws.ag[r] = exp2f(log2_prob(tot.ac, kLog2e, Mq1, Lsq1));
+        a.ws.xstar[r] = S.arg_index;
+        a.ws.ag[r] = exp2f(log2_prob(S.arg_carry, kLog2e, Mq1, Lsq1));
+        S.arg_index = 0x7fffffff;
+        S.arg_carry = 0.f;
       }
       __syncwarp();
     }
