@@ -31,9 +31,9 @@ static_assert(sizeof(WsHeader) == 256, "header is 256 bytes");
 struct LossLayout {
   int64_t R = 0, N = 0, nwblk = 0;
   size_t hdr = 0;
-  // float[R] each: the log2-domain normaliser of z_p/T, z_q/T and z_q, kept in two parts:
-  // M = max_v z_v s (s = log2(e)/T, rounded product) and Ls = log2 sum_v 2^(z_v s - M),
-  // so log2 p~_v = fma(z_v, s, -M) - Ls holds its precision for large logits.
+  // float[R] each: the normaliser of z_p/T, z_q/T and z_q in two parts: the raw logit
+  // maximum M = max_v z_v and Ls = log2 sum_v 2^((z_v - M) s) with s = log2(e)/T, so that
+  // log2 p~_v = (z_v - M) s - Ls; the maximum's own term is exactly 2^0 = 1.
   size_t Mp = 0, Lsp = 0, Mq = 0, Lsq = 0, Mq1 = 0, Lsq1 = 0;
   size_t ag = 0, as = 0, qlt = 0;   // float[R] a^greedy, a^sample, sum_{lq<lp} q~
   size_t dEg = 0, dEs = 0;          // float[R] dE_n / da_{n,j}
@@ -242,10 +242,8 @@ __device__ __forceinline__ uint4 ldg_stream(const uint4* p) {
   return v;
 }
 
-// Online log2-sum-exp state of the values z*s: M = running max of the rounded products
-// z*s, S = sum_v 2^(fma(z_v, s, -M)).  Every term, the max's included, is formed the same
-// way as the later evaluation fma(z, s, -M) - log2(S), so the max element's own rounding
-// cancels.
+// Online log2-sum-exp state of the values z*s: M = running raw maximum of z and
+// S = sum_v 2^((z_v - M) s).  The maximum's own term is exactly 1.
 struct Lse {
   float M, S;
 };
@@ -254,31 +252,44 @@ __device__ __forceinline__ void lse_init(Lse& a) {
   a.S = 0.f;
 }
 __device__ __forceinline__ void lse_push(Lse& a, float z, float s) {
-  const float x = __fmul_rn(z, s);
-  if (x > a.M) {
-    a.S = a.S * ex2(a.M - x) + ex2(fmaf(z, s, -x));
-    a.M = x;
+  if (z > a.M) {
+    a.S = a.S * ex2((a.M - z) * s) + 1.f;  // M == -inf: ex2(-inf) = 0 and S was 0
+    a.M = z;
   } else if (a.M != -INFINITY) {
-    a.S += ex2(fmaf(z, s, -a.M));
+    a.S += ex2((z - a.M) * s);
   }
 }
-__device__ __forceinline__ Lse lse_merge(Lse a, Lse b) {
+__device__ __forceinline__ Lse lse_merge(Lse a, Lse b, float s) {
   Lse r;
   r.M = fmaxf(a.M, b.M);
   if (r.M == -INFINITY) {
     r.S = 0.f;
   } else {
-    float sa = (a.M == -INFINITY) ? 0.f : a.S * ex2(a.M - r.M);
-    float sb = (b.M == -INFINITY) ? 0.f : b.S * ex2(b.M - r.M);
+    const float sa = (a.M == -INFINITY) ? 0.f : a.S * ex2((a.M - r.M) * s);
+    const float sb = (b.M == -INFINITY) ? 0.f : b.S * ex2((b.M - r.M) * s);
     r.S = sa + sb;
   }
   return r;
 }
-// log2(S) of the normaliser, accurate log (once per row); the normaliser is M + log2(S).
+// Ls = log2(S), accurate log (once per row).
 __device__ __forceinline__ float lse_ls(Lse a) { return log2f(a.S); }
-// log2 of the scaled probability of logit z: fma(z, s, -M) - Ls.
-__device__ __forceinline__ float log2_prob(float z, float s, float M, float Ls) {
-  return fmaf(z, s, -M) - Ls;
+// log2 of the scaled probability of logit z: (z - M) s - Ls.
+__device__ __forceinline__ float log2_prob(float z, float s, float M, float Ls) { return fmaf(z - M, s, -Ls); }
+
+// f32(bf16 half of w) + c in one instruction (the widening happens inside the add).
+__device__ __forceinline__ float bf16lo_add(uint32_t w, float c) {
+  float d;
+  asm("{\n\t.reg .b16 lo, hi;\n\tmov.b32 {lo, hi}, %1;\n\tadd.rn.f32.bf16 %0, lo, %2;\n\t}"
+      : "=f"(d)
+      : "r"(w), "f"(c));
+  return d;
+}
+__device__ __forceinline__ float bf16hi_add(uint32_t w, float c) {
+  float d;
+  asm("{\n\t.reg .b16 lo, hi;\n\tmov.b32 {lo, hi}, %1;\n\tadd.rn.f32.bf16 %0, hi, %2;\n\t}"
+      : "=f"(d)
+      : "r"(w), "f"(c));
+  return d;
 }
 
 // Argmax with the lowest index on ties, carrying one extra value.

@@ -45,14 +45,14 @@ struct RowState {
   Lse lp, lq, lr;
 };
 
-__device__ __forceinline__ RowState merge_state(const RowState& a, const RowState& b) {
+__device__ __forceinline__ RowState merge_state(const RowState& a, const RowState& b, float sT) {
   RowState o;
   o.q = amax_merge(a.q, b.q);
   o.p = amax_merge(a.p, b.p);
   o.r = amax_merge(a.r, b.r);
-  o.lp = lse_merge(a.lp, b.lp);
-  o.lq = lse_merge(a.lq, b.lq);
-  o.lr = lse_merge(a.lr, b.lr);
+  o.lp = lse_merge(a.lp, b.lp, sT);
+  o.lq = lse_merge(a.lq, b.lq, sT);
+  o.lr = lse_merge(a.lr, b.lr, sT);
   return o;
 }
 
@@ -123,12 +123,12 @@ __global__ void __launch_bounds__(kRowThreads) reward_rows(RewardRowArgs a) {
         visit(v, load_elem<T>(zq + v), load_elem<T>(zp + v), REF ? load_elem<T>(zr + v) : 0.f);
     }
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) st = merge_state(st, shfl_state(st, off));
+    for (int off = 16; off > 0; off >>= 1) st = merge_state(st, shfl_state(st, off), a.sT);
     if (lane == 0) red[warp] = st;
     __syncthreads();
     if (threadIdx.x == 0) {
       RowState t = red[0];
-      for (int w = 1; w < kRowWarps; ++w) t = merge_state(t, red[w]);
+      for (int w = 1; w < kRowWarps; ++w) t = merge_state(t, red[w], a.sT);
       uint8_t acc, acc_ref = 0;
       if (!SAMPLING) {
         acc = (t.q.i == t.p.i) ? 1 : 0;

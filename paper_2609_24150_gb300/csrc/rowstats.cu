@@ -2,9 +2,9 @@
 //
 // For every logit row r = (window n, depth j) this computes, from z_p (target)
 // and z_q (draft):
-//   (M, Ls)  the log2-domain normalisers of z_p/T and z_q/T (the temperature-scaled
-//            distributions of Sec. 2.3) and of z_q (the unscaled draft of Eq.
-//            acc_greedy): M = max_v z_v s, Ls = log2 sum_v 2^(z_v s - M),
+//   (M, Ls)  the normalisers of z_p/T and z_q/T (the temperature-scaled distributions
+//            of Sec. 2.3) and of z_q (the unscaled draft of Eq. acc_greedy):
+//            M = max_v z_v, Ls = log2 sum_v 2^((z_v - M) s),
 //   x*       argmax_v z_p (lowest index on ties) and a^greedy = q(x*) (Eq. acc_greedy),
 //   a^sample = sum_v min(p~_v, q~_v)   (Eq. acc_sample),
 //   Qlt      = sum_{v: q~_v < p~_v} q~_v, which the backward of a^sample needs.
@@ -51,11 +51,11 @@ struct Phase1 {
   Amax am;
 };
 
-__device__ __forceinline__ Phase1 merge1(const Phase1& a, const Phase1& b) {
+__device__ __forceinline__ Phase1 merge1(const Phase1& a, const Phase1& b, float sT) {
   Phase1 r;
-  r.p = lse_merge(a.p, b.p);
-  r.q = lse_merge(a.q, b.q);
-  r.q1 = lse_merge(a.q1, b.q1);
+  r.p = lse_merge(a.p, b.p, sT);
+  r.q = lse_merge(a.q, b.q, sT);
+  r.q1 = lse_merge(a.q1, b.q1, kLog2e);
   r.am = amax_merge(a.am, b.am);
   return r;
 }
@@ -114,7 +114,7 @@ __global__ void __launch_bounds__(kGenericThreads) rowstats_generic(RowStatsArgs
 
     // block reduction of phase 1 (fixed butterfly + fixed warp order: deterministic)
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) acc = merge1(acc, shfl1(acc, off));
+    for (int off = 16; off > 0; off >>= 1) acc = merge1(acc, shfl1(acc, off), a.sT);
     if (lane == 0) red1[warp] = acc;
     __syncthreads();
     if (warp == 0) {
@@ -128,7 +128,7 @@ __global__ void __launch_bounds__(kGenericThreads) rowstats_generic(RowStatsArgs
         amax_init(x.am);
       }
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) x = merge1(x, shfl1(x, off));
+      for (int off = 16; off > 0; off >>= 1) x = merge1(x, shfl1(x, off), a.sT);
       if (lane == 0) row1 = x;
     }
     __syncthreads();

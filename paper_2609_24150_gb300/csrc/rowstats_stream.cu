@@ -53,7 +53,7 @@ constexpr int kBarRow = 1, kBarSum = 2;
 // ab among equal av contains the first occurrence; the position inside that vector is
 // found in the second pass, by the one thread that streams the vector again.
 struct RowPart {
-  float pM, pS, qM, qS, q1M, q1S;  // online log2-sum-exp states (M = max of z*s)
+  float pM, pS, qM, qS, q1M, q1S;  // online log2-sum-exp states (M = raw max of z)
   float av;
   int32_t ab;
 };
@@ -76,11 +76,11 @@ __device__ __forceinline__ void part_init(RowPart& a) {
 }
 
 // Butterfly reductions over a warp: every lane ends with the same, order-fixed result.
-__device__ __forceinline__ void warp_lse(float& M, float& S) {
+__device__ __forceinline__ void warp_lse(float& M, float& S, float scale) {
   float m = M;
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
-  float s = (M == -INFINITY) ? 0.f : S * ex2(M - m);
+  float s = (M == -INFINITY) ? 0.f : S * ex2((M - m) * scale);
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
   M = m;
@@ -98,10 +98,10 @@ __device__ __forceinline__ void warp_amax(float& v, int32_t& i) {
   }
 }
 template <bool NEED_Q1>
-__device__ __forceinline__ void warp_part(RowPart& a) {
-  warp_lse(a.pM, a.pS);
-  warp_lse(a.qM, a.qS);
-  if (NEED_Q1) warp_lse(a.q1M, a.q1S);
+__device__ __forceinline__ void warp_part(RowPart& a, float sT) {
+  warp_lse(a.pM, a.pS, sT);
+  warp_lse(a.qM, a.qS, sT);
+  if (NEED_Q1) warp_lse(a.q1M, a.q1S, kLog2e);
   warp_amax(a.av, a.ab);
 }
 // A vector's maximum beats the running one: remember it and where its vector starts.
@@ -114,36 +114,27 @@ __device__ __forceinline__ void amax_vec(RowPart& A, float vmax, int base) {
 // ---------------------------------------------------------------- per-chunk arithmetic
 
 // Fold NW bf16 words (2 NW values) of one tensor into (M, S); vmax is their maximum.
-// Each value costs one fma (the bf16 operand is widened inside the instruction), one
-// ex2, and half a packed add.
+// Each value costs one mixed-precision add (z - M, the bf16 widened inside the add), half
+// a packed multiply by s, one ex2 and half a packed add.
 template <int NW>
 __device__ __forceinline__ void lse_words(float& M, float& S, const uint32_t* w, float vmax, float s) {
-  const float xm = __fmul_rn(vmax, s);
-  if (xm > M) {
-    S *= ex2(M - xm);  // M == -inf: ex2(-inf) = 0 and S is still 0
-    M = xm;
+  if (vmax > M) {
+    S *= ex2((M - vmax) * s);  // M == -inf: ex2(-inf) = 0 and S is still 0
+    M = vmax;
   }
   if (M == -INFINITY) return;
   const float nM = -M;
-#ifdef AAL_SCALAR_ACC
-  float acc0 = 0.f, acc1 = 0.f;
+  const float2 s2 = make_float2(s, s), zero2 = make_float2(0.f, 0.f);
+  float2 acc0 = zero2, acc1 = zero2;
 #pragma unroll
   for (int k = 0; k < NW; ++k) {
-    acc0 += ex2(fmaf(bf16_lo(w[k]), s, nM));
-    acc1 += ex2(fmaf(bf16_hi(w[k]), s, nM));
-  }
-  S += acc0 + acc1;
-#else
-  float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
-#pragma unroll
-  for (int k = 0; k < NW; ++k) {
-    const float2 e = make_float2(ex2(fmaf(bf16_lo(w[k]), s, nM)), ex2(fmaf(bf16_hi(w[k]), s, nM)));
+    const float2 x = f2fma(make_float2(bf16lo_add(w[k], nM), bf16hi_add(w[k], nM)), s2, zero2);
+    const float2 e = make_float2(ex2(x.x), ex2(x.y));
     if (k & 1) acc1 = f2add(acc1, e);
     else acc0 = f2add(acc0, e);
   }
   const float2 t = f2add(acc0, acc1);
   S += t.x + t.y;
-#endif
 }
 
 // Phase 1 on NV 16-byte vectors of bf16 per tensor; vector v holds elements
@@ -181,27 +172,22 @@ __device__ __forceinline__ void phase1_bf16(RowPart& A, const uint4* pv, const u
   if (NEED_Q1) lse_words<NW>(A.q1M, A.q1S, qw, qm, kLog2e);
 }
 
-// Phase 2 on one 16-byte vector of bf16 per tensor, with the row normalisers folded into
-// one addend each (nLp = -(M_p + Ls_p)): log2 p~ = fma(z_p, s, nLp).
+// Phase 2 on one 16-byte vector of bf16 per tensor.  With C = M + Ls/s, log2 p~ = (z - C) s;
+// since s > 0 the min and the comparison are taken on u = z - C (one mixed-precision add
+// each) and only the min is scaled.
 __device__ __forceinline__ void phase2_bf16(float2& smin2, float2& sqlt2, const uint4& pw, const uint4& qw,
-                                            float s, float nLp, float nLq) {
+                                            float s, float nCp, float nCq) {
   const uint32_t pa[4] = {pw.x, pw.y, pw.z, pw.w};
   const uint32_t qa[4] = {qw.x, qw.y, qw.z, qw.w};
+  const float2 s2 = make_float2(s, s), zero2 = make_float2(0.f, 0.f);
 #pragma unroll
   for (int k = 0; k < 4; ++k) {
-    const float lp0 = fmaf(bf16_lo(pa[k]), s, nLp), lp1 = fmaf(bf16_hi(pa[k]), s, nLp);
-    const float lq0 = fmaf(bf16_lo(qa[k]), s, nLq), lq1 = fmaf(bf16_hi(qa[k]), s, nLq);
-#ifdef AAL_SCALAR_ACC
-    const float e0 = ex2(fminf(lp0, lq0)), e1 = ex2(fminf(lp1, lq1));
-    smin2.x += e0;
-    smin2.y += e1;
-    sqlt2.x = fmaf(e0, set_lt(lq0, lp0), sqlt2.x);
-    sqlt2.y = fmaf(e1, set_lt(lq1, lp1), sqlt2.y);
-#else
-    const float2 e = make_float2(ex2(fminf(lp0, lq0)), ex2(fminf(lp1, lq1)));
+    const float up0 = bf16lo_add(pa[k], nCp), up1 = bf16hi_add(pa[k], nCp);
+    const float uq0 = bf16lo_add(qa[k], nCq), uq1 = bf16hi_add(qa[k], nCq);
+    const float2 x = f2fma(make_float2(fminf(up0, uq0), fminf(up1, uq1)), s2, zero2);
+    const float2 e = make_float2(ex2(x.x), ex2(x.y));
     smin2 = f2add(smin2, e);
-    sqlt2 = f2fma(e, make_float2(set_lt(lq0, lp0), set_lt(lq1, lp1)), sqlt2);
-#endif
+    sqlt2 = f2fma(e, make_float2(set_lt(uq0, up0), set_lt(uq1, up1)), sqlt2);
   }
 }
 
@@ -253,15 +239,14 @@ __device__ __forceinline__ void find_first(const uint4& pw, const uint4& qw, flo
 
 template <int N>
 __device__ __forceinline__ void lse_vals(float& M, float& S, const float* v, float vmax, float s) {
-  const float xm = __fmul_rn(vmax, s);
-  if (xm > M) {
-    S *= ex2(M - xm);
-    M = xm;
+  if (vmax > M) {
+    S *= ex2((M - vmax) * s);
+    M = vmax;
   }
   if (M == -INFINITY) return;
   float acc = 0.f;
 #pragma unroll
-  for (int e = 0; e < N; ++e) acc += ex2(fmaf(v[e], s, -M));
+  for (int e = 0; e < N; ++e) acc += ex2((v[e] - M) * s);
   S += acc;
 }
 
@@ -285,18 +270,17 @@ __device__ __forceinline__ void phase1_vec(RowPart& A, const uint4& pw, const ui
 
 template <typename T>
 __device__ __forceinline__ void phase2_vec(float& smin, float& sqlt, const uint4& pw, const uint4& qw, float sT,
-                                           float Mp, float Lsp, float Mq, float Lsq) {
+                                           float nCp, float nCq) {
   constexpr int E = 16 / sizeof(T);
   float pv[8], qv[8];
   unpack_vec<T>(pw, pv);
   unpack_vec<T>(qw, qv);
 #pragma unroll
   for (int e = 0; e < E; ++e) {
-    const float lp = fmaf(pv[e], sT, -Mp) - Lsp;
-    const float lq = fmaf(qv[e], sT, -Mq) - Lsq;
-    const float t = ex2(fminf(lp, lq));
+    const float up = pv[e] + nCp, uq = qv[e] + nCq;
+    const float t = ex2(fminf(up, uq) * sT);
     smin += t;
-    sqlt += (lq < lp) ? t : 0.f;
+    sqlt += (uq < up) ? t : 0.f;
   }
 }
 
@@ -400,22 +384,22 @@ __global__ void __launch_bounds__(kThreads, 1) rowstats_stream(RowStatsArgs a, i
         __syncwarp();
         if (lane == 0) mbar_arrive(&S.empty[pos.slot]);
       }
-      warp_part<NEED_Q1>(A);
+      warp_part<NEED_Q1>(A, a.sT);
       if (lane == 0) S.red[warp] = A;
       named_barrier(kBarRow, kConsumers);
       // every warp combines the warp partials itself (lanes >= kWarps carry the identity)
       RowPart tot;
       if (lane < kWarps) tot = S.red[lane];
       else part_init(tot);
-      warp_part<NEED_Q1>(tot);
+      warp_part<NEED_Q1>(tot, a.sT);
       const float Mp = tot.pM, Lsp = log2f(tot.pS);
       const float Mq = tot.qM, Lsq = log2f(tot.qS);
 
       // pass 2: overlap sums
       float smin = 0.f, sqlt = 0.f;
       float2 smin2 = make_float2(0.f, 0.f), sqlt2 = make_float2(0.f, 0.f);
-      // one-float normalisers for the overlap pass: |error| <= ulp(M + Ls) / 2 in log2 units
-      const float nLp = -(Mp + Lsp), nLq = -(Mq + Lsq);
+      // overlap pass in unscaled units: log2 p~ = (z - Cp) s with Cp = Mp + Lsp / s
+      const float nCp = -(Mp + Lsp / a.sT), nCq = -(Mq + Lsq / a.sT);
       // the vector that holds the first z_p maximum: chunk cstar, vector istar, thread tstar
       const int cstar = tot.ab == 0x7fffffff ? -1 : tot.ab / CH;
       const int istar = tot.ab == 0x7fffffff ? 0 : (tot.ab - cstar * CH) / E;
@@ -436,11 +420,11 @@ __global__ void __launch_bounds__(kThreads, 1) rowstats_stream(RowStatsArgs a, i
 #pragma unroll
             for (int v = 0; v < kNV; ++v) {
               const int i = t + v * kConsumers;
-              phase2_bf16(smin2, sqlt2, P[i], Q[i], a.sT, nLp, nLq);
+              phase2_bf16(smin2, sqlt2, P[i], Q[i], a.sT, nCp, nCq);
             }
           } else {
             const int nvec = min(CH, V - e0) / E;
-            for (int i = t; i < nvec; i += kConsumers) phase2_vec<T>(smin, sqlt, P[i], Q[i], a.sT, Mp, Lsp, Mq, Lsq);
+            for (int i = t; i < nvec; i += kConsumers) phase2_vec<T>(smin, sqlt, P[i], Q[i], a.sT, nCp, nCq);
           }
         }
         __syncwarp();
