@@ -159,6 +159,23 @@ AAL_API aal_status aal_accept_reward(const aal_reward_problem* prob, const void*
                              size_t workspace_bytes, int32_t* tau, int32_t* tau_ref,
                              float* rollout_len, float* advantage, void* stream);
 
+/* The same reward for the draft alone (R = tau^theta), taken from the statistics that
+ * aal_loss_fwd left in `loss_workspace` instead of from the logits: the forward already
+ * streams z_p and z_q and records, per row, x* = argmax z_p, the draft's greedy token
+ * S_k = argmax z_q (lowest index on ties), z_p(S_k) and the normalisers.  No logit is read,
+ * so a training step that computes the loss and the GRPO reward over the same logits
+ * (Sec. 3.4 with the surrogate of Sec. 3.2 / 3.3) reads them once for both.
+ *   rprob     N, K, V, dtype must equal lprob's.  AAL_GREEDY works after any loss mode;
+ *             AAL_SAMPLING needs a loss mode with the sampling term at the same temperature
+ *             (the normalisers of p~ and q~ at T); otherwise AAL_ERR_INVALID_ARG.
+ *   lprob, loss_workspace  the problem and workspace of a completed aal_loss_fwd (same stream).
+ *   workspace  at least aal_reward_workspace_size(rprob) bytes.
+ * Outputs as for aal_accept_reward (no reference draft). */
+AAL_API aal_status aal_accept_reward_from_loss(const aal_reward_problem* rprob, const aal_problem* lprob,
+                                               const void* loss_workspace, size_t loss_workspace_bytes,
+                                               void* workspace, size_t workspace_bytes, int32_t* tau,
+                                               float* rollout_len, float* advantage, void* stream);
+
 /* aal_accept_reward without a workspace argument: the scratch lives in a fixed array inside
  * the library.  The paper has no counterpart; this exists for callers that cannot allocate
  * device memory -- e.g. a training loop whose device memory is all reserved up front by its

@@ -29,6 +29,7 @@ from .aal import (  # noqa: F401
     AalRewardProblem,
     aal_abi_version,
     aal_accept_reward,
+    aal_accept_reward_from_loss,
     aal_accept_reward_noalloc,
     aal_check_device_status,
     aal_loss_bwd,

@@ -76,13 +76,15 @@ def library() -> ctypes.CDLL:
     lib.aal_loss_bwd.argtypes = [P, vp, vp, vp, vp, sz, ctypes.c_float, vp, vp]
     lib.aal_accept_reward.argtypes = [RP, vp, vp, vp, vp, sz, vp, vp, vp, vp, vp]
     lib.aal_accept_reward_noalloc.argtypes = [RP, vp, vp, vp, vp, vp, vp, vp, vp]
+    lib.aal_accept_reward_from_loss.argtypes = [RP, P, vp, sz, vp, sz, vp, vp, vp, vp]
     lib.aal_check_device_status.argtypes = [vp, vp]
     lib.aal_status_string.argtypes = [ctypes.c_int]
     lib.aal_status_string.restype = ctypes.c_char_p
     lib.aal_abi_version.argtypes = []
     lib.aal_abi_version.restype = ctypes.c_int32
     for f in ("aal_workspace_size", "aal_reward_workspace_size", "aal_loss_fwd", "aal_loss_bwd",
-              "aal_accept_reward", "aal_accept_reward_noalloc", "aal_check_device_status"):
+              "aal_accept_reward", "aal_accept_reward_noalloc", "aal_accept_reward_from_loss",
+              "aal_check_device_status"):
         getattr(lib, f).restype = ctypes.c_int
     _LIB = lib
     return lib
@@ -205,6 +207,19 @@ def aal_accept_reward(problem: AalRewardProblem, draft, target, ref_draft, works
         _ptr(rollout_len, "rollout_len", torch.float32, nroll),
         _ptr(advantage, "advantage", torch.float32, nroll), _stream(stream))
     _check(code, "aal_accept_reward")
+
+
+def aal_accept_reward_from_loss(problem: AalRewardProblem, loss_problem_: AalProblem, loss_workspace,
+                                workspace, tau, rollout_len, advantage, stream=None):
+    """The draft's reward from the statistics of a completed aal_loss_fwd (no logit pass)."""
+    N = problem.N
+    nroll = N // max(1, problem.windows_per_rollout)
+    code = library().aal_accept_reward_from_loss(
+        ctypes.byref(problem), ctypes.byref(loss_problem_), _ptr(loss_workspace, "loss_workspace"),
+        _nbytes(loss_workspace), _ptr(workspace, "workspace"), _nbytes(workspace),
+        _ptr(tau, "tau", torch.int32, N), _ptr(rollout_len, "rollout_len", torch.float32, nroll),
+        _ptr(advantage, "advantage", torch.float32, nroll), _stream(stream))
+    _check(code, "aal_accept_reward_from_loss")
 
 
 def aal_accept_reward_noalloc(problem: AalRewardProblem, draft, target, ref_draft, tau, tau_ref,

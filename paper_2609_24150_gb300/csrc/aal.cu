@@ -215,6 +215,61 @@ aal_status aal_accept_reward(const aal_reward_problem* prob, const void* draft, 
   return cuda_status(launch_reward_groups(ga, s));
 }
 
+aal_status aal_accept_reward_from_loss(const aal_reward_problem* rprob, const aal_problem* lprob,
+                                       const void* loss_workspace, size_t loss_workspace_bytes, void* workspace,
+                                       size_t workspace_bytes, int32_t* tau, float* rollout_len, float* advantage,
+                                       void* stream) {
+  aal_status st = check_reward(rprob);
+  if (st != AAL_OK) return st;
+  st = check_problem(lprob);
+  if (st != AAL_OK) return st;
+  if (rprob->N != lprob->N || rprob->K != lprob->K || rprob->V != lprob->V || rprob->dtype != lprob->dtype)
+    return AAL_ERR_INVALID_ARG;
+  const bool sampling = rprob->mode == AAL_SAMPLING;
+  // the sampling acceptance needs the loss's temperature-scaled normalisers at this T
+  if (sampling && (!(lprob->mode & AAL_SAMPLING) || lprob->temperature != rprob->temperature))
+    return AAL_ERR_INVALID_ARG;
+  if (rprob->N == 0) return AAL_OK;
+  if (tau == nullptr || rollout_len == nullptr || advantage == nullptr || !aligned(tau, 4) ||
+      !aligned(rollout_len, 4) || !aligned(advantage, 4))
+    return AAL_ERR_INVALID_ARG;
+  const LossLayout LL = loss_layout(lprob->N, lprob->K);
+  if (loss_workspace == nullptr || !aligned(loss_workspace, 256) || loss_workspace_bytes < LL.total)
+    return AAL_ERR_WORKSPACE;
+  const RewardLayout L = reward_layout(rprob->N, rprob->K);
+  if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < L.total) return AAL_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  char* base = static_cast<char*>(workspace);
+  WsHeader* hdr = reinterpret_cast<WsHeader*>(base + L.hdr);
+  if (cudaMemsetAsync(hdr, 0, sizeof(WsHeader), s) != cudaSuccess) return AAL_ERR_CUDA;
+
+  RewardStatsArgs fa;
+  fa.ws = loss_ws(const_cast<void*>(loss_workspace), LL);
+  fa.R = LL.R;
+  fa.K = (int32_t)rprob->K;
+  fa.sampling = sampling;
+  fa.sT = sampling ? kLog2e / rprob->temperature : 0.f;
+  fa.seed = rprob->seed;
+  fa.row_offset = rprob->row_offset;
+  fa.acc = reinterpret_cast<uint8_t*>(base + L.acc);
+  if (launch_reward_flags_from_stats(fa, s) != cudaSuccess) return AAL_ERR_CUDA;
+
+  RewardGroupArgs ga;
+  ga.acc = fa.acc;
+  ga.acc_ref = nullptr;
+  ga.rbuf = reinterpret_cast<float*>(base + L.rbuf);
+  ga.N = rprob->N;
+  ga.K = (int32_t)rprob->K;
+  ga.wpr = rprob->windows_per_rollout;
+  ga.rpg = rprob->rollouts_per_group;
+  ga.adv_clip = rprob->adv_clip;
+  ga.tau = tau;
+  ga.tau_ref = nullptr;
+  ga.rollout_len = rollout_len;
+  ga.advantage = advantage;
+  return cuda_status(launch_reward_groups(ga, s));
+}
+
 aal_status aal_check_device_status(void* workspace, void* stream) {
   if (workspace == nullptr || !aligned(workspace, 256)) return AAL_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);

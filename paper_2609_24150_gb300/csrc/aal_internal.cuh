@@ -38,6 +38,8 @@ struct LossLayout {
   size_t ag = 0, as = 0, qlt = 0;   // float[R] a^greedy, a^sample, sum_{lq<lp} q~
   size_t dEg = 0, dEs = 0;          // float[R] dE_n / da_{n,j}
   size_t xstar = 0;                 // int32[R] target argmax
+  size_t yhat = 0;                  // int32[R] draft argmax (the greedy draft token)
+  size_t zpy = 0;                   // float[R] z_p at the draft argmax
   size_t cpart = 0;                 // float2[R][kMaxCluster] per-CTA (overlap, Qlt) partials
   size_t wpart = 0;                 // double[nwblk][4] window-kernel block partials
   size_t total = 0;
@@ -72,6 +74,8 @@ inline LossLayout loss_layout(int64_t N, int64_t K) {
   L.dEg = take(R * 4);
   L.dEs = take(R * 4);
   L.xstar = take(R * 4);
+  L.yhat = take(R * 4);
+  L.zpy = take(R * 4);
   L.cpart = take(R * kMaxCluster * 8);
   L.wpart = take((size_t)(L.nwblk > 0 ? L.nwblk : 1) * 4 * 8);
   L.total = off;
@@ -105,6 +109,8 @@ struct LossWs {
   WsHeader* hdr;
   float *Mp, *Lsp, *Mq, *Lsq, *Mq1, *Lsq1, *ag, *as, *qlt, *dEg, *dEs;
   int32_t* xstar;
+  int32_t* yhat;
+  float* zpy;
   float2* cpart;
   double* wpart;
 };
@@ -125,6 +131,8 @@ inline LossWs loss_ws(void* base, const LossLayout& L) {
   w.dEg = reinterpret_cast<float*>(b + L.dEg);
   w.dEs = reinterpret_cast<float*>(b + L.dEs);
   w.xstar = reinterpret_cast<int32_t*>(b + L.xstar);
+  w.yhat = reinterpret_cast<int32_t*>(b + L.yhat);
+  w.zpy = reinterpret_cast<float*>(b + L.zpy);
   w.cpart = reinterpret_cast<float2*>(b + L.cpart);
   w.wpart = reinterpret_cast<double*>(b + L.wpart);
   return w;
@@ -186,6 +194,18 @@ struct RewardRowArgs {
   WsHeader* hdr;
 };
 
+// Acceptance flags from the statistics a loss forward left in its workspace.
+struct RewardStatsArgs {
+  LossWs ws;
+  int64_t R;
+  int32_t K;
+  bool sampling;
+  float sT;
+  uint64_t seed;
+  int64_t row_offset;
+  uint8_t* acc;
+};
+
 struct RewardGroupArgs {
   const uint8_t* acc;
   const uint8_t* acc_ref;  // null without a reference draft
@@ -208,6 +228,7 @@ cudaError_t launch_window(const WindowArgs& a, cudaStream_t s);
 cudaError_t launch_backward(const BackwardArgs& a, bool bf16, cudaStream_t s);
 cudaError_t launch_reward_rows(const RewardRowArgs& a, bool bf16, cudaStream_t s);
 cudaError_t launch_reward_groups(const RewardGroupArgs& a, cudaStream_t s);
+cudaError_t launch_reward_flags_from_stats(const RewardStatsArgs& a, cudaStream_t s);
 
 // ---------------------------------------------------------------------------
 // Device helpers.

@@ -241,7 +241,32 @@ __global__ void __launch_bounds__(kGroupThreads) reward_groups(RewardGroupArgs a
   }
 }
 
+// One thread per row: the acceptance of the draft's greedy token from the loss forward's
+// statistics (x*, the draft argmax y = S_k and z_p(y), and the normalisers), no logit pass.
+// Sampling: log2 q~(y) = (z_q(y) - M_q) s - Ls_q = -Ls_q because y is where z_q peaks.
+__global__ void __launch_bounds__(256) reward_flags_from_stats(RewardStatsArgs a) {
+  const int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= a.R) return;
+  uint8_t acc;
+  if (!a.sampling) {
+    acc = (a.ws.yhat[r] == a.ws.xstar[r]) ? 1 : 0;
+  } else {
+    const int64_t n = r / a.K;
+    const uint32_t k = (uint32_t)(r - n * a.K);
+    const float u = philox_uniform(a.seed, (uint64_t)(a.row_offset + n), k);
+    const float d = log2_prob(a.ws.zpy[r], a.sT, a.ws.Mp[r], a.ws.Lsp[r]) + a.ws.Lsq[r];
+    acc = (u < exp2f(fminf(d, 0.f))) ? 1 : 0;
+  }
+  a.acc[r] = acc;
+}
+
 }  // namespace
+
+cudaError_t launch_reward_flags_from_stats(const RewardStatsArgs& a, cudaStream_t s) {
+  if (a.R < 1) return cudaSuccess;
+  reward_flags_from_stats<<<(unsigned)((a.R + 255) / 256), 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_reward_rows(const RewardRowArgs& a, bool bf16, cudaStream_t s) {
   return bf16 ? dispatch<uint16_t>(a, s) : dispatch<float>(a, s);

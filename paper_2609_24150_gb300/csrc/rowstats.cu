@@ -48,7 +48,8 @@ __device__ __forceinline__ void unpack<uint16_t>(const uint4& w, float* out) {
 
 struct Phase1 {
   Lse p, q, q1;
-  Amax am;
+  Amax am;  // target argmax, carrying z_q there
+  Amax aq;  // draft argmax, carrying z_p there
 };
 
 __device__ __forceinline__ Phase1 merge1(const Phase1& a, const Phase1& b, float sT) {
@@ -57,6 +58,7 @@ __device__ __forceinline__ Phase1 merge1(const Phase1& a, const Phase1& b, float
   r.q = lse_merge(a.q, b.q, sT);
   r.q1 = lse_merge(a.q1, b.q1, kLog2e);
   r.am = amax_merge(a.am, b.am);
+  r.aq = amax_merge(a.aq, b.aq);
   return r;
 }
 
@@ -66,6 +68,7 @@ __device__ __forceinline__ Phase1 shfl1(const Phase1& a, int off) {
   b.q = shfl_lse(a.q, off);
   b.q1 = shfl_lse(a.q1, off);
   b.am = shfl_amax(a.am, off);
+  b.aq = shfl_amax(a.aq, off);
   return b;
 }
 
@@ -85,11 +88,17 @@ __global__ void __launch_bounds__(kGenericThreads) rowstats_generic(RowStatsArgs
     lse_init(acc.q);
     lse_init(acc.q1);
     amax_init(acc.am);
+    amax_init(acc.aq);
     auto visit = [&](int64_t v, float p, float q) {
       if (p > acc.am.v) {
         acc.am.v = p;
         acc.am.i = (int32_t)v;
         acc.am.carry = q;
+      }
+      if (q > acc.aq.v) {
+        acc.aq.v = q;
+        acc.aq.i = (int32_t)v;
+        acc.aq.carry = p;
       }
       if (a.need_p) lse_push(acc.p, p, a.sT);
       if (a.need_q) lse_push(acc.q, q, a.sT);
@@ -126,6 +135,7 @@ __global__ void __launch_bounds__(kGenericThreads) rowstats_generic(RowStatsArgs
         lse_init(x.q);
         lse_init(x.q1);
         amax_init(x.am);
+        amax_init(x.aq);
       }
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) x = merge1(x, shfl1(x, off), a.sT);
@@ -186,6 +196,8 @@ __global__ void __launch_bounds__(kGenericThreads) rowstats_generic(RowStatsArgs
       a.ws.Mq1[r] = Mq1;
       a.ws.Lsq1[r] = Lsq1;
       a.ws.xstar[r] = tot.am.i;
+      a.ws.yhat[r] = tot.aq.i;
+      a.ws.zpy[r] = tot.aq.carry;
       a.ws.ag[r] = exp2f(log2_prob(tot.am.carry, kLog2e, Mq1, Lsq1));
       a.ws.cpart[r * kMaxCluster] = make_float2(s_min, s_qlt);
     }

@@ -54,8 +54,10 @@ constexpr int kBarRow = 1, kBarSum = 2;
 // found in the second pass, by the one thread that streams the vector again.
 struct RowPart {
   float pM, pS, qM, qS, q1M, q1S;  // online log2-sum-exp states (M = raw max of z)
-  float av;
+  float av;                        // target: largest z_p and the first vector holding it
   int32_t ab;
+  float qv;                        // draft: largest z_q and the first vector holding it
+  int32_t qb;
 };
 
 struct Smem {
@@ -65,14 +67,22 @@ struct Smem {
   float2 red2[2][kWarps];
   int32_t arg_index;  // x*, written by the thread that finds it in the second pass
   float arg_carry;    // z_q at x*
+  int32_t yarg_index;  // the draft argmax, found the same way
+  float yarg_carry;    // z_p there
   int abort_flag;
 };
 
+// Running maxima start at a finite floor far below any logit, so the online updates need
+// no -inf special cases: a floor term contributes 2^(-huge) = 0.
+constexpr float kMaxFloor = -1e30f;
+
 __device__ __forceinline__ void part_init(RowPart& a) {
-  a.pM = a.qM = a.q1M = -INFINITY;
+  a.pM = a.qM = a.q1M = kMaxFloor;
   a.pS = a.qS = a.q1S = 0.f;
   a.av = -INFINITY;
   a.ab = 0x7fffffff;
+  a.qv = -INFINITY;
+  a.qb = 0x7fffffff;
 }
 
 // Butterfly reductions over a warp: every lane ends with the same, order-fixed result.
@@ -80,7 +90,7 @@ __device__ __forceinline__ void warp_lse(float& M, float& S, float scale) {
   float m = M;
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
-  float s = (M == -INFINITY) ? 0.f : S * ex2((M - m) * scale);
+  float s = S * ex2((M - m) * scale);
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
   M = m;
@@ -103,12 +113,13 @@ __device__ __forceinline__ void warp_part(RowPart& a, float sT) {
   warp_lse(a.qM, a.qS, sT);
   if (NEED_Q1) warp_lse(a.q1M, a.q1S, kLog2e);
   warp_amax(a.av, a.ab);
+  warp_amax(a.qv, a.qb);
 }
 // A vector's maximum beats the running one: remember it and where its vector starts.
-__device__ __forceinline__ void amax_vec(RowPart& A, float vmax, int base) {
-  const bool take = vmax > A.av;
-  A.av = take ? vmax : A.av;
-  A.ab = take ? base : A.ab;
+__device__ __forceinline__ void amax_vec(float& best, int32_t& at, float vmax, int base) {
+  const bool take = vmax > best;
+  best = take ? vmax : best;
+  at = take ? base : at;
 }
 
 // ---------------------------------------------------------------- per-chunk arithmetic
@@ -118,11 +129,9 @@ __device__ __forceinline__ void amax_vec(RowPart& A, float vmax, int base) {
 // a packed multiply by s, one ex2 and half a packed add.
 template <int NW>
 __device__ __forceinline__ void lse_words(float& M, float& S, const uint32_t* w, float vmax, float s) {
-  if (vmax > M) {
-    S *= ex2((M - vmax) * s);  // M == -inf: ex2(-inf) = 0 and S is still 0
-    M = vmax;
-  }
-  if (M == -INFINITY) return;
+  const float m = fmaxf(M, vmax);  // branch-free: rescale by 2^((M - m) s), 1 when unchanged
+  S *= ex2((M - m) * s);
+  M = m;
   const float nM = -M;
   const float2 s2 = make_float2(s, s), zero2 = make_float2(0.f, 0.f);
   float2 acc0 = zero2, acc1 = zero2;
@@ -155,18 +164,17 @@ __device__ __forceinline__ void phase1_bf16(RowPart& A, const uint4* pv, const u
     qw[4 * v + 2] = qv[v].z;
     qw[4 * v + 3] = qv[v].w;
   }
-  float pm = -INFINITY;
+  float pm = -INFINITY, qm = -INFINITY;
 #pragma unroll
-  for (int v = 0; v < NV; ++v) {  // per-vector maxima of z_p, in element order
-    const uint32_t m2 = bmax2(bmax2(pw[4 * v], pw[4 * v + 1]), bmax2(pw[4 * v + 2], pw[4 * v + 3]));
-    const float vm = fmaxf(bf16_lo(m2), bf16_hi(m2));
-    amax_vec(A, vm, idx0 + v * vstride);
-    pm = fmaxf(pm, vm);
+  for (int v = 0; v < NV; ++v) {  // per-vector maxima of z_p and z_q, in element order
+    const uint32_t mp = bmax2(bmax2(pw[4 * v], pw[4 * v + 1]), bmax2(pw[4 * v + 2], pw[4 * v + 3]));
+    const uint32_t mq = bmax2(bmax2(qw[4 * v], qw[4 * v + 1]), bmax2(qw[4 * v + 2], qw[4 * v + 3]));
+    const float vp = fmaxf(bf16_lo(mp), bf16_hi(mp)), vq = fmaxf(bf16_lo(mq), bf16_hi(mq));
+    amax_vec(A.av, A.ab, vp, idx0 + v * vstride);
+    amax_vec(A.qv, A.qb, vq, idx0 + v * vstride);
+    pm = fmaxf(pm, vp);
+    qm = fmaxf(qm, vq);
   }
-  uint32_t qmw = qw[0];
-#pragma unroll
-  for (int k = 1; k < NW; ++k) qmw = bmax2(qmw, qw[k]);
-  const float qm = fmaxf(bf16_lo(qmw), bf16_hi(qmw));
   lse_words<NW>(A.pM, A.pS, pw, pm, sT);
   lse_words<NW>(A.qM, A.qS, qw, qm, sT);
   if (NEED_Q1) lse_words<NW>(A.q1M, A.q1S, qw, qm, kLog2e);
@@ -239,11 +247,9 @@ __device__ __forceinline__ void find_first(const uint4& pw, const uint4& qw, flo
 
 template <int N>
 __device__ __forceinline__ void lse_vals(float& M, float& S, const float* v, float vmax, float s) {
-  if (vmax > M) {
-    S *= ex2((M - vmax) * s);
-    M = vmax;
-  }
-  if (M == -INFINITY) return;
+  const float m = fmaxf(M, vmax);
+  S *= ex2((M - m) * s);
+  M = m;
   float acc = 0.f;
 #pragma unroll
   for (int e = 0; e < N; ++e) acc += ex2((v[e] - M) * s);
@@ -262,7 +268,8 @@ __device__ __forceinline__ void phase1_vec(RowPart& A, const uint4& pw, const ui
     pm = fmaxf(pm, pv[e]);
     qm = fmaxf(qm, qv[e]);
   }
-  amax_vec(A, pm, idx0);
+  amax_vec(A.av, A.ab, pm, idx0);
+  amax_vec(A.qv, A.qb, qm, idx0);
   lse_vals<E>(A.pM, A.pS, pv, pm, sT);
   lse_vals<E>(A.qM, A.qS, qv, qm, sT);
   if (NEED_Q1) lse_vals<E>(A.q1M, A.q1S, qv, qm, kLog2e);
@@ -319,6 +326,8 @@ __global__ void __launch_bounds__(kThreads, 1) rowstats_stream(RowStatsArgs a, i
     S.abort_flag = 0;
     S.arg_index = 0x7fffffff;
     S.arg_carry = 0.f;
+    S.yarg_index = 0x7fffffff;
+    S.yarg_carry = 0.f;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   __syncthreads();
@@ -404,6 +413,9 @@ __global__ void __launch_bounds__(kThreads, 1) rowstats_stream(RowStatsArgs a, i
       const int cstar = tot.ab == 0x7fffffff ? -1 : tot.ab / CH;
       const int istar = tot.ab == 0x7fffffff ? 0 : (tot.ab - cstar * CH) / E;
       const int tstar = istar % kConsumers;
+      const int cyh = tot.qb == 0x7fffffff ? -1 : tot.qb / CH;  // same for the draft argmax
+      const int iyh = tot.qb == 0x7fffffff ? 0 : (tot.qb - cyh * CH) / E;
+      const int tyh = iyh % kConsumers;
       for (int c = 0; c < nch; ++c, pos.next()) {
         if (wait_phase(&S.full[pos.slot], pos.phase, abort_flag, limit_ns, hdr)) {
           const int e0 = c * CH;
@@ -415,6 +427,13 @@ __global__ void __launch_bounds__(kThreads, 1) rowstats_stream(RowStatsArgs a, i
             find_first<T>(P[istar], Q[istar], tot.av, &at, &carry);
             S.arg_index = tot.ab + at;
             S.arg_carry = carry;
+          }
+          if (c == cyh && t == tyh) {
+            int at;
+            float carry;
+            find_first<T>(Q[iyh], P[iyh], tot.qv, &at, &carry);
+            S.yarg_index = tot.qb + at;
+            S.yarg_carry = carry;
           }
           if (sizeof(T) == 2 && c < nfull) {
 #pragma unroll
@@ -456,8 +475,12 @@ __global__ void __launch_bounds__(kThreads, 1) rowstats_stream(RowStatsArgs a, i
         a.ws.Lsq1[r] = Lsq1;
         a.ws.xstar[r] = S.arg_index;
         a.ws.ag[r] = exp2f(log2_prob(S.arg_carry, kLog2e, Mq1, Lsq1));
+        a.ws.yhat[r] = S.yarg_index;
+        a.ws.zpy[r] = S.yarg_carry;
         S.arg_index = 0x7fffffff;
         S.arg_carry = 0.f;
+        S.yarg_index = 0x7fffffff;
+        S.yarg_carry = 0.f;
       }
       __syncwarp();
     }

@@ -141,3 +141,24 @@ def test_binding_refuses_cpu_tensors():
     with pytest.raises(ValueError, match="CUDA"):
         aal.aal_loss_fwd(p, t, t, None, torch.zeros(1024, dtype=torch.uint8),
                          torch.zeros(1), None)
+
+
+def test_reward_from_loss_argument_checks():
+    lib = aal.library()
+    lp = _prob(N=8, K=4, V=100, mode=aal.AAL_GREEDY, temperature=0.0)
+    code, lsize = _ws_size(lp)
+    rp = _rprob(N=8, K=4, V=100)
+    fake = 1 << 24
+    out = ctypes.c_size_t(0)
+    assert lib.aal_reward_workspace_size(ctypes.byref(rp), ctypes.byref(out)) == 0
+    rsize = out.value
+    call = lambda r, l, lws=fake, lb=lsize: lib.aal_accept_reward_from_loss(
+        ctypes.byref(r), ctypes.byref(l), lws, lb, fake, rsize, fake, fake, fake, None)
+    # shapes must match the loss problem
+    assert call(_rprob(N=8, K=4, V=101), lp) == aal.AAL_ERR_INVALID_ARG
+    # sampling acceptance needs a loss with the sampling term at the same temperature
+    assert call(_rprob(N=8, K=4, V=100, mode=aal.AAL_SAMPLING), lp) == aal.AAL_ERR_INVALID_ARG
+    lps = _prob(N=8, K=4, V=100, mode=aal.AAL_BOTH, temperature=0.9)
+    assert call(_rprob(N=8, K=4, V=100, mode=aal.AAL_SAMPLING, temperature=1.0), lps) == aal.AAL_ERR_INVALID_ARG
+    # the loss workspace must be large enough
+    assert call(rp, lp, fake, lsize - 1) == aal.AAL_ERR_WORKSPACE

@@ -146,3 +146,64 @@ def test_full_prompt_group_sampled_windows(reward_group, mode):
     rl = got["rollout_len"]
     R = got["tau"].astype(np.float64) - got["tau_ref"]
     np.testing.assert_allclose(rl, R.reshape(16, 256).mean(1), atol=1e-6)
+
+
+@pytest.mark.parametrize("dtype,V", [(torch.float32, 1000), (torch.bfloat16, 1001), (torch.bfloat16, 4096),
+                                     (torch.bfloat16, 32000), (torch.bfloat16, 8200)])
+@pytest.mark.parametrize("mode,T", [(aal.AAL_GREEDY, 1.0), (aal.AAL_SAMPLING, 1.0), (aal.AAL_SAMPLING, 0.7)])
+def test_reward_from_loss_statistics(dtype, V, mode, T):
+    """The reward taken from a loss forward's statistics equals the one from a logit pass
+    (greedy bit-exactly; sampling apart from draws on the threshold) and the oracle's."""
+    wpr, rpg = 4, 4
+    target, draft, _ = synth.make_reward_logits(0, seed=V, windows_per_rollout=wpr, rollouts_per_group=rpg * 2,
+                                                K=6, V=V, dtype=dtype)
+    draft[::3] = target[::3]
+    t, d = target.to(DEV), draft.to(DEV)
+    N = t.shape[0]
+    lprob = aal.loss_problem(d, aal.AAL_BOTH, T, 0.5, 0.5)
+    lws = torch.empty(aal.aal_workspace_size(lprob), dtype=torch.uint8, device=DEV)
+    loss = torch.empty(1, device=DEV)
+    aal.aal_loss_fwd(lprob, d, t, None, lws, loss)
+    rprob = aal.reward_problem(d, mode, T, 2.0, 17, 5000, wpr, rpg)
+    rws = torch.empty(aal.aal_reward_workspace_size(rprob), dtype=torch.uint8, device=DEV)
+    tau = torch.full((N,), -1, dtype=torch.int32, device=DEV)
+    rl = torch.full((N // wpr,), float("nan"), device=DEV)
+    adv = torch.full((N // wpr,), float("nan"), device=DEV)
+    aal.aal_accept_reward_from_loss(rprob, lprob, lws, rws, tau, rl, adv)
+    torch.cuda.synchronize()
+    got = dict(tau=tau.cpu().numpy(), rollout_len=rl.cpu().numpy(), advantage=adv.cpu().numpy())
+    logit = run_reward(t, d, None, mode, T, seed=17, row_offset=5000, wpr=wpr, rpg=rpg, clip=2.0)
+    exp = oracle.accept_reward(target, draft, None, OMODE[mode], T, 17, 5000, wpr, rpg, 2.0)
+    _, _, amb = oracle_chunked(t, d, None, mode, T, 17, 5000, np.arange(N))
+    keep = ~amb
+    np.testing.assert_array_equal(got["tau"][keep], exp["tau"][keep])
+    np.testing.assert_array_equal(got["tau"][keep], logit["tau"][keep])
+    if keep.all():
+        np.testing.assert_allclose(got["rollout_len"], exp["rollout_len"], rtol=0, atol=1e-6)
+        np.testing.assert_allclose(got["advantage"], exp["advantage"], rtol=0, atol=1e-5)
+
+
+def test_reward_from_loss_full_size_greedy():
+    """The bench's configuration: V=128256 bf16, 8192 windows of K=7, after the EAL+WTV forward."""
+    target, draft, _ = synth.make_logits("v128k", seed=3, device=DEV)
+    N = target.shape[0]
+    lprob = aal.loss_problem(draft, aal.AAL_BOTH, 1.0, 0.5, 0.5)
+    lws = torch.empty(aal.aal_workspace_size(lprob), dtype=torch.uint8, device=DEV)
+    loss = torch.empty(1, device=DEV)
+    aal.aal_loss_fwd(lprob, draft, target, None, lws, loss)
+    rprob = aal.reward_problem(draft, aal.AAL_GREEDY, 1.0, 5.0, 0, 0, 256, 16)
+    rws = torch.empty(aal.aal_reward_workspace_size(rprob), dtype=torch.uint8, device=DEV)
+    tau = torch.empty(N, dtype=torch.int32, device=DEV)
+    rl = torch.empty(N // 256, device=DEV)
+    adv = torch.empty(N // 256, device=DEV)
+    aal.aal_accept_reward_from_loss(rprob, lprob, lws, rws, tau, rl, adv)
+    logit = run_reward(target, draft, None, aal.AAL_GREEDY, wpr=256, rpg=16)
+    np.testing.assert_array_equal(tau.cpu().numpy(), logit["tau"])
+    np.testing.assert_array_equal(adv.cpu().numpy(), logit["advantage"])
+    # sampled windows against the oracle
+    rng = np.random.default_rng(4)
+    windows = np.array(sorted(set([0, N - 1] + list(rng.choice(N, 30, replace=False)))))
+    tau_o, _, _ = oracle_chunked(target, draft, None, aal.AAL_GREEDY, 1.0, 0, 0, windows)
+    np.testing.assert_array_equal(tau.cpu().numpy()[windows], tau_o)
+    del target, draft
+    torch.cuda.empty_cache()
