@@ -28,10 +28,10 @@ namespace {
 using namespace ptx;
 
 #ifndef AAL_STREAM_SLOTS
-#define AAL_STREAM_SLOTS 7
+#define AAL_STREAM_SLOTS 4
 #endif
 #ifndef AAL_STREAM_SLOT_KB
-#define AAL_STREAM_SLOT_KB 32
+#define AAL_STREAM_SLOT_KB 48
 #endif
 constexpr int kSlots = AAL_STREAM_SLOTS;               // ring slots
 constexpr int kSlotBytes = AAL_STREAM_SLOT_KB * 1024;  // half z_p, half z_q
