@@ -66,6 +66,21 @@ def dist_env():
     return ws, rank, local
 
 
+def max_over_ranks(x: float, ws_count: int, device=None) -> float:
+    """The largest value over all ranks (the job is as slow as its slowest rank)."""
+    if ws_count <= 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def rank_row_offset(rank: int, windows_per_rank: int) -> int:
+    """Global index of a rank's first window: each rank owns a contiguous block of windows, so
+    the counter-based draws of the sampling reward do not depend on the sharding."""
+    return rank * windows_per_rank
+
+
 def measured_peak():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -153,7 +168,7 @@ def run_ours(args, ws_count, rank, local):
     prob = aal.loss_problem(draft, aal.AAL_BOTH, MODE_T, W_G, W_S)
     ws = torch.empty(aal.aal_workspace_size(prob), dtype=torch.uint8, device=dev)
     loss = torch.empty(1, dtype=torch.float32, device=dev)
-    rprob = aal.reward_problem(draft, aal.AAL_GREEDY, 1.0, 5.0, 0, rank * N, wpr, RPG)
+    rprob = aal.reward_problem(draft, aal.AAL_GREEDY, 1.0, 5.0, 0, rank_row_offset(rank, N), wpr, RPG)
     rws = torch.empty(aal.aal_reward_workspace_size(rprob), dtype=torch.uint8, device=dev)
     tau = torch.empty(N, dtype=torch.int32, device=dev)
     nroll = N // wpr
@@ -194,11 +209,7 @@ def run_ours(args, ws_count, rank, local):
     if ws_count > 1:
         torch.distributed.barrier()
     clk = clocks.stop()
-    ms_total = t_start.elapsed_time(t_end)
-    if ws_count > 1:
-        tt = torch.tensor([ms_total], dtype=torch.float64, device=dev)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        ms_total = float(tt.item())
+    ms_total = max_over_ranks(t_start.elapsed_time(t_end), ws_count, dev)
     ms_step = ms_total / args.steps
     per = {"fwd": 0.0, "bwd": 0.0, "reward": 0.0}
     for i in range(args.steps):

@@ -1,0 +1,34 @@
+/*
+ * aal_debug.h -- failure-detection test hook of libaal.so.
+ *
+ * Not part of the computation: it lets a test make one of the library's bounded device
+ * waits run out on purpose, so that the timeout path can be checked on a GPU without a
+ * fault, a trap or a hang.
+ */
+#ifndef AAL_DEBUG_H_
+#define AAL_DEBUG_H_
+
+#include <stdint.h>
+
+#include "aal.h"
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Arms the next aal_loss_fwd that runs the TMA-streamed row kernel (sampling term, rows
+ * a multiple of 16 bytes) to leave the completion barrier of its `chunk`-th ring copy
+ * (counted from 0 in each CTA's stream) unarmed: the consumers of that chunk wait on a
+ * phase that nothing completes.  Every wait of that kernel, and of later ones, gives up
+ * after `wait_limit_ns` (0 restores the default of 1 s); the kernel then records
+ * AAL_ERR_TIMEOUT in the workspace status word, walks its remaining loops without waiting,
+ * drains its copies and returns, so aal_check_device_status() reports AAL_ERR_TIMEOUT and
+ * the context stays usable.  The results of that forward are not valid.  A negative
+ * `chunk` arms nothing.  The chunk setting is consumed by the next forward. */
+AAL_API void aal_debug_fail_next_forward(int64_t chunk, uint64_t wait_limit_ns);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* AAL_DEBUG_H_ */

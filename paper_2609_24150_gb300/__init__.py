@@ -32,6 +32,7 @@ from .aal import (  # noqa: F401
     aal_accept_reward_from_loss,
     aal_accept_reward_noalloc,
     aal_check_device_status,
+    aal_debug_fail_next_forward,
     aal_loss_bwd,
     aal_loss_fwd,
     aal_reward_workspace_size,

@@ -78,6 +78,8 @@ def library() -> ctypes.CDLL:
     lib.aal_accept_reward_noalloc.argtypes = [RP, vp, vp, vp, vp, vp, vp, vp, vp]
     lib.aal_accept_reward_from_loss.argtypes = [RP, P, vp, sz, vp, sz, vp, vp, vp, vp]
     lib.aal_check_device_status.argtypes = [vp, vp]
+    lib.aal_debug_fail_next_forward.argtypes = [ctypes.c_int64, ctypes.c_uint64]
+    lib.aal_debug_fail_next_forward.restype = None
     lib.aal_status_string.argtypes = [ctypes.c_int]
     lib.aal_status_string.restype = ctypes.c_char_p
     lib.aal_abi_version.argtypes = []
@@ -247,3 +249,9 @@ def aal_accept_reward_noalloc(problem: AalRewardProblem, draft, target, ref_draf
 def aal_check_device_status(workspace, stream=None) -> int:
     """Synchronise and return (and clear) the workspace's device status code."""
     return int(library().aal_check_device_status(_ptr(workspace, "workspace"), _stream(stream)))
+
+
+def aal_debug_fail_next_forward(chunk: int, wait_limit_ns: int = 0):
+    """Failure-detection test hook: leave one ring copy of the next streamed forward unarmed
+    so that its bounded waits run out (see include/aal_debug.h)."""
+    library().aal_debug_fail_next_forward(int(chunk), int(wait_limit_ns))

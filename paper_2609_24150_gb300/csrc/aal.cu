@@ -2,13 +2,20 @@
 #include <math.h>
 #include <string.h>
 
+#include <atomic>
+
 #include "aal_internal.cuh"
+#include "../../include/aal_debug.h"
 
 using namespace aal;
 
 namespace {
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// Failure-detection test hooks (include/aal_debug.h).
+std::atomic<uint64_t> g_wait_limit_ns{0};
+std::atomic<int64_t> g_skip_chunk{-1};
 
 aal_status check_shape(int64_t N, int64_t K, int64_t V, int32_t dtype) {
   if (N < 0 || K < 1 || V < 1) return AAL_ERR_INVALID_ARG;
@@ -48,9 +55,19 @@ aal_status cuda_status(cudaError_t e) { return e == cudaSuccess ? AAL_OK : AAL_E
 
 }  // namespace
 
+namespace aal {
+uint64_t debug_wait_limit_ns() { return g_wait_limit_ns.load(); }
+int64_t debug_take_skip_chunk() { return g_skip_chunk.exchange(-1); }
+}  // namespace aal
+
 extern "C" {
 
 int32_t aal_abi_version(void) { return 10000; }
+
+void aal_debug_fail_next_forward(int64_t chunk, uint64_t wait_limit_ns) {
+  g_wait_limit_ns.store(wait_limit_ns);
+  g_skip_chunk.store(chunk);
+}
 
 const char* aal_status_string(aal_status s) {
   switch (s) {
@@ -109,6 +126,7 @@ aal_status aal_loss_fwd(const aal_problem* prob, const void* draft, const void* 
   ra.need_q = sampling;
   ra.need_q1 = greedy && !(sampling && prob->temperature == 1.0f);
   ra.overlap = sampling;
+  ra.skip_chunk = debug_take_skip_chunk();
   ra.ws = ws;
   int cluster = 1;
   e = launch_rowstats(ra, bf16, s, &cluster);

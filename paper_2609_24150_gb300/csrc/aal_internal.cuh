@@ -150,6 +150,7 @@ struct RowStatsArgs {
   bool need_q;          // log-sum-exp of z_q / T   (sampling term)
   bool need_q1;         // log-sum-exp of z_q       (greedy term, when T != 1 or no sampling)
   bool overlap;         // second phase: sum min(p~, q~) and Qlt (sampling term)
+  int64_t skip_chunk;   // failure-detection test hook: a chunk whose copy is never armed (-1: none)
   LossWs ws;
 };
 
@@ -224,6 +225,10 @@ struct RewardGroupArgs {
 cudaError_t launch_rowstats(const RowStatsArgs& a, bool bf16, cudaStream_t s, int* cluster_used);
 cudaError_t launch_rowstats_stream(const RowStatsArgs& a, bool bf16, cudaStream_t s, uint64_t limit_ns);
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // bounded waits give up after 1 s
+
+// Failure-detection test hooks (include/aal_debug.h); both are 0 / -1 in normal use.
+uint64_t debug_wait_limit_ns();
+int64_t debug_take_skip_chunk();
 cudaError_t launch_window(const WindowArgs& a, cudaStream_t s);
 cudaError_t launch_backward(const BackwardArgs& a, bool bf16, cudaStream_t s);
 cudaError_t launch_reward_rows(const RewardRowArgs& a, bool bf16, cudaStream_t s);

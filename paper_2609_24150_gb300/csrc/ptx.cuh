@@ -92,6 +92,7 @@ template <bool CLUSTER = false>
 __device__ __forceinline__ bool wait_phase(uint64_t* b, uint32_t parity, volatile int* abort_flag,
                                            uint64_t limit_ns, WsHeader* hdr) {
   constexpr uint32_t kSuspendNs = 100000;
+  if (*abort_flag) return false;
   if (CLUSTER ? mbar_try_cluster(b, parity, kSuspendNs) : mbar_try(b, parity, kSuspendNs)) return !*abort_flag;
   const uint64_t t0 = now_ns();
   for (uint32_t it = 0; it < kSpinLimit; ++it) {

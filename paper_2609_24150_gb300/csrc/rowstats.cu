@@ -238,7 +238,8 @@ cudaError_t launch_rowstats(const RowStatsArgs& a, bool bf16, cudaStream_t s, in
                        ((reinterpret_cast<uintptr_t>(a.zq) | reinterpret_cast<uintptr_t>(a.zp)) % 16 == 0);
   if (a.overlap && aligned) {
     *cluster_used = 1;
-    return launch_rowstats_stream(a, bf16, s, kWaitLimitNs);
+    const uint64_t limit = debug_wait_limit_ns();
+    return launch_rowstats_stream(a, bf16, s, limit ? limit : kWaitLimitNs);
   }
   *cluster_used = 1;
   return bf16 ? launch_generic<uint16_t>(a, s) : launch_generic<float>(a, s);

@@ -1,0 +1,33 @@
+"""Failure detection on the GPU without a fault: a bounded device wait is made to run out
+(a ring copy whose barrier nothing completes), the kernel reports AAL_ERR_TIMEOUT through the
+workspace status word and returns, and the context stays usable for the next call."""
+
+import pytest
+import torch
+
+import paper_2609_24150_gb300 as aal
+import synth
+from tests.parity import LossRun, check_loss
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda:0"
+
+
+@pytest.mark.parametrize("chunk", [0, 1, 3])
+def test_bounded_wait_times_out_and_context_stays_usable(chunk):
+    target, draft, _ = synth.make_logits("tiny", seed=11, N=16, K=2, V=20000, dtype=torch.bfloat16)
+    t, d = target.to(DEV), draft.to(DEV)
+    prob = aal.loss_problem(d, aal.AAL_BOTH, 1.0, 0.5, 0.5)
+    ws = torch.empty(aal.aal_workspace_size(prob), dtype=torch.uint8, device=DEV)
+    loss = torch.empty(1, device=DEV)
+    aal.aal_debug_fail_next_forward(chunk, 50_000_000)        # waits give up after 50 ms
+    try:
+        aal.aal_loss_fwd(prob, d, t, None, ws, loss)
+        assert aal.aal_check_device_status(ws) == aal.AAL_ERR_TIMEOUT
+        assert aal.aal_check_device_status(ws) == aal.AAL_OK  # the status word was cleared
+    finally:
+        aal.aal_debug_fail_next_forward(-1, 0)                # default limit again
+    # the same context runs the next forward and backward correctly
+    run = LossRun(t, d, None, aal.AAL_BOTH, 1.0, 0.5, 0.5, dloss=16.0)
+    check_loss(run, t, d, None, aal.AAL_BOTH, 1.0, 0.5, 0.5, dloss=16.0)

@@ -1,0 +1,73 @@
+"""The N > 1 path on the CPU: two gloo ranks.
+
+Windows are independent, so ranks shard them with no collective on the data path; only the
+step time is reduced (max over ranks).  The reward's counter-based draws are keyed by the
+global window index, so a sharded run reproduces the unsharded one exactly, and per-rank
+loss partials (sum of w * E[L], |W|) combine into the global loss with one all-reduce.
+"""
+
+import multiprocessing as mp
+import os
+import socket
+
+import numpy as np
+import pytest
+import torch
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _worker(rank, world, port, out):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank), WORLD_SIZE=str(world))
+    import torch.distributed as dist
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        import bench
+        import oracle
+        import synth
+        res = {"max": bench.max_over_ranks(float(10 * (rank + 1)), world)}
+        # the whole batch, drawn identically on every rank; each rank keeps its shard
+        target, draft, _ = synth.make_logits("tiny", seed=3, N=8, K=4, V=64)
+        per = 8 // world
+        lo = bench.rank_row_offset(rank, per)
+        t, d = target[lo:lo + per], draft[lo:lo + per]
+        rw = oracle.accept_reward(t, d, None, 2, 0.9, seed=7, row_offset=lo, windows_per_rollout=2,
+                                  rollouts_per_group=2)
+        taus = [torch.zeros(per, dtype=torch.int64) for _ in range(world)]
+        dist.all_gather(taus, torch.as_tensor(rw["tau"]))
+        res["tau"] = torch.cat(taus).numpy()
+        fw = oracle.loss_forward(t, d, None, oracle.MODE_BOTH, 0.9, 0.5, 0.5)
+        part = torch.tensor([0.5 * fw["eal_g"].sum() + 0.5 * fw["eal_s"].sum(), float(fw["nvalid"])],
+                            dtype=torch.float64)
+        dist.all_reduce(part)
+        res["loss"] = float(-part[0] / part[1])
+        out.put((rank, res))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_two_gloo_ranks():
+    ctx = mp.get_context("spawn")
+    out = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_worker, args=(r, 2, port, out)) for r in range(2)]
+    for p in procs:
+        p.start()
+    results = dict(out.get(timeout=240) for _ in procs)
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    import oracle
+    import synth
+    target, draft, _ = synth.make_logits("tiny", seed=3, N=8, K=4, V=64)
+    whole = oracle.accept_reward(target, draft, None, 2, 0.9, seed=7, row_offset=0, windows_per_rollout=2,
+                                 rollouts_per_group=2)
+    ref_loss = oracle.loss_forward(target, draft, None, oracle.MODE_BOTH, 0.9, 0.5, 0.5)["loss"]
+    for r in range(2):
+        assert results[r]["max"] == 20.0
+        np.testing.assert_array_equal(results[r]["tau"], whole["tau"])
+        assert abs(results[r]["loss"] - ref_loss) < 1e-12
