@@ -47,3 +47,4 @@ from .reward import (  # noqa: F401
     simulated_accept_length,
 )
 from .philox import philox4x32_10, uniform01  # noqa: F401
+from .sequence import gather_windows, seq_loss_backward, seq_loss_forward  # noqa: F401

@@ -1,0 +1,95 @@
+"""Pins of the sliding-window sequence loss (oracle/sequence.py), CPU only."""
+
+from fractions import Fraction
+
+import numpy as np
+import pytest
+
+import oracle
+from oracle.sequence import gather_windows, seq_loss_backward, seq_loss_forward
+from tests.spec_sim import expected_accepted_length_greedy, expected_accepted_length_sampling
+
+
+def _rational_dist(rng, V, denom=10):
+    w = rng.integers(1, denom, size=V)
+    s = int(w.sum())
+    return [Fraction(int(x), s) for x in w]
+
+
+def test_every_window_equals_brute_force_verification():
+    """Each window starting at t covers positions t..t+K-1 of the sequence (truncated at its end)
+    and its E[L] equals enumerated speculative verification over exactly those positions."""
+    rng = np.random.default_rng(0)
+    Tn, K, V = 5, 3, 3
+    p = [_rational_dist(rng, V) for _ in range(Tn)]
+    q = [_rational_dist(rng, V) for _ in range(Tn)]
+    zp = np.log(np.array([[[float(x) for x in r] for r in p]]))
+    zq = np.log(np.array([[[float(x) for x in r] for r in q]]))
+    fw = seq_loss_forward(zp, zq, None, K, oracle.MODE_BOTH, 1.0, 1.0, 1.0)
+    pstar = [max(range(V), key=lambda v: (r[v], -v)) for r in p]
+    total = 0.0
+    for t in range(Tn):
+        span = range(t, min(t + K, Tn))
+        es = expected_accepted_length_sampling([p[i] for i in span], [q[i] for i in span])
+        eg = expected_accepted_length_greedy([pstar[i] for i in span], [q[i] for i in span])
+        assert abs(fw["eal_s"][t] - float(es)) < 1e-13
+        assert abs(fw["eal_g"][t] - float(eg)) < 1e-13
+        total += float(es) + float(eg)
+    assert fw["nvalid"] == Tn
+    assert abs(fw["loss"] + total / Tn) < 1e-13
+
+
+def test_invalid_positions_end_windows_and_start_none():
+    rng = np.random.default_rng(1)
+    B, Tn, K, V = 2, 6, 3, 4
+    zp = rng.normal(size=(B, Tn, V))
+    zq = rng.normal(size=(B, Tn, V))
+    mask = np.ones((B, Tn), dtype=np.uint8)
+    mask[0, 2] = 0
+    mask[1, 4:] = 0           # padding at the end of sequence 1
+    fw = seq_loss_forward(zp, zq, mask, K)
+    kn = fw["kn"].reshape(B, Tn)
+    assert list(kn[0]) == [2, 1, 0, 3, 2, 1]
+    assert list(kn[1]) == [3, 3, 2, 1, 0, 0]
+    assert fw["nvalid"] == 9
+
+
+def test_window_size_one_is_the_mean_acceptance():
+    rng = np.random.default_rng(2)
+    zp = rng.normal(size=(2, 7, 9))
+    zq = rng.normal(size=(2, 7, 9))
+    fw = seq_loss_forward(zp, zq, None, 1, oracle.MODE_SAMPLING, 0.8)
+    a = oracle.acceptance_sampling(zp, zq, 0.8)
+    assert abs(fw["loss"] + a.mean()) < 1e-14
+
+
+@pytest.mark.parametrize("mode,T", [(oracle.MODE_BOTH, 1.0), (oracle.MODE_SAMPLING, 0.7), (oracle.MODE_GREEDY, 1.0)])
+def test_sequence_gradient_by_finite_differences(mode, T):
+    """Positions shared by up to K windows: the summed gradient against central differences."""
+    rng = np.random.default_rng(3)
+    B, Tn, K, V = 1, 5, 3, 6
+    while True:
+        zp = rng.normal(0, 1.5, size=(B, Tn, V))
+        zq = zp + rng.normal(0, 1.0, size=(B, Tn, V))
+        pt = np.exp(oracle.log_softmax(zp, T)); qt = np.exp(oracle.log_softmax(zq, T))
+        if np.min(np.abs(pt - qt)) > 1e-3:
+            break
+    mask = np.ones((B, Tn), dtype=np.uint8)
+    mask[0, 3] = 0
+    kw = dict(mode=mode, T=T, w_greedy=0.4, w_sampling=0.6)
+    g = seq_loss_backward(zp, zq, mask, K, dloss=3.0, **kw)
+    h = 1e-6
+    for idx in np.ndindex(B, Tn, V):
+        a = zq.copy(); a[idx] += h
+        b = zq.copy(); b[idx] -= h
+        fd = 3.0 * (seq_loss_forward(zp, a, mask, K, **kw)["loss"] - seq_loss_forward(zp, b, mask, K, **kw)["loss"]) / (2 * h)
+        assert abs(fd - g[idx]) < 1e-7, (idx, fd, g[idx])
+
+
+def test_gathered_windows_point_back_to_their_positions():
+    zp = np.arange(2 * 4 * 3, dtype=np.float64).reshape(2, 4, 3)
+    wp, wq, wm, src = gather_windows(zp, zp, None, 3)
+    assert src[5].tolist() == [5, 6, 7]          # sequence 1, t = 1
+    assert src[7].tolist() == [7, -1, -1]         # last position of sequence 1
+    assert wm[7].tolist() == [1, 0, 0]
+    np.testing.assert_array_equal(wp[5, 1], zp[1, 2])
