@@ -4,7 +4,9 @@ A plain, slow, fp64 CPU restatement of what the paper defines: the per-position
 acceptance probabilities under greedy and sampling verification (Sec. 2.3,
 Eqs. acc_greedy / acc_sample), the speculative-window expected accepted length
 (Sec. 3.1, Eq. eal_generic), the EAL and WTV losses (Eqs. loss_eal / loss_tv)
-with their gradient with respect to the draft logits, and the GRPO stage's
+with their gradient with respect to the draft logits, over independent windows and
+over whole sequences (Sec. 3.3), the forward-KL anchor of the combined objectives
+(Sec. 4.1), and the GRPO stage's
 simulated acceptance length, debiased reward and group-normalised advantage
 (Sec. 3.4).  Every function computes its definition directly, with numpy in
 float64, so that a reader can check it against the paper by eye; nothing here
@@ -47,4 +49,18 @@ from .reward import (  # noqa: F401
     simulated_accept_length,
 )
 from .philox import philox4x32_10, uniform01  # noqa: F401
-from .sequence import gather_windows, seq_loss_backward, seq_loss_forward  # noqa: F401
+from .sequence import (  # noqa: F401
+    gather_windows,
+    seq_loss_backward,
+    seq_loss_forward,
+    seq_objective_backward,
+    seq_objective_forward,
+)
+from .anchor import (  # noqa: F401
+    MODE_KL,
+    anchor_backward,
+    anchor_forward,
+    kl_divergence,
+    objective_backward,
+    objective_forward,
+)

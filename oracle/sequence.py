@@ -3,9 +3,12 @@
 Sec. 3.3 (Fig. wtv and its description): the draft and the target each run once over a
 sequence, every position t gets its acceptance a_t, and a window of size gamma starts at
 every position and slides by one; the loss accumulates -E[L_t] over all window starts W.
-Windows that run past the end of a sequence, or into an invalid position, are truncated
-there (the same reading as for masked windows of the windowed layout), and a start belongs
-to W iff its own position is valid.
+The paper does not say what happens at the end of a sequence.  Two readings are offered:
+by default a window that runs past the end, or into an invalid position, is truncated there
+(the same reading as for masked windows of the windowed layout) and a start belongs to W iff
+its own position is valid; with ``full_windows`` only windows whose gamma positions are all
+valid and inside the sequence belong to W (for an unmasked sequence of length T, the starts
+0 .. T - gamma).
 
 The sequence loss is the windowed loss of losses.py applied to the gathered windows; its
 gradient with respect to a position's draft logits is the sum of the gradients of the rows
@@ -16,12 +19,13 @@ from __future__ import annotations
 
 import numpy as np
 
-from .losses import MODE_BOTH, as_f64, loss_backward, loss_forward
+from .losses import MODE_BOTH, as_f64, leading_valid_depths, loss_backward, loss_forward
 
 
-def gather_windows(target, draft, mask, K: int):
+def gather_windows(target, draft, mask, K: int, full_windows: bool = False):
     """[B][T][V] logits -> [B*T][K][V] windows (window n = b*T + t covers positions t..t+K-1)
-    and their [B*T][K] validity (position valid and inside the sequence)."""
+    and their [B*T][K] validity (position valid and inside the sequence; with ``full_windows``
+    every depth of a window with fewer than K leading valid positions is invalid)."""
     zp = as_f64(target)
     zq = as_f64(draft)
     B, T, V = zp.shape
@@ -40,27 +44,61 @@ def gather_windows(target, draft, mask, K: int):
                     wq[n, j] = zq[b, p]
                     wm[n, j] = 1 if valid[b, p] else 0
                     src[n, j] = b * T + p
+    if full_windows:
+        wm[leading_valid_depths(wm, B * T, K) < K] = 0
     return wp, wq, wm, src
 
 
 def seq_loss_forward(target, draft, mask, K: int, mode: int = MODE_BOTH, T: float = 1.0,
-                     w_greedy: float = 1.0, w_sampling: float = 1.0):
-    """The loss over every sliding window of every sequence (see the module docstring)."""
-    wp, wq, wm, _ = gather_windows(target, draft, mask, K)
-    return loss_forward(wp, wq, wm, mode, T, w_greedy, w_sampling)
+                     w_greedy: float = 1.0, w_sampling: float = 1.0, n_windows_total=None,
+                     full_windows: bool = False):
+    """The loss over every sliding window of every sequence (see the module docstring).
+    ``n_windows_total`` replaces |W| when the sequences given are a slice of a larger batch."""
+    wp, wq, wm, _ = gather_windows(target, draft, mask, K, full_windows)
+    return loss_forward(wp, wq, wm, mode, T, w_greedy, w_sampling, n_windows_total)
 
 
 def seq_loss_backward(target, draft, mask, K: int, mode: int = MODE_BOTH, T: float = 1.0,
-                      w_greedy: float = 1.0, w_sampling: float = 1.0, dloss: float = 1.0) -> np.ndarray:
+                      w_greedy: float = 1.0, w_sampling: float = 1.0, dloss: float = 1.0,
+                      n_windows_total=None, full_windows: bool = False) -> np.ndarray:
     """dloss * dL/dz_q per position, [B][T][V]: the window rows' gradients added back to the
-    positions they were gathered from."""
+    positions they were gathered from (|W| replaced by ``n_windows_total`` when given)."""
     zq = as_f64(draft)
     B, Tn, V = zq.shape
-    wp, wq, wm, src = gather_windows(target, draft, mask, K)
-    g = loss_backward(wp, wq, wm, mode, T, w_greedy, w_sampling, dloss)
+    wp, wq, wm, src = gather_windows(target, draft, mask, K, full_windows)
+    g = loss_backward(wp, wq, wm, mode, T, w_greedy, w_sampling, dloss, n_windows_total)
     out = np.zeros((B * Tn, V))
     for n in range(B * Tn):
         for j in range(K):
             if src[n, j] >= 0:
                 out[src[n, j]] += g[n, j]
     return out.reshape(B, Tn, V)
+
+
+def seq_objective_forward(target, draft, mask, K: int, mode: int = 5, T: float = 1.0,
+                          w_greedy: float = 1.0, w_sampling: float = 1.0, w_kl: float = 1.0,
+                          n_windows_total=None, n_positions_total=None, full_windows: bool = False):
+    """w_kl L_KL + w_g L_EAL + w_s L_WTV over whole sequences: the window terms as in
+    seq_loss_forward, the anchor once per valid position (anchor.py)."""
+    from .anchor import MODE_KL, anchor_forward
+    fw = seq_loss_forward(target, draft, mask, K, mode & 3, T, w_greedy, w_sampling, n_windows_total,
+                          full_windows)
+    if mode & MODE_KL:
+        an = anchor_forward(target, draft, mask, n_positions_total)
+        fw["loss"] += w_kl * an["loss"]
+        fw["kl"] = an["kl"]
+        fw["npos"] = an["npos"]
+    return fw
+
+
+def seq_objective_backward(target, draft, mask, K: int, mode: int = 5, T: float = 1.0,
+                           w_greedy: float = 1.0, w_sampling: float = 1.0, w_kl: float = 1.0,
+                           dloss: float = 1.0, n_windows_total=None, n_positions_total=None,
+                           full_windows: bool = False) -> np.ndarray:
+    """dloss * d(objective)/dz_q per position, [B][T][V]."""
+    from .anchor import MODE_KL, anchor_backward
+    g = seq_loss_backward(target, draft, mask, K, mode & 3, T, w_greedy, w_sampling, dloss,
+                          n_windows_total, full_windows)
+    if mode & MODE_KL:
+        g = g + anchor_backward(target, draft, mask, dloss * w_kl, n_positions_total)
+    return g

@@ -93,3 +93,50 @@ def test_gathered_windows_point_back_to_their_positions():
     assert src[7].tolist() == [7, -1, -1]         # last position of sequence 1
     assert wm[7].tolist() == [1, 0, 0]
     np.testing.assert_array_equal(wp[5, 1], zp[1, 2])
+
+
+def test_slice_around_a_position_gives_its_gradient():
+    """The full-size GPU tests check sampled positions against the oracle run on the positions
+    t-K+1 .. t+K-1 only, with |W| of the whole batch: every window containing t lies inside."""
+    rng = np.random.default_rng(4)
+    B, Tn, K, V = 2, 12, 3, 5
+    zp = rng.normal(size=(B, Tn, V))
+    zq = zp + rng.normal(size=(B, Tn, V))
+    mask = np.ones((B, Tn), dtype=np.uint8)
+    mask[1, 7] = 0
+    full = seq_loss_backward(zp, zq, mask, K, oracle.MODE_BOTH, 0.9, 0.3, 0.7, 2.0)
+    fw = seq_loss_forward(zp, zq, mask, K, oracle.MODE_BOTH, 0.9, 0.3, 0.7)
+    for b, t in [(0, 0), (0, 5), (1, 6), (1, 8), (1, 11)]:
+        lo, hi = max(0, t - K + 1), min(Tn, t + K)
+        g = seq_loss_backward(zp[b:b + 1, lo:hi], zq[b:b + 1, lo:hi], mask[b:b + 1, lo:hi], K,
+                              oracle.MODE_BOTH, 0.9, 0.3, 0.7, 2.0, n_windows_total=fw["nvalid"])
+        np.testing.assert_allclose(g[0, t - lo], full[b, t], rtol=0, atol=1e-15)
+
+
+def test_full_windows_reading_keeps_only_complete_windows():
+    """With full_windows, an unmasked sequence of length T has the windows starting at
+    0 .. T-K only, each equal to brute-force verification over its K positions; a hole removes
+    every window that would cover it."""
+    rng = np.random.default_rng(5)
+    Tn, K, V = 6, 3, 3
+    p = [_rational_dist(rng, V) for _ in range(Tn)]
+    q = [_rational_dist(rng, V) for _ in range(Tn)]
+    zp = np.log(np.array([[[float(x) for x in r] for r in p]]))
+    zq = np.log(np.array([[[float(x) for x in r] for r in q]]))
+    fw = seq_loss_forward(zp, zq, None, K, oracle.MODE_SAMPLING, full_windows=True)
+    assert fw["nvalid"] == Tn - K + 1
+    total = 0.0
+    for t in range(Tn):
+        if t <= Tn - K:
+            es = float(expected_accepted_length_sampling(p[t:t + K], q[t:t + K]))
+            assert abs(fw["eal_s"][t] - es) < 1e-13
+            total += es
+        else:
+            assert fw["eal_s"][t] == 0.0
+    assert abs(fw["loss"] + total / (Tn - K + 1)) < 1e-13
+    mask = np.ones((1, Tn), dtype=np.uint8)
+    mask[0, 3] = 0
+    fw = seq_loss_forward(zp, zq, mask, K, oracle.MODE_SAMPLING, full_windows=True)
+    assert list(fw["kn"]) == [3, 0, 0, 0, 0, 0]
+    g = seq_loss_backward(zp, zq, mask, K, oracle.MODE_SAMPLING, full_windows=True)
+    assert np.all(g[0, 3:] == 0) and np.any(g[0, :3] != 0)
