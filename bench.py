@@ -54,6 +54,7 @@ def parse():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-seq", action="store_true", help="skip the sequence-layout measurement")
     ap.add_argument("--windows", type=int, default=None,
                     help="run the first WINDOWS windows of the workload (profiling captures)")
     return ap.parse_args()
@@ -232,6 +233,10 @@ def run_ours(args, ws_count, rank, local):
     torch.cuda.synchronize()
     ms_reward_pass = r0.elapsed_time(r1) / reps
 
+    greedy_obj = None if args.no_seq else run_greedy_objective(aal, draft, target, grad, stream,
+                                                                max(5, args.steps // 2))
+    seq = None if args.no_seq else run_sequence_layout(aal, dev, stream, rank, max(5, args.steps // 2))
+
     b = algo_bytes(N, K, V)
     step_bytes = sum(b.values())
     R = N * K
@@ -279,6 +284,10 @@ def run_ours(args, ws_count, rank, local):
                      "algorithmic_bytes": b[dom]},
         "clocks": clk,
     }
+    if greedy_obj is not None:
+        res["greedy_objective"] = greedy_obj
+    if seq is not None:
+        res["sequence_layout"] = seq
 
     if rank == 0 and not args.no_e2e:
         res["e2e"] = run_e2e(args, aal, prob, rprob, draft, target, grad, ws, loss, rws, tau, rl, adv,
@@ -286,6 +295,77 @@ def run_ours(args, ws_count, rank, local):
     if rank == 0 and ws_count == 1 and not args.no_cpu_baseline:
         res["cpu_baseline"] = cpu_baseline(draft, target, args.cpu_seconds)
     return res
+
+
+def _time_fwd_bwd(aal, fwd, bwd, stream, reps):
+    """Mean fwd and bwd milliseconds over ``reps`` pairs, events on the launching stream."""
+    for _ in range(3):
+        fwd()
+        bwd()
+    torch.cuda.synchronize()
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(reps)]
+    for e in ev:
+        e[0].record(stream)
+        fwd()
+        e[1].record(stream)
+        bwd()
+        e[2].record(stream)
+    torch.cuda.synchronize()
+    return (sum(e[0].elapsed_time(e[1]) for e in ev) / reps, sum(e[1].elapsed_time(e[2]) for e in ev) / reps)
+
+
+def run_greedy_objective(aal, draft, target, grad, stream, reps):
+    """The paper's greedy-regime objective L_KL + 0.1 L_EAL (Sec. 4.1) on the same batch:
+    one pass over both rows forward (normalisers, x*, KL), target + draft read and the
+    gradient written backward."""
+    N, K, V = draft.shape
+    prob = aal.loss_problem(draft, aal.AAL_KL | aal.AAL_GREEDY, 1.0, 0.1, 0.0, 1.0)
+    ws = torch.empty(aal.aal_workspace_size(prob), dtype=torch.uint8, device=draft.device)
+    loss = torch.empty(1, dtype=torch.float32, device=draft.device)
+    fwd, bwd = _time_fwd_bwd(
+        aal, lambda: aal.aal_loss_fwd(prob, draft, target, None, ws, loss, None, stream),
+        lambda: aal.aal_loss_bwd(prob, draft, target, None, ws, 1.0, grad, stream), stream, reps)
+    assert aal.aal_check_device_status(ws) == aal.AAL_OK
+    R = N * K
+    row = V * draft.element_size()
+    fb, bb = 2 * R * row, 3 * R * row
+    out = {"workload": f"v128k: N={N} windows, K={K}, V={V} bf16; L_KL + 0.1 L_EAL fwd+bwd",
+           "ms": round(fwd + bwd, 4), "fwd_ms": round(fwd, 4), "bwd_ms": round(bwd, 4),
+           "gbs": round((fb + bb) / ((fwd + bwd) * 1e-3) / 1e9, 1),
+           "fwd_gbs": round(fb / (fwd * 1e-3) / 1e9, 1), "bwd_gbs": round(bb / (bwd * 1e-3) / 1e9, 1),
+           "rows_per_s": round(R / ((fwd + bwd) * 1e-3), 1), "loss": float(loss.item())}
+    del ws
+    return out
+
+
+def run_sequence_layout(aal, dev, stream, rank, reps):
+    """The same loss over the sequence layout (Sec. 3.3): 4 sequences x 2048 positions, a window
+    of K=7 starting at every position, logits stored once per position; fwd + bwd timed with
+    events on the launching stream.  Unmasked, so every row is read (and written) once."""
+    target, draft, _ = synth.make_seq_logits("seq_v128k", seed=rank, device=dev, masked=False)
+    B, T, V = draft.shape
+    K = synth.SEQUENCES["seq_v128k"].K
+    grad = torch.empty_like(draft)
+    prob = aal.seq_problem(draft, K, aal.AAL_BOTH, MODE_T, W_G, W_S)
+    ws = torch.empty(aal.aal_seq_workspace_size(prob), dtype=torch.uint8, device=dev)
+    loss = torch.empty(1, dtype=torch.float32, device=dev)
+    fwd, bwd = _time_fwd_bwd(
+        aal, lambda: aal.aal_seq_loss_fwd(prob, draft, target, None, ws, loss, None, stream),
+        lambda: aal.aal_seq_loss_bwd(prob, draft, target, None, ws, 1.0, grad, stream), stream, reps)
+    assert aal.aal_check_device_status(ws) == aal.AAL_OK
+    R = B * T
+    row = V * draft.element_size()
+    fb, bb = 2 * R * row, 3 * R * row
+    out = {"workload": f"seq_v128k: B={B} x T={T} positions, K={K}, V={V} bf16, unmasked; "
+                       "EAL+WTV 0.5/0.5 at T=1 fwd+bwd",
+           "ms": round(fwd + bwd, 4), "fwd_ms": round(fwd, 4), "bwd_ms": round(bwd, 4),
+           "gbs": round((fb + bb) / ((fwd + bwd) * 1e-3) / 1e9, 1),
+           "fwd_gbs": round(fb / (fwd * 1e-3) / 1e9, 1), "bwd_gbs": round(bb / (bwd * 1e-3) / 1e9, 1),
+           "positions_per_s": round(R / ((fwd + bwd) * 1e-3), 1),
+           "windows_per_s": round(R / ((fwd + bwd) * 1e-3), 1),
+           "loss": float(loss.item())}
+    del target, draft, grad, ws
+    return out
 
 
 def host_memory_bytes():

@@ -62,9 +62,13 @@ typedef enum {
 
 typedef enum { AAL_F32 = 0, AAL_BF16 = 1 } aal_dtype;
 
-/* Which loss terms to compute.  GREEDY: L_EAL (Eq. loss_eal); SAMPLING: L_WTV
- * (Eq. loss_tv); BOTH: w_greedy * L_EAL + w_sampling * L_WTV. */
-typedef enum { AAL_GREEDY = 1, AAL_SAMPLING = 2, AAL_BOTH = 3 } aal_mode;
+/* Which loss terms to compute (bits).  GREEDY: L_EAL (Eq. loss_eal); SAMPLING: L_WTV
+ * (Eq. loss_tv); BOTH: w_greedy * L_EAL + w_sampling * L_WTV.  KL adds w_kl * L_KL, the
+ * forward-KL anchor of the combined objectives (Sec. 4.1): the mean over valid positions of
+ * KL(p || q) = sum_v p(v) (log p(v) - log q(v)) at T = 1.  The greedy-regime objective of
+ * Sec. 4.1, L_KL + 0.1 L_EAL, is mode AAL_KL | AAL_GREEDY with w_kl = 1, w_greedy = 0.1;
+ * mode AAL_KL alone is the L_KL baseline.  Valid modes: 1 .. 7. */
+typedef enum { AAL_GREEDY = 1, AAL_SAMPLING = 2, AAL_BOTH = 3, AAL_KL = 4 } aal_mode;
 
 #define AAL_MAX_K 8
 
@@ -76,8 +80,8 @@ typedef enum { AAL_GREEDY = 1, AAL_SAMPLING = 2, AAL_BOTH = 3 } aal_mode;
  *                and > 0 when mode includes SAMPLING.  The greedy acceptance
  *                a = q(x*) (Eq. acc_greedy) always uses the unscaled draft, so T is
  *                ignored (and may be 0) for mode GREEDY.
- *   w_greedy, w_sampling  weights of the two terms (used by every mode; a term the mode
- *                does not select is not computed).  Must be finite. */
+ *   w_greedy, w_sampling, w_kl  weights of the terms (a term the mode does not select is
+ *                not computed and its weight is ignored).  Must be finite. */
 typedef struct {
   int64_t N, K, V;
   int32_t dtype;
@@ -85,15 +89,18 @@ typedef struct {
   float temperature;
   float w_greedy;
   float w_sampling;
+  float w_kl;
   int32_t reserved; /* must be 0 */
 } aal_problem;
 
 /* Bytes of device workspace a loss problem needs (host-only, launches nothing). */
 AAL_API aal_status aal_workspace_size(const aal_problem* prob, size_t* bytes);
 
-/* Forward of the loss (Sec. 3.2 Eq. loss_eal, Sec. 3.3 Eq. loss_tv):
+/* Forward of the loss (Sec. 3.2 Eq. loss_eal, Sec. 3.3 Eq. loss_tv, Sec. 4.1):
  *   L = -(1/|W|) sum_n [ w_g sum_{k=1}^{K_n} prod_{j<k} a^g_{n,j}
  *                       + w_s sum_{k=1}^{K_n} prod_{j<k} a^s_{n,j} ]
+ *       + w_kl (1/|P|) sum_{valid rows r} KL(p_r || q_r)     (mode bit AAL_KL; |P| = number
+ *                                                            of rows with mask 1; 0 if none)
  * with a^g = q(x*) (Eq. acc_greedy, x* = target argmax, lowest index on ties) and
  * a^s = sum_v min(p~, q~) = 1 - TV(p~, q~) (Eqs. acc_sample, rejection_rate).
  *   draft, target  [N][K][V] logits of the draft (z_q) and the target (z_p).
@@ -117,6 +124,57 @@ AAL_API aal_status aal_loss_fwd(const aal_problem* prob, const void* draft, cons
 AAL_API aal_status aal_loss_bwd(const aal_problem* prob, const void* draft, const void* target,
                         const uint8_t* mask, const void* workspace, size_t workspace_bytes,
                         float dloss, void* grad_draft, void* stream);
+
+/* Sequence layout (Sec. 3.3): the draft and the target run once over whole sequences, and a
+ * window of gamma = K positions starts at every position and slides by one, so each position
+ * is depth j of up to K windows.  Logits are stored once per position, not once per window.
+ *   B, seq_len, K, V  sequences, positions per sequence (>= 0), window size gamma
+ *                     (1..AAL_MAX_K), vocabulary size (>= 1).
+ *   dtype, mode, temperature, w_greedy, w_sampling, w_kl, reserved  as in aal_problem
+ *                     (the anchor averages over the valid positions).
+ *   full_windows      which windows belong to W (the paper leaves the end of a sequence open):
+ *                     0 = every start position, its window truncated at the end of the
+ *                     sequence or at its first invalid position (as a masked window of
+ *                     aal_loss_fwd); 1 = only windows whose K positions are all valid and
+ *                     inside the sequence (starts 0 .. seq_len - K of an unmasked sequence). */
+typedef struct {
+  int64_t B, seq_len, K, V;
+  int32_t dtype;
+  int32_t mode;
+  float temperature;
+  float w_greedy;
+  float w_sampling;
+  float w_kl;
+  int32_t full_windows;
+  int32_t reserved; /* must be 0 */
+} aal_seq_problem;
+
+/* Bytes of device workspace a sequence problem needs (host-only, launches nothing). */
+AAL_API aal_status aal_seq_workspace_size(const aal_seq_problem* prob, size_t* bytes);
+
+/* Forward of the loss over every sliding window of every sequence:
+ *   L = -(1/|W|) sum_{b,t} [ w_g E^g_{b,t} + w_s E^s_{b,t} ],
+ * where the window starting at position t of sequence b covers positions t .. t+K-1 and stops
+ * at the end of the sequence or at its first invalid position (K_{b,t} = the number of leading
+ * valid positions; the window is in W iff K_{b,t} >= 1, i.e. iff position t is valid, or with
+ * full_windows iff K_{b,t} = K).  E and the acceptances are those of aal_loss_fwd.
+ *   draft, target  [B][seq_len][V] logits (z_q, z_p), rows contiguous, 16-byte aligned bases.
+ *   mask           [B][seq_len] uint8, nonzero = valid position, or NULL (all valid).
+ *   workspace      at least aal_seq_workspace_size() bytes, 256-byte aligned.
+ *   loss           device float[1].
+ *   eal            device float[B*seq_len][2] or NULL: E^g, E^s of the window starting at each
+ *                  position (0 for a term not computed or a window not in W). */
+AAL_API aal_status aal_seq_loss_fwd(const aal_seq_problem* prob, const void* draft, const void* target,
+                                    const uint8_t* mask, void* workspace, size_t workspace_bytes,
+                                    float* loss, float* eal, void* stream);
+
+/* Backward of the sequence loss: grad_draft [B][seq_len][V] = dloss * dL/dz_q, each position's
+ * row summed over the windows that contain it (in a fixed order, so results are reproducible).
+ * Must follow aal_seq_loss_fwd on the same stream with the same problem, inputs and workspace.
+ * Positions in no window's valid prefix get exact zeros; ties follow aal_loss_bwd. */
+AAL_API aal_status aal_seq_loss_bwd(const aal_seq_problem* prob, const void* draft, const void* target,
+                                    const uint8_t* mask, const void* workspace, size_t workspace_bytes,
+                                    float dloss, void* grad_draft, void* stream);
 
 /* Simulated acceptance reward of the GRPO stage (Sec. 3.4).
  *   N, K, V, dtype       as for the loss; K is the window size gamma (1..AAL_MAX_K).

@@ -1,12 +1,12 @@
 """The forward-KL anchor of the combined objectives, float64 (test infrastructure only).
 
-Sec. 4.1: the greedy-regime draft is trained on L_KL + 0.1 L_EAL, where the anchor L_KL
-is the forward KL divergence between the target and the draft at each token position,
+Sec. 4.1: the greedy-regime draft is trained on L_KL + 0.1 L_EAL.  The anchor L_KL is a
+forward KL from the target to the draft, one per token position:
 KL(p_t || q_t) = sum_v p_t(v) (log p_t(v) - log q_t(v)).  The anchor uses the model
 distributions themselves (T = 1): the temperature of Sec. 4.1 is stated for p~ and q~,
 which only the acceptance terms use.
 
-Readings (the paper gives only "at each token position"):
+Readings (the paper says no more than that the KL is taken per token position):
   * the anchor is the mean of the per-position KL over the valid positions (mask 1),
     independent of any window; with none it is 0;
   * its weight w_kl enters the objective as  L = w_kl L_KL + w_g L_EAL + w_s L_WTV,

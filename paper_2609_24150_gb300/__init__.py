@@ -20,6 +20,7 @@ from .aal import (  # noqa: F401
     AAL_ERR_WORKSPACE,
     AAL_F32,
     AAL_GREEDY,
+    AAL_KL,
     AAL_MAX_K,
     AAL_NOALLOC_MAX_ROWS,
     AAL_OK,
@@ -27,6 +28,7 @@ from .aal import (  # noqa: F401
     AalError,
     AalProblem,
     AalRewardProblem,
+    AalSeqProblem,
     aal_abi_version,
     aal_accept_reward,
     aal_accept_reward_from_loss,
@@ -36,10 +38,14 @@ from .aal import (  # noqa: F401
     aal_loss_bwd,
     aal_loss_fwd,
     aal_reward_workspace_size,
+    aal_seq_loss_bwd,
+    aal_seq_loss_fwd,
+    aal_seq_workspace_size,
     aal_status_string,
     aal_workspace_size,
     library,
     library_path,
     loss_problem,
     reward_problem,
+    seq_problem,
 )

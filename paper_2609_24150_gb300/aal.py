@@ -21,6 +21,7 @@ AAL_BF16 = 1
 AAL_GREEDY = 1
 AAL_SAMPLING = 2
 AAL_BOTH = 3
+AAL_KL = 4          # mode bit: the forward-KL anchor
 
 AAL_MAX_K = 8
 AAL_NOALLOC_MAX_ROWS = 1 << 20   # N * K limit of aal_accept_reward_noalloc
@@ -37,7 +38,7 @@ class AalProblem(ctypes.Structure):
     _fields_ = [("N", ctypes.c_int64), ("K", ctypes.c_int64), ("V", ctypes.c_int64),
                 ("dtype", ctypes.c_int32), ("mode", ctypes.c_int32),
                 ("temperature", ctypes.c_float), ("w_greedy", ctypes.c_float),
-                ("w_sampling", ctypes.c_float), ("reserved", ctypes.c_int32)]
+                ("w_sampling", ctypes.c_float), ("w_kl", ctypes.c_float), ("reserved", ctypes.c_int32)]
 
 
 class AalRewardProblem(ctypes.Structure):
@@ -47,6 +48,15 @@ class AalRewardProblem(ctypes.Structure):
                 ("temperature", ctypes.c_float), ("adv_clip", ctypes.c_float),
                 ("seed", ctypes.c_uint64), ("row_offset", ctypes.c_int64),
                 ("windows_per_rollout", ctypes.c_int64), ("rollouts_per_group", ctypes.c_int64)]
+
+
+class AalSeqProblem(ctypes.Structure):
+    """Mirror of ``aal_seq_problem``."""
+    _fields_ = [("B", ctypes.c_int64), ("seq_len", ctypes.c_int64), ("K", ctypes.c_int64),
+                ("V", ctypes.c_int64), ("dtype", ctypes.c_int32), ("mode", ctypes.c_int32),
+                ("temperature", ctypes.c_float), ("w_greedy", ctypes.c_float),
+                ("w_sampling", ctypes.c_float), ("w_kl", ctypes.c_float),
+                ("full_windows", ctypes.c_int32), ("reserved", ctypes.c_int32)]
 
 
 class AalError(RuntimeError):
@@ -77,6 +87,10 @@ def library() -> ctypes.CDLL:
     lib.aal_accept_reward.argtypes = [RP, vp, vp, vp, vp, sz, vp, vp, vp, vp, vp]
     lib.aal_accept_reward_noalloc.argtypes = [RP, vp, vp, vp, vp, vp, vp, vp, vp]
     lib.aal_accept_reward_from_loss.argtypes = [RP, P, vp, sz, vp, sz, vp, vp, vp, vp]
+    SP = ctypes.POINTER(AalSeqProblem)
+    lib.aal_seq_workspace_size.argtypes = [SP, ctypes.POINTER(sz)]
+    lib.aal_seq_loss_fwd.argtypes = [SP, vp, vp, vp, vp, sz, vp, vp, vp]
+    lib.aal_seq_loss_bwd.argtypes = [SP, vp, vp, vp, vp, sz, ctypes.c_float, vp, vp]
     lib.aal_check_device_status.argtypes = [vp, vp]
     lib.aal_debug_fail_next_forward.argtypes = [ctypes.c_int64, ctypes.c_uint64]
     lib.aal_debug_fail_next_forward.restype = None
@@ -86,7 +100,7 @@ def library() -> ctypes.CDLL:
     lib.aal_abi_version.restype = ctypes.c_int32
     for f in ("aal_workspace_size", "aal_reward_workspace_size", "aal_loss_fwd", "aal_loss_bwd",
               "aal_accept_reward", "aal_accept_reward_noalloc", "aal_accept_reward_from_loss",
-              "aal_check_device_status"):
+              "aal_seq_workspace_size", "aal_seq_loss_fwd", "aal_seq_loss_bwd", "aal_check_device_status"):
         getattr(lib, f).restype = ctypes.c_int
     _LIB = lib
     return lib
@@ -134,14 +148,27 @@ def _check(code: int, where: str):
 
 
 def loss_problem(draft: torch.Tensor, mode: int, temperature: float = 1.0, w_greedy: float = 1.0,
-                 w_sampling: float = 1.0) -> AalProblem:
-    """Problem struct for [N][K][V] logits."""
+                 w_sampling: float = 1.0, w_kl: float = 1.0) -> AalProblem:
+    """Problem struct for [N][K][V] logits (``w_kl`` weighs the AAL_KL anchor)."""
     if draft.dim() != 3:
         raise ValueError("logits must be [N][K][V]")
     N, K, V = draft.shape
     if draft.dtype not in _DTYPES:
         raise ValueError(f"unsupported dtype {draft.dtype}")
-    return AalProblem(N, K, V, _DTYPES[draft.dtype], mode, temperature, w_greedy, w_sampling, 0)
+    return AalProblem(N, K, V, _DTYPES[draft.dtype], mode, temperature, w_greedy, w_sampling, w_kl, 0)
+
+
+def seq_problem(draft: torch.Tensor, K: int, mode: int, temperature: float = 1.0, w_greedy: float = 1.0,
+                w_sampling: float = 1.0, full_windows: bool = False, w_kl: float = 1.0) -> AalSeqProblem:
+    """Problem struct for [B][seq_len][V] logits with sliding windows of K positions
+    (``full_windows``: only windows with all K positions valid belong to W)."""
+    if draft.dim() != 3:
+        raise ValueError("logits must be [B][seq_len][V]")
+    B, S, V = draft.shape
+    if draft.dtype not in _DTYPES:
+        raise ValueError(f"unsupported dtype {draft.dtype}")
+    return AalSeqProblem(B, S, K, V, _DTYPES[draft.dtype], mode, temperature, w_greedy, w_sampling,
+                         w_kl, int(bool(full_windows)), 0)
 
 
 def reward_problem(draft: torch.Tensor, mode: int, temperature: float = 1.0, adv_clip: float = 5.0,
@@ -195,6 +222,33 @@ def aal_loss_bwd(problem: AalProblem, draft, target, mask, workspace, dloss: flo
         _ptr(mask, "mask", torch.uint8), _ptr(workspace, "workspace"), _nbytes(workspace),
         float(dloss), _ptr(grad, "grad"), _stream(stream))
     _check(code, "aal_loss_bwd")
+
+
+def aal_seq_workspace_size(problem: AalSeqProblem) -> int:
+    out = ctypes.c_size_t(0)
+    _check(library().aal_seq_workspace_size(ctypes.byref(problem), ctypes.byref(out)),
+           "aal_seq_workspace_size")
+    return out.value
+
+
+def aal_seq_loss_fwd(problem: AalSeqProblem, draft, target, mask, workspace, loss, eal=None, stream=None):
+    """Forward of the loss over every sliding window of every sequence; writes loss[0] (and
+    eal[B*seq_len][2] when given)."""
+    R = problem.B * problem.seq_len
+    code = library().aal_seq_loss_fwd(
+        ctypes.byref(problem), _ptr(draft, "draft"), _ptr(target, "target"),
+        _ptr(mask, "mask", torch.uint8, R), _ptr(workspace, "workspace"), _nbytes(workspace),
+        _ptr(loss, "loss", torch.float32, 1), _ptr(eal, "eal", torch.float32, 2 * R), _stream(stream))
+    _check(code, "aal_seq_loss_fwd")
+
+
+def aal_seq_loss_bwd(problem: AalSeqProblem, draft, target, mask, workspace, dloss: float, grad, stream=None):
+    """Backward of the sequence loss: grad = dloss * dL/d draft, summed over each position's windows."""
+    code = library().aal_seq_loss_bwd(
+        ctypes.byref(problem), _ptr(draft, "draft"), _ptr(target, "target"),
+        _ptr(mask, "mask", torch.uint8), _ptr(workspace, "workspace"), _nbytes(workspace),
+        float(dloss), _ptr(grad, "grad"), _stream(stream))
+    _check(code, "aal_seq_loss_bwd")
 
 
 def aal_accept_reward(problem: AalRewardProblem, draft, target, ref_draft, workspace, tau,

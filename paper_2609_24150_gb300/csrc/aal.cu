@@ -30,9 +30,9 @@ aal_status check_problem(const aal_problem* p) {
   if (p == nullptr) return AAL_ERR_INVALID_ARG;
   aal_status st = check_shape(p->N, p->K, p->V, p->dtype);
   if (st != AAL_OK) return st;
-  if (p->mode != AAL_GREEDY && p->mode != AAL_SAMPLING && p->mode != AAL_BOTH) return AAL_ERR_INVALID_ARG;
+  if (p->mode < 1 || p->mode > (AAL_BOTH | AAL_KL)) return AAL_ERR_INVALID_ARG;
   if ((p->mode & AAL_SAMPLING) && !(isfinite(p->temperature) && p->temperature > 0.f)) return AAL_ERR_INVALID_ARG;
-  if (!isfinite(p->w_greedy) || !isfinite(p->w_sampling)) return AAL_ERR_INVALID_ARG;
+  if (!isfinite(p->w_greedy) || !isfinite(p->w_sampling) || !isfinite(p->w_kl)) return AAL_ERR_INVALID_ARG;
   if (p->reserved != 0) return AAL_ERR_INVALID_ARG;
   return AAL_OK;
 }
@@ -51,7 +51,66 @@ aal_status check_reward(const aal_reward_problem* p) {
   return AAL_OK;
 }
 
+aal_status check_seq(const aal_seq_problem* p) {
+  if (p == nullptr) return AAL_ERR_INVALID_ARG;
+  if (p->B < 0 || p->seq_len < 0) return AAL_ERR_INVALID_ARG;
+  if (p->full_windows != 0 && p->full_windows != 1) return AAL_ERR_INVALID_ARG;
+  if (p->seq_len > 0 && p->B > INT64_MAX / p->seq_len) return AAL_ERR_INVALID_ARG;
+  // the checks of a windowed problem with one window per position (R * K * V elements bound
+  // the per-depth partials too)
+  const aal_problem q{p->B * p->seq_len, p->K, p->V, p->dtype, p->mode, p->temperature, p->w_greedy,
+                      p->w_sampling, p->w_kl, p->reserved};
+  return check_problem(&q);
+}
+
 aal_status cuda_status(cudaError_t e) { return e == cudaSuccess ? AAL_OK : AAL_ERR_CUDA; }
+
+// Per-row statistics of R logit rows (pass over z_p and z_q), shared by both layouts.
+cudaError_t launch_stats(const void* draft, const void* target, int64_t R, int64_t V, int32_t dtype,
+                         int32_t mode, float temperature, const LossWs& ws, cudaStream_t s, int* cluster) {
+  const bool greedy = (mode & AAL_GREEDY) != 0, sampling = (mode & AAL_SAMPLING) != 0;
+  const bool kl = (mode & AAL_KL) != 0;
+  RowStatsArgs ra;
+  ra.zq = draft;
+  ra.zp = target;
+  ra.R = R;
+  ra.V = V;
+  ra.sT = sampling ? kLog2e / temperature : 0.f;
+  ra.need_p = sampling;
+  ra.need_q = sampling;
+  ra.need_q1 = (greedy || kl) && !(sampling && temperature == 1.0f);
+  ra.overlap = sampling;
+  ra.need_kl = kl;
+  ra.skip_chunk = debug_take_skip_chunk();
+  ra.ws = ws;
+  *cluster = 1;
+  return launch_rowstats(ra, dtype == AAL_BF16, s, cluster);
+}
+
+// Gradient rows from the statistics and dE/da in the workspace, shared by both layouts.
+cudaError_t launch_grad(const void* draft, const void* target, const uint8_t* mask, int64_t R, int64_t V,
+                        int32_t dtype, int32_t mode, float temperature, float w_greedy, float w_sampling,
+                        float w_kl, float dloss, const LossWs& ws, void* grad, cudaStream_t s) {
+  const bool greedy = (mode & AAL_GREEDY) != 0, sampling = (mode & AAL_SAMPLING) != 0;
+  const bool kl = (mode & AAL_KL) != 0;
+  BackwardArgs ba;
+  ba.zq = draft;
+  ba.zp = target;
+  ba.grad = grad;
+  ba.R = R;
+  ba.V = V;
+  ba.K = 1;
+  ba.sT = sampling ? kLog2e / temperature : 0.f;
+  ba.invT = sampling ? 1.0f / temperature : 0.f;
+  ba.dloss = dloss;
+  ba.w_greedy = greedy ? w_greedy : 0.f;
+  ba.w_sampling = sampling ? w_sampling : 0.f;
+  ba.w_kl = kl ? w_kl : 0.f;
+  ba.mask = mask;
+  ba.q1_is_qT = (greedy || kl) && sampling && temperature == 1.0f;
+  ba.ws = ws;
+  return launch_backward(ba, dtype == AAL_BF16, s);
+}
 
 }  // namespace
 
@@ -62,7 +121,7 @@ int64_t debug_take_skip_chunk() { return g_skip_chunk.exchange(-1); }
 
 extern "C" {
 
-int32_t aal_abi_version(void) { return 10000; }
+int32_t aal_abi_version(void) { return 10100; }
 
 void aal_debug_fail_next_forward(int64_t chunk, uint64_t wait_limit_ns) {
   g_wait_limit_ns.store(wait_limit_ns);
@@ -111,25 +170,11 @@ aal_status aal_loss_fwd(const aal_problem* prob, const void* draft, const void* 
   if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < L.total) return AAL_ERR_WORKSPACE;
 
   const bool greedy = (prob->mode & AAL_GREEDY) != 0, sampling = (prob->mode & AAL_SAMPLING) != 0;
-  const bool bf16 = prob->dtype == AAL_BF16;
   LossWs ws = loss_ws(workspace, L);
   cudaError_t e = cudaMemsetAsync(ws.hdr, 0, sizeof(WsHeader), s);
   if (e != cudaSuccess) return AAL_ERR_CUDA;
-
-  RowStatsArgs ra;
-  ra.zq = draft;
-  ra.zp = target;
-  ra.R = L.R;
-  ra.V = prob->V;
-  ra.sT = sampling ? kLog2e / prob->temperature : 0.f;
-  ra.need_p = sampling;
-  ra.need_q = sampling;
-  ra.need_q1 = greedy && !(sampling && prob->temperature == 1.0f);
-  ra.overlap = sampling;
-  ra.skip_chunk = debug_take_skip_chunk();
-  ra.ws = ws;
   int cluster = 1;
-  e = launch_rowstats(ra, bf16, s, &cluster);
+  e = launch_stats(draft, target, L.R, prob->V, prob->dtype, prob->mode, prob->temperature, ws, s, &cluster);
   if (e != cudaSuccess) return AAL_ERR_CUDA;
 
   WindowArgs wa;
@@ -139,8 +184,10 @@ aal_status aal_loss_fwd(const aal_problem* prob, const void* draft, const void* 
   wa.cluster = cluster;
   wa.greedy = greedy;
   wa.sampling = sampling;
+  wa.kl = (prob->mode & AAL_KL) != 0;
   wa.w_greedy = prob->w_greedy;
   wa.w_sampling = prob->w_sampling;
+  wa.w_kl = prob->w_kl;
   wa.loss = loss;
   wa.eal = eal;
   wa.ws = ws;
@@ -151,7 +198,8 @@ aal_status aal_loss_fwd(const aal_problem* prob, const void* draft, const void* 
 aal_status aal_loss_bwd(const aal_problem* prob, const void* draft, const void* target,
                         const uint8_t* mask, const void* workspace, size_t workspace_bytes, float dloss,
                         void* grad_draft, void* stream) {
-  (void)mask;  // the forward folded the mask into dE/da (zero outside each window's valid prefix)
+  // the forward folded the mask into dE/da (zero outside each window's valid prefix); the
+  // anchor's rows are the valid positions themselves
   aal_status st = check_problem(prob);
   if (st != AAL_OK) return st;
   if (!isfinite(dloss)) return AAL_ERR_INVALID_ARG;
@@ -161,23 +209,82 @@ aal_status aal_loss_bwd(const aal_problem* prob, const void* draft, const void* 
     return AAL_ERR_INVALID_ARG;
   const LossLayout L = loss_layout(prob->N, prob->K);
   if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < L.total) return AAL_ERR_WORKSPACE;
-  const bool greedy = (prob->mode & AAL_GREEDY) != 0, sampling = (prob->mode & AAL_SAMPLING) != 0;
+  return cuda_status(launch_grad(draft, target, mask, L.R, prob->V, prob->dtype, prob->mode,
+                                 prob->temperature, prob->w_greedy, prob->w_sampling, prob->w_kl, dloss,
+                                 loss_ws(const_cast<void*>(workspace), L), grad_draft,
+                                 static_cast<cudaStream_t>(stream)));
+}
 
-  BackwardArgs ba;
-  ba.zq = draft;
-  ba.zp = target;
-  ba.grad = grad_draft;
-  ba.R = L.R;
-  ba.V = prob->V;
-  ba.K = (int32_t)prob->K;
-  ba.sT = sampling ? kLog2e / prob->temperature : 0.f;
-  ba.invT = sampling ? 1.0f / prob->temperature : 0.f;
-  ba.dloss = dloss;
-  ba.w_greedy = greedy ? prob->w_greedy : 0.f;
-  ba.w_sampling = sampling ? prob->w_sampling : 0.f;
-  ba.q1_is_qT = greedy && sampling && prob->temperature == 1.0f;
-  ba.ws = loss_ws(const_cast<void*>(workspace), L);
-  return cuda_status(launch_backward(ba, prob->dtype == AAL_BF16, static_cast<cudaStream_t>(stream)));
+aal_status aal_seq_workspace_size(const aal_seq_problem* prob, size_t* bytes) {
+  aal_status st = check_seq(prob);
+  if (st != AAL_OK) return st;
+  if (bytes == nullptr) return AAL_ERR_INVALID_ARG;
+  *bytes = seq_layout(prob->B, prob->seq_len, prob->K).total;
+  return AAL_OK;
+}
+
+aal_status aal_seq_loss_fwd(const aal_seq_problem* prob, const void* draft, const void* target,
+                            const uint8_t* mask, void* workspace, size_t workspace_bytes, float* loss,
+                            float* eal, void* stream) {
+  aal_status st = check_seq(prob);
+  if (st != AAL_OK) return st;
+  if (loss == nullptr || !aligned(loss, 4) || (eal != nullptr && !aligned(eal, 4))) return AAL_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int64_t R = prob->B * prob->seq_len;
+  if (R == 0) return cuda_status(cudaMemsetAsync(loss, 0, sizeof(float), s));
+  if (draft == nullptr || target == nullptr || !aligned(draft, 16) || !aligned(target, 16))
+    return AAL_ERR_INVALID_ARG;
+  const SeqLayout L = seq_layout(prob->B, prob->seq_len, prob->K);
+  if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < L.total) return AAL_ERR_WORKSPACE;
+
+  LossWs ws = loss_ws(workspace, L.base);
+  cudaError_t e = cudaMemsetAsync(ws.hdr, 0, sizeof(WsHeader), s);
+  if (e != cudaSuccess) return AAL_ERR_CUDA;
+  int cluster = 1;
+  e = launch_stats(draft, target, R, prob->V, prob->dtype, prob->mode, prob->temperature, ws, s, &cluster);
+  if (e != cudaSuccess) return AAL_ERR_CUDA;
+
+  char* base = static_cast<char*>(workspace);
+  SeqWindowArgs wa;
+  wa.mask = mask;
+  wa.B = prob->B;
+  wa.T = prob->seq_len;
+  wa.K = (int32_t)prob->K;
+  wa.full_windows = prob->full_windows != 0;
+  wa.cluster = cluster;
+  wa.greedy = (prob->mode & AAL_GREEDY) != 0;
+  wa.sampling = (prob->mode & AAL_SAMPLING) != 0;
+  wa.kl = (prob->mode & AAL_KL) != 0;
+  wa.w_greedy = prob->w_greedy;
+  wa.w_sampling = prob->w_sampling;
+  wa.w_kl = prob->w_kl;
+  wa.loss = loss;
+  wa.eal = eal;
+  wa.pg = reinterpret_cast<float*>(base + L.pg);
+  wa.ps = reinterpret_cast<float*>(base + L.ps);
+  wa.ws = ws;
+  wa.nwblk = L.base.nwblk;
+  return cuda_status(launch_seq_window(wa, s));
+}
+
+aal_status aal_seq_loss_bwd(const aal_seq_problem* prob, const void* draft, const void* target,
+                            const uint8_t* mask, const void* workspace, size_t workspace_bytes, float dloss,
+                            void* grad_draft, void* stream) {
+  // dE/da carries the windows' masks; the anchor's rows are the valid positions
+  aal_status st = check_seq(prob);
+  if (st != AAL_OK) return st;
+  if (!isfinite(dloss)) return AAL_ERR_INVALID_ARG;
+  const int64_t R = prob->B * prob->seq_len;
+  if (R == 0) return AAL_OK;
+  if (draft == nullptr || target == nullptr || grad_draft == nullptr || !aligned(draft, 16) ||
+      !aligned(target, 16) || !aligned(grad_draft, 16))
+    return AAL_ERR_INVALID_ARG;
+  const SeqLayout L = seq_layout(prob->B, prob->seq_len, prob->K);
+  if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < L.total) return AAL_ERR_WORKSPACE;
+  return cuda_status(launch_grad(draft, target, mask, R, prob->V, prob->dtype, prob->mode,
+                                 prob->temperature, prob->w_greedy, prob->w_sampling, prob->w_kl, dloss,
+                                 loss_ws(const_cast<void*>(workspace), L.base), grad_draft,
+                                 static_cast<cudaStream_t>(stream)));
 }
 
 aal_status aal_accept_reward(const aal_reward_problem* prob, const void* draft, const void* target,

@@ -11,6 +11,7 @@
 namespace aal {
 
 constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
 constexpr int kMaxCluster = 8;          // CTAs that may share one logit row
 constexpr uint32_t kStatusTimeout = 5;  // == AAL_ERR_TIMEOUT
 
@@ -24,7 +25,8 @@ struct WsHeader {
   int32_t nvalid;         // |W|, written by the forward
   int32_t cluster;        // CTAs per row used by the row-statistics kernel
   float loss;             // copy of the loss
-  float pad[59];
+  int32_t npos;           // valid positions (rows), the normaliser of the KL anchor
+  float pad[58];
 };
 static_assert(sizeof(WsHeader) == 256, "header is 256 bytes");
 
@@ -35,19 +37,22 @@ struct LossLayout {
   // maximum M = max_v z_v and Ls = log2 sum_v 2^((z_v - M) s) with s = log2(e)/T, so that
   // log2 p~_v = (z_v - M) s - Ls; the maximum's own term is exactly 2^0 = 1.
   size_t Mp = 0, Lsp = 0, Mq = 0, Lsq = 0, Mq1 = 0, Lsq1 = 0;
+  size_t Mp1 = 0, Lsp1 = 0;         // float[R] the normaliser of z_p at T = 1 (KL anchor)
+  size_t kl = 0;                    // float[R] KL(p || q) at T = 1 (KL anchor)
   size_t ag = 0, as = 0, qlt = 0;   // float[R] a^greedy, a^sample, sum_{lq<lp} q~
   size_t dEg = 0, dEs = 0;          // float[R] dE_n / da_{n,j}
   size_t xstar = 0;                 // int32[R] target argmax
   size_t yhat = 0;                  // int32[R] draft argmax (the greedy draft token)
   size_t zpy = 0;                   // float[R] z_p at the draft argmax
   size_t cpart = 0;                 // float2[R][kMaxCluster] per-CTA (overlap, Qlt) partials
-  size_t wpart = 0;                 // double[nwblk][4] window-kernel block partials
+  size_t wpart = 0;                 // double[nwblk][kWpart] window-kernel block partials
   size_t total = 0;
 };
 
 __host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 constexpr int kWindowThreads = 256;
+constexpr int kWpart = 8;  // block partials: sum E^g, sum E^s, |W|, sum KL, |positions|
 
 inline LossLayout loss_layout(int64_t N, int64_t K) {
   LossLayout L;
@@ -68,6 +73,9 @@ inline LossLayout loss_layout(int64_t N, int64_t K) {
   L.Lsq = take(R * 4);
   L.Mq1 = take(R * 4);
   L.Lsq1 = take(R * 4);
+  L.Mp1 = take(R * 4);
+  L.Lsp1 = take(R * 4);
+  L.kl = take(R * 4);
   L.ag = take(R * 4);
   L.as = take(R * 4);
   L.qlt = take(R * 4);
@@ -77,7 +85,31 @@ inline LossLayout loss_layout(int64_t N, int64_t K) {
   L.yhat = take(R * 4);
   L.zpy = take(R * 4);
   L.cpart = take(R * kMaxCluster * 8);
-  L.wpart = take((size_t)(L.nwblk > 0 ? L.nwblk : 1) * 4 * 8);
+  L.wpart = take((size_t)(L.nwblk > 0 ? L.nwblk : 1) * kWpart * 8);
+  L.total = off;
+  return L;
+}
+
+// Sequence layout: rows are positions (R = N = B*T, one window per start position) plus the
+// per-window, per-depth partials dE_t/da_{t+j}, which a gather sums into each position's dE/da.
+struct SeqLayout {
+  LossLayout base;
+  size_t pg = 0, ps = 0;  // float[B*T][K] each (greedy, sampling)
+  size_t total = 0;
+};
+
+inline SeqLayout seq_layout(int64_t B, int64_t T, int64_t K) {
+  SeqLayout L;
+  L.base = loss_layout(B * T, 1);
+  size_t off = L.base.total;
+  auto take = [&](size_t bytes) {
+    size_t o = off;
+    off = align_up(off + bytes, 256);
+    return o;
+  };
+  const size_t nk = (size_t)(B * T * K);
+  L.pg = take(nk * 4);
+  L.ps = take(nk * 4);
   L.total = off;
   return L;
 }
@@ -107,7 +139,7 @@ inline RewardLayout reward_layout(int64_t N, int64_t K) {
 // Pointers into a loss workspace.
 struct LossWs {
   WsHeader* hdr;
-  float *Mp, *Lsp, *Mq, *Lsq, *Mq1, *Lsq1, *ag, *as, *qlt, *dEg, *dEs;
+  float *Mp, *Lsp, *Mq, *Lsq, *Mq1, *Lsq1, *Mp1, *Lsp1, *kl, *ag, *as, *qlt, *dEg, *dEs;
   int32_t* xstar;
   int32_t* yhat;
   float* zpy;
@@ -125,6 +157,9 @@ inline LossWs loss_ws(void* base, const LossLayout& L) {
   w.Lsq = reinterpret_cast<float*>(b + L.Lsq);
   w.Mq1 = reinterpret_cast<float*>(b + L.Mq1);
   w.Lsq1 = reinterpret_cast<float*>(b + L.Lsq1);
+  w.Mp1 = reinterpret_cast<float*>(b + L.Mp1);
+  w.Lsp1 = reinterpret_cast<float*>(b + L.Lsp1);
+  w.kl = reinterpret_cast<float*>(b + L.kl);
   w.ag = reinterpret_cast<float*>(b + L.ag);
   w.as = reinterpret_cast<float*>(b + L.as);
   w.qlt = reinterpret_cast<float*>(b + L.qlt);
@@ -150,6 +185,7 @@ struct RowStatsArgs {
   bool need_q;          // log-sum-exp of z_q / T   (sampling term)
   bool need_q1;         // log-sum-exp of z_q       (greedy term, when T != 1 or no sampling)
   bool overlap;         // second phase: sum min(p~, q~) and Qlt (sampling term)
+  bool need_kl;         // KL(p || q) at T = 1 and the normaliser of z_p at T = 1 (anchor)
   int64_t skip_chunk;   // failure-detection test hook: a chunk whose copy is never armed (-1: none)
   LossWs ws;
 };
@@ -159,10 +195,26 @@ struct WindowArgs {
   int64_t N;
   int32_t K;
   int32_t cluster;      // partials per row in ws.cpart
-  bool greedy, sampling;
-  float w_greedy, w_sampling;
+  bool greedy, sampling, kl;
+  float w_greedy, w_sampling, w_kl;
   float* loss;          // device float[1]
   float* eal;           // device float[N][2] or null
+  LossWs ws;
+  int64_t nwblk;
+};
+
+struct SeqWindowArgs {
+  const uint8_t* mask;  // [B][T] or null
+  int64_t B, T;
+  int32_t K;
+  int32_t cluster;
+  bool greedy, sampling, kl;
+  bool full_windows;    // W = windows with all K positions valid
+  float w_greedy, w_sampling, w_kl;
+  float* loss;
+  float* eal;           // [B*T][2] or null
+  float* pg;            // [B*T][K]
+  float* ps;
   LossWs ws;
   int64_t nwblk;
 };
@@ -176,7 +228,9 @@ struct BackwardArgs {
   float sT, invT;
   float dloss;
   float w_greedy, w_sampling;  // 0 for a term the mode does not select
-  bool q1_is_qT;               // T == 1 with both terms: q = q~, one exponential per element
+  float w_kl;                  // 0 without the KL anchor
+  const uint8_t* mask;         // [R] position validity (the anchor's rows), or null
+  bool q1_is_qT;               // T == 1, sampling and a T = 1 term: q = q~, one exponential
   LossWs ws;
 };
 
@@ -230,6 +284,7 @@ constexpr uint64_t kWaitLimitNs = 1000000000ull;  // bounded waits give up after
 uint64_t debug_wait_limit_ns();
 int64_t debug_take_skip_chunk();
 cudaError_t launch_window(const WindowArgs& a, cudaStream_t s);
+cudaError_t launch_seq_window(const SeqWindowArgs& a, cudaStream_t s);
 cudaError_t launch_backward(const BackwardArgs& a, bool bf16, cudaStream_t s);
 cudaError_t launch_reward_rows(const RewardRowArgs& a, bool bf16, cudaStream_t s);
 cudaError_t launch_reward_groups(const RewardGroupArgs& a, cudaStream_t s);
@@ -316,6 +371,45 @@ __device__ __forceinline__ float bf16hi_add(uint32_t w, float c) {
       : "=f"(d)
       : "r"(w), "f"(c));
   return d;
+}
+
+// Online forward KL of one row at T = 1 (the anchor): with e_v = exp(z_p,v - M) and M the
+// running maximum of z_p, S = sum e_v and D = sum e_v (z_p,v - z_q,v), both rescaled when M
+// moves.  Then p_v = e_v / S and KL(p || q) = D / S - (M - M_q) - ln S + ln S_q.  A target
+// logit of -inf adds nothing (0 log 0 = 0).
+struct KlAcc {
+  float M, S, D;
+};
+__device__ __forceinline__ void kl_init(KlAcc& a) {
+  a.M = -INFINITY;
+  a.S = 0.f;
+  a.D = 0.f;
+}
+__device__ __forceinline__ void kl_push(KlAcc& a, float p, float q) {
+  if (p > a.M) {
+    const float r = ex2((a.M - p) * kLog2e);  // M == -inf: r = 0, and S, D were 0
+    a.S = fmaf(a.S, r, 1.f);
+    a.D = fmaf(a.D, r, p - q);
+    a.M = p;
+  } else if (p != -INFINITY) {
+    const float e = ex2((p - a.M) * kLog2e);
+    a.S += e;
+    a.D = fmaf(e, p - q, a.D);
+  }
+}
+__device__ __forceinline__ KlAcc kl_merge(KlAcc a, KlAcc b) {
+  KlAcc r;
+  r.M = fmaxf(a.M, b.M);
+  if (r.M == -INFINITY) {
+    r.S = 0.f;
+    r.D = 0.f;
+    return r;
+  }
+  const float sa = (a.M == -INFINITY) ? 0.f : ex2((a.M - r.M) * kLog2e);
+  const float sb = (b.M == -INFINITY) ? 0.f : ex2((b.M - r.M) * kLog2e);
+  r.S = a.S * sa + b.S * sb;
+  r.D = a.D * sa + b.D * sb;
+  return r;
 }
 
 // Argmax with the lowest index on ties, carrying one extra value.

@@ -4,10 +4,12 @@
 // g^s = -(dloss/|W|) w_s dE^s_n/da^s_{n,j} (dE/da from the window kernel):
 //   dz_u = g^g a^g (delta_{u,x*} - q(u))                 greedy term, Eq. acc_greedy
 //        + g^s (1/T) q~(u) (c_u - Qlt),  c_u = [q~_u < p~_u]   sampling term, Eq. acc_sample
+//        + c^kl (q(u) - p(u))                                  KL anchor (Sec. 4.1), T = 1
 // (the softmax Jacobian applied to d a / d q; at a tie q~_u = p~_u the min follows the
 // frozen p~, so c_u = 0).  q(u), q~(u) and c_u are recomputed from the logits and the
 // row's saved log-sum-exps; nothing of size V is materialised.  One pass: reads z_q
-// (and z_p when the sampling term is on), writes dz in the logits' dtype.
+// (and z_p when the sampling term or the anchor is on), writes dz in the logits' dtype.
+// c^kl = dloss w_kl / |positions| on valid positions, 0 elsewhere.
 #include "aal_internal.cuh"
 
 namespace aal {
@@ -69,13 +71,14 @@ __device__ __forceinline__ void st_stream(uint4* p, const uint4& v) {
 }
 
 struct RowCoef {
-  float sT, Mq, Lsq, Mp, Lsp, Mq1, Lsq1;
+  float sT, Mq, Lsq, Mp, Lsp, Mq1, Lsq1, Mp1, Lsp1;
+  float Ck;          // c^kl
   float cpos, cneg;  // g^s/T (1 - Qlt) and -g^s/T Qlt
   float Ag;          // g^g a^g
   int32_t xs;
 };
 
-template <bool GREEDY, bool SAMPLING, bool Q1_IS_QT>
+template <bool GREEDY, bool SAMPLING, bool Q1_IS_QT, bool KL>
 __device__ __forceinline__ float grad_elem(const RowCoef& c, float q, float p, int64_t u) {
   float d = 0.f, qt = 0.f;
   if (SAMPLING) {
@@ -84,26 +87,33 @@ __device__ __forceinline__ float grad_elem(const RowCoef& c, float q, float p, i
     qt = ex2(lq);
     d = qt * (lq < lp ? c.cpos : c.cneg);
   }
-  if (GREEDY) {
+  if (GREEDY || KL) {
     const float q1 = Q1_IS_QT ? qt : ex2(log2_prob(q, kLog2e, c.Mq1, c.Lsq1));
-    d = fmaf(-c.Ag, q1, d);
-    if (u == c.xs) d += c.Ag;
+    if (GREEDY) {
+      d = fmaf(-c.Ag, q1, d);
+      if (u == c.xs) d += c.Ag;
+    }
+    if (KL) d = fmaf(c.Ck, q1 - ex2(log2_prob(p, kLog2e, c.Mp1, c.Lsp1)), d);
   }
   return d;
 }
 
-template <typename T, bool VEC, bool GREEDY, bool SAMPLING, bool Q1_IS_QT>
+template <typename T, bool VEC, bool GREEDY, bool SAMPLING, bool Q1_IS_QT, bool KL>
 __global__ void __launch_bounds__(kBwdThreads) backward_kernel(BackwardArgs a) {
   const int nvalid = a.ws.hdr->nvalid;
   const float scale = nvalid > 0 ? -a.dloss / (float)nvalid : 0.f;
+  const int npos = KL ? a.ws.hdr->npos : 0;
+  const float kscale = npos > 0 ? a.dloss * a.w_kl / (float)npos : 0.f;
+  constexpr bool READ_P = SAMPLING || KL;
   constexpr int E = Io<T>::E;
   for (int64_t r = blockIdx.x; r < a.R; r += gridDim.x) {
     const float gg = GREEDY ? scale * a.w_greedy * a.ws.dEg[r] : 0.f;
     const float gs = SAMPLING ? scale * a.w_sampling * a.ws.dEs[r] : 0.f;
+    const float ck = (KL && (a.mask == nullptr || a.mask[r] != 0)) ? kscale : 0.f;
     T* out = static_cast<T*>(a.grad) + r * a.V;
     const T* zq = static_cast<const T*>(a.zq) + r * a.V;
     const T* zp = static_cast<const T*>(a.zp) + r * a.V;
-    if (gg == 0.f && gs == 0.f) {
+    if (gg == 0.f && gs == 0.f && ck == 0.f) {
       if (VEC) {
         uint4* o4 = reinterpret_cast<uint4*>(out);
         for (int64_t i = threadIdx.x; i < a.V / E; i += kBwdThreads) st_stream(o4 + i, make_uint4(0, 0, 0, 0));
@@ -118,8 +128,11 @@ __global__ void __launch_bounds__(kBwdThreads) backward_kernel(BackwardArgs a) {
     c.Lsq = SAMPLING ? a.ws.Lsq[r] : 0.f;
     c.Mp = SAMPLING ? a.ws.Mp[r] : 0.f;
     c.Lsp = SAMPLING ? a.ws.Lsp[r] : 0.f;
-    c.Mq1 = GREEDY ? a.ws.Mq1[r] : 0.f;
-    c.Lsq1 = GREEDY ? a.ws.Lsq1[r] : 0.f;
+    c.Mq1 = (GREEDY || KL) ? a.ws.Mq1[r] : 0.f;
+    c.Lsq1 = (GREEDY || KL) ? a.ws.Lsq1[r] : 0.f;
+    c.Mp1 = KL ? a.ws.Mp1[r] : 0.f;
+    c.Lsp1 = KL ? a.ws.Lsp1[r] : 0.f;
+    c.Ck = ck;
     const float qlt = SAMPLING ? a.ws.qlt[r] : 0.f;
     const float Bs = gs * a.invT;
     c.cpos = Bs * (1.f - qlt);
@@ -134,43 +147,49 @@ __global__ void __launch_bounds__(kBwdThreads) backward_kernel(BackwardArgs a) {
       for (int64_t i = threadIdx.x; i < nv; i += kBwdThreads) {
         float qv[E], pv[E], d[E];
         Io<T>::unpack(ldg_stream(q4 + i), qv);
-        if (SAMPLING) Io<T>::unpack(ldg_stream(p4 + i), pv);
+        if (READ_P) Io<T>::unpack(ldg_stream(p4 + i), pv);
 #pragma unroll
         for (int e = 0; e < E; ++e)
-          d[e] = grad_elem<GREEDY, SAMPLING, Q1_IS_QT>(c, qv[e], SAMPLING ? pv[e] : 0.f, i * E + e);
+          d[e] = grad_elem<GREEDY, SAMPLING, Q1_IS_QT, KL>(c, qv[e], READ_P ? pv[e] : 0.f, i * E + e);
         st_stream(o4 + i, Io<T>::pack(d));
       }
     } else {
       for (int64_t v = threadIdx.x; v < a.V; v += kBwdThreads) {
         const float q = load_elem<T>(zq + v);
-        const float p = SAMPLING ? load_elem<T>(zp + v) : 0.f;
-        Io<T>::store1(out + v, grad_elem<GREEDY, SAMPLING, Q1_IS_QT>(c, q, p, v));
+        const float p = READ_P ? load_elem<T>(zp + v) : 0.f;
+        Io<T>::store1(out + v, grad_elem<GREEDY, SAMPLING, Q1_IS_QT, KL>(c, q, p, v));
       }
     }
   }
 }
 
-template <typename T, bool VEC, bool G, bool S, bool Q>
+template <typename T, bool VEC, bool G, bool S, bool Q, bool KL>
 cudaError_t go(const BackwardArgs& a, cudaStream_t s) {
   int dev = 0, sms = 0, per_sm = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, backward_kernel<T, VEC, G, S, Q>, kBwdThreads, 0);
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, backward_kernel<T, VEC, G, S, Q, KL>, kBwdThreads, 0);
   if (per_sm < 1) per_sm = 1;
   int64_t grid = (int64_t)sms * per_sm;
   if (grid > a.R) grid = a.R;
   if (grid < 1) return cudaSuccess;
-  backward_kernel<T, VEC, G, S, Q><<<(unsigned)grid, kBwdThreads, 0, s>>>(a);
+  backward_kernel<T, VEC, G, S, Q, KL><<<(unsigned)grid, kBwdThreads, 0, s>>>(a);
   return cudaGetLastError();
 }
 
-template <typename T, bool VEC>
+template <typename T, bool VEC, bool KL>
 cudaError_t dispatch_mode(const BackwardArgs& a, cudaStream_t s) {
   const bool G = a.w_greedy != 0.f, S = a.w_sampling != 0.f;
-  if (G && S) return a.q1_is_qT ? go<T, VEC, true, true, true>(a, s) : go<T, VEC, true, true, false>(a, s);
-  if (G) return go<T, VEC, true, false, false>(a, s);
-  if (S) return go<T, VEC, false, true, false>(a, s);
-  return go<T, VEC, false, false, false>(a, s);
+  const bool Q = a.q1_is_qT && S && (G || KL);
+  if (G && S) return Q ? go<T, VEC, true, true, true, KL>(a, s) : go<T, VEC, true, true, false, KL>(a, s);
+  if (G) return go<T, VEC, true, false, false, KL>(a, s);
+  if (S) {
+    if constexpr (KL) {
+      if (Q) return go<T, VEC, false, true, true, KL>(a, s);
+    }
+    return go<T, VEC, false, true, false, KL>(a, s);
+  }
+  return go<T, VEC, false, false, false, KL>(a, s);
 }
 
 template <typename T>
@@ -178,7 +197,8 @@ cudaError_t dispatch(const BackwardArgs& a, cudaStream_t s) {
   const bool vec = ((a.V * (int64_t)sizeof(T)) % 16 == 0) &&
                    ((reinterpret_cast<uintptr_t>(a.zq) | reinterpret_cast<uintptr_t>(a.zp) |
                      reinterpret_cast<uintptr_t>(a.grad)) % 16 == 0);
-  return vec ? dispatch_mode<T, true>(a, s) : dispatch_mode<T, false>(a, s);
+  if (a.w_kl != 0.f) return vec ? dispatch_mode<T, true, true>(a, s) : dispatch_mode<T, false, true>(a, s);
+  return vec ? dispatch_mode<T, true, false>(a, s) : dispatch_mode<T, false, false>(a, s);
 }
 
 }  // namespace

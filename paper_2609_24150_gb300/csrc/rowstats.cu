@@ -7,7 +7,9 @@
 //            M = max_v z_v, Ls = log2 sum_v 2^((z_v - M) s),
 //   x*       argmax_v z_p (lowest index on ties) and a^greedy = q(x*) (Eq. acc_greedy),
 //   a^sample = sum_v min(p~_v, q~_v)   (Eq. acc_sample),
-//   Qlt      = sum_{v: q~_v < p~_v} q~_v, which the backward of a^sample needs.
+//   Qlt      = sum_{v: q~_v < p~_v} q~_v, which the backward of a^sample needs,
+//   KL(p || q) at T = 1 and the normaliser of z_p at T = 1, for the forward-KL anchor of
+//            the combined objectives (Sec. 4.1), in the same pass as the normalisers.
 // a^sample needs both normalisers before it can be summed, so it is a second phase
 // over the row.  This file holds the generic kernel: one CTA per row, both
 // phases streamed from global memory (the second mostly from L2), any V and any
@@ -48,6 +50,7 @@ __device__ __forceinline__ void unpack<uint16_t>(const uint4& w, float* out) {
 
 struct Phase1 {
   Lse p, q, q1;
+  KlAcc kl;
   Amax am;  // target argmax, carrying z_q there
   Amax aq;  // draft argmax, carrying z_p there
 };
@@ -57,6 +60,7 @@ __device__ __forceinline__ Phase1 merge1(const Phase1& a, const Phase1& b, float
   r.p = lse_merge(a.p, b.p, sT);
   r.q = lse_merge(a.q, b.q, sT);
   r.q1 = lse_merge(a.q1, b.q1, kLog2e);
+  r.kl = kl_merge(a.kl, b.kl);
   r.am = amax_merge(a.am, b.am);
   r.aq = amax_merge(a.aq, b.aq);
   return r;
@@ -67,6 +71,9 @@ __device__ __forceinline__ Phase1 shfl1(const Phase1& a, int off) {
   b.p = shfl_lse(a.p, off);
   b.q = shfl_lse(a.q, off);
   b.q1 = shfl_lse(a.q1, off);
+  b.kl.M = __shfl_xor_sync(0xffffffffu, a.kl.M, off);
+  b.kl.S = __shfl_xor_sync(0xffffffffu, a.kl.S, off);
+  b.kl.D = __shfl_xor_sync(0xffffffffu, a.kl.D, off);
   b.am = shfl_amax(a.am, off);
   b.aq = shfl_amax(a.aq, off);
   return b;
@@ -87,6 +94,7 @@ __global__ void __launch_bounds__(kGenericThreads) rowstats_generic(RowStatsArgs
     lse_init(acc.p);
     lse_init(acc.q);
     lse_init(acc.q1);
+    kl_init(acc.kl);
     amax_init(acc.am);
     amax_init(acc.aq);
     auto visit = [&](int64_t v, float p, float q) {
@@ -103,6 +111,7 @@ __global__ void __launch_bounds__(kGenericThreads) rowstats_generic(RowStatsArgs
       if (a.need_p) lse_push(acc.p, p, a.sT);
       if (a.need_q) lse_push(acc.q, q, a.sT);
       if (a.need_q1) lse_push(acc.q1, q, kLog2e);
+      if (a.need_kl) kl_push(acc.kl, p, q);
     };
     constexpr int E = Vec<T>::E;
     if (VEC) {
@@ -134,6 +143,7 @@ __global__ void __launch_bounds__(kGenericThreads) rowstats_generic(RowStatsArgs
         lse_init(x.p);
         lse_init(x.q);
         lse_init(x.q1);
+        kl_init(x.kl);
         amax_init(x.am);
         amax_init(x.aq);
       }
@@ -195,6 +205,12 @@ __global__ void __launch_bounds__(kGenericThreads) rowstats_generic(RowStatsArgs
       a.ws.Lsq[r] = Lsq;
       a.ws.Mq1[r] = Mq1;
       a.ws.Lsq1[r] = Lsq1;
+      if (a.need_kl) {
+        const float Lsp1 = log2f(tot.kl.S);
+        a.ws.Mp1[r] = tot.kl.M;
+        a.ws.Lsp1[r] = Lsp1;
+        a.ws.kl[r] = tot.kl.D / tot.kl.S - (tot.kl.M - Mq1) - kLn2 * (Lsp1 - Lsq1);
+      }
       a.ws.xstar[r] = tot.am.i;
       a.ws.yhat[r] = tot.aq.i;
       a.ws.zpy[r] = tot.aq.carry;
@@ -230,13 +246,13 @@ cudaError_t launch_generic(const RowStatsArgs& a, cudaStream_t s) {
 }  // namespace
 
 // The TMA-streamed kernel (rowstats_stream.cu) serves rows whose byte length is a
-// multiple of 16 when the sampling term needs the second pass; everything else takes the
-// generic kernel.
+// multiple of 16 when the sampling term needs the second pass and the KL anchor is off;
+// everything else takes the generic kernel.
 cudaError_t launch_rowstats(const RowStatsArgs& a, bool bf16, cudaStream_t s, int* cluster_used) {
   const int elt = bf16 ? 2 : 4;
   const bool aligned = ((a.V * elt) % 16 == 0) &&
                        ((reinterpret_cast<uintptr_t>(a.zq) | reinterpret_cast<uintptr_t>(a.zp)) % 16 == 0);
-  if (a.overlap && aligned) {
+  if (a.overlap && aligned && !a.need_kl) {
     *cluster_used = 1;
     const uint64_t limit = debug_wait_limit_ns();
     return launch_rowstats_stream(a, bf16, s, limit ? limit : kWaitLimitNs);

@@ -7,10 +7,13 @@ can consume the very same bytes without sharing any of the method's code.
 
 from .workloads import (  # noqa: F401
     REWARD,
+    SEQUENCES,
+    SeqWorkload,
     WORKLOADS,
     Workload,
     bytes_per_tensor,
     make_logits,
     make_reward_logits,
+    make_seq_logits,
     workload,
 )

@@ -61,6 +61,71 @@ REWARD = dict(prompts=64, rollouts_per_group=16, windows_per_rollout=256, K=8, V
               dtype=torch.bfloat16)
 
 
+# Sequence layout (Sec. 3.3): logits stored once per position, [B][seq_len][V], with sliding
+# windows of K positions.  The validity mask marks each sequence's prompt (not trained on) and
+# the padding after its end: the prompt length is uniform in [prompt_lo, prompt_hi) and the
+# sequence ends at a length uniform in [end_lo, seq_len].
+@dataclasses.dataclass(frozen=True)
+class SeqWorkload:
+    name: str
+    B: int
+    seq_len: int
+    K: int
+    V: int
+    dtype: torch.dtype
+    recipe: str
+    prompt: tuple
+    end_lo: int
+    description: str
+
+
+SEQUENCES = {
+    "seq_tiny": SeqWorkload(
+        "seq_tiny", 3, 37, 4, 1000, torch.float32, "gauss", (0, 6), 25,
+        "B=3 x 37 positions, K=4, V=1000, fp32, gauss recipe; prompts of 0-5 positions, "
+        "sequences ending at 25-37"),
+    "seq_v128k": SeqWorkload(
+        "seq_v128k", 4, 2048, 7, 128256, torch.bfloat16, "zipf", (32, 512), 1024,
+        "B=4 x 2048 positions, K=7, V=128256, bf16, zipf recipe; prompts of 32-511 positions, "
+        "sequences ending at 1024-2048"),
+}
+
+SEQ_ROWS_PER_CHUNK = 2048
+
+
+def make_seq_logits(name: str, seed: int = 0, device="cpu", B: Optional[int] = None,
+                    seq_len: Optional[int] = None, V: Optional[int] = None,
+                    dtype: Optional[torch.dtype] = None, masked: bool = True):
+    """Draw (target, draft, mask) for a sequence workload: [B][seq_len][V] logits and a
+    [B][seq_len] uint8 mask (1 = trained position), or None with ``masked=False``."""
+    w = SEQUENCES[name]
+    B = w.B if B is None else B
+    T = w.seq_len if seq_len is None else seq_len
+    V = w.V if V is None else V
+    dtype = w.dtype if dtype is None else dtype
+    g = _gen(device, seed)
+    R = B * T
+    target = torch.empty((R, V), dtype=dtype, device=device)
+    draft = torch.empty((R, V), dtype=dtype, device=device)
+    for r0 in range(0, R, SEQ_ROWS_PER_CHUNK):
+        r1 = min(R, r0 + SEQ_ROWS_PER_CHUNK)
+        zp, zq = _chunk(w.recipe, r1 - r0, V, g, device)
+        target[r0:r1].copy_(zp)
+        draft[r0:r1].copy_(zq)
+        del zp, zq
+    mask = None
+    if masked:
+        gm = torch.Generator(device="cpu")
+        gm.manual_seed(int(seed) + 7919)
+        lo, hi = w.prompt
+        prompt = torch.randint(min(lo, T), max(min(hi, T), min(lo, T) + 1), (B,), generator=gm)
+        end = torch.randint(min(w.end_lo, T), T + 1, (B,), generator=gm)
+        t = torch.arange(T)
+        mask = ((t[None, :] >= prompt[:, None]) & (t[None, :] < end[:, None])).to(torch.uint8)
+        mask = mask.to(device)
+    return target.view(B, T, V), draft.view(B, T, V), mask
+
+
 def workload(name: str) -> Workload:
     return WORKLOADS[name]
 
@@ -187,5 +252,5 @@ def human_gb(nbytes: int) -> str:
     return f"{nbytes / 1e9:.2f} GB"
 
 
-__all__ = ["Workload", "WORKLOADS", "REWARD", "workload", "make_logits",
-           "make_reward_logits", "bytes_per_tensor", "human_gb"]
+__all__ = ["Workload", "WORKLOADS", "REWARD", "SeqWorkload", "SEQUENCES", "workload", "make_logits",
+           "make_reward_logits", "make_seq_logits", "bytes_per_tensor", "human_gb"]

@@ -25,15 +25,17 @@ GRAD_RTOL = 1e-2
 TIE_BAND = 1e-5
 
 MODES = {"greedy": aal.AAL_GREEDY, "sampling": aal.AAL_SAMPLING, "both": aal.AAL_BOTH}
-ORACLE_MODES = {aal.AAL_GREEDY: oracle.MODE_GREEDY, aal.AAL_SAMPLING: oracle.MODE_SAMPLING,
-                aal.AAL_BOTH: oracle.MODE_BOTH}
+# the C modes are bit sets with the oracle's values: 1 EAL, 2 WTV, 4 the KL anchor
+ORACLE_MODES = {m: (oracle.MODE_GREEDY if m & aal.AAL_GREEDY else 0)
+                | (oracle.MODE_SAMPLING if m & aal.AAL_SAMPLING else 0)
+                | (oracle.MODE_KL if m & aal.AAL_KL else 0) for m in range(1, 8)}
 
 
 class LossRun:
     """Forward + backward of one problem through the C ABI; results stay on the device."""
 
-    def __init__(self, target, draft, mask, mode, T=1.0, wg=1.0, ws=1.0, dloss=1.0):
-        self.prob = aal.loss_problem(draft, mode, T, wg, ws)
+    def __init__(self, target, draft, mask, mode, T=1.0, wg=1.0, ws=1.0, dloss=1.0, wkl=1.0):
+        self.prob = aal.loss_problem(draft, mode, T, wg, ws, wkl)
         self.ws_buf = torch.empty(aal.aal_workspace_size(self.prob), dtype=torch.uint8,
                                   device=draft.device)
         N = draft.shape[0]
@@ -68,7 +70,7 @@ def grad_tolerance(target, draft, mask, omode, T, wg, ws, dloss, gref, nvalid, f
 
 
 def check_loss(run: LossRun, target, draft, mask, mode, T, wg, ws, dloss=1.0, windows=None,
-               n_windows_total=None):
+               n_windows_total=None, wkl=1.0, n_positions_total=None):
     """Compare loss / eal / gradient of ``run`` with the oracle (optionally on some windows)."""
     omode = ORACLE_MODES[mode]
     if windows is None:
@@ -80,7 +82,7 @@ def check_loss(run: LossRun, target, draft, mask, mode, T, wg, ws, dloss=1.0, wi
         t_h, d_h = target[idx].cpu(), draft[idx].cpu()
         m_h = None if mask is None else mask[idx].cpu().numpy()
         sel = np.asarray(windows)
-    fw = oracle.loss_forward(t_h, d_h, m_h, omode, T, wg, ws, n_windows_total)
+    fw = oracle.objective_forward(t_h, d_h, m_h, omode, T, wg, ws, wkl, n_windows_total, n_positions_total)
     nvalid = fw["nvalid"]
     eal = run.eal.cpu().numpy()[sel]
     if omode & oracle.MODE_GREEDY:
@@ -91,7 +93,8 @@ def check_loss(run: LossRun, target, draft, mask, mode, T, wg, ws, dloss=1.0, wi
         ref = fw["loss"]
         got = float(run.loss.item())
         assert abs(got - ref) <= LOSS_RTOL * abs(ref) + LOSS_ATOL, (got, ref)
-    gref = oracle.loss_backward(t_h, d_h, m_h, omode, T, wg, ws, dloss, n_windows_total)
+    gref = oracle.objective_backward(t_h, d_h, m_h, omode, T, wg, ws, wkl, dloss, n_windows_total,
+                                     n_positions_total)
     g = run.grad.cpu().double().numpy()[sel]
     tol = grad_tolerance(t_h, d_h, m_h, omode, T, wg, ws, dloss, gref, nvalid, fw)
     bad = np.abs(g - gref) > tol
@@ -111,3 +114,100 @@ def loss_from_eal(run: LossRun, mode, wg, ws, nvalid):
     if mode & aal.AAL_SAMPLING:
         num += ws * eal[:, 1].sum()
     return -num / nvalid if nvalid else 0.0
+
+
+# -------------------------------------------------------------------------- sequence layout
+
+class SeqRun:
+    """Forward + backward of one sequence-layout problem through the C ABI."""
+
+    def __init__(self, target, draft, mask, K, mode, T=1.0, wg=1.0, ws=1.0, dloss=1.0, full_windows=False,
+                 wkl=1.0):
+        self.prob = aal.seq_problem(draft, K, mode, T, wg, ws, full_windows, wkl)
+        self.ws_buf = torch.empty(aal.aal_seq_workspace_size(self.prob), dtype=torch.uint8,
+                                  device=draft.device)
+        R = draft.shape[0] * draft.shape[1]
+        self.loss = torch.full((1,), float("nan"), dtype=torch.float32, device=draft.device)
+        self.eal = torch.full((max(R, 1), 2), float("nan"), dtype=torch.float32, device=draft.device)
+        self.grad = torch.full_like(draft, float("nan"))
+        aal.aal_seq_loss_fwd(self.prob, draft, target, mask, self.ws_buf, self.loss,
+                             self.eal if R > 0 else None)
+        aal.aal_seq_loss_bwd(self.prob, draft, target, mask, self.ws_buf, dloss, self.grad)
+        torch.cuda.synchronize()
+        assert aal.aal_check_device_status(self.ws_buf) == aal.AAL_OK
+
+
+def seq_grad_tolerance(target, draft, mask, K, omode, T, wg, ws, dloss, gref, nvalid_total,
+                       full_windows=False):
+    """Per-position tolerance: GRAD_ATOL + GRAD_RTOL |g_ref| plus the near-tie widening of every
+    window row the position contributes to."""
+    wp, wq, wm, src = oracle.gather_windows(target, draft, mask, K, full_windows)
+    fw = oracle.loss_forward(wp, wq, wm, omode, T, wg, ws, nvalid_total)
+    widen = grad_tolerance(wp, wq, wm, omode, T, wg, ws, dloss, np.zeros(wq.shape), nvalid_total,
+                           fw) - GRAD_ATOL
+    Bq, Tq, V = gref.shape
+    extra = np.zeros((Bq * Tq, V))
+    for n, j in np.argwhere(src >= 0):
+        extra[src[n, j]] += widen[n, j]
+    return GRAD_ATOL + GRAD_RTOL * np.abs(gref) + extra.reshape(Bq, Tq, V)
+
+
+def _assert_grad(g, gref, tol, where=""):
+    bad = np.abs(g - gref) > tol
+    if bad.any():
+        i = tuple(np.argwhere(bad)[0])
+        raise AssertionError(f"{where}{int(bad.sum())} gradient elements off; first {i}: "
+                             f"gpu {g[i]!r} oracle {gref[i]!r} tol {tol[i]!r}")
+
+
+def check_seq_loss(run: SeqRun, target, draft, mask, K, mode, T, wg, ws, dloss=1.0, full_windows=False,
+                   wkl=1.0):
+    """Every output of a sequence-layout run against the oracle on all positions."""
+    omode = ORACLE_MODES[mode]
+    t_h, d_h = target.cpu(), draft.cpu()
+    m_h = None if mask is None else mask.cpu().numpy()
+    fw = oracle.seq_objective_forward(t_h, d_h, m_h, K, omode, T, wg, ws, wkl, full_windows=full_windows)
+    eal = run.eal.cpu().numpy()
+    if omode & oracle.MODE_GREEDY:
+        np.testing.assert_allclose(eal[:, 0], fw["eal_g"], rtol=LOSS_RTOL, atol=LOSS_ATOL)
+    if omode & oracle.MODE_SAMPLING:
+        np.testing.assert_allclose(eal[:, 1], fw["eal_s"], rtol=LOSS_RTOL, atol=LOSS_ATOL)
+    got, ref = float(run.loss.item()), fw["loss"]
+    assert abs(got - ref) <= LOSS_RTOL * abs(ref) + LOSS_ATOL, (got, ref)
+    gref = oracle.seq_objective_backward(t_h, d_h, m_h, K, omode, T, wg, ws, wkl, dloss,
+                                         full_windows=full_windows)
+    tol = seq_grad_tolerance(t_h, d_h, m_h, K, omode, T, wg, ws, dloss, gref, fw["nvalid"], full_windows)
+    _assert_grad(run.grad.cpu().double().numpy(), gref, tol)
+    return fw
+
+
+def check_seq_positions(run: SeqRun, target, draft, mask, K, mode, T, wg, ws, dloss, positions,
+                        nvalid_total, wkl=1.0, npos_total=None):
+    """Sampled check at full size: for each (b, t) the oracle runs on positions t-K+1 .. t+K-1 of
+    sequence b only (every window containing t, and the window starting at t, lie inside), with
+    |W| (and the anchor's |positions|) of the whole batch; the window starting at t and the
+    gradient row of t are compared."""
+    omode = ORACLE_MODES[mode]
+    Tn = draft.shape[1]
+    eal = run.eal.view(draft.shape[0], Tn, 2)
+    for b, t in positions:
+        lo, hi = max(0, t - K + 1), min(Tn, t + K)
+        t_h = target[b:b + 1, lo:hi].cpu()
+        d_h = draft[b:b + 1, lo:hi].cpu()
+        m_h = None if mask is None else mask[b:b + 1, lo:hi].cpu().numpy()
+        fw = oracle.seq_objective_forward(t_h, d_h, m_h, K, omode, T, wg, ws, wkl, nvalid_total, npos_total)
+        e = eal[b, t].cpu().numpy()
+        if omode & oracle.MODE_GREEDY:
+            np.testing.assert_allclose(e[0], fw["eal_g"][t - lo], rtol=LOSS_RTOL, atol=LOSS_ATOL)
+        if omode & oracle.MODE_SAMPLING:
+            np.testing.assert_allclose(e[1], fw["eal_s"][t - lo], rtol=LOSS_RTOL, atol=LOSS_ATOL)
+        gref = oracle.seq_objective_backward(t_h, d_h, m_h, K, omode, T, wg, ws, wkl, dloss, nvalid_total,
+                                             npos_total)
+        tol = seq_grad_tolerance(t_h, d_h, m_h, K, omode, T, wg, ws, dloss, gref, nvalid_total)
+        g = run.grad[b, t].cpu().double().numpy()
+        _assert_grad(g, gref[0, t - lo], tol[0, t - lo], where=f"position ({b}, {t}): ")
+
+
+def seq_window_counts(mask, B, Tn):
+    """|W| of a sequence batch: the number of valid positions (each starts one window)."""
+    return B * Tn if mask is None else int(mask.sum().item())

@@ -41,7 +41,7 @@ def test_library_exports_every_declared_symbol():
 
 
 def test_status_strings_and_version():
-    assert aal.aal_abi_version() == 10000
+    assert aal.aal_abi_version() == 10100
     for code in range(6):
         assert aal.aal_status_string(code).startswith("AAL_")
     assert aal.aal_status_string(99) == "unknown aal_status"
@@ -49,7 +49,7 @@ def test_status_strings_and_version():
 
 def _prob(**kw):
     d = dict(N=4, K=3, V=100, dtype=aal.AAL_BF16, mode=aal.AAL_BOTH, temperature=1.0,
-             w_greedy=0.5, w_sampling=0.5, reserved=0)
+             w_greedy=0.5, w_sampling=0.5, w_kl=1.0, reserved=0)
     d.update(kw)
     return aal.AalProblem(**d)
 
@@ -73,7 +73,9 @@ def test_workspace_size_grows_with_rows():
     (dict(N=-1), aal.AAL_ERR_INVALID_ARG),
     (dict(dtype=7), aal.AAL_ERR_INVALID_ARG),
     (dict(mode=0), aal.AAL_ERR_INVALID_ARG),
-    (dict(mode=4), aal.AAL_ERR_INVALID_ARG),
+    (dict(mode=8), aal.AAL_ERR_INVALID_ARG),
+    (dict(mode=-1), aal.AAL_ERR_INVALID_ARG),
+    (dict(w_kl=float("nan")), aal.AAL_ERR_INVALID_ARG),
     (dict(temperature=0.0), aal.AAL_ERR_INVALID_ARG),
     (dict(temperature=-1.0), aal.AAL_ERR_INVALID_ARG),
     (dict(temperature=float("nan")), aal.AAL_ERR_INVALID_ARG),
@@ -88,6 +90,9 @@ def test_bad_problems_are_rejected(kw, code):
 
 def test_greedy_mode_accepts_zero_temperature():
     assert _ws_size(_prob(mode=aal.AAL_GREEDY, temperature=0.0))[0] == aal.AAL_OK
+    assert _ws_size(_prob(mode=aal.AAL_GREEDY | aal.AAL_KL, temperature=0.0))[0] == aal.AAL_OK
+    assert _ws_size(_prob(mode=aal.AAL_KL, temperature=0.0))[0] == aal.AAL_OK
+    assert _ws_size(_prob(mode=aal.AAL_KL | aal.AAL_SAMPLING, temperature=0.0))[0] == aal.AAL_ERR_INVALID_ARG
 
 
 def test_null_and_misaligned_pointers_rejected_before_launch():
@@ -162,3 +167,57 @@ def test_reward_from_loss_argument_checks():
     assert call(_rprob(N=8, K=4, V=100, mode=aal.AAL_SAMPLING, temperature=1.0), lps) == aal.AAL_ERR_INVALID_ARG
     # the loss workspace must be large enough
     assert call(rp, lp, fake, lsize - 1) == aal.AAL_ERR_WORKSPACE
+
+
+def _sprob(**kw):
+    d = dict(B=2, seq_len=16, K=4, V=100, dtype=aal.AAL_BF16, mode=aal.AAL_BOTH, temperature=1.0,
+             w_greedy=0.5, w_sampling=0.5, w_kl=1.0, full_windows=0, reserved=0)
+    d.update(kw)
+    return aal.AalSeqProblem(**d)
+
+
+def _seq_ws(p):
+    out = ctypes.c_size_t(0)
+    return aal.library().aal_seq_workspace_size(ctypes.byref(p), ctypes.byref(out)), out.value
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(), aal.AAL_OK),
+    (dict(B=0), aal.AAL_OK),
+    (dict(seq_len=0), aal.AAL_OK),
+    (dict(K=20), aal.AAL_ERR_UNSUPPORTED),
+    (dict(K=0), aal.AAL_ERR_INVALID_ARG),
+    (dict(B=-1), aal.AAL_ERR_INVALID_ARG),
+    (dict(seq_len=-3), aal.AAL_ERR_INVALID_ARG),
+    (dict(B=2**40, seq_len=2**40), aal.AAL_ERR_INVALID_ARG),     # B * seq_len overflows
+    (dict(B=2**30, seq_len=2**20, V=2**20), aal.AAL_ERR_INVALID_ARG),  # logit bytes overflow
+    (dict(V=0), aal.AAL_ERR_INVALID_ARG),
+    (dict(mode=0), aal.AAL_ERR_INVALID_ARG),
+    (dict(temperature=0.0), aal.AAL_ERR_INVALID_ARG),
+    (dict(reserved=2), aal.AAL_ERR_INVALID_ARG),
+    (dict(full_windows=1), aal.AAL_OK),
+    (dict(full_windows=2), aal.AAL_ERR_INVALID_ARG),
+])
+def test_seq_problem_checks(kw, code):
+    assert _seq_ws(_sprob(**kw))[0] == code
+
+
+def test_seq_workspace_holds_per_depth_partials():
+    c1, s1 = _seq_ws(_sprob(K=1))
+    c8, s8 = _seq_ws(_sprob(K=8))
+    # two float[B*seq_len][K] arrays, each 256-byte aligned: 2 x (32*8*4 - 256) more bytes for K = 8
+    assert c1 == c8 == aal.AAL_OK and s8 - s1 == 2 * (32 * 8 * 4 - 256) and s1 % 256 == 0
+
+
+def test_seq_pointer_checks_before_launch():
+    lib = aal.library()
+    p = _sprob()
+    code, size = _seq_ws(p)
+    fake_ws, fake = 1 << 20, 1 << 24
+    assert lib.aal_seq_loss_fwd(ctypes.byref(p), None, fake, None, fake_ws, size, fake, None, None) == aal.AAL_ERR_INVALID_ARG
+    assert lib.aal_seq_loss_fwd(ctypes.byref(p), fake, fake + 8, None, fake_ws, size, fake, None, None) == aal.AAL_ERR_INVALID_ARG
+    assert lib.aal_seq_loss_fwd(ctypes.byref(p), fake, fake, None, fake_ws, size, None, None, None) == aal.AAL_ERR_INVALID_ARG
+    assert lib.aal_seq_loss_fwd(ctypes.byref(p), fake, fake, None, fake_ws, size - 1, fake, None, None) == aal.AAL_ERR_WORKSPACE
+    assert lib.aal_seq_loss_bwd(ctypes.byref(p), fake, fake, None, fake_ws, size, 1.0, None, None) == aal.AAL_ERR_INVALID_ARG
+    assert lib.aal_seq_loss_bwd(ctypes.byref(p), fake, fake, None, fake_ws, size, float("inf"), fake, None) == aal.AAL_ERR_INVALID_ARG
+    assert lib.aal_seq_loss_bwd(ctypes.byref(p), fake, fake, None, fake_ws + 128, size, 1.0, fake, None) == aal.AAL_ERR_WORKSPACE
