@@ -6,7 +6,7 @@ Eqs. acc_greedy / acc_sample), the speculative-window expected accepted length
 (Sec. 3.1, Eq. eal_generic), the EAL and WTV losses (Eqs. loss_eal / loss_tv)
 with their gradient with respect to the draft logits, over independent windows and
 over whole sequences (Sec. 3.3), the forward-KL anchor of the combined objectives
-(Sec. 4.1), and the GRPO stage's
+(Sec. 4.1), the GRPO stage's clipped policy-ratio surrogate (Sec. 3.4), and its
 simulated acceptance length, debiased reward and group-normalised advantage
 (Sec. 3.4).  Every function computes its definition directly, with numpy in
 float64, so that a reader can check it against the paper by eye; nothing here
@@ -56,6 +56,7 @@ from .sequence import (  # noqa: F401
     seq_objective_backward,
     seq_objective_forward,
 )
+from .grpo import grpo_backward, grpo_forward, policy_log_ratio, trajectory_log_probs  # noqa: F401
 from .anchor import (  # noqa: F401
     MODE_KL,
     anchor_backward,
