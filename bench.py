@@ -236,6 +236,7 @@ def run_ours(args, ws_count, rank, local):
     greedy_obj = None if args.no_seq else run_greedy_objective(aal, draft, target, grad, stream,
                                                                 max(5, args.steps // 2))
     seq = None if args.no_seq else run_sequence_layout(aal, dev, stream, rank, max(5, args.steps // 2))
+    grpo = None if args.no_seq else run_grpo_phase(aal, dev, stream, rank, max(5, args.steps // 2))
 
     b = algo_bytes(N, K, V)
     step_bytes = sum(b.values())
@@ -288,6 +289,8 @@ def run_ours(args, ws_count, rank, local):
         res["greedy_objective"] = greedy_obj
     if seq is not None:
         res["sequence_layout"] = seq
+    if grpo is not None:
+        res["grpo_phase_step"] = grpo
 
     if rank == 0 and not args.no_e2e:
         res["e2e"] = run_e2e(args, aal, prob, rprob, draft, target, grad, ws, loss, rws, tau, rl, adv,
@@ -335,6 +338,57 @@ def run_greedy_objective(aal, draft, target, grad, stream, reps):
            "fwd_gbs": round(fb / (fwd * 1e-3) / 1e9, 1), "bwd_gbs": round(bb / (bwd * 1e-3) / 1e9, 1),
            "rows_per_s": round(R / ((fwd + bwd) * 1e-3), 1), "loss": float(loss.item())}
     del ws
+    return out
+
+
+def run_grpo_phase(aal, dev, stream, rank, reps):
+    """The paper's GRPO-phase step, L_KL + 0.1 L_EAL + 0.1 L_GRPO (Sec. 3.4, 4.1), over one prompt
+    group of the reward workload (16 rollouts x 256 windows, K = 8, V = 128256 bf16, the reference
+    draft = the draft + N(0, 0.3^2)): aal_loss_fwd, aal_grpo_from_loss (reads the reference
+    once), aal_loss_bwd.  Groups of 16 single-window samples."""
+    target, draft, ref = synth.make_reward_logits(rank, seed=0, device=dev, with_ref=True, ref_from_draft=0.3)
+    N, K, V = draft.shape
+    grad = torch.empty_like(draft)
+    mode = aal.AAL_KL | aal.AAL_GREEDY | aal.AAL_GRPO
+    lprob = aal.loss_problem(draft, mode, 1.0, 0.1, 0.0, 1.0)
+    lws = torch.empty(aal.aal_workspace_size(lprob), dtype=torch.uint8, device=dev)
+    gprob = aal.grpo_problem(draft, 1, 16, 5.0, 0.2, 0.0, 10.0, 10.0, 0.1)
+    gws = torch.empty(aal.aal_grpo_workspace_size(gprob), dtype=torch.uint8, device=dev)
+    loss = torch.empty(1, dtype=torch.float32, device=dev)
+    gloss = torch.empty(1, dtype=torch.float32, device=dev)
+
+    def step():
+        aal.aal_loss_fwd(lprob, draft, target, None, lws, loss, None, stream)
+        aal.aal_grpo_from_loss(gprob, lprob, lws, ref, gws, gloss, stream=stream)
+        aal.aal_loss_bwd(lprob, draft, target, None, lws, 1.0, grad, stream)
+
+    for _ in range(3):
+        step()
+    torch.cuda.synchronize()
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(reps)]
+    for e in ev:
+        e[0].record(stream)
+        aal.aal_loss_fwd(lprob, draft, target, None, lws, loss, None, stream)
+        e[1].record(stream)
+        aal.aal_grpo_from_loss(gprob, lprob, lws, ref, gws, gloss, stream=stream)
+        e[2].record(stream)
+        aal.aal_loss_bwd(lprob, draft, target, None, lws, 1.0, grad, stream)
+        e[3].record(stream)
+    torch.cuda.synchronize()
+    assert aal.aal_check_device_status(lws) == aal.AAL_OK
+    ms = [sum(e[i].elapsed_time(e[i + 1]) for e in ev) / reps for i in range(3)]
+    R = N * K
+    row = V * draft.element_size()
+    b = [2 * R * row, R * row, 3 * R * row]
+    tot = sum(ms)
+    out = {"workload": f"reward group: {N} windows (16 rollouts x 256), K={K}, V={V} bf16; "
+                       "L_KL + 0.1 L_EAL + 0.1 L_GRPO, groups of 16 windows",
+           "ms": round(tot, 4), "fwd_ms": round(ms[0], 4), "grpo_ms": round(ms[1], 4), "bwd_ms": round(ms[2], 4),
+           "gbs": round(sum(b) / (tot * 1e-3) / 1e9, 1),
+           "fwd_gbs": round(b[0] / (ms[0] * 1e-3) / 1e9, 1), "grpo_gbs": round(b[1] / (ms[1] * 1e-3) / 1e9, 1),
+           "bwd_gbs": round(b[2] / (ms[2] * 1e-3) / 1e9, 1), "rows_per_s": round(R / (tot * 1e-3), 1),
+           "loss": float(loss.item()), "grpo_loss": float(gloss.item())}
+    del target, draft, ref, grad, lws, gws
     return out
 
 

@@ -67,8 +67,12 @@ typedef enum { AAL_F32 = 0, AAL_BF16 = 1 } aal_dtype;
  * forward-KL anchor of the combined objectives (Sec. 4.1): the mean over valid positions of
  * KL(p || q) = sum_v p(v) (log p(v) - log q(v)) at T = 1.  The greedy-regime objective of
  * Sec. 4.1, L_KL + 0.1 L_EAL, is mode AAL_KL | AAL_GREEDY with w_kl = 1, w_greedy = 0.1;
- * mode AAL_KL alone is the L_KL baseline.  Valid modes: 1 .. 7. */
-typedef enum { AAL_GREEDY = 1, AAL_SAMPLING = 2, AAL_BOTH = 3, AAL_KL = 4 } aal_mode;
+ * mode AAL_KL alone is the L_KL baseline.  AAL_GRPO makes aal_loss_bwd add the gradient of
+ * the GRPO surrogate (Sec. 3.4) whose per-row coefficients aal_grpo_from_loss writes into the
+ * loss workspace between the forward and the backward; aal_loss_fwd clears them, so without
+ * that call the term is zero, and the loss aal_loss_fwd reports never includes it (see
+ * aal_grpo_from_loss).  Valid modes: 1 .. 15 (AAL_GRPO only with aal_loss_*). */
+typedef enum { AAL_GREEDY = 1, AAL_SAMPLING = 2, AAL_BOTH = 3, AAL_KL = 4, AAL_GRPO = 8 } aal_mode;
 
 #define AAL_MAX_K 8
 
@@ -175,6 +179,63 @@ AAL_API aal_status aal_seq_loss_fwd(const aal_seq_problem* prob, const void* dra
 AAL_API aal_status aal_seq_loss_bwd(const aal_seq_problem* prob, const void* draft, const void* target,
                                     const uint8_t* mask, const void* workspace, size_t workspace_bytes,
                                     float dloss, void* grad_draft, void* stream);
+
+/* The GRPO surrogate of Sec. 3.4 over the windows of a completed aal_loss_fwd.
+ *   N, K, V, dtype       must equal the loss problem's (windows of K depths, no mask: every
+ *                        window is verified over all K depths).
+ *   windows_per_rollout, rollouts_per_group, adv_clip   grouping and C_A as in
+ *                        aal_reward_problem (N a multiple of their product); the paper's
+ *                        samples are single windows (windows_per_rollout = 1, groups of m).
+ *   eps_clip             PPO clip epsilon, in [0, 1).
+ *   rho_min, rho_max     the ratio's safety clip, 0 <= rho_min <= rho_max (finite).
+ *   log_rho_clip         clip of log rho before exponentiating (> 0; the paper uses 10).
+ *   w_grpo               weight of L_GRPO in the gradient the loss backward adds (finite). */
+typedef struct {
+  int64_t N, K, V;
+  int32_t dtype;
+  int32_t reserved; /* must be 0 */
+  int64_t windows_per_rollout;
+  int64_t rollouts_per_group;
+  float adv_clip;
+  float eps_clip;
+  float rho_min;
+  float rho_max;
+  float log_rho_clip;
+  float w_grpo;
+} aal_grpo_problem;
+
+AAL_API aal_status aal_grpo_workspace_size(const aal_grpo_problem* prob, size_t* bytes);
+
+/* GRPO stage of one batch (Sec. 3.4), from the statistics of a completed aal_loss_fwd whose mode
+ * includes AAL_GRPO plus one pass over the reference draft.  Per window t with the draft's greedy
+ * tokens S_k = argmax z_q (recorded by the forward):
+ *   tau^theta, tau^ref    leading runs of S_k = x*_k and of argmax z_ref = x*_k (greedy
+ *                         verification against the target's argmax, lowest index on ties);
+ *   A                     the clipped group-standardised advantage of R = tau^theta - tau^ref
+ *                         (as aal_accept_reward with the reference draft);
+ *   log rho_t             (1/K) sum_k [log pi_theta(S_k) - log pi_ref(S_k)] (softmax at T = 1),
+ *                         clipped to [-log_rho_clip, log_rho_clip];
+ *   rho_t                 exp(log rho_t) clipped to [rho_min, rho_max];
+ *   L_GRPO                -(1/N) sum_t min(rho_t A_t, clip(rho_t, 1 - eps, 1 + eps) A_t), the mean
+ *                         over equal groups of the groups' mean surrogates.
+ * R and A carry no gradient; the trajectory is held fixed.  The call writes, into the loss
+ * workspace, w_grpo times dL_GRPO/d log pi_theta(S_k) for every row, which the following
+ * aal_loss_bwd (same problem, mode with AAL_GRPO) turns into c (delta_{u,S_k} - q(u)); the
+ * objective whose gradient that backward writes is therefore the forward's loss plus
+ * w_grpo * L_GRPO.
+ *   gprob, lprob           the GRPO problem and the loss problem of the forward.
+ *   loss_workspace         the forward's workspace (read, and its GRPO coefficients written).
+ *   ref_draft              [N][K][V] logits of the frozen reference draft (16-byte aligned).
+ *   workspace              at least aal_grpo_workspace_size(gprob) bytes, 256-byte aligned.
+ *   grpo_loss              device float[1]: L_GRPO (unweighted).
+ *   tau, tau_ref           device int32[N] or NULL.
+ *   advantage              device float[N / windows_per_rollout] or NULL.
+ *   log_rho                device float[N] (the clipped log rho) or NULL. */
+AAL_API aal_status aal_grpo_from_loss(const aal_grpo_problem* gprob, const aal_problem* lprob,
+                                      void* loss_workspace, size_t loss_workspace_bytes,
+                                      const void* ref_draft, void* workspace, size_t workspace_bytes,
+                                      float* grpo_loss, int32_t* tau, int32_t* tau_ref, float* advantage,
+                                      float* log_rho, void* stream);
 
 /* Simulated acceptance reward of the GRPO stage (Sec. 3.4).
  *   N, K, V, dtype       as for the loss; K is the window size gamma (1..AAL_MAX_K).

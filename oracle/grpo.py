@@ -52,20 +52,31 @@ def policy_log_ratio(draft, ref_draft, log_rho_clip: float = LOG_RHO_CLIP):
 
 def grpo_forward(target, draft, ref_draft, windows_per_rollout: int = 1, rollouts_per_group: int = 1,
                  adv_clip: float = 5.0, eps_clip: float = 0.2, rho_min: float = 0.0,
-                 rho_max: float = 10.0, log_rho_clip: float = LOG_RHO_CLIP):
+                 rho_max: float = 10.0, log_rho_clip: float = LOG_RHO_CLIP,
+                 advantage_window=None, n_windows_total=None):
+    """``advantage_window`` and ``n_windows_total`` stand in for the advantages and N of a larger
+    batch when only some of its windows are passed in (then the loss is those windows' share)."""
     zq = as_f64(draft)
     N = zq.shape[0]
-    rw = accept_reward(target, draft, ref_draft, REWARD_GREEDY, windows_per_rollout=windows_per_rollout,
-                       rollouts_per_group=rollouts_per_group, adv_clip=adv_clip)
-    A = np.repeat(rw["advantage"], windows_per_rollout)           # per window
+    rw = None
+    if advantage_window is None:
+        rw = accept_reward(target, draft, ref_draft, REWARD_GREEDY, windows_per_rollout=windows_per_rollout,
+                           rollouts_per_group=rollouts_per_group, adv_clip=adv_clip)
+        A = np.repeat(rw["advantage"], windows_per_rollout)       # per window
+    else:
+        A = np.asarray(advantage_window, dtype=np.float64)
     log_rho, raw, S = policy_log_ratio(draft, ref_draft, log_rho_clip)
     rho_exp = np.exp(log_rho)
     rho = np.clip(rho_exp, rho_min, rho_max)
     surrogate = np.minimum(rho * A, np.clip(rho, 1.0 - eps_clip, 1.0 + eps_clip) * A)
     m = windows_per_rollout * rollouts_per_group
-    G = N // m
-    group_loss = np.array([-np.mean(surrogate[g * m:(g + 1) * m]) for g in range(G)])
-    loss = float(np.mean(group_loss)) if G > 0 else 0.0
+    if n_windows_total is None:
+        G = N // m
+        group_loss = np.array([-np.mean(surrogate[g * m:(g + 1) * m]) for g in range(G)])
+        loss = float(np.mean(group_loss)) if G > 0 else 0.0
+    else:   # equal groups: the mean of group means is the mean over all windows
+        group_loss = None
+        loss = float(-np.sum(surrogate) / n_windows_total)
     return dict(loss=loss, group_loss=group_loss, log_rho=log_rho, log_rho_raw=raw, rho=rho,
                 rho_exp=rho_exp, advantage_window=A, surrogate=surrogate, S=S, reward=rw)
 
@@ -73,14 +84,15 @@ def grpo_forward(target, draft, ref_draft, windows_per_rollout: int = 1, rollout
 def grpo_backward(target, draft, ref_draft, windows_per_rollout: int = 1, rollouts_per_group: int = 1,
                   adv_clip: float = 5.0, eps_clip: float = 0.2, rho_min: float = 0.0,
                   rho_max: float = 10.0, log_rho_clip: float = LOG_RHO_CLIP,
-                  dloss: float = 1.0) -> np.ndarray:
+                  dloss: float = 1.0, advantage_window=None, n_windows_total=None) -> np.ndarray:
     """dloss * dL_GRPO/dz_theta, [N][K][V] (see the module docstring)."""
     zq = as_f64(draft)
     N, K, V = zq.shape
     fw = grpo_forward(target, draft, ref_draft, windows_per_rollout, rollouts_per_group, adv_clip,
-                      eps_clip, rho_min, rho_max, log_rho_clip)
+                      eps_clip, rho_min, rho_max, log_rho_clip, advantage_window, n_windows_total)
     m = windows_per_rollout * rollouts_per_group
-    G = N // m
+    n_all = N if n_windows_total is None else int(n_windows_total)
+    G = n_all // m
     grad = np.zeros((N, K, V))
     if G == 0:
         return grad

@@ -20,12 +20,14 @@ from .aal import (  # noqa: F401
     AAL_ERR_WORKSPACE,
     AAL_F32,
     AAL_GREEDY,
+    AAL_GRPO,
     AAL_KL,
     AAL_MAX_K,
     AAL_NOALLOC_MAX_ROWS,
     AAL_OK,
     AAL_SAMPLING,
     AalError,
+    AalGrpoProblem,
     AalProblem,
     AalRewardProblem,
     AalSeqProblem,
@@ -35,6 +37,8 @@ from .aal import (  # noqa: F401
     aal_accept_reward_noalloc,
     aal_check_device_status,
     aal_debug_fail_next_forward,
+    aal_grpo_from_loss,
+    aal_grpo_workspace_size,
     aal_loss_bwd,
     aal_loss_fwd,
     aal_reward_workspace_size,
@@ -46,6 +50,7 @@ from .aal import (  # noqa: F401
     library,
     library_path,
     loss_problem,
+    grpo_problem,
     reward_problem,
     seq_problem,
 )

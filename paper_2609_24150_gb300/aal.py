@@ -22,6 +22,7 @@ AAL_GREEDY = 1
 AAL_SAMPLING = 2
 AAL_BOTH = 3
 AAL_KL = 4          # mode bit: the forward-KL anchor
+AAL_GRPO = 8        # mode bit: the backward adds the GRPO surrogate's gradient
 
 AAL_MAX_K = 8
 AAL_NOALLOC_MAX_ROWS = 1 << 20   # N * K limit of aal_accept_reward_noalloc
@@ -59,6 +60,16 @@ class AalSeqProblem(ctypes.Structure):
                 ("full_windows", ctypes.c_int32), ("reserved", ctypes.c_int32)]
 
 
+class AalGrpoProblem(ctypes.Structure):
+    """Mirror of ``aal_grpo_problem``."""
+    _fields_ = [("N", ctypes.c_int64), ("K", ctypes.c_int64), ("V", ctypes.c_int64),
+                ("dtype", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("windows_per_rollout", ctypes.c_int64), ("rollouts_per_group", ctypes.c_int64),
+                ("adv_clip", ctypes.c_float), ("eps_clip", ctypes.c_float),
+                ("rho_min", ctypes.c_float), ("rho_max", ctypes.c_float),
+                ("log_rho_clip", ctypes.c_float), ("w_grpo", ctypes.c_float)]
+
+
 class AalError(RuntimeError):
     def __init__(self, code: int, where: str):
         self.code = code
@@ -91,6 +102,9 @@ def library() -> ctypes.CDLL:
     lib.aal_seq_workspace_size.argtypes = [SP, ctypes.POINTER(sz)]
     lib.aal_seq_loss_fwd.argtypes = [SP, vp, vp, vp, vp, sz, vp, vp, vp]
     lib.aal_seq_loss_bwd.argtypes = [SP, vp, vp, vp, vp, sz, ctypes.c_float, vp, vp]
+    GP = ctypes.POINTER(AalGrpoProblem)
+    lib.aal_grpo_workspace_size.argtypes = [GP, ctypes.POINTER(sz)]
+    lib.aal_grpo_from_loss.argtypes = [GP, P, vp, sz, vp, vp, sz, vp, vp, vp, vp, vp, vp]
     lib.aal_check_device_status.argtypes = [vp, vp]
     lib.aal_debug_fail_next_forward.argtypes = [ctypes.c_int64, ctypes.c_uint64]
     lib.aal_debug_fail_next_forward.restype = None
@@ -100,7 +114,8 @@ def library() -> ctypes.CDLL:
     lib.aal_abi_version.restype = ctypes.c_int32
     for f in ("aal_workspace_size", "aal_reward_workspace_size", "aal_loss_fwd", "aal_loss_bwd",
               "aal_accept_reward", "aal_accept_reward_noalloc", "aal_accept_reward_from_loss",
-              "aal_seq_workspace_size", "aal_seq_loss_fwd", "aal_seq_loss_bwd", "aal_check_device_status"):
+              "aal_seq_workspace_size", "aal_seq_loss_fwd", "aal_seq_loss_bwd", "aal_check_device_status",
+              "aal_grpo_workspace_size", "aal_grpo_from_loss"):
         getattr(lib, f).restype = ctypes.c_int
     _LIB = lib
     return lib
@@ -222,6 +237,41 @@ def aal_loss_bwd(problem: AalProblem, draft, target, mask, workspace, dloss: flo
         _ptr(mask, "mask", torch.uint8), _ptr(workspace, "workspace"), _nbytes(workspace),
         float(dloss), _ptr(grad, "grad"), _stream(stream))
     _check(code, "aal_loss_bwd")
+
+
+def grpo_problem(draft: torch.Tensor, windows_per_rollout: int = 1, rollouts_per_group: int = 1,
+                 adv_clip: float = 5.0, eps_clip: float = 0.2, rho_min: float = 0.0, rho_max: float = 10.0,
+                 log_rho_clip: float = 10.0, w_grpo: float = 1.0) -> AalGrpoProblem:
+    """GRPO problem struct for the [N][K][V] windows of a loss problem."""
+    if draft.dim() != 3:
+        raise ValueError("logits must be [N][K][V]")
+    N, K, V = draft.shape
+    return AalGrpoProblem(N, K, V, _DTYPES[draft.dtype], 0, windows_per_rollout, rollouts_per_group,
+                          adv_clip, eps_clip, rho_min, rho_max, log_rho_clip, w_grpo)
+
+
+def aal_grpo_workspace_size(problem: AalGrpoProblem) -> int:
+    out = ctypes.c_size_t(0)
+    _check(library().aal_grpo_workspace_size(ctypes.byref(problem), ctypes.byref(out)),
+           "aal_grpo_workspace_size")
+    return out.value
+
+
+def aal_grpo_from_loss(problem: AalGrpoProblem, loss_problem_: AalProblem, loss_workspace, ref_draft,
+                       workspace, grpo_loss, tau=None, tau_ref=None, advantage=None, log_rho=None,
+                       stream=None):
+    """GRPO stage after aal_loss_fwd (mode with AAL_GRPO): L_GRPO, tau, tau_ref, advantages,
+    log rho; writes the surrogate's gradient coefficients into the loss workspace."""
+    N = problem.N
+    nroll = N // max(1, problem.windows_per_rollout)
+    code = library().aal_grpo_from_loss(
+        ctypes.byref(problem), ctypes.byref(loss_problem_), _ptr(loss_workspace, "loss_workspace"),
+        _nbytes(loss_workspace), _ptr(ref_draft, "ref_draft"), _ptr(workspace, "workspace"),
+        _nbytes(workspace), _ptr(grpo_loss, "grpo_loss", torch.float32, 1),
+        _ptr(tau, "tau", torch.int32, N), _ptr(tau_ref, "tau_ref", torch.int32, N),
+        _ptr(advantage, "advantage", torch.float32, nroll), _ptr(log_rho, "log_rho", torch.float32, N),
+        _stream(stream))
+    _check(code, "aal_grpo_from_loss")
 
 
 def aal_seq_workspace_size(problem: AalSeqProblem) -> int:

@@ -30,7 +30,7 @@ aal_status check_problem(const aal_problem* p) {
   if (p == nullptr) return AAL_ERR_INVALID_ARG;
   aal_status st = check_shape(p->N, p->K, p->V, p->dtype);
   if (st != AAL_OK) return st;
-  if (p->mode < 1 || p->mode > (AAL_BOTH | AAL_KL)) return AAL_ERR_INVALID_ARG;
+  if (p->mode < 1 || p->mode > (AAL_BOTH | AAL_KL | AAL_GRPO)) return AAL_ERR_INVALID_ARG;
   if ((p->mode & AAL_SAMPLING) && !(isfinite(p->temperature) && p->temperature > 0.f)) return AAL_ERR_INVALID_ARG;
   if (!isfinite(p->w_greedy) || !isfinite(p->w_sampling) || !isfinite(p->w_kl)) return AAL_ERR_INVALID_ARG;
   if (p->reserved != 0) return AAL_ERR_INVALID_ARG;
@@ -60,7 +60,27 @@ aal_status check_seq(const aal_seq_problem* p) {
   // the per-depth partials too)
   const aal_problem q{p->B * p->seq_len, p->K, p->V, p->dtype, p->mode, p->temperature, p->w_greedy,
                       p->w_sampling, p->w_kl, p->reserved};
-  return check_problem(&q);
+  aal_status st = check_problem(&q);
+  if (st != AAL_OK) return st;
+  if (p->mode & AAL_GRPO) return AAL_ERR_UNSUPPORTED;  // the GRPO stage runs over windows
+  return AAL_OK;
+}
+
+aal_status check_grpo(const aal_grpo_problem* p) {
+  if (p == nullptr) return AAL_ERR_INVALID_ARG;
+  aal_status st = check_shape(p->N, p->K, p->V, p->dtype);
+  if (st != AAL_OK) return st;
+  if (p->reserved != 0) return AAL_ERR_INVALID_ARG;
+  if (p->windows_per_rollout < 1 || p->rollouts_per_group < 1) return AAL_ERR_INVALID_ARG;
+  if (p->windows_per_rollout > INT64_MAX / p->rollouts_per_group) return AAL_ERR_INVALID_ARG;
+  if (p->N % (p->windows_per_rollout * p->rollouts_per_group) != 0) return AAL_ERR_INVALID_ARG;
+  if (!(isfinite(p->adv_clip) && p->adv_clip > 0.f)) return AAL_ERR_INVALID_ARG;
+  if (!(p->eps_clip >= 0.f && p->eps_clip < 1.f)) return AAL_ERR_INVALID_ARG;
+  if (!(isfinite(p->rho_min) && isfinite(p->rho_max) && p->rho_min >= 0.f && p->rho_min <= p->rho_max))
+    return AAL_ERR_INVALID_ARG;
+  if (!(isfinite(p->log_rho_clip) && p->log_rho_clip > 0.f)) return AAL_ERR_INVALID_ARG;
+  if (!isfinite(p->w_grpo)) return AAL_ERR_INVALID_ARG;
+  return AAL_OK;
 }
 
 aal_status cuda_status(cudaError_t e) { return e == cudaSuccess ? AAL_OK : AAL_ERR_CUDA; }
@@ -70,6 +90,7 @@ cudaError_t launch_stats(const void* draft, const void* target, int64_t R, int64
                          int32_t mode, float temperature, const LossWs& ws, cudaStream_t s, int* cluster) {
   const bool greedy = (mode & AAL_GREEDY) != 0, sampling = (mode & AAL_SAMPLING) != 0;
   const bool kl = (mode & AAL_KL) != 0;
+  const bool grpo = (mode & AAL_GRPO) != 0;  // log pi_theta(y) needs the T = 1 normaliser
   RowStatsArgs ra;
   ra.zq = draft;
   ra.zp = target;
@@ -78,7 +99,7 @@ cudaError_t launch_stats(const void* draft, const void* target, int64_t R, int64
   ra.sT = sampling ? kLog2e / temperature : 0.f;
   ra.need_p = sampling;
   ra.need_q = sampling;
-  ra.need_q1 = (greedy || kl) && !(sampling && temperature == 1.0f);
+  ra.need_q1 = (greedy || kl || grpo) && !(sampling && temperature == 1.0f);
   ra.overlap = sampling;
   ra.need_kl = kl;
   ra.skip_chunk = debug_take_skip_chunk();
@@ -93,6 +114,7 @@ cudaError_t launch_grad(const void* draft, const void* target, const uint8_t* ma
                         float w_kl, float dloss, const LossWs& ws, void* grad, cudaStream_t s) {
   const bool greedy = (mode & AAL_GREEDY) != 0, sampling = (mode & AAL_SAMPLING) != 0;
   const bool kl = (mode & AAL_KL) != 0;
+  const bool grpo = (mode & AAL_GRPO) != 0;
   BackwardArgs ba;
   ba.zq = draft;
   ba.zp = target;
@@ -106,8 +128,9 @@ cudaError_t launch_grad(const void* draft, const void* target, const uint8_t* ma
   ba.w_greedy = greedy ? w_greedy : 0.f;
   ba.w_sampling = sampling ? w_sampling : 0.f;
   ba.w_kl = kl ? w_kl : 0.f;
+  ba.grpo = grpo;
   ba.mask = mask;
-  ba.q1_is_qT = (greedy || kl) && sampling && temperature == 1.0f;
+  ba.q1_is_qT = (greedy || kl || grpo) && sampling && temperature == 1.0f;
   ba.ws = ws;
   return launch_backward(ba, dtype == AAL_BF16, s);
 }
@@ -173,6 +196,10 @@ aal_status aal_loss_fwd(const aal_problem* prob, const void* draft, const void* 
   LossWs ws = loss_ws(workspace, L);
   cudaError_t e = cudaMemsetAsync(ws.hdr, 0, sizeof(WsHeader), s);
   if (e != cudaSuccess) return AAL_ERR_CUDA;
+  if (prob->mode & AAL_GRPO) {  // no GRPO term until aal_grpo_from_loss writes one
+    e = cudaMemsetAsync(ws.cgr, 0, (size_t)L.R * sizeof(float), s);
+    if (e != cudaSuccess) return AAL_ERR_CUDA;
+  }
   int cluster = 1;
   e = launch_stats(draft, target, L.R, prob->V, prob->dtype, prob->mode, prob->temperature, ws, s, &cluster);
   if (e != cudaSuccess) return AAL_ERR_CUDA;
@@ -285,6 +312,89 @@ aal_status aal_seq_loss_bwd(const aal_seq_problem* prob, const void* draft, cons
                                  prob->temperature, prob->w_greedy, prob->w_sampling, prob->w_kl, dloss,
                                  loss_ws(const_cast<void*>(workspace), L.base), grad_draft,
                                  static_cast<cudaStream_t>(stream)));
+}
+
+aal_status aal_grpo_workspace_size(const aal_grpo_problem* prob, size_t* bytes) {
+  aal_status st = check_grpo(prob);
+  if (st != AAL_OK) return st;
+  if (bytes == nullptr) return AAL_ERR_INVALID_ARG;
+  *bytes = grpo_layout(prob->N, prob->K, prob->windows_per_rollout).total;
+  return AAL_OK;
+}
+
+aal_status aal_grpo_from_loss(const aal_grpo_problem* gprob, const aal_problem* lprob, void* loss_workspace,
+                              size_t loss_workspace_bytes, const void* ref_draft, void* workspace,
+                              size_t workspace_bytes, float* grpo_loss, int32_t* tau, int32_t* tau_ref,
+                              float* advantage, float* log_rho, void* stream) {
+  aal_status st = check_grpo(gprob);
+  if (st != AAL_OK) return st;
+  st = check_problem(lprob);
+  if (st != AAL_OK) return st;
+  if (!(lprob->mode & AAL_GRPO)) return AAL_ERR_INVALID_ARG;
+  if (gprob->N != lprob->N || gprob->K != lprob->K || gprob->V != lprob->V || gprob->dtype != lprob->dtype)
+    return AAL_ERR_INVALID_ARG;
+  if (grpo_loss == nullptr || !aligned(grpo_loss, 4) || (tau != nullptr && !aligned(tau, 4)) ||
+      (tau_ref != nullptr && !aligned(tau_ref, 4)) || (advantage != nullptr && !aligned(advantage, 4)) ||
+      (log_rho != nullptr && !aligned(log_rho, 4)))
+    return AAL_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (gprob->N == 0) return cuda_status(cudaMemsetAsync(grpo_loss, 0, sizeof(float), s));
+  if (ref_draft == nullptr || !aligned(ref_draft, 16)) return AAL_ERR_INVALID_ARG;
+  const LossLayout LL = loss_layout(lprob->N, lprob->K);
+  if (loss_workspace == nullptr || !aligned(loss_workspace, 256) || loss_workspace_bytes < LL.total)
+    return AAL_ERR_WORKSPACE;
+  const GrpoLayout L = grpo_layout(gprob->N, gprob->K, gprob->windows_per_rollout);
+  if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < L.total) return AAL_ERR_WORKSPACE;
+  char* base = static_cast<char*>(workspace);
+  WsHeader* hdr = reinterpret_cast<WsHeader*>(base + L.hdr);
+  if (cudaMemsetAsync(hdr, 0, sizeof(WsHeader), s) != cudaSuccess) return AAL_ERR_CUDA;
+  const LossWs lws = loss_ws(loss_workspace, LL);
+
+  GrpoRefArgs ra;
+  ra.zr = ref_draft;
+  ra.R = L.R;
+  ra.V = gprob->V;
+  ra.lws = lws;
+  ra.acc = reinterpret_cast<uint8_t*>(base + L.acc);
+  ra.acc_ref = reinterpret_cast<uint8_t*>(base + L.acc_ref);
+  ra.lpr = reinterpret_cast<float*>(base + L.lpr);
+  ra.hdr = hdr;
+  if (launch_grpo_ref_rows(ra, gprob->dtype == AAL_BF16, s) != cudaSuccess) return AAL_ERR_CUDA;
+
+  float* adv = advantage != nullptr ? advantage : reinterpret_cast<float*>(base + L.adv);
+  RewardGroupArgs ga;
+  ga.acc = ra.acc;
+  ga.acc_ref = ra.acc_ref;
+  ga.rbuf = reinterpret_cast<float*>(base + L.rbuf);
+  ga.N = gprob->N;
+  ga.K = (int32_t)gprob->K;
+  ga.wpr = gprob->windows_per_rollout;
+  ga.rpg = gprob->rollouts_per_group;
+  ga.adv_clip = gprob->adv_clip;
+  ga.tau = tau != nullptr ? tau : reinterpret_cast<int32_t*>(base + L.tau);
+  ga.tau_ref = tau_ref != nullptr ? tau_ref : reinterpret_cast<int32_t*>(base + L.tau_ref);
+  ga.rollout_len = reinterpret_cast<float*>(base + L.rl);
+  ga.advantage = adv;
+  if (launch_reward_groups(ga, s) != cudaSuccess) return AAL_ERR_CUDA;
+
+  GrpoWindowArgs wa;
+  wa.lws = lws;
+  wa.lpr = ra.lpr;
+  wa.adv = adv;
+  wa.N = gprob->N;
+  wa.K = (int32_t)gprob->K;
+  wa.wpr = gprob->windows_per_rollout;
+  wa.eps_clip = gprob->eps_clip;
+  wa.rho_min = gprob->rho_min;
+  wa.rho_max = gprob->rho_max;
+  wa.log_rho_clip = gprob->log_rho_clip;
+  wa.w_grpo = gprob->w_grpo;
+  wa.log_rho = log_rho;
+  wa.part = reinterpret_cast<double*>(base + L.part);
+  wa.nblk = L.nblk;
+  wa.hdr = hdr;
+  wa.loss = grpo_loss;
+  return cuda_status(launch_grpo_windows(wa, s));
 }
 
 aal_status aal_accept_reward(const aal_reward_problem* prob, const void* draft, const void* target,

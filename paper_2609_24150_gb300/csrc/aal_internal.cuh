@@ -39,6 +39,7 @@ struct LossLayout {
   size_t Mp = 0, Lsp = 0, Mq = 0, Lsq = 0, Mq1 = 0, Lsq1 = 0;
   size_t Mp1 = 0, Lsp1 = 0;         // float[R] the normaliser of z_p at T = 1 (KL anchor)
   size_t kl = 0;                    // float[R] KL(p || q) at T = 1 (KL anchor)
+  size_t cgr = 0;                   // float[R] GRPO coefficient of (delta_{u,y} - q(u)), w_grpo included
   size_t ag = 0, as = 0, qlt = 0;   // float[R] a^greedy, a^sample, sum_{lq<lp} q~
   size_t dEg = 0, dEs = 0;          // float[R] dE_n / da_{n,j}
   size_t xstar = 0;                 // int32[R] target argmax
@@ -76,6 +77,7 @@ inline LossLayout loss_layout(int64_t N, int64_t K) {
   L.Mp1 = take(R * 4);
   L.Lsp1 = take(R * 4);
   L.kl = take(R * 4);
+  L.cgr = take(R * 4);
   L.ag = take(R * 4);
   L.as = take(R * 4);
   L.qlt = take(R * 4);
@@ -139,7 +141,7 @@ inline RewardLayout reward_layout(int64_t N, int64_t K) {
 // Pointers into a loss workspace.
 struct LossWs {
   WsHeader* hdr;
-  float *Mp, *Lsp, *Mq, *Lsq, *Mq1, *Lsq1, *Mp1, *Lsp1, *kl, *ag, *as, *qlt, *dEg, *dEs;
+  float *Mp, *Lsp, *Mq, *Lsq, *Mq1, *Lsq1, *Mp1, *Lsp1, *kl, *cgr, *ag, *as, *qlt, *dEg, *dEs;
   int32_t* xstar;
   int32_t* yhat;
   float* zpy;
@@ -160,6 +162,7 @@ inline LossWs loss_ws(void* base, const LossLayout& L) {
   w.Mp1 = reinterpret_cast<float*>(b + L.Mp1);
   w.Lsp1 = reinterpret_cast<float*>(b + L.Lsp1);
   w.kl = reinterpret_cast<float*>(b + L.kl);
+  w.cgr = reinterpret_cast<float*>(b + L.cgr);
   w.ag = reinterpret_cast<float*>(b + L.ag);
   w.as = reinterpret_cast<float*>(b + L.as);
   w.qlt = reinterpret_cast<float*>(b + L.qlt);
@@ -229,6 +232,7 @@ struct BackwardArgs {
   float dloss;
   float w_greedy, w_sampling;  // 0 for a term the mode does not select
   float w_kl;                  // 0 without the KL anchor
+  bool grpo;                   // add dloss * cgr[r] (delta_{u,y_r} - q(u)) (the GRPO surrogate)
   const uint8_t* mask;         // [R] position validity (the anchor's rows), or null
   bool q1_is_qT;               // T == 1, sampling and a T = 1 term: q = q~, one exponential
   LossWs ws;
@@ -275,6 +279,70 @@ struct RewardGroupArgs {
   float* advantage;
 };
 
+// GRPO workspace (aal_grpo_from_loss): reward flags and buffers, log pi_ref at the draft's
+// greedy tokens, and block partials of the surrogate sum.
+struct GrpoLayout {
+  int64_t R = 0, N = 0, nroll = 0, nblk = 0;
+  size_t hdr = 0, acc = 0, acc_ref = 0, rbuf = 0, tau = 0, tau_ref = 0, rl = 0, adv = 0, lpr = 0, part = 0;
+  size_t total = 0;
+};
+
+constexpr int kGrpoThreads = 256;
+
+inline GrpoLayout grpo_layout(int64_t N, int64_t K, int64_t wpr) {
+  GrpoLayout L;
+  L.N = N;
+  L.R = N * K;
+  L.nroll = wpr > 0 ? N / wpr : 0;
+  L.nblk = (N + kGrpoThreads - 1) / kGrpoThreads;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    size_t o = off;
+    off = align_up(off + bytes, 256);
+    return o;
+  };
+  L.hdr = take(sizeof(WsHeader));
+  L.acc = take((size_t)L.R);
+  L.acc_ref = take((size_t)L.R);
+  L.rbuf = take((size_t)N * 4);
+  L.tau = take((size_t)N * 4);
+  L.tau_ref = take((size_t)N * 4);
+  L.rl = take((size_t)L.nroll * 4);
+  L.adv = take((size_t)L.nroll * 4);
+  L.lpr = take((size_t)L.R * 4);
+  L.part = take((size_t)(L.nblk > 0 ? L.nblk : 1) * 8);
+  L.total = off;
+  return L;
+}
+
+// Reference-draft pass: per row, log pi_ref at the draft's greedy token y (from the loss
+// workspace) and whether the reference's own greedy token matches x*.
+struct GrpoRefArgs {
+  const void* zr;      // reference draft logits [R][V]
+  int64_t R, V;
+  LossWs lws;          // x*, y of the loss forward
+  uint8_t* acc;        // [R] y == x*
+  uint8_t* acc_ref;    // [R] argmax z_ref == x*
+  float* lpr;          // [R] log pi_ref(y)
+  WsHeader* hdr;       // status word for the streamed pass's bounded waits
+};
+
+// Per window: log rho, the clipped surrogate, its per-row gradient coefficients.
+struct GrpoWindowArgs {
+  LossWs lws;          // Lsq1 (log pi_theta(y) = -ln2 Lsq1), cgr out
+  const float* lpr;
+  const float* adv;    // [N / wpr]
+  int64_t N;
+  int32_t K;
+  int64_t wpr;
+  float eps_clip, rho_min, rho_max, log_rho_clip, w_grpo;
+  float* log_rho;      // [N] or null
+  double* part;        // [nblk]
+  int64_t nblk;
+  WsHeader* hdr;       // of the GRPO workspace (last-block counter)
+  float* loss;         // [1] L_GRPO
+};
+
 // Launchers (return cudaGetLastError() of their launches).
 cudaError_t launch_rowstats(const RowStatsArgs& a, bool bf16, cudaStream_t s, int* cluster_used);
 cudaError_t launch_rowstats_stream(const RowStatsArgs& a, bool bf16, cudaStream_t s, uint64_t limit_ns);
@@ -289,6 +357,8 @@ cudaError_t launch_backward(const BackwardArgs& a, bool bf16, cudaStream_t s);
 cudaError_t launch_reward_rows(const RewardRowArgs& a, bool bf16, cudaStream_t s);
 cudaError_t launch_reward_groups(const RewardGroupArgs& a, cudaStream_t s);
 cudaError_t launch_reward_flags_from_stats(const RewardStatsArgs& a, cudaStream_t s);
+cudaError_t launch_grpo_ref_rows(const GrpoRefArgs& a, bool bf16, cudaStream_t s);
+cudaError_t launch_grpo_windows(const GrpoWindowArgs& a, cudaStream_t s);
 
 // ---------------------------------------------------------------------------
 // Device helpers.

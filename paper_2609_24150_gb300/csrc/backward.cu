@@ -5,11 +5,14 @@
 //   dz_u = g^g a^g (delta_{u,x*} - q(u))                 greedy term, Eq. acc_greedy
 //        + g^s (1/T) q~(u) (c_u - Qlt),  c_u = [q~_u < p~_u]   sampling term, Eq. acc_sample
 //        + c^kl (q(u) - p(u))                                  KL anchor (Sec. 4.1), T = 1
+//        + c^grpo (delta_{u,y} - q(u))                         GRPO surrogate (Sec. 3.4), y = argmax z_q
 // (the softmax Jacobian applied to d a / d q; at a tie q~_u = p~_u the min follows the
 // frozen p~, so c_u = 0).  q(u), q~(u) and c_u are recomputed from the logits and the
 // row's saved log-sum-exps; nothing of size V is materialised.  One pass: reads z_q
 // (and z_p when the sampling term or the anchor is on), writes dz in the logits' dtype.
-// c^kl = dloss w_kl / |positions| on valid positions, 0 elsewhere.
+// c^kl = dloss w_kl / |positions| on valid positions, 0 elsewhere; c^grpo = dloss times the
+// per-row coefficient aal_grpo_from_loss left in the workspace.  The greedy and GRPO terms
+// share q(u), so both run in the GREEDY instantiation.
 #include "aal_internal.cuh"
 
 namespace aal {
@@ -75,11 +78,15 @@ struct RowCoef {
   float Ck;          // c^kl
   float cpos, cneg;  // g^s/T (1 - Qlt) and -g^s/T Qlt
   float Ag;          // g^g a^g
-  int32_t xs;
+  float Cg;          // c^grpo
+  float Aq;          // Ag + Cg, the coefficient of -q(u)
+  int32_t xs, ys;
 };
 
+// Every term of element u except the greedy and GRPO spikes (+Ag at x*, +Cg at y), which
+// the callers add: once per 16-byte vector in the vector path, per element in the scalar one.
 template <bool GREEDY, bool SAMPLING, bool Q1_IS_QT, bool KL>
-__device__ __forceinline__ float grad_elem(const RowCoef& c, float q, float p, int64_t u) {
+__device__ __forceinline__ float grad_elem(const RowCoef& c, float q, float p) {
   float d = 0.f, qt = 0.f;
   if (SAMPLING) {
     const float lq = log2_prob(q, c.sT, c.Mq, c.Lsq);
@@ -89,10 +96,7 @@ __device__ __forceinline__ float grad_elem(const RowCoef& c, float q, float p, i
   }
   if (GREEDY || KL) {
     const float q1 = Q1_IS_QT ? qt : ex2(log2_prob(q, kLog2e, c.Mq1, c.Lsq1));
-    if (GREEDY) {
-      d = fmaf(-c.Ag, q1, d);
-      if (u == c.xs) d += c.Ag;
-    }
+    if (GREEDY) d = fmaf(-c.Aq, q1, d);
     if (KL) d = fmaf(c.Ck, q1 - ex2(log2_prob(p, kLog2e, c.Mp1, c.Lsp1)), d);
   }
   return d;
@@ -107,13 +111,14 @@ __global__ void __launch_bounds__(kBwdThreads) backward_kernel(BackwardArgs a) {
   constexpr bool READ_P = SAMPLING || KL;
   constexpr int E = Io<T>::E;
   for (int64_t r = blockIdx.x; r < a.R; r += gridDim.x) {
-    const float gg = GREEDY ? scale * a.w_greedy * a.ws.dEg[r] : 0.f;
+    const float gg = (GREEDY && a.w_greedy != 0.f) ? scale * a.w_greedy * a.ws.dEg[r] : 0.f;
+    const float cg = (GREEDY && a.grpo) ? a.dloss * a.ws.cgr[r] : 0.f;
     const float gs = SAMPLING ? scale * a.w_sampling * a.ws.dEs[r] : 0.f;
     const float ck = (KL && (a.mask == nullptr || a.mask[r] != 0)) ? kscale : 0.f;
     T* out = static_cast<T*>(a.grad) + r * a.V;
     const T* zq = static_cast<const T*>(a.zq) + r * a.V;
     const T* zp = static_cast<const T*>(a.zp) + r * a.V;
-    if (gg == 0.f && gs == 0.f && ck == 0.f) {
+    if (gg == 0.f && gs == 0.f && ck == 0.f && cg == 0.f) {
       if (VEC) {
         uint4* o4 = reinterpret_cast<uint4*>(out);
         for (int64_t i = threadIdx.x; i < a.V / E; i += kBwdThreads) st_stream(o4 + i, make_uint4(0, 0, 0, 0));
@@ -137,10 +142,16 @@ __global__ void __launch_bounds__(kBwdThreads) backward_kernel(BackwardArgs a) {
     const float Bs = gs * a.invT;
     c.cpos = Bs * (1.f - qlt);
     c.cneg = -Bs * qlt;
-    c.Ag = GREEDY ? gg * a.ws.ag[r] : 0.f;
-    c.xs = GREEDY ? a.ws.xstar[r] : -1;
+    c.Ag = gg != 0.f ? gg * a.ws.ag[r] : 0.f;
+    c.Cg = cg;
+    c.Aq = c.Ag + c.Cg;
+    c.xs = gg != 0.f ? a.ws.xstar[r] : -1;
+    c.ys = cg != 0.f ? a.ws.yhat[r] : -1;
     if (VEC) {
       const int64_t nv = a.V / E;
+      // the vectors and lanes of the spikes (-1: none)
+      const int64_t xv = c.xs >= 0 ? c.xs / E : -1, yv = c.ys >= 0 ? c.ys / E : -1;
+      const int xe = c.xs >= 0 ? c.xs % E : 0, ye = c.ys >= 0 ? c.ys % E : 0;
       const uint4* q4 = reinterpret_cast<const uint4*>(zq);
       const uint4* p4 = reinterpret_cast<const uint4*>(zp);
       uint4* o4 = reinterpret_cast<uint4*>(out);
@@ -149,15 +160,31 @@ __global__ void __launch_bounds__(kBwdThreads) backward_kernel(BackwardArgs a) {
         Io<T>::unpack(ldg_stream(q4 + i), qv);
         if (READ_P) Io<T>::unpack(ldg_stream(p4 + i), pv);
 #pragma unroll
-        for (int e = 0; e < E; ++e)
-          d[e] = grad_elem<GREEDY, SAMPLING, Q1_IS_QT, KL>(c, qv[e], READ_P ? pv[e] : 0.f, i * E + e);
+        for (int e = 0; e < E; ++e) d[e] = grad_elem<GREEDY, SAMPLING, Q1_IS_QT, KL>(c, qv[e], READ_P ? pv[e] : 0.f);
+        if (GREEDY) {  // the spikes, tested once per vector
+          if (i == xv) {
+#pragma unroll
+            for (int e = 0; e < E; ++e)
+              if (e == xe) d[e] += c.Ag;
+          }
+          if (i == yv) {
+#pragma unroll
+            for (int e = 0; e < E; ++e)
+              if (e == ye) d[e] += c.Cg;
+          }
+        }
         st_stream(o4 + i, Io<T>::pack(d));
       }
     } else {
       for (int64_t v = threadIdx.x; v < a.V; v += kBwdThreads) {
         const float q = load_elem<T>(zq + v);
         const float p = READ_P ? load_elem<T>(zp + v) : 0.f;
-        Io<T>::store1(out + v, grad_elem<GREEDY, SAMPLING, Q1_IS_QT, KL>(c, q, p, v));
+        float d = grad_elem<GREEDY, SAMPLING, Q1_IS_QT, KL>(c, q, p);
+        if (GREEDY) {
+          if (v == c.xs) d += c.Ag;
+          if (v == c.ys) d += c.Cg;
+        }
+        Io<T>::store1(out + v, d);
       }
     }
   }
@@ -179,7 +206,7 @@ cudaError_t go(const BackwardArgs& a, cudaStream_t s) {
 
 template <typename T, bool VEC, bool KL>
 cudaError_t dispatch_mode(const BackwardArgs& a, cudaStream_t s) {
-  const bool G = a.w_greedy != 0.f, S = a.w_sampling != 0.f;
+  const bool G = a.w_greedy != 0.f || a.grpo, S = a.w_sampling != 0.f;
   const bool Q = a.q1_is_qT && S && (G || KL);
   if (G && S) return Q ? go<T, VEC, true, true, true, KL>(a, s) : go<T, VEC, true, true, false, KL>(a, s);
   if (G) return go<T, VEC, true, false, false, KL>(a, s);

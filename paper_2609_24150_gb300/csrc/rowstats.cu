@@ -245,14 +245,16 @@ cudaError_t launch_generic(const RowStatsArgs& a, cudaStream_t s) {
 
 }  // namespace
 
-// The TMA-streamed kernel (rowstats_stream.cu) serves rows whose byte length is a
-// multiple of 16 when the sampling term needs the second pass and the KL anchor is off;
-// everything else takes the generic kernel.
+// The TMA-streamed kernel (rowstats_stream.cu) serves rows whose byte length is a multiple
+// of 16: in two passes with the sampling term, in one pass without it.  Unaligned rows, and
+// the KL anchor next to a sampling term at T != 1, take the generic kernel.
 cudaError_t launch_rowstats(const RowStatsArgs& a, bool bf16, cudaStream_t s, int* cluster_used) {
   const int elt = bf16 ? 2 : 4;
   const bool aligned = ((a.V * elt) % 16 == 0) &&
                        ((reinterpret_cast<uintptr_t>(a.zq) | reinterpret_cast<uintptr_t>(a.zp)) % 16 == 0);
-  if (a.overlap && aligned && !a.need_kl) {
+  // the streamed kernel takes the KL anchor only where the z_p normaliser it keeps is at T = 1
+  const bool kl_ok = !a.need_kl || !a.overlap || a.sT == kLog2e;
+  if (aligned && kl_ok) {
     *cluster_used = 1;
     const uint64_t limit = debug_wait_limit_ns();
     return launch_rowstats_stream(a, bf16, s, limit ? limit : kWaitLimitNs);

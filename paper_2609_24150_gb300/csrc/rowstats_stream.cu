@@ -16,6 +16,13 @@
 //     state, reduce it across the CTA at the end of the row, then fold each second-pass
 //     chunk into the overlap sums.  The producer keeps streaming through that reduction.
 //
+// Problems without the sampling term (greedy EAL, the KL anchor, the GRPO statistics) need
+// neither the second pass nor a temperature: they run the same kernel with one pass at T = 1,
+// where the normalisers of z_p and z_q are those of p and q themselves.  The first pass
+// finds the argmaxes only to the 16-byte vector; resolve_argmax then reads those two
+// vectors of each row again (64 bytes) to place x* and y exactly.  With the KL anchor the
+// first pass also folds D = sum_v e_v (z_p,v - z_q,v) next to the log-sum-exp of z_p.
+//
 // There is no cross-CTA communication, so all 152 SMs run one CTA each.  Every wait is
 // bounded (ptx::wait_phase); after a timeout every thread keeps walking the same loops
 // without waiting or computing, so all meet the same named barriers, the producer drains
@@ -54,6 +61,7 @@ constexpr int kBarRow = 1, kBarSum = 2;
 // found in the second pass, by the one thread that streams the vector again.
 struct RowPart {
   float pM, pS, qM, qS, q1M, q1S;  // online log2-sum-exp states (M = raw max of z)
+  float pD;                        // KL anchor: sum 2^((z_p - pM) s) (z_p - z_q), rescaled with pS
   float av;                        // target: largest z_p and the first vector holding it
   int32_t ab;
   float qv;                        // draft: largest z_q and the first vector holding it
@@ -63,7 +71,7 @@ struct RowPart {
 struct Smem {
   uint64_t full[kSlots];
   uint64_t empty[kSlots];
-  RowPart red[kWarps];
+  RowPart red[2][kWarps];  // by row parity
   float2 red2[2][kWarps];
   int32_t arg_index;  // x*, written by the thread that finds it in the second pass
   float arg_carry;    // z_q at x*
@@ -79,6 +87,7 @@ constexpr float kMaxFloor = -1e30f;
 __device__ __forceinline__ void part_init(RowPart& a) {
   a.pM = a.qM = a.q1M = kMaxFloor;
   a.pS = a.qS = a.q1S = 0.f;
+  a.pD = 0.f;
   a.av = -INFINITY;
   a.ab = 0x7fffffff;
   a.qv = -INFINITY;
@@ -107,9 +116,26 @@ __device__ __forceinline__ void warp_amax(float& v, int32_t& i) {
     }
   }
 }
-template <bool NEED_Q1>
+// (M, S, D): D rescales with S.
+__device__ __forceinline__ void warp_lse_kl(float& M, float& S, float& D, float scale) {
+  float m = M;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
+  const float r = ex2((M - m) * scale);
+  float s = S * r, d = D * r;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    s += __shfl_xor_sync(0xffffffffu, s, off);
+    d += __shfl_xor_sync(0xffffffffu, d, off);
+  }
+  M = m;
+  S = s;
+  D = d;
+}
+template <bool NEED_Q1, bool KL = false>
 __device__ __forceinline__ void warp_part(RowPart& a, float sT) {
-  warp_lse(a.pM, a.pS, sT);
+  if (KL) warp_lse_kl(a.pM, a.pS, a.pD, sT);
+  else warp_lse(a.pM, a.pS, sT);
   warp_lse(a.qM, a.qS, sT);
   if (NEED_Q1) warp_lse(a.q1M, a.q1S, kLog2e);
   warp_amax(a.av, a.ab);
@@ -146,9 +172,34 @@ __device__ __forceinline__ void lse_words(float& M, float& S, const uint32_t* w,
   S += t.x + t.y;
 }
 
+// lse_words for z_p with the KL sum: D += 2^((z_p - M) s) (z_p - z_q), rescaled with S.
+template <int NW>
+__device__ __forceinline__ void lse_kl_words(float& M, float& S, float& D, const uint32_t* pw,
+                                             const uint32_t* qw, float vmax, float s) {
+  const float m = fmaxf(M, vmax);
+  const float r = ex2((M - m) * s);
+  S *= r;
+  D *= r;
+  M = m;
+  const float nM = -M;
+  const float2 s2 = make_float2(s, s), zero2 = make_float2(0.f, 0.f);
+  float2 acc = zero2, dacc = zero2;
+#pragma unroll
+  for (int k = 0; k < NW; ++k) {
+    const float2 x = f2fma(make_float2(bf16lo_add(pw[k], nM), bf16hi_add(pw[k], nM)), s2, zero2);
+    const float2 e = make_float2(ex2(x.x), ex2(x.y));
+    acc = f2add(acc, e);
+    // z_p - z_q: the draft value widened, the target's bf16 widened inside the add
+    const float2 d = make_float2(bf16lo_add(pw[k], -bf16_lo(qw[k])), bf16hi_add(pw[k], -bf16_hi(qw[k])));
+    dacc = f2fma(e, d, dacc);
+  }
+  S += acc.x + acc.y;
+  D += dacc.x + dacc.y;
+}
+
 // Phase 1 on NV 16-byte vectors of bf16 per tensor; vector v holds elements
 // idx0 + v * vstride + [0, 8).
-template <int NV, bool NEED_Q1>
+template <int NV, bool NEED_Q1, bool KL = false>
 __device__ __forceinline__ void phase1_bf16(RowPart& A, const uint4* pv, const uint4* qv, int idx0, int vstride,
                                             float sT) {
   constexpr int NW = 4 * NV;
@@ -175,7 +226,8 @@ __device__ __forceinline__ void phase1_bf16(RowPart& A, const uint4* pv, const u
     pm = fmaxf(pm, vp);
     qm = fmaxf(qm, vq);
   }
-  lse_words<NW>(A.pM, A.pS, pw, pm, sT);
+  if (KL) lse_kl_words<NW>(A.pM, A.pS, A.pD, pw, qw, pm, sT);
+  else lse_words<NW>(A.pM, A.pS, pw, pm, sT);
   lse_words<NW>(A.qM, A.qS, qw, qm, sT);
   if (NEED_Q1) lse_words<NW>(A.q1M, A.q1S, qw, qm, kLog2e);
 }
@@ -256,7 +308,26 @@ __device__ __forceinline__ void lse_vals(float& M, float& S, const float* v, flo
   S += acc;
 }
 
-template <typename T, bool NEED_Q1>
+template <int N>
+__device__ __forceinline__ void lse_kl_vals(float& M, float& S, float& D, const float* p, const float* q,
+                                            float vmax, float s) {
+  const float m = fmaxf(M, vmax);
+  const float r = ex2((M - m) * s);
+  S *= r;
+  D *= r;
+  M = m;
+  float acc = 0.f, dacc = 0.f;
+#pragma unroll
+  for (int e = 0; e < N; ++e) {
+    const float x = ex2((p[e] - M) * s);
+    acc += x;
+    dacc = fmaf(x, p[e] - q[e], dacc);
+  }
+  S += acc;
+  D += dacc;
+}
+
+template <typename T, bool NEED_Q1, bool KL = false>
 __device__ __forceinline__ void phase1_vec(RowPart& A, const uint4& pw, const uint4& qw, int idx0, float sT) {
   constexpr int E = 16 / sizeof(T);
   float pv[8], qv[8];
@@ -270,7 +341,8 @@ __device__ __forceinline__ void phase1_vec(RowPart& A, const uint4& pw, const ui
   }
   amax_vec(A.av, A.ab, pm, idx0);
   amax_vec(A.qv, A.qb, qm, idx0);
-  lse_vals<E>(A.pM, A.pS, pv, pm, sT);
+  if (KL) lse_kl_vals<E>(A.pM, A.pS, A.pD, pv, qv, pm, sT);
+  else lse_vals<E>(A.pM, A.pS, pv, pm, sT);
   lse_vals<E>(A.qM, A.qS, qv, qm, sT);
   if (NEED_Q1) lse_vals<E>(A.q1M, A.q1S, qv, qm, kLog2e);
 }
@@ -304,7 +376,10 @@ struct RingPos {
 
 // ---------------------------------------------------------------- the kernel
 
-template <typename T, bool NEED_Q1>
+// PASSES = 2: the sampling term (normalisers at T, then the overlap sums).  PASSES = 1: no
+// sampling term; everything at T = 1 (sT is log2 e), argmaxes resolved by resolve_argmax.
+// KL: the anchor's D next to the z_p normaliser (which must then be at T = 1).
+template <typename T, bool NEED_Q1, int PASSES, bool KL>
 __global__ void __launch_bounds__(kThreads, 1) rowstats_stream(RowStatsArgs a, int nch, uint64_t limit_ns) {
   extern __shared__ __align__(1024) unsigned char smem[];
   unsigned char* ring = smem;
@@ -343,8 +418,8 @@ __global__ void __launch_bounds__(kThreads, 1) rowstats_stream(RowStatsArgs a, i
       for (int64_t r = blockIdx.x; r < a.R && !*abort_flag; r += gridDim.x) {
         const char* prow = static_cast<const char*>(a.zp) + r * a.V * ES;
         const char* qrow = static_cast<const char*>(a.zq) + r * a.V * ES;
-        for (int pass = 0; pass < 2 && !*abort_flag; ++pass) {
-          const uint64_t pol = pass == 0 ? keep : drop;
+        for (int pass = 0; pass < PASSES && !*abort_flag; ++pass) {
+          const uint64_t pol = (pass == 0 && PASSES == 2) ? keep : drop;
           for (int c = 0; c < nch; ++c) {
             if (!wait_phase(&S.empty[pos.slot], pos.phase ^ 1u, abort_flag, limit_ns, hdr)) break;
             const int e0 = c * CH;
@@ -376,6 +451,7 @@ __global__ void __launch_bounds__(kThreads, 1) rowstats_stream(RowStatsArgs a, i
     const int t = threadIdx.x;
     RingPos pos;
     uint32_t j = 0;
+    const float sT = PASSES == 2 ? a.sT : kLog2e;
     for (int64_t r = blockIdx.x; r < a.R; r += gridDim.x, ++j) {
       // pass 1: online normalisers and argmax
       RowPart A;
@@ -392,25 +468,50 @@ __global__ void __launch_bounds__(kThreads, 1) rowstats_stream(RowStatsArgs a, i
               pv[v] = P[t + v * kConsumers];
               qv[v] = Q[t + v * kConsumers];
             }
-            phase1_bf16<kNV, NEED_Q1>(A, pv, qv, e0 + t * E, kConsumers * E, a.sT);
+            phase1_bf16<kNV, NEED_Q1, KL>(A, pv, qv, e0 + t * E, kConsumers * E, sT);
           } else {
             const int nvec = min(CH, V - e0) / E;
-            for (int i = t; i < nvec; i += kConsumers) phase1_vec<T, NEED_Q1>(A, P[i], Q[i], e0 + i * E, a.sT);
+            for (int i = t; i < nvec; i += kConsumers) phase1_vec<T, NEED_Q1, KL>(A, P[i], Q[i], e0 + i * E, sT);
           }
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&S.empty[pos.slot]);
       }
-      warp_part<NEED_Q1>(A, a.sT);
-      if (lane == 0) S.red[warp] = A;
+      warp_part<NEED_Q1, KL>(A, sT);
+      if (lane == 0) S.red[j & 1][warp] = A;
       named_barrier(kBarRow, kConsumers);
       // every warp combines the warp partials itself (lanes >= kWarps carry the identity)
       RowPart tot;
-      if (lane < kWarps) tot = S.red[lane];
+      if (lane < kWarps) tot = S.red[j & 1][lane];
       else part_init(tot);
-      warp_part<NEED_Q1>(tot, a.sT);
+      warp_part<NEED_Q1, KL>(tot, sT);
       const float Mp = tot.pM, Lsp = log2f(tot.pS);
       const float Mq = tot.qM, Lsq = log2f(tot.qS);
+      if (KL && t == 0 && !*abort_flag) {  // both normalisers are at T = 1 here
+        const float Mq1 = NEED_Q1 ? tot.q1M : Mq;
+        const float Lsq1 = NEED_Q1 ? log2f(tot.q1S) : Lsq;
+        a.ws.Mp1[r] = Mp;
+        a.ws.Lsp1[r] = Lsp;
+        a.ws.kl[r] = tot.pD / tot.pS - (Mp - Mq1) - kLn2 * (Lsp - Lsq1);
+      }
+      if (PASSES == 1) {
+        if (t == 0) {
+          if (!*abort_flag) {
+            a.ws.Mp[r] = Mp;
+            a.ws.Lsp[r] = Lsp;
+            a.ws.Mq[r] = Mq;
+            a.ws.Lsq[r] = Lsq;
+            a.ws.Mq1[r] = Mq;
+            a.ws.Lsq1[r] = Lsq;
+            a.ws.cpart[r * kMaxCluster] = make_float2(0.f, 0.f);
+          }
+          // the first vector holding each maximum, which resolve_argmax turns into the element;
+          // -1 (no vector) after an abort, so that it reads nothing
+          a.ws.xstar[r] = *abort_flag ? -1 : tot.ab;
+          a.ws.yhat[r] = *abort_flag ? -1 : tot.qb;
+        }
+        continue;
+      }
 
       // pass 2: overlap sums
       float smin = 0.f, sqlt = 0.f;
@@ -499,9 +600,9 @@ __global__ void __launch_bounds__(kThreads, 1) rowstats_stream(RowStatsArgs a, i
 
 constexpr size_t kSmemBytes = (size_t)kSlots * kSlotBytes + sizeof(Smem);
 
-template <typename T, bool NEED_Q1>
+template <typename T, bool NEED_Q1, int PASSES, bool KL>
 cudaError_t launch_T(const RowStatsArgs& a, cudaStream_t s, int nch, uint64_t limit_ns) {
-  auto kern = rowstats_stream<T, NEED_Q1>;
+  auto kern = rowstats_stream<T, NEED_Q1, PASSES, KL>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
   if (e != cudaSuccess) return e;
   int dev = 0, sms = 0;
@@ -514,14 +615,77 @@ cudaError_t launch_T(const RowStatsArgs& a, cudaStream_t s, int nch, uint64_t li
   return cudaGetLastError();
 }
 
+// One thread per row: the first element equal to the row maximum inside the vector the
+// one-pass kernel recorded (x* for z_p, y for z_q), the other tensor's value there, and
+// a^greedy = q(x*).
+template <typename T>
+__global__ void __launch_bounds__(256) resolve_argmax(RowStatsArgs a) {
+  const int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= a.R) return;
+  constexpr int E = 16 / sizeof(T);
+  const T* zp = static_cast<const T*>(a.zp) + r * a.V;
+  const T* zq = static_cast<const T*>(a.zq) + r * a.V;
+  const int32_t xb = a.ws.xstar[r], yb = a.ws.yhat[r];
+  int32_t xs = 0, ys = 0;
+  float cx = 0.f, cy = 0.f;
+  // a vector is read only at an in-range, vector-aligned start (an all -inf row, or a row
+  // of an aborted launch, records none)
+  if (xb >= 0 && xb % E == 0 && (int64_t)xb + E <= a.V) {
+    const uint4 pw = *reinterpret_cast<const uint4*>(zp + xb), qw = *reinterpret_cast<const uint4*>(zq + xb);
+    float pv[8], qv[8];
+    unpack_vec<T>(pw, pv);
+    unpack_vec<T>(qw, qv);
+    float m = pv[0];
+    for (int e = 1; e < E; ++e) m = fmaxf(m, pv[e]);
+    int at = 0;
+    for (int e = E - 1; e >= 0; --e)
+      if (pv[e] == m) at = e;
+    xs = xb + at;
+    cx = qv[at];
+  }
+  if (yb >= 0 && yb % E == 0 && (int64_t)yb + E <= a.V) {
+    const uint4 pw = *reinterpret_cast<const uint4*>(zp + yb), qw = *reinterpret_cast<const uint4*>(zq + yb);
+    float pv[8], qv[8];
+    unpack_vec<T>(pw, pv);
+    unpack_vec<T>(qw, qv);
+    float m = qv[0];
+    for (int e = 1; e < E; ++e) m = fmaxf(m, qv[e]);
+    int at = 0;
+    for (int e = E - 1; e >= 0; --e)
+      if (qv[e] == m) at = e;
+    ys = yb + at;
+    cy = pv[at];
+  }
+  a.ws.xstar[r] = xs;
+  a.ws.yhat[r] = ys;
+  a.ws.zpy[r] = cy;
+  a.ws.ag[r] = exp2f(log2_prob(cx, kLog2e, a.ws.Mq1[r], a.ws.Lsq1[r]));
+}
+
+template <typename T>
+cudaError_t launch_one_pass(const RowStatsArgs& a, cudaStream_t s, int nch, uint64_t limit_ns) {
+  cudaError_t e = a.need_kl ? launch_T<T, false, 1, true>(a, s, nch, limit_ns)
+                            : launch_T<T, false, 1, false>(a, s, nch, limit_ns);
+  if (e != cudaSuccess) return e;
+  if (a.R < 1) return cudaSuccess;
+  resolve_argmax<T><<<(unsigned)((a.R + 255) / 256), 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+template <typename T>
+cudaError_t launch_two_pass(const RowStatsArgs& a, cudaStream_t s, int nch, uint64_t limit_ns) {
+  if (a.need_kl) return launch_T<T, false, 2, true>(a, s, nch, limit_ns);  // T = 1: no separate q1
+  return a.need_q1 ? launch_T<T, true, 2, false>(a, s, nch, limit_ns) : launch_T<T, false, 2, false>(a, s, nch, limit_ns);
+}
+
 }  // namespace
 
 cudaError_t launch_rowstats_stream(const RowStatsArgs& a, bool bf16, cudaStream_t s, uint64_t limit_ns) {
   const int elt = bf16 ? 2 : 4;
   const int64_t CH = kHalfSlot / elt;
   const int nch = (int)((a.V + CH - 1) / CH);
-  if (bf16) return a.need_q1 ? launch_T<uint16_t, true>(a, s, nch, limit_ns) : launch_T<uint16_t, false>(a, s, nch, limit_ns);
-  return a.need_q1 ? launch_T<float, true>(a, s, nch, limit_ns) : launch_T<float, false>(a, s, nch, limit_ns);
+  if (!a.overlap) return bf16 ? launch_one_pass<uint16_t>(a, s, nch, limit_ns) : launch_one_pass<float>(a, s, nch, limit_ns);
+  return bf16 ? launch_two_pass<uint16_t>(a, s, nch, limit_ns) : launch_two_pass<float>(a, s, nch, limit_ns);
 }
 
 }  // namespace aal

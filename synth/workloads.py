@@ -212,13 +212,16 @@ def make_logits(name: str, seed: int = 0, device="cpu", n_windows: Optional[int]
 def make_reward_logits(group: int, seed: int = 0, device="cpu", with_ref: bool = False,
                        windows_per_rollout: Optional[int] = None,
                        rollouts_per_group: Optional[int] = None, K: Optional[int] = None,
-                       V: Optional[int] = None, dtype: Optional[torch.dtype] = None):
+                       V: Optional[int] = None, dtype: Optional[torch.dtype] = None,
+                       ref_from_draft: Optional[float] = None):
     """Draw one prompt group of the reward workload: (target, draft, ref_draft | None).
 
     Rows are [rollouts_per_group * windows_per_rollout][K][V]; the group is drawn
     from its own generator seeded by (seed, group), so groups can be streamed one
     at a time. ``ref_draft`` (a frozen earlier draft) is the target plus its own
-    independent N(0, 1) noise.
+    independent N(0, 1) noise, or, with ``ref_from_draft = s``, the draft plus N(0, s^2)
+    noise: a snapshot of the draft a little way back in training, as the GRPO stage's
+    reference policy is.
     """
     wpr = REWARD["windows_per_rollout"] if windows_per_rollout is None else windows_per_rollout
     rpg = REWARD["rollouts_per_group"] if rollouts_per_group is None else rollouts_per_group
@@ -238,8 +241,14 @@ def make_reward_logits(group: int, seed: int = 0, device="cpu", with_ref: bool =
         draft[n0:n1].copy_((zp + torch.randn((rows, V), generator=g, device=device))
                            .view(n1 - n0, K, V))
         if with_ref:
-            ref[n0:n1].copy_((zp + torch.randn((rows, V), generator=g, device=device))
-                             .view(n1 - n0, K, V))
+            if ref_from_draft is None:
+                ref[n0:n1].copy_((zp + torch.randn((rows, V), generator=g, device=device))
+                                 .view(n1 - n0, K, V))
+            else:
+                zq = draft[n0:n1].view(rows, V).float()
+                ref[n0:n1].copy_((zq + ref_from_draft * torch.randn((rows, V), generator=g, device=device))
+                                 .view(n1 - n0, K, V))
+                del zq
         del zp
     return target, draft, ref
 

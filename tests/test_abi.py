@@ -73,7 +73,8 @@ def test_workspace_size_grows_with_rows():
     (dict(N=-1), aal.AAL_ERR_INVALID_ARG),
     (dict(dtype=7), aal.AAL_ERR_INVALID_ARG),
     (dict(mode=0), aal.AAL_ERR_INVALID_ARG),
-    (dict(mode=8), aal.AAL_ERR_INVALID_ARG),
+    (dict(mode=16), aal.AAL_ERR_INVALID_ARG),
+    (dict(mode=aal.AAL_GRPO | aal.AAL_KL | aal.AAL_GREEDY), aal.AAL_OK),
     (dict(mode=-1), aal.AAL_ERR_INVALID_ARG),
     (dict(w_kl=float("nan")), aal.AAL_ERR_INVALID_ARG),
     (dict(temperature=0.0), aal.AAL_ERR_INVALID_ARG),
@@ -221,3 +222,56 @@ def test_seq_pointer_checks_before_launch():
     assert lib.aal_seq_loss_bwd(ctypes.byref(p), fake, fake, None, fake_ws, size, 1.0, None, None) == aal.AAL_ERR_INVALID_ARG
     assert lib.aal_seq_loss_bwd(ctypes.byref(p), fake, fake, None, fake_ws, size, float("inf"), fake, None) == aal.AAL_ERR_INVALID_ARG
     assert lib.aal_seq_loss_bwd(ctypes.byref(p), fake, fake, None, fake_ws + 128, size, 1.0, fake, None) == aal.AAL_ERR_WORKSPACE
+
+
+def _gprob(**kw):
+    d = dict(N=8, K=4, V=100, dtype=aal.AAL_BF16, reserved=0, windows_per_rollout=1, rollouts_per_group=4,
+             adv_clip=5.0, eps_clip=0.2, rho_min=0.0, rho_max=10.0, log_rho_clip=10.0, w_grpo=0.1)
+    d.update(kw)
+    return aal.AalGrpoProblem(**d)
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(), aal.AAL_OK),
+    (dict(rollouts_per_group=3), aal.AAL_ERR_INVALID_ARG),      # 8 windows not a multiple of 3
+    (dict(eps_clip=1.0), aal.AAL_ERR_INVALID_ARG),
+    (dict(eps_clip=-0.1), aal.AAL_ERR_INVALID_ARG),
+    (dict(rho_min=2.0, rho_max=1.0), aal.AAL_ERR_INVALID_ARG),
+    (dict(rho_min=-1.0), aal.AAL_ERR_INVALID_ARG),
+    (dict(rho_max=float("inf")), aal.AAL_ERR_INVALID_ARG),
+    (dict(log_rho_clip=0.0), aal.AAL_ERR_INVALID_ARG),
+    (dict(w_grpo=float("nan")), aal.AAL_ERR_INVALID_ARG),
+    (dict(adv_clip=0.0), aal.AAL_ERR_INVALID_ARG),
+    (dict(reserved=1), aal.AAL_ERR_INVALID_ARG),
+    (dict(K=9), aal.AAL_ERR_UNSUPPORTED),
+])
+def test_grpo_problem_checks(kw, code):
+    out = ctypes.c_size_t(0)
+    p = _gprob(**kw)
+    assert aal.library().aal_grpo_workspace_size(ctypes.byref(p), ctypes.byref(out)) == code
+
+
+def test_grpo_needs_a_matching_loss_problem_with_the_grpo_bit():
+    lib = aal.library()
+    g = _gprob()
+    fake, fake_ws = 1 << 24, 1 << 20
+    big = 1 << 30
+    lp = _prob(N=8, K=4, mode=aal.AAL_GREEDY)                       # no AAL_GRPO bit
+    assert lib.aal_grpo_from_loss(ctypes.byref(g), ctypes.byref(lp), fake_ws, big, fake, fake_ws, big,
+                                  fake, None, None, None, None, None) == aal.AAL_ERR_INVALID_ARG
+    lp = _prob(N=8, K=3, mode=aal.AAL_GREEDY | aal.AAL_GRPO)        # shape differs
+    assert lib.aal_grpo_from_loss(ctypes.byref(g), ctypes.byref(lp), fake_ws, big, fake, fake_ws, big,
+                                  fake, None, None, None, None, None) == aal.AAL_ERR_INVALID_ARG
+    lp = _prob(N=8, K=4, mode=aal.AAL_GREEDY | aal.AAL_GRPO)
+    assert lib.aal_grpo_from_loss(ctypes.byref(g), ctypes.byref(lp), fake_ws, big, None, fake_ws, big,
+                                  fake, None, None, None, None, None) == aal.AAL_ERR_INVALID_ARG
+    assert lib.aal_grpo_from_loss(ctypes.byref(g), ctypes.byref(lp), fake_ws, big, fake, fake_ws, big,
+                                  None, None, None, None, None, None) == aal.AAL_ERR_INVALID_ARG
+    assert lib.aal_grpo_from_loss(ctypes.byref(g), ctypes.byref(lp), fake_ws, 16, fake, fake_ws, big,
+                                  fake, None, None, None, None, None) == aal.AAL_ERR_WORKSPACE
+    assert lib.aal_grpo_from_loss(ctypes.byref(g), ctypes.byref(lp), fake_ws, big, fake, fake_ws, 16,
+                                  fake, None, None, None, None, None) == aal.AAL_ERR_WORKSPACE
+
+
+def test_sequence_layout_refuses_the_grpo_bit():
+    assert _seq_ws(_sprob(mode=aal.AAL_GREEDY | aal.AAL_GRPO))[0] == aal.AAL_ERR_UNSUPPORTED

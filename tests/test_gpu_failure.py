@@ -14,11 +14,14 @@ pytestmark = pytest.mark.gpu
 DEV = "cuda:0"
 
 
-@pytest.mark.parametrize("chunk", [0, 1, 3])
-def test_bounded_wait_times_out_and_context_stays_usable(chunk):
+# 32 rows of V = 20000 bf16 (two ring chunks per pass), fewer rows than CTAs: each CTA
+# streams one row, chunks 0-1 in the first pass and 2-3 in the second (two-pass modes only)
+@pytest.mark.parametrize("mode,chunk", [(aal.AAL_BOTH, 0), (aal.AAL_BOTH, 1), (aal.AAL_BOTH, 3),
+                                        (aal.AAL_KL | aal.AAL_GREEDY, 0), (aal.AAL_KL | aal.AAL_GREEDY, 1)])
+def test_bounded_wait_times_out_and_context_stays_usable(mode, chunk):
     target, draft, _ = synth.make_logits("tiny", seed=11, N=16, K=2, V=20000, dtype=torch.bfloat16)
     t, d = target.to(DEV), draft.to(DEV)
-    prob = aal.loss_problem(d, aal.AAL_BOTH, 1.0, 0.5, 0.5)
+    prob = aal.loss_problem(d, mode, 1.0, 0.5, 0.5)
     ws = torch.empty(aal.aal_workspace_size(prob), dtype=torch.uint8, device=DEV)
     loss = torch.empty(1, device=DEV)
     aal.aal_debug_fail_next_forward(chunk, 50_000_000)        # waits give up after 50 ms
@@ -29,5 +32,5 @@ def test_bounded_wait_times_out_and_context_stays_usable(chunk):
     finally:
         aal.aal_debug_fail_next_forward(-1, 0)                # default limit again
     # the same context runs the next forward and backward correctly
-    run = LossRun(t, d, None, aal.AAL_BOTH, 1.0, 0.5, 0.5, dloss=16.0)
-    check_loss(run, t, d, None, aal.AAL_BOTH, 1.0, 0.5, 0.5, dloss=16.0)
+    run = LossRun(t, d, None, mode, 1.0, 0.5, 0.5, dloss=32.0)
+    check_loss(run, t, d, None, mode, 1.0, 0.5, 0.5, dloss=32.0)

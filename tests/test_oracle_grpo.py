@@ -127,3 +127,23 @@ def test_gradient_by_finite_differences(wpr, rpg, eps):
                     - grpo_forward(tgt, b, rf, wpr, rpg, eps_clip=eps)["loss"]) / (2 * h)
         assert abs(fd - g[idx]) < 1e-8, (idx, fd, g[idx])
     assert np.any(g != 0)
+
+
+def test_a_slice_with_the_batch_advantages_gives_its_rows():
+    """The full-size GPU test checks sampled windows against the oracle run on those windows
+    alone, given the whole batch's advantages and N: their gradient rows are unchanged."""
+    rng = np.random.default_rng(11)
+    N, K, V = 8, 2, 5
+    tgt = rng.normal(0, 2, size=(N, K, V))
+    dr = tgt + rng.normal(0, 1.5, size=(N, K, V))
+    rf = tgt + rng.normal(0, 1.5, size=(N, K, V))
+    full = grpo_forward(tgt, dr, rf, 1, 4)
+    g = grpo_backward(tgt, dr, rf, 1, 4, dloss=3.0)
+    sel = [1, 5, 6]
+    fs = grpo_forward(tgt[sel], dr[sel], rf[sel], 1, 4, advantage_window=full["advantage_window"][sel],
+                      n_windows_total=N)
+    gs = grpo_backward(tgt[sel], dr[sel], rf[sel], 1, 4, dloss=3.0,
+                       advantage_window=full["advantage_window"][sel], n_windows_total=N)
+    np.testing.assert_allclose(gs, g[sel], rtol=0, atol=1e-16)
+    np.testing.assert_allclose(fs["rho"], full["rho"][sel], rtol=0, atol=0)
+    assert abs(fs["loss"] - (-np.sum(full["surrogate"][sel]) / N)) < 1e-16
