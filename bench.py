@@ -54,7 +54,9 @@ def parse():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--no-seq", action="store_true", help="skip the sequence-layout measurement")
+    ap.add_argument("--no-seq", action="store_true", help="skip every line beside the step")
+    ap.add_argument("--lines", default="greedy,seq,grpo",
+                    help="lines measured beside the step (comma-separated from greedy, seq, grpo)")
     ap.add_argument("--windows", type=int, default=None,
                     help="run the first WINDOWS windows of the workload (profiling captures)")
     return ap.parse_args()
@@ -233,10 +235,11 @@ def run_ours(args, ws_count, rank, local):
     torch.cuda.synchronize()
     ms_reward_pass = r0.elapsed_time(r1) / reps
 
-    greedy_obj = None if args.no_seq else run_greedy_objective(aal, draft, target, grad, stream,
-                                                                max(5, args.steps // 2))
-    seq = None if args.no_seq else run_sequence_layout(aal, dev, stream, rank, max(5, args.steps // 2))
-    grpo = None if args.no_seq else run_grpo_phase(aal, dev, stream, rank, max(5, args.steps // 2))
+    lines = set() if args.no_seq else {x.strip() for x in args.lines.split(",") if x.strip()}
+    reps = max(5, args.steps // 2)
+    greedy_obj = run_greedy_objective(aal, draft, target, grad, stream, reps) if "greedy" in lines else None
+    seq = run_sequence_layout(aal, dev, stream, rank, reps) if "seq" in lines else None
+    grpo = run_grpo_phase(aal, dev, stream, rank, reps) if "grpo" in lines else None
 
     b = algo_bytes(N, K, V)
     step_bytes = sum(b.values())
