@@ -59,9 +59,13 @@ from .sequence import (  # noqa: F401
 from .grpo import grpo_backward, grpo_forward, policy_log_ratio, trajectory_log_probs  # noqa: F401
 from .anchor import (  # noqa: F401
     MODE_KL,
+    MODE_TV,
     anchor_backward,
     anchor_forward,
     kl_divergence,
     objective_backward,
     objective_forward,
+    total_variation,
+    tv_backward,
+    tv_forward,
 )

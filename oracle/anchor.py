@@ -70,22 +70,86 @@ def anchor_backward(target, draft, mask=None, dloss: float = 1.0, n_positions_to
 
 def objective_forward(target, draft, mask=None, mode: int = MODE_KL | 1, T: float = 1.0,
                       w_greedy: float = 1.0, w_sampling: float = 1.0, w_kl: float = 1.0,
-                      n_windows_total=None, n_positions_total=None):
-    """w_kl L_KL + w_g L_EAL + w_s L_WTV over [N][K][V] windows (terms selected by ``mode``)."""
+                      n_windows_total=None, n_positions_total=None, w_tv: float = 1.0):
+    """w_kl L_KL + w_g L_EAL + w_s L_WTV + w_tv L_TV over [N][K][V] windows (terms selected by
+    ``mode``)."""
     fw = loss_forward(target, draft, mask, mode & 3, T, w_greedy, w_sampling, n_windows_total)
     if mode & MODE_KL:
         an = anchor_forward(target, draft, mask, n_positions_total)
         fw["loss"] += w_kl * an["loss"]
         fw["kl"] = an["kl"]
         fw["npos"] = an["npos"]
+    if mode & MODE_TV:
+        tv = tv_forward(target, draft, mask, T, n_windows_total)
+        fw["loss"] += w_tv * tv["loss"]
+        fw["tv"] = tv["tv"]
+        fw["nvalid"] = tv["nvalid"]
     return fw
 
 
 def objective_backward(target, draft, mask=None, mode: int = MODE_KL | 1, T: float = 1.0,
                        w_greedy: float = 1.0, w_sampling: float = 1.0, w_kl: float = 1.0,
-                       dloss: float = 1.0, n_windows_total=None, n_positions_total=None) -> np.ndarray:
+                       dloss: float = 1.0, n_windows_total=None, n_positions_total=None,
+                       w_tv: float = 1.0) -> np.ndarray:
     """dloss * d(objective)/dz_q, [N][K][V]."""
     g = loss_backward(target, draft, mask, mode & 3, T, w_greedy, w_sampling, dloss, n_windows_total)
     if mode & MODE_KL:
         g = g + anchor_backward(target, draft, mask, dloss * w_kl, n_positions_total)
+    if mode & MODE_TV:
+        g = g + tv_backward(target, draft, mask, T, dloss * w_tv, n_windows_total)
     return g
+
+
+# ---------------------------------------------------------------------------------------
+# The L_TV baseline's auxiliary term (Sec. 4.1): the per-position total variation distance
+# averaged across the window, L_aux(t) = (1/gamma) sum_j TV(p~_{t+j}, q~_{t+j}), with
+# TV = (1/2) sum_v |p~(v) - q~(v)|.  Readings: a masked window averages over its K_n valid
+# leading positions (1/K_n; = 1/gamma without a mask), windows not in W add nothing, and
+# L_TV is the mean over W:  L_TV = (1/|W|) sum_{n in W} (1/K_n) sum_{j < K_n} TV_{n,j}.
+# Gradient: TV = 1 - sum_v min(p~, q~) (Sec. 3.3), so dTV/dz_u = -d a^sample/dz_u with the
+# subgradient of losses.loss_backward (the min follows the frozen p~ at a tie).
+
+MODE_TV = 16  # the L_TV auxiliary term, a mode bit
+
+
+def total_variation(target, draft, T: float) -> np.ndarray:
+    """TV(p~, q~) of every row, from its definition (1/2) sum_v |p~(v) - q~(v)|."""
+    pt = np.exp(log_softmax(as_f64(target), T))
+    qt = np.exp(log_softmax(as_f64(draft), T))
+    return 0.5 * np.sum(np.abs(pt - qt), axis=-1)
+
+
+def tv_forward(target, draft, mask=None, T: float = 1.0, n_windows_total=None):
+    from .losses import leading_valid_depths
+    zp = as_f64(target)
+    N, K, _ = zp.shape
+    kn = leading_valid_depths(mask, N, K)
+    tv = total_variation(zp, draft, T)
+    per = np.zeros(N)
+    for n in range(N):
+        if kn[n] >= 1:
+            per[n] = np.sum(tv[n, :kn[n]]) / kn[n]
+    nvalid = int(np.sum(kn >= 1)) if n_windows_total is None else int(n_windows_total)
+    loss = float(np.sum(per) / nvalid) if nvalid > 0 else 0.0
+    return dict(loss=loss, tv=tv, per_window=per, kn=kn, nvalid=nvalid)
+
+
+def tv_backward(target, draft, mask=None, T: float = 1.0, dloss: float = 1.0, n_windows_total=None) -> np.ndarray:
+    """dloss * dL_TV/dz_q, [N][K][V]."""
+    zp = as_f64(target)
+    zq = as_f64(draft)
+    fw = tv_forward(zp, zq, mask, T, n_windows_total)
+    grad = np.zeros_like(zq)
+    if fw["nvalid"] == 0:
+        return grad
+    lp = log_softmax(zp, T)
+    lq = log_softmax(zq, T)
+    qt = np.exp(lq)
+    c = (lq < lp).astype(np.float64)
+    qlt = np.sum(c * qt, axis=-1, keepdims=True)
+    da_s = (1.0 / T) * qt * (c - qlt)          # d a^sample / dz_u, as in losses.loss_backward
+    N, K, _ = zq.shape
+    for n in range(N):
+        for j in range(int(fw["kn"][n])):
+            grad[n, j] = -dloss / (fw["nvalid"] * fw["kn"][n]) * da_s[n, j]
+    return grad

@@ -77,10 +77,11 @@ def seq_loss_backward(target, draft, mask, K: int, mode: int = MODE_BOTH, T: flo
 
 def seq_objective_forward(target, draft, mask, K: int, mode: int = 5, T: float = 1.0,
                           w_greedy: float = 1.0, w_sampling: float = 1.0, w_kl: float = 1.0,
-                          n_windows_total=None, n_positions_total=None, full_windows: bool = False):
+                          n_windows_total=None, n_positions_total=None, full_windows: bool = False,
+                          w_tv: float = 1.0):
     """w_kl L_KL + w_g L_EAL + w_s L_WTV over whole sequences: the window terms as in
     seq_loss_forward, the anchor once per valid position (anchor.py)."""
-    from .anchor import MODE_KL, anchor_forward
+    from .anchor import MODE_KL, MODE_TV, anchor_forward, tv_forward
     fw = seq_loss_forward(target, draft, mask, K, mode & 3, T, w_greedy, w_sampling, n_windows_total,
                           full_windows)
     if mode & MODE_KL:
@@ -88,17 +89,32 @@ def seq_objective_forward(target, draft, mask, K: int, mode: int = 5, T: float =
         fw["loss"] += w_kl * an["loss"]
         fw["kl"] = an["kl"]
         fw["npos"] = an["npos"]
+    if mode & MODE_TV:   # the L_TV term over the same sliding windows
+        wp, wq, wm, _ = gather_windows(target, draft, mask, K, full_windows)
+        tv = tv_forward(wp, wq, wm, T, n_windows_total)
+        fw["loss"] += w_tv * tv["loss"]
+        fw["nvalid"] = tv["nvalid"]
     return fw
 
 
 def seq_objective_backward(target, draft, mask, K: int, mode: int = 5, T: float = 1.0,
                            w_greedy: float = 1.0, w_sampling: float = 1.0, w_kl: float = 1.0,
                            dloss: float = 1.0, n_windows_total=None, n_positions_total=None,
-                           full_windows: bool = False) -> np.ndarray:
+                           full_windows: bool = False, w_tv: float = 1.0) -> np.ndarray:
     """dloss * d(objective)/dz_q per position, [B][T][V]."""
-    from .anchor import MODE_KL, anchor_backward
+    from .anchor import MODE_KL, MODE_TV, anchor_backward, tv_backward
     g = seq_loss_backward(target, draft, mask, K, mode & 3, T, w_greedy, w_sampling, dloss,
                           n_windows_total, full_windows)
     if mode & MODE_KL:
         g = g + anchor_backward(target, draft, mask, dloss * w_kl, n_positions_total)
+    if mode & MODE_TV:   # window rows' gradients added back to their positions
+        B, Tn, V = as_f64(draft).shape
+        wp, wq, wm, src = gather_windows(target, draft, mask, K, full_windows)
+        gw = tv_backward(wp, wq, wm, T, dloss * w_tv, n_windows_total)
+        out = np.zeros((B * Tn, V))
+        for n in range(B * Tn):
+            for j in range(K):
+                if src[n, j] >= 0:
+                    out[src[n, j]] += gw[n, j]
+        g = g + out.reshape(B, Tn, V)
     return g

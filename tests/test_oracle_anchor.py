@@ -144,3 +144,58 @@ def test_sequence_objective_by_finite_differences():
         assert abs(fd - g[idx]) < 1e-7, (idx, fd, g[idx])
     fw = oracle.seq_objective_forward(zp, zq, mask, K, **kw)
     assert fw["npos"] == 4
+
+
+# ---------------------------------------------------------------------- the L_TV baseline term
+
+def test_total_variation_against_scipy_and_special_cases():
+    import scipy.spatial.distance as ssd
+    rng = np.random.default_rng(20)
+    zp = _logits(rng, 3, 2, 12)
+    zq = _logits(rng, 3, 2, 12)
+    tv = oracle.total_variation(zp, zq, 0.7)
+    pt = np.exp(oracle.log_softmax(zp, 0.7))
+    qt = np.exp(oracle.log_softmax(zq, 0.7))
+    for idx in np.ndindex(3, 2):
+        assert abs(tv[idx] - 0.5 * ssd.cityblock(pt[idx], qt[idx])) < 1e-14
+    np.testing.assert_allclose(tv, 1.0 - oracle.acceptance_sampling(zp, zq, 0.7), atol=1e-14)
+    assert np.all(oracle.total_variation(zp, zp, 1.3) < 1e-15)
+    a = np.array([[0.0, 0.0, -np.inf, -np.inf]])
+    b = np.array([[-np.inf, -np.inf, 0.0, 1.0]])
+    assert abs(oracle.total_variation(a, b, 1.0)[0] - 1.0) < 1e-15          # disjoint supports
+
+
+def test_tv_term_averages_each_window_over_its_valid_positions():
+    rng = np.random.default_rng(21)
+    zp = _logits(rng, 3, 4, 9)
+    zq = _logits(rng, 3, 4, 9)
+    mask = np.ones((3, 4), dtype=np.uint8)
+    mask[1, 2] = 0          # K_1 = 2
+    mask[2, 0] = 0          # window 2 not in W
+    fw = oracle.tv_forward(zp, zq, mask, 0.9)
+    tv = oracle.total_variation(zp, zq, 0.9)
+    want = (tv[0].mean() + tv[1, :2].mean()) / 2
+    assert fw["nvalid"] == 2 and abs(fw["loss"] - want) < 1e-15
+
+
+@pytest.mark.parametrize("mode,T", [(oracle.MODE_TV, 1.0), (oracle.MODE_KL | oracle.MODE_TV, 0.8),
+                                    (oracle.MODE_TV | 3, 1.2)])
+def test_tv_objective_by_finite_differences(mode, T):
+    rng = np.random.default_rng(22)
+    N, K, V = 2, 3, 6
+    while True:
+        zp = _logits(rng, N, K, V, scale=1.5)
+        zq = zp + _logits(rng, N, K, V, scale=1.0)
+        pt = np.exp(oracle.log_softmax(zp, T))
+        qt = np.exp(oracle.log_softmax(zq, T))
+        if np.min(np.abs(pt - qt)) > 1e-3:
+            break
+    mask = np.array([[1, 1, 0], [1, 1, 1]], dtype=np.uint8)
+    kw = dict(mode=mode, T=T, w_greedy=0.2, w_sampling=0.5, w_kl=1.0, w_tv=0.1)
+    g = objective_backward(zp, zq, mask, dloss=2.0, **kw)
+    h = 1e-6
+    for idx in np.ndindex(N, K, V):
+        a = zq.copy(); a[idx] += h
+        b = zq.copy(); b[idx] -= h
+        fd = 2.0 * (objective_forward(zp, a, mask, **kw)["loss"] - objective_forward(zp, b, mask, **kw)["loss"]) / (2 * h)
+        assert abs(fd - g[idx]) < 1e-7, (idx, fd, g[idx])

@@ -140,3 +140,25 @@ def test_full_windows_reading_keeps_only_complete_windows():
     assert list(fw["kn"]) == [3, 0, 0, 0, 0, 0]
     g = seq_loss_backward(zp, zq, mask, K, oracle.MODE_SAMPLING, full_windows=True)
     assert np.all(g[0, 3:] == 0) and np.any(g[0, :3] != 0)
+
+
+def test_sequence_tv_term_by_finite_differences():
+    rng = np.random.default_rng(8)
+    B, Tn, K, V = 1, 5, 3, 5
+    while True:
+        zp = rng.normal(0, 1.5, size=(B, Tn, V))
+        zq = zp + rng.normal(0, 1.0, size=(B, Tn, V))
+        pt = np.exp(oracle.log_softmax(zp, 0.9)); qt = np.exp(oracle.log_softmax(zq, 0.9))
+        if np.min(np.abs(pt - qt)) > 1e-3:
+            break
+    mask = np.ones((B, Tn), dtype=np.uint8)
+    mask[0, 3] = 0
+    kw = dict(mode=oracle.MODE_KL | oracle.MODE_TV, T=0.9, w_greedy=0.0, w_sampling=0.0, w_kl=1.0, w_tv=0.1)
+    g = oracle.seq_objective_backward(zp, zq, mask, K, dloss=2.0, **kw)
+    h = 1e-6
+    for idx in np.ndindex(B, Tn, V):
+        a = zq.copy(); a[idx] += h
+        b = zq.copy(); b[idx] -= h
+        fd = 2.0 * (oracle.seq_objective_forward(zp, a, mask, K, **kw)["loss"]
+                    - oracle.seq_objective_forward(zp, b, mask, K, **kw)["loss"]) / (2 * h)
+        assert abs(fd - g[idx]) < 1e-7, (idx, fd, g[idx])
