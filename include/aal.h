@@ -71,8 +71,11 @@ typedef enum { AAL_F32 = 0, AAL_BF16 = 1 } aal_dtype;
  * the GRPO surrogate (Sec. 3.4) whose per-row coefficients aal_grpo_from_loss writes into the
  * loss workspace between the forward and the backward; aal_loss_fwd clears them, so without
  * that call the term is zero, and the loss aal_loss_fwd reports never includes it (see
- * aal_grpo_from_loss).  Valid modes: 1 .. 15 (AAL_GRPO only with aal_loss_*). */
-typedef enum { AAL_GREEDY = 1, AAL_SAMPLING = 2, AAL_BOTH = 3, AAL_KL = 4, AAL_GRPO = 8 } aal_mode;
+ * aal_grpo_from_loss).  AAL_TV adds w_tv * L_TV, the auxiliary term of the L_KL + L_TV baseline
+ * (Sec. 4.1): each window's TV(p~, q~) = 1 - a^sample averaged over its K_n valid positions, then
+ * the mean over W; the baseline L_KL + 0.1 L_TV is mode AAL_KL | AAL_TV with w_tv = 0.1 (T as for
+ * the sampling term).  Valid modes: 1 .. 31 (AAL_GRPO only with aal_loss_*). */
+typedef enum { AAL_GREEDY = 1, AAL_SAMPLING = 2, AAL_BOTH = 3, AAL_KL = 4, AAL_GRPO = 8, AAL_TV = 16 } aal_mode;
 
 #define AAL_MAX_K 8
 
@@ -80,12 +83,12 @@ typedef enum { AAL_GREEDY = 1, AAL_SAMPLING = 2, AAL_BOTH = 3, AAL_KL = 4, AAL_G
  *   N, K, V      windows, window size gamma (1..AAL_MAX_K), vocabulary size (>= 1); N may be 0.
  *   dtype        aal_dtype of draft, target and the gradient.
  *   mode         aal_mode.
- *   temperature  T of the sampling term (Sec. 2.3: p~ ~ exp(log p / T)); must be finite
- *                and > 0 when mode includes SAMPLING.  The greedy acceptance
+ *   temperature  T of the sampling and TV terms (Sec. 2.3: p~ ~ exp(log p / T)); must be
+ *                finite and > 0 when mode includes SAMPLING or TV.  The greedy acceptance
  *                a = q(x*) (Eq. acc_greedy) always uses the unscaled draft, so T is
  *                ignored (and may be 0) for mode GREEDY.
- *   w_greedy, w_sampling, w_kl  weights of the terms (a term the mode does not select is
- *                not computed and its weight is ignored).  Must be finite. */
+ *   w_greedy, w_sampling, w_kl, w_tv  weights of the terms (a term the mode does not select
+ *                is not computed and its weight is ignored).  Must be finite. */
 typedef struct {
   int64_t N, K, V;
   int32_t dtype;
@@ -94,6 +97,7 @@ typedef struct {
   float w_greedy;
   float w_sampling;
   float w_kl;
+  float w_tv;
   int32_t reserved; /* must be 0 */
 } aal_problem;
 
@@ -105,6 +109,7 @@ AAL_API aal_status aal_workspace_size(const aal_problem* prob, size_t* bytes);
  *                       + w_s sum_{k=1}^{K_n} prod_{j<k} a^s_{n,j} ]
  *       + w_kl (1/|P|) sum_{valid rows r} KL(p_r || q_r)     (mode bit AAL_KL; |P| = number
  *                                                            of rows with mask 1; 0 if none)
+ *       + w_tv (1/|W|) sum_n (1/K_n) sum_{j<K_n} (1 - a^s_{n,j})    (mode bit AAL_TV)
  * with a^g = q(x*) (Eq. acc_greedy, x* = target argmax, lowest index on ties) and
  * a^s = sum_v min(p~, q~) = 1 - TV(p~, q~) (Eqs. acc_sample, rejection_rate).
  *   draft, target  [N][K][V] logits of the draft (z_q) and the target (z_p).
@@ -134,7 +139,7 @@ AAL_API aal_status aal_loss_bwd(const aal_problem* prob, const void* draft, cons
  * is depth j of up to K windows.  Logits are stored once per position, not once per window.
  *   B, seq_len, K, V  sequences, positions per sequence (>= 0), window size gamma
  *                     (1..AAL_MAX_K), vocabulary size (>= 1).
- *   dtype, mode, temperature, w_greedy, w_sampling, w_kl, reserved  as in aal_problem
+ *   dtype, mode, temperature, w_greedy, w_sampling, w_kl, w_tv, reserved  as in aal_problem
  *                     (the anchor averages over the valid positions).
  *   full_windows      which windows belong to W (the paper leaves the end of a sequence open):
  *                     0 = every start position, its window truncated at the end of the
@@ -149,6 +154,7 @@ typedef struct {
   float w_greedy;
   float w_sampling;
   float w_kl;
+  float w_tv;
   int32_t full_windows;
   int32_t reserved; /* must be 0 */
 } aal_seq_problem;

@@ -23,6 +23,7 @@ AAL_SAMPLING = 2
 AAL_BOTH = 3
 AAL_KL = 4          # mode bit: the forward-KL anchor
 AAL_GRPO = 8        # mode bit: the backward adds the GRPO surrogate's gradient
+AAL_TV = 16         # mode bit: the L_TV baseline's window-averaged TV term
 
 AAL_MAX_K = 8
 AAL_NOALLOC_MAX_ROWS = 1 << 20   # N * K limit of aal_accept_reward_noalloc
@@ -39,7 +40,8 @@ class AalProblem(ctypes.Structure):
     _fields_ = [("N", ctypes.c_int64), ("K", ctypes.c_int64), ("V", ctypes.c_int64),
                 ("dtype", ctypes.c_int32), ("mode", ctypes.c_int32),
                 ("temperature", ctypes.c_float), ("w_greedy", ctypes.c_float),
-                ("w_sampling", ctypes.c_float), ("w_kl", ctypes.c_float), ("reserved", ctypes.c_int32)]
+                ("w_sampling", ctypes.c_float), ("w_kl", ctypes.c_float), ("w_tv", ctypes.c_float),
+                ("reserved", ctypes.c_int32)]
 
 
 class AalRewardProblem(ctypes.Structure):
@@ -56,7 +58,7 @@ class AalSeqProblem(ctypes.Structure):
     _fields_ = [("B", ctypes.c_int64), ("seq_len", ctypes.c_int64), ("K", ctypes.c_int64),
                 ("V", ctypes.c_int64), ("dtype", ctypes.c_int32), ("mode", ctypes.c_int32),
                 ("temperature", ctypes.c_float), ("w_greedy", ctypes.c_float),
-                ("w_sampling", ctypes.c_float), ("w_kl", ctypes.c_float),
+                ("w_sampling", ctypes.c_float), ("w_kl", ctypes.c_float), ("w_tv", ctypes.c_float),
                 ("full_windows", ctypes.c_int32), ("reserved", ctypes.c_int32)]
 
 
@@ -163,18 +165,20 @@ def _check(code: int, where: str):
 
 
 def loss_problem(draft: torch.Tensor, mode: int, temperature: float = 1.0, w_greedy: float = 1.0,
-                 w_sampling: float = 1.0, w_kl: float = 1.0) -> AalProblem:
-    """Problem struct for [N][K][V] logits (``w_kl`` weighs the AAL_KL anchor)."""
+                 w_sampling: float = 1.0, w_kl: float = 1.0, w_tv: float = 1.0) -> AalProblem:
+    """Problem struct for [N][K][V] logits (``w_kl`` weighs the AAL_KL anchor, ``w_tv`` the
+    AAL_TV term)."""
     if draft.dim() != 3:
         raise ValueError("logits must be [N][K][V]")
     N, K, V = draft.shape
     if draft.dtype not in _DTYPES:
         raise ValueError(f"unsupported dtype {draft.dtype}")
-    return AalProblem(N, K, V, _DTYPES[draft.dtype], mode, temperature, w_greedy, w_sampling, w_kl, 0)
+    return AalProblem(N, K, V, _DTYPES[draft.dtype], mode, temperature, w_greedy, w_sampling, w_kl, w_tv, 0)
 
 
 def seq_problem(draft: torch.Tensor, K: int, mode: int, temperature: float = 1.0, w_greedy: float = 1.0,
-                w_sampling: float = 1.0, full_windows: bool = False, w_kl: float = 1.0) -> AalSeqProblem:
+                w_sampling: float = 1.0, full_windows: bool = False, w_kl: float = 1.0,
+                w_tv: float = 1.0) -> AalSeqProblem:
     """Problem struct for [B][seq_len][V] logits with sliding windows of K positions
     (``full_windows``: only windows with all K positions valid belong to W)."""
     if draft.dim() != 3:
@@ -183,7 +187,7 @@ def seq_problem(draft: torch.Tensor, K: int, mode: int, temperature: float = 1.0
     if draft.dtype not in _DTYPES:
         raise ValueError(f"unsupported dtype {draft.dtype}")
     return AalSeqProblem(B, S, K, V, _DTYPES[draft.dtype], mode, temperature, w_greedy, w_sampling,
-                         w_kl, int(bool(full_windows)), 0)
+                         w_kl, w_tv, int(bool(full_windows)), 0)
 
 
 def reward_problem(draft: torch.Tensor, mode: int, temperature: float = 1.0, adv_clip: float = 5.0,

@@ -30,9 +30,11 @@ aal_status check_problem(const aal_problem* p) {
   if (p == nullptr) return AAL_ERR_INVALID_ARG;
   aal_status st = check_shape(p->N, p->K, p->V, p->dtype);
   if (st != AAL_OK) return st;
-  if (p->mode < 1 || p->mode > (AAL_BOTH | AAL_KL | AAL_GRPO)) return AAL_ERR_INVALID_ARG;
-  if ((p->mode & AAL_SAMPLING) && !(isfinite(p->temperature) && p->temperature > 0.f)) return AAL_ERR_INVALID_ARG;
-  if (!isfinite(p->w_greedy) || !isfinite(p->w_sampling) || !isfinite(p->w_kl)) return AAL_ERR_INVALID_ARG;
+  if (p->mode < 1 || p->mode > (AAL_BOTH | AAL_KL | AAL_GRPO | AAL_TV)) return AAL_ERR_INVALID_ARG;
+  if ((p->mode & (AAL_SAMPLING | AAL_TV)) && !(isfinite(p->temperature) && p->temperature > 0.f))
+    return AAL_ERR_INVALID_ARG;
+  if (!isfinite(p->w_greedy) || !isfinite(p->w_sampling) || !isfinite(p->w_kl) || !isfinite(p->w_tv))
+    return AAL_ERR_INVALID_ARG;
   if (p->reserved != 0) return AAL_ERR_INVALID_ARG;
   return AAL_OK;
 }
@@ -59,7 +61,7 @@ aal_status check_seq(const aal_seq_problem* p) {
   // the checks of a windowed problem with one window per position (R * K * V elements bound
   // the per-depth partials too)
   const aal_problem q{p->B * p->seq_len, p->K, p->V, p->dtype, p->mode, p->temperature, p->w_greedy,
-                      p->w_sampling, p->w_kl, p->reserved};
+                      p->w_sampling, p->w_kl, p->w_tv, p->reserved};
   aal_status st = check_problem(&q);
   if (st != AAL_OK) return st;
   if (p->mode & AAL_GRPO) return AAL_ERR_UNSUPPORTED;  // the GRPO stage runs over windows
@@ -88,7 +90,8 @@ aal_status cuda_status(cudaError_t e) { return e == cudaSuccess ? AAL_OK : AAL_E
 // Per-row statistics of R logit rows (pass over z_p and z_q), shared by both layouts.
 cudaError_t launch_stats(const void* draft, const void* target, int64_t R, int64_t V, int32_t dtype,
                          int32_t mode, float temperature, const LossWs& ws, cudaStream_t s, int* cluster) {
-  const bool greedy = (mode & AAL_GREEDY) != 0, sampling = (mode & AAL_SAMPLING) != 0;
+  const bool greedy = (mode & AAL_GREEDY) != 0;
+  const bool sampling = (mode & (AAL_SAMPLING | AAL_TV)) != 0;  // both need a^sample
   const bool kl = (mode & AAL_KL) != 0;
   const bool grpo = (mode & AAL_GRPO) != 0;  // log pi_theta(y) needs the T = 1 normaliser
   RowStatsArgs ra;
@@ -112,7 +115,8 @@ cudaError_t launch_stats(const void* draft, const void* target, int64_t R, int64
 cudaError_t launch_grad(const void* draft, const void* target, const uint8_t* mask, int64_t R, int64_t V,
                         int32_t dtype, int32_t mode, float temperature, float w_greedy, float w_sampling,
                         float w_kl, float dloss, const LossWs& ws, void* grad, cudaStream_t s) {
-  const bool greedy = (mode & AAL_GREEDY) != 0, sampling = (mode & AAL_SAMPLING) != 0;
+  const bool greedy = (mode & AAL_GREEDY) != 0;
+  const bool sampling = (mode & (AAL_SAMPLING | AAL_TV)) != 0;
   const bool kl = (mode & AAL_KL) != 0;
   const bool grpo = (mode & AAL_GRPO) != 0;
   BackwardArgs ba;
@@ -126,7 +130,7 @@ cudaError_t launch_grad(const void* draft, const void* target, const uint8_t* ma
   ba.invT = sampling ? 1.0f / temperature : 0.f;
   ba.dloss = dloss;
   ba.w_greedy = greedy ? w_greedy : 0.f;
-  ba.w_sampling = sampling ? w_sampling : 0.f;
+  ba.w_sampling = sampling ? 1.f : 0.f;  // the window kernels fold w_s and w_tv into dE^s/da
   ba.w_kl = kl ? w_kl : 0.f;
   ba.grpo = grpo;
   ba.mask = mask;
@@ -144,7 +148,7 @@ int64_t debug_take_skip_chunk() { return g_skip_chunk.exchange(-1); }
 
 extern "C" {
 
-int32_t aal_abi_version(void) { return 10100; }
+int32_t aal_abi_version(void) { return 10200; }
 
 void aal_debug_fail_next_forward(int64_t chunk, uint64_t wait_limit_ns) {
   g_wait_limit_ns.store(wait_limit_ns);
@@ -212,9 +216,11 @@ aal_status aal_loss_fwd(const aal_problem* prob, const void* draft, const void* 
   wa.greedy = greedy;
   wa.sampling = sampling;
   wa.kl = (prob->mode & AAL_KL) != 0;
+  wa.tv = (prob->mode & AAL_TV) != 0;
   wa.w_greedy = prob->w_greedy;
   wa.w_sampling = prob->w_sampling;
   wa.w_kl = prob->w_kl;
+  wa.w_tv = prob->w_tv;
   wa.loss = loss;
   wa.eal = eal;
   wa.ws = ws;
@@ -282,9 +288,11 @@ aal_status aal_seq_loss_fwd(const aal_seq_problem* prob, const void* draft, cons
   wa.greedy = (prob->mode & AAL_GREEDY) != 0;
   wa.sampling = (prob->mode & AAL_SAMPLING) != 0;
   wa.kl = (prob->mode & AAL_KL) != 0;
+  wa.tv = (prob->mode & AAL_TV) != 0;
   wa.w_greedy = prob->w_greedy;
   wa.w_sampling = prob->w_sampling;
   wa.w_kl = prob->w_kl;
+  wa.w_tv = prob->w_tv;
   wa.loss = loss;
   wa.eal = eal;
   wa.pg = reinterpret_cast<float*>(base + L.pg);

@@ -41,7 +41,7 @@ struct LossLayout {
   size_t kl = 0;                    // float[R] KL(p || q) at T = 1 (KL anchor)
   size_t cgr = 0;                   // float[R] GRPO coefficient of (delta_{u,y} - q(u)), w_grpo included
   size_t ag = 0, as = 0, qlt = 0;   // float[R] a^greedy, a^sample, sum_{lq<lp} q~
-  size_t dEg = 0, dEs = 0;          // float[R] dE_n / da_{n,j}
+  size_t dEg = 0, dEs = 0;          // float[R] dE^g/da (unweighted); w_s dE^s/da + w_tv / K_n
   size_t xstar = 0;                 // int32[R] target argmax
   size_t yhat = 0;                  // int32[R] draft argmax (the greedy draft token)
   size_t zpy = 0;                   // float[R] z_p at the draft argmax
@@ -198,8 +198,8 @@ struct WindowArgs {
   int64_t N;
   int32_t K;
   int32_t cluster;      // partials per row in ws.cpart
-  bool greedy, sampling, kl;
-  float w_greedy, w_sampling, w_kl;
+  bool greedy, sampling, kl, tv;
+  float w_greedy, w_sampling, w_kl, w_tv;
   float* loss;          // device float[1]
   float* eal;           // device float[N][2] or null
   LossWs ws;
@@ -211,9 +211,9 @@ struct SeqWindowArgs {
   int64_t B, T;
   int32_t K;
   int32_t cluster;
-  bool greedy, sampling, kl;
+  bool greedy, sampling, kl, tv;
   bool full_windows;    // W = windows with all K positions valid
-  float w_greedy, w_sampling, w_kl;
+  float w_greedy, w_sampling, w_kl, w_tv;
   float* loss;
   float* eal;           // [B*T][2] or null
   float* pg;            // [B*T][K]

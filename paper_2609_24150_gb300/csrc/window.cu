@@ -40,10 +40,11 @@ __device__ __forceinline__ void block_sum(double (&x)[NV], double* sm) {
   __syncthreads();
 }
 
-constexpr int kSums = 5;  // sum E^g, sum E^s, |W|, sum KL, |positions|
+constexpr int kSums = 6;  // sum E^g, sum E^s, |W|, sum KL, |positions|, sum of window TV means
 
 // Block partials -> the last block to finish adds them in block order and writes the loss
 //   L = -(w_g sum E^g + w_s sum E^s) / |W| + w_kl sum KL / |positions|
+//       + w_tv sum_n (1/K_n) sum_j (1 - a^s_{n,j}) / |W|
 // (each term 0 when its count is 0), |W| and |positions|.
 template <typename Args>
 __device__ __forceinline__ void finish_loss(const Args& a, double (&x)[kSums], double* sm, bool* is_last) {
@@ -74,6 +75,7 @@ __device__ __forceinline__ void finish_loss(const Args& a, double (&x)[kSums], d
                        (a.sampling ? (double)a.w_sampling * t[1] : 0.0);
     double L = nvalid > 0 ? -num / (double)nvalid : 0.0;
     if (a.kl && npos > 0) L += (double)a.w_kl * t[3] / (double)npos;
+    if (a.tv && nvalid > 0) L += (double)a.w_tv * t[5] / (double)nvalid;
     const float loss = (float)L;
     *a.loss = loss;
     a.ws.hdr->loss = loss;
@@ -113,7 +115,8 @@ __global__ void __launch_bounds__(kWindowThreads) window_kernel(WindowArgs a) {
   __shared__ double sm[kSums * kWindowThreads / 32];
   __shared__ bool is_last;
   const int64_t n = (int64_t)blockIdx.x * kWindowThreads + threadIdx.x;
-  double eg = 0.0, es = 0.0, valid = 0.0, ksum = 0.0, kcnt = 0.0;
+  double eg = 0.0, es = 0.0, valid = 0.0, ksum = 0.0, kcnt = 0.0, tvs = 0.0;
+  const bool ov = a.sampling || a.tv;  // both terms are built from a^sample
   if (n < a.N) {
     const int K = a.K;
     int kn = K;
@@ -131,7 +134,7 @@ __global__ void __launch_bounds__(kWindowThreads) window_kernel(WindowArgs a) {
       if (j < K) {
         const int64_t r = r0 + j;
         if (a.greedy) ag[j] = a.ws.ag[r];
-        if (a.sampling) {
+        if (ov) {
           float2 t = a.ws.cpart[r * kMaxCluster];
           for (int c = 1; c < a.cluster; ++c) {
             const float2 u = a.ws.cpart[r * kMaxCluster + c];
@@ -151,11 +154,18 @@ __global__ void __launch_bounds__(kWindowThreads) window_kernel(WindowArgs a) {
       for (int j = 0; j < AAL_MAX_K; ++j)
         if (j < K) a.ws.dEg[r0 + j] = dE[j];
     }
-    if (a.sampling) {
-      Es = window_term(as, kn, dE);
+    if (ov) {
+      // the sampling-side coefficient of each row, weights folded in:
+      // w_s dE^s/da + w_tv / K_n (the TV term's derivative, with the sign of -a^s)
+      if (a.sampling) Es = window_term(as, kn, dE);
+      const float tvc = (a.tv && kn > 0) ? a.w_tv / (float)kn : 0.f;
+      float tsum = 0.f;
 #pragma unroll
-      for (int j = 0; j < AAL_MAX_K; ++j)
-        if (j < K) a.ws.dEs[r0 + j] = dE[j];
+      for (int j = 0; j < AAL_MAX_K; ++j) {
+        if (j < K) a.ws.dEs[r0 + j] = (a.sampling ? a.w_sampling * dE[j] : 0.f) + (j < kn ? tvc : 0.f);
+        if (j < kn) tsum += 1.f - as[j];
+      }
+      if (a.tv && kn > 0) tvs = tsum / (float)kn;
     }
     if (a.eal != nullptr) {
       a.eal[2 * n + 0] = Eg;
@@ -177,7 +187,7 @@ __global__ void __launch_bounds__(kWindowThreads) window_kernel(WindowArgs a) {
       kcnt = c;
     }
   }
-  double x[kSums] = {eg, es, valid, ksum, kcnt};
+  double x[kSums] = {eg, es, valid, ksum, kcnt, tvs};
   finish_loss(a, x, sm, &is_last);
 }
 
@@ -203,7 +213,8 @@ __global__ void __launch_bounds__(kWindowThreads) seq_window_kernel(SeqWindowArg
   __shared__ bool is_last;
   const int64_t N = a.B * a.T;
   const int64_t n = (int64_t)blockIdx.x * kWindowThreads + threadIdx.x;
-  double eg = 0.0, es = 0.0, valid = 0.0, ksum = 0.0, kcnt = 0.0;
+  double eg = 0.0, es = 0.0, valid = 0.0, ksum = 0.0, kcnt = 0.0, tvs = 0.0;
+  const bool ov = a.sampling || a.tv;
   if (n < N) {
     const int K = a.K;
     const int64_t t = n % a.T;
@@ -212,7 +223,7 @@ __global__ void __launch_bounds__(kWindowThreads) seq_window_kernel(SeqWindowArg
     if (a.full_windows && kn < K) kn = 0;
     valid = kn >= 1 ? 1.0 : 0.0;
     // this window's first row is position n: finish its per-row overlap sums here
-    if (a.sampling) {
+    if (ov) {
       float q;
       a.ws.as[n] = row_overlap(a.ws, n, a.cluster, &q);
       a.ws.qlt[n] = q;
@@ -224,7 +235,7 @@ __global__ void __launch_bounds__(kWindowThreads) seq_window_kernel(SeqWindowArg
       as[j] = 0.f;
       if (j < kn) {
         if (a.greedy) ag[j] = a.ws.ag[n + j];
-        if (a.sampling) as[j] = row_overlap(a.ws, n + j, a.cluster, nullptr);
+        if (ov) as[j] = row_overlap(a.ws, n + j, a.cluster, nullptr);
       }
     }
     float Eg = 0.f, Es = 0.f;
@@ -234,11 +245,16 @@ __global__ void __launch_bounds__(kWindowThreads) seq_window_kernel(SeqWindowArg
       for (int j = 0; j < AAL_MAX_K; ++j)
         if (j < K) a.pg[n * K + j] = dE[j];
     }
-    if (a.sampling) {
-      Es = window_term(as, kn, dE);
+    if (ov) {  // weighted partials, as in window_kernel
+      if (a.sampling) Es = window_term(as, kn, dE);
+      const float tvc = (a.tv && kn > 0) ? a.w_tv / (float)kn : 0.f;
+      float tsum = 0.f;
 #pragma unroll
-      for (int j = 0; j < AAL_MAX_K; ++j)
-        if (j < K) a.ps[n * K + j] = dE[j];
+      for (int j = 0; j < AAL_MAX_K; ++j) {
+        if (j < K) a.ps[n * K + j] = (a.sampling ? a.w_sampling * dE[j] : 0.f) + (j < kn ? tvc : 0.f);
+        if (j < kn) tsum += 1.f - as[j];
+      }
+      if (a.tv && kn > 0) tvs = tsum / (float)kn;
     }
     if (a.eal != nullptr) {
       a.eal[2 * n + 0] = Eg;
@@ -251,7 +267,7 @@ __global__ void __launch_bounds__(kWindowThreads) seq_window_kernel(SeqWindowArg
       kcnt = 1.0;
     }
   }
-  double x[kSums] = {eg, es, valid, ksum, kcnt};
+  double x[kSums] = {eg, es, valid, ksum, kcnt, tvs};
   finish_loss(a, x, sm, &is_last);
 }
 
@@ -266,7 +282,7 @@ __global__ void __launch_bounds__(256) seq_gather_kernel(SeqWindowArgs a) {
   for (int j = 0; j < K && j <= t; ++j) {
     const int64_t n = p - j;
     if (a.greedy) g += a.pg[n * K + j];
-    if (a.sampling) s += a.ps[n * K + j];
+    if (a.sampling || a.tv) s += a.ps[n * K + j];
   }
   a.ws.dEg[p] = g;
   a.ws.dEs[p] = s;

@@ -25,17 +25,18 @@ GRAD_RTOL = 1e-2
 TIE_BAND = 1e-5
 
 MODES = {"greedy": aal.AAL_GREEDY, "sampling": aal.AAL_SAMPLING, "both": aal.AAL_BOTH}
-# the C modes are bit sets with the oracle's values: 1 EAL, 2 WTV, 4 the KL anchor
+# the C modes are bit sets with the oracle's values: 1 EAL, 2 WTV, 4 the KL anchor, 16 the TV term
 ORACLE_MODES = {m: (oracle.MODE_GREEDY if m & aal.AAL_GREEDY else 0)
                 | (oracle.MODE_SAMPLING if m & aal.AAL_SAMPLING else 0)
-                | (oracle.MODE_KL if m & aal.AAL_KL else 0) for m in range(1, 8)}
+                | (oracle.MODE_KL if m & aal.AAL_KL else 0)
+                | (oracle.MODE_TV if m & aal.AAL_TV else 0) for m in range(1, 32) if m & ~aal.AAL_GRPO}
 
 
 class LossRun:
     """Forward + backward of one problem through the C ABI; results stay on the device."""
 
-    def __init__(self, target, draft, mask, mode, T=1.0, wg=1.0, ws=1.0, dloss=1.0, wkl=1.0):
-        self.prob = aal.loss_problem(draft, mode, T, wg, ws, wkl)
+    def __init__(self, target, draft, mask, mode, T=1.0, wg=1.0, ws=1.0, dloss=1.0, wkl=1.0, wtv=1.0):
+        self.prob = aal.loss_problem(draft, mode, T, wg, ws, wkl, wtv)
         self.ws_buf = torch.empty(aal.aal_workspace_size(self.prob), dtype=torch.uint8,
                                   device=draft.device)
         N = draft.shape[0]
@@ -49,10 +50,10 @@ class LossRun:
         assert aal.aal_check_device_status(self.ws_buf) == aal.AAL_OK
 
 
-def grad_tolerance(target, draft, mask, omode, T, wg, ws, dloss, gref, nvalid, fw):
-    """Per-element tolerance, widened at WTV near-ties (see module docstring)."""
+def grad_tolerance(target, draft, mask, omode, T, wg, ws, dloss, gref, nvalid, fw, wtv=0.0):
+    """Per-element tolerance, widened at WTV / TV near-ties (see module docstring)."""
     tol = GRAD_ATOL + GRAD_RTOL * np.abs(gref)
-    if not (omode & oracle.MODE_SAMPLING) or nvalid == 0:
+    if not (omode & (oracle.MODE_SAMPLING | oracle.MODE_TV)) or nvalid == 0:
         return tol
     zp = oracle.as_f64(target)
     zq = oracle.as_f64(draft)
@@ -63,14 +64,20 @@ def grad_tolerance(target, draft, mask, omode, T, wg, ws, dloss, gref, nvalid, f
     if not amb.any():
         return tol
     qt = np.exp(lq)
-    dEs = oracle.expected_length_partials(fw["a_s"], fw["kn"])
-    B = np.abs(dloss * ws * dEs / nvalid / T)[..., None]
+    kn = fw["kn"]
+    coef = np.zeros(amb.shape[:-1])
+    if omode & oracle.MODE_SAMPLING:
+        coef = coef + ws * oracle.expected_length_partials(fw["a_s"], kn)
+    if omode & oracle.MODE_TV:
+        depth = np.arange(coef.shape[-1])[None, :]
+        coef = coef + np.where(depth < kn[:, None], wtv / np.maximum(kn, 1)[:, None], 0.0)
+    B = np.abs(dloss * coef / nvalid / T)[..., None]
     dq = np.sum(np.where(amb, qt, 0.0), axis=-1, keepdims=True)
     return tol + B * qt * (amb + dq)
 
 
 def check_loss(run: LossRun, target, draft, mask, mode, T, wg, ws, dloss=1.0, windows=None,
-               n_windows_total=None, wkl=1.0, n_positions_total=None):
+               n_windows_total=None, wkl=1.0, n_positions_total=None, wtv=1.0):
     """Compare loss / eal / gradient of ``run`` with the oracle (optionally on some windows)."""
     omode = ORACLE_MODES[mode]
     if windows is None:
@@ -82,7 +89,7 @@ def check_loss(run: LossRun, target, draft, mask, mode, T, wg, ws, dloss=1.0, wi
         t_h, d_h = target[idx].cpu(), draft[idx].cpu()
         m_h = None if mask is None else mask[idx].cpu().numpy()
         sel = np.asarray(windows)
-    fw = oracle.objective_forward(t_h, d_h, m_h, omode, T, wg, ws, wkl, n_windows_total, n_positions_total)
+    fw = oracle.objective_forward(t_h, d_h, m_h, omode, T, wg, ws, wkl, n_windows_total, n_positions_total, wtv)
     nvalid = fw["nvalid"]
     eal = run.eal.cpu().numpy()[sel]
     if omode & oracle.MODE_GREEDY:
@@ -94,9 +101,9 @@ def check_loss(run: LossRun, target, draft, mask, mode, T, wg, ws, dloss=1.0, wi
         got = float(run.loss.item())
         assert abs(got - ref) <= LOSS_RTOL * abs(ref) + LOSS_ATOL, (got, ref)
     gref = oracle.objective_backward(t_h, d_h, m_h, omode, T, wg, ws, wkl, dloss, n_windows_total,
-                                     n_positions_total)
+                                     n_positions_total, wtv)
     g = run.grad.cpu().double().numpy()[sel]
-    tol = grad_tolerance(t_h, d_h, m_h, omode, T, wg, ws, dloss, gref, nvalid, fw)
+    tol = grad_tolerance(t_h, d_h, m_h, omode, T, wg, ws, dloss, gref, nvalid, fw, wtv if omode & oracle.MODE_TV else 0.0)
     bad = np.abs(g - gref) > tol
     if bad.any():
         i = tuple(np.argwhere(bad)[0])
@@ -122,8 +129,8 @@ class SeqRun:
     """Forward + backward of one sequence-layout problem through the C ABI."""
 
     def __init__(self, target, draft, mask, K, mode, T=1.0, wg=1.0, ws=1.0, dloss=1.0, full_windows=False,
-                 wkl=1.0):
-        self.prob = aal.seq_problem(draft, K, mode, T, wg, ws, full_windows, wkl)
+                 wkl=1.0, wtv=1.0):
+        self.prob = aal.seq_problem(draft, K, mode, T, wg, ws, full_windows, wkl, wtv)
         self.ws_buf = torch.empty(aal.aal_seq_workspace_size(self.prob), dtype=torch.uint8,
                                   device=draft.device)
         R = draft.shape[0] * draft.shape[1]
@@ -138,13 +145,13 @@ class SeqRun:
 
 
 def seq_grad_tolerance(target, draft, mask, K, omode, T, wg, ws, dloss, gref, nvalid_total,
-                       full_windows=False):
+                       full_windows=False, wtv=0.0):
     """Per-position tolerance: GRAD_ATOL + GRAD_RTOL |g_ref| plus the near-tie widening of every
     window row the position contributes to."""
     wp, wq, wm, src = oracle.gather_windows(target, draft, mask, K, full_windows)
     fw = oracle.loss_forward(wp, wq, wm, omode, T, wg, ws, nvalid_total)
     widen = grad_tolerance(wp, wq, wm, omode, T, wg, ws, dloss, np.zeros(wq.shape), nvalid_total,
-                           fw) - GRAD_ATOL
+                           fw, wtv) - GRAD_ATOL
     Bq, Tq, V = gref.shape
     extra = np.zeros((Bq * Tq, V))
     for n, j in np.argwhere(src >= 0):
@@ -161,12 +168,13 @@ def _assert_grad(g, gref, tol, where=""):
 
 
 def check_seq_loss(run: SeqRun, target, draft, mask, K, mode, T, wg, ws, dloss=1.0, full_windows=False,
-                   wkl=1.0):
+                   wkl=1.0, wtv=1.0):
     """Every output of a sequence-layout run against the oracle on all positions."""
     omode = ORACLE_MODES[mode]
     t_h, d_h = target.cpu(), draft.cpu()
     m_h = None if mask is None else mask.cpu().numpy()
-    fw = oracle.seq_objective_forward(t_h, d_h, m_h, K, omode, T, wg, ws, wkl, full_windows=full_windows)
+    fw = oracle.seq_objective_forward(t_h, d_h, m_h, K, omode, T, wg, ws, wkl, full_windows=full_windows,
+                                      w_tv=wtv)
     eal = run.eal.cpu().numpy()
     if omode & oracle.MODE_GREEDY:
         np.testing.assert_allclose(eal[:, 0], fw["eal_g"], rtol=LOSS_RTOL, atol=LOSS_ATOL)
@@ -175,8 +183,9 @@ def check_seq_loss(run: SeqRun, target, draft, mask, K, mode, T, wg, ws, dloss=1
     got, ref = float(run.loss.item()), fw["loss"]
     assert abs(got - ref) <= LOSS_RTOL * abs(ref) + LOSS_ATOL, (got, ref)
     gref = oracle.seq_objective_backward(t_h, d_h, m_h, K, omode, T, wg, ws, wkl, dloss,
-                                         full_windows=full_windows)
-    tol = seq_grad_tolerance(t_h, d_h, m_h, K, omode, T, wg, ws, dloss, gref, fw["nvalid"], full_windows)
+                                         full_windows=full_windows, w_tv=wtv)
+    tol = seq_grad_tolerance(t_h, d_h, m_h, K, omode, T, wg, ws, dloss, gref, fw["nvalid"], full_windows,
+                             wtv if omode & oracle.MODE_TV else 0.0)
     _assert_grad(run.grad.cpu().double().numpy(), gref, tol)
     return fw
 

@@ -41,7 +41,7 @@ def test_library_exports_every_declared_symbol():
 
 
 def test_status_strings_and_version():
-    assert aal.aal_abi_version() == 10100
+    assert aal.aal_abi_version() == 10200
     for code in range(6):
         assert aal.aal_status_string(code).startswith("AAL_")
     assert aal.aal_status_string(99) == "unknown aal_status"
@@ -49,7 +49,7 @@ def test_status_strings_and_version():
 
 def _prob(**kw):
     d = dict(N=4, K=3, V=100, dtype=aal.AAL_BF16, mode=aal.AAL_BOTH, temperature=1.0,
-             w_greedy=0.5, w_sampling=0.5, w_kl=1.0, reserved=0)
+             w_greedy=0.5, w_sampling=0.5, w_kl=1.0, w_tv=0.1, reserved=0)
     d.update(kw)
     return aal.AalProblem(**d)
 
@@ -73,7 +73,10 @@ def test_workspace_size_grows_with_rows():
     (dict(N=-1), aal.AAL_ERR_INVALID_ARG),
     (dict(dtype=7), aal.AAL_ERR_INVALID_ARG),
     (dict(mode=0), aal.AAL_ERR_INVALID_ARG),
-    (dict(mode=16), aal.AAL_ERR_INVALID_ARG),
+    (dict(mode=32), aal.AAL_ERR_INVALID_ARG),
+    (dict(mode=aal.AAL_KL | aal.AAL_TV), aal.AAL_OK),
+    (dict(mode=aal.AAL_TV, temperature=0.0), aal.AAL_ERR_INVALID_ARG),
+    (dict(w_tv=float("inf")), aal.AAL_ERR_INVALID_ARG),
     (dict(mode=aal.AAL_GRPO | aal.AAL_KL | aal.AAL_GREEDY), aal.AAL_OK),
     (dict(mode=-1), aal.AAL_ERR_INVALID_ARG),
     (dict(w_kl=float("nan")), aal.AAL_ERR_INVALID_ARG),
@@ -172,7 +175,7 @@ def test_reward_from_loss_argument_checks():
 
 def _sprob(**kw):
     d = dict(B=2, seq_len=16, K=4, V=100, dtype=aal.AAL_BF16, mode=aal.AAL_BOTH, temperature=1.0,
-             w_greedy=0.5, w_sampling=0.5, w_kl=1.0, full_windows=0, reserved=0)
+             w_greedy=0.5, w_sampling=0.5, w_kl=1.0, w_tv=0.1, full_windows=0, reserved=0)
     d.update(kw)
     return aal.AalSeqProblem(**d)
 

@@ -125,3 +125,49 @@ def test_sequence_full_size_sampled_positions():
                         seq_window_counts(mask, B, Tn), wkl=1.0, npos_total=npos)
     dead = torch.from_numpy(m == 0).to(DEV)
     assert torch.count_nonzero(run.grad[dead]).item() == 0
+
+
+# ------------------------------------------------------------------ the L_TV baseline term (AAL_TV)
+
+KL_TV = aal.AAL_KL | aal.AAL_TV
+
+
+@pytest.mark.parametrize("mode,T,wtv", [
+    (KL_TV, 1.0, 0.1),                                # the paper's L_KL + 0.1 L_TV baseline, T = 1
+    (KL_TV, 0.7, 0.1),                                # ... at T = 0.7 (generic kernel: anchor beside T != 1)
+    (aal.AAL_TV, 1.3, 1.0),                           # the TV term alone
+    (aal.AAL_TV | aal.AAL_BOTH, 1.0, 0.5),            # beside EAL and WTV: one sampling coefficient
+])
+@pytest.mark.parametrize("masked", [False, True])
+def test_tv_term_tiny_all_rows(mode, T, wtv, masked):
+    target, draft, _ = synth.make_logits("tiny", seed=31)
+    mask = None
+    if masked:
+        mask = torch.ones(32, 4, dtype=torch.uint8)
+        mask[2, 1] = 0
+        mask[6, 0] = 0
+        mask[7, 3] = 0
+    t, d, m = _dev(target, draft, mask)
+    dloss = 32.0 * 4
+    run = LossRun(t, d, m, mode, T, 0.3, 0.6, dloss=dloss, wkl=1.0, wtv=wtv)
+    check_loss(run, t, d, m, mode, T, 0.3, 0.6, dloss=dloss, wkl=1.0, wtv=wtv)
+
+
+@pytest.mark.parametrize("V,dtype", [(4104, torch.bfloat16), (4099, torch.float32)])
+def test_tv_term_sequence_layout(V, dtype):
+    target, draft, _ = synth.make_seq_logits("seq_tiny", seed=17, B=2, seq_len=13, V=V, dtype=dtype, masked=False)
+    mask = torch.ones(2, 13, dtype=torch.uint8)
+    mask[1, 9:] = 0
+    t, d, m = _dev(target, draft, mask)
+    for full in (False, True):
+        run = SeqRun(t, d, m, 4, KL_TV, 0.9, 0.0, 0.0, dloss=24.0, full_windows=full, wkl=1.0, wtv=0.1)
+        check_seq_loss(run, t, d, m, 4, KL_TV, 0.9, 0.0, 0.0, dloss=24.0, full_windows=full, wkl=1.0, wtv=0.1)
+
+
+def test_tv_baseline_full_size_sampled_windows():
+    """N = 8192 windows, K = 7, V = 128256 bf16 under L_KL + 0.1 L_TV at T = 1."""
+    target, draft, _ = synth.make_logits("v128k", seed=2, device=DEV)
+    N, K, V = draft.shape
+    run = LossRun(target, draft, None, KL_TV, 1.0, 0.0, 0.0, dloss=float(N * K), wkl=1.0, wtv=0.1)
+    check_loss(run, target, draft, None, KL_TV, 1.0, 0.0, 0.0, dloss=float(N * K), windows=[0, 3000, 8191],
+               n_windows_total=N, wkl=1.0, n_positions_total=N * K, wtv=0.1)
