@@ -140,7 +140,7 @@ def _weights(mode: int, w_greedy: float, w_sampling: float):
 
 
 def loss_forward(target, draft, mask=None, mode: int = MODE_BOTH, T: float = 1.0,
-                 w_greedy: float = 1.0, w_sampling: float = 1.0, n_windows_total=None):
+                 w_greedy: float = 1.0, w_sampling: float = 1.0, n_windows_total=None, xstar=None):
     """The EAL and WTV losses, Eq. loss_eal (Sec. 3.2) and Eq. loss_tv (Sec. 3.3).
 
     L_EAL = -(1/|W|) sum_t sum_k prod_{j<k} a^greedy_{t+j}
@@ -152,14 +152,28 @@ def loss_forward(target, draft, mask=None, mode: int = MODE_BOTH, T: float = 1.0
     overrides |W| when only some windows of a larger batch are passed in.
     Returns a dict with the loss, the per-window expected lengths and the
     per-position acceptances.
+
+    ``xstar`` ([N][K] token ids) gives the target's tokens directly (Sec. 3.2: for greedy
+    target-generated data x* is the ground-truth token); the target logits are then not
+    needed (``target`` may be None) and only the greedy term is defined.
     """
-    zp = as_f64(target)
     zq = as_f64(draft)
-    N, K, V = zp.shape
+    if xstar is not None:
+        if mode & MODE_SAMPLING:
+            raise ValueError("token ids define the greedy term only")
+        zp = None
+        N, K, V = zq.shape
+    else:
+        zp = as_f64(target)
+        N, K, V = zp.shape
     kn = leading_valid_depths(mask, N, K)
     nvalid = int(np.sum(kn >= 1)) if n_windows_total is None else int(n_windows_total)
     wg, ws = _weights(mode, w_greedy, w_sampling)
-    a_g, xstar = acceptance_greedy(zp, zq)
+    if xstar is None:
+        a_g, xstar = acceptance_greedy(zp, zq)
+    else:
+        xstar = np.asarray(xstar, dtype=np.int64).reshape(N, K)
+        a_g = np.exp(np.take_along_axis(log_softmax(zq, 1.0), xstar[..., None], axis=-1)[..., 0])
     eal_g = expected_length(a_g, kn) if mode & MODE_GREEDY else np.zeros(N)
     if mode & MODE_SAMPLING:
         a_s = acceptance_sampling(zp, zq, T)
@@ -177,7 +191,7 @@ def loss_forward(target, draft, mask=None, mode: int = MODE_BOTH, T: float = 1.0
 
 def loss_backward(target, draft, mask=None, mode: int = MODE_BOTH, T: float = 1.0,
                   w_greedy: float = 1.0, w_sampling: float = 1.0, dloss: float = 1.0,
-                  n_windows_total=None) -> np.ndarray:
+                  n_windows_total=None, xstar=None) -> np.ndarray:
     """dloss * dL/dz_q for every draft logit, [N][K][V] float64.
 
     The target is frozen (Sec. 3.2, 3.3): only the draft logits get a gradient.
@@ -194,10 +208,9 @@ def loss_backward(target, draft, mask=None, mode: int = MODE_BOTH, T: float = 1.
     at a tie q~_v = p~_v the min is taken to follow the frozen p~, so c_v = 0 there.
     The comparison is made on log-probabilities.
     """
-    zp = as_f64(target)
     zq = as_f64(draft)
-    N, K, V = zp.shape
-    fw = loss_forward(target, draft, mask, mode, T, w_greedy, w_sampling, n_windows_total)
+    N, K, V = zq.shape
+    fw = loss_forward(target, draft, mask, mode, T, w_greedy, w_sampling, n_windows_total, xstar)
     nvalid, kn = fw["nvalid"], fw["kn"]
     grad = np.zeros((N, K, V), dtype=np.float64)
     if nvalid == 0:
@@ -213,7 +226,7 @@ def loss_backward(target, draft, mask=None, mode: int = MODE_BOTH, T: float = 1.
         grad += scale * wg * dEg[..., None] * da_g
     if mode & MODE_SAMPLING:
         dEs = expected_length_partials(fw["a_s"], kn)
-        lp = log_softmax(zp, T)
+        lp = log_softmax(as_f64(target), T)
         lq = log_softmax(zq, T)
         qt = np.exp(lq)
         c = (lq < lp).astype(np.float64)

@@ -49,24 +49,39 @@ def gather_windows(target, draft, mask, K: int, full_windows: bool = False):
     return wp, wq, wm, src
 
 
+def _window_ids(xstar, src):
+    """[B][T] token ids -> the [B*T][K] ids of every window row (0 outside the sequence)."""
+    flat = np.asarray(xstar, dtype=np.int64).reshape(-1)
+    return np.where(src >= 0, flat[np.maximum(src, 0)], 0)
+
+
 def seq_loss_forward(target, draft, mask, K: int, mode: int = MODE_BOTH, T: float = 1.0,
                      w_greedy: float = 1.0, w_sampling: float = 1.0, n_windows_total=None,
-                     full_windows: bool = False):
+                     full_windows: bool = False, xstar=None):
     """The loss over every sliding window of every sequence (see the module docstring).
-    ``n_windows_total`` replaces |W| when the sequences given are a slice of a larger batch."""
-    wp, wq, wm, _ = gather_windows(target, draft, mask, K, full_windows)
-    return loss_forward(wp, wq, wm, mode, T, w_greedy, w_sampling, n_windows_total)
+    ``n_windows_total`` replaces |W| when the sequences given are a slice of a larger batch;
+    ``xstar`` ([B][T] token ids) replaces the target's argmax (greedy term only)."""
+    if xstar is not None:
+        target = np.zeros(as_f64(draft).shape)   # not read: the ids define x*
+    wp, wq, wm, src = gather_windows(target, draft, mask, K, full_windows)
+    ids = None if xstar is None else _window_ids(xstar, src)
+    return loss_forward(None if ids is not None else wp, wq, wm, mode, T, w_greedy, w_sampling,
+                        n_windows_total, ids)
 
 
 def seq_loss_backward(target, draft, mask, K: int, mode: int = MODE_BOTH, T: float = 1.0,
                       w_greedy: float = 1.0, w_sampling: float = 1.0, dloss: float = 1.0,
-                      n_windows_total=None, full_windows: bool = False) -> np.ndarray:
+                      n_windows_total=None, full_windows: bool = False, xstar=None) -> np.ndarray:
     """dloss * dL/dz_q per position, [B][T][V]: the window rows' gradients added back to the
     positions they were gathered from (|W| replaced by ``n_windows_total`` when given)."""
     zq = as_f64(draft)
     B, Tn, V = zq.shape
+    if xstar is not None:
+        target = np.zeros(zq.shape)
     wp, wq, wm, src = gather_windows(target, draft, mask, K, full_windows)
-    g = loss_backward(wp, wq, wm, mode, T, w_greedy, w_sampling, dloss, n_windows_total)
+    ids = None if xstar is None else _window_ids(xstar, src)
+    g = loss_backward(None if ids is not None else wp, wq, wm, mode, T, w_greedy, w_sampling, dloss,
+                      n_windows_total, ids)
     out = np.zeros((B * Tn, V))
     for n in range(B * Tn):
         for j in range(K):

@@ -311,3 +311,41 @@ def test_gradient_matches_central_differences(K, mode, T):
         fd = 2.0 * (oracle.loss_forward(zp, zplus, mask, **kw)["loss"]
                     - oracle.loss_forward(zp, zminus, mask, **kw)["loss"]) / (2 * h)
         assert abs(fd - g[idx]) < 1e-7, (idx, fd, g[idx])
+
+
+# ------------------------------------------------------------------ target token ids
+
+def test_token_ids_equal_a_target_peaked_on_them():
+    """x* given as ids (Sec. 3.2: the ground-truth token of greedy target-generated data) is
+    the same as target logits whose argmax is that id: a +60 peak on zero logits."""
+    rng = np.random.default_rng(40)
+    N, K, V = 3, 4, 11
+    zq = rng.normal(0, 2, size=(N, K, V))
+    ids = rng.integers(0, V, size=(N, K))
+    zp = np.zeros((N, K, V))
+    np.put_along_axis(zp, ids[..., None], 60.0, axis=-1)
+    mask = np.ones((N, K), dtype=np.uint8)
+    mask[1, 2] = 0
+    a = oracle.loss_forward(None, zq, mask, oracle.MODE_GREEDY, 1.0, 0.7, 0.0, xstar=ids)
+    b = oracle.loss_forward(zp, zq, mask, oracle.MODE_GREEDY, 1.0, 0.7, 0.0)
+    assert abs(a["loss"] - b["loss"]) < 1e-15 and np.array_equal(a["xstar"], ids)
+    ga = oracle.loss_backward(None, zq, mask, oracle.MODE_GREEDY, 1.0, 0.7, 0.0, 2.0, xstar=ids)
+    gb = oracle.loss_backward(zp, zq, mask, oracle.MODE_GREEDY, 1.0, 0.7, 0.0, 2.0)
+    np.testing.assert_array_equal(ga, gb)
+    with pytest.raises(ValueError):
+        oracle.loss_forward(None, zq, mask, oracle.MODE_BOTH, 1.0, xstar=ids)
+
+
+def test_token_id_gradient_by_finite_differences():
+    rng = np.random.default_rng(41)
+    N, K, V = 2, 3, 7
+    zq = rng.normal(0, 1.5, size=(N, K, V))
+    ids = rng.integers(0, V, size=(N, K))
+    g = oracle.loss_backward(None, zq, None, oracle.MODE_GREEDY, 1.0, 1.0, 0.0, 3.0, xstar=ids)
+    h = 1e-6
+    for idx in np.ndindex(N, K, V):
+        a = zq.copy(); a[idx] += h
+        b = zq.copy(); b[idx] -= h
+        fd = 3.0 * (oracle.loss_forward(None, a, None, 1, 1.0, 1.0, 0.0, xstar=ids)["loss"]
+                    - oracle.loss_forward(None, b, None, 1, 1.0, 1.0, 0.0, xstar=ids)["loss"]) / (2 * h)
+        assert abs(fd - g[idx]) < 1e-8

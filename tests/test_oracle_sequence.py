@@ -162,3 +162,19 @@ def test_sequence_tv_term_by_finite_differences():
         fd = 2.0 * (oracle.seq_objective_forward(zp, a, mask, K, **kw)["loss"]
                     - oracle.seq_objective_forward(zp, b, mask, K, **kw)["loss"]) / (2 * h)
         assert abs(fd - g[idx]) < 1e-7, (idx, fd, g[idx])
+
+
+def test_sequence_token_ids_equal_a_peaked_target():
+    rng = np.random.default_rng(9)
+    B, Tn, K, V = 2, 6, 3, 8
+    zq = rng.normal(0, 2, size=(B, Tn, V))
+    ids = rng.integers(0, V, size=(B, Tn))
+    zp = np.zeros((B, Tn, V))
+    np.put_along_axis(zp, ids[..., None], 60.0, axis=-1)
+    mask = np.ones((B, Tn), dtype=np.uint8)
+    mask[1, 4] = 0
+    a = seq_loss_forward(None, zq, mask, K, oracle.MODE_GREEDY, xstar=ids)
+    b = seq_loss_forward(zp, zq, mask, K, oracle.MODE_GREEDY)
+    assert abs(a["loss"] - b["loss"]) < 1e-15
+    np.testing.assert_array_equal(seq_loss_backward(None, zq, mask, K, oracle.MODE_GREEDY, dloss=2.0, xstar=ids),
+                                  seq_loss_backward(zp, zq, mask, K, oracle.MODE_GREEDY, dloss=2.0))
