@@ -55,8 +55,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-seq", action="store_true", help="skip every line beside the step")
-    ap.add_argument("--lines", default="greedy,seq,grpo",
-                    help="lines measured beside the step (comma-separated from greedy, seq, grpo)")
+    ap.add_argument("--lines", default="greedy,ids,seq,grpo",
+                    help="lines measured beside the step (comma-separated from greedy, ids, seq, grpo)")
     ap.add_argument("--windows", type=int, default=None,
                     help="run the first WINDOWS windows of the workload (profiling captures)")
     return ap.parse_args()
@@ -238,6 +238,7 @@ def run_ours(args, ws_count, rank, local):
     lines = set() if args.no_seq else {x.strip() for x in args.lines.split(",") if x.strip()}
     reps = max(5, args.steps // 2)
     greedy_obj = run_greedy_objective(aal, draft, target, grad, stream, reps) if "greedy" in lines else None
+    greedy_ids = run_greedy_ids(aal, draft, target, grad, stream, reps) if "ids" in lines else None
     seq = run_sequence_layout(aal, dev, stream, rank, reps) if "seq" in lines else None
     grpo = run_grpo_phase(aal, dev, stream, rank, reps) if "grpo" in lines else None
 
@@ -290,6 +291,8 @@ def run_ours(args, ws_count, rank, local):
     }
     if greedy_obj is not None:
         res["greedy_objective"] = greedy_obj
+    if greedy_ids is not None:
+        res["greedy_eal_token_ids"] = greedy_ids
     if seq is not None:
         res["sequence_layout"] = seq
     if grpo is not None:
@@ -392,6 +395,32 @@ def run_grpo_phase(aal, dev, stream, rank, reps):
            "bwd_gbs": round(b[2] / (ms[2] * 1e-3) / 1e9, 1), "rows_per_s": round(R / (tot * 1e-3), 1),
            "loss": float(loss.item()), "grpo_loss": float(gloss.item())}
     del target, draft, ref, grad, lws, gws
+    return out
+
+
+def run_greedy_ids(aal, draft, target, grad, stream, reps):
+    """L_EAL with x* given as target token ids (mode AAL_IDS; the ids are the target's argmax,
+    taken once outside the timed region): the forward reads the draft only, the backward reads
+    the draft and writes the gradient."""
+    N, K, V = draft.shape
+    ids = target.float().argmax(-1).to(torch.int32).contiguous() if V * N * K < 2**31 else \
+        torch.cat([target[i:i + 256].float().argmax(-1).to(torch.int32) for i in range(0, N, 256)])
+    prob = aal.loss_problem(draft, aal.AAL_GREEDY | aal.AAL_IDS, 1.0, 1.0, 0.0)
+    ws = torch.empty(aal.aal_workspace_size(prob), dtype=torch.uint8, device=draft.device)
+    loss = torch.empty(1, dtype=torch.float32, device=draft.device)
+    fwd, bwd = _time_fwd_bwd(
+        aal, lambda: aal.aal_loss_fwd(prob, draft, ids, None, ws, loss, None, stream),
+        lambda: aal.aal_loss_bwd(prob, draft, ids, None, ws, 1.0, grad, stream), stream, reps)
+    assert aal.aal_check_device_status(ws) == aal.AAL_OK
+    R = N * K
+    row = V * draft.element_size()
+    fb, bb = R * row + 4 * R, 2 * R * row
+    out = {"workload": f"v128k: N={N} windows, K={K}, V={V} bf16, x* as int32 ids; L_EAL fwd+bwd",
+           "ms": round(fwd + bwd, 4), "fwd_ms": round(fwd, 4), "bwd_ms": round(bwd, 4),
+           "gbs": round((fb + bb) / ((fwd + bwd) * 1e-3) / 1e9, 1),
+           "fwd_gbs": round(fb / (fwd * 1e-3) / 1e9, 1), "bwd_gbs": round(bb / (bwd * 1e-3) / 1e9, 1),
+           "rows_per_s": round(R / ((fwd + bwd) * 1e-3), 1), "loss": float(loss.item())}
+    del ws, ids
     return out
 
 

@@ -74,8 +74,16 @@ typedef enum { AAL_F32 = 0, AAL_BF16 = 1 } aal_dtype;
  * aal_grpo_from_loss).  AAL_TV adds w_tv * L_TV, the auxiliary term of the L_KL + L_TV baseline
  * (Sec. 4.1): each window's TV(p~, q~) = 1 - a^sample averaged over its K_n valid positions, then
  * the mean over W; the baseline L_KL + 0.1 L_TV is mode AAL_KL | AAL_TV with w_tv = 0.1 (T as for
- * the sampling term).  Valid modes: 1 .. 31 (AAL_GRPO only with aal_loss_*). */
-typedef enum { AAL_GREEDY = 1, AAL_SAMPLING = 2, AAL_BOTH = 3, AAL_KL = 4, AAL_GRPO = 8, AAL_TV = 16 } aal_mode;
+ * the sampling term).  AAL_IDS changes what `target` points to: int32 token ids, one per logit row
+ * ([N][K] or [B][seq_len]), taken as x* (Sec. 3.2: for greedy target-generated data x* is the
+ * ground-truth token) instead of target logits; then only the draft is read (half the forward's
+ * bytes, and the greedy backward never reads the target).  It combines with AAL_GREEDY and
+ * AAL_GRPO only (the other terms need p).  An id outside [0, V) records AAL_ERR_INVALID_ARG in the
+ * workspace status word (aal_check_device_status) and that row's a^greedy is 0.
+ * Valid modes: 1 .. 63 (AAL_GRPO only with aal_loss_*). */
+typedef enum {
+  AAL_GREEDY = 1, AAL_SAMPLING = 2, AAL_BOTH = 3, AAL_KL = 4, AAL_GRPO = 8, AAL_TV = 16, AAL_IDS = 32
+} aal_mode;
 
 #define AAL_MAX_K 8
 
@@ -321,8 +329,9 @@ AAL_API aal_status aal_accept_reward_noalloc(const aal_reward_problem* prob, con
                                              int32_t* tau_ref, float* rollout_len, float* advantage,
                                              void* stream);
 
-/* Synchronises `stream`, reads the device status word of a loss or reward workspace,
- * clears it, and returns AAL_OK or the recorded device error (AAL_ERR_TIMEOUT). */
+/* Synchronises `stream`, reads the device status word of a loss, reward or GRPO workspace,
+ * clears it, and returns AAL_OK or the recorded device error: AAL_ERR_TIMEOUT (a bounded wait
+ * ran out) or AAL_ERR_INVALID_ARG (a target token id outside [0, V) under AAL_IDS). */
 AAL_API aal_status aal_check_device_status(void* workspace, void* stream);
 
 /* Static description of a status code; never NULL. */

@@ -21,6 +21,7 @@ from .aal import (  # noqa: F401
     AAL_F32,
     AAL_GREEDY,
     AAL_GRPO,
+    AAL_IDS,
     AAL_KL,
     AAL_MAX_K,
     AAL_NOALLOC_MAX_ROWS,

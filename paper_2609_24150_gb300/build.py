@@ -18,7 +18,8 @@ CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libaal.so")
 SOURCES = ["aal.cu", "rowstats.cu", "rowstats_stream.cu", "window.cu", "backward.cu", "reward.cu",
-           "grpo.cu", "noalloc.cu"]
+           "grpo.cu", "onetensor.cu",
+           "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
          "-Xcompiler", "-fvisibility=hidden", "--extended-lambda"]

@@ -12,6 +12,8 @@ using namespace aal;
 namespace {
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+// target logits start on 16 bytes; target token ids (mode AAL_IDS) on 4
+size_t target_align(int32_t mode) { return (mode & AAL_IDS) ? 4 : 16; }
 
 // Failure-detection test hooks (include/aal_debug.h).
 std::atomic<uint64_t> g_wait_limit_ns{0};
@@ -30,7 +32,9 @@ aal_status check_problem(const aal_problem* p) {
   if (p == nullptr) return AAL_ERR_INVALID_ARG;
   aal_status st = check_shape(p->N, p->K, p->V, p->dtype);
   if (st != AAL_OK) return st;
-  if (p->mode < 1 || p->mode > (AAL_BOTH | AAL_KL | AAL_GRPO | AAL_TV)) return AAL_ERR_INVALID_ARG;
+  if (p->mode < 1 || p->mode > (AAL_BOTH | AAL_KL | AAL_GRPO | AAL_TV | AAL_IDS)) return AAL_ERR_INVALID_ARG;
+  if ((p->mode & AAL_IDS) && ((p->mode & (AAL_SAMPLING | AAL_KL | AAL_TV)) || !(p->mode & (AAL_GREEDY | AAL_GRPO))))
+    return AAL_ERR_INVALID_ARG;  // token ids define x* only: the greedy and GRPO terms
   if ((p->mode & (AAL_SAMPLING | AAL_TV)) && !(isfinite(p->temperature) && p->temperature > 0.f))
     return AAL_ERR_INVALID_ARG;
   if (!isfinite(p->w_greedy) || !isfinite(p->w_sampling) || !isfinite(p->w_kl) || !isfinite(p->w_tv))
@@ -87,9 +91,25 @@ aal_status check_grpo(const aal_grpo_problem* p) {
 
 aal_status cuda_status(cudaError_t e) { return e == cudaSuccess ? AAL_OK : AAL_ERR_CUDA; }
 
-// Per-row statistics of R logit rows (pass over z_p and z_q), shared by both layouts.
+// Per-row statistics of R logit rows (pass over z_p and z_q, or over z_q alone when `target`
+// holds token ids), shared by both layouts.
 cudaError_t launch_stats(const void* draft, const void* target, int64_t R, int64_t V, int32_t dtype,
                          int32_t mode, float temperature, const LossWs& ws, cudaStream_t s, int* cluster) {
+  if (mode & AAL_IDS) {
+    Stream1Args a;
+    a.z = draft;
+    a.R = R;
+    a.V = V;
+    a.lws = ws;
+    a.ids = static_cast<const int32_t*>(target);
+    a.acc = nullptr;
+    a.acc_ref = nullptr;
+    a.lpr = nullptr;
+    a.hdr = ws.hdr;
+    *cluster = 1;
+    (void)debug_take_skip_chunk();  // (the ring test hook applies to the two-tensor forward only)
+    return launch_one_tensor(a, dtype == AAL_BF16, true, s);
+  }
   const bool greedy = (mode & AAL_GREEDY) != 0;
   const bool sampling = (mode & (AAL_SAMPLING | AAL_TV)) != 0;  // both need a^sample
   const bool kl = (mode & AAL_KL) != 0;
@@ -148,7 +168,7 @@ int64_t debug_take_skip_chunk() { return g_skip_chunk.exchange(-1); }
 
 extern "C" {
 
-int32_t aal_abi_version(void) { return 10200; }
+int32_t aal_abi_version(void) { return 10300; }
 
 void aal_debug_fail_next_forward(int64_t chunk, uint64_t wait_limit_ns) {
   g_wait_limit_ns.store(wait_limit_ns);
@@ -191,7 +211,7 @@ aal_status aal_loss_fwd(const aal_problem* prob, const void* draft, const void* 
   if (loss == nullptr || !aligned(loss, 4) || (eal != nullptr && !aligned(eal, 4))) return AAL_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (prob->N == 0) return cuda_status(cudaMemsetAsync(loss, 0, sizeof(float), s));
-  if (draft == nullptr || target == nullptr || !aligned(draft, 16) || !aligned(target, 16))
+  if (draft == nullptr || target == nullptr || !aligned(draft, 16) || !aligned(target, target_align(prob->mode)))
     return AAL_ERR_INVALID_ARG;
   const LossLayout L = loss_layout(prob->N, prob->K);
   if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < L.total) return AAL_ERR_WORKSPACE;
@@ -238,7 +258,7 @@ aal_status aal_loss_bwd(const aal_problem* prob, const void* draft, const void* 
   if (!isfinite(dloss)) return AAL_ERR_INVALID_ARG;
   if (prob->N == 0) return AAL_OK;
   if (draft == nullptr || target == nullptr || grad_draft == nullptr || !aligned(draft, 16) ||
-      !aligned(target, 16) || !aligned(grad_draft, 16))
+      !aligned(target, target_align(prob->mode)) || !aligned(grad_draft, 16))
     return AAL_ERR_INVALID_ARG;
   const LossLayout L = loss_layout(prob->N, prob->K);
   if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < L.total) return AAL_ERR_WORKSPACE;
@@ -265,7 +285,7 @@ aal_status aal_seq_loss_fwd(const aal_seq_problem* prob, const void* draft, cons
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int64_t R = prob->B * prob->seq_len;
   if (R == 0) return cuda_status(cudaMemsetAsync(loss, 0, sizeof(float), s));
-  if (draft == nullptr || target == nullptr || !aligned(draft, 16) || !aligned(target, 16))
+  if (draft == nullptr || target == nullptr || !aligned(draft, 16) || !aligned(target, target_align(prob->mode)))
     return AAL_ERR_INVALID_ARG;
   const SeqLayout L = seq_layout(prob->B, prob->seq_len, prob->K);
   if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < L.total) return AAL_ERR_WORKSPACE;
@@ -312,7 +332,7 @@ aal_status aal_seq_loss_bwd(const aal_seq_problem* prob, const void* draft, cons
   const int64_t R = prob->B * prob->seq_len;
   if (R == 0) return AAL_OK;
   if (draft == nullptr || target == nullptr || grad_draft == nullptr || !aligned(draft, 16) ||
-      !aligned(target, 16) || !aligned(grad_draft, 16))
+      !aligned(target, target_align(prob->mode)) || !aligned(grad_draft, 16))
     return AAL_ERR_INVALID_ARG;
   const SeqLayout L = seq_layout(prob->B, prob->seq_len, prob->K);
   if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < L.total) return AAL_ERR_WORKSPACE;
@@ -358,16 +378,17 @@ aal_status aal_grpo_from_loss(const aal_grpo_problem* gprob, const aal_problem* 
   if (cudaMemsetAsync(hdr, 0, sizeof(WsHeader), s) != cudaSuccess) return AAL_ERR_CUDA;
   const LossWs lws = loss_ws(loss_workspace, LL);
 
-  GrpoRefArgs ra;
-  ra.zr = ref_draft;
+  Stream1Args ra;
+  ra.z = ref_draft;
   ra.R = L.R;
   ra.V = gprob->V;
   ra.lws = lws;
+  ra.ids = nullptr;
   ra.acc = reinterpret_cast<uint8_t*>(base + L.acc);
   ra.acc_ref = reinterpret_cast<uint8_t*>(base + L.acc_ref);
   ra.lpr = reinterpret_cast<float*>(base + L.lpr);
   ra.hdr = hdr;
-  if (launch_grpo_ref_rows(ra, gprob->dtype == AAL_BF16, s) != cudaSuccess) return AAL_ERR_CUDA;
+  if (launch_one_tensor(ra, gprob->dtype == AAL_BF16, false, s) != cudaSuccess) return AAL_ERR_CUDA;
 
   float* adv = advantage != nullptr ? advantage : reinterpret_cast<float*>(base + L.adv);
   RewardGroupArgs ga;
@@ -522,7 +543,9 @@ aal_status aal_check_device_status(void* workspace, void* stream) {
   if (cudaMemcpy(&word, &hdr->status, sizeof(word), cudaMemcpyDeviceToHost) != cudaSuccess) return AAL_ERR_CUDA;
   if (word == 0) return AAL_OK;
   if (cudaMemset(&hdr->status, 0, sizeof(word)) != cudaSuccess) return AAL_ERR_CUDA;
-  return word == kStatusTimeout ? AAL_ERR_TIMEOUT : AAL_ERR_CUDA;
+  if (word == kStatusTimeout) return AAL_ERR_TIMEOUT;
+  if (word == (uint32_t)AAL_ERR_INVALID_ARG) return AAL_ERR_INVALID_ARG;  // a token id outside [0, V)
+  return AAL_ERR_CUDA;
 }
 
 }  // extern "C"

@@ -315,16 +315,18 @@ inline GrpoLayout grpo_layout(int64_t N, int64_t K, int64_t wpr) {
   return L;
 }
 
-// Reference-draft pass: per row, log pi_ref at the draft's greedy token y (from the loss
-// workspace) and whether the reference's own greedy token matches x*.
-struct GrpoRefArgs {
-  const void* zr;      // reference draft logits [R][V]
+// One pass over the rows of a single tensor (onetensor.cu).  REF: the GRPO reference-draft
+// pass, log pi_ref at the draft's greedy token y (from the loss workspace) and both
+// acceptance flags.  IDS: the loss forward with x* given as token ids (only the draft read).
+struct Stream1Args {
+  const void* z;       // [R][V] logits: the reference draft (REF) or the draft (IDS)
   int64_t R, V;
-  LossWs lws;          // x*, y of the loss forward
-  uint8_t* acc;        // [R] y == x*
-  uint8_t* acc_ref;    // [R] argmax z_ref == x*
-  float* lpr;          // [R] log pi_ref(y)
-  WsHeader* hdr;       // status word for the streamed pass's bounded waits
+  LossWs lws;          // REF: x*, y of the loss forward; IDS: the statistics written
+  const int32_t* ids;  // IDS: [R] target token ids
+  uint8_t* acc;        // REF: [R] y == x*
+  uint8_t* acc_ref;    // REF: [R] argmax z_ref == x*
+  float* lpr;          // REF: [R] log pi_ref(y)
+  WsHeader* hdr;       // status word (bounded waits; out-of-range ids)
 };
 
 // Per window: log rho, the clipped surrogate, its per-row gradient coefficients.
@@ -357,7 +359,7 @@ cudaError_t launch_backward(const BackwardArgs& a, bool bf16, cudaStream_t s);
 cudaError_t launch_reward_rows(const RewardRowArgs& a, bool bf16, cudaStream_t s);
 cudaError_t launch_reward_groups(const RewardGroupArgs& a, cudaStream_t s);
 cudaError_t launch_reward_flags_from_stats(const RewardStatsArgs& a, cudaStream_t s);
-cudaError_t launch_grpo_ref_rows(const GrpoRefArgs& a, bool bf16, cudaStream_t s);
+cudaError_t launch_one_tensor(const Stream1Args& a, bool bf16, bool ids, cudaStream_t s);
 cudaError_t launch_grpo_windows(const GrpoWindowArgs& a, cudaStream_t s);
 
 // ---------------------------------------------------------------------------

@@ -117,7 +117,7 @@ __global__ void __launch_bounds__(kBwdThreads) backward_kernel(BackwardArgs a) {
     const float ck = (KL && (a.mask == nullptr || a.mask[r] != 0)) ? kscale : 0.f;
     T* out = static_cast<T*>(a.grad) + r * a.V;
     const T* zq = static_cast<const T*>(a.zq) + r * a.V;
-    const T* zp = static_cast<const T*>(a.zp) + r * a.V;
+    const T* zp = READ_P ? static_cast<const T*>(a.zp) + r * a.V : nullptr;  // (token ids otherwise)
     if (gg == 0.f && gs == 0.f && ck == 0.f && cg == 0.f) {
       if (VEC) {
         uint4* o4 = reinterpret_cast<uint4*>(out);
@@ -221,8 +221,10 @@ cudaError_t dispatch_mode(const BackwardArgs& a, cudaStream_t s) {
 
 template <typename T>
 cudaError_t dispatch(const BackwardArgs& a, cudaStream_t s) {
+  // z_p is read only by the sampling term and the anchor (and may be token ids otherwise)
+  const bool reads_p = a.w_sampling != 0.f || a.w_kl != 0.f;
   const bool vec = ((a.V * (int64_t)sizeof(T)) % 16 == 0) &&
-                   ((reinterpret_cast<uintptr_t>(a.zq) | reinterpret_cast<uintptr_t>(a.zp) |
+                   ((reinterpret_cast<uintptr_t>(a.zq) | (reads_p ? reinterpret_cast<uintptr_t>(a.zp) : 0) |
                      reinterpret_cast<uintptr_t>(a.grad)) % 16 == 0);
   if (a.w_kl != 0.f) return vec ? dispatch_mode<T, true, true>(a, s) : dispatch_mode<T, false, true>(a, s);
   return vec ? dispatch_mode<T, true, false>(a, s) : dispatch_mode<T, false, false>(a, s);

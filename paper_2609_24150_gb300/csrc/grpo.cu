@@ -4,10 +4,9 @@
 // the draft's greedy token y = S_k = argmax z_theta and the draft's T = 1 normaliser, so
 // log pi_theta(y) = -ln 2 * Ls_q1 (y is where z_theta peaks).  What is left needs the
 // reference draft only:
-//   grpo_ref_rows   one pass over z_ref: its normaliser, its own greedy token (for tau^ref)
-//                   and z_ref(y), giving log pi_ref(y) and both acceptance flags.  Rows whose
-//                   byte length is a multiple of 16 are streamed through a shared-memory ring
-//                   by TMA (grpo_ref_stream); the others take a plain vectorised loop;
+//   one-tensor pass one pass over z_ref (onetensor.cu, mode REF): its normaliser, its own
+//                   greedy token (for tau^ref) and z_ref(y), giving log pi_ref(y) and both
+//                   acceptance flags;
 //   reward_groups   tau, tau^ref, R = tau - tau^ref, rollout means, clipped advantages
 //                   (the kernel of aal_accept_reward);
 //   grpo_windows    per window: log rho = (1/K) sum_k [log pi_theta(y_k) - log pi_ref(y_k)]
@@ -18,397 +17,10 @@
 //                   term is the minimum and every clip is inside, else 0.
 // The group loss is the mean over a group's windows and L_GRPO the mean over equal-sized
 // groups, which is -(1/N) sum_t surrogate_t.
-#include "ptx.cuh"
+#include "aal_internal.cuh"
 
 namespace aal {
 namespace {
-
-using namespace ptx;
-
-constexpr int kRefThreads = 256;
-
-template <typename T>
-struct RefVec;
-template <>
-struct RefVec<float> {
-  static constexpr int E = 4;
-  __device__ static void unpack(const uint4& w, float* o) {
-    o[0] = __uint_as_float(w.x);
-    o[1] = __uint_as_float(w.y);
-    o[2] = __uint_as_float(w.z);
-    o[3] = __uint_as_float(w.w);
-  }
-};
-template <>
-struct RefVec<uint16_t> {
-  static constexpr int E = 8;
-  __device__ static void unpack(const uint4& w, float* o) {
-    o[0] = bf16_lo(w.x);
-    o[1] = bf16_hi(w.x);
-    o[2] = bf16_lo(w.y);
-    o[3] = bf16_hi(w.y);
-    o[4] = bf16_lo(w.z);
-    o[5] = bf16_hi(w.z);
-    o[6] = bf16_lo(w.w);
-    o[7] = bf16_hi(w.w);
-  }
-};
-
-struct RefAcc {
-  Lse l;
-  Amax am;
-};
-
-__device__ __forceinline__ void ref_push(RefAcc& a, int64_t v, float z) {
-  if (z > a.am.v) {
-    a.am.v = z;
-    a.am.i = (int32_t)v;
-  }
-  lse_push(a.l, z, kLog2e);
-}
-
-__device__ __forceinline__ RefAcc ref_merge(const RefAcc& a, const RefAcc& b) {
-  RefAcc r;
-  r.l = lse_merge(a.l, b.l, kLog2e);
-  r.am = amax_merge(a.am, b.am);
-  return r;
-}
-
-__device__ __forceinline__ RefAcc ref_shfl(const RefAcc& a, int off) {
-  RefAcc b;
-  b.l = shfl_lse(a.l, off);
-  b.am = shfl_amax(a.am, off);
-  return b;
-}
-
-// One CTA per row (grid-stride over rows), 16-byte loads, two in flight per thread.
-template <typename T, bool VEC>
-__global__ void __launch_bounds__(kRefThreads) grpo_ref_rows(GrpoRefArgs a) {
-  __shared__ RefAcc red[kRefThreads / 32];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  for (int64_t r = blockIdx.x; r < a.R; r += gridDim.x) {
-    const T* z = static_cast<const T*>(a.zr) + r * a.V;
-    RefAcc acc;
-    lse_init(acc.l);
-    amax_init(acc.am);
-    if (VEC) {
-      constexpr int E = RefVec<T>::E;
-      const int64_t nv = a.V / E;
-      const uint4* z4 = reinterpret_cast<const uint4*>(z);
-      int64_t i = threadIdx.x;
-      for (; i + kRefThreads < nv; i += 2 * kRefThreads) {
-        const uint4 w0 = ldg_stream(z4 + i);
-        const uint4 w1 = ldg_stream(z4 + i + kRefThreads);
-        float f[E];
-        RefVec<T>::unpack(w0, f);
-#pragma unroll
-        for (int e = 0; e < E; ++e) ref_push(acc, i * E + e, f[e]);
-        RefVec<T>::unpack(w1, f);
-#pragma unroll
-        for (int e = 0; e < E; ++e) ref_push(acc, (i + kRefThreads) * E + e, f[e]);
-      }
-      if (i < nv) {
-        float f[E];
-        RefVec<T>::unpack(ldg_stream(z4 + i), f);
-#pragma unroll
-        for (int e = 0; e < E; ++e) ref_push(acc, i * E + e, f[e]);
-      }
-    } else {
-      for (int64_t v = threadIdx.x; v < a.V; v += kRefThreads) ref_push(acc, v, load_elem<T>(z + v));
-    }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) acc = ref_merge(acc, ref_shfl(acc, off));
-    if (lane == 0) red[warp] = acc;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      RefAcc t = red[0];
-      for (int w = 1; w < kRefThreads / 32; ++w) t = ref_merge(t, red[w]);
-      const int32_t y = a.lws.yhat[r], xs = a.lws.xstar[r];
-      // y is a valid index unless the draft row was all -inf (undefined input): read nothing then
-      const float zy = (y >= 0 && (int64_t)y < a.V) ? load_elem<T>(z + y) : -INFINITY;
-      a.lpr[r] = (zy - t.l.M) - kLn2 * lse_ls(t.l);
-      a.acc[r] = (y == xs) ? 1 : 0;
-      a.acc_ref[r] = (t.am.i == xs) ? 1 : 0;
-    }
-    __syncthreads();  // red is reused by the next row
-  }
-}
-
-template <typename T, bool VEC>
-cudaError_t go_ref(const GrpoRefArgs& a, cudaStream_t s) {
-  int dev = 0, sms = 0, per_sm = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, grpo_ref_rows<T, VEC>, kRefThreads, 0);
-  if (per_sm < 1) per_sm = 1;
-  int64_t grid = (int64_t)sms * per_sm;
-  if (grid > a.R) grid = a.R;
-  if (grid < 1) return cudaSuccess;
-  grpo_ref_rows<T, VEC><<<(unsigned)grid, kRefThreads, 0, s>>>(a);
-  return cudaGetLastError();
-}
-
-template <typename T>
-cudaError_t dispatch_ref(const GrpoRefArgs& a, cudaStream_t s) {
-  const bool vec = ((a.V * (int64_t)sizeof(T)) % 16 == 0) && (reinterpret_cast<uintptr_t>(a.zr) % 16 == 0);
-  return vec ? go_ref<T, true>(a, s) : go_ref<T, false>(a, s);
-}
-
-// ---------------------------------------------------------------- streamed reference pass
-// One CTA per SM, persistent over rows.  A producer thread copies each row of z_ref in
-// 48 KB chunks into a 4-slot ring (1-D TMA bulk copies, completion counted on an mbarrier
-// per slot, evict_first: nothing is read twice); 16 consumer warps fold each chunk into
-// an online log2-sum-exp and a per-16-byte-vector running maximum.  y and x* are known
-// before the row starts, so the thread that holds y's vector reads z_ref(y), and the one
-// that holds x*'s vector reads z_ref(x*) and the first position in that vector with the
-// same value.  At the end of the row:
-//   log pi_ref(y) = (z_ref(y) - M) - ln 2 * log2 S,
-//   argmax z_ref == x*  iff  z_ref(x*) = M, the first vector holding M is x*'s, and no
-//                           earlier element of that vector equals z_ref(x*).
-// Every wait is bounded as in the loss forward (status word of the GRPO workspace).
-constexpr int kRSlots = 4;
-constexpr int kRSlotBytes = 48 * 1024;
-constexpr int kRWarps = 16;
-constexpr int kRConsumers = 32 * kRWarps;
-constexpr int kRThreads = 32 + kRConsumers;
-constexpr int kRVecPerChunk = kRSlotBytes / 16;
-constexpr int kRNV = kRVecPerChunk / kRConsumers;
-static_assert(kRNV * kRConsumers == kRVecPerChunk, "consumers must tile a chunk");
-constexpr int kRBarRow = 1;
-
-struct RefPart {
-  float M, S;    // online log2-sum-exp (M = raw max)
-  float av;      // largest value and the first vector (element index) holding it
-  int32_t ab;
-};
-
-struct RefSmem {
-  uint64_t full[kRSlots];
-  uint64_t empty[kRSlots];
-  RefPart red[2][kRWarps];
-  float zy[2], zx[2];   // z_ref(y), z_ref(x*), by row parity
-  int32_t fx[2];        // first index of x*'s vector whose value equals z_ref(x*)
-  int abort_flag;
-};
-
-constexpr float kRefFloor = -1e30f;
-
-__device__ __forceinline__ void refpart_init(RefPart& a) {
-  a.M = kRefFloor;
-  a.S = 0.f;
-  a.av = -INFINITY;
-  a.ab = 0x7fffffff;
-}
-
-__device__ __forceinline__ void refpart_warp(RefPart& a) {
-  float m = a.M;
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
-  float s = a.S * ex2((a.M - m) * kLog2e);
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
-  a.M = m;
-  a.S = s;
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) {
-    const float v2 = __shfl_xor_sync(0xffffffffu, a.av, off);
-    const int32_t i2 = __shfl_xor_sync(0xffffffffu, a.ab, off);
-    if (v2 > a.av || (v2 == a.av && i2 < a.ab)) {
-      a.av = v2;
-      a.ab = i2;
-    }
-  }
-}
-
-// Fold one 16-byte vector (E values, the first at element idx0) into the part.
-template <typename T>
-__device__ __forceinline__ void ref_vec(RefPart& A, const uint4& w, int idx0) {
-  constexpr int E = RefVec<T>::E;
-  float f[E];
-  RefVec<T>::unpack(w, f);
-  float vm = f[0];
-#pragma unroll
-  for (int e = 1; e < E; ++e) vm = fmaxf(vm, f[e]);
-  if (vm > A.av) {
-    A.av = vm;
-    A.ab = idx0;
-  }
-  const float m = fmaxf(A.M, vm);
-  A.S *= ex2((A.M - m) * kLog2e);
-  A.M = m;
-  float acc = 0.f;
-#pragma unroll
-  for (int e = 0; e < E; ++e) acc += ex2((f[e] - m) * kLog2e);
-  A.S += acc;
-}
-
-template <typename T>
-__device__ __forceinline__ float ref_elem(const uint4& w, int e) {
-  constexpr int E = RefVec<T>::E;
-  float f[E];
-  RefVec<T>::unpack(w, f);
-  float v = f[0];
-#pragma unroll
-  for (int k = 1; k < E; ++k)
-    if (k == e) v = f[k];
-  return v;
-}
-
-// The first lane k <= e of the vector whose value equals lane e's.
-template <typename T>
-__device__ __forceinline__ int ref_first_equal(const uint4& w, int e) {
-  constexpr int E = RefVec<T>::E;
-  float f[E];
-  RefVec<T>::unpack(w, f);
-  const float v = ref_elem<T>(w, e);
-  int first = e;
-#pragma unroll
-  for (int k = E - 1; k >= 0; --k)
-    if (k <= e && f[k] == v) first = k;
-  return first;
-}
-
-template <typename T>
-__global__ void __launch_bounds__(kRThreads, 1) grpo_ref_stream(GrpoRefArgs a, WsHeader* hdr, int nch,
-                                                                  uint64_t limit_ns) {
-  extern __shared__ __align__(1024) unsigned char smem[];
-  unsigned char* ring = smem;
-  RefSmem& S = *reinterpret_cast<RefSmem*>(smem + kRSlots * kRSlotBytes);
-  volatile int* abort_flag = &S.abort_flag;
-  constexpr int ES = sizeof(T);
-  constexpr int E = 16 / ES;
-  constexpr int CH = kRSlotBytes / ES;  // elements per chunk
-  const int V = (int)a.V;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-
-  if (threadIdx.x == 0) {
-    for (int k = 0; k < kRSlots; ++k) {
-      mbar_init(&S.full[k], 1);
-      mbar_init(&S.empty[k], kRWarps);
-    }
-    S.abort_flag = 0;
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-  }
-  __syncthreads();
-
-  if (warp == kRWarps) {
-    // ------------------------------------------------------------ producer
-    if (lane == 0) {
-      const uint64_t drop = policy_evict_first();
-      int slot = 0;
-      uint32_t phase = 0, armed = 0, last_phase = 0;
-      for (int64_t r = blockIdx.x; r < a.R && !*abort_flag; r += gridDim.x) {
-        const char* row = static_cast<const char*>(a.zr) + r * a.V * ES;
-        for (int c = 0; c < nch; ++c) {
-          if (!wait_phase(&S.empty[slot], phase ^ 1u, abort_flag, limit_ns, hdr)) break;
-          const int e0 = c * CH;
-          const uint32_t bytes = (uint32_t)(min(CH, V - e0) * ES);
-          mbar_expect_tx(&S.full[slot], bytes);
-          bulk_load(ring + slot * kRSlotBytes, row + (int64_t)e0 * ES, bytes, &S.full[slot], drop);
-          armed |= 1u << slot;
-          last_phase = (last_phase & ~(1u << slot)) | (phase << slot);
-          if (++slot == kRSlots) {
-            slot = 0;
-            phase ^= 1u;
-          }
-        }
-      }
-      for (int k = 0; k < kRSlots; ++k) {  // drain the last copy of every slot
-        if (!(armed & (1u << k))) continue;
-        const uint32_t ph = (last_phase >> k) & 1u;
-        const uint64_t t0 = now_ns();
-        for (uint32_t it = 0; it < kSpinLimit && !mbar_try(&S.full[k], ph, 100000); ++it)
-          if (now_ns() - t0 > limit_ns) break;
-      }
-    }
-  } else {
-    // ------------------------------------------------------------ consumers
-    const int t = threadIdx.x;
-    int slot = 0;
-    uint32_t phase = 0, j = 0;
-    for (int64_t r = blockIdx.x; r < a.R; r += gridDim.x, ++j) {
-      const int32_t y = a.lws.yhat[r], xs = a.lws.xstar[r];
-      // owners of y's and x*'s vectors (none when an index is out of range)
-      const bool y_ok = y >= 0 && y < V, x_ok = xs >= 0 && xs < V;
-      const int cy = y_ok ? y / CH : -1, iy = y_ok ? (y - cy * CH) / E : 0, ey = y_ok ? y % E : 0;
-      const int cx = x_ok ? xs / CH : -1, ix = x_ok ? (xs - cx * CH) / E : 0, ex = x_ok ? xs % E : 0;
-      // S.zy/zx/fx[j & 1] are written by the owners before this row's barrier and read by
-      // thread 0 after it; the owners of row j + 2 write them only after thread 0 has passed
-      // the barrier of row j + 1, so nothing is reset (an absent owner is known from y_ok/x_ok)
-      RefPart A;
-      refpart_init(A);
-      for (int c = 0; c < nch; ++c) {
-        if (wait_phase(&S.full[slot], phase, abort_flag, limit_ns, hdr)) {
-          const int e0 = c * CH;
-          const uint4* Z = reinterpret_cast<const uint4*>(ring + slot * kRSlotBytes);
-          if (e0 + CH <= V) {
-            uint4 w[kRNV];
-#pragma unroll
-            for (int v = 0; v < kRNV; ++v) w[v] = Z[t + v * kRConsumers];
-#pragma unroll
-            for (int v = 0; v < kRNV; ++v) ref_vec<T>(A, w[v], e0 + (t + v * kRConsumers) * E);
-          } else {
-            const int nvec = (V - e0) / E;
-            for (int i = t; i < nvec; i += kRConsumers) ref_vec<T>(A, Z[i], e0 + i * E);
-          }
-          if (c == cy && t == iy % kRConsumers) S.zy[j & 1] = ref_elem<T>(Z[iy], ey);
-          if (c == cx && t == ix % kRConsumers) {
-            S.zx[j & 1] = ref_elem<T>(Z[ix], ex);
-            S.fx[j & 1] = cx * CH + ix * E + ref_first_equal<T>(Z[ix], ex);
-          }
-        }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&S.empty[slot]);
-        if (++slot == kRSlots) {
-          slot = 0;
-          phase ^= 1u;
-        }
-      }
-      refpart_warp(A);
-      if (lane == 0) S.red[j & 1][warp] = A;
-      named_barrier(kRBarRow, kRConsumers);
-      if (t == 0 && !*abort_flag) {
-        RefPart tot = S.red[j & 1][0];
-        for (int w = 1; w < kRWarps; ++w) {
-          const RefPart b = S.red[j & 1][w];
-          const float m = fmaxf(tot.M, b.M);
-          tot.S = tot.S * ex2((tot.M - m) * kLog2e) + b.S * ex2((b.M - m) * kLog2e);
-          tot.M = m;
-          if (b.av > tot.av || (b.av == tot.av && b.ab < tot.ab)) {
-            tot.av = b.av;
-            tot.ab = b.ab;
-          }
-        }
-        const bool first_is_x = x_ok && S.zx[j & 1] == tot.av && tot.ab == xs - ex && S.fx[j & 1] == xs;
-        const float zy = y_ok ? S.zy[j & 1] : -INFINITY;
-        a.lpr[r] = (zy - tot.M) - kLn2 * log2f(tot.S);
-        a.acc[r] = (y == xs) ? 1 : 0;
-        a.acc_ref[r] = first_is_x ? 1 : 0;
-      }
-    }
-  }
-  __syncwarp();
-  __syncthreads();
-}
-
-constexpr size_t kRSmemBytes = (size_t)kRSlots * kRSlotBytes + sizeof(RefSmem);
-
-template <typename T>
-cudaError_t go_ref_stream(const GrpoRefArgs& a, WsHeader* hdr, cudaStream_t s, uint64_t limit_ns) {
-  auto kern = grpo_ref_stream<T>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kRSmemBytes);
-  if (e != cudaSuccess) return e;
-  int dev = 0, sms = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  int64_t grid = sms;
-  if (grid > a.R) grid = a.R;
-  if (grid < 1) return cudaSuccess;
-  const int CH = kRSlotBytes / (int)sizeof(T);
-  const int nch = (int)((a.V + CH - 1) / CH);
-  kern<<<(unsigned)grid, kRThreads, kRSmemBytes, s>>>(a, hdr, nch, limit_ns);
-  return cudaGetLastError();
-}
 
 __global__ void __launch_bounds__(kGrpoThreads) grpo_windows(GrpoWindowArgs a) {
   __shared__ double sm[kGrpoThreads / 32];
@@ -466,17 +78,6 @@ __global__ void __launch_bounds__(kGrpoThreads) grpo_windows(GrpoWindowArgs a) {
 }
 
 }  // namespace
-
-cudaError_t launch_grpo_ref_rows(const GrpoRefArgs& a, bool bf16, cudaStream_t s) {
-  const int64_t elt = bf16 ? 2 : 4;
-  const bool aligned = (a.V * elt) % 16 == 0 && reinterpret_cast<uintptr_t>(a.zr) % 16 == 0;
-  if (aligned && a.hdr != nullptr) {
-    const uint64_t limit = debug_wait_limit_ns();
-    return bf16 ? go_ref_stream<uint16_t>(a, a.hdr, s, limit ? limit : kWaitLimitNs)
-                : go_ref_stream<float>(a, a.hdr, s, limit ? limit : kWaitLimitNs);
-  }
-  return bf16 ? dispatch_ref<uint16_t>(a, s) : dispatch_ref<float>(a, s);
-}
 
 cudaError_t launch_grpo_windows(const GrpoWindowArgs& a, cudaStream_t s) {
   if (a.nblk < 1) return cudaSuccess;

@@ -41,7 +41,7 @@ def test_library_exports_every_declared_symbol():
 
 
 def test_status_strings_and_version():
-    assert aal.aal_abi_version() == 10200
+    assert aal.aal_abi_version() == 10300
     for code in range(6):
         assert aal.aal_status_string(code).startswith("AAL_")
     assert aal.aal_status_string(99) == "unknown aal_status"
@@ -73,7 +73,13 @@ def test_workspace_size_grows_with_rows():
     (dict(N=-1), aal.AAL_ERR_INVALID_ARG),
     (dict(dtype=7), aal.AAL_ERR_INVALID_ARG),
     (dict(mode=0), aal.AAL_ERR_INVALID_ARG),
-    (dict(mode=32), aal.AAL_ERR_INVALID_ARG),
+    (dict(mode=64), aal.AAL_ERR_INVALID_ARG),
+    (dict(mode=aal.AAL_IDS | aal.AAL_GREEDY), aal.AAL_OK),
+    (dict(mode=aal.AAL_IDS | aal.AAL_GRPO), aal.AAL_OK),
+    (dict(mode=aal.AAL_IDS), aal.AAL_ERR_INVALID_ARG),
+    (dict(mode=aal.AAL_IDS | aal.AAL_BOTH), aal.AAL_ERR_INVALID_ARG),
+    (dict(mode=aal.AAL_IDS | aal.AAL_GREEDY | aal.AAL_KL), aal.AAL_ERR_INVALID_ARG),
+    (dict(mode=aal.AAL_IDS | aal.AAL_GREEDY | aal.AAL_TV), aal.AAL_ERR_INVALID_ARG),
     (dict(mode=aal.AAL_KL | aal.AAL_TV), aal.AAL_OK),
     (dict(mode=aal.AAL_TV, temperature=0.0), aal.AAL_ERR_INVALID_ARG),
     (dict(w_tv=float("inf")), aal.AAL_ERR_INVALID_ARG),
