@@ -44,11 +44,14 @@ from .reward import (  # noqa: F401
     debiased_reward,
     greedy_trajectory,
     group_advantages,
+    REWARD_SAMPLED_DRAFT,
     rollout_lengths,
+    sampled_trajectory,
     sampling_accepts,
+    sampling_accepts_at,
     simulated_accept_length,
 )
-from .philox import philox4x32_10, uniform01  # noqa: F401
+from .philox import gumbel_uniforms, philox4x32_10, uniform01  # noqa: F401
 from .sequence import (  # noqa: F401
     gather_windows,
     seq_loss_backward,

@@ -58,3 +58,17 @@ def uniform01(seed: int, window, depth) -> np.ndarray:
                                 seed & 0xFFFFFFFF, (seed >> 32) & 0xFFFFFFFF)
     m = (x0.astype(np.uint64) >> np.uint64(9)).astype(np.float64)
     return (2.0 * m + 1.0) * 2.0 ** -24
+
+
+def gumbel_uniforms(seed: int, window: int, depth: int, V: int) -> np.ndarray:
+    """The V uniforms of the sampled-draft reward's Gumbel-max draw for window n, depth k:
+    element v takes output word v mod 4 of counter (n_lo, n_hi, k, 1 + v div 4) (word 3 = 0 is
+    the acceptance draw's counter, so the two never share a counter), mapped to (0, 1) as
+    uniform01 maps x0."""
+    n = np.uint64(window)
+    c3 = np.arange((V + 3) // 4, dtype=np.uint64) + np.uint64(1)
+    words = philox4x32_10(np.full_like(c3, n & _MASK32), np.full_like(c3, n >> _SH32),
+                          np.full_like(c3, np.uint64(depth)), c3, seed & 0xFFFFFFFF, (seed >> 32) & 0xFFFFFFFF)
+    x = np.stack(words, axis=1).reshape(-1)[:V]            # element v = 4 c + w
+    m = (x.astype(np.uint64) >> np.uint64(9)).astype(np.float64)
+    return (2.0 * m + 1.0) * 2.0 ** -24

@@ -13,10 +13,11 @@ from __future__ import annotations
 import numpy as np
 
 from .losses import argmax_lowest, as_f64, log_softmax
-from .philox import uniform01
+from .philox import gumbel_uniforms, uniform01
 
 REWARD_GREEDY = 1
 REWARD_SAMPLING = 2
+REWARD_SAMPLED_DRAFT = 6   # sampling verification with the drafted token sampled from q~
 
 
 def greedy_trajectory(z) -> np.ndarray:
@@ -41,6 +42,29 @@ def simulated_accept_length(accept: np.ndarray) -> np.ndarray:
             total += prod
         tau[n] = total
     return tau
+
+
+def sampled_trajectory(draft, T: float, seed: int, row_offset: int = 0) -> np.ndarray:
+    """S_k ~ q~_k drawn by the Gumbel-max method: S_k = argmax_v (z_k(v)/T + G_v) with
+    G_v = -log(-log U_v), U_v the counter-based uniforms of gumbel_uniforms for (window
+    row_offset + n, depth k); lowest index on ties.  (Sec. 2.3: under sampling verification the
+    draft samples its token from q~.)"""
+    zq = as_f64(draft)
+    N, K, V = zq.shape
+    S = np.zeros((N, K), dtype=np.int64)
+    for n in range(N):
+        for k in range(K):
+            U = gumbel_uniforms(seed, row_offset + n, k, V)
+            S[n, k] = int(np.argmax(zq[n, k] / T - np.log(-np.log(U))))
+    return S
+
+
+def sampling_accepts_at(target, draft, T: float, u: np.ndarray, S: np.ndarray):
+    """Acceptance of given drafted tokens S under sampling verification: u < min(1, p~(S)/q~(S))."""
+    lp = np.take_along_axis(log_softmax(as_f64(target), T), S[..., None], axis=-1)[..., 0]
+    lq = np.take_along_axis(log_softmax(as_f64(draft), T), S[..., None], axis=-1)[..., 0]
+    thr = np.minimum(1.0, np.exp(lp - lq))
+    return (u < thr).astype(np.int64), thr
 
 
 def sampling_accepts(target, draft, T: float, u: np.ndarray):
@@ -99,7 +123,9 @@ def accept_reward(target, draft, ref_draft=None, mode: int = REWARD_GREEDY, T: f
     """The reward pipeline of Sec. 3.4 for N windows of [K][V] logits.
 
     Greedy: accepted iff S_k = x*_k (draft argmax equals target argmax).
-    Sampling: accepted iff u(seed, row_offset + n, k) < min(1, p~(S_k)/q~(S_k)).
+    Sampling: accepted iff u(seed, row_offset + n, k) < min(1, p~(S_k)/q~(S_k)), with S_k the
+    draft's argmax, or (REWARD_SAMPLED_DRAFT) S_k sampled from q~ by sampled_trajectory; the
+    reference draft's tokens are drawn with the same uniforms.
     The reference draft, when given, is verified the same way with the same
     uniforms.  Returns tau, R, rollout lengths, advantages and (for sampling) the
     acceptance thresholds of both drafts, so a comparison can set aside draws that
@@ -109,7 +135,7 @@ def accept_reward(target, draft, ref_draft=None, mode: int = REWARD_GREEDY, T: f
     N, K, V = zp.shape
     xstar = argmax_lowest(zp)
     u = None
-    if mode == REWARD_SAMPLING:
+    if mode in (REWARD_SAMPLING, REWARD_SAMPLED_DRAFT):
         n_idx = np.arange(N, dtype=np.uint64)[:, None] + np.uint64(row_offset)
         k_idx = np.arange(K, dtype=np.uint64)[None, :]
         u = uniform01(seed, n_idx, k_idx)
@@ -117,6 +143,8 @@ def accept_reward(target, draft, ref_draft=None, mode: int = REWARD_GREEDY, T: f
     def verify(z):
         if mode == REWARD_GREEDY:
             return (greedy_trajectory(z) == xstar).astype(np.int64), None
+        if mode == REWARD_SAMPLED_DRAFT:
+            return sampling_accepts_at(zp, z, T, u, sampled_trajectory(z, T, seed, row_offset))
         return sampling_accepts(zp, z, T, u)
 
     acc, thr = verify(draft)

@@ -178,3 +178,38 @@ def test_uniform_chi_square_and_serial_correlation():
     assert abs(chi2 - (bins - 1)) < 6 * math.sqrt(2 * (bins - 1))
     r = np.corrcoef(u[:-1], u[1:])[0, 1]
     assert abs(r) < 6 / math.sqrt(n)
+
+
+# ------------------------------------------------------------------ sampled draft tokens
+
+def test_gumbel_max_draws_follow_the_scaled_draft_distribution():
+    """S ~ q~ (Sec. 2.3): over 40000 windows with the same logits, the frequencies of the
+    Gumbel-max tokens match q~ within 5 binomial standard deviations per token."""
+    import oracle
+    V, T, n = 6, 0.8, 40000
+    z = np.array([1.0, 0.2, -0.5, 2.0, 0.0, 1.5])
+    draft = np.broadcast_to(z, (n, 1, V))
+    S = oracle.sampled_trajectory(draft, T, seed=123)[:, 0]
+    q = np.exp(oracle.log_softmax(z, T))
+    freq = np.bincount(S, minlength=V) / n
+    assert np.all(np.abs(freq - q) <= 5 * np.sqrt(q * (1 - q) / n)), (freq, q)
+
+
+def test_sampled_draft_reward_has_the_wtv_expected_length():
+    """Accepting a token drawn from q~ with probability min(1, p~/q~) accepts with probability
+    sum_v min(p~, q~) = a^sample at every depth, independently, so the mean of tau over many
+    windows is the WTV expected length sum_k prod_{j<=k} a^s_j."""
+    import oracle
+    rng = np.random.default_rng(5)
+    K, V, T, n = 3, 5, 1.2, 20000
+    zp = rng.normal(0, 1.5, size=(K, V))
+    zq = zp + rng.normal(0, 1.0, size=(K, V))
+    tgt = np.broadcast_to(zp, (n, K, V))
+    dr = np.broadcast_to(zq, (n, K, V))
+    out = oracle.accept_reward(tgt, dr, None, oracle.REWARD_SAMPLED_DRAFT, T=T, seed=9)
+    a = oracle.acceptance_sampling(zp, zq, T)
+    want = sum(np.prod(a[:k + 1]) for k in range(K))
+    tau = out["tau"].astype(np.float64)
+    assert abs(tau.mean() - want) <= 5 * tau.std() / np.sqrt(n), (tau.mean(), want)
+    ref = oracle.accept_reward(tgt, dr, dr, oracle.REWARD_SAMPLED_DRAFT, T=T, seed=9)
+    np.testing.assert_array_equal(ref["tau"], ref["tau_ref"])     # common random numbers
