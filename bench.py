@@ -234,6 +234,16 @@ def run_ours(args, ws_count, rank, local):
     r1.record(stream)
     torch.cuda.synchronize()
     ms_reward_pass = r0.elapsed_time(r1) / reps
+    # the same with the drafted token sampled from q~ (Gumbel-max, one Philox word per entry)
+    sprob = aal.reward_problem(draft, aal.AAL_SAMPLING | aal.AAL_SAMPLED_DRAFT, 1.0, 5.0, 0,
+                               rank_row_offset(rank, N), wpr, RPG)
+    aal.aal_accept_reward(sprob, draft, target, None, rws, tau, None, rl, adv, stream)
+    r0.record(stream)
+    for _ in range(reps):
+        aal.aal_accept_reward(sprob, draft, target, None, rws, tau, None, rl, adv, stream)
+    r1.record(stream)
+    torch.cuda.synchronize()
+    ms_reward_sampled = r0.elapsed_time(r1) / reps
 
     lines = set() if args.no_seq else {x.strip() for x in args.lines.split(",") if x.strip()}
     reps = max(5, args.steps // 2)
@@ -276,6 +286,9 @@ def run_ours(args, ws_count, rank, local):
         "rows_per_s": round(R * ws_count / (ms_step * 1e-3), 1),
         "breakdown_ms": {k: round(v, 4) for k, v in per.items()},
         "breakdown_gbs": {k: round(b[k] / (per[k] * 1e-3) / 1e9, 1) for k in ("fwd", "bwd")},
+        "reward_sampled_draft": {"ms": round(ms_reward_sampled, 4),
+                                 "gbs": round(2 * R * V * 2 / (ms_reward_sampled * 1e-3) / 1e9, 1),
+                                 "note": "aal_accept_reward, AAL_SAMPLING | AAL_SAMPLED_DRAFT at T = 1"},
         "reward_logit_pass": {"ms": round(ms_reward_pass, 4),
                               "gbs": round(2 * R * V * 2 / (ms_reward_pass * 1e-3) / 1e9, 1),
                               "note": "aal_accept_reward streaming draft + target itself"},

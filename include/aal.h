@@ -251,6 +251,10 @@ AAL_API aal_status aal_grpo_from_loss(const aal_grpo_problem* gprob, const aal_p
                                       float* grpo_loss, int32_t* tau, int32_t* tau_ref, float* advantage,
                                       float* log_rho, void* stream);
 
+/* Reward mode flag: with AAL_SAMPLING, the drafted token is drawn from q~ instead of taken as
+ * the draft's argmax (aal_reward_problem.mode = AAL_SAMPLING | AAL_SAMPLED_DRAFT). */
+#define AAL_SAMPLED_DRAFT 4
+
 /* Simulated acceptance reward of the GRPO stage (Sec. 3.4).
  *   N, K, V, dtype       as for the loss; K is the window size gamma (1..AAL_MAX_K).
  *   mode                 AAL_GREEDY: draft token S_k = argmax z_q is accepted iff it
@@ -258,6 +262,12 @@ AAL_API aal_status aal_grpo_from_loss(const aal_grpo_problem* gprob, const aal_p
  *                        AAL_SAMPLING: S_k is accepted iff u < min(1, p~(S_k)/q~(S_k))
  *                        (Sec. 2.3) with u = Philox4x32-10 uniform keyed by
  *                        (seed; window row_offset + n, depth k).
+ *                        AAL_SAMPLING | AAL_SAMPLED_DRAFT: the same acceptance, with S_k drawn
+ *                        from q~ (sampling verification's own draft token) by Gumbel-max:
+ *                        S_k = argmax_v (z_q(v)/T + G_v), G_v = -ln(-ln U_v), U_v = word v mod 4
+ *                        of Philox4x32-10 at counter (n_lo, n_hi, k, 1 + v div 4) mapped like u;
+ *                        the reference draft uses the same G.  Its expected tau is the WTV
+ *                        expected length.  (Not with aal_accept_reward_from_loss.)
  *   temperature          T for AAL_SAMPLING (finite, > 0).
  *   seed, row_offset     Philox key and the global index of window 0 (so a batch can be
  *                        streamed in pieces with the same draws).

@@ -26,6 +26,7 @@ from .aal import (  # noqa: F401
     AAL_MAX_K,
     AAL_NOALLOC_MAX_ROWS,
     AAL_OK,
+    AAL_SAMPLED_DRAFT,
     AAL_SAMPLING,
     AAL_TV,
     AalError,

@@ -25,6 +25,7 @@ AAL_KL = 4          # mode bit: the forward-KL anchor
 AAL_GRPO = 8        # mode bit: the backward adds the GRPO surrogate's gradient
 AAL_TV = 16         # mode bit: the L_TV baseline's window-averaged TV term
 AAL_IDS = 32        # mode bit: `target` holds int32 token ids (x*), not logits
+AAL_SAMPLED_DRAFT = 4   # reward mode flag (with AAL_SAMPLING): the drafted token is drawn from q~
 
 AAL_MAX_K = 8
 AAL_NOALLOC_MAX_ROWS = 1 << 20   # N * K limit of aal_accept_reward_noalloc

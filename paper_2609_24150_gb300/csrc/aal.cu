@@ -47,8 +47,9 @@ aal_status check_reward(const aal_reward_problem* p) {
   if (p == nullptr) return AAL_ERR_INVALID_ARG;
   aal_status st = check_shape(p->N, p->K, p->V, p->dtype);
   if (st != AAL_OK) return st;
-  if (p->mode != AAL_GREEDY && p->mode != AAL_SAMPLING) return AAL_ERR_INVALID_ARG;
-  if (p->mode == AAL_SAMPLING && !(isfinite(p->temperature) && p->temperature > 0.f)) return AAL_ERR_INVALID_ARG;
+  if (p->mode != AAL_GREEDY && p->mode != AAL_SAMPLING && p->mode != (AAL_SAMPLING | AAL_SAMPLED_DRAFT))
+    return AAL_ERR_INVALID_ARG;
+  if ((p->mode & AAL_SAMPLING) && !(isfinite(p->temperature) && p->temperature > 0.f)) return AAL_ERR_INVALID_ARG;
   if (p->windows_per_rollout < 1 || p->rollouts_per_group < 1) return AAL_ERR_INVALID_ARG;
   if (p->windows_per_rollout > INT64_MAX / p->rollouts_per_group) return AAL_ERR_INVALID_ARG;
   if (p->N % (p->windows_per_rollout * p->rollouts_per_group) != 0) return AAL_ERR_INVALID_ARG;
@@ -168,7 +169,7 @@ int64_t debug_take_skip_chunk() { return g_skip_chunk.exchange(-1); }
 
 extern "C" {
 
-int32_t aal_abi_version(void) { return 10300; }
+int32_t aal_abi_version(void) { return 10400; }
 
 void aal_debug_fail_next_forward(int64_t chunk, uint64_t wait_limit_ns) {
   g_wait_limit_ns.store(wait_limit_ns);
@@ -445,8 +446,9 @@ aal_status aal_accept_reward(const aal_reward_problem* prob, const void* draft, 
   WsHeader* hdr = reinterpret_cast<WsHeader*>(base + L.hdr);
   if (cudaMemsetAsync(hdr, 0, sizeof(WsHeader), s) != cudaSuccess) return AAL_ERR_CUDA;
 
-  const bool sampling = prob->mode == AAL_SAMPLING;
+  const bool sampling = (prob->mode & AAL_SAMPLING) != 0;
   RewardRowArgs ra;
+  ra.sampled_draft = (prob->mode & AAL_SAMPLED_DRAFT) != 0;
   ra.zq = draft;
   ra.zp = target;
   ra.zr = ref_draft;
@@ -489,6 +491,8 @@ aal_status aal_accept_reward_from_loss(const aal_reward_problem* rprob, const aa
   if (st != AAL_OK) return st;
   if (rprob->N != lprob->N || rprob->K != lprob->K || rprob->V != lprob->V || rprob->dtype != lprob->dtype)
     return AAL_ERR_INVALID_ARG;
+  // a sampled draft token needs the logits (one noise draw per vocabulary entry)
+  if (rprob->mode & AAL_SAMPLED_DRAFT) return AAL_ERR_INVALID_ARG;
   const bool sampling = rprob->mode == AAL_SAMPLING;
   // the sampling acceptance needs the loss's temperature-scaled normalisers at this T
   if (sampling && (!(lprob->mode & AAL_SAMPLING) || lprob->temperature != rprob->temperature))

@@ -245,6 +245,7 @@ struct RewardRowArgs {
   int64_t R, V;
   int32_t K;
   bool sampling;
+  bool sampled_draft;  // the drafted token is drawn from q~ (Gumbel-max) instead of argmax z_q
   float sT;
   uint64_t seed;
   int64_t row_offset;
@@ -534,6 +535,16 @@ __device__ __forceinline__ float philox_uniform(uint64_t seed, uint64_t n, uint3
   uint4 c = make_uint4((uint32_t)n, (uint32_t)(n >> 32), k, 0u);
   uint4 x = philox4x32_10(c, (uint32_t)seed, (uint32_t)(seed >> 32));
   return (float)((x.x >> 9) * 2u + 1u) * 5.9604644775390625e-08f;  // * 2^-24
+}
+
+// The four uniforms of counter (n_lo, n_hi, k, c3), mapped like philox_uniform: the Gumbel-max
+// draw of the sampled-draft reward gives vocabulary element v word v mod 4 of c3 = 1 + v div 4.
+__device__ __forceinline__ float4 philox_uniform4(uint64_t seed, uint64_t n, uint32_t k, uint32_t c3) {
+  uint4 x = philox4x32_10(make_uint4((uint32_t)n, (uint32_t)(n >> 32), k, c3), (uint32_t)seed,
+                          (uint32_t)(seed >> 32));
+  constexpr float s = 5.9604644775390625e-08f;  // 2^-24
+  return make_float4((float)((x.x >> 9) * 2u + 1u) * s, (float)((x.y >> 9) * 2u + 1u) * s,
+                     (float)((x.z >> 9) * 2u + 1u) * s, (float)((x.w >> 9) * 2u + 1u) * s);
 }
 
 // Bounded wait support: every spin in this library gives up after this many polls.

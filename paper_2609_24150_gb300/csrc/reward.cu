@@ -5,7 +5,10 @@
 //   lowest index on ties.  Greedy verification accepts iff S_k == x*_k.  Sampling
 //   verification accepts iff u < min(1, p~(S_k)/q~(S_k)) (Sec. 2.3), with
 //   u = Philox4x32-10(counter (n_lo, n_hi, k, 0), key seed) and n the global window
-//   index; it needs the log-sum-exps of z_p/T and z_q/T, streamed online.
+//   index; it needs the log-sum-exps of z_p/T and z_q/T, streamed online.  With a sampled
+//   draft (sampled_draft) S_k is instead drawn from q~ by the Gumbel-max method: S_k =
+//   argmax_v (z_q(v)/T + G_v), G_v = -ln(-ln U_v), U_v from counter (n_lo, n_hi, k, 1 + v/4)
+//   word v mod 4; the reference draft draws with the same G (common random numbers).
 // Group kernel, per group of rollouts:
 //   tau = sum_{k=1}^{K} prod_{j<=k} accept_j (the leading run), R = tau - tau^ref
 //   (Eq. debiased_reward), rollout length = mean R over the rollout's windows,
@@ -45,6 +48,40 @@ struct RowState {
   Lse lp, lq, lr;
 };
 
+// Running best of a perturbed key (Gumbel-max), with z of the drawn tensor and z_p there.
+struct Draw {
+  float key;
+  int32_t i;
+  float z, zp;
+};
+__device__ __forceinline__ void draw_init(Draw& d) {
+  d.key = -INFINITY;
+  d.i = 0x7fffffff;
+  d.z = 0.f;
+  d.zp = 0.f;
+}
+__device__ __forceinline__ Draw draw_merge(const Draw& a, const Draw& b) {
+  return (b.key > a.key || (b.key == a.key && b.i < a.i)) ? b : a;
+}
+__device__ __forceinline__ Draw shfl_draw(const Draw& a, int off) {
+  Draw b;
+  b.key = __shfl_xor_sync(0xffffffffu, a.key, off);
+  b.i = __shfl_xor_sync(0xffffffffu, a.i, off);
+  b.z = __shfl_xor_sync(0xffffffffu, a.z, off);
+  b.zp = __shfl_xor_sync(0xffffffffu, a.zp, off);
+  return b;
+}
+__device__ __forceinline__ void draw_push(Draw& d, float key, int64_t v, float z, float zp) {
+  if (key > d.key) {
+    d.key = key;
+    d.i = (int32_t)v;
+    d.z = z;
+    d.zp = zp;
+  }
+}
+// The Gumbel noise in log2 units: G log2(e) = -log2(-ln U) = -log2(-ln2 * log2 U).
+__device__ __forceinline__ float gumbel2(float U) { return -__log2f(-kLn2 * __log2f(U)); }
+
 __device__ __forceinline__ RowState merge_state(const RowState& a, const RowState& b, float sT) {
   RowState o;
   o.q = amax_merge(a.q, b.q);
@@ -76,9 +113,10 @@ __device__ __forceinline__ void init_state(RowState& s) {
   lse_init(s.lr);
 }
 
-template <typename T, bool VEC, bool SAMPLING, bool REF>
+template <typename T, bool VEC, bool SAMPLING, bool REF, bool SAMPLED = false>
 __global__ void __launch_bounds__(kRowThreads) reward_rows(RewardRowArgs a) {
   __shared__ RowState red[kRowWarps];
+  __shared__ Draw dred[2][kRowWarps];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   for (int64_t r = blockIdx.x; r < a.R; r += gridDim.x) {
     const T* zq = static_cast<const T*>(a.zq) + r * a.V;
@@ -86,6 +124,16 @@ __global__ void __launch_bounds__(kRowThreads) reward_rows(RewardRowArgs a) {
     const T* zr = REF ? static_cast<const T*>(a.zr) + r * a.V : nullptr;
     RowState st;
     init_state(st);
+    Draw dq, dr;  // sampled draft tokens (SAMPLED)
+    draw_init(dq);
+    draw_init(dr);
+    const int64_t n_glob = a.row_offset + r / a.K;
+    const uint32_t k_depth = (uint32_t)(r % a.K);
+    auto draw = [&](int64_t v, float q, float p, float rr, float U) {
+      const float g = gumbel2(U);
+      draw_push(dq, fmaf(q, a.sT, g), v, q, p);
+      if (REF) draw_push(dr, fmaf(rr, a.sT, g), v, rr, p);
+    };
     auto visit = [&](int64_t v, float q, float p, float rr) {
       if (q > st.q.v) {
         st.q.v = q;
@@ -117,13 +165,42 @@ __global__ void __launch_bounds__(kRowThreads) reward_rows(RewardRowArgs a) {
         if (REF) unpack_any<T>(ldg_stream(reinterpret_cast<const uint4*>(zr) + i), rv);
 #pragma unroll
         for (int e = 0; e < E; ++e) visit(i * E + e, qv[e], pv[e], REF ? rv[e] : 0.f);
+        if (SAMPLED) {  // E is a multiple of 4: whole counters
+#pragma unroll
+          for (int h = 0; h < E / 4; ++h) {
+            const int64_t v0 = i * E + 4 * h;
+            const float4 U = philox_uniform4(a.seed, (uint64_t)n_glob, k_depth, (uint32_t)(1 + v0 / 4));
+            draw(v0 + 0, qv[4 * h + 0], pv[4 * h + 0], REF ? rv[4 * h + 0] : 0.f, U.x);
+            draw(v0 + 1, qv[4 * h + 1], pv[4 * h + 1], REF ? rv[4 * h + 1] : 0.f, U.y);
+            draw(v0 + 2, qv[4 * h + 2], pv[4 * h + 2], REF ? rv[4 * h + 2] : 0.f, U.z);
+            draw(v0 + 3, qv[4 * h + 3], pv[4 * h + 3], REF ? rv[4 * h + 3] : 0.f, U.w);
+          }
+        }
       }
     } else {
-      for (int64_t v = threadIdx.x; v < a.V; v += kRowThreads)
-        visit(v, load_elem<T>(zq + v), load_elem<T>(zp + v), REF ? load_elem<T>(zr + v) : 0.f);
+      for (int64_t v = threadIdx.x; v < a.V; v += kRowThreads) {
+        const float q = load_elem<T>(zq + v), p = load_elem<T>(zp + v), rr = REF ? load_elem<T>(zr + v) : 0.f;
+        visit(v, q, p, rr);
+        if (SAMPLED) {
+          const float4 U4 = philox_uniform4(a.seed, (uint64_t)n_glob, k_depth, (uint32_t)(1 + v / 4));
+          const int w = (int)(v & 3);
+          draw(v, q, p, rr, w == 0 ? U4.x : w == 1 ? U4.y : w == 2 ? U4.z : U4.w);
+        }
+      }
     }
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) st = merge_state(st, shfl_state(st, off), a.sT);
+    if (SAMPLED) {
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) {
+        dq = draw_merge(dq, shfl_draw(dq, off));
+        if (REF) dr = draw_merge(dr, shfl_draw(dr, off));
+      }
+      if (lane == 0) {
+        dred[0][warp] = dq;
+        dred[1][warp] = dr;
+      }
+    }
     if (lane == 0) red[warp] = st;
     __syncthreads();
     if (threadIdx.x == 0) {
@@ -138,12 +215,25 @@ __global__ void __launch_bounds__(kRowThreads) reward_rows(RewardRowArgs a) {
         const uint32_t k = (uint32_t)(r - n * a.K);
         const float u = philox_uniform(a.seed, (uint64_t)(a.row_offset + n), k);
         const float Lsp = lse_ls(t.lp), Lsq = lse_ls(t.lq);
+        // the drafted token S: the draft's argmax, or its Gumbel-max draw
+        float zqS = t.q.v, zpS = t.q.carry, zrS = t.r.v, zpR = t.r.carry;
+        if (SAMPLED) {
+          Draw bq = dred[0][0], br = dred[1][0];
+          for (int w = 1; w < kRowWarps; ++w) {
+            bq = draw_merge(bq, dred[0][w]);
+            if (REF) br = draw_merge(br, dred[1][w]);
+          }
+          zqS = bq.z;
+          zpS = bq.zp;
+          zrS = br.z;
+          zpR = br.zp;
+        }
         // log2 p~(S) - log2 q~(S)
-        const float d = log2_prob(t.q.carry, a.sT, t.lp.M, Lsp) - log2_prob(t.q.v, a.sT, t.lq.M, Lsq);
+        const float d = log2_prob(zpS, a.sT, t.lp.M, Lsp) - log2_prob(zqS, a.sT, t.lq.M, Lsq);
         acc = (u < exp2f(fminf(d, 0.f))) ? 1 : 0;
         if (REF) {
           const float Lsr = lse_ls(t.lr);
-          const float dr = log2_prob(t.r.carry, a.sT, t.lp.M, Lsp) - log2_prob(t.r.v, a.sT, t.lr.M, Lsr);
+          const float dr = log2_prob(zpR, a.sT, t.lp.M, Lsp) - log2_prob(zrS, a.sT, t.lr.M, Lsr);
           acc_ref = (u < exp2f(fminf(dr, 0.f))) ? 1 : 0;
         }
       }
@@ -154,23 +244,25 @@ __global__ void __launch_bounds__(kRowThreads) reward_rows(RewardRowArgs a) {
   }
 }
 
-template <typename T, bool VEC, bool S, bool R>
+template <typename T, bool VEC, bool S, bool R, bool D = false>
 cudaError_t go(const RewardRowArgs& a, cudaStream_t s) {
   int dev = 0, sms = 0, per_sm = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, reward_rows<T, VEC, S, R>, kRowThreads, 0);
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, reward_rows<T, VEC, S, R, D>, kRowThreads, 0);
   if (per_sm < 1) per_sm = 1;
   int64_t grid = (int64_t)sms * per_sm;
   if (grid > a.R) grid = a.R;
   if (grid < 1) return cudaSuccess;
-  reward_rows<T, VEC, S, R><<<(unsigned)grid, kRowThreads, 0, s>>>(a);
+  reward_rows<T, VEC, S, R, D><<<(unsigned)grid, kRowThreads, 0, s>>>(a);
   return cudaGetLastError();
 }
 
 template <typename T, bool VEC>
 cudaError_t dispatch_flags(const RewardRowArgs& a, cudaStream_t s) {
   const bool ref = a.zr != nullptr;
+  if (a.sampling && a.sampled_draft)
+    return ref ? go<T, VEC, true, true, true>(a, s) : go<T, VEC, true, false, true>(a, s);
   if (a.sampling) return ref ? go<T, VEC, true, true>(a, s) : go<T, VEC, true, false>(a, s);
   return ref ? go<T, VEC, false, true>(a, s) : go<T, VEC, false, false>(a, s);
 }

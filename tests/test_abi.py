@@ -41,7 +41,7 @@ def test_library_exports_every_declared_symbol():
 
 
 def test_status_strings_and_version():
-    assert aal.aal_abi_version() == 10300
+    assert aal.aal_abi_version() == 10400
     for code in range(6):
         assert aal.aal_status_string(code).startswith("AAL_")
     assert aal.aal_status_string(99) == "unknown aal_status"
@@ -138,6 +138,9 @@ def _rprob(**kw):
     (dict(), aal.AAL_OK),
     (dict(mode=aal.AAL_BOTH), aal.AAL_ERR_INVALID_ARG),
     (dict(mode=aal.AAL_SAMPLING, temperature=0.0), aal.AAL_ERR_INVALID_ARG),
+    (dict(mode=aal.AAL_SAMPLING | aal.AAL_SAMPLED_DRAFT), aal.AAL_OK),
+    (dict(mode=aal.AAL_GREEDY | aal.AAL_SAMPLED_DRAFT), aal.AAL_ERR_INVALID_ARG),
+    (dict(mode=aal.AAL_SAMPLED_DRAFT), aal.AAL_ERR_INVALID_ARG),
     (dict(windows_per_rollout=3), aal.AAL_ERR_INVALID_ARG),     # 8 windows not a multiple of 6
     (dict(rollouts_per_group=0), aal.AAL_ERR_INVALID_ARG),
     (dict(adv_clip=0.0), aal.AAL_ERR_INVALID_ARG),
