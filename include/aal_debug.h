@@ -16,15 +16,16 @@
 extern "C" {
 #endif
 
-/* Arms the next aal_loss_fwd that runs the TMA-streamed row kernel (sampling term, rows
- * a multiple of 16 bytes) to leave the completion barrier of its `chunk`-th ring copy
- * (counted from 0 in each CTA's stream) unarmed: the consumers of that chunk wait on a
- * phase that nothing completes.  Every wait of that kernel, and of later ones, gives up
+/* Arms the next forward pass that streams logits through a TMA ring (aal_loss_fwd or
+ * aal_seq_loss_fwd on rows a multiple of 16 bytes, including the token-id form, or the
+ * reference-draft pass of aal_grpo_from_loss) to leave the completion barrier of its
+ * `chunk`-th ring copy (counted from 0 in each CTA's stream) unarmed: the consumers of that
+ * chunk wait on a phase that nothing completes.  Every wait of that kernel, and of later ones, gives up
  * after `wait_limit_ns` (0 restores the default of 1 s); the kernel then records
  * AAL_ERR_TIMEOUT in the workspace status word, walks its remaining loops without waiting,
  * drains its copies and returns, so aal_check_device_status() reports AAL_ERR_TIMEOUT and
- * the context stays usable.  The results of that forward are not valid.  A negative
- * `chunk` arms nothing.  The chunk setting is consumed by the next forward. */
+ * the context stays usable.  The results of that call are not valid.  A negative
+ * `chunk` arms nothing.  The chunk setting is consumed by the next forward or GRPO call. */
 AAL_API void aal_debug_fail_next_forward(int64_t chunk, uint64_t wait_limit_ns);
 
 #ifdef __cplusplus

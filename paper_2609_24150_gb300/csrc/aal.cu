@@ -107,8 +107,8 @@ cudaError_t launch_stats(const void* draft, const void* target, int64_t R, int64
     a.acc_ref = nullptr;
     a.lpr = nullptr;
     a.hdr = ws.hdr;
+    a.skip_chunk = debug_take_skip_chunk();
     *cluster = 1;
-    (void)debug_take_skip_chunk();  // (the ring test hook applies to the two-tensor forward only)
     return launch_one_tensor(a, dtype == AAL_BF16, true, s);
   }
   const bool greedy = (mode & AAL_GREEDY) != 0;
@@ -389,6 +389,7 @@ aal_status aal_grpo_from_loss(const aal_grpo_problem* gprob, const aal_problem* 
   ra.acc_ref = reinterpret_cast<uint8_t*>(base + L.acc_ref);
   ra.lpr = reinterpret_cast<float*>(base + L.lpr);
   ra.hdr = hdr;
+  ra.skip_chunk = debug_take_skip_chunk();
   if (launch_one_tensor(ra, gprob->dtype == AAL_BF16, false, s) != cudaSuccess) return AAL_ERR_CUDA;
 
   float* adv = advantage != nullptr ? advantage : reinterpret_cast<float*>(base + L.adv);

@@ -328,6 +328,7 @@ struct Stream1Args {
   uint8_t* acc_ref;    // REF: [R] argmax z_ref == x*
   float* lpr;          // REF: [R] log pi_ref(y)
   WsHeader* hdr;       // status word (bounded waits; out-of-range ids)
+  int64_t skip_chunk;  // failure-detection test hook: a chunk whose copy is never armed (-1: none)
 };
 
 // Per window: log rho, the clipped surrogate, its per-row gradient coefficients.

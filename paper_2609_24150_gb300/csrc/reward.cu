@@ -13,7 +13,7 @@
 //   tau = sum_{k=1}^{K} prod_{j<=k} accept_j (the leading run), R = tau - tau^ref
 //   (Eq. debiased_reward), rollout length = mean R over the rollout's windows,
 //   A = clip((x - mean)/(std + 1e-6), -C_A, C_A) with the population std (Eq. advantage).
-#include "aal_internal.cuh"
+#include "ptx.cuh"
 
 namespace aal {
 namespace {
@@ -244,6 +244,222 @@ __global__ void __launch_bounds__(kRowThreads) reward_rows(RewardRowArgs a) {
   }
 }
 
+// ---------------------------------------------------------------- sampled draft, vector path
+// The sampled-draft reward is bound by arithmetic, not bytes: one Philox4x32-10 call per four
+// vocabulary entries and two logarithms per entry.  This path keeps everything per 16-byte vector
+// and branch-free: the log-sum-exps fold a vector's values after one rescale to the vector maximum
+// (as in the streamed forward), the Gumbel keys of a vector are maxed first and the element is
+// looked up only when the vector beats the running best, and the first Philox round, whose two
+// products depend only on the row (window, depth), is computed once per row.
+struct PhiloxRow {
+  uint32_t x0, x1, x2k, x3;  // round-1 output except the c3 term: x2 = x2k ^ c3
+  uint32_t k0[10], k1[10];   // round keys
+};
+
+__device__ __forceinline__ PhiloxRow philox_row(uint64_t seed, uint64_t n, uint32_t k) {
+  PhiloxRow P;
+  uint32_t a = (uint32_t)seed, b = (uint32_t)(seed >> 32);
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    P.k0[r] = a;
+    P.k1[r] = b;
+    a += 0x9E3779B9u;
+    b += 0xBB67AE85u;
+  }
+  const uint32_t c0 = (uint32_t)n, c1 = (uint32_t)(n >> 32), c2 = k;
+  const uint32_t hi0 = __umulhi(0xD2511F53u, c0), lo0 = 0xD2511F53u * c0;
+  const uint32_t hi1 = __umulhi(0xCD9E8D57u, c2), lo1 = 0xCD9E8D57u * c2;
+  P.x0 = hi1 ^ c1 ^ P.k0[0];
+  P.x1 = lo1;
+  P.x2k = hi0 ^ P.k1[0];
+  P.x3 = lo0;
+  return P;
+}
+
+// The four words of counter (n_lo, n_hi, k, c3): rounds 2..10 after the row's round 1.
+__device__ __forceinline__ uint4 philox_rest(const PhiloxRow& P, uint32_t c3) {
+  uint4 c = make_uint4(P.x0, P.x1, P.x2k ^ c3, P.x3);
+#pragma unroll
+  for (int r = 1; r < 10; ++r) {
+    // each 32 x 32 -> 64 product in one multiply: high and low halves together
+    const uint64_t p0 = (uint64_t)0xD2511F53u * c.x, p1 = (uint64_t)0xCD9E8D57u * c.z;
+    c = make_uint4((uint32_t)(p1 >> 32) ^ c.y ^ P.k0[r], (uint32_t)p1, (uint32_t)(p0 >> 32) ^ c.w ^ P.k1[r],
+                   (uint32_t)p0);
+  }
+  return c;
+}
+
+// ((w >> 9) * 2 + 1) * 2^-24 without an integer-to-float conversion: the 23 high bits as the
+// mantissa of a float in [1, 2), minus (1 - 2^-24) (exact: the result is an odd multiple of
+// 2^-24 below 1).
+__device__ __forceinline__ float word_uniform(uint32_t w) {
+  return __uint_as_float(0x3F800000u | (w >> 9)) - 0.99999994039535522461f;
+}
+
+// Fold E values into (M, S) at scale s after one rescale to max(M, vector max).
+template <int E>
+__device__ __forceinline__ void lse_fold(Lse& L, const float* z, float s) {
+  float vm = z[0];
+#pragma unroll
+  for (int e = 1; e < E; ++e) vm = fmaxf(vm, z[e]);
+  const float m = fmaxf(L.M, vm);
+  float acc = 0.f;
+#pragma unroll
+  for (int e = 0; e < E; ++e) acc += ex2((z[e] - m) * s);
+  L.S = L.S * ex2((L.M - m) * s) + acc;
+  L.M = m;
+}
+
+// Offer E Gumbel keys of one vector (elements v0 ..) to a running draw.
+template <int E>
+__device__ __forceinline__ void draw_fold(Draw& d, const float* key, const float* z, const float* zp, int64_t v0) {
+  float km = key[0];
+#pragma unroll
+  for (int e = 1; e < E; ++e) km = fmaxf(km, key[e]);
+  if (km > d.key) {  // rare once the running best has settled
+    int at = 0;
+#pragma unroll
+    for (int e = E - 1; e >= 0; --e)
+      if (key[e] == km) at = e;
+    float zz = z[0], pp = zp[0];
+#pragma unroll
+    for (int e = 1; e < E; ++e)
+      if (e == at) {
+        zz = z[e];
+        pp = zp[e];
+      }
+    d.key = km;
+    d.i = (int32_t)(v0 + at);
+    d.z = zz;
+    d.zp = pp;
+  }
+}
+
+// lse_fold for a bf16 vector in its packed form: the maximum by max.bf16x2, z - m with the bf16
+// widened inside the add, the scale and the sums on f32 pairs.
+__device__ __forceinline__ void lse_fold_bf16(Lse& L, const uint4& w, float s) {
+  const uint32_t mw = ptx::bmax2(ptx::bmax2(w.x, w.y), ptx::bmax2(w.z, w.w));
+  const float m = fmaxf(L.M, fmaxf(bf16_lo(mw), bf16_hi(mw)));
+  const float nm = -m;
+  const float2 s2 = make_float2(s, s), zero2 = make_float2(0.f, 0.f);
+  const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+  float2 acc = zero2;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const float2 x = ptx::f2fma(make_float2(bf16lo_add(ww[k], nm), bf16hi_add(ww[k], nm)), s2, zero2);
+    acc = ptx::f2add(acc, make_float2(ex2(x.x), ex2(x.y)));
+  }
+  L.S = L.S * ex2((L.M - m) * s) + (acc.x + acc.y);
+  L.M = m;
+}
+
+template <typename T, bool REF>
+__global__ void __launch_bounds__(kRowThreads, REF ? 4 : 5) reward_sampled_rows(RewardRowArgs a) {
+  __shared__ RowState red[kRowWarps];
+  __shared__ Draw dred[2][kRowWarps];
+  constexpr int E = 16 / sizeof(T);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  for (int64_t r = blockIdx.x; r < a.R; r += gridDim.x) {
+    const uint4* q4 = reinterpret_cast<const uint4*>(static_cast<const T*>(a.zq) + r * a.V);
+    const uint4* p4 = reinterpret_cast<const uint4*>(static_cast<const T*>(a.zp) + r * a.V);
+    const uint4* r4 = REF ? reinterpret_cast<const uint4*>(static_cast<const T*>(a.zr) + r * a.V) : nullptr;
+    const int64_t n_glob = a.row_offset + r / a.K;
+    const uint32_t k_depth = (uint32_t)(r % a.K);
+    const PhiloxRow P = philox_row(a.seed, (uint64_t)n_glob, k_depth);
+    RowState st;
+    init_state(st);
+    // running maxima start at a finite floor, so lse_fold needs no -inf case (a -inf logit
+    // then adds 2^(-inf) = 0)
+    st.lp.M = st.lq.M = st.lr.M = -1e30f;
+    Draw dq, dr;
+    draw_init(dq);
+    draw_init(dr);
+    const int64_t nv = a.V / E;
+    for (int64_t i = threadIdx.x; i < nv; i += kRowThreads) {
+      float qv[E], pv[E], rv[E], g[E], kq[E], kr[E];
+      const uint4 qw = ldg_stream(q4 + i), pw = ldg_stream(p4 + i);
+      uint4 rw = make_uint4(0, 0, 0, 0);
+      if (REF) rw = ldg_stream(r4 + i);
+      unpack_any<T>(qw, qv);
+      unpack_any<T>(pw, pv);
+      if (REF) unpack_any<T>(rw, rv);
+#pragma unroll
+      for (int h = 0; h < E / 4; ++h) {
+        const uint4 w = philox_rest(P, (uint32_t)(1 + (i * E) / 4 + h));
+        g[4 * h + 0] = gumbel2(word_uniform(w.x));
+        g[4 * h + 1] = gumbel2(word_uniform(w.y));
+        g[4 * h + 2] = gumbel2(word_uniform(w.z));
+        g[4 * h + 3] = gumbel2(word_uniform(w.w));
+      }
+#pragma unroll
+      for (int e = 0; e < E; ++e) {
+        kq[e] = fmaf(qv[e], a.sT, g[e]);
+        if (REF) kr[e] = fmaf(rv[e], a.sT, g[e]);
+      }
+      draw_fold<E>(dq, kq, qv, pv, i * E);
+      if (REF) draw_fold<E>(dr, kr, rv, pv, i * E);
+      if (sizeof(T) == 2) {
+        lse_fold_bf16(st.lp, pw, a.sT);
+        lse_fold_bf16(st.lq, qw, a.sT);
+        if (REF) lse_fold_bf16(st.lr, rw, a.sT);
+      } else {
+        lse_fold<E>(st.lp, pv, a.sT);
+        lse_fold<E>(st.lq, qv, a.sT);
+        if (REF) lse_fold<E>(st.lr, rv, a.sT);
+      }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      st.lp = lse_merge(st.lp, shfl_lse(st.lp, off), a.sT);
+      st.lq = lse_merge(st.lq, shfl_lse(st.lq, off), a.sT);
+      if (REF) st.lr = lse_merge(st.lr, shfl_lse(st.lr, off), a.sT);
+      dq = draw_merge(dq, shfl_draw(dq, off));
+      if (REF) dr = draw_merge(dr, shfl_draw(dr, off));
+    }
+    if (lane == 0) {
+      red[warp] = st;
+      dred[0][warp] = dq;
+      dred[1][warp] = dr;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      RowState t = red[0];
+      Draw bq = dred[0][0], br = dred[1][0];
+      for (int w = 1; w < kRowWarps; ++w) {
+        t.lp = lse_merge(t.lp, red[w].lp, a.sT);
+        t.lq = lse_merge(t.lq, red[w].lq, a.sT);
+        if (REF) t.lr = lse_merge(t.lr, red[w].lr, a.sT);
+        bq = draw_merge(bq, dred[0][w]);
+        if (REF) br = draw_merge(br, dred[1][w]);
+      }
+      const float u = philox_uniform(a.seed, (uint64_t)n_glob, k_depth);
+      const float Lsp = lse_ls(t.lp), Lsq = lse_ls(t.lq);
+      const float d = log2_prob(bq.zp, a.sT, t.lp.M, Lsp) - log2_prob(bq.z, a.sT, t.lq.M, Lsq);
+      a.acc[r] = (u < exp2f(fminf(d, 0.f))) ? 1 : 0;
+      if (REF) {
+        const float Lsr = lse_ls(t.lr);
+        const float dd = log2_prob(br.zp, a.sT, t.lp.M, Lsp) - log2_prob(br.z, a.sT, t.lr.M, Lsr);
+        a.acc_ref[r] = (u < exp2f(fminf(dd, 0.f))) ? 1 : 0;
+      }
+    }
+    __syncthreads();
+  }
+}
+
+template <typename T, bool REF>
+cudaError_t go_sampled(const RewardRowArgs& a, cudaStream_t s) {
+  int dev = 0, sms = 0, per_sm = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, reward_sampled_rows<T, REF>, kRowThreads, 0);
+  if (per_sm < 1) per_sm = 1;
+  int64_t grid = (int64_t)sms * per_sm;
+  if (grid > a.R) grid = a.R;
+  if (grid < 1) return cudaSuccess;
+  reward_sampled_rows<T, REF><<<(unsigned)grid, kRowThreads, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
 template <typename T, bool VEC, bool S, bool R, bool D = false>
 cudaError_t go(const RewardRowArgs& a, cudaStream_t s) {
   int dev = 0, sms = 0, per_sm = 0;
@@ -261,8 +477,10 @@ cudaError_t go(const RewardRowArgs& a, cudaStream_t s) {
 template <typename T, bool VEC>
 cudaError_t dispatch_flags(const RewardRowArgs& a, cudaStream_t s) {
   const bool ref = a.zr != nullptr;
-  if (a.sampling && a.sampled_draft)
+  if (a.sampling && a.sampled_draft) {
+    if (VEC) return ref ? go_sampled<T, true>(a, s) : go_sampled<T, false>(a, s);
     return ref ? go<T, VEC, true, true, true>(a, s) : go<T, VEC, true, false, true>(a, s);
+  }
   if (a.sampling) return ref ? go<T, VEC, true, true>(a, s) : go<T, VEC, true, false>(a, s);
   return ref ? go<T, VEC, false, true>(a, s) : go<T, VEC, false, false>(a, s);
 }
