@@ -107,6 +107,14 @@ __device__ __forceinline__ bool wait_phase(uint64_t* b, uint32_t parity, volatil
 
 // ---------------------------------------------------------------- packed arithmetic
 // Two fp32 lanes per instruction (sm_100+), IEEE round-to-nearest like the scalar forms.
+#ifndef AAL_F2_ASM
+#define AAL_F2_ASM 0
+#endif
+#if !AAL_F2_ASM
+// the compiler's own pair operations: it places the pairs in registers itself
+__device__ __forceinline__ float2 f2fma(float2 a, float2 b, float2 c) { return __ffma2_rn(a, b, c); }
+__device__ __forceinline__ float2 f2add(float2 a, float2 b) { return __fadd2_rn(a, b); }
+#else
 __device__ __forceinline__ float2 f2fma(float2 a, float2 b, float2 c) {
   float2 d;
   asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\tmov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
@@ -123,6 +131,7 @@ __device__ __forceinline__ float2 f2add(float2 a, float2 b) {
       : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
   return d;
 }
+#endif
 __device__ __forceinline__ uint32_t bmax2(uint32_t a, uint32_t b) {
   uint32_t d;
   asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));

@@ -50,6 +50,10 @@ constexpr int kVecPerChunk = kHalfSlot / 16;
 constexpr int kWarps = AAL_STREAM_WARPS;  // consumer warps
 constexpr int kConsumers = 32 * kWarps;
 constexpr int kThreads = 32 + kConsumers;
+#ifndef AAL_STREAM_CTAS
+#define AAL_STREAM_CTAS 1
+#endif
+constexpr int kCtasPerSm = AAL_STREAM_CTAS;  // resident CTAs per SM (each with its own ring)
 constexpr int kNV = kVecPerChunk / kConsumers;  // 16-byte vectors per thread per full chunk
 static_assert(kNV * kConsumers == kVecPerChunk, "consumers must tile a chunk");
 constexpr int kBarRow = 1, kBarSum = 2;
@@ -380,7 +384,7 @@ struct RingPos {
 // sampling term; everything at T = 1 (sT is log2 e), argmaxes resolved by resolve_argmax.
 // KL: the anchor's D next to the z_p normaliser (which must then be at T = 1).
 template <typename T, bool NEED_Q1, int PASSES, bool KL>
-__global__ void __launch_bounds__(kThreads, 1) rowstats_stream(RowStatsArgs a, int nch, uint64_t limit_ns) {
+__global__ void __launch_bounds__(kThreads, kCtasPerSm) rowstats_stream(RowStatsArgs a, int nch, uint64_t limit_ns) {
   extern __shared__ __align__(1024) unsigned char smem[];
   unsigned char* ring = smem;
   Smem& S = *reinterpret_cast<Smem*>(smem + kSlots * kSlotBytes);
@@ -608,7 +612,7 @@ cudaError_t launch_T(const RowStatsArgs& a, cudaStream_t s, int nch, uint64_t li
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  int64_t grid = sms;
+  int64_t grid = (int64_t)sms * kCtasPerSm;
   if (grid > a.R) grid = a.R;
   if (grid < 1) return cudaSuccess;
   kern<<<(unsigned)grid, kThreads, kSmemBytes, s>>>(a, nch, limit_ns);
