@@ -38,6 +38,8 @@ sys.path.insert(0, ROOT)
 import synth  # noqa: E402
 
 WORKLOAD = "v128k"
+STEP_WORKLOAD = ("v128k: N=8192 windows (B=4 x T=2048), K=7, V=128256 bf16; EAL+WTV 0.5/0.5 at T=1 fwd+bwd, "
+                 "greedy reward 16 rollouts x 256 windows")
 MODE_T, W_G, W_S = 1.0, 0.5, 0.5
 WPR, RPG = 256, 16           # reward: windows per rollout, rollouts per group
 KERNELS_PER_STEP = 5         # row stats + window combine, backward, reward flags + groups
@@ -278,8 +280,7 @@ def run_ours(args, ws_count, rank, local):
         "dtype": "bf16",
         "data": "synthetic (seeded Zipf target logits over a random vocabulary permutation, "
                 "draft = target + N(0,1)); no model weights",
-        "config": {"workload": f"{WORKLOAD}: N=8192 windows (B=4 x T=2048), K=7, V=128256 bf16; "
-                               "EAL+WTV 0.5/0.5 at T=1 fwd+bwd, greedy reward 16 rollouts x 256 windows",
+        "config": {"workload": STEP_WORKLOAD,
                    "N": N, "K": K, "V": V, "rows_per_step": R,
                    "bytes_per_step": step_bytes, "l2": "inputs larger than L2 (14.7 GB per tensor)",
                    "parallelism": f"replicas x{ws_count} (independent windows)"},
@@ -576,7 +577,7 @@ def run_reference(args, ws_count, rank):
             "value": round(value, 4), "unit": "GB/s", "n_gpus": ws_count, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(dt * 1e3, 3), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": f"{WORKLOAD}: N=8192, K=7, V=128256 bf16 (each step: a {n}-window sample)"},
+            "config": {"workload": STEP_WORKLOAD, "sample": f"each step times the oracle on a {n}-window sample"},
             "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
                              "sample": f"{n} windows ({n * K} rows x V={V}) per step, numpy fp64, one thread"},
             "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
