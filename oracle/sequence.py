@@ -133,3 +133,41 @@ def seq_objective_backward(target, draft, mask, K: int, mode: int = 5, T: float 
                     out[src[n, j]] += gw[n, j]
         g = g + out.reshape(B, Tn, V)
     return g
+
+
+# ---------------------------------------------------------------------------------------
+# The GRPO stage over sequences (Sec. 3.4): the three forward passes run once per sequence
+# and the window samples are sliced from them.  Windows are given by their start positions
+# (flat index b*T + t, each window inside its sequence); the surrogate is grpo.py's over the
+# sliced windows, and a position's gradient row adds the rows of every window that covers it.
+
+def slice_windows(x, starts, K: int):
+    """[B][T][V] -> the [N][K][V] windows starting at the given flat positions."""
+    z = as_f64(x)
+    B, T, V = z.shape
+    flat = z.reshape(B * T, V)
+    starts = np.asarray(starts, dtype=np.int64)
+    for s in starts:
+        if s < 0 or s % T + K > T:
+            raise ValueError("a window must lie inside its sequence")
+    return np.stack([flat[s:s + K] for s in starts]) if len(starts) else np.zeros((0, K, V))
+
+
+def seq_grpo_forward(target, draft, ref, starts, K: int, **grpo_kw):
+    from .grpo import grpo_forward
+    return grpo_forward(slice_windows(target, starts, K), slice_windows(draft, starts, K),
+                        slice_windows(ref, starts, K), **grpo_kw)
+
+
+def seq_grpo_backward(target, draft, ref, starts, K: int, dloss: float = 1.0, **grpo_kw) -> np.ndarray:
+    """dloss * dL_GRPO/dz_theta per position, [B][T][V]."""
+    from .grpo import grpo_backward
+    zq = as_f64(draft)
+    B, T, V = zq.shape
+    g = grpo_backward(slice_windows(target, starts, K), slice_windows(draft, starts, K),
+                      slice_windows(ref, starts, K), dloss=dloss, **grpo_kw)
+    out = np.zeros((B * T, V))
+    for n, s in enumerate(np.asarray(starts, dtype=np.int64)):
+        for k in range(K):
+            out[s + k] += g[n, k]
+    return out.reshape(B, T, V)

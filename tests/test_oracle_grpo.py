@@ -147,3 +147,36 @@ def test_a_slice_with_the_batch_advantages_gives_its_rows():
     np.testing.assert_allclose(gs, g[sel], rtol=0, atol=1e-16)
     np.testing.assert_allclose(fs["rho"], full["rho"][sel], rtol=0, atol=0)
     assert abs(fs["loss"] - (-np.sum(full["surrogate"][sel]) / N)) < 1e-16
+
+
+def test_sequence_grpo_gradient_by_finite_differences():
+    """Overlapping windows sliced from one sequence pass (Sec. 3.4): the per-position gradient
+    adds every covering window's row; checked against central differences of the loss."""
+    from oracle.sequence import seq_grpo_backward, seq_grpo_forward
+    rng = np.random.default_rng(17)
+    B, T, K, V = 2, 9, 3, 5
+    for _ in range(200):
+        tgt = rng.normal(0, 2, size=(B, T, V))
+        dr = rng.normal(0, 1, size=(B, T, V))
+        S = np.where(rng.random((B, T)) < 0.6, np.argmax(tgt, -1), rng.integers(0, V, (B, T)))
+        np.put_along_axis(dr, S[..., None], np.max(dr, -1, keepdims=True) + 3.0, axis=-1)
+        rf = dr + rng.normal(0, 0.4, size=(B, T, V))
+        Sr = np.where(rng.random((B, T)) < 0.4, rng.integers(0, V, (B, T)), S)
+        np.put_along_axis(rf, Sr[..., None], np.max(rf, -1, keepdims=True) + 1.5, axis=-1)
+        starts = [0, 1, 2, 4, 9 + 0, 9 + 3, 9 + 5, 9 + 6]          # two groups of four, overlapping
+        kw = dict(windows_per_rollout=1, rollouts_per_group=4, eps_clip=0.25)
+        fw = seq_grpo_forward(tgt, dr, rf, starts, K, **kw)
+        if np.min(np.abs(fw["rho"] - 1.25)) > 1e-3 and np.min(np.abs(fw["rho"] - 0.75)) > 1e-3 \
+                and np.any(fw["advantage_window"] != 0):
+            break
+    else:
+        raise AssertionError("no admissible input")
+    g = seq_grpo_backward(tgt, dr, rf, starts, K, dloss=2.0, **kw)
+    h = 1e-6
+    for idx in np.ndindex(B, T, V):
+        a = dr.copy(); a[idx] += h
+        b = dr.copy(); b[idx] -= h
+        fd = 2.0 * (seq_grpo_forward(tgt, a, rf, starts, K, **kw)["loss"]
+                    - seq_grpo_forward(tgt, b, rf, starts, K, **kw)["loss"]) / (2 * h)
+        assert abs(fd - g[idx]) < 1e-8, (idx, fd, g[idx])
+    assert np.all(g[0, 7:] == 0) and np.any(g != 0)        # positions 7, 8 of sequence 0 are in no window
