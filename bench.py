@@ -57,8 +57,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-seq", action="store_true", help="skip every line beside the step")
-    ap.add_argument("--lines", default="greedy,ids,seq,grpo",
-                    help="lines measured beside the step (comma-separated from greedy, ids, seq, grpo)")
+    ap.add_argument("--lines", default="greedy,ids,seq,grpo,seqgrpo",
+                    help="lines measured beside the step (comma-separated from greedy, ids, seq, grpo, seqgrpo)")
     ap.add_argument("--windows", type=int, default=None,
                     help="run the first WINDOWS windows of the workload (profiling captures)")
     return ap.parse_args()
@@ -253,6 +253,7 @@ def run_ours(args, ws_count, rank, local):
     greedy_ids = run_greedy_ids(aal, draft, target, grad, stream, reps) if "ids" in lines else None
     seq = run_sequence_layout(aal, dev, stream, rank, reps) if "seq" in lines else None
     grpo = run_grpo_phase(aal, dev, stream, rank, reps) if "grpo" in lines else None
+    seq_grpo = run_seq_grpo_phase(aal, dev, stream, rank, reps) if "seqgrpo" in lines else None
 
     b = algo_bytes(N, K, V)
     step_bytes = sum(b.values())
@@ -311,6 +312,8 @@ def run_ours(args, ws_count, rank, local):
         res["sequence_layout"] = seq
     if grpo is not None:
         res["grpo_phase_step"] = grpo
+    if seq_grpo is not None:
+        res["seq_grpo_phase_step"] = seq_grpo
 
     if rank == 0 and not args.no_e2e:
         res["e2e"] = run_e2e(args, aal, prob, rprob, draft, target, grad, ws, loss, rws, tau, rl, adv,
@@ -435,6 +438,62 @@ def run_greedy_ids(aal, draft, target, grad, stream, reps):
            "fwd_gbs": round(fb / (fwd * 1e-3) / 1e9, 1), "bwd_gbs": round(bb / (bwd * 1e-3) / 1e9, 1),
            "rows_per_s": round(R / ((fwd + bwd) * 1e-3), 1), "loss": float(loss.item())}
     del ws, ids
+    return out
+
+
+def run_seq_grpo_phase(aal, dev, stream, rank, reps):
+    """The GRPO-phase step over sequences (Sec. 3.4): seq_v128k (4 x 2048 positions, K = 7, V = 128256
+    bf16, prompt and padding masks), L_KL + 0.1 L_EAL over every sliding window plus 0.1 L_GRPO over
+    8 anchors per sequence with groups of 16 consecutive windows; the reference draft = the draft +
+    N(0, 0.3^2).  aal_seq_loss_fwd, aal_seq_grpo_from_loss (reads the reference once per position),
+    aal_seq_loss_bwd."""
+    target, draft, mask = synth.make_seq_logits("seq_v128k", seed=rank, device=dev)
+    B, T, V = draft.shape
+    K, m = synth.SEQUENCES["seq_v128k"].K, 16
+    g = torch.Generator(device=dev).manual_seed(rank)
+    ref = (draft.float() + 0.3 * torch.randn(draft.shape, generator=g, device=dev)).to(draft.dtype)
+    valid = mask.cpu()
+    starts = []
+    for b in range(B):
+        v = torch.nonzero(valid[b]).flatten()
+        lo, hi = int(v[0]), int(v[-1]) - K - m
+        for a in torch.linspace(lo, hi, 8).long().tolist():
+            starts += [b * T + a + i for i in range(m)]
+    starts = torch.tensor(sorted(starts), dtype=torch.int32, device=dev)
+    N = starts.numel()
+    grad = torch.empty_like(draft)
+    sprob = aal.seq_problem(draft, K, aal.AAL_KL | aal.AAL_GREEDY | aal.AAL_GRPO, 1.0, 0.1, 0.0, False, 1.0)
+    lws = torch.empty(aal.aal_seq_workspace_size(sprob), dtype=torch.uint8, device=dev)
+    gprob = aal.grpo_seq_problem(N, draft, K, 1, m, w_grpo=0.1)
+    gws = torch.empty(aal.aal_seq_grpo_workspace_size(gprob, sprob), dtype=torch.uint8, device=dev)
+    loss = torch.empty(1, dtype=torch.float32, device=dev)
+    gloss = torch.empty(1, dtype=torch.float32, device=dev)
+    calls = [lambda: aal.aal_seq_loss_fwd(sprob, draft, target, mask, lws, loss, None, stream),
+             lambda: aal.aal_seq_grpo_from_loss(gprob, sprob, lws, ref, starts, gws, gloss, stream=stream),
+             lambda: aal.aal_seq_loss_bwd(sprob, draft, target, mask, lws, 1.0, grad, stream)]
+    for _ in range(3):
+        for c in calls:
+            c()
+    torch.cuda.synchronize()
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(reps)]
+    for e in ev:
+        for i, c in enumerate(calls):
+            e[i].record(stream)
+            c()
+        e[3].record(stream)
+    torch.cuda.synchronize()
+    assert aal.aal_check_device_status(lws) == aal.AAL_OK and aal.aal_check_device_status(gws) == aal.AAL_OK
+    ms = [sum(e[i].elapsed_time(e[i + 1]) for e in ev) / reps for i in range(3)]
+    R = B * T
+    row = V * draft.element_size()
+    b = [2 * R * row, R * row, 3 * R * row]   # masked rows are still read; the masked backward rows are written
+    tot = sum(ms)
+    out = {"workload": f"seq_v128k: B={B} x T={T} positions, K={K}, V={V} bf16, masked; L_KL + 0.1 L_EAL + "
+                       f"0.1 L_GRPO over {N} windows (8 anchors per sequence x groups of {m})",
+           "ms": round(tot, 4), "fwd_ms": round(ms[0], 4), "grpo_ms": round(ms[1], 4), "bwd_ms": round(ms[2], 4),
+           "gbs": round(sum(b) / (tot * 1e-3) / 1e9, 1), "positions_per_s": round(R / (tot * 1e-3), 1),
+           "loss": float(loss.item()), "grpo_loss": float(gloss.item())}
+    del target, draft, ref, grad, lws, gws
     return out
 
 

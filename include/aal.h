@@ -80,7 +80,7 @@ typedef enum { AAL_F32 = 0, AAL_BF16 = 1 } aal_dtype;
  * bytes, and the greedy backward never reads the target).  It combines with AAL_GREEDY and
  * AAL_GRPO only (the other terms need p).  An id outside [0, V) records AAL_ERR_INVALID_ARG in the
  * workspace status word (aal_check_device_status) and that row's a^greedy is 0.
- * Valid modes: 1 .. 63 (AAL_GRPO only with aal_loss_*). */
+ * Valid modes: 1 .. 63. */
 typedef enum {
   AAL_GREEDY = 1, AAL_SAMPLING = 2, AAL_BOTH = 3, AAL_KL = 4, AAL_GRPO = 8, AAL_TV = 16, AAL_IDS = 32
 } aal_mode;
@@ -250,6 +250,28 @@ AAL_API aal_status aal_grpo_from_loss(const aal_grpo_problem* gprob, const aal_p
                                       const void* ref_draft, void* workspace, size_t workspace_bytes,
                                       float* grpo_loss, int32_t* tau, int32_t* tau_ref, float* advantage,
                                       float* log_rho, void* stream);
+
+/* The GRPO stage over sequences (Sec. 3.4: the forward passes run once per sequence and the window
+ * samples are sliced from them), after aal_seq_loss_fwd with a mode that includes AAL_GRPO.
+ *   gprob      N = the number of windows; K, V, dtype equal the sequence problem's; grouping,
+ *              clips and w_grpo as for aal_grpo_from_loss (N a multiple of
+ *              windows_per_rollout * rollouts_per_group).
+ *   starts     device int32[N]: the flat start position b * seq_len + t of each window, in
+ *              ascending order, each window inside its sequence (t + K <= seq_len).  Windows may
+ *              overlap.  A start that breaks this is reported as AAL_ERR_INVALID_ARG through the
+ *              status word of `workspace` (aal_check_device_status) and its window reads nothing.
+ *   ref_draft  [B][seq_len][V] logits of the reference draft: read once, every position.
+ *   workspace  at least aal_seq_grpo_workspace_size() bytes, 256-byte aligned.
+ * Outputs as for aal_grpo_from_loss (tau, tau_ref, log_rho per window).  The loss workspace
+ * receives, per position, the sum over the windows that cover it of their coefficients, so the
+ * following aal_seq_loss_bwd adds the gradient of w_grpo * L_GRPO to every covered position. */
+AAL_API aal_status aal_seq_grpo_workspace_size(const aal_grpo_problem* gprob, const aal_seq_problem* sprob,
+                                               size_t* bytes);
+AAL_API aal_status aal_seq_grpo_from_loss(const aal_grpo_problem* gprob, const aal_seq_problem* sprob,
+                                          void* loss_workspace, size_t loss_workspace_bytes,
+                                          const void* ref_draft, const int32_t* starts, void* workspace,
+                                          size_t workspace_bytes, float* grpo_loss, int32_t* tau,
+                                          int32_t* tau_ref, float* advantage, float* log_rho, void* stream);
 
 /* Reward mode flag: with AAL_SAMPLING, the drafted token is drawn from q~ instead of taken as
  * the draft's argmax (aal_reward_problem.mode = AAL_SAMPLING | AAL_SAMPLED_DRAFT). */

@@ -42,6 +42,8 @@ from .aal import (  # noqa: F401
     aal_debug_fail_next_forward,
     aal_grpo_from_loss,
     aal_grpo_workspace_size,
+    aal_seq_grpo_from_loss,
+    aal_seq_grpo_workspace_size,
     aal_loss_bwd,
     aal_loss_fwd,
     aal_reward_workspace_size,
@@ -54,6 +56,7 @@ from .aal import (  # noqa: F401
     library_path,
     loss_problem,
     grpo_problem,
+    grpo_seq_problem,
     reward_problem,
     seq_problem,
 )

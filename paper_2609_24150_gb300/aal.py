@@ -109,6 +109,8 @@ def library() -> ctypes.CDLL:
     GP = ctypes.POINTER(AalGrpoProblem)
     lib.aal_grpo_workspace_size.argtypes = [GP, ctypes.POINTER(sz)]
     lib.aal_grpo_from_loss.argtypes = [GP, P, vp, sz, vp, vp, sz, vp, vp, vp, vp, vp, vp]
+    lib.aal_seq_grpo_workspace_size.argtypes = [GP, SP, ctypes.POINTER(sz)]
+    lib.aal_seq_grpo_from_loss.argtypes = [GP, SP, vp, sz, vp, vp, vp, sz, vp, vp, vp, vp, vp, vp]
     lib.aal_check_device_status.argtypes = [vp, vp]
     lib.aal_debug_fail_next_forward.argtypes = [ctypes.c_int64, ctypes.c_uint64]
     lib.aal_debug_fail_next_forward.restype = None
@@ -119,7 +121,8 @@ def library() -> ctypes.CDLL:
     for f in ("aal_workspace_size", "aal_reward_workspace_size", "aal_loss_fwd", "aal_loss_bwd",
               "aal_accept_reward", "aal_accept_reward_noalloc", "aal_accept_reward_from_loss",
               "aal_seq_workspace_size", "aal_seq_loss_fwd", "aal_seq_loss_bwd", "aal_check_device_status",
-              "aal_grpo_workspace_size", "aal_grpo_from_loss"):
+              "aal_grpo_workspace_size", "aal_grpo_from_loss", "aal_seq_grpo_workspace_size",
+              "aal_seq_grpo_from_loss"):
         getattr(lib, f).restype = ctypes.c_int
     _LIB = lib
     return lib
@@ -278,6 +281,42 @@ def aal_grpo_from_loss(problem: AalGrpoProblem, loss_problem_: AalProblem, loss_
         _ptr(advantage, "advantage", torch.float32, nroll), _ptr(log_rho, "log_rho", torch.float32, N),
         _stream(stream))
     _check(code, "aal_grpo_from_loss")
+
+
+def grpo_seq_problem(n_windows: int, draft: torch.Tensor, K: int, windows_per_rollout: int = 1,
+                     rollouts_per_group: int = 1, adv_clip: float = 5.0, eps_clip: float = 0.2,
+                     rho_min: float = 0.0, rho_max: float = 10.0, log_rho_clip: float = 10.0,
+                     w_grpo: float = 1.0) -> AalGrpoProblem:
+    """GRPO problem struct for n_windows windows of K positions sliced from [B][T][V] logits."""
+    if draft.dim() != 3:
+        raise ValueError("logits must be [B][seq_len][V]")
+    V = draft.shape[2]
+    return AalGrpoProblem(n_windows, K, V, _DTYPES[draft.dtype], 0, windows_per_rollout, rollouts_per_group,
+                          adv_clip, eps_clip, rho_min, rho_max, log_rho_clip, w_grpo)
+
+
+def aal_seq_grpo_workspace_size(problem: AalGrpoProblem, seq_problem_: AalSeqProblem) -> int:
+    out = ctypes.c_size_t(0)
+    _check(library().aal_seq_grpo_workspace_size(ctypes.byref(problem), ctypes.byref(seq_problem_),
+                                                 ctypes.byref(out)), "aal_seq_grpo_workspace_size")
+    return out.value
+
+
+def aal_seq_grpo_from_loss(problem: AalGrpoProblem, seq_problem_: AalSeqProblem, loss_workspace, ref_draft,
+                           starts, workspace, grpo_loss, tau=None, tau_ref=None, advantage=None, log_rho=None,
+                           stream=None):
+    """GRPO stage over windows sliced from sequences (ascending flat start positions), after
+    aal_seq_loss_fwd with AAL_GRPO; writes the per-position gradient coefficients."""
+    N = problem.N
+    nroll = N // max(1, problem.windows_per_rollout)
+    code = library().aal_seq_grpo_from_loss(
+        ctypes.byref(problem), ctypes.byref(seq_problem_), _ptr(loss_workspace, "loss_workspace"),
+        _nbytes(loss_workspace), _ptr(ref_draft, "ref_draft"), _ptr(starts, "starts", torch.int32, N),
+        _ptr(workspace, "workspace"), _nbytes(workspace), _ptr(grpo_loss, "grpo_loss", torch.float32, 1),
+        _ptr(tau, "tau", torch.int32, N), _ptr(tau_ref, "tau_ref", torch.int32, N),
+        _ptr(advantage, "advantage", torch.float32, nroll), _ptr(log_rho, "log_rho", torch.float32, N),
+        _stream(stream))
+    _check(code, "aal_seq_grpo_from_loss")
 
 
 def aal_seq_workspace_size(problem: AalSeqProblem) -> int:

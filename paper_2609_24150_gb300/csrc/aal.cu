@@ -67,10 +67,7 @@ aal_status check_seq(const aal_seq_problem* p) {
   // the per-depth partials too)
   const aal_problem q{p->B * p->seq_len, p->K, p->V, p->dtype, p->mode, p->temperature, p->w_greedy,
                       p->w_sampling, p->w_kl, p->w_tv, p->reserved};
-  aal_status st = check_problem(&q);
-  if (st != AAL_OK) return st;
-  if (p->mode & AAL_GRPO) return AAL_ERR_UNSUPPORTED;  // the GRPO stage runs over windows
-  return AAL_OK;
+  return check_problem(&q);
 }
 
 aal_status check_grpo(const aal_grpo_problem* p) {
@@ -294,6 +291,10 @@ aal_status aal_seq_loss_fwd(const aal_seq_problem* prob, const void* draft, cons
   LossWs ws = loss_ws(workspace, L.base);
   cudaError_t e = cudaMemsetAsync(ws.hdr, 0, sizeof(WsHeader), s);
   if (e != cudaSuccess) return AAL_ERR_CUDA;
+  if (prob->mode & AAL_GRPO) {  // no GRPO term until aal_seq_grpo_from_loss writes one
+    e = cudaMemsetAsync(ws.cgr, 0, (size_t)R * sizeof(float), s);
+    if (e != cudaSuccess) return AAL_ERR_CUDA;
+  }
   int cluster = 1;
   e = launch_stats(draft, target, R, prob->V, prob->dtype, prob->mode, prob->temperature, ws, s, &cluster);
   if (e != cudaSuccess) return AAL_ERR_CUDA;
@@ -411,6 +412,9 @@ aal_status aal_grpo_from_loss(const aal_grpo_problem* gprob, const aal_problem* 
   GrpoWindowArgs wa;
   wa.lws = lws;
   wa.lpr = ra.lpr;
+  wa.starts = nullptr;
+  wa.RP = 0;
+  wa.cw = nullptr;
   wa.adv = adv;
   wa.N = gprob->N;
   wa.K = (int32_t)gprob->K;
@@ -426,6 +430,118 @@ aal_status aal_grpo_from_loss(const aal_grpo_problem* gprob, const aal_problem* 
   wa.hdr = hdr;
   wa.loss = grpo_loss;
   return cuda_status(launch_grpo_windows(wa, s));
+}
+
+aal_status aal_seq_grpo_workspace_size(const aal_grpo_problem* gprob, const aal_seq_problem* sprob, size_t* bytes) {
+  aal_status st = check_grpo(gprob);
+  if (st != AAL_OK) return st;
+  st = check_seq(sprob);
+  if (st != AAL_OK) return st;
+  if (bytes == nullptr) return AAL_ERR_INVALID_ARG;
+  *bytes = seq_grpo_layout(gprob->N, gprob->K, gprob->windows_per_rollout, sprob->B * sprob->seq_len).total;
+  return AAL_OK;
+}
+
+aal_status aal_seq_grpo_from_loss(const aal_grpo_problem* gprob, const aal_seq_problem* sprob, void* loss_workspace,
+                                  size_t loss_workspace_bytes, const void* ref_draft, const int32_t* starts,
+                                  void* workspace, size_t workspace_bytes, float* grpo_loss, int32_t* tau,
+                                  int32_t* tau_ref, float* advantage, float* log_rho, void* stream) {
+  aal_status st = check_grpo(gprob);
+  if (st != AAL_OK) return st;
+  st = check_seq(sprob);
+  if (st != AAL_OK) return st;
+  if (!(sprob->mode & AAL_GRPO)) return AAL_ERR_INVALID_ARG;
+  if (gprob->K != sprob->K || gprob->V != sprob->V || gprob->dtype != sprob->dtype) return AAL_ERR_INVALID_ARG;
+  if (grpo_loss == nullptr || !aligned(grpo_loss, 4) || (tau != nullptr && !aligned(tau, 4)) ||
+      (tau_ref != nullptr && !aligned(tau_ref, 4)) || (advantage != nullptr && !aligned(advantage, 4)) ||
+      (log_rho != nullptr && !aligned(log_rho, 4)))
+    return AAL_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int64_t RP = sprob->B * sprob->seq_len;
+  if (RP == 0) return cuda_status(cudaMemsetAsync(grpo_loss, 0, sizeof(float), s));
+  if (ref_draft == nullptr || !aligned(ref_draft, 16)) return AAL_ERR_INVALID_ARG;
+  if (gprob->N > 0 && (starts == nullptr || !aligned(starts, 4))) return AAL_ERR_INVALID_ARG;
+  const SeqLayout SL = seq_layout(sprob->B, sprob->seq_len, sprob->K);
+  if (loss_workspace == nullptr || !aligned(loss_workspace, 256) || loss_workspace_bytes < SL.total)
+    return AAL_ERR_WORKSPACE;
+  const SeqGrpoLayout L = seq_grpo_layout(gprob->N, gprob->K, gprob->windows_per_rollout, RP);
+  if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < L.total) return AAL_ERR_WORKSPACE;
+  char* base = static_cast<char*>(workspace);
+  WsHeader* hdr = reinterpret_cast<WsHeader*>(base + L.g.hdr);
+  if (cudaMemsetAsync(hdr, 0, sizeof(WsHeader), s) != cudaSuccess) return AAL_ERR_CUDA;
+  const LossWs lws = loss_ws(loss_workspace, SL.base);
+
+  // the reference pass over every position: log pi_ref at the draft's token, both flags
+  Stream1Args ra;
+  ra.z = ref_draft;
+  ra.R = RP;
+  ra.V = gprob->V;
+  ra.lws = lws;
+  ra.ids = nullptr;
+  ra.acc = reinterpret_cast<uint8_t*>(base + L.acc_pos);
+  ra.acc_ref = reinterpret_cast<uint8_t*>(base + L.accr_pos);
+  ra.lpr = reinterpret_cast<float*>(base + L.lpr_pos);
+  ra.hdr = hdr;
+  ra.skip_chunk = debug_take_skip_chunk();
+  if (launch_one_tensor(ra, gprob->dtype == AAL_BF16, false, s) != cudaSuccess) return AAL_ERR_CUDA;
+
+  if (gprob->N == 0) {  // no windows: no GRPO term
+    if (cudaMemsetAsync(lws.cgr, 0, (size_t)RP * sizeof(float), s) != cudaSuccess) return AAL_ERR_CUDA;
+    return cuda_status(cudaMemsetAsync(grpo_loss, 0, sizeof(float), s));
+  }
+  SeqGrpoArgs qa;
+  qa.starts = starts;
+  qa.N = gprob->N;
+  qa.T = sprob->seq_len;
+  qa.RP = RP;
+  qa.K = (int32_t)gprob->K;
+  qa.acc_pos = ra.acc;
+  qa.accr_pos = ra.acc_ref;
+  qa.acc = reinterpret_cast<uint8_t*>(base + L.g.acc);
+  qa.acc_ref = reinterpret_cast<uint8_t*>(base + L.g.acc_ref);
+  qa.cw = reinterpret_cast<float*>(base + L.cw);
+  qa.cgr = lws.cgr;
+  qa.hdr = hdr;
+  if (launch_seq_grpo_gather(qa, s) != cudaSuccess) return AAL_ERR_CUDA;
+
+  float* adv = advantage != nullptr ? advantage : reinterpret_cast<float*>(base + L.g.adv);
+  RewardGroupArgs ga;
+  ga.acc = qa.acc;
+  ga.acc_ref = qa.acc_ref;
+  ga.rbuf = reinterpret_cast<float*>(base + L.g.rbuf);
+  ga.N = gprob->N;
+  ga.K = (int32_t)gprob->K;
+  ga.wpr = gprob->windows_per_rollout;
+  ga.rpg = gprob->rollouts_per_group;
+  ga.adv_clip = gprob->adv_clip;
+  ga.tau = tau != nullptr ? tau : reinterpret_cast<int32_t*>(base + L.g.tau);
+  ga.tau_ref = tau_ref != nullptr ? tau_ref : reinterpret_cast<int32_t*>(base + L.g.tau_ref);
+  ga.rollout_len = reinterpret_cast<float*>(base + L.g.rl);
+  ga.advantage = adv;
+  if (launch_reward_groups(ga, s) != cudaSuccess) return AAL_ERR_CUDA;
+
+  GrpoWindowArgs wa;
+  wa.lws = lws;
+  wa.lpr = ra.lpr;
+  wa.starts = starts;
+  wa.RP = RP;
+  wa.cw = reinterpret_cast<float*>(base + L.cw);
+  wa.adv = adv;
+  wa.N = gprob->N;
+  wa.K = (int32_t)gprob->K;
+  wa.wpr = gprob->windows_per_rollout;
+  wa.eps_clip = gprob->eps_clip;
+  wa.rho_min = gprob->rho_min;
+  wa.rho_max = gprob->rho_max;
+  wa.log_rho_clip = gprob->log_rho_clip;
+  wa.w_grpo = gprob->w_grpo;
+  wa.log_rho = log_rho;
+  wa.part = reinterpret_cast<double*>(base + L.g.part);
+  wa.nblk = L.g.nblk;
+  wa.hdr = hdr;
+  wa.loss = grpo_loss;
+  if (launch_grpo_windows(wa, s) != cudaSuccess) return AAL_ERR_CUDA;
+  return cuda_status(launch_seq_grpo_scatter(qa, s));
 }
 
 aal_status aal_accept_reward(const aal_reward_problem* prob, const void* draft, const void* target,

@@ -331,10 +331,54 @@ struct Stream1Args {
   int64_t skip_chunk;  // failure-detection test hook: a chunk whose copy is never armed (-1: none)
 };
 
+// GRPO over sequences (aal_seq_grpo_from_loss): per-position flags and log pi_ref from the
+// reference pass, the windows' rows gathered from them, and the windows' coefficients before
+// they are added per position.
+struct SeqGrpoLayout {
+  GrpoLayout g;        // per-window buffers (acc, acc_ref, rewards, advantages, partials)
+  int64_t RP = 0;      // positions B*T
+  size_t acc_pos = 0, accr_pos = 0, lpr_pos = 0, cw = 0;
+  size_t total = 0;
+};
+
+inline SeqGrpoLayout seq_grpo_layout(int64_t N, int64_t K, int64_t wpr, int64_t positions) {
+  SeqGrpoLayout L;
+  L.g = grpo_layout(N, K, wpr);
+  L.RP = positions;
+  size_t off = L.g.total;
+  auto take = [&](size_t bytes) {
+    size_t o = off;
+    off = align_up(off + bytes, 256);
+    return o;
+  };
+  L.acc_pos = take((size_t)positions);
+  L.accr_pos = take((size_t)positions);
+  L.lpr_pos = take((size_t)positions * 4);
+  L.cw = take((size_t)(N * K) * 4);
+  L.total = off;
+  return L;
+}
+
+struct SeqGrpoArgs {
+  const int32_t* starts;  // [N] flat start position of each window (ascending)
+  int64_t N, T, RP;
+  int32_t K;
+  const uint8_t* acc_pos;
+  const uint8_t* accr_pos;
+  uint8_t* acc;           // [N][K] gathered
+  uint8_t* acc_ref;
+  const float* cw;        // [N][K] coefficients of the window rows
+  float* cgr;             // [RP] per position (loss workspace)
+  WsHeader* hdr;          // status word: AAL_ERR_INVALID_ARG for a bad start
+};
+
 // Per window: log rho, the clipped surrogate, its per-row gradient coefficients.
 struct GrpoWindowArgs {
   LossWs lws;          // Lsq1 (log pi_theta(y) = -ln2 Lsq1), cgr out
   const float* lpr;
+  const int32_t* starts;  // null: window rows are n*K + k; else positions starts[n] + k
+  int64_t RP;             // with starts: the number of positions
+  float* cw;              // with starts: the window rows' coefficients ([N][K]), not lws.cgr
   const float* adv;    // [N / wpr]
   int64_t N;
   int32_t K;
@@ -363,6 +407,8 @@ cudaError_t launch_reward_groups(const RewardGroupArgs& a, cudaStream_t s);
 cudaError_t launch_reward_flags_from_stats(const RewardStatsArgs& a, cudaStream_t s);
 cudaError_t launch_one_tensor(const Stream1Args& a, bool bf16, bool ids, cudaStream_t s);
 cudaError_t launch_grpo_windows(const GrpoWindowArgs& a, cudaStream_t s);
+cudaError_t launch_seq_grpo_gather(const SeqGrpoArgs& a, cudaStream_t s);
+cudaError_t launch_seq_grpo_scatter(const SeqGrpoArgs& a, cudaStream_t s);
 
 // ---------------------------------------------------------------------------
 // Device helpers.

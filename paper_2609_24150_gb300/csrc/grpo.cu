@@ -29,9 +29,16 @@ __global__ void __launch_bounds__(kGrpoThreads) grpo_windows(GrpoWindowArgs a) {
   double surr = 0.0;
   if (t < a.N) {
     const int K = a.K;
+    // the window's rows: n*K + k, or (sequence layout) positions start + k, whose bounds the
+    // gather kernel has checked (a bad start reads position 0 here and is reported there)
+    int64_t row0 = t * K;
+    if (a.starts != nullptr) {
+      const int64_t st = a.starts[t];
+      row0 = (st >= 0 && st + K <= a.RP) ? st : 0;
+    }
     float sum = 0.f;
     for (int k = 0; k < K; ++k) {
-      const int64_t r = t * K + k;
+      const int64_t r = row0 + k;
       sum += -kLn2 * a.lws.Lsq1[r] - a.lpr[r];
     }
     const float raw = sum / (float)K;
@@ -45,7 +52,8 @@ __global__ void __launch_bounds__(kGrpoThreads) grpo_windows(GrpoWindowArgs a) {
     const bool inside = raw >= -a.log_rho_clip && raw <= a.log_rho_clip && rho_e >= a.rho_min &&
                         rho_e <= a.rho_max;
     const float coef = (unclipped && inside) ? a.w_grpo * (-1.f / (float)a.N) * A * rho_e / (float)K : 0.f;
-    for (int k = 0; k < K; ++k) a.lws.cgr[t * K + k] = coef;
+    float* out = a.starts != nullptr ? a.cw + t * K : a.lws.cgr + t * K;
+    for (int k = 0; k < K; ++k) out[k] = coef;
     if (a.log_rho != nullptr) a.log_rho[t] = lr;
     surr = s;
   }
@@ -78,6 +86,55 @@ __global__ void __launch_bounds__(kGrpoThreads) grpo_windows(GrpoWindowArgs a) {
 }
 
 }  // namespace
+
+// Sequence layout: each window row (n, k) takes the flags of position starts[n] + k.  A start
+// outside [0, RP - K], across a sequence end, or below the previous one records
+// AAL_ERR_INVALID_ARG and its rows read nothing (flags 0).
+__global__ void __launch_bounds__(256) seq_grpo_gather(SeqGrpoArgs a) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= a.N * a.K) return;
+  const int64_t n = i / a.K;
+  const int k = (int)(i - n * a.K);
+  const int64_t st = a.starts[n];
+  const bool ok = st >= 0 && st + a.K <= a.RP && (st % a.T) + a.K <= a.T && (n == 0 || a.starts[n - 1] <= st);
+  if (!ok && k == 0) atomicExch(&a.hdr->status, 1u);  // == AAL_ERR_INVALID_ARG
+  a.acc[i] = ok ? a.acc_pos[st + k] : 0;
+  a.acc_ref[i] = ok ? a.accr_pos[st + k] : 0;
+}
+
+// Per position p: the coefficients of the window rows that land on it, windows in start order
+// (starts ascending, so they are the windows with start in [p - K + 1, p], found by binary
+// search): a fixed order of at most K terms, no atomics.
+__global__ void __launch_bounds__(256) seq_grpo_scatter(SeqGrpoArgs a) {
+  const int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (p >= a.RP) return;
+  const int64_t lo_start = p - a.K + 1;
+  int64_t lo = 0, hi = a.N;  // first window with start >= lo_start
+  while (lo < hi) {
+    const int64_t mid = (lo + hi) >> 1;
+    if (a.starts[mid] < lo_start) lo = mid + 1;
+    else hi = mid;
+  }
+  float c = 0.f;
+  for (int64_t n = lo; n < a.N && a.starts[n] <= p; ++n) {
+    const int64_t k = p - a.starts[n];
+    if (k >= 0 && k < a.K) c += a.cw[n * a.K + k];
+  }
+  a.cgr[p] = c;
+}
+
+cudaError_t launch_seq_grpo_gather(const SeqGrpoArgs& a, cudaStream_t s) {
+  const int64_t n = a.N * a.K;
+  if (n < 1) return cudaSuccess;
+  seq_grpo_gather<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_seq_grpo_scatter(const SeqGrpoArgs& a, cudaStream_t s) {
+  if (a.RP < 1) return cudaSuccess;
+  seq_grpo_scatter<<<(unsigned)((a.RP + 255) / 256), 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_grpo_windows(const GrpoWindowArgs& a, cudaStream_t s) {
   if (a.nblk < 1) return cudaSuccess;

@@ -285,5 +285,20 @@ def test_grpo_needs_a_matching_loss_problem_with_the_grpo_bit():
                                   fake, None, None, None, None, None) == aal.AAL_ERR_WORKSPACE
 
 
-def test_sequence_layout_refuses_the_grpo_bit():
-    assert _seq_ws(_sprob(mode=aal.AAL_GREEDY | aal.AAL_GRPO))[0] == aal.AAL_ERR_UNSUPPORTED
+def test_sequence_grpo_checks():
+    lib = aal.library()
+    sp = _sprob(B=2, seq_len=16, K=4, mode=aal.AAL_GREEDY | aal.AAL_GRPO)
+    assert _seq_ws(sp)[0] == aal.AAL_OK
+    g = _gprob(N=8, K=4)
+    out = ctypes.c_size_t(0)
+    assert lib.aal_seq_grpo_workspace_size(ctypes.byref(g), ctypes.byref(sp), ctypes.byref(out)) == aal.AAL_OK
+    size = out.value
+    fake, fake_ws, big = 1 << 24, 1 << 20, 1 << 30
+    args = lambda gp, spp, starts, ws_bytes: (ctypes.byref(gp), ctypes.byref(spp), fake_ws, big, fake, starts,
+                                              fake_ws, ws_bytes, fake, None, None, None, None, None)
+    assert lib.aal_seq_grpo_from_loss(*args(g, sp, None, size)) == aal.AAL_ERR_INVALID_ARG      # no starts
+    assert lib.aal_seq_grpo_from_loss(*args(g, sp, fake + 2, size)) == aal.AAL_ERR_INVALID_ARG  # misaligned
+    assert lib.aal_seq_grpo_from_loss(*args(g, sp, fake, size - 1)) == aal.AAL_ERR_WORKSPACE
+    assert lib.aal_seq_grpo_from_loss(*args(_gprob(N=8, K=3), sp, fake, size)) == aal.AAL_ERR_INVALID_ARG
+    no_grpo = _sprob(B=2, seq_len=16, K=4, mode=aal.AAL_GREEDY)
+    assert lib.aal_seq_grpo_from_loss(*args(g, no_grpo, fake, size)) == aal.AAL_ERR_INVALID_ARG
