@@ -486,7 +486,10 @@ def run_seq_grpo_phase(aal, dev, stream, rank, reps):
     ms = [sum(e[i].elapsed_time(e[i + 1]) for e in ev) / reps for i in range(3)]
     R = B * T
     row = V * draft.element_size()
-    b = [2 * R * row, R * row, 3 * R * row]   # masked rows are still read; the masked backward rows are written
+    n_valid = int(mask.sum().item())
+    # forward and reference pass read every position; the backward reads draft and target of a
+    # valid position and writes its row, and only writes the zero row of a masked one
+    b = [2 * R * row, R * row, (3 * n_valid + (R - n_valid)) * row]
     tot = sum(ms)
     out = {"workload": f"seq_v128k: B={B} x T={T} positions, K={K}, V={V} bf16, masked; L_KL + 0.1 L_EAL + "
                        f"0.1 L_GRPO over {N} windows (8 anchors per sequence x groups of {m})",
