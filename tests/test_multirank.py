@@ -3,7 +3,8 @@
 Windows are independent, so ranks shard them with no collective on the data path; only the
 step time is reduced (max over ranks).  The reward's counter-based draws are keyed by the
 global window index, so a sharded run reproduces the unsharded one exactly, and per-rank
-loss partials (sum of w * E[L], |W|) combine into the global loss with one all-reduce.
+loss partials (sum of w * E[L], |W|; with the anchor also sum KL and |positions|) combine
+into the global loss with one all-reduce, for windows and for sharded sequences.
 """
 
 import multiprocessing as mp
@@ -45,6 +46,18 @@ def _worker(rank, world, port, out):
                             dtype=torch.float64)
         dist.all_reduce(part)
         res["loss"] = float(-part[0] / part[1])
+        # sequence layout, sequences sharded: the partials of L_KL + 0.1 L_EAL are
+        # (sum E^g, |W|, sum KL, |positions|), one all-reduce of four numbers
+        st, sd, sm = synth.make_seq_logits("seq_tiny", seed=4, B=4, seq_len=11, V=50)
+        bper = 4 // world
+        b0 = rank * bper
+        ts, ds, ms = st[b0:b0 + bper], sd[b0:b0 + bper], sm[b0:b0 + bper].numpy()
+        fe = oracle.seq_loss_forward(ts, ds, ms, 3, oracle.MODE_GREEDY)
+        an = oracle.anchor_forward(ts, ds, ms)
+        sp = torch.tensor([fe["eal_g"].sum(), float(fe["nvalid"]), float(np.sum(an["kl"][an["valid"]])),
+                           float(an["npos"])], dtype=torch.float64)
+        dist.all_reduce(sp)
+        res["seq_loss"] = float(-0.1 * sp[0] / sp[1] + sp[2] / sp[3])
         out.put((rank, res))
     finally:
         dist.destroy_process_group()
@@ -67,7 +80,11 @@ def test_two_gloo_ranks():
     whole = oracle.accept_reward(target, draft, None, 2, 0.9, seed=7, row_offset=0, windows_per_rollout=2,
                                  rollouts_per_group=2)
     ref_loss = oracle.loss_forward(target, draft, None, oracle.MODE_BOTH, 0.9, 0.5, 0.5)["loss"]
+    st, sd, sm = synth.make_seq_logits("seq_tiny", seed=4, B=4, seq_len=11, V=50)
+    ref_seq = oracle.seq_objective_forward(st, sd, sm.numpy(), 3, oracle.MODE_KL | oracle.MODE_GREEDY, 1.0,
+                                           0.1, 0.0, 1.0)["loss"]
     for r in range(2):
         assert results[r]["max"] == 20.0
         np.testing.assert_array_equal(results[r]["tau"], whole["tau"])
         assert abs(results[r]["loss"] - ref_loss) < 1e-12
+        assert abs(results[r]["seq_loss"] - ref_seq) < 1e-12
