@@ -1,0 +1,58 @@
+"""The step as a CUDA graph: aal_loss_fwd, aal_loss_bwd and aal_accept_reward_from_loss launch
+only kernels and async memsets on the caller's stream, so they can be captured once and replayed
+(for callers with many small batches, where launch latency matters).  Replays must reproduce
+eager launches bit for bit (every reduction has a fixed order)."""
+
+import pytest
+import torch
+
+import paper_2609_24150_gb300 as aal
+import synth
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda:0"
+
+
+@pytest.mark.parametrize("mode,T", [(aal.AAL_BOTH, 1.0), (aal.AAL_KL | aal.AAL_GREEDY, 1.0), (aal.AAL_SAMPLING, 0.8)])
+def test_step_replays_bit_exactly(mode, T):
+    target, draft, mask = synth.make_logits("v32k", seed=6, n_windows=256)
+    t, d, m = target.to(DEV), draft.to(DEV), mask.to(DEV)
+    N = d.shape[0]
+    prob = aal.loss_problem(d, mode, T, 0.4, 0.6, 1.0)
+    rprob = aal.reward_problem(d, aal.AAL_GREEDY, windows_per_rollout=16, rollouts_per_group=16)
+    ws = torch.empty(aal.aal_workspace_size(prob), dtype=torch.uint8, device=DEV)
+    rws = torch.empty(aal.aal_reward_workspace_size(rprob), dtype=torch.uint8, device=DEV)
+    loss = torch.empty(1, device=DEV)
+    eal = torch.empty(N, 2, device=DEV)
+    grad = torch.empty_like(d)
+    tau = torch.empty(N, dtype=torch.int32, device=DEV)
+    rl = torch.empty(N // 16, device=DEV)
+    adv = torch.empty(N // 16, device=DEV)
+
+    def step():
+        aal.aal_loss_fwd(prob, d, t, m, ws, loss, eal)
+        aal.aal_loss_bwd(prob, d, t, m, ws, 2.0, grad)
+        aal.aal_accept_reward_from_loss(rprob, prob, ws, rws, tau, rl, adv)
+
+    step()
+    torch.cuda.synchronize()
+    ref = [x.clone() for x in (loss, eal, grad, tau, adv)]
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):          # warm the launchers on the capture stream
+        step()
+    torch.cuda.current_stream().wait_stream(s)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        step()
+    for x in (loss, eal, grad):
+        x.fill_(float("nan"))
+    tau.fill_(-1)
+    for _ in range(2):
+        g.replay()
+        torch.cuda.synchronize()
+        assert aal.aal_check_device_status(ws) == aal.AAL_OK
+        for a, b in zip((loss, eal, grad, tau, adv), ref):
+            assert torch.equal(a, b)
