@@ -559,19 +559,22 @@ def run_e2e(args, aal, prob, rprob, draft, target, grad, ws, loss, rws, tau, rl,
     if avail is not None and need > avail // 3:
         return {"value": None, "unit": "GB/s", "skipped": f"pinned inputs need {need / 1e9:.1f} GB, "
                 f"host has {avail / 1e9:.1f} GB available"}
-    d_h = torch.empty(draft.shape, dtype=draft.dtype, pin_memory=True)
-    t_h = torch.empty(target.shape, dtype=target.dtype, pin_memory=True)
-    d_h.copy_(draft)
-    t_h.copy_(target)
+    # both inputs staged in ONE pinned allocation and copied into one device buffer whose two
+    # halves are the kernels' inputs: on this host two separate 14.7 GB pinned allocations copied
+    # at 85-210 GB/s, one allocation at a steady ~200 GB/s
+    both_h = torch.empty((2,) + tuple(draft.shape), dtype=draft.dtype, pin_memory=True)
+    both_h[0].copy_(draft)
+    both_h[1].copy_(target)
+    both = torch.empty((2,) + tuple(draft.shape), dtype=draft.dtype, device=draft.device)
+    d_in, t_in = both[0], both[1]
     loss_h = torch.empty(1, dtype=torch.float32, pin_memory=True)
     adv_h = torch.empty(adv.shape, dtype=torch.float32, pin_memory=True)
     rl_h = torch.empty(rl.shape, dtype=torch.float32, pin_memory=True)
 
     def e2e_step():
-        draft.copy_(d_h, non_blocking=True)
-        target.copy_(t_h, non_blocking=True)
-        aal.aal_loss_fwd(prob, draft, target, None, ws, loss, None, stream)
-        aal.aal_loss_bwd(prob, draft, target, None, ws, 1.0, grad, stream)
+        both.copy_(both_h, non_blocking=True)
+        aal.aal_loss_fwd(prob, d_in, t_in, None, ws, loss, None, stream)
+        aal.aal_loss_bwd(prob, d_in, t_in, None, ws, 1.0, grad, stream)
         aal.aal_accept_reward_from_loss(rprob, prob, ws, rws, tau, rl, adv, stream)
         loss_h.copy_(loss, non_blocking=True)
         adv_h.copy_(adv, non_blocking=True)
@@ -587,7 +590,7 @@ def run_e2e(args, aal, prob, rprob, draft, target, grad, ws, loss, rws, tau, rl,
     z.record(stream)
     torch.cuda.synchronize()
     ms = a.elapsed_time(z) / args.e2e_steps
-    del d_h, t_h
+    del both_h, both
     return {"value": round(step_bytes / (ms * 1e-3) / 1e9, 1), "unit": "GB/s", "ms_per_step": round(ms, 3),
             "h2d_bytes_per_step": need, "d2h_bytes_per_step": 4 + 2 * 4 * adv.numel(),
             "steps": args.e2e_steps}
