@@ -105,6 +105,15 @@ __device__ __forceinline__ bool wait_phase(uint64_t* b, uint32_t parity, volatil
   return false;
 }
 
+// Consumer side of a ring slot: a phase that has already completed is taken after one
+// non-blocking test, without reading the abort flag; otherwise the bounded wait above.
+// After an abort a consumer may so still read a landed (or stale) slot: its results are
+// discarded, since every output write is guarded by the abort flag.
+__device__ __forceinline__ bool wait_full(uint64_t* b, uint32_t parity, volatile int* abort_flag,
+                                          uint64_t limit_ns, WsHeader* hdr) {
+  return mbar_test(b, parity) || wait_phase(b, parity, abort_flag, limit_ns, hdr);
+}
+
 // ---------------------------------------------------------------- packed arithmetic
 // Two fp32 lanes per instruction (sm_100+), IEEE round-to-nearest like the scalar forms.
 #ifndef AAL_F2_ASM

@@ -25,8 +25,9 @@
 //
 // There is no cross-CTA communication, so all 152 SMs run one CTA each.  Every wait is
 // bounded (ptx::wait_phase); after a timeout every thread keeps walking the same loops
-// without waiting or computing, so all meet the same named barriers, the producer drains
-// its copies, and the kernel returns with AAL_ERR_TIMEOUT in the workspace status word.
+// without waiting (a consumer still folds a chunk it finds landed, into results that are
+// never written), so all meet the same named barriers, the producer drains its copies,
+// and the kernel returns with AAL_ERR_TIMEOUT in the workspace status word.
 #include "ptx.cuh"
 
 namespace aal {
@@ -201,8 +202,24 @@ __device__ __forceinline__ void lse_kl_words(float& M, float& S, float& D, const
   D += dacc.x + dacc.y;
 }
 
+// The first of a thread's NV vectors whose maximum (vm[v], packed bf16 pair) equals m:
+// the running argmax moves there.  Called only when m beats the running maximum, which
+// after the first chunks of a row is rare.
+template <int NV>
+__device__ __forceinline__ void first_vec_at(float& best, int32_t& at, const uint32_t* vm, float m, int idx0,
+                                             int vstride) {
+  int v0 = NV - 1;
+#pragma unroll
+  for (int v = NV - 2; v >= 0; --v)
+    if (fmaxf(bf16_lo(vm[v]), bf16_hi(vm[v])) == m) v0 = v;
+  best = m;
+  at = idx0 + v0 * vstride;
+}
+
 // Phase 1 on NV 16-byte vectors of bf16 per tensor; vector v holds elements
-// idx0 + v * vstride + [0, 8).
+// idx0 + v * vstride + [0, 8).  The maxima are taken on packed bf16 pairs: per vector, then
+// over the thread's vectors; only a maximum that beats the running one looks for its vector
+// (the first in element order, as a strict per-vector update in that order would).
 template <int NV, bool NEED_Q1, bool KL = false>
 __device__ __forceinline__ void phase1_bf16(RowPart& A, const uint4* pv, const uint4* qv, int idx0, int vstride,
                                             float sT) {
@@ -219,17 +236,21 @@ __device__ __forceinline__ void phase1_bf16(RowPart& A, const uint4* pv, const u
     qw[4 * v + 2] = qv[v].z;
     qw[4 * v + 3] = qv[v].w;
   }
-  float pm = -INFINITY, qm = -INFINITY;
+  uint32_t vp[NV], vq[NV];
 #pragma unroll
-  for (int v = 0; v < NV; ++v) {  // per-vector maxima of z_p and z_q, in element order
-    const uint32_t mp = bmax2(bmax2(pw[4 * v], pw[4 * v + 1]), bmax2(pw[4 * v + 2], pw[4 * v + 3]));
-    const uint32_t mq = bmax2(bmax2(qw[4 * v], qw[4 * v + 1]), bmax2(qw[4 * v + 2], qw[4 * v + 3]));
-    const float vp = fmaxf(bf16_lo(mp), bf16_hi(mp)), vq = fmaxf(bf16_lo(mq), bf16_hi(mq));
-    amax_vec(A.av, A.ab, vp, idx0 + v * vstride);
-    amax_vec(A.qv, A.qb, vq, idx0 + v * vstride);
-    pm = fmaxf(pm, vp);
-    qm = fmaxf(qm, vq);
+  for (int v = 0; v < NV; ++v) {  // per-vector maxima of z_p and z_q, packed
+    vp[v] = bmax2(bmax2(pw[4 * v], pw[4 * v + 1]), bmax2(pw[4 * v + 2], pw[4 * v + 3]));
+    vq[v] = bmax2(bmax2(qw[4 * v], qw[4 * v + 1]), bmax2(qw[4 * v + 2], qw[4 * v + 3]));
   }
+  uint32_t cp = vp[0], cq = vq[0];
+#pragma unroll
+  for (int v = 1; v < NV; ++v) {
+    cp = bmax2(cp, vp[v]);
+    cq = bmax2(cq, vq[v]);
+  }
+  const float pm = fmaxf(bf16_lo(cp), bf16_hi(cp)), qm = fmaxf(bf16_lo(cq), bf16_hi(cq));
+  if (pm > A.av) first_vec_at<NV>(A.av, A.ab, vp, pm, idx0, vstride);
+  if (qm > A.qv) first_vec_at<NV>(A.qv, A.qb, vq, qm, idx0, vstride);
   if (KL) lse_kl_words<NW>(A.pM, A.pS, A.pD, pw, qw, pm, sT);
   else lse_words<NW>(A.pM, A.pS, pw, pm, sT);
   lse_words<NW>(A.qM, A.qS, qw, qm, sT);
@@ -461,7 +482,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) rowstats_stream(RowStats
       RowPart A;
       part_init(A);
       for (int c = 0; c < nch; ++c, pos.next()) {
-        if (wait_phase(&S.full[pos.slot], pos.phase, abort_flag, limit_ns, hdr)) {
+        if (wait_full(&S.full[pos.slot], pos.phase, abort_flag, limit_ns, hdr)) {
           const int e0 = c * CH;
           const uint4* P = reinterpret_cast<const uint4*>(ring + pos.slot * kSlotBytes);
           const uint4* Q = reinterpret_cast<const uint4*>(ring + pos.slot * kSlotBytes + kHalfSlot);
@@ -475,7 +496,10 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) rowstats_stream(RowStats
             phase1_bf16<kNV, NEED_Q1, KL>(A, pv, qv, e0 + t * E, kConsumers * E, sT);
           } else {
             const int nvec = min(CH, V - e0) / E;
-            for (int i = t; i < nvec; i += kConsumers) phase1_vec<T, NEED_Q1, KL>(A, P[i], Q[i], e0 + i * E, sT);
+            for (int i = t; i < nvec; i += kConsumers) {
+              if (sizeof(T) == 2) phase1_bf16<1, NEED_Q1, KL>(A, P + i, Q + i, e0 + i * E, 0, sT);
+              else phase1_vec<T, NEED_Q1, KL>(A, P[i], Q[i], e0 + i * E, sT);
+            }
           }
         }
         __syncwarp();
@@ -530,7 +554,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) rowstats_stream(RowStats
       const int iyh = tot.qb == 0x7fffffff ? 0 : (tot.qb - cyh * CH) / E;
       const int tyh = iyh % kConsumers;
       for (int c = 0; c < nch; ++c, pos.next()) {
-        if (wait_phase(&S.full[pos.slot], pos.phase, abort_flag, limit_ns, hdr)) {
+        if (wait_full(&S.full[pos.slot], pos.phase, abort_flag, limit_ns, hdr)) {
           const int e0 = c * CH;
           const uint4* P = reinterpret_cast<const uint4*>(ring + pos.slot * kSlotBytes);
           const uint4* Q = reinterpret_cast<const uint4*>(ring + pos.slot * kSlotBytes + kHalfSlot);
@@ -556,7 +580,10 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) rowstats_stream(RowStats
             }
           } else {
             const int nvec = min(CH, V - e0) / E;
-            for (int i = t; i < nvec; i += kConsumers) phase2_vec<T>(smin, sqlt, P[i], Q[i], a.sT, nCp, nCq);
+            for (int i = t; i < nvec; i += kConsumers) {
+              if (sizeof(T) == 2) phase2_bf16(smin2, sqlt2, P[i], Q[i], a.sT, nCp, nCq);
+              else phase2_vec<T>(smin, sqlt, P[i], Q[i], a.sT, nCp, nCq);
+            }
           }
         }
         __syncwarp();
