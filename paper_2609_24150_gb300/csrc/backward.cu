@@ -103,7 +103,7 @@ __device__ __forceinline__ float grad_elem(const RowCoef& c, float q, float p) {
 }
 
 template <typename T, bool VEC, bool GREEDY, bool SAMPLING, bool Q1_IS_QT, bool KL>
-__global__ void __launch_bounds__(kBwdThreads) backward_kernel(BackwardArgs a) {
+__device__ __forceinline__ void backward_rows(const BackwardArgs& a) {
   const int nvalid = a.ws.hdr->nvalid;
   const float scale = nvalid > 0 ? -a.dloss / (float)nvalid : 0.f;
   const int npos = KL ? a.ws.hdr->npos : 0;
@@ -191,16 +191,31 @@ __global__ void __launch_bounds__(kBwdThreads) backward_kernel(BackwardArgs a) {
 }
 
 template <typename T, bool VEC, bool G, bool S, bool Q, bool KL>
+__global__ void __launch_bounds__(kBwdThreads) backward_kernel(BackwardArgs a) {
+  backward_rows<T, VEC, G, S, Q, KL>(a);
+}
+// The anchor's bf16 vector instances (two exponentials an element) are held to 40
+// registers, six blocks an SM, for enough loads in flight (unbounded they took 48, five
+// blocks); the others fit six or more unbounded, and fp32 ones would spill at 40.
+template <typename T, bool G, bool S, bool Q>
+__global__ void __launch_bounds__(kBwdThreads, 6) backward_kernel_kl(BackwardArgs a) {
+  backward_rows<T, true, G, S, Q, true>(a);
+}
+
+template <typename T, bool VEC, bool G, bool S, bool Q, bool KL>
 cudaError_t go(const BackwardArgs& a, cudaStream_t s) {
   int dev = 0, sms = 0, per_sm = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, backward_kernel<T, VEC, G, S, Q, KL>, kBwdThreads, 0);
+  void (*kern)(BackwardArgs);
+  if constexpr (VEC && KL && sizeof(T) == 2) kern = backward_kernel_kl<T, G, S, Q>;
+  else kern = backward_kernel<T, VEC, G, S, Q, KL>;
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kBwdThreads, 0);
   if (per_sm < 1) per_sm = 1;
   int64_t grid = (int64_t)sms * per_sm;
   if (grid > a.R) grid = a.R;
   if (grid < 1) return cudaSuccess;
-  backward_kernel<T, VEC, G, S, Q, KL><<<(unsigned)grid, kBwdThreads, 0, s>>>(a);
+  kern<<<(unsigned)grid, kBwdThreads, 0, s>>>(a);
   return cudaGetLastError();
 }
 
