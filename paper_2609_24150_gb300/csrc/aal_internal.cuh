@@ -422,6 +422,13 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
+// log2(x) on the MUFU unit; denormal inputs flush to zero (callers pass normal values only).
+__device__ __forceinline__ float lg2(float x) {
+  float y;
+  asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
 

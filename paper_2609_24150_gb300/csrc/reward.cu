@@ -79,8 +79,9 @@ __device__ __forceinline__ void draw_push(Draw& d, float key, int64_t v, float z
     d.zp = zp;
   }
 }
-// The Gumbel noise in log2 units: G log2(e) = -log2(-ln U) = -log2(-ln2 * log2 U).
-__device__ __forceinline__ float gumbel2(float U) { return -__log2f(-kLn2 * __log2f(U)); }
+// The Gumbel noise in log2 units: G log2(e) = -log2(-ln U) = -log2(-ln2 * log2 U).  Both
+// logarithms see normal numbers only: U >= 2^-24, and -ln2 * log2 U >= 5.9e-8 (U <= 1 - 2^-24).
+__device__ __forceinline__ float gumbel2(float U) { return -lg2(-kLn2 * lg2(U)); }
 
 __device__ __forceinline__ RowState merge_state(const RowState& a, const RowState& b, float sT) {
   RowState o;
@@ -310,9 +311,10 @@ __device__ __forceinline__ void lse_fold(Lse& L, const float* z, float s) {
   L.M = m;
 }
 
-// Offer E Gumbel keys of one vector (elements v0 ..) to a running draw.
-template <int E>
-__device__ __forceinline__ void draw_fold(Draw& d, const float* key, const float* z, const float* zp, int64_t v0) {
+// Offer E Gumbel keys of one vector (elements v0 ..) to a running draw; the target's vector
+// (pw, packed) is unpacked only when the vector wins.
+template <typename T, int E>
+__device__ __forceinline__ void draw_fold(Draw& d, const float* key, const float* z, const uint4& pw, int64_t v0) {
   float km = key[0];
 #pragma unroll
   for (int e = 1; e < E; ++e) km = fmaxf(km, key[e]);
@@ -321,6 +323,8 @@ __device__ __forceinline__ void draw_fold(Draw& d, const float* key, const float
 #pragma unroll
     for (int e = E - 1; e >= 0; --e)
       if (key[e] == km) at = e;
+    float zp[E];
+    unpack_any<T>(pw, zp);
     float zz = z[0], pp = zp[0];
 #pragma unroll
     for (int e = 1; e < E; ++e)
@@ -381,7 +385,7 @@ __global__ void __launch_bounds__(kRowThreads, REF ? 4 : 5) reward_sampled_rows(
       uint4 rw = make_uint4(0, 0, 0, 0);
       if (REF) rw = ldg_stream(r4 + i);
       unpack_any<T>(qw, qv);
-      unpack_any<T>(pw, pv);
+      if (sizeof(T) != 2) unpack_any<T>(pw, pv);  // (the bf16 path folds z_p packed)
       if (REF) unpack_any<T>(rw, rv);
 #pragma unroll
       for (int h = 0; h < E / 4; ++h) {
@@ -396,8 +400,8 @@ __global__ void __launch_bounds__(kRowThreads, REF ? 4 : 5) reward_sampled_rows(
         kq[e] = fmaf(qv[e], a.sT, g[e]);
         if (REF) kr[e] = fmaf(rv[e], a.sT, g[e]);
       }
-      draw_fold<E>(dq, kq, qv, pv, i * E);
-      if (REF) draw_fold<E>(dr, kr, rv, pv, i * E);
+      draw_fold<T, E>(dq, kq, qv, pw, i * E);
+      if (REF) draw_fold<T, E>(dr, kr, rv, pw, i * E);
       if (sizeof(T) == 2) {
         lse_fold_bf16(st.lp, pw, a.sT);
         lse_fold_bf16(st.lq, qw, a.sT);
