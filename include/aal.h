@@ -145,6 +145,24 @@ AAL_API aal_status aal_loss_bwd(const aal_problem* prob, const void* draft, cons
                         const uint8_t* mask, const void* workspace, size_t workspace_bytes,
                         float dloss, void* grad_draft, void* stream);
 
+/* Forward and backward in one call: the loss, eal and workspace of aal_loss_fwd and the
+ * gradient of aal_loss_bwd with the same dloss, bit for bit (same arguments, layouts and
+ * rules as those two calls; dloss must be known before the forward, as it is for a loss
+ * that is a fixed weight times the objective).  The result equals the two calls; the
+ * difference is the traffic.  With bf16 rows whose byte length is a multiple of 16, the
+ * K rows of each window are streamed by K CTAs together (one cooperative launch, one CTA
+ * per SM), and the gradient is written while the rows are still in L2: the logits are read
+ * from HBM once (2 V b per row, plus V b gradient written) instead of twice (the separate
+ * forward's 2 V b and the backward's 3 V b).  Other problems (fp32, unaligned rows, token
+ * ids, the anchor beside a sampling term at T != 1) run the two calls inside this one.
+ * AAL_GRPO is rejected with AAL_ERR_UNSUPPORTED: its coefficients come from
+ * aal_grpo_from_loss, between the forward and the backward.  A bounded device wait that ran
+ * out (a ring copy, or the group barrier between the K CTAs of a window) is reported by
+ * aal_check_device_status as AAL_ERR_TIMEOUT, and then no output may be used. */
+AAL_API aal_status aal_loss_fwd_bwd(const aal_problem* prob, const void* draft, const void* target,
+                                    const uint8_t* mask, void* workspace, size_t workspace_bytes,
+                                    float dloss, float* loss, float* eal, void* grad_draft, void* stream);
+
 /* Sequence layout (Sec. 3.3): the draft and the target run once over whole sequences, and a
  * window of gamma = K positions starts at every position and slides by one, so each position
  * is depth j of up to K windows.  Logits are stored once per position, not once per window.

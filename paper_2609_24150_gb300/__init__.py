@@ -46,6 +46,7 @@ from .aal import (  # noqa: F401
     aal_seq_grpo_workspace_size,
     aal_loss_bwd,
     aal_loss_fwd,
+    aal_loss_fwd_bwd,
     aal_reward_workspace_size,
     aal_seq_loss_bwd,
     aal_seq_loss_fwd,

@@ -99,6 +99,7 @@ def library() -> ctypes.CDLL:
     lib.aal_reward_workspace_size.argtypes = [RP, ctypes.POINTER(sz)]
     lib.aal_loss_fwd.argtypes = [P, vp, vp, vp, vp, sz, vp, vp, vp]
     lib.aal_loss_bwd.argtypes = [P, vp, vp, vp, vp, sz, ctypes.c_float, vp, vp]
+    lib.aal_loss_fwd_bwd.argtypes = [P, vp, vp, vp, vp, sz, ctypes.c_float, vp, vp, vp, vp]
     lib.aal_accept_reward.argtypes = [RP, vp, vp, vp, vp, sz, vp, vp, vp, vp, vp]
     lib.aal_accept_reward_noalloc.argtypes = [RP, vp, vp, vp, vp, vp, vp, vp, vp]
     lib.aal_accept_reward_from_loss.argtypes = [RP, P, vp, sz, vp, sz, vp, vp, vp, vp]
@@ -118,7 +119,7 @@ def library() -> ctypes.CDLL:
     lib.aal_status_string.restype = ctypes.c_char_p
     lib.aal_abi_version.argtypes = []
     lib.aal_abi_version.restype = ctypes.c_int32
-    for f in ("aal_workspace_size", "aal_reward_workspace_size", "aal_loss_fwd", "aal_loss_bwd",
+    for f in ("aal_workspace_size", "aal_reward_workspace_size", "aal_loss_fwd", "aal_loss_bwd", "aal_loss_fwd_bwd",
               "aal_accept_reward", "aal_accept_reward_noalloc", "aal_accept_reward_from_loss",
               "aal_seq_workspace_size", "aal_seq_loss_fwd", "aal_seq_loss_bwd", "aal_check_device_status",
               "aal_grpo_workspace_size", "aal_grpo_from_loss", "aal_seq_grpo_workspace_size",
@@ -246,6 +247,19 @@ def aal_loss_bwd(problem: AalProblem, draft, target, mask, workspace, dloss: flo
         _ptr(mask, "mask", torch.uint8), _ptr(workspace, "workspace"), _nbytes(workspace),
         float(dloss), _ptr(grad, "grad"), _stream(stream))
     _check(code, "aal_loss_bwd")
+
+
+def aal_loss_fwd_bwd(problem: AalProblem, draft, target, mask, workspace, dloss: float, loss, grad, eal=None,
+                     stream=None):
+    """Forward and backward in one call: loss[0] (and eal[N][2]) as aal_loss_fwd, grad as
+    aal_loss_bwd with the same dloss; the logits are read from HBM once."""
+    N = problem.N
+    code = library().aal_loss_fwd_bwd(
+        ctypes.byref(problem), _ptr(draft, "draft"), _ptr(target, "target"),
+        _ptr(mask, "mask", torch.uint8, N * problem.K), _ptr(workspace, "workspace"),
+        _nbytes(workspace), float(dloss), _ptr(loss, "loss", torch.float32, 1),
+        _ptr(eal, "eal", torch.float32, 2 * N), _ptr(grad, "grad"), _stream(stream))
+    _check(code, "aal_loss_fwd_bwd")
 
 
 def grpo_problem(draft: torch.Tensor, windows_per_rollout: int = 1, rollouts_per_group: int = 1,

@@ -89,6 +89,29 @@ aal_status check_grpo(const aal_grpo_problem* p) {
 
 aal_status cuda_status(cudaError_t e) { return e == cudaSuccess ? AAL_OK : AAL_ERR_CUDA; }
 
+// The statistics pass over z_p and z_q for the mode's terms (takes the test hook's chunk).
+RowStatsArgs stats_args(const void* draft, const void* target, int64_t R, int64_t V, int32_t mode,
+                        float temperature, const LossWs& ws) {
+  const bool greedy = (mode & AAL_GREEDY) != 0;
+  const bool sampling = (mode & (AAL_SAMPLING | AAL_TV)) != 0;  // both need a^sample
+  const bool kl = (mode & AAL_KL) != 0;
+  const bool grpo = (mode & AAL_GRPO) != 0;  // log pi_theta(y) needs the T = 1 normaliser
+  RowStatsArgs ra;
+  ra.zq = draft;
+  ra.zp = target;
+  ra.R = R;
+  ra.V = V;
+  ra.sT = sampling ? kLog2e / temperature : 0.f;
+  ra.need_p = sampling;
+  ra.need_q = sampling;
+  ra.need_q1 = (greedy || kl || grpo) && !(sampling && temperature == 1.0f);
+  ra.overlap = sampling;
+  ra.need_kl = kl;
+  ra.skip_chunk = debug_take_skip_chunk();
+  ra.ws = ws;
+  return ra;
+}
+
 // Per-row statistics of R logit rows (pass over z_p and z_q, or over z_q alone when `target`
 // holds token ids), shared by both layouts.
 cudaError_t launch_stats(const void* draft, const void* target, int64_t R, int64_t V, int32_t dtype,
@@ -108,31 +131,14 @@ cudaError_t launch_stats(const void* draft, const void* target, int64_t R, int64
     *cluster = 1;
     return launch_one_tensor(a, dtype == AAL_BF16, true, s);
   }
-  const bool greedy = (mode & AAL_GREEDY) != 0;
-  const bool sampling = (mode & (AAL_SAMPLING | AAL_TV)) != 0;  // both need a^sample
-  const bool kl = (mode & AAL_KL) != 0;
-  const bool grpo = (mode & AAL_GRPO) != 0;  // log pi_theta(y) needs the T = 1 normaliser
-  RowStatsArgs ra;
-  ra.zq = draft;
-  ra.zp = target;
-  ra.R = R;
-  ra.V = V;
-  ra.sT = sampling ? kLog2e / temperature : 0.f;
-  ra.need_p = sampling;
-  ra.need_q = sampling;
-  ra.need_q1 = (greedy || kl || grpo) && !(sampling && temperature == 1.0f);
-  ra.overlap = sampling;
-  ra.need_kl = kl;
-  ra.skip_chunk = debug_take_skip_chunk();
-  ra.ws = ws;
   *cluster = 1;
-  return launch_rowstats(ra, dtype == AAL_BF16, s, cluster);
+  return launch_rowstats(stats_args(draft, target, R, V, mode, temperature, ws), dtype == AAL_BF16, s, cluster);
 }
 
-// Gradient rows from the statistics and dE/da in the workspace, shared by both layouts.
-cudaError_t launch_grad(const void* draft, const void* target, const uint8_t* mask, int64_t R, int64_t V,
-                        int32_t dtype, int32_t mode, float temperature, float w_greedy, float w_sampling,
-                        float w_kl, float dloss, const LossWs& ws, void* grad, cudaStream_t s) {
+// The gradient pass for the mode's terms.
+BackwardArgs grad_args(const void* draft, const void* target, const uint8_t* mask, int64_t R, int64_t V,
+                       int32_t mode, float temperature, float w_greedy, float w_kl, float dloss, const LossWs& ws,
+                       void* grad) {
   const bool greedy = (mode & AAL_GREEDY) != 0;
   const bool sampling = (mode & (AAL_SAMPLING | AAL_TV)) != 0;
   const bool kl = (mode & AAL_KL) != 0;
@@ -154,7 +160,39 @@ cudaError_t launch_grad(const void* draft, const void* target, const uint8_t* ma
   ba.mask = mask;
   ba.q1_is_qT = (greedy || kl || grpo) && sampling && temperature == 1.0f;
   ba.ws = ws;
-  return launch_backward(ba, dtype == AAL_BF16, s);
+  return ba;
+}
+
+// Gradient rows from the statistics and dE/da in the workspace, shared by both layouts.
+cudaError_t launch_grad(const void* draft, const void* target, const uint8_t* mask, int64_t R, int64_t V,
+                        int32_t dtype, int32_t mode, float temperature, float w_greedy, float w_sampling,
+                        float w_kl, float dloss, const LossWs& ws, void* grad, cudaStream_t s) {
+  (void)w_sampling;  // folded into dE^s/da by the window kernels
+  return launch_backward(grad_args(draft, target, mask, R, V, mode, temperature, w_greedy, w_kl, dloss, ws, grad),
+                         dtype == AAL_BF16, s);
+}
+
+// The window terms of an [N][K] problem.
+WindowArgs window_args(const aal_problem* prob, const uint8_t* mask, int cluster, float* loss, float* eal,
+                       const LossWs& ws, int64_t nwblk) {
+  WindowArgs wa;
+  wa.mask = mask;
+  wa.N = prob->N;
+  wa.K = (int32_t)prob->K;
+  wa.cluster = cluster;
+  wa.greedy = (prob->mode & AAL_GREEDY) != 0;
+  wa.sampling = (prob->mode & AAL_SAMPLING) != 0;
+  wa.kl = (prob->mode & AAL_KL) != 0;
+  wa.tv = (prob->mode & AAL_TV) != 0;
+  wa.w_greedy = prob->w_greedy;
+  wa.w_sampling = prob->w_sampling;
+  wa.w_kl = prob->w_kl;
+  wa.w_tv = prob->w_tv;
+  wa.loss = loss;
+  wa.eal = eal;
+  wa.ws = ws;
+  wa.nwblk = nwblk;
+  return wa;
 }
 
 }  // namespace
@@ -166,7 +204,7 @@ int64_t debug_take_skip_chunk() { return g_skip_chunk.exchange(-1); }
 
 extern "C" {
 
-int32_t aal_abi_version(void) { return 10400; }
+int32_t aal_abi_version(void) { return 10500; }
 
 void aal_debug_fail_next_forward(int64_t chunk, uint64_t wait_limit_ns) {
   g_wait_limit_ns.store(wait_limit_ns);
@@ -214,7 +252,6 @@ aal_status aal_loss_fwd(const aal_problem* prob, const void* draft, const void* 
   const LossLayout L = loss_layout(prob->N, prob->K);
   if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < L.total) return AAL_ERR_WORKSPACE;
 
-  const bool greedy = (prob->mode & AAL_GREEDY) != 0, sampling = (prob->mode & AAL_SAMPLING) != 0;
   LossWs ws = loss_ws(workspace, L);
   cudaError_t e = cudaMemsetAsync(ws.hdr, 0, sizeof(WsHeader), s);
   if (e != cudaSuccess) return AAL_ERR_CUDA;
@@ -225,25 +262,7 @@ aal_status aal_loss_fwd(const aal_problem* prob, const void* draft, const void* 
   int cluster = 1;
   e = launch_stats(draft, target, L.R, prob->V, prob->dtype, prob->mode, prob->temperature, ws, s, &cluster);
   if (e != cudaSuccess) return AAL_ERR_CUDA;
-
-  WindowArgs wa;
-  wa.mask = mask;
-  wa.N = prob->N;
-  wa.K = (int32_t)prob->K;
-  wa.cluster = cluster;
-  wa.greedy = greedy;
-  wa.sampling = sampling;
-  wa.kl = (prob->mode & AAL_KL) != 0;
-  wa.tv = (prob->mode & AAL_TV) != 0;
-  wa.w_greedy = prob->w_greedy;
-  wa.w_sampling = prob->w_sampling;
-  wa.w_kl = prob->w_kl;
-  wa.w_tv = prob->w_tv;
-  wa.loss = loss;
-  wa.eal = eal;
-  wa.ws = ws;
-  wa.nwblk = L.nwblk;
-  return cuda_status(launch_window(wa, s));
+  return cuda_status(launch_window(window_args(prob, mask, cluster, loss, eal, ws, L.nwblk), s));
 }
 
 aal_status aal_loss_bwd(const aal_problem* prob, const void* draft, const void* target,
@@ -264,6 +283,49 @@ aal_status aal_loss_bwd(const aal_problem* prob, const void* draft, const void* 
                                  prob->temperature, prob->w_greedy, prob->w_sampling, prob->w_kl, dloss,
                                  loss_ws(const_cast<void*>(workspace), L), grad_draft,
                                  static_cast<cudaStream_t>(stream)));
+}
+
+aal_status aal_loss_fwd_bwd(const aal_problem* prob, const void* draft, const void* target,
+                            const uint8_t* mask, void* workspace, size_t workspace_bytes, float dloss,
+                            float* loss, float* eal, void* grad_draft, void* stream) {
+  aal_status st = check_problem(prob);
+  if (st != AAL_OK) return st;
+  if (prob->mode & AAL_GRPO) return AAL_ERR_UNSUPPORTED;  // its coefficients come between the two
+  if (!isfinite(dloss)) return AAL_ERR_INVALID_ARG;
+  if (loss == nullptr || !aligned(loss, 4) || (eal != nullptr && !aligned(eal, 4))) return AAL_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (prob->N == 0) return cuda_status(cudaMemsetAsync(loss, 0, sizeof(float), s));
+  if (draft == nullptr || target == nullptr || grad_draft == nullptr || !aligned(draft, 16) ||
+      !aligned(target, target_align(prob->mode)) || !aligned(grad_draft, 16))
+    return AAL_ERR_INVALID_ARG;
+  const LossLayout L = loss_layout(prob->N, prob->K);
+  if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < L.total) return AAL_ERR_WORKSPACE;
+
+  // the fused kernel: bf16 rows of 16-byte multiples, both logit tensors, and (as for the
+  // streamed forward) the anchor beside a sampling term only at T = 1
+  const bool sampling = (prob->mode & (AAL_SAMPLING | AAL_TV)) != 0, kl = (prob->mode & AAL_KL) != 0;
+  const bool fusable = prob->dtype == AAL_BF16 && !(prob->mode & AAL_IDS) && (prob->V * 2) % 16 == 0 &&
+                       !(kl && sampling && prob->temperature != 1.0f);
+  if (fusable) {
+    LossWs ws = loss_ws(workspace, L);
+    if (cudaMemsetAsync(ws.hdr, 0, sizeof(WsHeader), s) != cudaSuccess) return AAL_ERR_CUDA;
+    if (cudaMemsetAsync(ws.gcnt, 0, (size_t)kMaxGroups * 4, s) != cudaSuccess) return AAL_ERR_CUDA;
+    if (launch_count_valid(mask, prob->N, (int32_t)prob->K, ws.hdr, s) != cudaSuccess) return AAL_ERR_CUDA;
+    FusedArgs f;
+    f.st = stats_args(draft, target, L.R, prob->V, prob->mode, prob->temperature, ws);
+    f.bw = grad_args(draft, target, mask, L.R, prob->V, prob->mode, prob->temperature, prob->w_greedy,
+                     prob->w_kl, dloss, ws, grad_draft);
+    f.win = window_args(prob, mask, 1, loss, eal, ws, L.nwblk);
+    f.groups = 0;
+    const uint64_t limit = debug_wait_limit_ns();
+    bool launched = false;
+    if (launch_fused(f, s, limit ? limit : kWaitLimitNs, &launched) != cudaSuccess) return AAL_ERR_CUDA;
+    // the loss from the statistics the fused kernel wrote, as aal_loss_fwd forms it
+    if (launched) return cuda_status(launch_window(f.win, s));
+  }
+  st = aal_loss_fwd(prob, draft, target, mask, workspace, workspace_bytes, loss, eal, stream);
+  if (st != AAL_OK) return st;
+  return aal_loss_bwd(prob, draft, target, mask, workspace, workspace_bytes, dloss, grad_draft, stream);
 }
 
 aal_status aal_seq_workspace_size(const aal_seq_problem* prob, size_t* bytes) {

@@ -13,6 +13,7 @@ namespace aal {
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr int kMaxCluster = 8;          // CTAs that may share one logit row
+constexpr int kMaxGroups = 1024;        // fused forward + backward: groups of K CTAs per launch
 constexpr uint32_t kStatusTimeout = 5;  // == AAL_ERR_TIMEOUT
 
 // ---------------------------------------------------------------------------
@@ -47,6 +48,7 @@ struct LossLayout {
   size_t zpy = 0;                   // float[R] z_p at the draft argmax
   size_t cpart = 0;                 // float2[R][kMaxCluster] per-CTA (overlap, Qlt) partials
   size_t wpart = 0;                 // double[nwblk][kWpart] window-kernel block partials
+  size_t gcnt = 0;                  // uint32[kMaxGroups] fused forward + backward: group arrivals
   size_t total = 0;
 };
 
@@ -88,6 +90,7 @@ inline LossLayout loss_layout(int64_t N, int64_t K) {
   L.zpy = take(R * 4);
   L.cpart = take(R * kMaxCluster * 8);
   L.wpart = take((size_t)(L.nwblk > 0 ? L.nwblk : 1) * kWpart * 8);
+  L.gcnt = take((size_t)kMaxGroups * 4);
   L.total = off;
   return L;
 }
@@ -147,6 +150,7 @@ struct LossWs {
   float* zpy;
   float2* cpart;
   double* wpart;
+  uint32_t* gcnt;
 };
 
 inline LossWs loss_ws(void* base, const LossLayout& L) {
@@ -173,6 +177,7 @@ inline LossWs loss_ws(void* base, const LossLayout& L) {
   w.zpy = reinterpret_cast<float*>(b + L.zpy);
   w.cpart = reinterpret_cast<float2*>(b + L.cpart);
   w.wpart = reinterpret_cast<double*>(b + L.wpart);
+  w.gcnt = reinterpret_cast<uint32_t*>(b + L.gcnt);
   return w;
 }
 
@@ -236,6 +241,15 @@ struct BackwardArgs {
   const uint8_t* mask;         // [R] position validity (the anchor's rows), or null
   bool q1_is_qT;               // T == 1, sampling and a T = 1 term: q = q~, one exponential
   LossWs ws;
+};
+
+// The fused forward + backward of [N][K][V] windows (aal_loss_fwd_bwd): groups of K CTAs,
+// CTA k of group g taking depth k of windows g, g + G, ...
+struct FusedArgs {
+  RowStatsArgs st;   // the statistics passes (zq, zp, R, V, sT, flags, test hook, workspace)
+  BackwardArgs bw;   // the gradient pass (grad, dloss, weights, position mask, invT)
+  WindowArgs win;    // the window terms (mask [N][K], N, K, which terms, w_sampling, w_tv)
+  int32_t groups;    // G
 };
 
 struct RewardRowArgs {
@@ -409,6 +423,10 @@ cudaError_t launch_one_tensor(const Stream1Args& a, bool bf16, bool ids, cudaStr
 cudaError_t launch_grpo_windows(const GrpoWindowArgs& a, cudaStream_t s);
 cudaError_t launch_seq_grpo_gather(const SeqGrpoArgs& a, cudaStream_t s);
 cudaError_t launch_seq_grpo_scatter(const SeqGrpoArgs& a, cudaStream_t s);
+cudaError_t launch_count_valid(const uint8_t* mask, int64_t N, int32_t K, WsHeader* hdr, cudaStream_t s);
+// Launches the fused forward + backward when the problem's flags have an instantiation and the
+// device can hold at least one group; *launched tells whether it did.
+cudaError_t launch_fused(const FusedArgs& f, cudaStream_t s, uint64_t limit_ns, bool* launched);
 
 // ---------------------------------------------------------------------------
 // Device helpers.
@@ -427,6 +445,34 @@ __device__ __forceinline__ float lg2(float x) {
   float y;
   asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+
+// Expected length of one window term and its partials (Sec. 3.1, Eq. eal_generic): with
+// P_k = prod_{j<k} a_j, E = sum_{k=1}^{kn} P_k and dE/da_j = P_j S_j, S_{kn-1} = 1,
+// S_j = 1 + a_{j+1} S_{j+1} (0 for j >= kn).  Shared by the window kernels and the fused
+// forward + backward, so both give bitwise the same partials.
+__device__ __forceinline__ float window_term(const float* a, int kn, float* dE) {
+  float P[AAL_MAX_K + 1];
+  P[0] = 1.f;
+  float E = 0.f;
+#pragma unroll
+  for (int j = 0; j < AAL_MAX_K; ++j) {
+    if (j < kn) {
+      P[j + 1] = P[j] * a[j];
+      E += P[j + 1];
+    }
+  }
+  float S = 1.f;
+#pragma unroll
+  for (int j = AAL_MAX_K - 1; j >= 0; --j) {
+    if (j < kn) {
+      dE[j] = P[j] * S;
+      S = 1.f + a[j] * S;
+    } else {
+      dE[j] = 0.f;
+    }
+  }
+  return E;
 }
 
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }

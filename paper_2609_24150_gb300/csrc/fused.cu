@@ -1,0 +1,484 @@
+// Forward and backward of the window losses in one call (aal_loss_fwd_bwd), GB300 path.
+//
+// The separate calls stream every row three times: twice in the forward (statistics from
+// HBM, overlap sums from L2) and once more from HBM in the backward, which must wait for the
+// window terms of all K depths.  Here the K rows of a window are held by K CTAs at the same
+// time (a group), so that the gradient pass can follow the statistics while the rows are
+// still in L2: per row, pass 1 from HBM, pass 2 (sampling term only) from L2, a group barrier
+// that gives every CTA its window's acceptances, and pass 3 from L2 writing the gradient.
+// The logits cross HBM once per step instead of twice.
+//
+// * Launch: cooperative, one CTA per SM (the ring takes ~193 KB of shared memory), grid =
+//   G groups x K CTAs; CTA k of group g takes depth k of windows g, g + G, ...  A cooperative
+//   launch has all its CTAs resident at once, so a group never waits on a CTA that is not
+//   running.
+// * Group barrier: once its row's statistics are in the workspace, thread 0 of each CTA adds
+//   one to the group's counter (release) and waits (acquire, bounded like the ring waits) for
+//   K arrivals per window.  It then reads the window's a^greedy, a^sample and mask, forms
+//   dE^g/da and dE^s/da with the window kernels' function (window_term) and the row's gradient
+//   coefficients with the backward's (row_coef), so that the gradient equals the one of
+//   aal_loss_fwd + aal_loss_bwd bit for bit.  The loss is left to the window kernel, which runs
+//   after this one over the statistics written here, exactly as in aal_loss_fwd.
+// * The counts of valid windows and positions that scale the gradient are taken from the mask
+//   by count_valid before the launch (the separate forward gets them from its window kernel).
+// * Failure: every wait is bounded.  A CTA that gave up keeps walking its rows without waiting
+//   and still adds its arrivals, so its group does not wait on it for the whole limit; the
+//   workspace status word reports AAL_ERR_TIMEOUT and the outputs are not to be used.
+#include "grad_elem.cuh"
+#include "stream_core.cuh"
+
+namespace aal {
+namespace {
+
+constexpr int kBarCoef = 3;  // named barrier: the row's gradient coefficients are in shared memory
+
+struct FusedSmem {
+  Smem s;
+  RowCoef coef;
+  int32_t live;  // the row's gradient has a nonzero term
+};
+
+constexpr size_t kFusedSmemBytes = (size_t)kSlots * kSlotBytes + sizeof(FusedSmem);
+
+// PASSES = 2 with the sampling (or TV) term, 1 without; NEED_Q1, KL as in rowstats_stream;
+// GREEDY and Q1_IS_QT as in the backward.  bf16 rows only (16-byte multiples).
+template <bool NEED_Q1, int PASSES, bool KL, bool GREEDY, bool Q1_IS_QT>
+__global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, uint64_t limit_ns) {
+  using T = uint16_t;
+  constexpr bool SAMPLING = PASSES == 2;
+  constexpr int E = 8;                // bf16 elements per 16-byte vector
+  constexpr int CH = kHalfSlot / 2;   // elements per chunk per tensor
+  extern __shared__ __align__(1024) unsigned char smem[];
+  unsigned char* ring = smem;
+  FusedSmem& F = *reinterpret_cast<FusedSmem*>(smem + kSlots * kSlotBytes);
+  Smem& S = F.s;
+  const RowStatsArgs& a = f.st;
+  volatile int* abort_flag = &S.abort_flag;
+  WsHeader* hdr = a.ws.hdr;
+  const int V = (int)a.V;
+  const int nfull = V / CH;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int K = f.win.K;
+  const int64_t N = f.win.N;
+  const int G = f.groups;
+  const int g = blockIdx.x / K, k = blockIdx.x % K;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kSlots; ++s) {
+      mbar_init(&S.full[s], 1);
+      mbar_init(&S.empty[s], kWarps);
+    }
+    S.abort_flag = 0;
+    S.arg_index = 0x7fffffff;
+    S.arg_carry = 0.f;
+    S.yarg_index = 0x7fffffff;
+    S.yarg_carry = 0.f;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+
+  if (warp == kWarps) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      const uint64_t keep = policy_evict_last(), drop = policy_evict_first();
+      RingPos pos;
+      int64_t seq = 0;
+      uint32_t armed = 0, last_phase = 0;
+      for (int64_t n = g; n < N && !*abort_flag; n += G) {
+        const int64_t r = n * K + k;
+        const char* prow = static_cast<const char*>(a.zp) + r * a.V * 2;
+        const char* qrow = static_cast<const char*>(a.zq) + r * a.V * 2;
+        // statistics passes keep the row in L2; the gradient pass is its last use
+        for (int pass = 0; pass < PASSES + 1 && !*abort_flag; ++pass) {
+          const uint64_t pol = pass < PASSES ? keep : drop;
+          for (int c = 0; c < nch; ++c) {
+            if (!wait_phase(&S.empty[pos.slot], pos.phase ^ 1u, abort_flag, limit_ns, hdr)) break;
+            const int e0 = c * CH;
+            const uint32_t bytes = (uint32_t)(min(CH, V - e0) * 2);
+            if (seq != a.skip_chunk) {  // (the test hook leaves one chunk's barrier unarmed)
+              mbar_expect_tx(&S.full[pos.slot], 2u * bytes);
+              bulk_load(ring + pos.slot * kSlotBytes, prow + (int64_t)e0 * 2, bytes, &S.full[pos.slot], pol);
+              bulk_load(ring + pos.slot * kSlotBytes + kHalfSlot, qrow + (int64_t)e0 * 2, bytes, &S.full[pos.slot],
+                        pol);
+              armed |= 1u << pos.slot;
+              last_phase = (last_phase & ~(1u << pos.slot)) | (pos.phase << pos.slot);
+            }
+            pos.next();
+            ++seq;
+          }
+        }
+      }
+      for (int s = 0; s < kSlots; ++s) {
+        if (!(armed & (1u << s))) continue;
+        const uint32_t ph = (last_phase >> s) & 1u;
+        const uint64_t t0 = now_ns();
+        for (uint32_t it = 0; it < kSpinLimit && !mbar_try(&S.full[s], ph, 100000); ++it)
+          if (now_ns() - t0 > limit_ns) break;
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ consumers
+    const int t = threadIdx.x;
+    RingPos pos;
+    uint32_t j = 0;
+    const float sT = PASSES == 2 ? a.sT : kLog2e;
+    // the backward's scales (thread 0 forms the coefficients)
+    float scale = 0.f, kscale = 0.f;
+    if (t == 0) {
+      const int nvalid = hdr->nvalid;
+      scale = nvalid > 0 ? -f.bw.dloss / (float)nvalid : 0.f;
+      const int npos = KL ? hdr->npos : 0;
+      kscale = npos > 0 ? f.bw.dloss * f.bw.w_kl / (float)npos : 0.f;
+    }
+    for (int64_t n = g; n < N; n += G, ++j) {
+      const int64_t r = n * K + k;
+      // ---- pass 1: online normalisers and argmax (HBM)
+      RowPart A;
+      part_init(A);
+      for (int c = 0; c < nch; ++c, pos.next()) {
+        if (wait_full(&S.full[pos.slot], pos.phase, abort_flag, limit_ns, hdr)) {
+          const int e0 = c * CH;
+          const uint4* P = reinterpret_cast<const uint4*>(ring + pos.slot * kSlotBytes);
+          const uint4* Q = reinterpret_cast<const uint4*>(ring + pos.slot * kSlotBytes + kHalfSlot);
+          if (c < nfull) {
+            uint4 pv[kNV], qv[kNV];
+#pragma unroll
+            for (int v = 0; v < kNV; ++v) {
+              pv[v] = P[t + v * kConsumers];
+              qv[v] = Q[t + v * kConsumers];
+            }
+            phase1_bf16<kNV, NEED_Q1, KL>(A, pv, qv, e0 + t * E, kConsumers * E, sT);
+          } else {
+            const int nvec = (V - e0) / E;
+            for (int i = t; i < nvec; i += kConsumers) phase1_bf16<1, NEED_Q1, KL>(A, P + i, Q + i, e0 + i * E, 0, sT);
+          }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&S.empty[pos.slot]);
+      }
+      warp_part<NEED_Q1, KL>(A, sT);
+      if (lane == 0) S.red[j & 1][warp] = A;
+      named_barrier(kBarRow, kConsumers);
+      RowPart tot;
+      if (lane < kWarps) tot = S.red[j & 1][lane];
+      else part_init(tot);
+      warp_part<NEED_Q1, KL>(tot, sT);
+      const float Mp = tot.pM, Lsp = log2f(tot.pS);
+      const float Mq = tot.qM, Lsq = log2f(tot.qS);
+      RowStat st{};  // thread 0: what the row's coefficients need
+      if (KL && t == 0) {  // both normalisers are at T = 1 here
+        const float Mq1 = NEED_Q1 ? tot.q1M : Mq;
+        const float Lsq1 = NEED_Q1 ? log2f(tot.q1S) : Lsq;
+        if (!*abort_flag) {
+          a.ws.Mp1[r] = Mp;
+          a.ws.Lsp1[r] = Lsp;
+          a.ws.kl[r] = tot.pD / tot.pS - (Mp - Mq1) - kLn2 * (Lsp - Lsq1);
+        }
+        st.Mp1 = Mp;
+        st.Lsp1 = Lsp;
+      }
+      if (PASSES == 1) {
+        if (t == 0) {
+          // x* and y to the element: their vectors are read again, from L2
+          const T* zp = static_cast<const T*>(a.zp) + r * a.V;
+          const T* zq = static_cast<const T*>(a.zq) + r * a.V;
+          const bool ok = !*abort_flag;
+          int32_t xs, ys;
+          float cx, cy;
+          resolve_vectors<T>(zp, zq, a.V, ok ? tot.ab : -1, ok ? tot.qb : -1, &xs, &cx, &ys, &cy);
+          const float ag = exp2f(log2_prob(cx, kLog2e, Mq, Lsq));
+          if (ok) {
+            a.ws.Mp[r] = Mp;
+            a.ws.Lsp[r] = Lsp;
+            a.ws.Mq[r] = Mq;
+            a.ws.Lsq[r] = Lsq;
+            a.ws.Mq1[r] = Mq;
+            a.ws.Lsq1[r] = Lsq;
+            a.ws.cpart[r * kMaxCluster] = make_float2(0.f, 0.f);
+            a.ws.xstar[r] = xs;
+            a.ws.yhat[r] = ys;
+            a.ws.zpy[r] = cy;
+            a.ws.ag[r] = ag;
+          }
+          st.Mq1 = Mq;
+          st.Lsq1 = Lsq;
+          st.ag = ag;
+          st.xs = xs;
+          st.ys = ys;
+        }
+      } else {
+        // ---- pass 2: overlap sums (L2)
+        float smin = 0.f, sqlt = 0.f;
+        float2 smin2 = make_float2(0.f, 0.f), sqlt2 = make_float2(0.f, 0.f);
+        const float nCp = -(Mp + Lsp / a.sT), nCq = -(Mq + Lsq / a.sT);
+        const int cstar = tot.ab == 0x7fffffff ? -1 : tot.ab / CH;
+        const int istar = tot.ab == 0x7fffffff ? 0 : (tot.ab - cstar * CH) / E;
+        const int tstar = istar % kConsumers;
+        const int cyh = tot.qb == 0x7fffffff ? -1 : tot.qb / CH;
+        const int iyh = tot.qb == 0x7fffffff ? 0 : (tot.qb - cyh * CH) / E;
+        const int tyh = iyh % kConsumers;
+        for (int c = 0; c < nch; ++c, pos.next()) {
+          if (wait_full(&S.full[pos.slot], pos.phase, abort_flag, limit_ns, hdr)) {
+            const int e0 = c * CH;
+            const uint4* P = reinterpret_cast<const uint4*>(ring + pos.slot * kSlotBytes);
+            const uint4* Q = reinterpret_cast<const uint4*>(ring + pos.slot * kSlotBytes + kHalfSlot);
+            if (c == cstar && t == tstar) {
+              int at;
+              float carry;
+              find_first<T>(P[istar], Q[istar], tot.av, &at, &carry);
+              S.arg_index = tot.ab + at;
+              S.arg_carry = carry;
+            }
+            if (c == cyh && t == tyh) {
+              int at;
+              float carry;
+              find_first<T>(Q[iyh], P[iyh], tot.qv, &at, &carry);
+              S.yarg_index = tot.qb + at;
+              S.yarg_carry = carry;
+            }
+            if (c < nfull) {
+#pragma unroll
+              for (int v = 0; v < kNV; ++v) {
+                const int i = t + v * kConsumers;
+                phase2_bf16(smin2, sqlt2, P[i], Q[i], a.sT, nCp, nCq);
+              }
+            } else {
+              const int nvec = (V - e0) / E;
+              for (int i = t; i < nvec; i += kConsumers) phase2_bf16(smin2, sqlt2, P[i], Q[i], a.sT, nCp, nCq);
+            }
+          }
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&S.empty[pos.slot]);
+        }
+        smin += smin2.x + smin2.y;
+        sqlt += sqlt2.x + sqlt2.y;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) {
+          smin += __shfl_xor_sync(0xffffffffu, smin, off);
+          sqlt += __shfl_xor_sync(0xffffffffu, sqlt, off);
+        }
+        if (lane == 0) S.red2[j & 1][warp] = make_float2(smin, sqlt);
+        named_barrier(kBarSum, kConsumers);
+        if (t == 0) {
+          float2 x = S.red2[j & 1][0];
+          for (int w = 1; w < kWarps; ++w) {
+            x.x += S.red2[j & 1][w].x;
+            x.y += S.red2[j & 1][w].y;
+          }
+          const float Mq1 = NEED_Q1 ? tot.q1M : Mq;
+          const float Lsq1 = NEED_Q1 ? log2f(tot.q1S) : Lsq;
+          const float ag = exp2f(log2_prob(S.arg_carry, kLog2e, Mq1, Lsq1));
+          if (!*abort_flag) {
+            a.ws.cpart[r * kMaxCluster] = x;
+            a.ws.Mp[r] = Mp;
+            a.ws.Lsp[r] = Lsp;
+            a.ws.Mq[r] = Mq;
+            a.ws.Lsq[r] = Lsq;
+            a.ws.Mq1[r] = Mq1;
+            a.ws.Lsq1[r] = Lsq1;
+            a.ws.xstar[r] = S.arg_index;
+            a.ws.ag[r] = ag;
+            a.ws.yhat[r] = S.yarg_index;
+            a.ws.zpy[r] = S.yarg_carry;
+          }
+          st.Mq = Mq;
+          st.Lsq = Lsq;
+          st.Mp = Mp;
+          st.Lsp = Lsp;
+          st.Mq1 = Mq1;
+          st.Lsq1 = Lsq1;
+          st.qlt = x.y;
+          st.ag = ag;
+          st.xs = S.arg_index;
+          st.ys = S.yarg_index;
+          S.arg_index = 0x7fffffff;
+          S.arg_carry = 0.f;
+          S.yarg_index = 0x7fffffff;
+          S.yarg_carry = 0.f;
+        }
+      }
+
+      // ---- group barrier, then the row's coefficients (thread 0)
+      if (t == 0) {
+        red_release_add(&a.ws.gcnt[g], 1u);
+        bool ok = !*abort_flag;
+        if (ok) {
+          const uint32_t target = (j + 1u) * (uint32_t)K;
+          const uint64_t t0 = now_ns();
+          for (uint32_t it = 0; ld_acquire(&a.ws.gcnt[g]) < target; ++it) {
+            if (*abort_flag || it >= kSpinLimit || now_ns() - t0 > limit_ns) {
+              if (!*abort_flag) {
+                *abort_flag = 1;
+                atomicExch(&hdr->status, kStatusTimeout);
+              }
+              ok = false;
+              break;
+            }
+            __nanosleep(128);
+          }
+        }
+        int32_t live = 0;
+        if (ok) {
+          // the window's terms, as the window kernel forms them (rows n K .. n K + K - 1)
+          const int64_t r0 = n * K;
+          int kn = K;
+          if (f.win.mask != nullptr) {
+            kn = 0;
+            while (kn < K && f.win.mask[r0 + kn] != 0) ++kn;
+          }
+          const bool ov = f.win.sampling || f.win.tv;
+          float agv[AAL_MAX_K], asv[AAL_MAX_K], dE[AAL_MAX_K];
+#pragma unroll
+          for (int jj = 0; jj < AAL_MAX_K; ++jj) {
+            agv[jj] = 0.f;
+            asv[jj] = 0.f;
+            if (jj < K) {
+              if (f.win.greedy) agv[jj] = __ldcg(&a.ws.ag[r0 + jj]);
+              if (ov) asv[jj] = __ldcg(&a.ws.cpart[(r0 + jj) * kMaxCluster]).x;
+            }
+          }
+          float dEg = 0.f, dEs = 0.f;
+          if (f.win.greedy) {
+            window_term(agv, kn, dE);
+            dEg = dE[k];
+          }
+          if (ov) {
+            if (f.win.sampling) window_term(asv, kn, dE);
+            const float tvc = (f.win.tv && kn > 0) ? f.win.w_tv / (float)kn : 0.f;
+            dEs = (f.win.sampling ? f.win.w_sampling * dE[k] : 0.f) + (k < kn ? tvc : 0.f);
+          }
+          const bool with_greedy = GREEDY && f.bw.w_greedy != 0.f;
+          const bool pos_valid = f.bw.mask == nullptr || f.bw.mask[r] != 0;
+          RowCoef c;
+          live = row_coef<GREEDY, SAMPLING, KL>(f.bw, scale, kscale, with_greedy ? dEg : 0.f, SAMPLING ? dEs : 0.f,
+                                                0.f, pos_valid, st, c)
+                     ? 1
+                     : 0;
+          F.coef = c;
+        }
+        F.live = live;
+      }
+      named_barrier(kBarCoef, kConsumers);
+
+      // ---- pass 3: the gradient row (L2)
+      const int32_t live = F.live;
+      const RowCoef c = F.coef;
+      const int64_t xv = (live && c.xs >= 0) ? c.xs / E : -1;
+      const int xe = c.xs >= 0 ? c.xs % E : 0;
+      uint4* out4 = reinterpret_cast<uint4*>(static_cast<T*>(f.bw.grad) + r * a.V);
+      const uint4 zero4 = make_uint4(0, 0, 0, 0);
+      for (int cc = 0; cc < nch; ++cc, pos.next()) {
+        if (wait_full(&S.full[pos.slot], pos.phase, abort_flag, limit_ns, hdr)) {
+          const int e0 = cc * CH;
+          const int64_t vb = e0 / E;
+          const uint4* P = reinterpret_cast<const uint4*>(ring + pos.slot * kSlotBytes);
+          const uint4* Q = reinterpret_cast<const uint4*>(ring + pos.slot * kSlotBytes + kHalfSlot);
+          if (cc < nfull) {
+#pragma unroll
+            for (int v = 0; v < kNV; ++v) {
+              const int i = t + v * kConsumers;
+              st_stream(out4 + vb + i,
+                        live ? grad_vec<T, GREEDY, SAMPLING, Q1_IS_QT, KL>(c, Q[i], P[i], vb + i, xv, xe, -1, 0) : zero4);
+            }
+          } else {
+            const int nvec = (V - e0) / E;
+            for (int i = t; i < nvec; i += kConsumers)
+              st_stream(out4 + vb + i,
+                        live ? grad_vec<T, GREEDY, SAMPLING, Q1_IS_QT, KL>(c, Q[i], P[i], vb + i, xv, xe, -1, 0) : zero4);
+          }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&S.empty[pos.slot]);
+      }
+    }
+  }
+  __syncwarp();
+  __syncthreads();
+}
+
+// |W| (windows whose depth 0 is valid) and |positions| (valid rows) from the [N][K] mask, one
+// block; integer sums, so the order does not matter.
+__global__ void __launch_bounds__(1024) count_valid(const uint8_t* mask, int64_t N, int32_t K, WsHeader* hdr) {
+  __shared__ unsigned long long sw, sp;
+  if (threadIdx.x == 0) {
+    sw = 0ull;
+    sp = 0ull;
+  }
+  __syncthreads();
+  unsigned long long w = 0, p = 0;
+  if (mask == nullptr) {
+    if (threadIdx.x == 0) {
+      w = (unsigned long long)N;
+      p = (unsigned long long)(N * K);
+    }
+  } else {
+    for (int64_t n = threadIdx.x; n < N; n += blockDim.x) w += mask[n * K] != 0;
+    for (int64_t r = threadIdx.x; r < N * K; r += blockDim.x) p += mask[r] != 0;
+  }
+  atomicAdd(&sw, w);
+  atomicAdd(&sp, p);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    hdr->nvalid = (int32_t)sw;
+    hdr->npos = (int32_t)sp;
+  }
+}
+
+template <bool NQ1, int P, bool KL, bool GR, bool Q>
+cudaError_t go_fused(const FusedArgs& f0, cudaStream_t s, uint64_t limit_ns, bool* launched) {
+  auto kern = fused_rows<NQ1, P, KL, GR, Q>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFusedSmemBytes);
+  if (e != cudaSuccess) return e;
+  int dev = 0, sms = 0, per_sm = 0, coop = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev);
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, kFusedSmemBytes);
+  if (e != cudaSuccess) return e;
+  const int64_t K = f0.win.K;
+  int64_t G = (int64_t)sms * per_sm / K;
+  if (G > f0.win.N) G = f0.win.N;
+  if (G > kMaxGroups) G = kMaxGroups;
+  if (!coop || G < 1) return cudaSuccess;  // *launched stays false: the caller runs the two calls
+  FusedArgs f = f0;
+  f.groups = (int32_t)G;
+  const int elt = 2;
+  const int nch = (int)((f.st.V + kHalfSlot / elt - 1) / (kHalfSlot / elt));
+  void* args[] = {&f, (void*)&nch, &limit_ns};
+  e = cudaLaunchCooperativeKernel((const void*)kern, dim3((unsigned)(G * K)), dim3(kThreads), args, kFusedSmemBytes, s);
+  if (e == cudaSuccess) *launched = true;
+  return e;
+}
+
+}  // namespace
+
+cudaError_t launch_count_valid(const uint8_t* mask, int64_t N, int32_t K, WsHeader* hdr, cudaStream_t s) {
+  count_valid<<<1, 1024, 0, s>>>(mask, N, K, hdr);
+  return cudaGetLastError();
+}
+
+// The instantiation for the problem's flags, or none (launched = false) for a combination
+// this path does not take.
+cudaError_t launch_fused(const FusedArgs& f, cudaStream_t s, uint64_t limit_ns, bool* launched) {
+  *launched = false;
+  const bool two = f.st.overlap, kl = f.st.need_kl, nq1 = f.st.need_q1 && two;
+  const bool greedy = f.bw.w_greedy != 0.f && !f.bw.grpo;
+  const bool q = f.bw.q1_is_qT && two && (greedy || kl);
+  if (!two) {
+    if (greedy && !kl) return go_fused<false, 1, false, true, false>(f, s, limit_ns, launched);
+    if (!greedy && kl) return go_fused<false, 1, true, false, false>(f, s, limit_ns, launched);
+    if (greedy && kl) return go_fused<false, 1, true, true, false>(f, s, limit_ns, launched);
+    return cudaSuccess;
+  }
+  if (kl) {
+    if (nq1 || !q) return cudaSuccess;
+    return greedy ? go_fused<false, 2, true, true, true>(f, s, limit_ns, launched)
+                  : go_fused<false, 2, true, false, true>(f, s, limit_ns, launched);
+  }
+  if (!greedy && !nq1 && !q) return go_fused<false, 2, false, false, false>(f, s, limit_ns, launched);
+  if (greedy && !nq1 && q) return go_fused<false, 2, false, true, true>(f, s, limit_ns, launched);
+  if (greedy && nq1 && !q) return go_fused<true, 2, false, true, false>(f, s, limit_ns, launched);
+  return cudaSuccess;
+}
+
+}  // namespace aal

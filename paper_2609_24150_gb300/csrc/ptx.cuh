@@ -79,6 +79,18 @@ __device__ __forceinline__ void named_barrier(int id, int n) {
   __syncwarp();
   asm volatile("barrier.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
 }
+// GPU-scope release add and acquire load on a global counter (the fused kernel's group
+// barrier): a CTA's row statistics, written before its release, are visible to a CTA whose
+// acquire load sees the count.
+__device__ __forceinline__ void red_release_add(uint32_t* p, uint32_t v) {
+  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
 __device__ __forceinline__ uint64_t now_ns() {
   uint64_t t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));

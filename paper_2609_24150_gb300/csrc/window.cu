@@ -86,31 +86,6 @@ __device__ __forceinline__ void finish_loss(const Args& a, double (&x)[kSums], d
   }
 }
 
-// Expected length and its partials for one window term; returns E.
-__device__ __forceinline__ float window_term(const float* a, int kn, float* dE) {
-  float P[AAL_MAX_K + 1];
-  P[0] = 1.f;
-  float E = 0.f;
-#pragma unroll
-  for (int j = 0; j < AAL_MAX_K; ++j) {
-    if (j < kn) {
-      P[j + 1] = P[j] * a[j];
-      E += P[j + 1];
-    }
-  }
-  float S = 1.f;
-#pragma unroll
-  for (int j = AAL_MAX_K - 1; j >= 0; --j) {
-    if (j < kn) {
-      dE[j] = P[j] * S;
-      S = 1.f + a[j] * S;
-    } else {
-      dE[j] = 0.f;
-    }
-  }
-  return E;
-}
-
 __global__ void __launch_bounds__(kWindowThreads) window_kernel(WindowArgs a) {
   __shared__ double sm[kSums * kWindowThreads / 32];
   __shared__ bool is_last;

@@ -25,7 +25,7 @@ def _declared():
 
 def test_header_declares_the_entry_points():
     names = _declared()
-    assert {"aal_loss_fwd", "aal_loss_bwd", "aal_accept_reward", "aal_workspace_size",
+    assert {"aal_loss_fwd", "aal_loss_bwd", "aal_loss_fwd_bwd", "aal_accept_reward", "aal_workspace_size",
             "aal_reward_workspace_size", "aal_check_device_status", "aal_status_string",
             "aal_abi_version"} <= names
 
@@ -41,7 +41,7 @@ def test_library_exports_every_declared_symbol():
 
 
 def test_status_strings_and_version():
-    assert aal.aal_abi_version() == 10400
+    assert aal.aal_abi_version() == 10500
     for code in range(6):
         assert aal.aal_status_string(code).startswith("AAL_")
     assert aal.aal_status_string(99) == "unknown aal_status"
@@ -125,6 +125,16 @@ def test_null_and_misaligned_pointers_rejected_before_launch():
     # backward: NULL gradient, non-finite upstream gradient
     assert lib.aal_loss_bwd(ctypes.byref(p), fake, fake, None, fake_ws, size, 1.0, None, None) == aal.AAL_ERR_INVALID_ARG
     assert lib.aal_loss_bwd(ctypes.byref(p), fake, fake, None, fake_ws, size, float("nan"), fake, None) == aal.AAL_ERR_INVALID_ARG
+    # the one-call forward + backward: every check of both calls, and GRPO refused
+    fb = lambda prob, d=fake, ws=fake_ws, sz=size, dl=1.0, loss=fake, grad=fake: lib.aal_loss_fwd_bwd(
+        ctypes.byref(prob), d, fake, None, ws, sz, dl, loss, None, grad, None)
+    assert fb(p, grad=None) == aal.AAL_ERR_INVALID_ARG
+    assert fb(p, loss=None) == aal.AAL_ERR_INVALID_ARG
+    assert fb(p, d=fake + 2) == aal.AAL_ERR_INVALID_ARG
+    assert fb(p, dl=float("inf")) == aal.AAL_ERR_INVALID_ARG
+    assert fb(p, sz=size - 1) == aal.AAL_ERR_WORKSPACE
+    assert fb(_prob(mode=aal.AAL_GRPO | aal.AAL_GREEDY)) == aal.AAL_ERR_UNSUPPORTED
+    assert fb(_prob(K=9)) == aal.AAL_ERR_UNSUPPORTED
 
 
 def _rprob(**kw):

@@ -1,0 +1,150 @@
+"""The one-call forward + backward (aal_loss_fwd_bwd).
+
+It must give the loss, the per-window expected lengths and the gradient of aal_loss_fwd followed
+by aal_loss_bwd bit for bit: on the fused path (bf16 rows of 16-byte multiples; every flag
+combination it instantiates, masks, fewer windows than CTA groups, K = 1 and K = 8, full-size
+rows) and on the problems it hands to the two calls (fp32, unaligned rows, token ids, the
+anchor beside the sampling term at T != 1).  A few cases are also checked against the oracle
+directly, and the group barrier's bounded wait is driven to a timeout without a fault.
+"""
+
+import pytest
+import torch
+
+import paper_2609_24150_gb300 as aal
+import synth
+from tests.parity import LossRun, check_loss
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda:0"
+G, S, B, KL, TV, IDS = aal.AAL_GREEDY, aal.AAL_SAMPLING, aal.AAL_BOTH, aal.AAL_KL, aal.AAL_TV, aal.AAL_IDS
+
+
+class FusedRun:
+    """aal_loss_fwd_bwd of one problem; the same fields as LossRun."""
+
+    def __init__(self, target, draft, mask, mode, T=1.0, wg=1.0, ws=1.0, dloss=1.0, wkl=1.0, wtv=1.0):
+        self.prob = aal.loss_problem(draft, mode, T, wg, ws, wkl, wtv)
+        self.ws_buf = torch.empty(aal.aal_workspace_size(self.prob), dtype=torch.uint8, device=draft.device)
+        N = draft.shape[0]
+        self.loss = torch.full((1,), float("nan"), dtype=torch.float32, device=draft.device)
+        self.eal = torch.full((max(N, 1), 2), float("nan"), dtype=torch.float32, device=draft.device)
+        self.grad = torch.full_like(draft, float("nan"))
+        aal.aal_loss_fwd_bwd(self.prob, draft, target, mask, self.ws_buf, dloss, self.loss, self.grad,
+                             self.eal if N > 0 else None)
+        torch.cuda.synchronize()
+        assert aal.aal_check_device_status(self.ws_buf) == aal.AAL_OK
+
+
+def _bits(x):
+    return x.view(torch.int16) if x.element_size() == 2 else x.view(torch.int32)
+
+
+def assert_same(f, s):
+    assert torch.equal(_bits(f.loss), _bits(s.loss)), (f.loss.item(), s.loss.item())
+    assert torch.equal(_bits(f.eal), _bits(s.eal))
+    diff = _bits(f.grad) != _bits(s.grad)
+    assert not diff.any(), f"{int(diff.sum())} gradient elements differ, first at {diff.nonzero()[0].tolist()}"
+
+
+def _inputs(N, K, V, seed, masked=False, dtype=torch.bfloat16):
+    t, d, _ = synth.make_logits("tiny", seed=seed, N=N, K=K, V=V, dtype=dtype)
+    mask = None
+    if masked:
+        g = torch.Generator().manual_seed(seed + 1)
+        mask = (torch.rand((N, K), generator=g) >= 0.15).to(torch.uint8)
+        mask[0, 0] = 0                        # a window outside W
+        mask[1, :] = 1                        # a full window
+        mask = mask.to(DEV)
+    return t.to(DEV), d.to(DEV), mask
+
+
+# (N, K, V, mode, T, wg, ws, wkl, wtv, masked): each fused instantiation at least once
+CASES = [
+    (24, 7, 4104, B, 1.0, 0.5, 0.5, 1.0, 1.0, False),       # two passes, q = q~ at T = 1
+    (40, 5, 20000, S, 0.7, 1.0, 1.0, 1.0, 1.0, True),       # sampling only, T != 1, two chunks a row
+    (16, 8, 8192, B, 1.5, 0.5, 0.5, 1.0, 1.0, False),       # greedy q beside q~ at T != 1
+    (33, 3, 1000, G, 1.0, 1.0, 0.0, 1.0, 1.0, True),        # one pass, argmaxes resolved from L2
+    (20, 4, 3000, KL | G, 1.0, 0.1, 0.0, 1.0, 1.0, False),  # one pass with the anchor
+    (20, 4, 3000, KL, 1.0, 0.0, 0.0, 1.0, 1.0, True),       # the anchor alone
+    (12, 6, 6000, KL | B, 1.0, 0.1, 0.1, 1.0, 1.0, True),   # two passes with the anchor
+    (12, 6, 6000, KL | TV, 1.0, 0.0, 0.0, 1.0, 0.1, False), # TV term + anchor, no greedy term
+    (3, 7, 128256, B, 1.0, 0.5, 0.5, 1.0, 1.0, False),      # fewer windows than groups, full rows
+    (200, 1, 2048, B, 1.0, 0.5, 0.5, 1.0, 1.0, False),      # K = 1: groups of one CTA
+]
+
+
+@pytest.mark.parametrize("N,K,V,mode,T,wg,ws,wkl,wtv,masked", CASES)
+@pytest.mark.parametrize("dloss_is_w", [False, True])
+def test_fused_equals_two_calls(N, K, V, mode, T, wg, ws, wkl, wtv, masked, dloss_is_w):
+    t, d, m = _inputs(N, K, V, seed=N + K + V, masked=masked)
+    dloss = float(N) if dloss_is_w else 1.0   # |W|-sized upstream gradient makes the absolute term bind
+    f = FusedRun(t, d, m, mode, T, wg, ws, dloss, wkl, wtv)
+    s = LossRun(t, d, m, mode, T, wg, ws, dloss, wkl, wtv)
+    assert_same(f, s)
+
+
+def test_fused_no_valid_window():
+    t, d, _ = _inputs(8, 4, 4096, seed=5)
+    m = torch.zeros((8, 4), dtype=torch.uint8, device=DEV)
+    f = FusedRun(t, d, m, B, 1.0, 0.5, 0.5)
+    assert f.loss.item() == 0.0 and not f.grad.float().abs().gt(0).any()
+    assert_same(f, LossRun(t, d, m, B, 1.0, 0.5, 0.5))
+
+
+@pytest.mark.parametrize("mode,T,dtype,V", [
+    (B, 1.0, torch.float32, 4096),        # fp32 logits
+    (B, 1.0, torch.bfloat16, 1001),       # rows that are not 16-byte multiples
+    (KL | S, 0.8, torch.bfloat16, 4096),  # the anchor beside the sampling term at T != 1
+])
+def test_problems_the_two_calls_take(mode, T, dtype, V):
+    t, d, m = _inputs(10, 3, V, seed=V, masked=True, dtype=dtype)
+    assert_same(FusedRun(t, d, m, mode, T, 0.5, 0.5), LossRun(t, d, m, mode, T, 0.5, 0.5))
+
+
+def test_token_ids_take_the_two_calls():
+    t, d, _ = _inputs(10, 3, 4096, seed=9)
+    ids = t.float().argmax(-1).to(torch.int32).contiguous()
+    assert_same(FusedRun(ids, d, None, G | IDS, 1.0, 1.0, 0.0), LossRun(ids, d, None, G | IDS, 1.0, 1.0, 0.0))
+
+
+def test_grpo_is_refused():
+    t, d, _ = _inputs(4, 2, 1024, seed=1)
+    with pytest.raises(aal.AalError):
+        FusedRun(t, d, None, G | aal.AAL_GRPO, 1.0, 1.0, 0.0)
+
+
+@pytest.mark.parametrize("mode,T,wg,ws", [(B, 1.0, 0.5, 0.5), (KL | G, 1.0, 0.1, 0.0), (S, 1.3, 0.0, 1.0)])
+def test_fused_against_the_oracle(mode, T, wg, ws):
+    t, d, m = _inputs(24, 5, 3000, seed=17, masked=True)
+    check_loss(FusedRun(t, d, m, mode, T, wg, ws, dloss=24.0), t, d, m, mode, T, wg, ws, dloss=24.0)
+
+
+def test_group_barrier_and_ring_time_out_and_context_stays_usable():
+    """One ring copy of every CTA is left unarmed: its waits run out (50 ms), the CTAs that gave
+    up still add their group arrivals, and the call returns with AAL_ERR_TIMEOUT recorded."""
+    t, d, _ = _inputs(16, 2, 20000, seed=11)
+    prob = aal.loss_problem(d, B, 1.0, 0.5, 0.5)
+    ws = torch.empty(aal.aal_workspace_size(prob), dtype=torch.uint8, device=DEV)
+    loss = torch.empty(1, device=DEV)
+    grad = torch.empty_like(d)
+    aal.aal_debug_fail_next_forward(3, 50_000_000)
+    try:
+        aal.aal_loss_fwd_bwd(prob, d, t, None, ws, 1.0, loss, grad)
+        assert aal.aal_check_device_status(ws) == aal.AAL_ERR_TIMEOUT
+        assert aal.aal_check_device_status(ws) == aal.AAL_OK
+    finally:
+        aal.aal_debug_fail_next_forward(-1, 0)
+    assert_same(FusedRun(t, d, None, B, 1.0, 0.5, 0.5), LossRun(t, d, None, B, 1.0, 0.5, 0.5))
+
+
+def test_v128k_full_size_fused_equals_two_calls():
+    t, d, _ = synth.make_logits("v128k", seed=0, device=DEV)
+    f = FusedRun(t, d, None, B, 1.0, 0.5, 0.5)
+    s = LossRun(t, d, None, B, 1.0, 0.5, 0.5)
+    assert_same(f, s)
+    del f, s
+    f = FusedRun(t, d, None, KL | G, 1.0, 0.1, 0.0)
+    s = LossRun(t, d, None, KL | G, 1.0, 0.1, 0.0)
+    assert_same(f, s)
