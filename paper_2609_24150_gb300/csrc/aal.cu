@@ -309,7 +309,7 @@ aal_status aal_loss_fwd_bwd(const aal_problem* prob, const void* draft, const vo
   if (fusable) {
     LossWs ws = loss_ws(workspace, L);
     if (cudaMemsetAsync(ws.hdr, 0, sizeof(WsHeader), s) != cudaSuccess) return AAL_ERR_CUDA;
-    if (cudaMemsetAsync(ws.gcnt, 0, (size_t)kMaxGroups * 4, s) != cudaSuccess) return AAL_ERR_CUDA;
+    if (cudaMemsetAsync(ws.mbox, 0xff, (size_t)L.R * 8, s) != cudaSuccess) return AAL_ERR_CUDA;  // kMboxEmpty
     if (launch_count_valid(mask, prob->N, (int32_t)prob->K, ws.hdr, s) != cudaSuccess) return AAL_ERR_CUDA;
     FusedArgs f;
     f.st = stats_args(draft, target, L.R, prob->V, prob->mode, prob->temperature, ws);

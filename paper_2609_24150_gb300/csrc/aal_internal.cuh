@@ -14,6 +14,7 @@ constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr int kMaxCluster = 8;          // CTAs that may share one logit row
 constexpr int kMaxGroups = 1024;        // fused forward + backward: groups of K CTAs per launch
+constexpr uint64_t kMboxEmpty = ~0ull;  // a mailbox word not yet written (no arithmetic result has these bits)
 constexpr uint32_t kStatusTimeout = 5;  // == AAL_ERR_TIMEOUT
 
 // ---------------------------------------------------------------------------
@@ -48,7 +49,7 @@ struct LossLayout {
   size_t zpy = 0;                   // float[R] z_p at the draft argmax
   size_t cpart = 0;                 // float2[R][kMaxCluster] per-CTA (overlap, Qlt) partials
   size_t wpart = 0;                 // double[nwblk][kWpart] window-kernel block partials
-  size_t gcnt = 0;                  // uint32[kMaxGroups] fused forward + backward: group arrivals
+  size_t mbox = 0;                  // uint64[R] fused forward + backward: (a^greedy, a^sample) per row
   size_t total = 0;
 };
 
@@ -90,7 +91,7 @@ inline LossLayout loss_layout(int64_t N, int64_t K) {
   L.zpy = take(R * 4);
   L.cpart = take(R * kMaxCluster * 8);
   L.wpart = take((size_t)(L.nwblk > 0 ? L.nwblk : 1) * kWpart * 8);
-  L.gcnt = take((size_t)kMaxGroups * 4);
+  L.mbox = take(R * 8);
   L.total = off;
   return L;
 }
@@ -150,7 +151,7 @@ struct LossWs {
   float* zpy;
   float2* cpart;
   double* wpart;
-  uint32_t* gcnt;
+  uint64_t* mbox;
 };
 
 inline LossWs loss_ws(void* base, const LossLayout& L) {
@@ -177,7 +178,7 @@ inline LossWs loss_ws(void* base, const LossLayout& L) {
   w.zpy = reinterpret_cast<float*>(b + L.zpy);
   w.cpart = reinterpret_cast<float2*>(b + L.cpart);
   w.wpart = reinterpret_cast<double*>(b + L.wpart);
-  w.gcnt = reinterpret_cast<uint32_t*>(b + L.gcnt);
+  w.mbox = reinterpret_cast<uint64_t*>(b + L.mbox);
   return w;
 }
 

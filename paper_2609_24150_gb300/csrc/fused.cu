@@ -12,18 +12,21 @@
 //   G groups x K CTAs; CTA k of group g takes depth k of windows g, g + G, ...  A cooperative
 //   launch has all its CTAs resident at once, so a group never waits on a CTA that is not
 //   running.
-// * Group barrier: once its row's statistics are in the workspace, thread 0 of each CTA adds
-//   one to the group's counter (release) and waits (acquire, bounded like the ring waits) for
-//   K arrivals per window.  It then reads the window's a^greedy, a^sample and mask, forms
-//   dE^g/da and dE^s/da with the window kernels' function (window_term) and the row's gradient
-//   coefficients with the backward's (row_coef), so that the gradient equals the one of
+// * Window exchange: once its row's statistics are in the workspace, thread 0 of each CTA
+//   publishes the row's (a^greedy, a^sample) as one 64-bit word in a per-row mailbox that the
+//   call filled with an all-ones sentinel, and warp 0 polls (bounded, like the ring waits; lane
+//   j the word of depth j) the K words of its window until none is the sentinel: the value is its own ready flag, so one L2 round
+//   trip brings the data.  It then forms dE^g/da and dE^s/da with the window kernels' function
+//   (window_term) and the row's gradient coefficients with the backward's (row_coef), from the
+//   same floats the window kernel reads later, so that the gradient equals the one of
 //   aal_loss_fwd + aal_loss_bwd bit for bit.  The loss is left to the window kernel, which runs
-//   after this one over the statistics written here, exactly as in aal_loss_fwd.
+//   after this one over the statistics written here, exactly as in aal_loss_fwd.  The anchor
+//   alone needs no window term and so no wait.
 // * The counts of valid windows and positions that scale the gradient are taken from the mask
 //   by count_valid before the launch (the separate forward gets them from its window kernel).
 // * Failure: every wait is bounded.  A CTA that gave up keeps walking its rows without waiting
-//   and still adds its arrivals, so its group does not wait on it for the whole limit; the
-//   workspace status word reports AAL_ERR_TIMEOUT and the outputs are not to be used.
+//   and still publishes a word for each, so its group does not wait on it for the whole limit;
+//   the workspace status word reports AAL_ERR_TIMEOUT and the outputs are not to be used.
 #include "grad_elem.cuh"
 #include "stream_core.cuh"
 
@@ -166,6 +169,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
       const float Mp = tot.pM, Lsp = log2f(tot.pS);
       const float Mq = tot.qM, Lsq = log2f(tot.qS);
       RowStat st{};  // thread 0: what the row's coefficients need
+      float st_as = 0.f;  // thread 0: the row's a^sample (two passes)
       if (KL && t == 0) {  // both normalisers are at T = 1 here
         const float Mq1 = NEED_Q1 ? tot.q1M : Mq;
         const float Lsq1 = NEED_Q1 ? log2f(tot.q1S) : Lsq;
@@ -288,6 +292,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
           st.Mq1 = Mq1;
           st.Lsq1 = Lsq1;
           st.qlt = x.y;
+          st_as = x.x;
           st.ag = ag;
           st.xs = S.arg_index;
           st.ys = S.yarg_index;
@@ -298,65 +303,81 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
         }
       }
 
-      // ---- group barrier, then the row's coefficients (thread 0)
-      if (t == 0) {
-        red_release_add(&a.ws.gcnt[g], 1u);
-        bool ok = !*abort_flag;
-        if (ok) {
-          const uint32_t target = (j + 1u) * (uint32_t)K;
+      // ---- the window's acceptances (warp 0: lane j polls depth j), the row's coefficients (thread 0)
+      if (warp == 0) {
+        const bool ov = f.win.sampling || f.win.tv;
+        const bool need = f.win.greedy || ov;  // the anchor alone needs no window term
+        const int64_t r0 = n * K;
+        if (lane == 0) {
+          // publish this row's (a^greedy, a^sample): one 64-bit word, its own ready flag
+          const float as_r = PASSES == 2 ? st_as : 0.f;
+          uint64_t word = ((uint64_t)__float_as_uint(as_r) << 32) | __float_as_uint(st.ag);
+          if (word == kMboxEmpty) word = 0;  // (bit patterns no arithmetic yields; never sent)
+          st_relaxed(&a.ws.mbox[r], word);
+        }
+        // one reading of the abort flag for the whole warp (another warp may raise it meanwhile)
+        bool ok = __shfl_sync(0xffffffffu, *abort_flag == 0 ? 1 : 0, 0) != 0;
+        uint64_t w = 0;
+        if (ok && need) {
           const uint64_t t0 = now_ns();
-          for (uint32_t it = 0; ld_acquire(&a.ws.gcnt[g]) < target; ++it) {
-            if (*abort_flag || it >= kSpinLimit || now_ns() - t0 > limit_ns) {
+          for (uint32_t it = 0;; ++it) {
+            if (lane < K) w = ld_relaxed(&a.ws.mbox[r0 + lane]);
+            if (__all_sync(0xffffffffu, lane >= K || w != kMboxEmpty)) break;
+            // lane 0 decides for the warp whether to give up
+            int quit = 0;
+            if (lane == 0 && (*abort_flag || it >= kSpinLimit || now_ns() - t0 > limit_ns)) {
               if (!*abort_flag) {
                 *abort_flag = 1;
                 atomicExch(&hdr->status, kStatusTimeout);
               }
+              quit = 1;
+            }
+            if (__shfl_sync(0xffffffffu, quit, 0)) {
               ok = false;
               break;
             }
-            __nanosleep(128);
+            __nanosleep(64);
           }
         }
-        int32_t live = 0;
-        if (ok) {
-          // the window's terms, as the window kernel forms them (rows n K .. n K + K - 1)
-          const int64_t r0 = n * K;
-          int kn = K;
-          if (f.win.mask != nullptr) {
-            kn = 0;
-            while (kn < K && f.win.mask[r0 + kn] != 0) ++kn;
-          }
-          const bool ov = f.win.sampling || f.win.tv;
-          float agv[AAL_MAX_K], asv[AAL_MAX_K], dE[AAL_MAX_K];
+        float agv[AAL_MAX_K], asv[AAL_MAX_K];
 #pragma unroll
-          for (int jj = 0; jj < AAL_MAX_K; ++jj) {
-            agv[jj] = 0.f;
-            asv[jj] = 0.f;
-            if (jj < K) {
-              if (f.win.greedy) agv[jj] = __ldcg(&a.ws.ag[r0 + jj]);
-              if (ov) asv[jj] = __ldcg(&a.ws.cpart[(r0 + jj) * kMaxCluster]).x;
-            }
-          }
-          float dEg = 0.f, dEs = 0.f;
-          if (f.win.greedy) {
-            window_term(agv, kn, dE);
-            dEg = dE[k];
-          }
-          if (ov) {
-            if (f.win.sampling) window_term(asv, kn, dE);
-            const float tvc = (f.win.tv && kn > 0) ? f.win.w_tv / (float)kn : 0.f;
-            dEs = (f.win.sampling ? f.win.w_sampling * dE[k] : 0.f) + (k < kn ? tvc : 0.f);
-          }
-          const bool with_greedy = GREEDY && f.bw.w_greedy != 0.f;
-          const bool pos_valid = f.bw.mask == nullptr || f.bw.mask[r] != 0;
-          RowCoef c;
-          live = row_coef<GREEDY, SAMPLING, KL>(f.bw, scale, kscale, with_greedy ? dEg : 0.f, SAMPLING ? dEs : 0.f,
-                                                0.f, pos_valid, st, c)
-                     ? 1
-                     : 0;
-          F.coef = c;
+        for (int jj = 0; jj < AAL_MAX_K; ++jj) {  // to lane 0 (0 beyond K, or without the term)
+          const float g_ = __shfl_sync(0xffffffffu, __uint_as_float((uint32_t)w), jj);
+          const float s_ = __shfl_sync(0xffffffffu, __uint_as_float((uint32_t)(w >> 32)), jj);
+          agv[jj] = (jj < K && need && f.win.greedy) ? g_ : 0.f;
+          asv[jj] = (jj < K && need && ov) ? s_ : 0.f;
         }
-        F.live = live;
+        if (lane == 0) {
+          int32_t live = 0;
+          if (ok) {
+            // the window's terms, as the window kernel forms them (rows n K .. n K + K - 1)
+            int kn = K;
+            if (f.win.mask != nullptr) {
+              kn = 0;
+              while (kn < K && f.win.mask[r0 + kn] != 0) ++kn;
+            }
+            float dE[AAL_MAX_K];
+            float dEg = 0.f, dEs = 0.f;
+            if (f.win.greedy) {
+              window_term(agv, kn, dE);
+              dEg = dE[k];
+            }
+            if (ov) {
+              if (f.win.sampling) window_term(asv, kn, dE);
+              const float tvc = (f.win.tv && kn > 0) ? f.win.w_tv / (float)kn : 0.f;
+              dEs = (f.win.sampling ? f.win.w_sampling * dE[k] : 0.f) + (k < kn ? tvc : 0.f);
+            }
+            const bool with_greedy = GREEDY && f.bw.w_greedy != 0.f;
+            const bool pos_valid = f.bw.mask == nullptr || f.bw.mask[r] != 0;
+            RowCoef c;
+            live = row_coef<GREEDY, SAMPLING, KL>(f.bw, scale, kscale, with_greedy ? dEg : 0.f,
+                                                  SAMPLING ? dEs : 0.f, 0.f, pos_valid, st, c)
+                       ? 1
+                       : 0;
+            F.coef = c;
+          }
+          F.live = live;
+        }
       }
       named_barrier(kBarCoef, kConsumers);
 

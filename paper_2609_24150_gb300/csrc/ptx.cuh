@@ -79,15 +79,14 @@ __device__ __forceinline__ void named_barrier(int id, int n) {
   __syncwarp();
   asm volatile("barrier.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
 }
-// GPU-scope release add and acquire load on a global counter (the fused kernel's group
-// barrier): a CTA's row statistics, written before its release, are visible to a CTA whose
-// acquire load sees the count.
-__device__ __forceinline__ void red_release_add(uint32_t* p, uint32_t v) {
-  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+// GPU-scope relaxed 64-bit store and load (single-copy atomic, coherent in L2): the fused
+// kernel's mailbox words, whose value is their own ready flag.
+__device__ __forceinline__ void st_relaxed(uint64_t* p, uint64_t v) {
+  asm volatile("st.relaxed.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
 }
-__device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
-  uint32_t v;
-  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+__device__ __forceinline__ uint64_t ld_relaxed(const uint64_t* p) {
+  uint64_t v;
+  asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
   return v;
 }
 
