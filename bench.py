@@ -42,7 +42,7 @@ STEP_WORKLOAD = ("v128k: N=8192 windows (B=4 x T=2048), K=7, V=128256 bf16; EAL+
                  "greedy reward 16 rollouts x 256 windows")
 MODE_T, W_G, W_S = 1.0, 0.5, 0.5
 WPR, RPG = 256, 16           # reward: windows per rollout, rollouts per group
-KERNELS_PER_STEP = 5         # row stats + window combine, backward, reward flags + groups
+KERNELS_PER_STEP = 5         # valid counts, fused forward + backward, window combine, reward flags + groups
 FALLBACK_HBM_GBS = 6800.0
 
 
@@ -181,8 +181,7 @@ def run_ours(args, ws_count, rank, local):
     adv = torch.empty(nroll, dtype=torch.float32, device=dev)
 
     def step(d, t):
-        aal.aal_loss_fwd(prob, d, t, None, ws, loss, None, stream)
-        aal.aal_loss_bwd(prob, d, t, None, ws, 1.0, grad, stream)
+        aal.aal_loss_fwd_bwd(prob, d, t, None, ws, 1.0, loss, grad, None, stream)
         aal.aal_accept_reward_from_loss(rprob, prob, ws, rws, tau, rl, adv, stream)
 
     for _ in range(args.warmup):
@@ -191,7 +190,7 @@ def run_ours(args, ws_count, rank, local):
     assert aal.aal_check_device_status(ws) == aal.AAL_OK
 
     # timed region: per-call events on the launching stream
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
     clocks = ClockSampler(local)
     clocks.start()
     time.sleep(0.3)
@@ -203,12 +202,10 @@ def run_ours(args, ws_count, rank, local):
     t_start.record(stream)
     for i in range(args.steps):
         ev[i][0].record(stream)
-        aal.aal_loss_fwd(prob, draft, target, None, ws, loss, None, stream)
+        aal.aal_loss_fwd_bwd(prob, draft, target, None, ws, 1.0, loss, grad, None, stream)
         ev[i][1].record(stream)
-        aal.aal_loss_bwd(prob, draft, target, None, ws, 1.0, grad, stream)
-        ev[i][2].record(stream)
         aal.aal_accept_reward_from_loss(rprob, prob, ws, rws, tau, rl, adv, stream)
-        ev[i][3].record(stream)
+        ev[i][2].record(stream)
     t_end.record(stream)
     torch.cuda.synchronize()
     if ws_count > 1:
@@ -216,12 +213,16 @@ def run_ours(args, ws_count, rank, local):
     clk = clocks.stop()
     ms_total = max_over_ranks(t_start.elapsed_time(t_end), ws_count, dev)
     ms_step = ms_total / args.steps
-    per = {"fwd": 0.0, "bwd": 0.0, "reward": 0.0}
+    per = {"fwd_bwd": 0.0, "reward": 0.0}
     for i in range(args.steps):
-        per["fwd"] += ev[i][0].elapsed_time(ev[i][1])
-        per["bwd"] += ev[i][1].elapsed_time(ev[i][2])
-        per["reward"] += ev[i][2].elapsed_time(ev[i][3])
+        per["fwd_bwd"] += ev[i][0].elapsed_time(ev[i][1])
+        per["reward"] += ev[i][1].elapsed_time(ev[i][2])
     per = {k: v / args.steps for k, v in per.items()}
+    # the same forward and backward as two calls (aal_loss_fwd, aal_loss_bwd), for comparison
+    reps2 = max(5, args.steps // 4)
+    fwd2, bwd2 = _time_fwd_bwd(
+        aal, lambda: aal.aal_loss_fwd(prob, draft, target, None, ws, loss, None, stream),
+        lambda: aal.aal_loss_bwd(prob, draft, target, None, ws, 1.0, grad, stream), stream, reps2)
     assert aal.aal_check_device_status(ws) == aal.AAL_OK
     loss_val = float(loss.item())
 
@@ -261,11 +262,13 @@ def run_ours(args, ws_count, rank, local):
     value = step_bytes * ws_count / (ms_step * 1e-3) / 1e9
     peak, peak_src = measured_peak()
 
-    # dominant kernel: the call with the largest share; its algorithmic bytes / its time
-    dom = max(("fwd", "bwd"), key=per.get)
-    dom_kernel = {"fwd": "rowstats_stream (aal_loss_fwd)", "bwd": "backward_kernel (aal_loss_bwd)"}[dom]
-    achieved = b[dom] / (per[dom] * 1e-3) / 1e9
-    traffic = recorded_traffic(dom)
+    # dominant kernel: the fused forward + backward (all but the reward's ~0.5% of the step).
+    # Algorithmic bytes per launch as counted for the metric (2 reads forward, 2 reads + 1 write
+    # backward); the fused kernel's own minimum traffic is 2 reads + 1 write, reported beside.
+    fb_bytes = b["fwd"] + b["bwd"]
+    min_traffic = 3 * R * V * draft.element_size()
+    achieved = fb_bytes / (per["fwd_bwd"] * 1e-3) / 1e9
+    traffic = recorded_traffic("fused")
 
     res = {
         "metric": "fused EAL/WTV fwd+bwd GB/s and logit-rows/s at V=128256 (with the GRPO acceptance reward)",
@@ -287,21 +290,30 @@ def run_ours(args, ws_count, rank, local):
                    "parallelism": f"replicas x{ws_count} (independent windows)"},
         "rows_per_s": round(R * ws_count / (ms_step * 1e-3), 1),
         "breakdown_ms": {k: round(v, 4) for k, v in per.items()},
-        "breakdown_gbs": {k: round(b[k] / (per[k] * 1e-3) / 1e9, 1) for k in ("fwd", "bwd")},
+        "two_call_step": {"note": "the same loss and gradient as aal_loss_fwd + aal_loss_bwd (bitwise equal)",
+                          "ms": round(fwd2 + bwd2, 4), "fwd_ms": round(fwd2, 4), "bwd_ms": round(bwd2, 4),
+                          "gbs": round(fb_bytes / ((fwd2 + bwd2) * 1e-3) / 1e9, 1),
+                          "fwd_gbs": round(b["fwd"] / (fwd2 * 1e-3) / 1e9, 1),
+                          "bwd_gbs": round(b["bwd"] / (bwd2 * 1e-3) / 1e9, 1)},
         "reward_sampled_draft": {"ms": round(ms_reward_sampled, 4),
                                  "gbs": round(2 * R * V * 2 / (ms_reward_sampled * 1e-3) / 1e9, 1),
                                  "note": "aal_accept_reward, AAL_SAMPLING | AAL_SAMPLED_DRAFT at T = 1"},
         "reward_logit_pass": {"ms": round(ms_reward_pass, 4),
                               "gbs": round(2 * R * V * 2 / (ms_reward_pass * 1e-3) / 1e9, 1),
                               "note": "aal_accept_reward streaming draft + target itself"},
-        "fwd_bwd_gbs": round((b["fwd"] + b["bwd"]) / ((per["fwd"] + per["bwd"]) * 1e-3) / 1e9, 1),
+        "fwd_bwd_gbs": round(fb_bytes / (per["fwd_bwd"] * 1e-3) / 1e9, 1),
         "frac_of_peak": round(value / ws_count / peak, 4),
         "loss": loss_val,
         "gpu_launches": KERNELS_PER_STEP * args.steps,
-        "roofline": {"bound": "hbm", "kernel": dom_kernel, "achieved": round(achieved, 1),
+        "roofline": {"bound": "hbm", "kernel": "fused_rows (aal_loss_fwd_bwd)", "achieved": round(achieved, 1),
                      "peak": peak, "peak_source": peak_src, "unit": "GB/s",
                      "frac": round(achieved / peak, 4), "traffic": traffic,
-                     "algorithmic_bytes": b[dom]},
+                     "algorithmic_bytes": fb_bytes,
+                     "min_traffic_bytes": min_traffic,
+                     "frac_of_min_traffic": round(min_traffic / (per["fwd_bwd"] * 1e-3) / 1e9 / peak, 4),
+                     "note": "algorithmic bytes count the forward (2 V b per row) and the backward (3 V b) as "
+                             "the metric does; the fused kernel reads each row from HBM once (3 V b per row "
+                             "with the gradient write), so frac_of_min_traffic is its DRAM utilisation"},
         "clocks": clk,
     }
     if greedy_obj is not None:
@@ -340,6 +352,21 @@ def _time_fwd_bwd(aal, fwd, bwd, stream, reps):
     return (sum(e[0].elapsed_time(e[1]) for e in ev) / reps, sum(e[1].elapsed_time(e[2]) for e in ev) / reps)
 
 
+def _time_call(fn, stream, reps):
+    """Mean milliseconds of ``fn`` over ``reps`` calls, events on the launching stream."""
+    for _ in range(3):
+        fn()
+    torch.cuda.synchronize()
+    a = torch.cuda.Event(enable_timing=True)
+    z = torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(reps):
+        fn()
+    z.record(stream)
+    torch.cuda.synchronize()
+    return a.elapsed_time(z) / reps
+
+
 def run_greedy_objective(aal, draft, target, grad, stream, reps):
     """The paper's greedy-regime objective L_KL + 0.1 L_EAL (Sec. 4.1) on the same batch:
     one pass over both rows forward (normalisers, x*, KL), target + draft read and the
@@ -351,15 +378,18 @@ def run_greedy_objective(aal, draft, target, grad, stream, reps):
     fwd, bwd = _time_fwd_bwd(
         aal, lambda: aal.aal_loss_fwd(prob, draft, target, None, ws, loss, None, stream),
         lambda: aal.aal_loss_bwd(prob, draft, target, None, ws, 1.0, grad, stream), stream, reps)
+    fused = _time_call(lambda: aal.aal_loss_fwd_bwd(prob, draft, target, None, ws, 1.0, loss, grad, None, stream),
+                       stream, reps)
     assert aal.aal_check_device_status(ws) == aal.AAL_OK
     R = N * K
     row = V * draft.element_size()
     fb, bb = 2 * R * row, 3 * R * row
     out = {"workload": f"v128k: N={N} windows, K={K}, V={V} bf16; L_KL + 0.1 L_EAL fwd+bwd",
-           "ms": round(fwd + bwd, 4), "fwd_ms": round(fwd, 4), "bwd_ms": round(bwd, 4),
-           "gbs": round((fb + bb) / ((fwd + bwd) * 1e-3) / 1e9, 1),
+           "ms": round(fused, 4), "gbs": round((fb + bb) / (fused * 1e-3) / 1e9, 1),
+           "rows_per_s": round(R / (fused * 1e-3), 1), "call": "aal_loss_fwd_bwd",
+           "two_call_ms": round(fwd + bwd, 4), "fwd_ms": round(fwd, 4), "bwd_ms": round(bwd, 4),
            "fwd_gbs": round(fb / (fwd * 1e-3) / 1e9, 1), "bwd_gbs": round(bb / (bwd * 1e-3) / 1e9, 1),
-           "rows_per_s": round(R / ((fwd + bwd) * 1e-3), 1), "loss": float(loss.item())}
+           "loss": float(loss.item())}
     del ws
     return out
 
@@ -585,8 +615,7 @@ def run_e2e(args, aal, prob, rprob, draft, target, grad, ws, loss, rws, tau, rl,
                 ready[b].record(copy_stream)
             stream.wait_event(ready[b])
             d_in, t_in = bufs[b][0], bufs[b][1]
-            aal.aal_loss_fwd(prob, d_in, t_in, None, ws, loss, None, stream)
-            aal.aal_loss_bwd(prob, d_in, t_in, None, ws, 1.0, grad, stream)
+            aal.aal_loss_fwd_bwd(prob, d_in, t_in, None, ws, 1.0, loss, grad, None, stream)
             aal.aal_accept_reward_from_loss(rprob, prob, ws, rws, tau, rl, adv, stream)
             free[b].record(stream)
             loss_h.copy_(loss, non_blocking=True)

@@ -13,6 +13,7 @@
 #pragma once
 
 #include "aal_internal.cuh"
+#include "ptx.cuh"
 
 namespace aal {
 
@@ -70,8 +71,12 @@ __device__ __forceinline__ void st_stream(uint4* p, const uint4& v) {
                : "memory");
 }
 
+// log2 q~_u = (z_q,u + nCq) s and log2 p~_u = (z_p,u + nCp) s with nC = -(M + Ls / s): the
+// same per-row constants, and the same comparison c_u = [z_q,u + nCq < z_p,u + nCp], as the
+// forward's overlap pass, so the gradient's c_u is the one the forward's Qlt summed over.
+// nCq1, nCp1: the same at T = 1 (s = log2 e) for q and p.
 struct RowCoef {
-  float sT, Mq, Lsq, Mp, Lsp, Mq1, Lsq1, Mp1, Lsp1;
+  float sT, nCq, nCp, nCq1, nCp1;
   float Ck;          // c^kl
   float cpos, cneg;  // g^s/T (1 - Qlt) and -g^s/T Qlt
   float Ag;          // g^g a^g
@@ -126,14 +131,10 @@ __device__ __forceinline__ bool row_coef(const BackwardArgs& a, float scale, flo
   const float ck = (KL && pos_valid) ? kscale : 0.f;
   if (gg == 0.f && gs == 0.f && ck == 0.f && cg == 0.f) return false;
   c.sT = a.sT;
-  c.Mq = SAMPLING ? st.Mq : 0.f;
-  c.Lsq = SAMPLING ? st.Lsq : 0.f;
-  c.Mp = SAMPLING ? st.Mp : 0.f;
-  c.Lsp = SAMPLING ? st.Lsp : 0.f;
-  c.Mq1 = (GREEDY || KL) ? st.Mq1 : 0.f;
-  c.Lsq1 = (GREEDY || KL) ? st.Lsq1 : 0.f;
-  c.Mp1 = KL ? st.Mp1 : 0.f;
-  c.Lsp1 = KL ? st.Lsp1 : 0.f;
+  c.nCq = SAMPLING ? -(st.Mq + st.Lsq / a.sT) : 0.f;
+  c.nCp = SAMPLING ? -(st.Mp + st.Lsp / a.sT) : 0.f;
+  c.nCq1 = (GREEDY || KL) ? -(st.Mq1 + st.Lsq1 / kLog2e) : 0.f;
+  c.nCp1 = KL ? -(st.Mp1 + st.Lsp1 / kLog2e) : 0.f;
   c.Ck = ck;
   const float qlt = SAMPLING ? st.qlt : 0.f;
   const float Bs = gs * a.invT;
@@ -149,19 +150,50 @@ __device__ __forceinline__ bool row_coef(const BackwardArgs& a, float scale, flo
 
 // Every term of element u except the greedy and GRPO spikes (+Ag at x*, +Cg at y), which
 // the callers add: once per 16-byte vector in the vector paths, per element in the scalar one.
+// (On the element's logits widened to fp32: the vector path below reaches the same values with
+// the bf16 widened inside the adds.)
 template <bool GREEDY, bool SAMPLING, bool Q1_IS_QT, bool KL>
 __device__ __forceinline__ float grad_elem(const RowCoef& c, float q, float p) {
   float d = 0.f, qt = 0.f;
   if (SAMPLING) {
-    const float lq = log2_prob(q, c.sT, c.Mq, c.Lsq);
-    const float lp = log2_prob(p, c.sT, c.Mp, c.Lsp);
-    qt = ex2(lq);
-    d = qt * (lq < lp ? c.cpos : c.cneg);
+    const float uq = q + c.nCq, up = p + c.nCp;
+    qt = ex2(uq * c.sT);
+    d = qt * (uq < up ? c.cpos : c.cneg);
   }
   if (GREEDY || KL) {
-    const float q1 = Q1_IS_QT ? qt : ex2(log2_prob(q, kLog2e, c.Mq1, c.Lsq1));
+    const float q1 = Q1_IS_QT ? qt : ex2((q + c.nCq1) * kLog2e);
     if (GREEDY) d = fmaf(-c.Aq, q1, d);
-    if (KL) d = fmaf(c.Ck, q1 - ex2(log2_prob(p, kLog2e, c.Mp1, c.Lsp1)), d);
+    if (KL) d = fmaf(c.Ck, q1 - ex2((p + c.nCp1) * kLog2e), d);
+  }
+  return d;
+}
+
+// grad_elem on the two bf16 halves of a word of z_q (qw) and of z_p (pw): each widened inside
+// a mixed-precision add, the scalings on fp32 pairs.  Bitwise the same as grad_elem on the
+// widened values (the widening is exact, and x * s is one rounding either way).
+template <bool GREEDY, bool SAMPLING, bool Q1_IS_QT, bool KL>
+__device__ __forceinline__ float2 grad_pair_bf16(const RowCoef& c, uint32_t qw, uint32_t pw) {
+  float2 d = make_float2(0.f, 0.f), qt = make_float2(0.f, 0.f);
+  if (SAMPLING) {
+    const float uq0 = bf16lo_add(qw, c.nCq), uq1 = bf16hi_add(qw, c.nCq);
+    const float up0 = bf16lo_add(pw, c.nCp), up1 = bf16hi_add(pw, c.nCp);
+    const float2 x = ptx::f2fma(make_float2(uq0, uq1), make_float2(c.sT, c.sT), make_float2(0.f, 0.f));
+    qt = make_float2(ex2(x.x), ex2(x.y));
+    d = make_float2(qt.x * (uq0 < up0 ? c.cpos : c.cneg), qt.y * (uq1 < up1 ? c.cpos : c.cneg));
+  }
+  if (GREEDY || KL) {
+    float2 q1 = qt;
+    if (!Q1_IS_QT) {
+      const float2 x = ptx::f2fma(make_float2(bf16lo_add(qw, c.nCq1), bf16hi_add(qw, c.nCq1)),
+                                  make_float2(kLog2e, kLog2e), make_float2(0.f, 0.f));
+      q1 = make_float2(ex2(x.x), ex2(x.y));
+    }
+    if (GREEDY) d = make_float2(fmaf(-c.Aq, q1.x, d.x), fmaf(-c.Aq, q1.y, d.y));
+    if (KL) {
+      const float2 x = ptx::f2fma(make_float2(bf16lo_add(pw, c.nCp1), bf16hi_add(pw, c.nCp1)),
+                                  make_float2(kLog2e, kLog2e), make_float2(0.f, 0.f));
+      d = make_float2(fmaf(c.Ck, q1.x - ex2(x.x), d.x), fmaf(c.Ck, q1.y - ex2(x.y), d.y));
+    }
   }
   return d;
 }
@@ -173,11 +205,23 @@ __device__ __forceinline__ uint4 grad_vec(const RowCoef& c, const uint4& qw, con
                                           int64_t xv, int xe, int64_t yv, int ye) {
   constexpr int E = Io<T>::E;
   constexpr bool READ_P = SAMPLING || KL;
-  float qv[E], pv[E], d[E];
-  Io<T>::unpack(qw, qv);
-  if (READ_P) Io<T>::unpack(pw, pv);
+  float d[E];
+  if constexpr (sizeof(T) == 2) {
+    const uint32_t qa[4] = {qw.x, qw.y, qw.z, qw.w};
+    const uint32_t pa[4] = {pw.x, pw.y, pw.z, pw.w};
 #pragma unroll
-  for (int e = 0; e < E; ++e) d[e] = grad_elem<GREEDY, SAMPLING, Q1_IS_QT, KL>(c, qv[e], READ_P ? pv[e] : 0.f);
+    for (int k = 0; k < 4; ++k) {
+      const float2 dd = grad_pair_bf16<GREEDY, SAMPLING, Q1_IS_QT, KL>(c, qa[k], READ_P ? pa[k] : 0u);
+      d[2 * k] = dd.x;
+      d[2 * k + 1] = dd.y;
+    }
+  } else {
+    float qv[E], pv[E];
+    Io<T>::unpack(qw, qv);
+    if (READ_P) Io<T>::unpack(pw, pv);
+#pragma unroll
+    for (int e = 0; e < E; ++e) d[e] = grad_elem<GREEDY, SAMPLING, Q1_IS_QT, KL>(c, qv[e], READ_P ? pv[e] : 0.f);
+  }
   if (GREEDY) {  // the spikes, tested once per vector
     if (i == xv) {
 #pragma unroll
