@@ -707,7 +707,8 @@ def main():
 
 
 def recorded_traffic(which):
-    """DRAM bytes per launch from the committed ncu summary, if the kernel is unchanged since."""
+    """DRAM bytes per launch from the committed ncu summary, if none of the kernel's sources has
+    changed since."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
@@ -716,12 +717,20 @@ def recorded_traffic(which):
         return None
     if not rec:
         return None
-    src = os.path.join(ROOT, "paper_2609_24150_gb300", "csrc", rec["source"])
+    sha = sources_sha(rec["sources"])
+    return rec["dram_bytes_per_launch"] if sha is not None and sha == rec["sources_sha256_16"] else None
+
+
+def sources_sha(names):
+    """First 16 hex digits of the SHA-256 of the named csrc files, concatenated in order."""
+    h = hashlib.sha256()
     try:
-        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        for n in names:
+            with open(os.path.join(ROOT, "paper_2609_24150_gb300", "csrc", n), "rb") as f:
+                h.update(f.read())
     except OSError:
         return None
-    return rec["dram_bytes_per_launch"] if sha == rec["source_sha256_16"] else None
+    return h.hexdigest()[:16]
 
 
 if __name__ == "__main__":
