@@ -467,6 +467,10 @@ cudaError_t go_fused(const FusedArgs& f0, cudaStream_t s, uint64_t limit_ns, boo
   const int nch = (int)((f.st.V + kHalfSlot / elt - 1) / (kHalfSlot / elt));
   void* args[] = {&f, (void*)&nch, &limit_ns};
   e = cudaLaunchCooperativeKernel((const void*)kern, dim3((unsigned)(G * K)), dim3(kThreads), args, kFusedSmemBytes, s);
+  if (e == cudaErrorCooperativeLaunchTooLarge) {  // fewer SMs available than the device has (shared
+    cudaGetLastError();                           // device): the caller runs the two calls instead
+    return cudaSuccess;
+  }
   if (e == cudaSuccess) *launched = true;
   return e;
 }

@@ -5,7 +5,7 @@ by aal_loss_bwd bit for bit: on the fused path (bf16 rows of 16-byte multiples; 
 combination it instantiates, masks, fewer windows than CTA groups, K = 1 and K = 8, full-size
 rows) and on the problems it hands to the two calls (fp32, unaligned rows, token ids, the
 anchor beside the sampling term at T != 1).  A few cases are also checked against the oracle
-directly, and the group barrier's bounded wait is driven to a timeout without a fault.
+directly, and the bounded waits are driven to a timeout without a fault.
 """
 
 import pytest
@@ -123,7 +123,8 @@ def test_fused_against_the_oracle(mode, T, wg, ws):
 
 def test_group_barrier_and_ring_time_out_and_context_stays_usable():
     """One ring copy of every CTA is left unarmed: its waits run out (50 ms), the CTAs that gave
-    up still add their group arrivals, and the call returns with AAL_ERR_TIMEOUT recorded."""
+    up still publish their rows' mailbox words (so no window's exchange waits the whole limit),
+    and the call returns with AAL_ERR_TIMEOUT recorded."""
     t, d, _ = _inputs(16, 2, 20000, seed=11)
     prob = aal.loss_problem(d, B, 1.0, 0.5, 0.5)
     ws = torch.empty(aal.aal_workspace_size(prob), dtype=torch.uint8, device=DEV)
@@ -147,4 +148,12 @@ def test_v128k_full_size_fused_equals_two_calls():
     del f, s
     f = FusedRun(t, d, None, KL | G, 1.0, 0.1, 0.0)
     s = LossRun(t, d, None, KL | G, 1.0, 0.1, 0.0)
+    assert_same(f, s)
+
+
+def test_v152k_full_size_fused_equals_two_calls():
+    """K = 6 (25 groups of 6 CTAs), V = 151936, low-overlap rows, WTV at T = 1.5."""
+    t, d, _ = synth.make_logits("v152k", seed=0, device=DEV)
+    f = FusedRun(t, d, None, S, 1.5, 0.0, 1.0)
+    s = LossRun(t, d, None, S, 1.5, 0.0, 1.0)
     assert_same(f, s)
