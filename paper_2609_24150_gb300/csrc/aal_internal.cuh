@@ -453,22 +453,23 @@ __device__ __forceinline__ float lg2(float x) {
 // S_j = 1 + a_{j+1} S_{j+1} (0 for j >= kn).  Shared by the window kernels and the fused
 // forward + backward, so both give bitwise the same partials.
 __device__ __forceinline__ float window_term(const float* a, int kn, float* dE) {
+  // every rounding spelled out (no contraction), so that every kernel forms the same bits
   float P[AAL_MAX_K + 1];
   P[0] = 1.f;
   float E = 0.f;
 #pragma unroll
   for (int j = 0; j < AAL_MAX_K; ++j) {
     if (j < kn) {
-      P[j + 1] = P[j] * a[j];
-      E += P[j + 1];
+      P[j + 1] = __fmul_rn(P[j], a[j]);
+      E = __fadd_rn(E, P[j + 1]);
     }
   }
   float S = 1.f;
 #pragma unroll
   for (int j = AAL_MAX_K - 1; j >= 0; --j) {
     if (j < kn) {
-      dE[j] = P[j] * S;
-      S = 1.f + a[j] * S;
+      dE[j] = __fmul_rn(P[j], S);
+      S = __fmaf_rn(a[j], S, 1.f);
     } else {
       dE[j] = 0.f;
     }

@@ -72,11 +72,12 @@ template <typename T, bool VEC, bool G, bool S, bool Q, bool KL>
 __global__ void __launch_bounds__(kBwdThreads) backward_kernel(BackwardArgs a) {
   backward_rows<T, VEC, G, S, Q, KL>(a);
 }
-// The anchor's bf16 vector instances (two exponentials an element) are held to 40
-// registers, six blocks an SM, for enough loads in flight (unbounded they took 48, five
-// blocks); the others fit six or more unbounded, and fp32 ones would spill at 40.
+// The anchor's bf16 vector instances (two exponentials an element) are bounded for enough
+// loads in flight: six blocks an SM (40 registers) without the sampling term (unbounded they
+// took 48, five blocks), five with it (at 40 registers they spilled; measured 6.47 against
+// 6.50 ms); the others fit six or more unbounded, and fp32 ones would spill at 40.
 template <typename T, bool G, bool S, bool Q>
-__global__ void __launch_bounds__(kBwdThreads, 6) backward_kernel_kl(BackwardArgs a) {
+__global__ void __launch_bounds__(kBwdThreads, S ? 5 : 6) backward_kernel_kl(BackwardArgs a) {
   backward_rows<T, true, G, S, Q, true>(a);
 }
 

@@ -365,7 +365,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
             if (ov) {
               if (f.win.sampling) window_term(asv, kn, dE);
               const float tvc = (f.win.tv && kn > 0) ? f.win.w_tv / (float)kn : 0.f;
-              dEs = (f.win.sampling ? f.win.w_sampling * dE[k] : 0.f) + (k < kn ? tvc : 0.f);
+              dEs = __fadd_rn(f.win.sampling ? __fmul_rn(f.win.w_sampling, dE[k]) : 0.f, k < kn ? tvc : 0.f);
             }
             const bool with_greedy = GREEDY && f.bw.w_greedy != 0.f;
             const bool pos_valid = f.bw.mask == nullptr || f.bw.mask[r] != 0;

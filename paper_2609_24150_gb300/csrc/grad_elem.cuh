@@ -82,6 +82,8 @@ struct RowCoef {
   float Ag;          // g^g a^g
   float Cg;          // c^grpo
   float Aq;          // Ag + Cg, the coefficient of -q(u)
+  float q1c;         // Ck - Aq: the coefficient of q(u) in every term but the sampling one
+  float cposq, cnegq;  // cpos + q1c, cneg + q1c: with q = q~ (T = 1) the element's whole q~ factor
   int32_t xs, ys;
 };
 
@@ -125,24 +127,29 @@ __device__ __forceinline__ RowStat load_row_stat(const LossWs& ws, int64_t r, bo
 template <bool GREEDY, bool SAMPLING, bool KL>
 __device__ __forceinline__ bool row_coef(const BackwardArgs& a, float scale, float kscale, float dEg, float dEs,
                                          float cgr, bool pos_valid, const RowStat& st, RowCoef& c) {
-  const float gg = (GREEDY && a.w_greedy != 0.f) ? scale * a.w_greedy * dEg : 0.f;
-  const float cg = (GREEDY && a.grpo) ? a.dloss * cgr : 0.f;
-  const float gs = SAMPLING ? scale * a.w_sampling * dEs : 0.f;
+  // every rounding spelled out (no contraction into fused multiply-adds), so that each kernel
+  // that includes this forms the same bits
+  const float gg = (GREEDY && a.w_greedy != 0.f) ? __fmul_rn(__fmul_rn(scale, a.w_greedy), dEg) : 0.f;
+  const float cg = (GREEDY && a.grpo) ? __fmul_rn(a.dloss, cgr) : 0.f;
+  const float gs = SAMPLING ? __fmul_rn(__fmul_rn(scale, a.w_sampling), dEs) : 0.f;
   const float ck = (KL && pos_valid) ? kscale : 0.f;
   if (gg == 0.f && gs == 0.f && ck == 0.f && cg == 0.f) return false;
   c.sT = a.sT;
-  c.nCq = SAMPLING ? -(st.Mq + st.Lsq / a.sT) : 0.f;
-  c.nCp = SAMPLING ? -(st.Mp + st.Lsp / a.sT) : 0.f;
-  c.nCq1 = (GREEDY || KL) ? -(st.Mq1 + st.Lsq1 / kLog2e) : 0.f;
-  c.nCp1 = KL ? -(st.Mp1 + st.Lsp1 / kLog2e) : 0.f;
+  c.nCq = SAMPLING ? -__fadd_rn(st.Mq, __fdiv_rn(st.Lsq, a.sT)) : 0.f;
+  c.nCp = SAMPLING ? -__fadd_rn(st.Mp, __fdiv_rn(st.Lsp, a.sT)) : 0.f;
+  c.nCq1 = (GREEDY || KL) ? -__fadd_rn(st.Mq1, __fdiv_rn(st.Lsq1, kLog2e)) : 0.f;
+  c.nCp1 = KL ? -__fadd_rn(st.Mp1, __fdiv_rn(st.Lsp1, kLog2e)) : 0.f;
   c.Ck = ck;
   const float qlt = SAMPLING ? st.qlt : 0.f;
-  const float Bs = gs * a.invT;
-  c.cpos = Bs * (1.f - qlt);
-  c.cneg = -Bs * qlt;
-  c.Ag = gg != 0.f ? gg * st.ag : 0.f;
+  const float Bs = __fmul_rn(gs, a.invT);
+  c.cpos = __fmul_rn(Bs, __fsub_rn(1.f, qlt));
+  c.cneg = -__fmul_rn(Bs, qlt);
+  c.Ag = gg != 0.f ? __fmul_rn(gg, st.ag) : 0.f;
   c.Cg = cg;
-  c.Aq = c.Ag + c.Cg;
+  c.Aq = __fadd_rn(c.Ag, c.Cg);
+  c.q1c = __fsub_rn(c.Ck, c.Aq);
+  c.cposq = __fadd_rn(c.cpos, c.q1c);
+  c.cnegq = __fadd_rn(c.cneg, c.q1c);
   c.xs = gg != 0.f ? st.xs : -1;
   c.ys = cg != 0.f ? st.ys : -1;
   return true;
@@ -152,48 +159,45 @@ __device__ __forceinline__ bool row_coef(const BackwardArgs& a, float scale, flo
 // the callers add: once per 16-byte vector in the vector paths, per element in the scalar one.
 // (On the element's logits widened to fp32: the vector path below reaches the same values with
 // the bf16 widened inside the adds.)
+// The terms are grouped by exponential: q~(u) (c_u ? cpos : cneg) + q(u) (Ck - Aq) - Ck p(u),
+// and with q = q~ the first two share one factor, q~(u) (c_u ? cposq : cnegq).
 template <bool GREEDY, bool SAMPLING, bool Q1_IS_QT, bool KL>
 __device__ __forceinline__ float grad_elem(const RowCoef& c, float q, float p) {
-  float d = 0.f, qt = 0.f;
+  float d = 0.f;
   if (SAMPLING) {
     const float uq = q + c.nCq, up = p + c.nCp;
-    qt = ex2(uq * c.sT);
-    d = qt * (uq < up ? c.cpos : c.cneg);
+    const float qt = ex2(uq * c.sT);
+    if (Q1_IS_QT) d = qt * (uq < up ? c.cposq : c.cnegq);
+    else d = qt * (uq < up ? c.cpos : c.cneg);
   }
-  if (GREEDY || KL) {
-    const float q1 = Q1_IS_QT ? qt : ex2((q + c.nCq1) * kLog2e);
-    if (GREEDY) d = fmaf(-c.Aq, q1, d);
-    if (KL) d = fmaf(c.Ck, q1 - ex2((p + c.nCp1) * kLog2e), d);
-  }
+  if ((GREEDY || KL) && !(SAMPLING && Q1_IS_QT)) d = fmaf(ex2((q + c.nCq1) * kLog2e), c.q1c, d);
+  if (KL) d = fmaf(ex2((p + c.nCp1) * kLog2e), -c.Ck, d);
   return d;
 }
 
 // grad_elem on the two bf16 halves of a word of z_q (qw) and of z_p (pw): each widened inside
-// a mixed-precision add, the scalings on fp32 pairs.  Bitwise the same as grad_elem on the
-// widened values (the widening is exact, and x * s is one rounding either way).
+// a mixed-precision add, the products and sums on fp32 pairs.  The same values as grad_elem on
+// the widened logits (the widening is exact and every product or fused add is one rounding
+// either way), up to the sign of an exact zero.
 template <bool GREEDY, bool SAMPLING, bool Q1_IS_QT, bool KL>
 __device__ __forceinline__ float2 grad_pair_bf16(const RowCoef& c, uint32_t qw, uint32_t pw) {
-  float2 d = make_float2(0.f, 0.f), qt = make_float2(0.f, 0.f);
+  const float2 zero2 = make_float2(0.f, 0.f), l2e2 = make_float2(kLog2e, kLog2e);
+  float2 d = zero2;
   if (SAMPLING) {
     const float uq0 = bf16lo_add(qw, c.nCq), uq1 = bf16hi_add(qw, c.nCq);
     const float up0 = bf16lo_add(pw, c.nCp), up1 = bf16hi_add(pw, c.nCp);
-    const float2 x = ptx::f2fma(make_float2(uq0, uq1), make_float2(c.sT, c.sT), make_float2(0.f, 0.f));
-    qt = make_float2(ex2(x.x), ex2(x.y));
-    d = make_float2(qt.x * (uq0 < up0 ? c.cpos : c.cneg), qt.y * (uq1 < up1 ? c.cpos : c.cneg));
+    const float2 x = ptx::f2fma(make_float2(uq0, uq1), make_float2(c.sT, c.sT), zero2);
+    const float2 qt = make_float2(ex2(x.x), ex2(x.y));
+    const float a = Q1_IS_QT ? c.cposq : c.cpos, b = Q1_IS_QT ? c.cnegq : c.cneg;
+    d = ptx::f2fma(qt, make_float2(uq0 < up0 ? a : b, uq1 < up1 ? a : b), zero2);
   }
-  if (GREEDY || KL) {
-    float2 q1 = qt;
-    if (!Q1_IS_QT) {
-      const float2 x = ptx::f2fma(make_float2(bf16lo_add(qw, c.nCq1), bf16hi_add(qw, c.nCq1)),
-                                  make_float2(kLog2e, kLog2e), make_float2(0.f, 0.f));
-      q1 = make_float2(ex2(x.x), ex2(x.y));
-    }
-    if (GREEDY) d = make_float2(fmaf(-c.Aq, q1.x, d.x), fmaf(-c.Aq, q1.y, d.y));
-    if (KL) {
-      const float2 x = ptx::f2fma(make_float2(bf16lo_add(pw, c.nCp1), bf16hi_add(pw, c.nCp1)),
-                                  make_float2(kLog2e, kLog2e), make_float2(0.f, 0.f));
-      d = make_float2(fmaf(c.Ck, q1.x - ex2(x.x), d.x), fmaf(c.Ck, q1.y - ex2(x.y), d.y));
-    }
+  if ((GREEDY || KL) && !(SAMPLING && Q1_IS_QT)) {
+    const float2 x = ptx::f2fma(make_float2(bf16lo_add(qw, c.nCq1), bf16hi_add(qw, c.nCq1)), l2e2, zero2);
+    d = ptx::f2fma(make_float2(ex2(x.x), ex2(x.y)), make_float2(c.q1c, c.q1c), d);
+  }
+  if (KL) {
+    const float2 x = ptx::f2fma(make_float2(bf16lo_add(pw, c.nCp1), bf16hi_add(pw, c.nCp1)), l2e2, zero2);
+    d = ptx::f2fma(make_float2(ex2(x.x), ex2(x.y)), make_float2(-c.Ck, -c.Ck), d);
   }
   return d;
 }

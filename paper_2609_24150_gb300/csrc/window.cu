@@ -137,7 +137,7 @@ __global__ void __launch_bounds__(kWindowThreads) window_kernel(WindowArgs a) {
       float tsum = 0.f;
 #pragma unroll
       for (int j = 0; j < AAL_MAX_K; ++j) {
-        if (j < K) a.ws.dEs[r0 + j] = (a.sampling ? a.w_sampling * dE[j] : 0.f) + (j < kn ? tvc : 0.f);
+        if (j < K) a.ws.dEs[r0 + j] = __fadd_rn(a.sampling ? __fmul_rn(a.w_sampling, dE[j]) : 0.f, j < kn ? tvc : 0.f);
         if (j < kn) tsum += 1.f - as[j];
       }
       if (a.tv && kn > 0) tvs = tsum / (float)kn;
@@ -226,7 +226,7 @@ __global__ void __launch_bounds__(kWindowThreads) seq_window_kernel(SeqWindowArg
       float tsum = 0.f;
 #pragma unroll
       for (int j = 0; j < AAL_MAX_K; ++j) {
-        if (j < K) a.ps[n * K + j] = (a.sampling ? a.w_sampling * dE[j] : 0.f) + (j < kn ? tvc : 0.f);
+        if (j < K) a.ps[n * K + j] = __fadd_rn(a.sampling ? __fmul_rn(a.w_sampling, dE[j]) : 0.f, j < kn ? tvc : 0.f);
         if (j < kn) tsum += 1.f - as[j];
       }
       if (a.tv && kn > 0) tvs = tsum / (float)kn;
