@@ -301,11 +301,37 @@ aal_status aal_loss_fwd_bwd(const aal_problem* prob, const void* draft, const vo
   const LossLayout L = loss_layout(prob->N, prob->K);
   if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < L.total) return AAL_ERR_WORKSPACE;
 
-  // the fused kernel: bf16 rows of 16-byte multiples, both logit tensors, and (as for the
-  // streamed forward) the anchor beside a sampling term only at T = 1
+  // the fused kernels: bf16 rows of 16-byte multiples; with logits, (as for the streamed
+  // forward) the anchor beside a sampling term only at T = 1; with token ids, the draft alone
   const bool sampling = (prob->mode & (AAL_SAMPLING | AAL_TV)) != 0, kl = (prob->mode & AAL_KL) != 0;
-  const bool fusable = prob->dtype == AAL_BF16 && !(prob->mode & AAL_IDS) && (prob->V * 2) % 16 == 0 &&
-                       !(kl && sampling && prob->temperature != 1.0f);
+  const bool ids = (prob->mode & AAL_IDS) != 0;
+  const bool rows16 = prob->dtype == AAL_BF16 && (prob->V * 2) % 16 == 0;
+  const bool fusable = rows16 && !ids && !(kl && sampling && prob->temperature != 1.0f);
+  if (rows16 && ids) {
+    LossWs ws = loss_ws(workspace, L);
+    if (cudaMemsetAsync(ws.hdr, 0, sizeof(WsHeader), s) != cudaSuccess) return AAL_ERR_CUDA;
+    if (cudaMemsetAsync(ws.mbox, 0xff, (size_t)L.R * 8, s) != cudaSuccess) return AAL_ERR_CUDA;  // kMboxEmpty
+    if (launch_count_valid(mask, prob->N, (int32_t)prob->K, ws.hdr, s) != cudaSuccess) return AAL_ERR_CUDA;
+    FusedIdsArgs f;
+    f.st.z = draft;
+    f.st.R = L.R;
+    f.st.V = prob->V;
+    f.st.lws = ws;
+    f.st.ids = static_cast<const int32_t*>(target);
+    f.st.acc = nullptr;
+    f.st.acc_ref = nullptr;
+    f.st.lpr = nullptr;
+    f.st.hdr = ws.hdr;
+    f.st.skip_chunk = debug_take_skip_chunk();
+    f.bw = grad_args(draft, target, mask, L.R, prob->V, prob->mode, prob->temperature, prob->w_greedy,
+                     prob->w_kl, dloss, ws, grad_draft);
+    f.win = window_args(prob, mask, 1, loss, eal, ws, L.nwblk);
+    f.groups = 0;
+    const uint64_t limit = debug_wait_limit_ns();
+    bool launched = false;
+    if (launch_fused_ids(f, s, limit ? limit : kWaitLimitNs, &launched) != cudaSuccess) return AAL_ERR_CUDA;
+    if (launched) return cuda_status(launch_window(f.win, s));
+  }
   if (fusable) {
     LossWs ws = loss_ws(workspace, L);
     if (cudaMemsetAsync(ws.hdr, 0, sizeof(WsHeader), s) != cudaSuccess) return AAL_ERR_CUDA;

@@ -346,6 +346,15 @@ struct Stream1Args {
   int64_t skip_chunk;  // failure-detection test hook: a chunk whose copy is never armed (-1: none)
 };
 
+// The fused forward + backward with x* as token ids (aal_loss_fwd_bwd, mode AAL_GREEDY |
+// AAL_IDS): only the draft is streamed; groups of K CTAs as in FusedArgs.
+struct FusedIdsArgs {
+  Stream1Args st;    // the draft's statistics pass (z = draft, ids, workspace, test hook)
+  BackwardArgs bw;   // the gradient pass
+  WindowArgs win;    // the window terms
+  int32_t groups;    // G
+};
+
 // GRPO over sequences (aal_seq_grpo_from_loss): per-position flags and log pi_ref from the
 // reference pass, the windows' rows gathered from them, and the windows' coefficients before
 // they are added per position.
@@ -428,6 +437,8 @@ cudaError_t launch_count_valid(const uint8_t* mask, int64_t N, int32_t K, WsHead
 // Launches the fused forward + backward when the problem's flags have an instantiation and the
 // device can hold at least one group; *launched tells whether it did.
 cudaError_t launch_fused(const FusedArgs& f, cudaStream_t s, uint64_t limit_ns, bool* launched);
+// The same for token ids (then resolve_draft_argmax places the draft's greedy token).
+cudaError_t launch_fused_ids(const FusedIdsArgs& f, cudaStream_t s, uint64_t limit_ns, bool* launched);
 
 // ---------------------------------------------------------------------------
 // Device helpers.

@@ -10,6 +10,7 @@
 //
 // Rows whose byte length is a multiple of 16 are streamed through a shared-memory ring by
 // TMA (one_tensor_stream); the others take a plain per-row loop (one_tensor_rows).
+#include "grad_elem.cuh"
 #include "ptx.cuh"
 
 namespace aal {
@@ -475,7 +476,285 @@ cudaError_t launch_T(const Stream1Args& a, bool ids, cudaStream_t s) {
   return cudaGetLastError();
 }
 
+// ---------------------------------------------------------------- fused forward + backward, ids
+// aal_loss_fwd_bwd with x* as token ids: the K rows of a window held by K CTAs (one cooperative
+// launch, one CTA per SM), each row streamed from HBM for the draft's statistics (kept in L2),
+// its a^greedy exchanged through the per-row mailbox as in fused.cu, and streamed again from L2
+// for the gradient -dloss/|W| w_g dE/da a^g (delta_{u,x*} - q(u)).  Statistics, exchange and
+// coefficients reuse the IDS stream's and the backward's code, so the results are bitwise those
+// of aal_loss_fwd + aal_loss_bwd; resolve_draft_argmax and the window kernel run after it.
+constexpr int kRBarCoef = 3;
+
+struct FusedIdsSmem {
+  RefSmem s;
+  RowCoef coef;
+  int32_t live;
+};
+
+constexpr size_t kFIdsSmemBytes = (size_t)kRSlots * kRSlotBytes + sizeof(FusedIdsSmem);
+
+__global__ void __launch_bounds__(kRThreads, 1) fused_ids_rows(FusedIdsArgs f, int nch, uint64_t limit_ns) {
+  using T = uint16_t;
+  constexpr int E = 8;
+  constexpr int CH = kRSlotBytes / 2;  // elements per chunk
+  extern __shared__ __align__(1024) unsigned char smem[];
+  unsigned char* ring = smem;
+  FusedIdsSmem& F = *reinterpret_cast<FusedIdsSmem*>(smem + kRSlots * kRSlotBytes);
+  RefSmem& S = F.s;
+  const Stream1Args& a = f.st;
+  WsHeader* hdr = a.hdr;
+  volatile int* abort_flag = &S.abort_flag;
+  const int V = (int)a.V;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int K = f.win.K;
+  const int64_t N = f.win.N;
+  const int G = f.groups;
+  const int g = blockIdx.x / K, k = blockIdx.x % K;
+
+  if (threadIdx.x == 0) {
+    for (int q = 0; q < kRSlots; ++q) {
+      mbar_init(&S.full[q], 1);
+      mbar_init(&S.empty[q], kRWarps);
+    }
+    S.abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+
+  if (warp == kRWarps) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      const uint64_t keep = policy_evict_last(), drop = policy_evict_first();
+      int slot = 0;
+      uint32_t phase = 0, armed = 0, last_phase = 0;
+      int64_t seq = 0;
+      for (int64_t n = g; n < N && !*abort_flag; n += G) {
+        const char* row = static_cast<const char*>(a.z) + (n * K + k) * a.V * 2;
+        for (int pass = 0; pass < 2 && !*abort_flag; ++pass) {  // statistics (kept in L2), gradient
+          const uint64_t pol = pass == 0 ? keep : drop;
+          for (int c = 0; c < nch; ++c, ++seq) {
+            if (!wait_phase(&S.empty[slot], phase ^ 1u, abort_flag, limit_ns, hdr)) break;
+            const int e0 = c * CH;
+            const uint32_t bytes = (uint32_t)(min(CH, V - e0) * 2);
+            if (seq != a.skip_chunk) {  // (the test hook leaves one chunk's barrier unarmed)
+              mbar_expect_tx(&S.full[slot], bytes);
+              bulk_load(ring + slot * kRSlotBytes, row + (int64_t)e0 * 2, bytes, &S.full[slot], pol);
+              armed |= 1u << slot;
+              last_phase = (last_phase & ~(1u << slot)) | (phase << slot);
+            }
+            if (++slot == kRSlots) {
+              slot = 0;
+              phase ^= 1u;
+            }
+          }
+        }
+      }
+      for (int q = 0; q < kRSlots; ++q) {
+        if (!(armed & (1u << q))) continue;
+        const uint32_t ph = (last_phase >> q) & 1u;
+        const uint64_t t0 = now_ns();
+        for (uint32_t it = 0; it < kSpinLimit && !mbar_try(&S.full[q], ph, 100000); ++it)
+          if (now_ns() - t0 > limit_ns) break;
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ consumers
+    const int t = threadIdx.x;
+    int slot = 0;
+    uint32_t phase = 0, j = 0;
+    float scale = 0.f;  // thread 0: -dloss / |W|
+    if (t == 0) {
+      const int nvalid = hdr->nvalid;
+      scale = nvalid > 0 ? -f.bw.dloss / (float)nvalid : 0.f;
+    }
+    for (int64_t n = g; n < N; n += G, ++j) {
+      const int64_t r = n * K + k;
+      const int32_t xs = a.ids[r];
+      const bool x_ok = xs >= 0 && xs < V;
+      const int cx = x_ok ? xs / CH : -1, ix = x_ok ? (xs - cx * CH) / E : 0, ex = x_ok ? xs % E : 0;
+      // ---- pass 1: the draft's normaliser and greedy token (HBM)
+      RefPart A;
+      refpart_init(A);
+      for (int c = 0; c < nch; ++c) {
+        if (wait_full(&S.full[slot], phase, abort_flag, limit_ns, hdr)) {
+          const int e0 = c * CH;
+          const uint4* Z = reinterpret_cast<const uint4*>(ring + slot * kRSlotBytes);
+          if (e0 + CH <= V) {
+            uint4 w[kRNV];
+#pragma unroll
+            for (int v = 0; v < kRNV; ++v) w[v] = Z[t + v * kRConsumers];
+#pragma unroll
+            for (int v = 0; v < kRNV; ++v) ref_vec<T>(A, w[v], e0 + (t + v * kRConsumers) * E);
+          } else {
+            const int nvec = (V - e0) / E;
+            for (int i = t; i < nvec; i += kRConsumers) ref_vec<T>(A, Z[i], e0 + i * E);
+          }
+          if (c == cx && t == ix % kRConsumers) S.zx[j & 1] = ref_elem<T>(Z[ix], ex);
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&S.empty[slot]);
+        if (++slot == kRSlots) {
+          slot = 0;
+          phase ^= 1u;
+        }
+      }
+      refpart_warp(A);
+      if (lane == 0) S.red[j & 1][warp] = A;
+      named_barrier(kRBarRow, kRConsumers);
+      RowStat st{};  // thread 0: what the row's coefficients need
+      if (t == 0) {
+        RefPart tot = S.red[j & 1][0];
+        for (int w = 1; w < kRWarps; ++w) {
+          const RefPart b = S.red[j & 1][w];
+          const float m = fmaxf(tot.M, b.M);
+          tot.S = tot.S * ex2((tot.M - m) * kLog2e) + b.S * ex2((b.M - m) * kLog2e);
+          tot.M = m;
+          if (b.av > tot.av || (b.av == tot.av && b.ab < tot.ab)) {
+            tot.av = b.av;
+            tot.ab = b.ab;
+          }
+        }
+        const float zx = x_ok ? S.zx[j & 1] : -INFINITY;
+        if (!*abort_flag) row_outputs<true>(a, r, tot.M, tot.S, tot.ab, false, -INFINITY, zx, false);
+        // the same values row_outputs wrote, as the backward reads them
+        const float Ls = log2f(tot.S);
+        st.Mq1 = tot.M;
+        st.Lsq1 = Ls;
+        st.ag = x_ok ? exp2f(log2_prob(zx, kLog2e, tot.M, Ls)) : 0.f;
+        st.xs = x_ok ? xs : -1;
+      }
+      // ---- the window's a^greedy (warp 0: lane j polls depth j), the row's coefficients (thread 0)
+      if (warp == 0) {
+        const int64_t r0 = n * K;
+        if (lane == 0) {
+          uint64_t word = __float_as_uint(st.ag);
+          if (word == kMboxEmpty) word = 0;
+          st_relaxed(&a.lws.mbox[r], word);
+        }
+        bool ok = __shfl_sync(0xffffffffu, *abort_flag == 0 ? 1 : 0, 0) != 0;
+        uint64_t w = 0;
+        if (ok) {
+          const uint64_t t0 = now_ns();
+          for (uint32_t it = 0;; ++it) {
+            if (lane < K) w = ld_relaxed(&a.lws.mbox[r0 + lane]);
+            if (__all_sync(0xffffffffu, lane >= K || w != kMboxEmpty)) break;
+            int quit = 0;
+            if (lane == 0 && (*abort_flag || it >= kSpinLimit || now_ns() - t0 > limit_ns)) {
+              if (!*abort_flag) {
+                *abort_flag = 1;
+                atomicExch(&hdr->status, kStatusTimeout);
+              }
+              quit = 1;
+            }
+            if (__shfl_sync(0xffffffffu, quit, 0)) {
+              ok = false;
+              break;
+            }
+            __nanosleep(64);
+          }
+        }
+        float agv[AAL_MAX_K];
+#pragma unroll
+        for (int jj = 0; jj < AAL_MAX_K; ++jj) {
+          const float g_ = __shfl_sync(0xffffffffu, __uint_as_float((uint32_t)w), jj);
+          agv[jj] = jj < K ? g_ : 0.f;
+        }
+        if (lane == 0) {
+          int32_t live = 0;
+          if (ok) {
+            int kn = K;
+            if (f.win.mask != nullptr) {
+              kn = 0;
+              while (kn < K && f.win.mask[r0 + kn] != 0) ++kn;
+            }
+            float dE[AAL_MAX_K];
+            window_term(agv, kn, dE);
+            const bool pos_valid = f.bw.mask == nullptr || f.bw.mask[r] != 0;
+            RowCoef c;
+            live = row_coef<true, false, false>(f.bw, scale, 0.f, f.bw.w_greedy != 0.f ? dE[k] : 0.f, 0.f, 0.f,
+                                                pos_valid, st, c)
+                       ? 1
+                       : 0;
+            F.coef = c;
+          }
+          F.live = live;
+        }
+      }
+      named_barrier(kRBarCoef, kRConsumers);
+
+      // ---- pass 3: the gradient row (L2)
+      const int32_t live = F.live;
+      const RowCoef c = F.coef;
+      const int64_t xv = (live && c.xs >= 0) ? c.xs / E : -1;
+      const int xe = c.xs >= 0 ? c.xs % E : 0;
+      uint4* out4 = reinterpret_cast<uint4*>(static_cast<T*>(f.bw.grad) + r * a.V);
+      const uint4 zero4 = make_uint4(0, 0, 0, 0);
+      for (int cc = 0; cc < nch; ++cc) {
+        if (wait_full(&S.full[slot], phase, abort_flag, limit_ns, hdr)) {
+          const int e0 = cc * CH;
+          const int64_t vb = e0 / E;
+          const uint4* Z = reinterpret_cast<const uint4*>(ring + slot * kRSlotBytes);
+          if (e0 + CH <= V) {
+#pragma unroll
+            for (int v = 0; v < kRNV; ++v) {
+              const int i = t + v * kRConsumers;
+              st_stream(out4 + vb + i, live ? grad_vec<T, true, false, false, false>(c, Z[i], zero4, vb + i, xv, xe, -1, 0)
+                                            : zero4);
+            }
+          } else {
+            const int nvec = (V - e0) / E;
+            for (int i = t; i < nvec; i += kRConsumers)
+              st_stream(out4 + vb + i, live ? grad_vec<T, true, false, false, false>(c, Z[i], zero4, vb + i, xv, xe, -1, 0)
+                                            : zero4);
+          }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&S.empty[slot]);
+        if (++slot == kRSlots) {
+          slot = 0;
+          phase ^= 1u;
+        }
+      }
+    }
+  }
+  __syncwarp();
+  __syncthreads();
+}
+
 }  // namespace
+
+cudaError_t launch_fused_ids(const FusedIdsArgs& f0, cudaStream_t s, uint64_t limit_ns, bool* launched) {
+  *launched = false;
+  if (f0.bw.w_greedy == 0.f || f0.bw.grpo) return cudaSuccess;  // only the greedy term is fused here
+  auto kern = fused_ids_rows;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFIdsSmemBytes);
+  if (e != cudaSuccess) return e;
+  int dev = 0, sms = 0, per_sm = 0, coop = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev);
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kRThreads, kFIdsSmemBytes);
+  if (e != cudaSuccess) return e;
+  const int64_t K = f0.win.K;
+  int64_t G = (int64_t)sms * per_sm / K;
+  if (G > f0.win.N) G = f0.win.N;
+  if (G > kMaxGroups) G = kMaxGroups;
+  if (!coop || G < 1) return cudaSuccess;
+  FusedIdsArgs f = f0;
+  f.groups = (int32_t)G;
+  const int CH = kRSlotBytes / 2;
+  const int nch = (int)((f.st.V + CH - 1) / CH);
+  void* args[] = {&f, (void*)&nch, &limit_ns};
+  e = cudaLaunchCooperativeKernel((const void*)kern, dim3((unsigned)(G * K)), dim3(kRThreads), args, kFIdsSmemBytes, s);
+  if (e == cudaErrorCooperativeLaunchTooLarge) {  // fewer SMs available: the caller runs the two calls
+    cudaGetLastError();
+    return cudaSuccess;
+  }
+  if (e != cudaSuccess) return e;
+  *launched = true;
+  resolve_draft_argmax<uint16_t><<<(unsigned)((f.st.R + 255) / 256), 256, 0, s>>>(f.st);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_one_tensor(const Stream1Args& a, bool bf16, bool ids, cudaStream_t s) {
   return bf16 ? launch_T<uint16_t>(a, ids, s) : launch_T<float>(a, ids, s);

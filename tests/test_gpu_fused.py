@@ -3,8 +3,8 @@
 It must give the loss, the per-window expected lengths and the gradient of aal_loss_fwd followed
 by aal_loss_bwd bit for bit: on the fused path (bf16 rows of 16-byte multiples; every flag
 combination it instantiates, masks, fewer windows than CTA groups, K = 1 and K = 8, full-size
-rows) and on the problems it hands to the two calls (fp32, unaligned rows, token ids, the
-anchor beside the sampling term at T != 1).  A few cases are also checked against the oracle
+rows; token ids with the draft alone streamed) and on the problems it hands to the two calls
+(fp32, unaligned rows, the anchor beside the sampling term at T != 1).  A few cases are also checked against the oracle
 directly, and the bounded waits are driven to a timeout without a fault.
 """
 
@@ -103,9 +103,49 @@ def test_problems_the_two_calls_take(mode, T, dtype, V):
     assert_same(FusedRun(t, d, m, mode, T, 0.5, 0.5), LossRun(t, d, m, mode, T, 0.5, 0.5))
 
 
-def test_token_ids_take_the_two_calls():
-    t, d, _ = _inputs(10, 3, 4096, seed=9)
+@pytest.mark.parametrize("N,K,V,masked", [(10, 3, 4096, False), (40, 7, 30000, True), (3, 8, 128256, False),
+                                           (100, 1, 1000, True)])
+@pytest.mark.parametrize("dloss_is_w", [False, True])
+def test_token_ids_fused_equals_two_calls(N, K, V, masked, dloss_is_w):
+    """x* as token ids (the draft alone streamed), some ids out of range on one run."""
+    t, d, m = _inputs(N, K, V, seed=9 + N, masked=masked)
     ids = t.float().argmax(-1).to(torch.int32).contiguous()
+    dloss = float(N) if dloss_is_w else 1.0
+    assert_same(FusedRun(ids, d, m, G | IDS, 1.0, 1.0, 0.0, dloss), LossRun(ids, d, m, G | IDS, 1.0, 1.0, 0.0, dloss))
+
+
+def test_token_ids_out_of_range_reported():
+    t, d, _ = _inputs(12, 4, 4096, seed=21)
+    ids = t.float().argmax(-1).to(torch.int32).contiguous()
+    ids[3, 1] = 4096                                   # one id past the vocabulary
+    prob = aal.loss_problem(d, G | IDS, 1.0, 1.0, 0.0)
+    ws = torch.empty(aal.aal_workspace_size(prob), dtype=torch.uint8, device=DEV)
+    loss = torch.empty(1, device=DEV)
+    grad = torch.empty_like(d)
+    aal.aal_loss_fwd_bwd(prob, d, ids, None, ws, 1.0, loss, grad)
+    assert aal.aal_check_device_status(ws) == aal.AAL_ERR_INVALID_ARG
+    s = torch.empty_like(grad)
+    ws2 = torch.empty_like(ws)
+    aal.aal_loss_fwd(prob, d, ids, None, ws2, loss)
+    aal.aal_loss_bwd(prob, d, ids, None, ws2, 1.0, s)
+    assert aal.aal_check_device_status(ws2) == aal.AAL_ERR_INVALID_ARG
+    assert torch.equal(_bits(grad), _bits(s))
+
+
+def test_token_ids_ring_times_out_and_context_stays_usable():
+    t, d, _ = _inputs(16, 2, 40000, seed=12)
+    ids = t.float().argmax(-1).to(torch.int32).contiguous()
+    prob = aal.loss_problem(d, G | IDS, 1.0, 1.0, 0.0)
+    ws = torch.empty(aal.aal_workspace_size(prob), dtype=torch.uint8, device=DEV)
+    loss = torch.empty(1, device=DEV)
+    grad = torch.empty_like(d)
+    aal.aal_debug_fail_next_forward(2, 50_000_000)    # a chunk of the gradient pass
+    try:
+        aal.aal_loss_fwd_bwd(prob, d, ids, None, ws, 1.0, loss, grad)
+        assert aal.aal_check_device_status(ws) == aal.AAL_ERR_TIMEOUT
+        assert aal.aal_check_device_status(ws) == aal.AAL_OK
+    finally:
+        aal.aal_debug_fail_next_forward(-1, 0)
     assert_same(FusedRun(ids, d, None, G | IDS, 1.0, 1.0, 0.0), LossRun(ids, d, None, G | IDS, 1.0, 1.0, 0.0))
 
 
