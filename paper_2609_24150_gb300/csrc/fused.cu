@@ -308,44 +308,13 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
         const bool ov = f.win.sampling || f.win.tv;
         const bool need = f.win.greedy || ov;  // the anchor alone needs no window term
         const int64_t r0 = n * K;
-        if (lane == 0) {
-          // publish this row's (a^greedy, a^sample): one 64-bit word, its own ready flag
-          const float as_r = PASSES == 2 ? st_as : 0.f;
-          uint64_t word = ((uint64_t)__float_as_uint(as_r) << 32) | __float_as_uint(st.ag);
-          if (word == kMboxEmpty) word = 0;  // (bit patterns no arithmetic yields; never sent)
-          st_relaxed(&a.ws.mbox[r], word);
-        }
-        // one reading of the abort flag for the whole warp (another warp may raise it meanwhile)
-        bool ok = __shfl_sync(0xffffffffu, *abort_flag == 0 ? 1 : 0, 0) != 0;
-        uint64_t w = 0;
-        if (ok && need) {
-          const uint64_t t0 = now_ns();
-          for (uint32_t it = 0;; ++it) {
-            if (lane < K) w = ld_relaxed(&a.ws.mbox[r0 + lane]);
-            if (__all_sync(0xffffffffu, lane >= K || w != kMboxEmpty)) break;
-            // lane 0 decides for the warp whether to give up
-            int quit = 0;
-            if (lane == 0 && (*abort_flag || it >= kSpinLimit || now_ns() - t0 > limit_ns)) {
-              if (!*abort_flag) {
-                *abort_flag = 1;
-                atomicExch(&hdr->status, kStatusTimeout);
-              }
-              quit = 1;
-            }
-            if (__shfl_sync(0xffffffffu, quit, 0)) {
-              ok = false;
-              break;
-            }
-            __nanosleep(64);
-          }
-        }
         float agv[AAL_MAX_K], asv[AAL_MAX_K];
+        const bool ok = window_exchange(a.ws.mbox, r, r0, K, lane, st.ag, PASSES == 2 ? st_as : 0.f, need,
+                                        abort_flag, hdr, limit_ns, agv, asv);
 #pragma unroll
-        for (int jj = 0; jj < AAL_MAX_K; ++jj) {  // to lane 0 (0 beyond K, or without the term)
-          const float g_ = __shfl_sync(0xffffffffu, __uint_as_float((uint32_t)w), jj);
-          const float s_ = __shfl_sync(0xffffffffu, __uint_as_float((uint32_t)(w >> 32)), jj);
-          agv[jj] = (jj < K && need && f.win.greedy) ? g_ : 0.f;
-          asv[jj] = (jj < K && need && ov) ? s_ : 0.f;
+        for (int jj = 0; jj < AAL_MAX_K; ++jj) {  // only the terms the window kernel forms
+          if (!f.win.greedy) agv[jj] = 0.f;
+          if (!ov) asv[jj] = 0.f;
         }
         if (lane == 0) {
           int32_t live = 0;

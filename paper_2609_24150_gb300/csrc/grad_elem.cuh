@@ -241,4 +241,51 @@ __device__ __forceinline__ uint4 grad_vec(const RowCoef& c, const uint4& qw, con
   return Io<T>::pack(d);
 }
 
+// The window exchange of the fused forward + backward, run by one whole warp: lane 0 publishes
+// this row's (a^greedy, a^sample) as one 64-bit word in the per-row mailbox (preset to
+// kMboxEmpty, so the word is its own ready flag), then lane j polls the word of depth j of the
+// window (rows r0 .. r0 + K - 1) until none is empty, bounded like the ring waits.  When `need`
+// is false (no window term) nothing is polled.  Returns, to every lane, whether the window's
+// words arrived; on lane 0, ag[j] and as[j] hold depth j's values (0 beyond K).  The abort flag
+// is read once for the warp (another warp may raise it meanwhile).
+__device__ __forceinline__ bool window_exchange(uint64_t* mbox, int64_t r, int64_t r0, int K, int lane, float ag_r,
+                                                float as_r, bool need, volatile int* abort_flag, WsHeader* hdr,
+                                                uint64_t limit_ns, float* ag, float* as) {
+  if (lane == 0) {
+    uint64_t word = ((uint64_t)__float_as_uint(as_r) << 32) | __float_as_uint(ag_r);
+    if (word == kMboxEmpty) word = 0;  // (bit patterns no arithmetic yields; never sent)
+    ptx::st_relaxed(&mbox[r], word);
+  }
+  bool ok = __shfl_sync(0xffffffffu, *abort_flag == 0 ? 1 : 0, 0) != 0;
+  uint64_t w = 0;
+  if (ok && need) {
+    const uint64_t t0 = ptx::now_ns();
+    for (uint32_t it = 0;; ++it) {
+      if (lane < K) w = ptx::ld_relaxed(&mbox[r0 + lane]);
+      if (__all_sync(0xffffffffu, lane >= K || w != kMboxEmpty)) break;
+      int quit = 0;  // lane 0 decides for the warp whether to give up
+      if (lane == 0 && (*abort_flag || it >= kSpinLimit || ptx::now_ns() - t0 > limit_ns)) {
+        if (!*abort_flag) {
+          *abort_flag = 1;
+          atomicExch(&hdr->status, kStatusTimeout);
+        }
+        quit = 1;
+      }
+      if (__shfl_sync(0xffffffffu, quit, 0)) {
+        ok = false;
+        break;
+      }
+      __nanosleep(64);
+    }
+  }
+#pragma unroll
+  for (int jj = 0; jj < AAL_MAX_K; ++jj) {
+    const float g_ = __shfl_sync(0xffffffffu, __uint_as_float((uint32_t)w), jj);
+    const float s_ = __shfl_sync(0xffffffffu, __uint_as_float((uint32_t)(w >> 32)), jj);
+    ag[jj] = (jj < K && need) ? g_ : 0.f;
+    as[jj] = (jj < K && need) ? s_ : 0.f;
+  }
+  return ok;
+}
+
 }  // namespace aal

@@ -626,39 +626,9 @@ __global__ void __launch_bounds__(kRThreads, 1) fused_ids_rows(FusedIdsArgs f, i
       // ---- the window's a^greedy (warp 0: lane j polls depth j), the row's coefficients (thread 0)
       if (warp == 0) {
         const int64_t r0 = n * K;
-        if (lane == 0) {
-          uint64_t word = __float_as_uint(st.ag);
-          if (word == kMboxEmpty) word = 0;
-          st_relaxed(&a.lws.mbox[r], word);
-        }
-        bool ok = __shfl_sync(0xffffffffu, *abort_flag == 0 ? 1 : 0, 0) != 0;
-        uint64_t w = 0;
-        if (ok) {
-          const uint64_t t0 = now_ns();
-          for (uint32_t it = 0;; ++it) {
-            if (lane < K) w = ld_relaxed(&a.lws.mbox[r0 + lane]);
-            if (__all_sync(0xffffffffu, lane >= K || w != kMboxEmpty)) break;
-            int quit = 0;
-            if (lane == 0 && (*abort_flag || it >= kSpinLimit || now_ns() - t0 > limit_ns)) {
-              if (!*abort_flag) {
-                *abort_flag = 1;
-                atomicExch(&hdr->status, kStatusTimeout);
-              }
-              quit = 1;
-            }
-            if (__shfl_sync(0xffffffffu, quit, 0)) {
-              ok = false;
-              break;
-            }
-            __nanosleep(64);
-          }
-        }
-        float agv[AAL_MAX_K];
-#pragma unroll
-        for (int jj = 0; jj < AAL_MAX_K; ++jj) {
-          const float g_ = __shfl_sync(0xffffffffu, __uint_as_float((uint32_t)w), jj);
-          agv[jj] = jj < K ? g_ : 0.f;
-        }
+        float agv[AAL_MAX_K], asv[AAL_MAX_K];
+        const bool ok = window_exchange(a.lws.mbox, r, r0, K, lane, st.ag, 0.f, true, abort_flag, hdr, limit_ns,
+                                        agv, asv);
         if (lane == 0) {
           int32_t live = 0;
           if (ok) {
