@@ -72,6 +72,8 @@ CASES = [
     (12, 6, 6000, KL | TV, 1.0, 0.0, 0.0, 1.0, 0.1, False), # TV term + anchor, no greedy term
     (3, 7, 128256, B, 1.0, 0.5, 0.5, 1.0, 1.0, False),      # fewer windows than groups, full rows
     (200, 1, 2048, B, 1.0, 0.5, 0.5, 1.0, 1.0, False),      # K = 1: groups of one CTA
+    (30, 3, 8, B, 1.0, 0.5, 0.5, 1.0, 1.0, True),           # one 16-byte vector a row
+    (30, 4, 24, KL | G, 1.0, 0.1, 0.0, 1.0, 1.0, False),    # three vectors a row, one pass
 ]
 
 
@@ -104,7 +106,7 @@ def test_problems_the_two_calls_take(mode, T, dtype, V):
 
 
 @pytest.mark.parametrize("N,K,V,masked", [(10, 3, 4096, False), (40, 7, 30000, True), (3, 8, 128256, False),
-                                           (100, 1, 1000, True)])
+                                           (100, 1, 1000, True), (20, 5, 8, True)])
 @pytest.mark.parametrize("dloss_is_w", [False, True])
 def test_token_ids_fused_equals_two_calls(N, K, V, masked, dloss_is_w):
     """x* as token ids (the draft alone streamed), some ids out of range on one run."""
