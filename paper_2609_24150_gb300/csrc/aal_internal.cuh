@@ -251,6 +251,8 @@ struct FusedArgs {
   BackwardArgs bw;   // the gradient pass (grad, dloss, weights, position mask, invT)
   WindowArgs win;    // the window terms (mask [N][K], N, K, which terms, w_sampling, w_tv)
   int32_t groups;    // G
+  int32_t solos;     // S solo CTAs after the groups' G K, each taking whole windows
+  int64_t n_group;   // windows 0 .. n_group - 1 go to the groups, the rest to the solo CTAs
 };
 
 struct RewardRowArgs {

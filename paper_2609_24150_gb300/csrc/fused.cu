@@ -12,6 +12,11 @@
 //   G groups x K CTAs; CTA k of group g takes depth k of windows g, g + G, ...  A cooperative
 //   launch has all its CTAs resident at once, so a group never waits on a CTA that is not
 //   running.
+// * Solo CTAs: the SMs that G K leaves over (152 - 147 at K = 7) each take whole windows of
+//   the last windows: the statistics of the window's K rows one after another, the K rows'
+//   coefficients from its own acceptances (no exchange), then the K gradient rows.  The host
+//   gives them as many windows as balances the two kinds; their rows stay in L2 across K rows'
+//   time instead of one.
 // * Window exchange: once its row's statistics are in the workspace, thread 0 of each CTA
 //   publishes the row's (a^greedy, a^sample) as one 64-bit word in a per-row mailbox that the
 //   call filled with an all-ones sentinel, and warp 0 polls (bounded, like the ring waits; lane
@@ -27,6 +32,8 @@
 // * Failure: every wait is bounded.  A CTA that gave up keeps walking its rows without waiting
 //   and still publishes a word for each, so its group does not wait on it for the whole limit;
 //   the workspace status word reports AAL_ERR_TIMEOUT and the outputs are not to be used.
+#include <algorithm>
+
 #include "grad_elem.cuh"
 #include "stream_core.cuh"
 
@@ -39,6 +46,11 @@ struct FusedSmem {
   Smem s;
   RowCoef coef;
   int32_t live;  // the row's gradient has a nonzero term
+  // a solo CTA's window: its rows' statistics and acceptances, then their coefficients
+  RowStat solo_st[AAL_MAX_K];
+  float solo_ag[AAL_MAX_K], solo_as[AAL_MAX_K];
+  RowCoef solo_coef[AAL_MAX_K];
+  int32_t solo_live[AAL_MAX_K];
 };
 
 constexpr size_t kFusedSmemBytes = (size_t)kSlots * kSlotBytes + sizeof(FusedSmem);
@@ -64,12 +76,15 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
   const int K = f.win.K;
   const int64_t N = f.win.N;
   const int G = f.groups;
-  const int g = blockIdx.x / K, k = blockIdx.x % K;
+  const int64_t NG = f.n_group;        // windows 0 .. NG - 1 go to the groups, the rest to the solo CTAs
+  const bool solo = (int)blockIdx.x >= G * K;
+  const int g = blockIdx.x / K, k = blockIdx.x % K;  // (a group's CTA)
+  const int so = (int)blockIdx.x - G * K;            // (a solo CTA)
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kSlots; ++s) {
-      mbar_init(&S.full[s], 1);
-      mbar_init(&S.empty[s], kWarps);
+    for (int q = 0; q < kSlots; ++q) {
+      mbar_init(&S.full[q], 1);
+      mbar_init(&S.empty[q], kWarps);
     }
     S.abort_flag = 0;
     S.arg_index = 0x7fffffff;
@@ -87,12 +102,12 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
       RingPos pos;
       int64_t seq = 0;
       uint32_t armed = 0, last_phase = 0;
-      for (int64_t n = g; n < N && !*abort_flag; n += G) {
-        const int64_t r = n * K + k;
+      // passes [p0, p1) of row r: the statistics passes keep the row in L2, the gradient pass
+      // (pass PASSES) is its last use
+      auto issue = [&](int64_t r, int p0, int p1) {
         const char* prow = static_cast<const char*>(a.zp) + r * a.V * 2;
         const char* qrow = static_cast<const char*>(a.zq) + r * a.V * 2;
-        // statistics passes keep the row in L2; the gradient pass is its last use
-        for (int pass = 0; pass < PASSES + 1 && !*abort_flag; ++pass) {
+        for (int pass = p0; pass < p1 && !*abort_flag; ++pass) {
           const uint64_t pol = pass < PASSES ? keep : drop;
           for (int c = 0; c < nch; ++c) {
             if (!wait_phase(&S.empty[pos.slot], pos.phase ^ 1u, abort_flag, limit_ns, hdr)) break;
@@ -110,12 +125,21 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
             ++seq;
           }
         }
+      };
+      if (!solo) {
+        for (int64_t n = g; n < NG && !*abort_flag; n += G) issue(n * K + k, 0, PASSES + 1);
+      } else {
+        // a whole window: the statistics of its K rows, then their gradients
+        for (int64_t n = NG + so; n < N && !*abort_flag; n += f.solos) {
+          for (int kk = 0; kk < K; ++kk) issue(n * K + kk, 0, PASSES);
+          for (int kk = 0; kk < K; ++kk) issue(n * K + kk, PASSES, PASSES + 1);
+        }
       }
-      for (int s = 0; s < kSlots; ++s) {
-        if (!(armed & (1u << s))) continue;
-        const uint32_t ph = (last_phase >> s) & 1u;
+      for (int q = 0; q < kSlots; ++q) {
+        if (!(armed & (1u << q))) continue;
+        const uint32_t ph = (last_phase >> q) & 1u;
         const uint64_t t0 = now_ns();
-        for (uint32_t it = 0; it < kSpinLimit && !mbar_try(&S.full[s], ph, 100000); ++it)
+        for (uint32_t it = 0; it < kSpinLimit && !mbar_try(&S.full[q], ph, 100000); ++it)
           if (now_ns() - t0 > limit_ns) break;
       }
     }
@@ -123,7 +147,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
     // ------------------------------------------------------------ consumers
     const int t = threadIdx.x;
     RingPos pos;
-    uint32_t j = 0;
+    uint32_t j = 0;  // rows walked (parity of the reduction buffers)
     const float sT = PASSES == 2 ? a.sT : kLog2e;
     // the backward's scales (thread 0 forms the coefficients)
     float scale = 0.f, kscale = 0.f;
@@ -133,8 +157,11 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
       const int npos = KL ? hdr->npos : 0;
       kscale = npos > 0 ? f.bw.dloss * f.bw.w_kl / (float)npos : 0.f;
     }
-    for (int64_t n = g; n < N; n += G, ++j) {
-      const int64_t r = n * K + k;
+    const bool ov = f.win.sampling || f.win.tv;
+
+    // The statistics passes of row r: writes its statistics to the workspace; thread 0 gets what
+    // the row's coefficients need (st) and its a^sample (st_as).
+    auto stats_row = [&](int64_t r, RowStat& st, float& st_as) {
       // ---- pass 1: online normalisers and argmax (HBM)
       RowPart A;
       part_init(A);
@@ -168,8 +195,6 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
       warp_part<NEED_Q1, KL>(tot, sT);
       const float Mp = tot.pM, Lsp = log2f(tot.pS);
       const float Mq = tot.qM, Lsq = log2f(tot.qS);
-      RowStat st{};  // thread 0: what the row's coefficients need
-      float st_as = 0.f;  // thread 0: the row's a^sample (two passes)
       if (KL && t == 0) {  // both normalisers are at T = 1 here
         const float Mq1 = NEED_Q1 ? tot.q1M : Mq;
         const float Lsq1 = NEED_Q1 ? log2f(tot.q1S) : Lsq;
@@ -302,57 +327,41 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
           S.yarg_carry = 0.f;
         }
       }
+      ++j;
+    };
 
-      // ---- the window's acceptances (warp 0: lane j polls depth j), the row's coefficients (thread 0)
-      if (warp == 0) {
-        const bool ov = f.win.sampling || f.win.tv;
-        const bool need = f.win.greedy || ov;  // the anchor alone needs no window term
-        const int64_t r0 = n * K;
-        float agv[AAL_MAX_K], asv[AAL_MAX_K];
-        const bool ok = window_exchange(a.ws.mbox, r, r0, K, lane, st.ag, PASSES == 2 ? st_as : 0.f, need,
-                                        abort_flag, hdr, limit_ns, agv, asv);
-#pragma unroll
-        for (int jj = 0; jj < AAL_MAX_K; ++jj) {  // only the terms the window kernel forms
-          if (!f.win.greedy) agv[jj] = 0.f;
-          if (!ov) asv[jj] = 0.f;
-        }
-        if (lane == 0) {
-          int32_t live = 0;
-          if (ok) {
-            // the window's terms, as the window kernel forms them (rows n K .. n K + K - 1)
-            int kn = K;
-            if (f.win.mask != nullptr) {
-              kn = 0;
-              while (kn < K && f.win.mask[r0 + kn] != 0) ++kn;
-            }
-            float dE[AAL_MAX_K];
-            float dEg = 0.f, dEs = 0.f;
-            if (f.win.greedy) {
-              window_term(agv, kn, dE);
-              dEg = dE[k];
-            }
-            if (ov) {
-              if (f.win.sampling) window_term(asv, kn, dE);
-              const float tvc = (f.win.tv && kn > 0) ? f.win.w_tv / (float)kn : 0.f;
-              dEs = __fadd_rn(f.win.sampling ? __fmul_rn(f.win.w_sampling, dE[k]) : 0.f, k < kn ? tvc : 0.f);
-            }
-            const bool with_greedy = GREEDY && f.bw.w_greedy != 0.f;
-            const bool pos_valid = f.bw.mask == nullptr || f.bw.mask[r] != 0;
-            RowCoef c;
-            live = row_coef<GREEDY, SAMPLING, KL>(f.bw, scale, kscale, with_greedy ? dEg : 0.f,
-                                                  SAMPLING ? dEs : 0.f, 0.f, pos_valid, st, c)
-                       ? 1
-                       : 0;
-            F.coef = c;
-          }
-          F.live = live;
-        }
+    // Thread 0: the coefficients of depth kk of window n (row r) from the window's acceptances
+    // (agv, asv; 0 beyond K and for a term the window kernel does not form), as the window
+    // kernel forms its terms and the backward its coefficients.  Returns whether any is nonzero.
+    auto coef_row = [&](int64_t n, int kk, int64_t r, const float* agv, const float* asv, const RowStat& st,
+                        RowCoef& c) -> int32_t {
+      const int64_t r0 = n * K;
+      int kn = K;
+      if (f.win.mask != nullptr) {
+        kn = 0;
+        while (kn < K && f.win.mask[r0 + kn] != 0) ++kn;
       }
-      named_barrier(kBarCoef, kConsumers);
+      float dE[AAL_MAX_K];
+      float dEg = 0.f, dEs = 0.f;
+      if (f.win.greedy) {
+        window_term(agv, kn, dE);
+        dEg = dE[kk];
+      }
+      if (ov) {
+        if (f.win.sampling) window_term(asv, kn, dE);
+        const float tvc = (f.win.tv && kn > 0) ? f.win.w_tv / (float)kn : 0.f;
+        dEs = __fadd_rn(f.win.sampling ? __fmul_rn(f.win.w_sampling, dE[kk]) : 0.f, kk < kn ? tvc : 0.f);
+      }
+      const bool with_greedy = GREEDY && f.bw.w_greedy != 0.f;
+      const bool pos_valid = f.bw.mask == nullptr || f.bw.mask[r] != 0;
+      return row_coef<GREEDY, SAMPLING, KL>(f.bw, scale, kscale, with_greedy ? dEg : 0.f, SAMPLING ? dEs : 0.f, 0.f,
+                                            pos_valid, st, c)
+                 ? 1
+                 : 0;
+    };
 
-      // ---- pass 3: the gradient row (L2)
-      const int32_t live = F.live;
-      const RowCoef c = F.coef;
+    // ---- pass 3: the gradient row (L2)
+    auto grad_row = [&](int64_t r, const RowCoef& c, int32_t live) {
       const int64_t xv = (live && c.xs >= 0) ? c.xs / E : -1;
       const int xe = c.xs >= 0 ? c.xs % E : 0;
       uint4* out4 = reinterpret_cast<uint4*>(static_cast<T*>(f.bw.grad) + r * a.V);
@@ -379,6 +388,69 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&S.empty[pos.slot]);
+      }
+    };
+
+    if (!solo) {
+      // one row of each of the group's windows: statistics, the window exchange, the gradient
+      for (int64_t n = g; n < NG; n += G) {
+        const int64_t r = n * K + k;
+        RowStat st{};
+        float st_as = 0.f;
+        stats_row(r, st, st_as);
+        if (warp == 0) {
+          const bool need = f.win.greedy || ov;  // the anchor alone needs no window term
+          float agv[AAL_MAX_K], asv[AAL_MAX_K];
+          const bool ok = window_exchange(a.ws.mbox, r, n * K, K, lane, st.ag, PASSES == 2 ? st_as : 0.f, need,
+                                          abort_flag, hdr, limit_ns, agv, asv);
+#pragma unroll
+          for (int jj = 0; jj < AAL_MAX_K; ++jj) {  // only the terms the window kernel forms
+            if (!f.win.greedy) agv[jj] = 0.f;
+            if (!ov) asv[jj] = 0.f;
+          }
+          if (lane == 0) {
+            RowCoef c;
+            F.live = ok ? coef_row(n, k, r, agv, asv, st, c) : 0;
+            if (F.live) F.coef = c;
+          }
+        }
+        named_barrier(kBarCoef, kConsumers);
+        const RowCoef c = F.coef;
+        grad_row(r, c, F.live);
+      }
+    } else {
+      // whole windows: the statistics of the K rows, their coefficients from those rows alone
+      // (no exchange), then the K gradient rows
+      for (int64_t n = NG + so; n < N; n += f.solos) {
+        for (int kk = 0; kk < K; ++kk) {
+          RowStat st{};
+          float st_as = 0.f;
+          stats_row(n * K + kk, st, st_as);
+          if (t == 0) {
+            F.solo_st[kk] = st;
+            F.solo_ag[kk] = f.win.greedy ? st.ag : 0.f;
+            F.solo_as[kk] = ov && PASSES == 2 ? st_as : 0.f;
+          }
+        }
+        if (t == 0) {
+          float agv[AAL_MAX_K], asv[AAL_MAX_K];
+#pragma unroll
+          for (int jj = 0; jj < AAL_MAX_K; ++jj) {
+            agv[jj] = jj < K ? F.solo_ag[jj] : 0.f;
+            asv[jj] = jj < K ? F.solo_as[jj] : 0.f;
+          }
+          for (int kk = 0; kk < K; ++kk) {
+            RowCoef c;
+            const bool ok = !*abort_flag;
+            F.solo_live[kk] = ok ? coef_row(n, kk, n * K + kk, agv, asv, F.solo_st[kk], c) : 0;
+            if (F.solo_live[kk]) F.solo_coef[kk] = c;
+          }
+        }
+        named_barrier(kBarCoef, kConsumers);
+        for (int kk = 0; kk < K; ++kk) {
+          const RowCoef c = F.solo_coef[kk];
+          grad_row(n * K + kk, c, F.solo_live[kk]);
+        }
       }
     }
   }
@@ -430,12 +502,28 @@ cudaError_t go_fused(const FusedArgs& f0, cudaStream_t s, uint64_t limit_ns, boo
   if (G > f0.win.N) G = f0.win.N;
   if (G > kMaxGroups) G = kMaxGroups;
   if (!coop || G < 1) return cudaSuccess;  // *launched stays false: the caller runs the two calls
+  // The SMs left over by the groups (sms per_sm - G K of them) take whole windows alone: a
+  // group finishes a window in one row's time, a solo CTA in K, so with m windows per solo CTA
+  // the step ends after max(ceil((N - m S) / G), m K) row times.  Take the best m near the
+  // balance point N / (G K + S), or no solo CTAs.
+  const int64_t N = f0.win.N;
+  const int64_t S = (int64_t)sms * per_sm - G * K;
+  int64_t best_m = 0;
+  if (S > 0) {
+    auto cost = [&](int64_t m) { return std::max((N - m * S + G - 1) / G, m * K); };
+    const int64_t m0 = N / (G * K + S);
+    for (int64_t m = m0; m <= m0 + 1; ++m)
+      if (m > 0 && m * S <= N && cost(m) < cost(best_m)) best_m = m;
+  }
   FusedArgs f = f0;
   f.groups = (int32_t)G;
+  f.solos = best_m > 0 ? (int32_t)S : 0;
+  f.n_group = N - best_m * f.solos;
   const int elt = 2;
   const int nch = (int)((f.st.V + kHalfSlot / elt - 1) / (kHalfSlot / elt));
   void* args[] = {&f, (void*)&nch, &limit_ns};
-  e = cudaLaunchCooperativeKernel((const void*)kern, dim3((unsigned)(G * K)), dim3(kThreads), args, kFusedSmemBytes, s);
+  e = cudaLaunchCooperativeKernel((const void*)kern, dim3((unsigned)(G * K + f.solos)), dim3(kThreads), args,
+                                  kFusedSmemBytes, s);
   if (e == cudaErrorCooperativeLaunchTooLarge) {  // fewer SMs available than the device has (shared
     cudaGetLastError();                           // device): the caller runs the two calls instead
     return cudaSuccess;

@@ -2,8 +2,8 @@
 
 It must give the loss, the per-window expected lengths and the gradient of aal_loss_fwd followed
 by aal_loss_bwd bit for bit: on the fused path (bf16 rows of 16-byte multiples; every flag
-combination it instantiates, masks, fewer windows than CTA groups, K = 1 and K = 8, full-size
-rows; token ids with the draft alone streamed) and on the problems it hands to the two calls
+combination it instantiates, masks, fewer windows than CTA groups, K = 1 and K = 8, windows
+enough for the solo CTAs, full-size rows; token ids with the draft alone streamed) and on the problems it hands to the two calls
 (fp32, unaligned rows, the anchor beside the sampling term at T != 1).  A few cases are also checked against the oracle
 directly, and the bounded waits are driven to a timeout without a fault.
 """
@@ -77,9 +77,41 @@ CASES = [
 ]
 
 
-@pytest.mark.parametrize("N,K,V,mode,T,wg,ws,wkl,wtv,masked", CASES)
+# Windows enough that the SMs the groups leave over (152 - G K) take whole windows as solo CTAs:
+# again each instantiation once.  N = G K + S balances one window per solo CTA; 304, two.
+SOLO_CASES = [
+    (152, 7, 4104, B, 1.0, 0.5, 0.5, 1.0, 1.0, False),
+    (304, 7, 2000, S, 0.7, 1.0, 1.0, 1.0, 1.0, True),
+    (152, 5, 8192, B, 1.5, 0.5, 0.5, 1.0, 1.0, False),
+    (152, 3, 1000, G, 1.0, 1.0, 0.0, 1.0, 1.0, True),
+    (152, 6, 3000, KL | G, 1.0, 0.1, 0.0, 1.0, 1.0, False),
+    (152, 6, 3000, KL, 1.0, 0.0, 0.0, 1.0, 1.0, True),
+    (152, 5, 6000, KL | B, 1.0, 0.1, 0.1, 1.0, 1.0, True),
+    (152, 7, 6000, KL | TV, 1.0, 0.0, 0.0, 1.0, 0.1, False),
+]
+
+
+def solo_windows(N, K, sms):
+    """The windows the launch gives to solo CTAs (one CTA per SM, as the ring's shared memory
+    allows): m per solo CTA, m minimising max(ceil((N - m S) / G), m K)."""
+    G = min(sms // K, N, 1024)
+    S = sms - G * K
+    cost = lambda m: max(-(-(N - m * S) // G), m * K)
+    best = 0
+    if S > 0:
+        m0 = N // (G * K + S)
+        for m in (m0, m0 + 1):
+            if m > 0 and m * S <= N and cost(m) < cost(best):
+                best = m
+    return best * S if best else 0
+
+
+@pytest.mark.parametrize("N,K,V,mode,T,wg,ws,wkl,wtv,masked", CASES + SOLO_CASES)
 @pytest.mark.parametrize("dloss_is_w", [False, True])
 def test_fused_equals_two_calls(N, K, V, mode, T, wg, ws, wkl, wtv, masked, dloss_is_w):
+    if (N, K, V, mode, T, wg, ws, wkl, wtv, masked) in SOLO_CASES:
+        sms = torch.cuda.get_device_properties(0).multi_processor_count
+        assert solo_windows(N, K, sms) > 0, "the case no longer reaches the solo CTAs"
     t, d, m = _inputs(N, K, V, seed=N + K + V, masked=masked)
     dloss = float(N) if dloss_is_w else 1.0   # |W|-sized upstream gradient makes the absolute term bind
     f = FusedRun(t, d, m, mode, T, wg, ws, dloss, wkl, wtv)
@@ -163,11 +195,12 @@ def test_fused_against_the_oracle(mode, T, wg, ws):
     check_loss(FusedRun(t, d, m, mode, T, wg, ws, dloss=24.0), t, d, m, mode, T, wg, ws, dloss=24.0)
 
 
-def test_group_barrier_and_ring_time_out_and_context_stays_usable():
+@pytest.mark.parametrize("N,K", [(16, 2), (152, 7)])   # groups only; groups and solo CTAs
+def test_group_barrier_and_ring_time_out_and_context_stays_usable(N, K):
     """One ring copy of every CTA is left unarmed: its waits run out (50 ms), the CTAs that gave
     up still publish their rows' mailbox words (so no window's exchange waits the whole limit),
     and the call returns with AAL_ERR_TIMEOUT recorded."""
-    t, d, _ = _inputs(16, 2, 20000, seed=11)
+    t, d, _ = _inputs(N, K, 20000, seed=11)
     prob = aal.loss_problem(d, B, 1.0, 0.5, 0.5)
     ws = torch.empty(aal.aal_workspace_size(prob), dtype=torch.uint8, device=DEV)
     loss = torch.empty(1, device=DEV)
