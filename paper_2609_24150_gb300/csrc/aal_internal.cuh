@@ -355,7 +355,26 @@ struct FusedIdsArgs {
   BackwardArgs bw;   // the gradient pass
   WindowArgs win;    // the window terms
   int32_t groups;    // G
+  int32_t solos;     // S solo CTAs after the groups' G K, each taking whole windows
+  int64_t n_group;   // windows 0 .. n_group - 1 go to the groups, the rest to the solo CTAs
 };
+
+// Windows per solo CTA for the fused kernels: G groups finish a window each in one row's time,
+// each of S solo CTAs one in K row times, so with m windows per solo CTA the launch ends after
+// max(ceil((N - m S) / G), m K) row times.  The best m near the balance point N / (G K + S),
+// or 0 (no solo CTAs) when none shortens the launch.
+inline int64_t solo_windows_each(int64_t N, int64_t K, int64_t G, int64_t S) {
+  if (S <= 0 || G <= 0) return 0;
+  auto cost = [&](int64_t m) {
+    const int64_t a = (N - m * S + G - 1) / G, b = m * K;
+    return a > b ? a : b;
+  };
+  int64_t best = 0;
+  const int64_t m0 = N / (G * K + S);
+  for (int64_t m = m0; m <= m0 + 1; ++m)
+    if (m > 0 && m * S <= N && cost(m) < cost(best)) best = m;
+  return best;
+}
 
 // GRPO over sequences (aal_seq_grpo_from_loss): per-position flags and log pi_ref from the
 // reference pass, the windows' rows gathered from them, and the windows' coefficients before

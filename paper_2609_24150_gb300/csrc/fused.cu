@@ -32,8 +32,6 @@
 // * Failure: every wait is bounded.  A CTA that gave up keeps walking its rows without waiting
 //   and still publishes a word for each, so its group does not wait on it for the whole limit;
 //   the workspace status word reports AAL_ERR_TIMEOUT and the outputs are not to be used.
-#include <algorithm>
-
 #include "grad_elem.cuh"
 #include "stream_core.cuh"
 
@@ -502,23 +500,13 @@ cudaError_t go_fused(const FusedArgs& f0, cudaStream_t s, uint64_t limit_ns, boo
   if (G > f0.win.N) G = f0.win.N;
   if (G > kMaxGroups) G = kMaxGroups;
   if (!coop || G < 1) return cudaSuccess;  // *launched stays false: the caller runs the two calls
-  // The SMs left over by the groups (sms per_sm - G K of them) take whole windows alone: a
-  // group finishes a window in one row's time, a solo CTA in K, so with m windows per solo CTA
-  // the step ends after max(ceil((N - m S) / G), m K) row times.  Take the best m near the
-  // balance point N / (G K + S), or no solo CTAs.
-  const int64_t N = f0.win.N;
+  // the SMs left over by the groups take whole windows alone
   const int64_t S = (int64_t)sms * per_sm - G * K;
-  int64_t best_m = 0;
-  if (S > 0) {
-    auto cost = [&](int64_t m) { return std::max((N - m * S + G - 1) / G, m * K); };
-    const int64_t m0 = N / (G * K + S);
-    for (int64_t m = m0; m <= m0 + 1; ++m)
-      if (m > 0 && m * S <= N && cost(m) < cost(best_m)) best_m = m;
-  }
+  const int64_t m = solo_windows_each(f0.win.N, K, G, S);
   FusedArgs f = f0;
   f.groups = (int32_t)G;
-  f.solos = best_m > 0 ? (int32_t)S : 0;
-  f.n_group = N - best_m * f.solos;
+  f.solos = m > 0 ? (int32_t)S : 0;
+  f.n_group = f0.win.N - m * f.solos;
   const int elt = 2;
   const int nch = (int)((f.st.V + kHalfSlot / elt - 1) / (kHalfSlot / elt));
   void* args[] = {&f, (void*)&nch, &limit_ns};

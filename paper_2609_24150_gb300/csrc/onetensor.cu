@@ -483,12 +483,17 @@ cudaError_t launch_T(const Stream1Args& a, bool ids, cudaStream_t s) {
 // for the gradient -dloss/|W| w_g dE/da a^g (delta_{u,x*} - q(u)).  Statistics, exchange and
 // coefficients reuse the IDS stream's and the backward's code, so the results are bitwise those
 // of aal_loss_fwd + aal_loss_bwd; resolve_draft_argmax and the window kernel run after it.
+// The SMs that G K leaves over take whole windows as solo CTAs, as in fused.cu.
 constexpr int kRBarCoef = 3;
 
 struct FusedIdsSmem {
   RefSmem s;
   RowCoef coef;
   int32_t live;
+  // a solo CTA's window: its rows' statistics, then their coefficients
+  RowStat solo_st[AAL_MAX_K];
+  RowCoef solo_coef[AAL_MAX_K];
+  int32_t solo_live[AAL_MAX_K];
 };
 
 constexpr size_t kFIdsSmemBytes = (size_t)kRSlots * kRSlotBytes + sizeof(FusedIdsSmem);
@@ -509,7 +514,10 @@ __global__ void __launch_bounds__(kRThreads, 1) fused_ids_rows(FusedIdsArgs f, i
   const int K = f.win.K;
   const int64_t N = f.win.N;
   const int G = f.groups;
-  const int g = blockIdx.x / K, k = blockIdx.x % K;
+  const int64_t NG = f.n_group;  // windows 0 .. NG - 1 go to the groups, the rest to the solo CTAs
+  const bool solo = (int)blockIdx.x >= G * K;
+  const int g = blockIdx.x / K, k = blockIdx.x % K;  // (a group's CTA)
+  const int so = (int)blockIdx.x - G * K;            // (a solo CTA)
 
   if (threadIdx.x == 0) {
     for (int q = 0; q < kRSlots; ++q) {
@@ -528,25 +536,36 @@ __global__ void __launch_bounds__(kRThreads, 1) fused_ids_rows(FusedIdsArgs f, i
       int slot = 0;
       uint32_t phase = 0, armed = 0, last_phase = 0;
       int64_t seq = 0;
-      for (int64_t n = g; n < N && !*abort_flag; n += G) {
-        const char* row = static_cast<const char*>(a.z) + (n * K + k) * a.V * 2;
-        for (int pass = 0; pass < 2 && !*abort_flag; ++pass) {  // statistics (kept in L2), gradient
-          const uint64_t pol = pass == 0 ? keep : drop;
-          for (int c = 0; c < nch; ++c, ++seq) {
-            if (!wait_phase(&S.empty[slot], phase ^ 1u, abort_flag, limit_ns, hdr)) break;
-            const int e0 = c * CH;
-            const uint32_t bytes = (uint32_t)(min(CH, V - e0) * 2);
-            if (seq != a.skip_chunk) {  // (the test hook leaves one chunk's barrier unarmed)
-              mbar_expect_tx(&S.full[slot], bytes);
-              bulk_load(ring + slot * kRSlotBytes, row + (int64_t)e0 * 2, bytes, &S.full[slot], pol);
-              armed |= 1u << slot;
-              last_phase = (last_phase & ~(1u << slot)) | (phase << slot);
-            }
-            if (++slot == kRSlots) {
-              slot = 0;
-              phase ^= 1u;
-            }
+      // pass 0 (statistics, kept in L2) or 1 (gradient, the row's last use) of row r
+      auto issue = [&](int64_t r, int pass) {
+        const char* row = static_cast<const char*>(a.z) + r * a.V * 2;
+        const uint64_t pol = pass == 0 ? keep : drop;
+        for (int c = 0; c < nch && !*abort_flag; ++c, ++seq) {
+          if (!wait_phase(&S.empty[slot], phase ^ 1u, abort_flag, limit_ns, hdr)) break;
+          const int e0 = c * CH;
+          const uint32_t bytes = (uint32_t)(min(CH, V - e0) * 2);
+          if (seq != a.skip_chunk) {  // (the test hook leaves one chunk's barrier unarmed)
+            mbar_expect_tx(&S.full[slot], bytes);
+            bulk_load(ring + slot * kRSlotBytes, row + (int64_t)e0 * 2, bytes, &S.full[slot], pol);
+            armed |= 1u << slot;
+            last_phase = (last_phase & ~(1u << slot)) | (phase << slot);
           }
+          if (++slot == kRSlots) {
+            slot = 0;
+            phase ^= 1u;
+          }
+        }
+      };
+      if (!solo) {
+        for (int64_t n = g; n < NG && !*abort_flag; n += G) {
+          issue(n * K + k, 0);
+          issue(n * K + k, 1);
+        }
+      } else {
+        // a whole window: the statistics of its K rows, then their gradients
+        for (int64_t n = NG + so; n < N && !*abort_flag; n += f.solos) {
+          for (int kk = 0; kk < K; ++kk) issue(n * K + kk, 0);
+          for (int kk = 0; kk < K; ++kk) issue(n * K + kk, 1);
         }
       }
       for (int q = 0; q < kRSlots; ++q) {
@@ -561,18 +580,19 @@ __global__ void __launch_bounds__(kRThreads, 1) fused_ids_rows(FusedIdsArgs f, i
     // ------------------------------------------------------------ consumers
     const int t = threadIdx.x;
     int slot = 0;
-    uint32_t phase = 0, j = 0;
-    float scale = 0.f;  // thread 0: -dloss / |W|
+    uint32_t phase = 0, j = 0;  // j: rows walked (parity of the reduction buffers)
+    float scale = 0.f;          // thread 0: -dloss / |W|
     if (t == 0) {
       const int nvalid = hdr->nvalid;
       scale = nvalid > 0 ? -f.bw.dloss / (float)nvalid : 0.f;
     }
-    for (int64_t n = g; n < N; n += G, ++j) {
-      const int64_t r = n * K + k;
+
+    // ---- pass 1 of row r: the draft's normaliser and greedy token (HBM), written to the
+    // workspace; thread 0 gets what the row's coefficients need
+    auto stats_row = [&](int64_t r, RowStat& st) {
       const int32_t xs = a.ids[r];
       const bool x_ok = xs >= 0 && xs < V;
       const int cx = x_ok ? xs / CH : -1, ix = x_ok ? (xs - cx * CH) / E : 0, ex = x_ok ? xs % E : 0;
-      // ---- pass 1: the draft's normaliser and greedy token (HBM)
       RefPart A;
       refpart_init(A);
       for (int c = 0; c < nch; ++c) {
@@ -601,7 +621,6 @@ __global__ void __launch_bounds__(kRThreads, 1) fused_ids_rows(FusedIdsArgs f, i
       refpart_warp(A);
       if (lane == 0) S.red[j & 1][warp] = A;
       named_barrier(kRBarRow, kRConsumers);
-      RowStat st{};  // thread 0: what the row's coefficients need
       if (t == 0) {
         RefPart tot = S.red[j & 1][0];
         for (int w = 1; w < kRWarps; ++w) {
@@ -623,38 +642,28 @@ __global__ void __launch_bounds__(kRThreads, 1) fused_ids_rows(FusedIdsArgs f, i
         st.ag = x_ok ? exp2f(log2_prob(zx, kLog2e, tot.M, Ls)) : 0.f;
         st.xs = x_ok ? xs : -1;
       }
-      // ---- the window's a^greedy (warp 0: lane j polls depth j), the row's coefficients (thread 0)
-      if (warp == 0) {
-        const int64_t r0 = n * K;
-        float agv[AAL_MAX_K], asv[AAL_MAX_K];
-        const bool ok = window_exchange(a.lws.mbox, r, r0, K, lane, st.ag, 0.f, true, abort_flag, hdr, limit_ns,
-                                        agv, asv);
-        if (lane == 0) {
-          int32_t live = 0;
-          if (ok) {
-            int kn = K;
-            if (f.win.mask != nullptr) {
-              kn = 0;
-              while (kn < K && f.win.mask[r0 + kn] != 0) ++kn;
-            }
-            float dE[AAL_MAX_K];
-            window_term(agv, kn, dE);
-            const bool pos_valid = f.bw.mask == nullptr || f.bw.mask[r] != 0;
-            RowCoef c;
-            live = row_coef<true, false, false>(f.bw, scale, 0.f, f.bw.w_greedy != 0.f ? dE[k] : 0.f, 0.f, 0.f,
-                                                pos_valid, st, c)
-                       ? 1
-                       : 0;
-            F.coef = c;
-          }
-          F.live = live;
-        }
-      }
-      named_barrier(kRBarCoef, kRConsumers);
+      ++j;
+    };
 
-      // ---- pass 3: the gradient row (L2)
-      const int32_t live = F.live;
-      const RowCoef c = F.coef;
+    // Thread 0: the coefficients of depth kk of window n (row r) from the window's a^greedy
+    // (agv), as the window kernel forms its terms and the backward its coefficients.
+    auto coef_row = [&](int64_t n, int kk, int64_t r, const float* agv, const RowStat& st, RowCoef& c) -> int32_t {
+      int kn = K;
+      if (f.win.mask != nullptr) {
+        kn = 0;
+        while (kn < K && f.win.mask[n * K + kn] != 0) ++kn;
+      }
+      float dE[AAL_MAX_K];
+      window_term(agv, kn, dE);
+      const bool pos_valid = f.bw.mask == nullptr || f.bw.mask[r] != 0;
+      return row_coef<true, false, false>(f.bw, scale, 0.f, f.bw.w_greedy != 0.f ? dE[kk] : 0.f, 0.f, 0.f,
+                                          pos_valid, st, c)
+                 ? 1
+                 : 0;
+    };
+
+    // ---- pass 2 of row r: the gradient row (L2)
+    auto grad_row = [&](int64_t r, const RowCoef& c, int32_t live) {
       const int64_t xv = (live && c.xs >= 0) ? c.xs / E : -1;
       const int xe = c.xs >= 0 ? c.xs % E : 0;
       uint4* out4 = reinterpret_cast<uint4*>(static_cast<T*>(f.bw.grad) + r * a.V);
@@ -685,6 +694,54 @@ __global__ void __launch_bounds__(kRThreads, 1) fused_ids_rows(FusedIdsArgs f, i
           phase ^= 1u;
         }
       }
+    };
+
+    if (!solo) {
+      // one row of each of the group's windows: statistics, the window exchange (warp 0: lane j
+      // polls depth j), the coefficients (thread 0), the gradient
+      for (int64_t n = g; n < NG; n += G) {
+        const int64_t r = n * K + k;
+        RowStat st{};
+        stats_row(r, st);
+        if (warp == 0) {
+          float agv[AAL_MAX_K], asv[AAL_MAX_K];
+          const bool ok = window_exchange(a.lws.mbox, r, n * K, K, lane, st.ag, 0.f, true, abort_flag, hdr, limit_ns,
+                                          agv, asv);
+          if (lane == 0) {
+            RowCoef c;
+            F.live = ok ? coef_row(n, k, r, agv, st, c) : 0;
+            if (F.live) F.coef = c;
+          }
+        }
+        named_barrier(kRBarCoef, kRConsumers);
+        const RowCoef c = F.coef;
+        grad_row(r, c, F.live);
+      }
+    } else {
+      // whole windows: the statistics of the K rows, their coefficients from those rows alone
+      // (no exchange), then the K gradient rows
+      for (int64_t n = NG + so; n < N; n += f.solos) {
+        for (int kk = 0; kk < K; ++kk) {
+          RowStat st{};
+          stats_row(n * K + kk, st);
+          if (t == 0) F.solo_st[kk] = st;
+        }
+        if (t == 0) {
+          float agv[AAL_MAX_K];
+#pragma unroll
+          for (int jj = 0; jj < AAL_MAX_K; ++jj) agv[jj] = jj < K ? F.solo_st[jj].ag : 0.f;
+          for (int kk = 0; kk < K; ++kk) {
+            RowCoef c;
+            F.solo_live[kk] = !*abort_flag ? coef_row(n, kk, n * K + kk, agv, F.solo_st[kk], c) : 0;
+            if (F.solo_live[kk]) F.solo_coef[kk] = c;
+          }
+        }
+        named_barrier(kRBarCoef, kRConsumers);
+        for (int kk = 0; kk < K; ++kk) {
+          const RowCoef c = F.solo_coef[kk];
+          grad_row(n * K + kk, c, F.solo_live[kk]);
+        }
+      }
     }
   }
   __syncwarp();
@@ -710,12 +767,18 @@ cudaError_t launch_fused_ids(const FusedIdsArgs& f0, cudaStream_t s, uint64_t li
   if (G > f0.win.N) G = f0.win.N;
   if (G > kMaxGroups) G = kMaxGroups;
   if (!coop || G < 1) return cudaSuccess;
+  // the SMs left over by the groups take whole windows alone
+  const int64_t S = (int64_t)sms * per_sm - G * K;
+  const int64_t m = solo_windows_each(f0.win.N, K, G, S);
   FusedIdsArgs f = f0;
   f.groups = (int32_t)G;
+  f.solos = m > 0 ? (int32_t)S : 0;
+  f.n_group = f0.win.N - m * f.solos;
   const int CH = kRSlotBytes / 2;
   const int nch = (int)((f.st.V + CH - 1) / CH);
   void* args[] = {&f, (void*)&nch, &limit_ns};
-  e = cudaLaunchCooperativeKernel((const void*)kern, dim3((unsigned)(G * K)), dim3(kRThreads), args, kFIdsSmemBytes, s);
+  e = cudaLaunchCooperativeKernel((const void*)kern, dim3((unsigned)(G * K + f.solos)), dim3(kRThreads), args,
+                                  kFIdsSmemBytes, s);
   if (e == cudaErrorCooperativeLaunchTooLarge) {  // fewer SMs available: the caller runs the two calls
     cudaGetLastError();
     return cudaSuccess;

@@ -138,7 +138,8 @@ def test_problems_the_two_calls_take(mode, T, dtype, V):
 
 
 @pytest.mark.parametrize("N,K,V,masked", [(10, 3, 4096, False), (40, 7, 30000, True), (3, 8, 128256, False),
-                                           (100, 1, 1000, True), (20, 5, 8, True)])
+                                           (100, 1, 1000, True), (20, 5, 8, True),
+                                           (152, 7, 4096, True), (304, 5, 2000, False)])   # with solo CTAs
 @pytest.mark.parametrize("dloss_is_w", [False, True])
 def test_token_ids_fused_equals_two_calls(N, K, V, masked, dloss_is_w):
     """x* as token ids (the draft alone streamed), some ids out of range on one run."""
@@ -166,14 +167,15 @@ def test_token_ids_out_of_range_reported():
     assert torch.equal(_bits(grad), _bits(s))
 
 
-def test_token_ids_ring_times_out_and_context_stays_usable():
-    t, d, _ = _inputs(16, 2, 40000, seed=12)
+@pytest.mark.parametrize("N,K", [(16, 2), (152, 7)])   # groups only; groups and solo CTAs
+def test_token_ids_ring_times_out_and_context_stays_usable(N, K):
+    t, d, _ = _inputs(N, K, 40000, seed=12)
     ids = t.float().argmax(-1).to(torch.int32).contiguous()
     prob = aal.loss_problem(d, G | IDS, 1.0, 1.0, 0.0)
     ws = torch.empty(aal.aal_workspace_size(prob), dtype=torch.uint8, device=DEV)
     loss = torch.empty(1, device=DEV)
     grad = torch.empty_like(d)
-    aal.aal_debug_fail_next_forward(2, 50_000_000)    # a chunk of the gradient pass
+    aal.aal_debug_fail_next_forward(2, 50_000_000)    # a group's gradient chunk, a solo CTA's statistics chunk
     try:
         aal.aal_loss_fwd_bwd(prob, d, ids, None, ws, 1.0, loss, grad)
         assert aal.aal_check_device_status(ws) == aal.AAL_ERR_TIMEOUT
