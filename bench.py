@@ -268,7 +268,7 @@ def run_ours(args, ws_count, rank, local):
     fb_bytes = b["fwd"] + b["bwd"]
     min_traffic = 3 * R * V * draft.element_size()
     achieved = fb_bytes / (per["fwd_bwd"] * 1e-3) / 1e9
-    traffic = recorded_traffic("fused")
+    traffic = recorded_traffic("fused") if args.windows is None else None  # recorded at the full batch
 
     res = {
         "metric": "fused EAL/WTV fwd+bwd GB/s and logit-rows/s at V=128256 (with the GRPO acceptance reward)",
