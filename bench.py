@@ -724,13 +724,40 @@ def recorded_traffic(which):
     return rec["dram_bytes_per_launch"] if sha is not None and sha == rec["sources_sha256_16"] else None
 
 
+def code_text(src):
+    """C/CUDA source without its comments, trailing blanks and empty lines: the part of a file
+    that can change the compiled kernel (string and character literals are kept whole)."""
+    out, i, n = [], 0, len(src)
+    while i < n:
+        c = src[i]
+        if c in "\"'":
+            j = i + 1
+            while j < n and src[j] != c:
+                j += 2 if src[j] == "\\" else 1
+            out.append(src[i:j + 1])
+            i = j + 1
+        elif src.startswith("//", i):
+            j = src.find("\n", i)
+            i = n if j < 0 else j
+        elif src.startswith("/*", i):
+            j = src.find("*/", i + 2)
+            i = n if j < 0 else j + 2
+        else:
+            out.append(c)
+            i += 1
+    lines = (line.rstrip() for line in "".join(out).splitlines())
+    return "\n".join(line for line in lines if line)
+
+
 def sources_sha(names):
-    """First 16 hex digits of the SHA-256 of the named csrc files, concatenated in order."""
+    """First 16 hex digits of the SHA-256 of the named csrc files' code (code_text), concatenated
+    in order: a comment edit keeps a recorded capture valid, a code edit voids it."""
     h = hashlib.sha256()
     try:
         for n in names:
-            with open(os.path.join(ROOT, "paper_2609_24150_gb300", "csrc", n), "rb") as f:
-                h.update(f.read())
+            with open(os.path.join(ROOT, "paper_2609_24150_gb300", "csrc", n), encoding="utf-8") as f:
+                h.update(code_text(f.read()).encode())
+                h.update(b"\0")
     except OSError:
         return None
     return h.hexdigest()[:16]

@@ -9,19 +9,19 @@
 // The logits cross HBM once per step instead of twice.
 //
 // * Launch: cooperative, one CTA per SM (the ring takes ~193 KB of shared memory), grid =
-//   G groups x K CTAs; CTA k of group g takes depth k of windows g, g + G, ...  A cooperative
-//   launch has all its CTAs resident at once, so a group never waits on a CTA that is not
-//   running.
-// * Solo CTAs: the SMs that G K leaves over (152 - 147 at K = 7) each take whole windows of
-//   the last windows: the statistics of the window's K rows one after another, the K rows'
-//   coefficients from its own acceptances (no exchange), then the K gradient rows.  The host
-//   gives them as many windows as balances the two kinds; their rows stay in L2 across K rows'
-//   time instead of one.
+//   G groups x K CTAs + S solo CTAs; CTA k of group g takes depth k of windows g, g + G, ...
+//   A cooperative launch has all its CTAs resident at once, so a group never waits on a CTA
+//   that is not running.
+// * Solo CTAs: the S = 152 - G K SMs the groups leave over (5 at K = 7) each take whole
+//   windows from the end of the batch: the statistics of the window's K rows one after
+//   another, the K rows' coefficients from its own acceptances (no exchange), then the K
+//   gradient rows.  The host gives them as many windows as balances the two kinds
+//   (solo_windows_each); their rows stay in L2 for K rows' time instead of one.
 // * Window exchange: once its row's statistics are in the workspace, thread 0 of each CTA
 //   publishes the row's (a^greedy, a^sample) as one 64-bit word in a per-row mailbox that the
 //   call filled with an all-ones sentinel, and warp 0 polls (bounded, like the ring waits; lane
-//   j the word of depth j) the K words of its window until none is the sentinel: the value is its own ready flag, so one L2 round
-//   trip brings the data.  It then forms dE^g/da and dE^s/da with the window kernels' function
+//   j the word of depth j) the K words of its window until none is the sentinel.  The value is
+//   its own ready flag, so one L2 round trip brings the data.  It then forms dE^g/da and dE^s/da with the window kernels' function
 //   (window_term) and the row's gradient coefficients with the backward's (row_coef), from the
 //   same floats the window kernel reads later, so that the gradient equals the one of
 //   aal_loss_fwd + aal_loss_bwd bit for bit.  The loss is left to the window kernel, which runs
