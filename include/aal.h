@@ -152,7 +152,8 @@ AAL_API aal_status aal_loss_bwd(const aal_problem* prob, const void* draft, cons
  * that is a fixed weight times the objective).  The result equals the two calls; the
  * difference is the traffic.  With bf16 rows whose byte length is a multiple of 16, the
  * K rows of each window are streamed by K CTAs together (one cooperative launch, one CTA
- * per SM), and the gradient is written while the rows are still in L2: the logits are read
+ * per SM; the SMs left over take whole windows alone), and the gradient is written while
+ * the rows are still in L2: the logits are read
  * from HBM once (2 V b per row, plus V b gradient written) instead of twice (the separate
  * forward's 2 V b and the backward's 3 V b).  With token ids (AAL_GREEDY | AAL_IDS) only the
  * draft is streamed the same way: V b read and V b written per row, instead of V b + 2 V b.
