@@ -157,8 +157,7 @@ AAL_API aal_status aal_loss_bwd(const aal_problem* prob, const void* draft, cons
  * from HBM once (2 V b per row, plus V b gradient written) instead of twice (the separate
  * forward's 2 V b and the backward's 3 V b).  With token ids (AAL_GREEDY | AAL_IDS) only the
  * draft is streamed the same way: V b read and V b written per row, instead of V b + 2 V b.
- * Other problems (fp32, unaligned rows, the anchor beside a sampling term at T != 1) run the
- * two calls inside this one.
+ * Other problems (fp32, unaligned rows) run the two calls inside this one.
  * AAL_GRPO is rejected with AAL_ERR_UNSUPPORTED: its coefficients come from
  * aal_grpo_from_loss, between the forward and the backward.  A bounded device wait that ran
  * out (a ring copy, or the group barrier between the K CTAs of a window) is reported by

@@ -301,12 +301,10 @@ aal_status aal_loss_fwd_bwd(const aal_problem* prob, const void* draft, const vo
   const LossLayout L = loss_layout(prob->N, prob->K);
   if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < L.total) return AAL_ERR_WORKSPACE;
 
-  // the fused kernels: bf16 rows of 16-byte multiples; with logits, (as for the streamed
-  // forward) the anchor beside a sampling term only at T = 1; with token ids, the draft alone
-  const bool sampling = (prob->mode & (AAL_SAMPLING | AAL_TV)) != 0, kl = (prob->mode & AAL_KL) != 0;
+  // the fused kernels: bf16 rows of 16-byte multiples; with token ids, the draft alone
   const bool ids = (prob->mode & AAL_IDS) != 0;
   const bool rows16 = prob->dtype == AAL_BF16 && (prob->V * 2) % 16 == 0;
-  const bool fusable = rows16 && !ids && !(kl && sampling && prob->temperature != 1.0f);
+  const bool fusable = rows16 && !ids;
   if (rows16 && ids) {
     LossWs ws = loss_ws(workspace, L);
     if (cudaMemsetAsync(ws.hdr, 0, sizeof(WsHeader), s) != cudaSuccess) return AAL_ERR_CUDA;

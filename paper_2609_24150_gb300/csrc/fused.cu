@@ -53,9 +53,9 @@ struct FusedSmem {
 
 constexpr size_t kFusedSmemBytes = (size_t)kSlots * kSlotBytes + sizeof(FusedSmem);
 
-// PASSES = 2 with the sampling (or TV) term, 1 without; NEED_Q1, KL as in rowstats_stream;
+// PASSES = 2 with the sampling (or TV) term, 1 without; NEED_Q1, KL, P1 as in rowstats_stream;
 // GREEDY and Q1_IS_QT as in the backward.  bf16 rows only (16-byte multiples).
-template <bool NEED_Q1, int PASSES, bool KL, bool GREEDY, bool Q1_IS_QT>
+template <bool NEED_Q1, int PASSES, bool KL, bool GREEDY, bool Q1_IS_QT, bool P1 = false>
 __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, uint64_t limit_ns) {
   using T = uint16_t;
   constexpr bool SAMPLING = PASSES == 2;
@@ -175,34 +175,35 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
               pv[v] = P[t + v * kConsumers];
               qv[v] = Q[t + v * kConsumers];
             }
-            phase1_bf16<kNV, NEED_Q1, KL>(A, pv, qv, e0 + t * E, kConsumers * E, sT);
+            phase1_bf16<kNV, NEED_Q1, KL, P1>(A, pv, qv, e0 + t * E, kConsumers * E, sT);
           } else {
             const int nvec = (V - e0) / E;
-            for (int i = t; i < nvec; i += kConsumers) phase1_bf16<1, NEED_Q1, KL>(A, P + i, Q + i, e0 + i * E, 0, sT);
+            for (int i = t; i < nvec; i += kConsumers)
+              phase1_bf16<1, NEED_Q1, KL, P1>(A, P + i, Q + i, e0 + i * E, 0, sT);
           }
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&S.empty[pos.slot]);
       }
-      warp_part<NEED_Q1, KL>(A, sT);
+      warp_part<NEED_Q1, KL, P1>(A, sT);
       if (lane == 0) S.red[j & 1][warp] = A;
       named_barrier(kBarRow, kConsumers);
       RowPart tot;
       if (lane < kWarps) tot = S.red[j & 1][lane];
       else part_init(tot);
-      warp_part<NEED_Q1, KL>(tot, sT);
+      warp_part<NEED_Q1, KL, P1>(tot, sT);
       const float Mp = tot.pM, Lsp = log2f(tot.pS);
       const float Mq = tot.qM, Lsq = log2f(tot.qS);
-      if (KL && t == 0) {  // both normalisers are at T = 1 here
-        const float Mq1 = NEED_Q1 ? tot.q1M : Mq;
-        const float Lsq1 = NEED_Q1 ? log2f(tot.q1S) : Lsq;
+      if (KL && t == 0) {
+        float Mp1, Lsp1, kl;
+        kl_stats<NEED_Q1, P1>(tot, Mp, Lsp, Mq, Lsq, Mp1, Lsp1, kl);
         if (!*abort_flag) {
-          a.ws.Mp1[r] = Mp;
-          a.ws.Lsp1[r] = Lsp;
-          a.ws.kl[r] = tot.pD / tot.pS - (Mp - Mq1) - kLn2 * (Lsp - Lsq1);
+          a.ws.Mp1[r] = Mp1;
+          a.ws.Lsp1[r] = Lsp1;
+          a.ws.kl[r] = kl;
         }
-        st.Mp1 = Mp;
-        st.Lsp1 = Lsp;
+        st.Mp1 = Mp1;
+        st.Lsp1 = Lsp1;
       }
       if (PASSES == 1) {
         if (t == 0) {
@@ -484,9 +485,9 @@ __global__ void __launch_bounds__(1024) count_valid(const uint8_t* mask, int64_t
   }
 }
 
-template <bool NQ1, int P, bool KL, bool GR, bool Q>
+template <bool NQ1, int P, bool KL, bool GR, bool Q, bool P1 = false>
 cudaError_t go_fused(const FusedArgs& f0, cudaStream_t s, uint64_t limit_ns, bool* launched) {
-  auto kern = fused_rows<NQ1, P, KL, GR, Q>;
+  auto kern = fused_rows<NQ1, P, KL, GR, Q, P1>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFusedSmemBytes);
   if (e != cudaSuccess) return e;
   int dev = 0, sms = 0, per_sm = 0, coop = 0;
@@ -540,10 +541,14 @@ cudaError_t launch_fused(const FusedArgs& f, cudaStream_t s, uint64_t limit_ns, 
     if (greedy && kl) return go_fused<false, 1, true, true, false>(f, s, limit_ns, launched);
     return cudaSuccess;
   }
-  if (kl) {
-    if (nq1 || !q) return cudaSuccess;
-    return greedy ? go_fused<false, 2, true, true, true>(f, s, limit_ns, launched)
-                  : go_fused<false, 2, true, false, true>(f, s, limit_ns, launched);
+  if (kl) {  // at T = 1 q = q~ (one z_q state); else z_q and z_p both kept at T = 1 beside T
+    if (q && !nq1)
+      return greedy ? go_fused<false, 2, true, true, true>(f, s, limit_ns, launched)
+                    : go_fused<false, 2, true, false, true>(f, s, limit_ns, launched);
+    if (nq1 && !q)
+      return greedy ? go_fused<true, 2, true, true, false, true>(f, s, limit_ns, launched)
+                    : go_fused<true, 2, true, false, false, true>(f, s, limit_ns, launched);
+    return cudaSuccess;
   }
   if (!greedy && !nq1 && !q) return go_fused<false, 2, false, false, false>(f, s, limit_ns, launched);
   if (greedy && !nq1 && q) return go_fused<false, 2, false, true, true>(f, s, limit_ns, launched);

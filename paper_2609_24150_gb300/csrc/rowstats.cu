@@ -252,9 +252,7 @@ cudaError_t launch_rowstats(const RowStatsArgs& a, bool bf16, cudaStream_t s, in
   const int elt = bf16 ? 2 : 4;
   const bool aligned = ((a.V * elt) % 16 == 0) &&
                        ((reinterpret_cast<uintptr_t>(a.zq) | reinterpret_cast<uintptr_t>(a.zp)) % 16 == 0);
-  // the streamed kernel takes the KL anchor only where the z_p normaliser it keeps is at T = 1
-  const bool kl_ok = !a.need_kl || !a.overlap || a.sT == kLog2e;
-  if (aligned && kl_ok) {
+  if (aligned) {
     *cluster_used = 1;
     const uint64_t limit = debug_wait_limit_ns();
     return launch_rowstats_stream(a, bf16, s, limit ? limit : kWaitLimitNs);

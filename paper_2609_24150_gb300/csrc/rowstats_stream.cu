@@ -21,7 +21,8 @@
 // where the normalisers of z_p and z_q are those of p and q themselves.  The first pass
 // finds the argmaxes only to the 16-byte vector; resolve_argmax then reads those two
 // vectors of each row again (64 bytes) to place x* and y exactly.  With the KL anchor the
-// first pass also folds D = sum_v e_v (z_p,v - z_q,v) next to the log-sum-exp of z_p.
+// first pass also folds D = sum_v e_v (z_p,v - z_q,v) next to the log-sum-exp of z_p at
+// T = 1; beside a sampling term at T != 1 that is a second z_p state, next to the one at T.
 //
 // There is no cross-CTA communication, so all 152 SMs run one CTA each.  Every wait is
 // bounded (ptx::wait_phase); after a timeout every thread keeps walking the same loops
@@ -38,8 +39,9 @@ using namespace ptx;
 
 // PASSES = 2: the sampling term (normalisers at T, then the overlap sums).  PASSES = 1: no
 // sampling term; everything at T = 1 (sT is log2 e), argmaxes resolved by resolve_argmax.
-// KL: the anchor's D next to the z_p normaliser (which must then be at T = 1).
-template <typename T, bool NEED_Q1, int PASSES, bool KL>
+// KL: the anchor's D next to the z_p normaliser at T = 1: the pass's own when it runs at T = 1,
+// else (P1, with NEED_Q1) a second z_p state at T = 1 beside the one at T.
+template <typename T, bool NEED_Q1, int PASSES, bool KL, bool P1 = false>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm) rowstats_stream(RowStatsArgs a, int nch, uint64_t limit_ns) {
   extern __shared__ __align__(1024) unsigned char smem[];
   unsigned char* ring = smem;
@@ -128,34 +130,34 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) rowstats_stream(RowStats
               pv[v] = P[t + v * kConsumers];
               qv[v] = Q[t + v * kConsumers];
             }
-            phase1_bf16<kNV, NEED_Q1, KL>(A, pv, qv, e0 + t * E, kConsumers * E, sT);
+            phase1_bf16<kNV, NEED_Q1, KL, P1>(A, pv, qv, e0 + t * E, kConsumers * E, sT);
           } else {
             const int nvec = min(CH, V - e0) / E;
             for (int i = t; i < nvec; i += kConsumers) {
-              if (sizeof(T) == 2) phase1_bf16<1, NEED_Q1, KL>(A, P + i, Q + i, e0 + i * E, 0, sT);
-              else phase1_vec<T, NEED_Q1, KL>(A, P[i], Q[i], e0 + i * E, sT);
+              if (sizeof(T) == 2) phase1_bf16<1, NEED_Q1, KL, P1>(A, P + i, Q + i, e0 + i * E, 0, sT);
+              else phase1_vec<T, NEED_Q1, KL, P1>(A, P[i], Q[i], e0 + i * E, sT);
             }
           }
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&S.empty[pos.slot]);
       }
-      warp_part<NEED_Q1, KL>(A, sT);
+      warp_part<NEED_Q1, KL, P1>(A, sT);
       if (lane == 0) S.red[j & 1][warp] = A;
       named_barrier(kBarRow, kConsumers);
       // every warp combines the warp partials itself (lanes >= kWarps carry the identity)
       RowPart tot;
       if (lane < kWarps) tot = S.red[j & 1][lane];
       else part_init(tot);
-      warp_part<NEED_Q1, KL>(tot, sT);
+      warp_part<NEED_Q1, KL, P1>(tot, sT);
       const float Mp = tot.pM, Lsp = log2f(tot.pS);
       const float Mq = tot.qM, Lsq = log2f(tot.qS);
-      if (KL && t == 0 && !*abort_flag) {  // both normalisers are at T = 1 here
-        const float Mq1 = NEED_Q1 ? tot.q1M : Mq;
-        const float Lsq1 = NEED_Q1 ? log2f(tot.q1S) : Lsq;
-        a.ws.Mp1[r] = Mp;
-        a.ws.Lsp1[r] = Lsp;
-        a.ws.kl[r] = tot.pD / tot.pS - (Mp - Mq1) - kLn2 * (Lsp - Lsq1);
+      if (KL && t == 0 && !*abort_flag) {
+        float Mp1, Lsp1, kl;
+        kl_stats<NEED_Q1, P1>(tot, Mp, Lsp, Mq, Lsq, Mp1, Lsp1, kl);
+        a.ws.Mp1[r] = Mp1;
+        a.ws.Lsp1[r] = Lsp1;
+        a.ws.kl[r] = kl;
       }
       if (PASSES == 1) {
         if (t == 0) {
@@ -266,9 +268,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) rowstats_stream(RowStats
 
 constexpr size_t kSmemBytes = (size_t)kSlots * kSlotBytes + sizeof(Smem);
 
-template <typename T, bool NEED_Q1, int PASSES, bool KL>
+template <typename T, bool NEED_Q1, int PASSES, bool KL, bool P1 = false>
 cudaError_t launch_T(const RowStatsArgs& a, cudaStream_t s, int nch, uint64_t limit_ns) {
-  auto kern = rowstats_stream<T, NEED_Q1, PASSES, KL>;
+  auto kern = rowstats_stream<T, NEED_Q1, PASSES, KL, P1>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
   if (e != cudaSuccess) return e;
   int dev = 0, sms = 0;
@@ -312,7 +314,9 @@ cudaError_t launch_one_pass(const RowStatsArgs& a, cudaStream_t s, int nch, uint
 
 template <typename T>
 cudaError_t launch_two_pass(const RowStatsArgs& a, cudaStream_t s, int nch, uint64_t limit_ns) {
-  if (a.need_kl) return launch_T<T, false, 2, true>(a, s, nch, limit_ns);  // T = 1: no separate q1
+  if (a.need_kl)  // at T = 1 the pass's normalisers are the anchor's; else both are kept
+    return a.need_q1 ? launch_T<T, true, 2, true, true>(a, s, nch, limit_ns)
+                     : launch_T<T, false, 2, true>(a, s, nch, limit_ns);
   return a.need_q1 ? launch_T<T, true, 2, false>(a, s, nch, limit_ns) : launch_T<T, false, 2, false>(a, s, nch, limit_ns);
 }
 

@@ -43,6 +43,8 @@ constexpr int kBarRow = 1, kBarSum = 2;
 struct RowPart {
   float pM, pS, qM, qS, q1M, q1S;  // online log2-sum-exp states (M = raw max of z)
   float pD;                        // KL anchor: sum 2^((z_p - pM) s) (z_p - z_q), rescaled with pS
+  float p1M, p1S;                  // KL anchor beside an overlap at T != 1 (P1): z_p at T = 1,
+                                   // and pD then rescales with p1S
   float av;                        // target: largest z_p and the first vector holding it
   int32_t ab;
   float qv;                        // draft: largest z_q and the first vector holding it
@@ -66,8 +68,8 @@ struct Smem {
 constexpr float kMaxFloor = -1e30f;
 
 __device__ __forceinline__ void part_init(RowPart& a) {
-  a.pM = a.qM = a.q1M = kMaxFloor;
-  a.pS = a.qS = a.q1S = 0.f;
+  a.pM = a.qM = a.q1M = a.p1M = kMaxFloor;
+  a.pS = a.qS = a.q1S = a.p1S = 0.f;
   a.pD = 0.f;
   a.av = -INFINITY;
   a.ab = 0x7fffffff;
@@ -113,10 +115,16 @@ __device__ __forceinline__ void warp_lse_kl(float& M, float& S, float& D, float 
   S = s;
   D = d;
 }
-template <bool NEED_Q1, bool KL = false>
+template <bool NEED_Q1, bool KL = false, bool P1 = false>
 __device__ __forceinline__ void warp_part(RowPart& a, float sT) {
-  if (KL) warp_lse_kl(a.pM, a.pS, a.pD, sT);
-  else warp_lse(a.pM, a.pS, sT);
+  if (KL && P1) {
+    warp_lse(a.pM, a.pS, sT);
+    warp_lse_kl(a.p1M, a.p1S, a.pD, kLog2e);
+  } else if (KL) {
+    warp_lse_kl(a.pM, a.pS, a.pD, sT);
+  } else {
+    warp_lse(a.pM, a.pS, sT);
+  }
   warp_lse(a.qM, a.qS, sT);
   if (NEED_Q1) warp_lse(a.q1M, a.q1S, kLog2e);
   warp_amax(a.av, a.ab);
@@ -196,7 +204,7 @@ __device__ __forceinline__ void first_vec_at(float& best, int32_t& at, const uin
 // idx0 + v * vstride + [0, 8).  The maxima are taken on packed bf16 pairs: per vector, then
 // over the thread's vectors; only a maximum that beats the running one looks for its vector
 // (the first in element order, as a strict per-vector update in that order would).
-template <int NV, bool NEED_Q1, bool KL = false>
+template <int NV, bool NEED_Q1, bool KL = false, bool P1 = false>
 __device__ __forceinline__ void phase1_bf16(RowPart& A, const uint4* pv, const uint4* qv, int idx0, int vstride,
                                             float sT) {
   constexpr int NW = 4 * NV;
@@ -227,8 +235,14 @@ __device__ __forceinline__ void phase1_bf16(RowPart& A, const uint4* pv, const u
   const float pm = fmaxf(bf16_lo(cp), bf16_hi(cp)), qm = fmaxf(bf16_lo(cq), bf16_hi(cq));
   if (pm > A.av) first_vec_at<NV>(A.av, A.ab, vp, pm, idx0, vstride);
   if (qm > A.qv) first_vec_at<NV>(A.qv, A.qb, vq, qm, idx0, vstride);
-  if (KL) lse_kl_words<NW>(A.pM, A.pS, A.pD, pw, qw, pm, sT);
-  else lse_words<NW>(A.pM, A.pS, pw, pm, sT);
+  if (KL && P1) {
+    lse_words<NW>(A.pM, A.pS, pw, pm, sT);
+    lse_kl_words<NW>(A.p1M, A.p1S, A.pD, pw, qw, pm, kLog2e);
+  } else if (KL) {
+    lse_kl_words<NW>(A.pM, A.pS, A.pD, pw, qw, pm, sT);
+  } else {
+    lse_words<NW>(A.pM, A.pS, pw, pm, sT);
+  }
   lse_words<NW>(A.qM, A.qS, qw, qm, sT);
   if (NEED_Q1) lse_words<NW>(A.q1M, A.q1S, qw, qm, kLog2e);
 }
@@ -328,7 +342,7 @@ __device__ __forceinline__ void lse_kl_vals(float& M, float& S, float& D, const 
   D += dacc;
 }
 
-template <typename T, bool NEED_Q1, bool KL = false>
+template <typename T, bool NEED_Q1, bool KL = false, bool P1 = false>
 __device__ __forceinline__ void phase1_vec(RowPart& A, const uint4& pw, const uint4& qw, int idx0, float sT) {
   constexpr int E = 16 / sizeof(T);
   float pv[8], qv[8];
@@ -342,10 +356,30 @@ __device__ __forceinline__ void phase1_vec(RowPart& A, const uint4& pw, const ui
   }
   amax_vec(A.av, A.ab, pm, idx0);
   amax_vec(A.qv, A.qb, qm, idx0);
-  if (KL) lse_kl_vals<E>(A.pM, A.pS, A.pD, pv, qv, pm, sT);
-  else lse_vals<E>(A.pM, A.pS, pv, pm, sT);
+  if (KL && P1) {
+    lse_vals<E>(A.pM, A.pS, pv, pm, sT);
+    lse_kl_vals<E>(A.p1M, A.p1S, A.pD, pv, qv, pm, kLog2e);
+  } else if (KL) {
+    lse_kl_vals<E>(A.pM, A.pS, A.pD, pv, qv, pm, sT);
+  } else {
+    lse_vals<E>(A.pM, A.pS, pv, pm, sT);
+  }
   lse_vals<E>(A.qM, A.qS, qv, qm, sT);
   if (NEED_Q1) lse_vals<E>(A.q1M, A.q1S, qv, qm, kLog2e);
+}
+
+// The anchor's row statistics from a row's reduced state (Mp, Lsp: z_p's normaliser at the
+// pass's temperature; Mq, Lsq: z_q's): z_p's normaliser at T = 1, kept apart when the
+// overlap runs at T != 1 (P1), and KL(p || q) = D / S_p - (Mp1 - Mq1) - ln 2 (Lsp1 - Lsq1)
+// in nats, with q's normaliser at T = 1.
+template <bool NEED_Q1, bool P1>
+__device__ __forceinline__ void kl_stats(const RowPart& tot, float Mp, float Lsp, float Mq, float Lsq, float& Mp1,
+                                         float& Lsp1, float& kl) {
+  const float Mq1 = NEED_Q1 ? tot.q1M : Mq;
+  const float Lsq1 = NEED_Q1 ? log2f(tot.q1S) : Lsq;
+  Mp1 = P1 ? tot.p1M : Mp;
+  Lsp1 = P1 ? log2f(tot.p1S) : Lsp;
+  kl = tot.pD / (P1 ? tot.p1S : tot.pS) - (Mp1 - Mq1) - kLn2 * (Lsp1 - Lsq1);
 }
 
 template <typename T>

@@ -134,7 +134,7 @@ KL_TV = aal.AAL_KL | aal.AAL_TV
 
 @pytest.mark.parametrize("mode,T,wtv", [
     (KL_TV, 1.0, 0.1),                                # the paper's L_KL + 0.1 L_TV baseline, T = 1
-    (KL_TV, 0.7, 0.1),                                # ... at T = 0.7 (generic kernel: anchor beside T != 1)
+    (KL_TV, 0.7, 0.1),                                # ... at T = 0.7 (z_p kept at T = 1 beside T)
     (aal.AAL_TV, 1.3, 1.0),                           # the TV term alone
     (aal.AAL_TV | aal.AAL_BOTH, 1.0, 0.5),            # beside EAL and WTV: one sampling coefficient
 ])

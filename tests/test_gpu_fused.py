@@ -4,7 +4,7 @@ It must give the loss, the per-window expected lengths and the gradient of aal_l
 by aal_loss_bwd bit for bit: on the fused path (bf16 rows of 16-byte multiples; every flag
 combination it instantiates, masks, fewer windows than CTA groups, K = 1 and K = 8, windows
 enough for the solo CTAs, full-size rows; token ids with the draft alone streamed) and on the problems it hands to the two calls
-(fp32, unaligned rows, the anchor beside the sampling term at T != 1).  A few cases are also checked against the oracle
+(fp32, unaligned rows).  A few cases are also checked against the oracle
 directly, and the bounded waits are driven to a timeout without a fault.
 """
 
@@ -70,6 +70,8 @@ CASES = [
     (20, 4, 3000, KL, 1.0, 0.0, 0.0, 1.0, 1.0, True),       # the anchor alone
     (12, 6, 6000, KL | B, 1.0, 0.1, 0.1, 1.0, 1.0, True),   # two passes with the anchor
     (12, 6, 6000, KL | TV, 1.0, 0.0, 0.0, 1.0, 0.1, False), # TV term + anchor, no greedy term
+    (10, 3, 4096, KL | S, 0.8, 0.5, 0.5, 1.0, 1.0, True),   # the anchor beside WTV at T != 1: z_p and z_q at 1 and T
+    (14, 5, 9000, KL | B, 1.5, 0.1, 0.5, 1.0, 1.0, False),  # ... and beside EAL too
     (3, 7, 128256, B, 1.0, 0.5, 0.5, 1.0, 1.0, False),      # fewer windows than groups, full rows
     (200, 1, 2048, B, 1.0, 0.5, 0.5, 1.0, 1.0, False),      # K = 1: groups of one CTA
     (30, 3, 8, B, 1.0, 0.5, 0.5, 1.0, 1.0, True),           # one 16-byte vector a row
@@ -88,6 +90,8 @@ SOLO_CASES = [
     (152, 6, 3000, KL, 1.0, 0.0, 0.0, 1.0, 1.0, True),
     (152, 5, 6000, KL | B, 1.0, 0.1, 0.1, 1.0, 1.0, True),
     (152, 7, 6000, KL | TV, 1.0, 0.0, 0.0, 1.0, 0.1, False),
+    (152, 5, 3000, KL | S, 0.8, 0.0, 1.0, 1.0, 1.0, True),
+    (152, 6, 2000, KL | B, 1.5, 0.1, 0.5, 1.0, 1.0, False),
 ]
 
 
@@ -130,7 +134,7 @@ def test_fused_no_valid_window():
 @pytest.mark.parametrize("mode,T,dtype,V", [
     (B, 1.0, torch.float32, 4096),        # fp32 logits
     (B, 1.0, torch.bfloat16, 1001),       # rows that are not 16-byte multiples
-    (KL | S, 0.8, torch.bfloat16, 4096),  # the anchor beside the sampling term at T != 1
+    (KL | S, 0.8, torch.float32, 4096),   # the anchor beside the sampling term at T != 1, fp32
 ])
 def test_problems_the_two_calls_take(mode, T, dtype, V):
     t, d, m = _inputs(10, 3, V, seed=V, masked=True, dtype=dtype)
@@ -191,7 +195,8 @@ def test_grpo_is_refused():
         FusedRun(t, d, None, G | aal.AAL_GRPO, 1.0, 1.0, 0.0)
 
 
-@pytest.mark.parametrize("mode,T,wg,ws", [(B, 1.0, 0.5, 0.5), (KL | G, 1.0, 0.1, 0.0), (S, 1.3, 0.0, 1.0)])
+@pytest.mark.parametrize("mode,T,wg,ws", [(B, 1.0, 0.5, 0.5), (KL | G, 1.0, 0.1, 0.0), (S, 1.3, 0.0, 1.0),
+                                         (KL | B, 0.7, 0.1, 0.5)])
 def test_fused_against_the_oracle(mode, T, wg, ws):
     t, d, m = _inputs(24, 5, 3000, seed=17, masked=True)
     check_loss(FusedRun(t, d, m, mode, T, wg, ws, dloss=24.0), t, d, m, mode, T, wg, ws, dloss=24.0)
