@@ -90,7 +90,8 @@ def test_anchor_gradient_matches_torch_autograd():
     np.testing.assert_allclose(g, tq.grad.numpy(), rtol=1e-12, atol=1e-15)
 
 
-@pytest.mark.parametrize("mode,T", [(MODE_KL | 1, 1.0), (MODE_KL | 2, 0.8), (MODE_KL | 3, 1.0), (MODE_KL, 1.0)])
+@pytest.mark.parametrize("mode,T", [(MODE_KL | 1, 1.0), (MODE_KL | 2, 0.8), (MODE_KL | 3, 1.0), (MODE_KL | 3, 1.5),
+                                    (MODE_KL, 1.0)])
 def test_objective_gradient_by_finite_differences(mode, T):
     rng = np.random.default_rng(5)
     N, K, V = 2, 3, 7
