@@ -133,25 +133,35 @@ class ClockSampler:
             self.proc.kill()
         self.file.flush()
         self.file.seek(0)
-        rows = [l.strip().split(", ") for l in self.file.read().splitlines() if l.strip()]
+        text = self.file.read()
         os.unlink(self.file.name)
-        sm, mx, reasons = [], [], set()
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for r in rows:
-            if len(r) < 9:
-                continue
-            try:
-                sm.append(float(r[1]))
-                mx.append(float(r[2]))
-            except ValueError:
-                continue
-            for nm, v in zip(names, r[5:9]):
-                if v.strip() == "Active":
-                    reasons.add(nm)
-        if not sm:
-            return None
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
-                "reasons": sorted(reasons)}
+        return summarize_clocks(text)
+
+
+def summarize_clocks(text):
+    """The clock record of the timed region from nvidia-smi's CSV samples (ClockSampler.FIELDS,
+    no header, no units): median SM clock, the largest max clock, the sample count and every
+    throttle reason seen active in any sample.  Malformed or partial lines are skipped; None
+    without a usable sample."""
+    sm, mx, reasons = [], [], set()
+    names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+    for line in text.splitlines():
+        r = [x.strip() for x in line.strip().split(",")]
+        if len(r) < 9:
+            continue
+        try:
+            s, m = float(r[1]), float(r[2])
+        except ValueError:
+            continue
+        sm.append(s)
+        mx.append(m)
+        for nm, v in zip(names, r[5:9]):
+            if v == "Active":
+                reasons.add(nm)
+    if not sm:
+        return None
+    return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+            "reasons": sorted(reasons)}
 
 
 # ----------------------------------------------------------------------------- our arm

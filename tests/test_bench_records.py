@@ -1,5 +1,6 @@
-"""bench.py's check that a recorded ncu traffic capture still describes the kernel's code:
-the hash covers the code of the listed sources and ignores their comments."""
+"""Host logic of bench.py: the check that a recorded ncu traffic capture still describes the
+kernel's code (the hash covers the code of the listed sources and ignores their comments), and
+the clock record of the timed region from nvidia-smi's samples."""
 
 import bench
 
@@ -27,3 +28,25 @@ def test_sources_sha_ignores_comment_edits_only(tmp_path, monkeypatch):
     (csrc / "k.cu").write_text("__global__ void k() { int z; }\n")
     assert bench.sources_sha(["k.cu"]) != a
     assert bench.sources_sha(["missing.cu"]) is None
+
+
+def test_clock_summary_takes_the_median_and_every_active_reason():
+    text = "\n".join([
+        "0, 2070, 2070, 900.5, 0x0000000000000000, Not Active, Not Active, Not Active, Not Active",
+        "0, 1965, 2070, 1400.1, 0x0000000000000004, Not Active, Not Active, Not Active, Active",
+        "0, 2070, 2070, 1200.0, 0x0000000000000000, Not Active, Not Active, Not Active, Not Active",
+        "0, [N/A], 2070, 1200.0, 0x0, Not Active, Not Active, Not Active, Not Active",   # skipped
+        "0, 2070, 2070",                                                                 # partial
+        "",
+    ])
+    c = bench.summarize_clocks(text)
+    assert c == {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "samples": 3, "reasons": ["sw_power_cap"]}
+
+
+def test_clock_summary_reports_thermal_and_hardware_slowdowns():
+    text = ("0, 1500, 2070, 800, 0x48, Active, Not Active, Active, Not Active\n"
+            "0, 1400, 2070, 800, 0x48, Not Active, Active, Not Active, Not Active\n")
+    c = bench.summarize_clocks(text)
+    assert c["sm_mhz"] == 1450.0 and c["samples"] == 2
+    assert c["reasons"] == ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown"]
+    assert bench.summarize_clocks("") is None
