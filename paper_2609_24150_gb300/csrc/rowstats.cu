@@ -246,8 +246,8 @@ cudaError_t launch_generic(const RowStatsArgs& a, cudaStream_t s) {
 }  // namespace
 
 // The TMA-streamed kernel (rowstats_stream.cu) serves rows whose byte length is a multiple
-// of 16: in two passes with the sampling term, in one pass without it.  Unaligned rows, and
-// the KL anchor next to a sampling term at T != 1, take the generic kernel.
+// of 16: in two passes with the sampling term, in one pass without it.  Unaligned rows take
+// the generic kernel.
 cudaError_t launch_rowstats(const RowStatsArgs& a, bool bf16, cudaStream_t s, int* cluster_used) {
   const int elt = bf16 ? 2 : 4;
   const bool aligned = ((a.V * elt) % 16 == 0) &&
