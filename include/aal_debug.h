@@ -1,9 +1,10 @@
 /*
- * aal_debug.h -- failure-detection test hook of libaal.so.
+ * aal_debug.h -- test hooks of libaal.so.
  *
- * Not part of the computation: it lets a test make one of the library's bounded device
+ * Not part of the computation: one lets a test make one of the library's bounded device
  * waits run out on purpose, so that the timeout path can be checked on a GPU without a
- * fault, a trap or a hang.
+ * fault, a trap or a hang; the other exposes a host-side launch decision so that it can be
+ * checked without a GPU.
  */
 #ifndef AAL_DEBUG_H_
 #define AAL_DEBUG_H_
@@ -27,6 +28,14 @@ extern "C" {
  * the context stays usable.  The results of that call are not valid.  A negative
  * `chunk` arms nothing.  The chunk setting is consumed by the next forward or GRPO call. */
 AAL_API void aal_debug_fail_next_forward(int64_t chunk, uint64_t wait_limit_ns);
+
+/* Windows per solo CTA in the launch of aal_loss_fwd_bwd's fused kernels, as the host chooses
+ * it: N windows of K rows, G groups of K CTAs (each group finishes one window per row time)
+ * and S spare CTAs (each takes whole windows, K row times each).  Returns an m >= 0 with
+ * m S <= N that minimises the launch's length in row times, max(ceil((N - m S) / G), m K),
+ * and 0 whenever no solo CTAs (m = 0) is as short; 0 when G <= 0 or S <= 0.  Pure host
+ * arithmetic: no GPU is touched. */
+AAL_API int64_t aal_debug_solo_windows(int64_t N, int32_t K, int32_t G, int32_t S);
 
 #ifdef __cplusplus
 }

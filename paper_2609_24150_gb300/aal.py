@@ -115,6 +115,8 @@ def library() -> ctypes.CDLL:
     lib.aal_check_device_status.argtypes = [vp, vp]
     lib.aal_debug_fail_next_forward.argtypes = [ctypes.c_int64, ctypes.c_uint64]
     lib.aal_debug_fail_next_forward.restype = None
+    lib.aal_debug_solo_windows.argtypes = [ctypes.c_int64, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32]
+    lib.aal_debug_solo_windows.restype = ctypes.c_int64
     lib.aal_status_string.argtypes = [ctypes.c_int]
     lib.aal_status_string.restype = ctypes.c_char_p
     lib.aal_abi_version.argtypes = []
@@ -418,3 +420,9 @@ def aal_debug_fail_next_forward(chunk: int, wait_limit_ns: int = 0):
     """Failure-detection test hook: leave one ring copy of the next streamed forward unarmed
     so that its bounded waits run out (see include/aal_debug.h)."""
     library().aal_debug_fail_next_forward(int(chunk), int(wait_limit_ns))
+
+
+def aal_debug_solo_windows(N: int, K: int, G: int, S: int) -> int:
+    """Test hook: windows per solo CTA that the fused call's launch chooses for N windows of K
+    rows, G groups and S spare CTAs (host arithmetic; see include/aal_debug.h)."""
+    return int(library().aal_debug_solo_windows(int(N), int(K), int(G), int(S)))

@@ -204,11 +204,15 @@ int64_t debug_take_skip_chunk() { return g_skip_chunk.exchange(-1); }
 
 extern "C" {
 
-int32_t aal_abi_version(void) { return 10500; }
+int32_t aal_abi_version(void) { return 10501; }
 
 void aal_debug_fail_next_forward(int64_t chunk, uint64_t wait_limit_ns) {
   g_wait_limit_ns.store(wait_limit_ns);
   g_skip_chunk.store(chunk);
+}
+
+int64_t aal_debug_solo_windows(int64_t N, int32_t K, int32_t G, int32_t S) {
+  return aal::solo_windows_each(N, K, G, S);
 }
 
 const char* aal_status_string(aal_status s) {

@@ -41,7 +41,7 @@ def test_library_exports_every_declared_symbol():
 
 
 def test_status_strings_and_version():
-    assert aal.aal_abi_version() == 10500
+    assert aal.aal_abi_version() == 10501
     for code in range(6):
         assert aal.aal_status_string(code).startswith("AAL_")
     assert aal.aal_status_string(99) == "unknown aal_status"
@@ -312,3 +312,32 @@ def test_sequence_grpo_checks():
     assert lib.aal_seq_grpo_from_loss(*args(_gprob(N=8, K=3), sp, fake, size)) == aal.AAL_ERR_INVALID_ARG
     no_grpo = _sprob(B=2, seq_len=16, K=4, mode=aal.AAL_GREEDY)
     assert lib.aal_seq_grpo_from_loss(*args(g, no_grpo, fake, size)) == aal.AAL_ERR_INVALID_ARG
+
+
+def _launch_rows(N, K, G, S, m):
+    """Row times of the fused launch: G groups take the first N - m S windows, one per row time
+    each; S solo CTAs take m windows each, K row times per window."""
+    return max(-(-(N - m * S) // G), m * K)
+
+
+@pytest.mark.parametrize("K", [1, 2, 3, 4, 5, 6, 7, 8])
+def test_solo_window_split_is_optimal(K):
+    """The fused call's split of windows between CTA groups and solo CTAs, against a brute
+    force over every m, for the SM count of a GB300 and of smaller parts."""
+    for ctas in (152, 148, 132, 64, 13):
+        for N in list(range(0, 400)) + [1000, 4096, 8191, 8192, 8193, 65536, 10**6 + 7]:
+            G = min(ctas // K, N, 1024)
+            S = ctas - G * K
+            m = aal.aal_debug_solo_windows(N, K, G, S)
+            if G <= 0 or S <= 0:
+                assert m == 0
+                continue
+            assert 0 <= m and m * S <= N
+            lo, hi = max(0, N // (G * K + S) - 3), min(N // S, N // (G * K + S) + 3)
+            best = min(_launch_rows(N, K, G, S, j) for j in [0] + list(range(lo, hi + 1)))
+            if N <= 400:   # the whole range as well, not just around the balance point
+                best = min(best, min(_launch_rows(N, K, G, S, j) for j in range(0, N // S + 1)))
+            assert _launch_rows(N, K, G, S, m) == best, (N, K, ctas, m)
+            if _launch_rows(N, K, G, S, 0) == best:
+                assert m == 0, (N, K, ctas, m)
+
