@@ -97,17 +97,10 @@ SOLO_CASES = [
 
 def solo_windows(N, K, sms):
     """The windows the launch gives to solo CTAs (one CTA per SM, as the ring's shared memory
-    allows): m per solo CTA, m minimising max(ceil((N - m S) / G), m K)."""
+    allows): the library's own split (checked against a brute force in test_abi)."""
     G = min(sms // K, N, 1024)
     S = sms - G * K
-    cost = lambda m: max(-(-(N - m * S) // G), m * K)
-    best = 0
-    if S > 0:
-        m0 = N // (G * K + S)
-        for m in (m0, m0 + 1):
-            if m > 0 and m * S <= N and cost(m) < cost(best):
-                best = m
-    return best * S if best else 0
+    return aal.aal_debug_solo_windows(N, K, G, S) * S if G > 0 and S > 0 else 0
 
 
 @pytest.mark.parametrize("N,K,V,mode,T,wg,ws,wkl,wtv,masked", CASES + SOLO_CASES)
