@@ -100,7 +100,18 @@ typedef enum {
  *                a = q(x*) (Eq. acc_greedy) always uses the unscaled draft, so T is
  *                ignored (and may be 0) for mode GREEDY.
  *   w_greedy, w_sampling, w_kl, w_tv  weights of the terms (a term the mode does not select
- *                is not computed and its weight is ignored).  Must be finite. */
+ *                is not computed and its weight is ignored).  Must be finite.
+ *   global_counts, n_windows_global, n_positions_global   data-parallel normalisers.  With
+ *                global_counts = 0 (the default; this field was "reserved, must be 0" before ABI
+ *                1.6, and the two fields after it are then not read) the loss divides by this
+ *                call's own |W| and |P|.  With global_counts = 1 it divides by n_windows_global
+ *                (|W| of the whole data-parallel batch, Sec. 3.2's 1/|W|: the windows whose depth
+ *                0 is valid, summed over the ranks) and n_positions_global (|P| of the whole
+ *                batch, the KL anchor's normaliser), each in [0, 2^31 - 1].  A batch sharded by
+ *                windows over ranks then needs no collective on the data path and no rescaled
+ *                dloss: the loss of the whole batch is the sum of the ranks' losses, and each
+ *                rank's gradient rows are those of the whole batch's loss, bit for bit.  The
+ *                backward uses the forward's normalisers (kept in the workspace). */
 typedef struct {
   int64_t N, K, V;
   int32_t dtype;
@@ -110,7 +121,9 @@ typedef struct {
   float w_sampling;
   float w_kl;
   float w_tv;
-  int32_t reserved; /* must be 0 */
+  int32_t global_counts;      /* 0 or 1 */
+  int64_t n_windows_global;   /* read only when global_counts = 1 */
+  int64_t n_positions_global; /* read only when global_counts = 1 */
 } aal_problem;
 
 /* Bytes of device workspace a loss problem needs (host-only, launches nothing). */
@@ -171,8 +184,10 @@ AAL_API aal_status aal_loss_fwd_bwd(const aal_problem* prob, const void* draft, 
  * is depth j of up to K windows.  Logits are stored once per position, not once per window.
  *   B, seq_len, K, V  sequences, positions per sequence (>= 0), window size gamma
  *                     (1..AAL_MAX_K), vocabulary size (>= 1).
- *   dtype, mode, temperature, w_greedy, w_sampling, w_kl, w_tv, reserved  as in aal_problem
- *                     (the anchor averages over the valid positions).
+ *   dtype, mode, temperature, w_greedy, w_sampling, w_kl, w_tv, global_counts,
+ *   n_windows_global, n_positions_global   as in aal_problem (the anchor averages over the
+ *                     valid positions; a batch is sharded over ranks by whole sequences, and
+ *                     n_windows_global counts the windows in W of all of them).
  *   full_windows      which windows belong to W (the paper leaves the end of a sequence open):
  *                     0 = every start position, its window truncated at the end of the
  *                     sequence or at its first invalid position (as a masked window of
@@ -188,7 +203,9 @@ typedef struct {
   float w_kl;
   float w_tv;
   int32_t full_windows;
-  int32_t reserved; /* must be 0 */
+  int32_t global_counts;      /* 0 or 1, as in aal_problem */
+  int64_t n_windows_global;   /* read only when global_counts = 1 */
+  int64_t n_positions_global; /* read only when global_counts = 1 */
 } aal_seq_problem;
 
 /* Bytes of device workspace a sequence problem needs (host-only, launches nothing). */

@@ -43,7 +43,8 @@ class AalProblem(ctypes.Structure):
                 ("dtype", ctypes.c_int32), ("mode", ctypes.c_int32),
                 ("temperature", ctypes.c_float), ("w_greedy", ctypes.c_float),
                 ("w_sampling", ctypes.c_float), ("w_kl", ctypes.c_float), ("w_tv", ctypes.c_float),
-                ("reserved", ctypes.c_int32)]
+                ("global_counts", ctypes.c_int32), ("n_windows_global", ctypes.c_int64),
+                ("n_positions_global", ctypes.c_int64)]
 
 
 class AalRewardProblem(ctypes.Structure):
@@ -61,7 +62,8 @@ class AalSeqProblem(ctypes.Structure):
                 ("V", ctypes.c_int64), ("dtype", ctypes.c_int32), ("mode", ctypes.c_int32),
                 ("temperature", ctypes.c_float), ("w_greedy", ctypes.c_float),
                 ("w_sampling", ctypes.c_float), ("w_kl", ctypes.c_float), ("w_tv", ctypes.c_float),
-                ("full_windows", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+                ("full_windows", ctypes.c_int32), ("global_counts", ctypes.c_int32),
+                ("n_windows_global", ctypes.c_int64), ("n_positions_global", ctypes.c_int64)]
 
 
 class AalGrpoProblem(ctypes.Structure):
@@ -172,30 +174,45 @@ def _check(code: int, where: str):
         raise AalError(code, where)
 
 
+def _global(n_windows_global, n_positions_global):
+    """(global_counts, |W|, |P|) fields: both counts given, or neither (this call's own)."""
+    if (n_windows_global is None) != (n_positions_global is None):
+        raise ValueError("give both global counts (|W| and |P| of the whole batch) or neither")
+    if n_windows_global is None:
+        return 0, 0, 0
+    return 1, int(n_windows_global), int(n_positions_global)
+
+
 def loss_problem(draft: torch.Tensor, mode: int, temperature: float = 1.0, w_greedy: float = 1.0,
-                 w_sampling: float = 1.0, w_kl: float = 1.0, w_tv: float = 1.0) -> AalProblem:
+                 w_sampling: float = 1.0, w_kl: float = 1.0, w_tv: float = 1.0,
+                 n_windows_global: Optional[int] = None, n_positions_global: Optional[int] = None) -> AalProblem:
     """Problem struct for [N][K][V] logits (``w_kl`` weighs the AAL_KL anchor, ``w_tv`` the
-    AAL_TV term)."""
+    AAL_TV term).  ``n_windows_global`` / ``n_positions_global``: |W| and |P| of a whole
+    data-parallel batch that this call is one shard of (the loss and gradient are normalised by
+    them instead of the shard's own)."""
     if draft.dim() != 3:
         raise ValueError("logits must be [N][K][V]")
     N, K, V = draft.shape
     if draft.dtype not in _DTYPES:
         raise ValueError(f"unsupported dtype {draft.dtype}")
-    return AalProblem(N, K, V, _DTYPES[draft.dtype], mode, temperature, w_greedy, w_sampling, w_kl, w_tv, 0)
+    return AalProblem(N, K, V, _DTYPES[draft.dtype], mode, temperature, w_greedy, w_sampling, w_kl, w_tv,
+                      *_global(n_windows_global, n_positions_global))
 
 
 def seq_problem(draft: torch.Tensor, K: int, mode: int, temperature: float = 1.0, w_greedy: float = 1.0,
                 w_sampling: float = 1.0, full_windows: bool = False, w_kl: float = 1.0,
-                w_tv: float = 1.0) -> AalSeqProblem:
+                w_tv: float = 1.0, n_windows_global: Optional[int] = None,
+                n_positions_global: Optional[int] = None) -> AalSeqProblem:
     """Problem struct for [B][seq_len][V] logits with sliding windows of K positions
-    (``full_windows``: only windows with all K positions valid belong to W)."""
+    (``full_windows``: only windows with all K positions valid belong to W; the global counts
+    as in loss_problem, for a batch sharded by whole sequences)."""
     if draft.dim() != 3:
         raise ValueError("logits must be [B][seq_len][V]")
     B, S, V = draft.shape
     if draft.dtype not in _DTYPES:
         raise ValueError(f"unsupported dtype {draft.dtype}")
     return AalSeqProblem(B, S, K, V, _DTYPES[draft.dtype], mode, temperature, w_greedy, w_sampling,
-                         w_kl, w_tv, int(bool(full_windows)), 0)
+                         w_kl, w_tv, int(bool(full_windows)), *_global(n_windows_global, n_positions_global))
 
 
 def reward_problem(draft: torch.Tensor, mode: int, temperature: float = 1.0, adv_clip: float = 5.0,

@@ -39,7 +39,10 @@ aal_status check_problem(const aal_problem* p) {
     return AAL_ERR_INVALID_ARG;
   if (!isfinite(p->w_greedy) || !isfinite(p->w_sampling) || !isfinite(p->w_kl) || !isfinite(p->w_tv))
     return AAL_ERR_INVALID_ARG;
-  if (p->reserved != 0) return AAL_ERR_INVALID_ARG;
+  if (p->global_counts != 0 && p->global_counts != 1) return AAL_ERR_INVALID_ARG;
+  if (p->global_counts == 1 && !(p->n_windows_global >= 0 && p->n_windows_global <= INT32_MAX &&
+                                 p->n_positions_global >= 0 && p->n_positions_global <= INT32_MAX))
+    return AAL_ERR_INVALID_ARG;
   return AAL_OK;
 }
 
@@ -65,8 +68,11 @@ aal_status check_seq(const aal_seq_problem* p) {
   if (p->seq_len > 0 && p->B > INT64_MAX / p->seq_len) return AAL_ERR_INVALID_ARG;
   // the checks of a windowed problem with one window per position (R * K * V elements bound
   // the per-depth partials too)
-  const aal_problem q{p->B * p->seq_len, p->K, p->V, p->dtype, p->mode, p->temperature, p->w_greedy,
-                      p->w_sampling, p->w_kl, p->w_tv, p->reserved};
+  const aal_problem q{p->B * p->seq_len, p->K,          p->V,          p->dtype,
+                      p->mode,           p->temperature, p->w_greedy, p->w_sampling,
+                      p->w_kl,           p->w_tv,       p->global_counts,
+                      p->global_counts == 1 ? p->n_windows_global : 0,
+                      p->global_counts == 1 ? p->n_positions_global : 0};
   return check_problem(&q);
 }
 
@@ -192,6 +198,8 @@ WindowArgs window_args(const aal_problem* prob, const uint8_t* mask, int cluster
   wa.eal = eal;
   wa.ws = ws;
   wa.nwblk = nwblk;
+  wa.nvalid_g = prob->global_counts == 1 ? (int32_t)prob->n_windows_global : -1;
+  wa.npos_g = prob->global_counts == 1 ? (int32_t)prob->n_positions_global : -1;
   return wa;
 }
 
@@ -204,7 +212,7 @@ int64_t debug_take_skip_chunk() { return g_skip_chunk.exchange(-1); }
 
 extern "C" {
 
-int32_t aal_abi_version(void) { return 10501; }
+int32_t aal_abi_version(void) { return 10600; }
 
 void aal_debug_fail_next_forward(int64_t chunk, uint64_t wait_limit_ns) {
   g_wait_limit_ns.store(wait_limit_ns);
@@ -313,8 +321,10 @@ aal_status aal_loss_fwd_bwd(const aal_problem* prob, const void* draft, const vo
     LossWs ws = loss_ws(workspace, L);
     if (cudaMemsetAsync(ws.hdr, 0, sizeof(WsHeader), s) != cudaSuccess) return AAL_ERR_CUDA;
     if (cudaMemsetAsync(ws.mbox, 0xff, (size_t)L.R * 8, s) != cudaSuccess) return AAL_ERR_CUDA;  // kMboxEmpty
-    if (launch_count_valid(mask, prob->N, (int32_t)prob->K, ws.hdr, s) != cudaSuccess) return AAL_ERR_CUDA;
     FusedIdsArgs f;
+    f.win = window_args(prob, mask, 1, loss, eal, ws, L.nwblk);
+    if (launch_count_valid(mask, prob->N, (int32_t)prob->K, f.win.nvalid_g, f.win.npos_g, ws.hdr, s) != cudaSuccess)
+      return AAL_ERR_CUDA;
     f.st.z = draft;
     f.st.R = L.R;
     f.st.V = prob->V;
@@ -327,7 +337,6 @@ aal_status aal_loss_fwd_bwd(const aal_problem* prob, const void* draft, const vo
     f.st.skip_chunk = debug_take_skip_chunk();
     f.bw = grad_args(draft, target, mask, L.R, prob->V, prob->mode, prob->temperature, prob->w_greedy,
                      prob->w_kl, dloss, ws, grad_draft);
-    f.win = window_args(prob, mask, 1, loss, eal, ws, L.nwblk);
     f.groups = 0;
     const uint64_t limit = debug_wait_limit_ns();
     bool launched = false;
@@ -338,12 +347,13 @@ aal_status aal_loss_fwd_bwd(const aal_problem* prob, const void* draft, const vo
     LossWs ws = loss_ws(workspace, L);
     if (cudaMemsetAsync(ws.hdr, 0, sizeof(WsHeader), s) != cudaSuccess) return AAL_ERR_CUDA;
     if (cudaMemsetAsync(ws.mbox, 0xff, (size_t)L.R * 8, s) != cudaSuccess) return AAL_ERR_CUDA;  // kMboxEmpty
-    if (launch_count_valid(mask, prob->N, (int32_t)prob->K, ws.hdr, s) != cudaSuccess) return AAL_ERR_CUDA;
     FusedArgs f;
+    f.win = window_args(prob, mask, 1, loss, eal, ws, L.nwblk);
+    if (launch_count_valid(mask, prob->N, (int32_t)prob->K, f.win.nvalid_g, f.win.npos_g, ws.hdr, s) != cudaSuccess)
+      return AAL_ERR_CUDA;
     f.st = stats_args(draft, target, L.R, prob->V, prob->mode, prob->temperature, ws);
     f.bw = grad_args(draft, target, mask, L.R, prob->V, prob->mode, prob->temperature, prob->w_greedy,
                      prob->w_kl, dloss, ws, grad_draft);
-    f.win = window_args(prob, mask, 1, loss, eal, ws, L.nwblk);
     f.groups = 0;
     const uint64_t limit = debug_wait_limit_ns();
     bool launched = false;
@@ -411,6 +421,8 @@ aal_status aal_seq_loss_fwd(const aal_seq_problem* prob, const void* draft, cons
   wa.ps = reinterpret_cast<float*>(base + L.ps);
   wa.ws = ws;
   wa.nwblk = L.base.nwblk;
+  wa.nvalid_g = prob->global_counts == 1 ? (int32_t)prob->n_windows_global : -1;
+  wa.npos_g = prob->global_counts == 1 ? (int32_t)prob->n_positions_global : -1;
   return cuda_status(launch_seq_window(wa, s));
 }
 

@@ -210,6 +210,7 @@ struct WindowArgs {
   float* eal;           // device float[N][2] or null
   LossWs ws;
   int64_t nwblk;
+  int32_t nvalid_g, npos_g;  // data-parallel |W| and |P| of the whole batch, or -1: this call's
 };
 
 struct SeqWindowArgs {
@@ -226,6 +227,7 @@ struct SeqWindowArgs {
   float* ps;
   LossWs ws;
   int64_t nwblk;
+  int32_t nvalid_g, npos_g;  // data-parallel |W| and |P| of the whole batch, or -1: this call's
 };
 
 struct BackwardArgs {
@@ -454,7 +456,8 @@ cudaError_t launch_one_tensor(const Stream1Args& a, bool bf16, bool ids, cudaStr
 cudaError_t launch_grpo_windows(const GrpoWindowArgs& a, cudaStream_t s);
 cudaError_t launch_seq_grpo_gather(const SeqGrpoArgs& a, cudaStream_t s);
 cudaError_t launch_seq_grpo_scatter(const SeqGrpoArgs& a, cudaStream_t s);
-cudaError_t launch_count_valid(const uint8_t* mask, int64_t N, int32_t K, WsHeader* hdr, cudaStream_t s);
+cudaError_t launch_count_valid(const uint8_t* mask, int64_t N, int32_t K, int32_t nvalid_g, int32_t npos_g,
+                               WsHeader* hdr, cudaStream_t s);
 // Launches the fused forward + backward when the problem's flags have an instantiation and the
 // device can hold at least one group; *launched tells whether it did.
 cudaError_t launch_fused(const FusedArgs& f, cudaStream_t s, uint64_t limit_ns, bool* launched);

@@ -458,8 +458,10 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
 }
 
 // |W| (windows whose depth 0 is valid) and |positions| (valid rows) from the [N][K] mask, one
-// block; integer sums, so the order does not matter.
-__global__ void __launch_bounds__(1024) count_valid(const uint8_t* mask, int64_t N, int32_t K, WsHeader* hdr) {
+// block; integer sums, so the order does not matter.  Data-parallel normalisers given by the
+// caller (nvalid_g, npos_g >= 0) replace the counts.
+__global__ void __launch_bounds__(1024) count_valid(const uint8_t* mask, int64_t N, int32_t K, int32_t nvalid_g,
+                                                    int32_t npos_g, WsHeader* hdr) {
   __shared__ unsigned long long sw, sp;
   if (threadIdx.x == 0) {
     sw = 0ull;
@@ -480,8 +482,8 @@ __global__ void __launch_bounds__(1024) count_valid(const uint8_t* mask, int64_t
   atomicAdd(&sp, p);
   __syncthreads();
   if (threadIdx.x == 0) {
-    hdr->nvalid = (int32_t)sw;
-    hdr->npos = (int32_t)sp;
+    hdr->nvalid = nvalid_g >= 0 ? nvalid_g : (int32_t)sw;
+    hdr->npos = npos_g >= 0 ? npos_g : (int32_t)sp;
   }
 }
 
@@ -523,8 +525,9 @@ cudaError_t go_fused(const FusedArgs& f0, cudaStream_t s, uint64_t limit_ns, boo
 
 }  // namespace
 
-cudaError_t launch_count_valid(const uint8_t* mask, int64_t N, int32_t K, WsHeader* hdr, cudaStream_t s) {
-  count_valid<<<1, 1024, 0, s>>>(mask, N, K, hdr);
+cudaError_t launch_count_valid(const uint8_t* mask, int64_t N, int32_t K, int32_t nvalid_g, int32_t npos_g,
+                               WsHeader* hdr, cudaStream_t s) {
+  count_valid<<<1, 1024, 0, s>>>(mask, N, K, nvalid_g, npos_g, hdr);
   return cudaGetLastError();
 }
 

@@ -69,8 +69,9 @@ __device__ __forceinline__ void finish_loss(const Args& a, double (&x)[kSums], d
   }
   block_sum<kWindowThreads, kSums>(t, sm);
   if (threadIdx.x == 0) {
-    const int nvalid = (int)t[2];
-    const int npos = (int)t[4];
+    // the data-parallel normalisers of the whole batch when the caller gives them
+    const int nvalid = a.nvalid_g >= 0 ? a.nvalid_g : (int)t[2];
+    const int npos = a.npos_g >= 0 ? a.npos_g : (int)t[4];
     const double num = (a.greedy ? (double)a.w_greedy * t[0] : 0.0) +
                        (a.sampling ? (double)a.w_sampling * t[1] : 0.0);
     double L = nvalid > 0 ? -num / (double)nvalid : 0.0;

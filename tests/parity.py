@@ -24,6 +24,39 @@ GRAD_ATOL = 1e-5
 GRAD_RTOL = 1e-2
 TIE_BAND = 1e-5
 
+# What the widened bands set aside, per test (reset by the autouse fixture in conftest.py):
+#   elems / tie_elems: gradient elements compared, and those whose fp64 log-probabilities lie
+#     within TIE_BAND of each other without being equal (their subgradient side is ambiguous);
+#   rescued: elements outside the unwidened tolerance that the widening accepted;
+#   windows / thr_windows: reward windows compared, and those set aside because a draw that
+#     decided their leading run lies within the threshold band of the reward tests.
+BAND = {"elems": 0, "tie_elems": 0, "rescued": 0, "windows": 0, "thr_windows": 0}
+BAND_LIMITS = {"tie": 1e-3, "rescued": 1e-3, "thr": 1e-2}
+
+
+def band_reset():
+    for k in BAND:
+        BAND[k] = 0
+
+
+def note_thr(set_aside, total):
+    BAND["thr_windows"] += int(set_aside)
+    BAND["windows"] += int(total)
+
+
+def band_shares():
+    e, w = max(BAND["elems"], 1), max(BAND["windows"], 1)
+    return {"tie": BAND["tie_elems"] / e, "rescued": BAND["rescued"] / e, "thr": BAND["thr_windows"] / w}
+
+
+def assert_bands():
+    """The widened bands set aside at most BAND_LIMITS of what a test compared: a systematic
+    error near the ties or thresholds would show up as far more."""
+    sh = band_shares()
+    for k, lim in BAND_LIMITS.items():
+        assert sh[k] <= lim, f"band {k}: {sh[k]:.3g} of the compared items (limit {lim}); counts {BAND}"
+
+
 MODES = {"greedy": aal.AAL_GREEDY, "sampling": aal.AAL_SAMPLING, "both": aal.AAL_BOTH}
 # the C modes are bit sets with the oracle's values: 1 EAL, 2 WTV, 4 the KL anchor, 16 the TV term
 ORACLE_MODES = {m: (oracle.MODE_GREEDY if m & aal.AAL_GREEDY else 0)
@@ -53,6 +86,7 @@ class LossRun:
 def grad_tolerance(target, draft, mask, omode, T, wg, ws, dloss, gref, nvalid, fw, wtv=0.0):
     """Per-element tolerance, widened at WTV / TV near-ties (see module docstring)."""
     tol = GRAD_ATOL + GRAD_RTOL * np.abs(gref)
+    BAND["elems"] += int(np.prod(np.shape(gref)))
     if not (omode & (oracle.MODE_SAMPLING | oracle.MODE_TV)) or nvalid == 0:
         return tol
     zp = oracle.as_f64(target)
@@ -61,6 +95,7 @@ def grad_tolerance(target, draft, mask, omode, T, wg, ws, dloss, gref, nvalid, f
     lq = oracle.log_softmax(zq, T)
     amb = np.abs(lq - lp) < TIE_BAND
     amb &= (lq != lp)  # exact ties are decided identically on both sides
+    BAND["tie_elems"] += int(amb.sum())
     if not amb.any():
         return tol
     qt = np.exp(lq)
@@ -105,6 +140,7 @@ def check_loss(run: LossRun, target, draft, mask, mode, T, wg, ws, dloss=1.0, wi
     g = run.grad.cpu().double().numpy()[sel]
     tol = grad_tolerance(t_h, d_h, m_h, omode, T, wg, ws, dloss, gref, nvalid, fw, wtv if omode & oracle.MODE_TV else 0.0)
     bad = np.abs(g - gref) > tol
+    BAND["rescued"] += int(np.sum((np.abs(g - gref) > GRAD_ATOL + GRAD_RTOL * np.abs(gref)) & ~bad))
     if bad.any():
         i = tuple(np.argwhere(bad)[0])
         raise AssertionError(f"{int(bad.sum())} gradient elements off; first {i}: "
@@ -161,6 +197,7 @@ def seq_grad_tolerance(target, draft, mask, K, omode, T, wg, ws, dloss, gref, nv
 
 def _assert_grad(g, gref, tol, where=""):
     bad = np.abs(g - gref) > tol
+    BAND["rescued"] += int(np.sum((np.abs(g - gref) > GRAD_ATOL + GRAD_RTOL * np.abs(gref)) & ~bad))
     if bad.any():
         i = tuple(np.argwhere(bad)[0])
         raise AssertionError(f"{where}{int(bad.sum())} gradient elements off; first {i}: "

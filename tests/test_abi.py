@@ -41,7 +41,7 @@ def test_library_exports_every_declared_symbol():
 
 
 def test_status_strings_and_version():
-    assert aal.aal_abi_version() == 10501
+    assert aal.aal_abi_version() == 10600
     for code in range(6):
         assert aal.aal_status_string(code).startswith("AAL_")
     assert aal.aal_status_string(99) == "unknown aal_status"
@@ -49,7 +49,7 @@ def test_status_strings_and_version():
 
 def _prob(**kw):
     d = dict(N=4, K=3, V=100, dtype=aal.AAL_BF16, mode=aal.AAL_BOTH, temperature=1.0,
-             w_greedy=0.5, w_sampling=0.5, w_kl=1.0, w_tv=0.1, reserved=0)
+             w_greedy=0.5, w_sampling=0.5, w_kl=1.0, w_tv=0.1, global_counts=0)
     d.update(kw)
     return aal.AalProblem(**d)
 
@@ -90,7 +90,13 @@ def test_workspace_size_grows_with_rows():
     (dict(temperature=-1.0), aal.AAL_ERR_INVALID_ARG),
     (dict(temperature=float("nan")), aal.AAL_ERR_INVALID_ARG),
     (dict(w_greedy=float("inf")), aal.AAL_ERR_INVALID_ARG),
-    (dict(reserved=1), aal.AAL_ERR_INVALID_ARG),
+    (dict(global_counts=2), aal.AAL_ERR_INVALID_ARG),
+    (dict(global_counts=-1), aal.AAL_ERR_INVALID_ARG),
+    (dict(global_counts=1, n_windows_global=10, n_positions_global=30), aal.AAL_OK),
+    (dict(global_counts=1, n_windows_global=0, n_positions_global=0), aal.AAL_OK),
+    (dict(global_counts=1, n_windows_global=-1, n_positions_global=30), aal.AAL_ERR_INVALID_ARG),
+    (dict(global_counts=1, n_windows_global=10, n_positions_global=2**31), aal.AAL_ERR_INVALID_ARG),
+    (dict(global_counts=0, n_windows_global=-5, n_positions_global=-5), aal.AAL_OK),  # not read
     (dict(V=2**31), aal.AAL_ERR_UNSUPPORTED),
     (dict(N=2**60, V=2**20), aal.AAL_ERR_INVALID_ARG),
 ])
@@ -194,7 +200,7 @@ def test_reward_from_loss_argument_checks():
 
 def _sprob(**kw):
     d = dict(B=2, seq_len=16, K=4, V=100, dtype=aal.AAL_BF16, mode=aal.AAL_BOTH, temperature=1.0,
-             w_greedy=0.5, w_sampling=0.5, w_kl=1.0, w_tv=0.1, full_windows=0, reserved=0)
+             w_greedy=0.5, w_sampling=0.5, w_kl=1.0, w_tv=0.1, full_windows=0, global_counts=0)
     d.update(kw)
     return aal.AalSeqProblem(**d)
 
@@ -217,7 +223,9 @@ def _seq_ws(p):
     (dict(V=0), aal.AAL_ERR_INVALID_ARG),
     (dict(mode=0), aal.AAL_ERR_INVALID_ARG),
     (dict(temperature=0.0), aal.AAL_ERR_INVALID_ARG),
-    (dict(reserved=2), aal.AAL_ERR_INVALID_ARG),
+    (dict(global_counts=2), aal.AAL_ERR_INVALID_ARG),
+    (dict(global_counts=1, n_windows_global=64, n_positions_global=64), aal.AAL_OK),
+    (dict(global_counts=1, n_windows_global=2**31, n_positions_global=64), aal.AAL_ERR_INVALID_ARG),
     (dict(full_windows=1), aal.AAL_OK),
     (dict(full_windows=2), aal.AAL_ERR_INVALID_ARG),
 ])
@@ -341,3 +349,25 @@ def test_solo_window_split_is_optimal(K):
             if _launch_rows(N, K, G, S, 0) == best:
                 assert m == 0, (N, K, ctas, m)
 
+
+
+def test_problem_struct_layout():
+    """The ctypes mirrors have the header's layout: the data-parallel fields follow the int32 that
+    was "reserved" before ABI 1.6 (so a caller that zeroes it never has them read)."""
+    P, S = aal.AalProblem, aal.AalSeqProblem
+    assert P.global_counts.offset == 52 and P.n_windows_global.offset == 56 and P.n_positions_global.offset == 64
+    assert ctypes.sizeof(P) == 72
+    assert S.full_windows.offset == 60 and S.global_counts.offset == 64 and S.n_windows_global.offset == 72
+    assert ctypes.sizeof(S) == 88
+
+
+def test_global_counts_need_both():
+    import torch
+    d = torch.empty(2, 3, 8, dtype=torch.bfloat16)
+    p = aal.loss_problem(d, aal.AAL_BOTH, n_windows_global=10, n_positions_global=30)
+    assert (p.global_counts, p.n_windows_global, p.n_positions_global) == (1, 10, 30)
+    assert aal.loss_problem(d, aal.AAL_BOTH).global_counts == 0
+    with pytest.raises(ValueError):
+        aal.loss_problem(d, aal.AAL_BOTH, n_windows_global=10)
+    s = aal.seq_problem(d, 2, aal.AAL_KL | aal.AAL_GREEDY, n_windows_global=6, n_positions_global=6)
+    assert (s.global_counts, s.n_windows_global, s.n_positions_global) == (1, 6, 6)

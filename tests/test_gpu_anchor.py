@@ -9,7 +9,7 @@ import torch
 import oracle
 import paper_2609_24150_gb300 as aal
 import synth
-from tests.parity import (LossRun, SeqRun, check_loss, check_seq_loss, check_seq_positions,
+from tests.parity import (LossRun, SeqRun, assert_bands, check_loss, check_seq_loss, check_seq_positions,
                           seq_window_counts)
 
 pytestmark = pytest.mark.gpu
@@ -95,6 +95,7 @@ def test_full_size_sampled_windows_greedy_objective():
     windows = [0, 1, 4095, 8191]
     check_loss(run, target, draft, None, KL_G, 0.0, 0.1, 0.0, dloss=float(N * K), windows=windows,
                n_windows_total=N, wkl=1.0, n_positions_total=N * K)
+    assert_bands()
     assert np.isfinite(run.loss.item())
 
 
@@ -123,6 +124,7 @@ def test_sequence_full_size_sampled_positions():
         positions += [(b, int(valid[0])), (b, int(valid[-1])), (b, int(valid[len(valid) // 2]))]
     check_seq_positions(run, target, draft, mask, K, KL_G, 0.0, 0.1, 0.0, float(npos), positions,
                         seq_window_counts(mask, B, Tn), wkl=1.0, npos_total=npos)
+    assert_bands()
     dead = torch.from_numpy(m == 0).to(DEV)
     assert torch.count_nonzero(run.grad[dead]).item() == 0
 
@@ -171,3 +173,4 @@ def test_tv_baseline_full_size_sampled_windows():
     run = LossRun(target, draft, None, KL_TV, 1.0, 0.0, 0.0, dloss=float(N * K), wkl=1.0, wtv=0.1)
     check_loss(run, target, draft, None, KL_TV, 1.0, 0.0, 0.0, dloss=float(N * K), windows=[0, 3000, 8191],
                n_windows_total=N, wkl=1.0, n_positions_total=N * K, wtv=0.1)
+    assert_bands()

@@ -7,7 +7,7 @@ import torch
 import oracle
 import paper_2609_24150_gb300 as aal
 import synth
-from tests.parity import LossRun, check_loss, loss_from_eal
+from tests.parity import LossRun, assert_bands, check_loss, loss_from_eal
 
 pytestmark = pytest.mark.gpu
 
@@ -85,6 +85,7 @@ def test_masked_v32k_sampled_windows():
         run = LossRun(target, draft, mask, mode, T, wg, ws, dloss=float(nvalid))
         check_loss(run, target, draft, mask, mode, T, wg, ws, dloss=float(nvalid), windows=windows,
                    n_windows_total=nvalid)
+        assert_bands()
         implied = loss_from_eal(run, mode, wg, ws, nvalid)
         assert abs(float(run.loss.item()) - implied) <= 1e-5 * abs(implied) + 1e-7
         # masked windows contribute nothing and their rows get exact zeros
@@ -193,6 +194,7 @@ def test_v128k_full_size_sampled_windows(v128k):
     windows = sorted(set([0, 1, N - 1] + list(rng.choice(N, 21, replace=False))))
     check_loss(run, target, draft, None, aal.AAL_BOTH, 1.0, 0.5, 0.5, dloss=float(N),
                windows=windows, n_windows_total=N)
+    assert_bands()
     implied = loss_from_eal(run, aal.AAL_BOTH, 0.5, 0.5, N)
     assert abs(float(run.loss.item()) - implied) <= 1e-5 * abs(implied)
     # every gradient row is finite and sums to 0 (softmax shift invariance) up to the bf16
@@ -223,6 +225,7 @@ def test_v152k_full_size_temperature_sweep(v152k, T):
     windows = sorted(set([0, N - 1] + list(rng.choice(N, 14, replace=False))))
     check_loss(run, target, draft, None, aal.AAL_SAMPLING, T, 0.0, 1.0, dloss=float(N),
                windows=windows, n_windows_total=N)
+    assert_bands()
     # rows whose draft equals the target have an exactly zero WTV gradient, at full size
     for n0 in range(0, N, 512):
         same = (target[n0:n0 + 512] == draft[n0:n0 + 512]).all(-1)

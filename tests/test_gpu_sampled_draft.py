@@ -11,6 +11,7 @@ import torch
 import oracle
 import paper_2609_24150_gb300 as aal
 import synth
+from tests.parity import note_thr
 from tests.test_gpu_reward import run_reward
 
 pytestmark = pytest.mark.gpu
@@ -48,6 +49,7 @@ def oracle_windows(target, draft, ref, T, seed, row_offset, windows):
             zz = oracle.as_f64(z)[0]
             a |= any(_gap(zz[k], T, seed, row_offset + int(n), k) < KEY_BAND for k in range(upto))
         amb.append(a)
+    note_thr(int(np.sum(amb)), len(amb))
     return np.array(taus), np.array(taurs), np.array(amb)
 
 

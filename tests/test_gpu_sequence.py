@@ -10,7 +10,7 @@ import torch
 
 import paper_2609_24150_gb300 as aal
 import synth
-from tests.parity import (LOSS_ATOL, LOSS_RTOL, LossRun, SeqRun, check_seq_loss, check_seq_positions,
+from tests.parity import (LOSS_ATOL, LOSS_RTOL, LossRun, SeqRun, assert_bands, check_seq_loss, check_seq_positions,
                           seq_window_counts)
 
 pytestmark = pytest.mark.gpu
@@ -188,6 +188,7 @@ def test_full_size_sampled_positions(seq_v128k, mode, T, wg, ws):
                       (b, Tn - 1), (b, int(rng.integers(first, last + 1)))]
     positions = sorted({(b, t) for b, t in positions if 0 <= t < Tn})
     check_seq_positions(run, target, draft, mask, K, mode, T, wg, ws, dloss, positions, nvalid)
+    assert_bands()
     eal = run.eal.double().cpu().numpy()
     num = (wg * eal[:, 0].sum() if mode & aal.AAL_GREEDY else 0.0) + \
           (ws * eal[:, 1].sum() if mode & aal.AAL_SAMPLING else 0.0)
