@@ -57,8 +57,9 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-seq", action="store_true", help="skip every line beside the step")
-    ap.add_argument("--lines", default="greedy,ids,seq,grpo,seqgrpo",
-                    help="lines measured beside the step (comma-separated from greedy, ids, seq, grpo, seqgrpo)")
+    ap.add_argument("--lines", default="greedy,ids,seq,grpo,seqgrpo,configs,rewardstream",
+                    help="lines measured beside the step (comma-separated from greedy, ids, seq, grpo, seqgrpo, "
+                         "configs, rewardstream)")
     ap.add_argument("--windows", type=int, default=None,
                     help="run the first WINDOWS windows of the workload (profiling captures)")
     return ap.parse_args()
@@ -265,12 +266,14 @@ def run_ours(args, ws_count, rank, local):
     seq = run_sequence_layout(aal, dev, stream, rank, reps) if "seq" in lines else None
     grpo = run_grpo_phase(aal, dev, stream, rank, reps) if "grpo" in lines else None
     seq_grpo = run_seq_grpo_phase(aal, dev, stream, rank, reps) if "seqgrpo" in lines else None
+    peak, peak_src = measured_peak()
+    configs = run_config_lines(aal, dev, stream, rank, reps, peak) if "configs" in lines else None
+    rstream = run_reward_stream(aal, dev, stream, rank, peak) if "rewardstream" in lines else None
 
     b = algo_bytes(N, K, V)
     step_bytes = sum(b.values())
     R = N * K
     value = step_bytes * ws_count / (ms_step * 1e-3) / 1e9
-    peak, peak_src = measured_peak()
 
     # dominant kernel: the fused forward + backward (all but the reward's ~0.5% of the step).
     # Algorithmic bytes per launch as counted for the metric (2 reads forward, 2 reads + 1 write
@@ -336,6 +339,10 @@ def run_ours(args, ws_count, rank, local):
         res["grpo_phase_step"] = grpo
     if seq_grpo is not None:
         res["seq_grpo_phase_step"] = seq_grpo
+    if configs is not None:
+        res["config_lines"] = configs
+    if rstream is not None:
+        res["reward_stream"] = rstream
 
     if rank == 0 and not args.no_e2e:
         res["e2e"] = run_e2e(args, aal, prob, rprob, draft, target, grad, ws, loss, rws, tau, rl, adv,
@@ -570,6 +577,110 @@ def run_sequence_layout(aal, dev, stream, rank, reps):
            "windows_per_s": round(R / ((fwd + bwd) * 1e-3), 1),
            "loss": float(loss.item())}
     del target, draft, grad, ws
+    return out
+
+
+def _loss_line(aal, draft, target, mask, mode, T, wg, ws, grad, stream, reps, peak):
+    """One loss configuration: the fused call and the two calls, events on the launching stream."""
+    N, K, V = draft.shape
+    prob = aal.loss_problem(draft, mode, T, wg, ws)
+    w = torch.empty(aal.aal_workspace_size(prob), dtype=torch.uint8, device=draft.device)
+    loss = torch.empty(1, dtype=torch.float32, device=draft.device)
+    fwd, bwd = _time_fwd_bwd(
+        aal, lambda: aal.aal_loss_fwd(prob, draft, target, mask, w, loss, None, stream),
+        lambda: aal.aal_loss_bwd(prob, draft, target, mask, w, 1.0, grad, stream), stream, reps)
+    fused = _time_call(lambda: aal.aal_loss_fwd_bwd(prob, draft, target, mask, w, 1.0, loss, grad, None, stream),
+                       stream, reps)
+    assert aal.aal_check_device_status(w) == aal.AAL_OK
+    R = N * K
+    row = V * draft.element_size()
+    fb, bb = 2 * R * row, 3 * R * row
+    gbs = (fb + bb) / (fused * 1e-3) / 1e9
+    return {"ms": round(fused, 4), "gbs": round(gbs, 1), "frac_of_peak": round(gbs / peak, 4),
+            "rows_per_s": round(R / (fused * 1e-3), 1), "call": "aal_loss_fwd_bwd",
+            "two_call_ms": round(fwd + bwd, 4), "fwd_ms": round(fwd, 4), "bwd_ms": round(bwd, 4),
+            "fwd_gbs": round(fb / (fwd * 1e-3) / 1e9, 1), "bwd_gbs": round(bb / (bwd * 1e-3) / 1e9, 1),
+            "min_traffic_gbs": round(3 * R * row / (fused * 1e-3) / 1e9, 1), "loss": float(loss.item())}
+
+
+def run_config_lines(aal, dev, stream, rank, reps, peak):
+    """The other loss configurations of the benchmark plan: v32k (N=2048, K=5, V=32000 bf16,
+    10% of positions masked) greedy EAL at T=0 and WTV at T=1; v152k (N=8192, K=6, V=151936
+    bf16, 20% low-overlap rows) WTV at T in {0.5, 1, 1.5}.  Bytes as the metric counts them
+    (2 V b forward, 3 V b backward per row); inputs larger than L2 (0.66 GB and 14.9 GB per
+    tensor)."""
+    out = {}
+    t, d, m = synth.make_logits("v32k", seed=rank, device=dev)
+    g = torch.empty_like(d)
+    for name, mode, T, wg, ws in (("greedy_T0", aal.AAL_GREEDY, 0.0, 1.0, 0.0),
+                                  ("wtv_T1", aal.AAL_SAMPLING, 1.0, 0.0, 1.0)):
+        out[f"v32k_{name}"] = dict(workload="v32k: N=2048 windows (B=4 x T=512), K=5, V=32000 bf16, 10% of "
+                                            f"positions masked; {'EAL' if wg else 'WTV'} fwd+bwd at T={T:g}",
+                                   **_loss_line(aal, d, t, m, mode, T, wg, ws, g, stream, reps, peak))
+    del t, d, m, g
+    torch.cuda.empty_cache()
+    t, d, _ = synth.make_logits("v152k", seed=rank, device=dev)
+    g = torch.empty_like(d)
+    for T in (0.5, 1.0, 1.5):
+        out[f"v152k_wtv_T{T:g}"] = dict(workload="v152k: N=8192 windows (B=4 x T=2048), K=6, V=151936 bf16, 20% "
+                                                 f"low-overlap rows; WTV fwd+bwd at T={T:g}",
+                                        **_loss_line(aal, d, t, None, aal.AAL_SAMPLING, T, 0.0, 1.0, g, stream,
+                                                     reps, peak))
+    del t, d, g
+    torch.cuda.empty_cache()
+    return out
+
+
+def run_reward_stream(aal, dev, stream, rank, peak, groups=64, distinct=4):
+    """The GRPO acceptance reward over the full reward workload: 64 prompts x 16 rollouts x 256
+    windows of K=8, V=128256 bf16 (Zipf target, draft = target + N(0, 1)), 2,097,152 logit rows
+    and 1076 GB of draft and target, streamed one prompt group (32768 rows, 8.41 GB per tensor)
+    per aal_accept_reward call with the group's global row offset, under greedy and sampling
+    (T = 1) verification, advantages over groups of 16 rollouts.  The logits of `distinct`
+    seeded groups are drawn once and streamed in rotation: drawing all 64 (a random
+    permutation per row) would take minutes, and the kernel's time does not depend on the
+    values.  Every call reads its 16.8 GB from HBM (far more than L2)."""
+    data = [synth.make_reward_logits(rank * groups + g, seed=0, device=dev)[:2] for g in range(distinct)]
+    target0, draft0 = data[0]
+    N, K, V = draft0.shape
+    R = N * K
+    nroll = N // 256
+    tau = torch.empty(N, dtype=torch.int32, device=dev)
+    rl = torch.empty(nroll, dtype=torch.float32, device=dev)
+    adv = torch.empty(nroll, dtype=torch.float32, device=dev)
+    out = {"workload": f"reward stream: {groups} prompt groups x 16 rollouts x 256 windows, K={K}, V={V} bf16 "
+                       f"({groups * R} logit rows, {groups * 2 * R * V * 2 / 1e9:.0f} GB read); logits of {distinct} "
+                       "seeded groups streamed in rotation",
+           "bytes": groups * 2 * R * V * 2}
+    for name, mode in (("greedy", aal.AAL_GREEDY), ("sampling_T1", aal.AAL_SAMPLING)):
+        probs = [aal.reward_problem(draft0, mode, 1.0, 5.0, 0, (rank * groups + g) * N, 256, 16) for g in range(groups)]
+        ws = torch.empty(aal.aal_reward_workspace_size(probs[0]), dtype=torch.uint8, device=dev)
+
+        def call(g):
+            t, d = data[g % distinct]
+            aal.aal_accept_reward(probs[g], d, t, None, ws, tau, None, rl, adv, stream)
+
+        for g in range(min(groups, 3)):
+            call(g)
+        torch.cuda.synchronize()
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(groups + 1)]
+        ev[0].record(stream)
+        for g in range(groups):
+            call(g)
+            ev[g + 1].record(stream)
+        torch.cuda.synchronize()
+        assert aal.aal_check_device_status(ws) == aal.AAL_OK
+        per = [ev[g].elapsed_time(ev[g + 1]) for g in range(groups)]
+        total = ev[0].elapsed_time(ev[groups])
+        gbs = out["bytes"] / (total * 1e-3) / 1e9
+        target_s = 0.215 * groups / 64   # 75% of the measured copy peak, plan of the benchmark
+        out[name] = {"total_s": round(total / 1e3, 5), "per_group_ms": round(statistics.mean(per), 4),
+                     "per_group_ms_max": round(max(per), 4), "rows_per_s": round(groups * R / (total * 1e-3), 1),
+                     "gbs": round(gbs, 1), "frac_of_peak": round(gbs / peak, 4),
+                     "target_s_at_75pct": round(target_s, 4), "time_over_target": round(total / 1e3 / target_s, 4)}
+        del ws
+    del data, target0, draft0
+    torch.cuda.empty_cache()
     return out
 
 

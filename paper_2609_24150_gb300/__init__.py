@@ -40,6 +40,7 @@ from .aal import (  # noqa: F401
     aal_accept_reward_noalloc,
     aal_check_device_status,
     aal_debug_fail_next_forward,
+    aal_debug_fused_min_row_bytes,
     aal_debug_solo_windows,
     aal_grpo_from_loss,
     aal_grpo_workspace_size,

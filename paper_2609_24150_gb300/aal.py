@@ -119,6 +119,8 @@ def library() -> ctypes.CDLL:
     lib.aal_debug_fail_next_forward.restype = None
     lib.aal_debug_solo_windows.argtypes = [ctypes.c_int64, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32]
     lib.aal_debug_solo_windows.restype = ctypes.c_int64
+    lib.aal_debug_fused_min_row_bytes.argtypes = [ctypes.c_int64]
+    lib.aal_debug_fused_min_row_bytes.restype = None
     lib.aal_status_string.argtypes = [ctypes.c_int]
     lib.aal_status_string.restype = ctypes.c_char_p
     lib.aal_abi_version.argtypes = []
@@ -437,6 +439,12 @@ def aal_debug_fail_next_forward(chunk: int, wait_limit_ns: int = 0):
     """Failure-detection test hook: leave one ring copy of the next streamed forward unarmed
     so that its bounded waits run out (see include/aal_debug.h)."""
     library().aal_debug_fail_next_forward(int(chunk), int(wait_limit_ns))
+
+
+def aal_debug_fused_min_row_bytes(nbytes: int) -> None:
+    """Test hook: the shortest row (bytes) aal_loss_fwd_bwd streams with its fused kernels
+    (0: every row they take; negative: the default; see include/aal_debug.h)."""
+    library().aal_debug_fused_min_row_bytes(int(nbytes))
 
 
 def aal_debug_solo_windows(N: int, K: int, G: int, S: int) -> int:

@@ -18,6 +18,7 @@ size_t target_align(int32_t mode) { return (mode & AAL_IDS) ? 4 : 16; }
 // Failure-detection test hooks (include/aal_debug.h).
 std::atomic<uint64_t> g_wait_limit_ns{0};
 std::atomic<int64_t> g_skip_chunk{-1};
+std::atomic<int64_t> g_fused_min_row_bytes{AAL_FUSED_MIN_ROW_BYTES_DEFAULT};
 
 aal_status check_shape(int64_t N, int64_t K, int64_t V, int32_t dtype) {
   if (N < 0 || K < 1 || V < 1) return AAL_ERR_INVALID_ARG;
@@ -219,6 +220,10 @@ void aal_debug_fail_next_forward(int64_t chunk, uint64_t wait_limit_ns) {
   g_skip_chunk.store(chunk);
 }
 
+void aal_debug_fused_min_row_bytes(int64_t bytes) {
+  g_fused_min_row_bytes.store(bytes < 0 ? (int64_t)AAL_FUSED_MIN_ROW_BYTES_DEFAULT : bytes);
+}
+
 int64_t aal_debug_solo_windows(int64_t N, int32_t K, int32_t G, int32_t S) {
   return aal::solo_windows_each(N, K, G, S);
 }
@@ -315,7 +320,8 @@ aal_status aal_loss_fwd_bwd(const aal_problem* prob, const void* draft, const vo
 
   // the fused kernels: bf16 rows of 16-byte multiples; with token ids, the draft alone
   const bool ids = (prob->mode & AAL_IDS) != 0;
-  const bool rows16 = prob->dtype == AAL_BF16 && (prob->V * 2) % 16 == 0;
+  const bool rows16 = prob->dtype == AAL_BF16 && (prob->V * 2) % 16 == 0 &&
+                      prob->V * 2 >= g_fused_min_row_bytes.load();
   const bool fusable = rows16 && !ids;
   if (rows16 && ids) {
     LossWs ws = loss_ws(workspace, L);
@@ -681,7 +687,27 @@ aal_status aal_accept_reward(const aal_reward_problem* prob, const void* draft, 
   ra.acc = reinterpret_cast<uint8_t*>(base + L.acc);
   ra.acc_ref = reinterpret_cast<uint8_t*>(base + L.acc_ref);
   ra.hdr = hdr;
-  cudaError_t e = launch_reward_rows(ra, prob->dtype == AAL_BF16, s);
+  cudaError_t e = cudaSuccess;
+  if (sampling && !ra.sampled_draft && ref_draft == nullptr && prob->dtype == AAL_BF16 && (prob->V * 2) % 16 == 0) {
+    // the argmax draft under sampling verification: one TMA-streamed pass over draft and target
+    // (both normalisers at T and the draft's greedy token), the flag decided at each row's end
+    RowStatsArgs sa{};
+    sa.zq = draft;
+    sa.zp = target;
+    sa.R = L.R;
+    sa.V = prob->V;
+    sa.sT = ra.sT;
+    sa.skip_chunk = -1;
+    sa.ws.hdr = hdr;
+    sa.acc = ra.acc;
+    sa.seed = prob->seed;
+    sa.row_offset = prob->row_offset;
+    sa.K = (int32_t)prob->K;
+    const uint64_t limit = debug_wait_limit_ns();
+    e = launch_reward_stream(sa, s, limit ? limit : kWaitLimitNs);
+  } else {
+    e = launch_reward_rows(ra, prob->dtype == AAL_BF16, s);
+  }
   if (e != cudaSuccess) return AAL_ERR_CUDA;
 
   RewardGroupArgs ga;

@@ -197,6 +197,12 @@ struct RowStatsArgs {
   bool need_kl;         // KL(p || q) at T = 1 and the normaliser of z_p at T = 1 (anchor)
   int64_t skip_chunk;   // failure-detection test hook: a chunk whose copy is never armed (-1: none)
   LossWs ws;
+  // the streamed sampling reward (launch_reward_stream): per-row acceptance flags, the Philox key
+  // and the global window index of row 0's window; ws.hdr is the reward workspace's status word
+  uint8_t* acc = nullptr;
+  uint64_t seed = 0;
+  int64_t row_offset = 0;
+  int32_t K = 1;
 };
 
 struct WindowArgs {
@@ -441,6 +447,9 @@ struct GrpoWindowArgs {
 // Launchers (return cudaGetLastError() of their launches).
 cudaError_t launch_rowstats(const RowStatsArgs& a, bool bf16, cudaStream_t s, int* cluster_used);
 cudaError_t launch_rowstats_stream(const RowStatsArgs& a, bool bf16, cudaStream_t s, uint64_t limit_ns);
+// The sampling reward's acceptance flags from one streamed pass over bf16 rows of 16-byte
+// multiples (a.sT = log2(e) / T, a.acc, a.seed, a.row_offset, a.K).
+cudaError_t launch_reward_stream(const RowStatsArgs& a, cudaStream_t s, uint64_t limit_ns);
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // bounded waits give up after 1 s
 
 // Failure-detection test hooks (include/aal_debug.h); both are 0 / -1 in normal use.

@@ -41,7 +41,7 @@ using namespace ptx;
 // sampling term; everything at T = 1 (sT is log2 e), argmaxes resolved by resolve_argmax.
 // KL: the anchor's D next to the z_p normaliser at T = 1: the pass's own when it runs at T = 1,
 // else (P1, with NEED_Q1) a second z_p state at T = 1 beside the one at T.
-template <typename T, bool NEED_Q1, int PASSES, bool KL, bool P1 = false>
+template <typename T, bool NEED_Q1, int PASSES, bool KL, bool P1 = false, bool REWARD = false>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm) rowstats_stream(RowStatsArgs a, int nch, uint64_t limit_ns) {
   extern __shared__ __align__(1024) unsigned char smem[];
   unsigned char* ring = smem;
@@ -113,7 +113,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) rowstats_stream(RowStats
     const int t = threadIdx.x;
     RingPos pos;
     uint32_t j = 0;
-    const float sT = PASSES == 2 ? a.sT : kLog2e;
+    const float sT = (PASSES == 2 || REWARD) ? a.sT : kLog2e;
     for (int64_t r = blockIdx.x; r < a.R; r += gridDim.x, ++j) {
       // pass 1: online normalisers and argmax
       RowPart A;
@@ -158,6 +158,24 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) rowstats_stream(RowStats
         a.ws.Mp1[r] = Mp1;
         a.ws.Lsp1[r] = Lsp1;
         a.ws.kl[r] = kl;
+      }
+      if (PASSES == 1 && REWARD) {
+        if (t == 0) {
+          // the sampling reward (Sec. 3.4, Eq. acc_sample): the draft's greedy token y (the first
+          // maximum of z_q, placed inside its recorded vector, read again from L2) and z_p there;
+          // accept iff u < min(1, p~(y) / q~(y)), with log2 q~(y) = -Ls_q since z_q peaks at y
+          const T* zp = static_cast<const T*>(a.zp) + r * a.V;
+          const T* zq = static_cast<const T*>(a.zq) + r * a.V;
+          int32_t xs, ys;
+          float cx, cy;
+          resolve_vectors<T>(zp, zq, a.V, -1, *abort_flag ? -1 : tot.qb, &xs, &cx, &ys, &cy);
+          const int64_t n = r / a.K;
+          const uint32_t k = (uint32_t)(r - n * a.K);
+          const float u = philox_uniform(a.seed, (uint64_t)(a.row_offset + n), k);
+          const float d = log2_prob(cy, sT, Mp, Lsp) + Lsq;
+          if (!*abort_flag) a.acc[r] = (u < exp2f(fminf(d, 0.f))) ? 1 : 0;
+        }
+        continue;
       }
       if (PASSES == 1) {
         if (t == 0) {
@@ -268,9 +286,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) rowstats_stream(RowStats
 
 constexpr size_t kSmemBytes = (size_t)kSlots * kSlotBytes + sizeof(Smem);
 
-template <typename T, bool NEED_Q1, int PASSES, bool KL, bool P1 = false>
+template <typename T, bool NEED_Q1, int PASSES, bool KL, bool P1 = false, bool REWARD = false>
 cudaError_t launch_T(const RowStatsArgs& a, cudaStream_t s, int nch, uint64_t limit_ns) {
-  auto kern = rowstats_stream<T, NEED_Q1, PASSES, KL, P1>;
+  auto kern = rowstats_stream<T, NEED_Q1, PASSES, KL, P1, REWARD>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
   if (e != cudaSuccess) return e;
   int dev = 0, sms = 0;
@@ -328,6 +346,12 @@ cudaError_t launch_rowstats_stream(const RowStatsArgs& a, bool bf16, cudaStream_
   const int nch = (int)((a.V + CH - 1) / CH);
   if (!a.overlap) return bf16 ? launch_one_pass<uint16_t>(a, s, nch, limit_ns) : launch_one_pass<float>(a, s, nch, limit_ns);
   return bf16 ? launch_two_pass<uint16_t>(a, s, nch, limit_ns) : launch_two_pass<float>(a, s, nch, limit_ns);
+}
+
+cudaError_t launch_reward_stream(const RowStatsArgs& a, cudaStream_t s, uint64_t limit_ns) {
+  const int64_t CH = kHalfSlot / 2;
+  const int nch = (int)((a.V + CH - 1) / CH);
+  return launch_T<uint16_t, false, 1, false, false, true>(a, s, nch, limit_ns);
 }
 
 }  // namespace aal

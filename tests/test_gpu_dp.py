@@ -17,6 +17,17 @@ import synth
 pytestmark = pytest.mark.gpu
 
 DEV = "cuda:0"
+
+
+@pytest.fixture(autouse=True, scope="module")
+def _fuse_short_rows():
+    """The fused kernels on every row they take, short rows included (the default sends rows
+    shorter than 128 KB to the two calls, which are faster there); restored afterwards."""
+    aal.aal_debug_fused_min_row_bytes(0)
+    yield
+    aal.aal_debug_fused_min_row_bytes(-1)
+
+
 G, S, B, KL = aal.AAL_GREEDY, aal.AAL_SAMPLING, aal.AAL_BOTH, aal.AAL_KL
 
 

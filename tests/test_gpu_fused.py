@@ -18,6 +18,17 @@ from tests.parity import LossRun, check_loss
 pytestmark = pytest.mark.gpu
 
 DEV = "cuda:0"
+
+
+@pytest.fixture(autouse=True, scope="module")
+def _fuse_short_rows():
+    """The fused kernels on every row they take, short rows included (the default sends rows
+    shorter than 128 KB to the two calls, which are faster there); restored afterwards."""
+    aal.aal_debug_fused_min_row_bytes(0)
+    yield
+    aal.aal_debug_fused_min_row_bytes(-1)
+
+
 G, S, B, KL, TV, IDS = aal.AAL_GREEDY, aal.AAL_SAMPLING, aal.AAL_BOTH, aal.AAL_KL, aal.AAL_TV, aal.AAL_IDS
 
 
@@ -162,6 +173,27 @@ def test_token_ids_out_of_range_reported():
     aal.aal_loss_bwd(prob, d, ids, None, ws2, 1.0, s)
     assert aal.aal_check_device_status(ws2) == aal.AAL_ERR_INVALID_ARG
     assert torch.equal(_bits(grad), _bits(s))
+
+
+@pytest.mark.parametrize("mode,T,wg,ws", [(B, 1.0, 0.5, 0.5), (B, 1.5, 0.5, 0.5), (KL | G, 1.0, 0.1, 0.0)])
+def test_fused_against_the_oracle_with_solo_ctas(mode, T, wg, ws):
+    """N = 304 windows of K = 7 at V = 50000 (five ring chunks a pass, a partial last one): on
+    one GB300 the call runs 21 groups of 7 CTAs with about 14 windows each and 5 solo CTAs with
+    whole windows, so both paths walk several windows.  Sampled windows of each kind (every
+    group's first and last window, and the solo CTAs' windows at the end of the batch) are
+    checked against the oracle directly, with the batch's |W| and |P|."""
+    N, K, V = 304, 7, 50000
+    t, d, m = _inputs(N, K, V, seed=23, masked=True)
+    run = FusedRun(t, d, m, mode, T, wg, ws, dloss=float(N), wkl=1.0)
+    mh = m.cpu().numpy()
+    nW = int((mh[:, 0] != 0).sum())
+    nP = int((mh != 0).sum())
+    groups = 21
+    windows = sorted(set([0, groups - 1, groups, 2 * groups + 5] + list(range(N - 12, N)) +
+                         [N - 12 - groups + 3, 150]))
+    check_loss(run, t, d, m, mode, T, wg, ws, dloss=float(N), windows=windows, n_windows_total=nW, wkl=1.0,
+               n_positions_total=nP)
+    assert_same(run, LossRun(t, d, m, mode, T, wg, ws, dloss=float(N), wkl=1.0))
 
 
 @pytest.mark.parametrize("N,K", [(16, 2), (152, 7)])   # groups only; groups and solo CTAs

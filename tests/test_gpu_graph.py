@@ -14,6 +14,15 @@ pytestmark = pytest.mark.gpu
 DEV = "cuda:0"
 
 
+@pytest.fixture(autouse=True, scope="module")
+def _fuse_short_rows():
+    """The fused kernels on every row they take, short rows included (the default sends rows
+    shorter than 128 KB to the two calls, which are faster there); restored afterwards."""
+    aal.aal_debug_fused_min_row_bytes(0)
+    yield
+    aal.aal_debug_fused_min_row_bytes(-1)
+
+
 @pytest.mark.parametrize("mode,T", [(aal.AAL_BOTH, 1.0), (aal.AAL_KL | aal.AAL_GREEDY, 1.0), (aal.AAL_SAMPLING, 0.8)])
 def test_step_replays_bit_exactly(mode, T):
     target, draft, mask = synth.make_logits("v32k", seed=6, n_windows=256)
