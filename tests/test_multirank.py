@@ -4,7 +4,10 @@ Windows are independent, so ranks shard them with no collective on the data path
 step time is reduced (max over ranks).  The reward's counter-based draws are keyed by the
 global window index, so a sharded run reproduces the unsharded one exactly, and per-rank
 loss partials (sum of w * E[L], |W|; with the anchor also sum KL and |positions|) combine
-into the global loss with one all-reduce, for windows and for sharded sequences.
+into the global loss with one all-reduce, for windows and for sharded sequences.  With the
+data-parallel normalisers (the library's global_counts), one all-reduce of two integers before
+the step gives |W| and |P| of the whole batch, and the ranks' losses normalised by them sum to
+the whole batch's loss (the GPU side of that is tests/test_gpu_dp.py).
 """
 
 import multiprocessing as mp
@@ -58,6 +61,21 @@ def _worker(rank, world, port, out):
                            float(an["npos"])], dtype=torch.float64)
         dist.all_reduce(sp)
         res["seq_loss"] = float(-0.1 * sp[0] / sp[1] + sp[2] / sp[3])
+        # data-parallel normalisers (the library's global_counts): each rank counts its shard's |W|
+        # (windows whose depth 0 is valid) and |P| (valid positions), one all-reduce of the two
+        # integers gives the whole batch's, and each rank's objective normalised by them; the
+        # ranks' losses then sum to the whole batch's, with no collective on the data path
+        tg, dg, mg = synth.make_logits("tiny", seed=5, N=8, K=4, V=64, mask_rate=0.3)
+        ml = mg[lo:lo + per].numpy()
+        counts = torch.tensor([int((ml[:, 0] != 0).sum()), int((ml != 0).sum())], dtype=torch.int64)
+        dist.all_reduce(counts)
+        nW, nP = int(counts[0]), int(counts[1])
+        omode = oracle.MODE_KL | oracle.MODE_BOTH
+        lr = oracle.objective_forward(tg[lo:lo + per], dg[lo:lo + per], ml, omode, 0.9, 0.5, 0.5, 1.0, nW, nP)["loss"]
+        tot = torch.tensor([lr], dtype=torch.float64)
+        dist.all_reduce(tot)
+        res["dp_counts"] = (nW, nP)
+        res["dp_loss"] = float(tot[0])
         out.put((rank, res))
     finally:
         dist.destroy_process_group()
@@ -83,7 +101,12 @@ def test_two_gloo_ranks():
     st, sd, sm = synth.make_seq_logits("seq_tiny", seed=4, B=4, seq_len=11, V=50)
     ref_seq = oracle.seq_objective_forward(st, sd, sm.numpy(), 3, oracle.MODE_KL | oracle.MODE_GREEDY, 1.0,
                                            0.1, 0.0, 1.0)["loss"]
+    tg, dg, mg = synth.make_logits("tiny", seed=5, N=8, K=4, V=64, mask_rate=0.3)
+    mh = mg.numpy()
+    ref_dp = oracle.objective_forward(tg, dg, mh, oracle.MODE_KL | oracle.MODE_BOTH, 0.9, 0.5, 0.5, 1.0)["loss"]
     for r in range(2):
+        assert results[r]["dp_counts"] == (int((mh[:, 0] != 0).sum()), int((mh != 0).sum()))
+        assert abs(results[r]["dp_loss"] - ref_dp) < 1e-12
         assert results[r]["max"] == 20.0
         np.testing.assert_array_equal(results[r]["tau"], whole["tau"])
         assert abs(results[r]["loss"] - ref_loss) < 1e-12
