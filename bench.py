@@ -831,7 +831,8 @@ def cpu_baseline(draft, target, seconds, cores=None):
     t0 = time.perf_counter()
     _oracle_step(target[:1].cpu(), draft[:1].cpu(), 0)
     one = time.perf_counter() - t0
-    n = int(max(cores, min(draft.shape[0], cores * max(1, round(seconds / max(one, 1e-3))))))
+    # as many windows as each core does in about `seconds`, at most 1024 (3.7 GB of shared sample)
+    n = int(max(cores, min(draft.shape[0], 1024, cores * max(1, round(seconds / max(one, 1e-3))))))
     pool = OraclePool(target[:n], draft[:n], cores)
     try:
         t0 = time.perf_counter()
