@@ -32,6 +32,8 @@
 // * Failure: every wait is bounded.  A CTA that gave up keeps walking its rows without waiting
 //   and still publishes a word for each, so its group does not wait on it for the whole limit;
 //   the workspace status word reports AAL_ERR_TIMEOUT and the outputs are not to be used.
+#include <type_traits>
+
 #include "grad_elem.cuh"
 #include "stream_core.cuh"
 
@@ -233,6 +235,8 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
           st.ag = ag;
           st.xs = xs;
           st.ys = ys;
+          // a group CTA's row: its mailbox word as soon as it is known (the exchange then only polls)
+          if (!solo) ptx::st_relaxed(&a.ws.mbox[r], mbox_word(ag, 0.f));
         }
       } else {
         // ---- pass 2: overlap sums (L2)
@@ -320,6 +324,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
           st.ag = ag;
           st.xs = S.arg_index;
           st.ys = S.yarg_index;
+          if (!solo) ptx::st_relaxed(&a.ws.mbox[r], mbox_word(ag, x.x));
           S.arg_index = 0x7fffffff;
           S.arg_carry = 0.f;
           S.yarg_index = 0x7fffffff;
@@ -332,8 +337,9 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
     // Thread 0: the coefficients of depth kk of window n (row r) from the window's acceptances
     // (agv, asv; 0 beyond K and for a term the window kernel does not form), as the window
     // kernel forms its terms and the backward its coefficients.  Returns whether any is nonzero.
+    // LOCAL_DONE: the row-local part of c was formed already (row_coef_local).
     auto coef_row = [&](int64_t n, int kk, int64_t r, const float* agv, const float* asv, const RowStat& st,
-                        RowCoef& c) -> int32_t {
+                        RowCoef& c, auto local_done) -> int32_t {
       const int64_t r0 = n * K;
       int kn = K;
       if (f.win.mask != nullptr) {
@@ -353,8 +359,8 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
       }
       const bool with_greedy = GREEDY && f.bw.w_greedy != 0.f;
       const bool pos_valid = f.bw.mask == nullptr || f.bw.mask[r] != 0;
-      return row_coef<GREEDY, SAMPLING, KL>(f.bw, scale, kscale, with_greedy ? dEg : 0.f, SAMPLING ? dEs : 0.f, 0.f,
-                                            pos_valid, st, c)
+      return row_coef<GREEDY, SAMPLING, KL, decltype(local_done)::value>(
+                 f.bw, scale, kscale, with_greedy ? dEg : 0.f, SAMPLING ? dEs : 0.f, 0.f, pos_valid, st, c)
                  ? 1
                  : 0;
     };
@@ -400,16 +406,19 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
         if (warp == 0) {
           const bool need = f.win.greedy || ov;  // the anchor alone needs no window term
           float agv[AAL_MAX_K], asv[AAL_MAX_K];
+          // the row's word was published with its statistics; the row-local coefficients are
+          // formed while the first poll of the window's words is in flight
+          RowCoef c;
           const bool ok = window_exchange(a.ws.mbox, r, n * K, K, lane, st.ag, PASSES == 2 ? st_as : 0.f, need,
-                                          abort_flag, hdr, limit_ns, agv, asv);
+                                          abort_flag, hdr, limit_ns, agv, asv, false,
+                                          [&]() { row_coef_local<GREEDY, SAMPLING, KL>(f.bw, st, c); });
 #pragma unroll
           for (int jj = 0; jj < AAL_MAX_K; ++jj) {  // only the terms the window kernel forms
             if (!f.win.greedy) agv[jj] = 0.f;
             if (!ov) asv[jj] = 0.f;
           }
           if (lane == 0) {
-            RowCoef c;
-            F.live = ok ? coef_row(n, k, r, agv, asv, st, c) : 0;
+            F.live = ok ? coef_row(n, k, r, agv, asv, st, c, std::true_type()) : 0;
             if (F.live) F.coef = c;
           }
         }
@@ -441,7 +450,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
           for (int kk = 0; kk < K; ++kk) {
             RowCoef c;
             const bool ok = !*abort_flag;
-            F.solo_live[kk] = ok ? coef_row(n, kk, n * K + kk, agv, asv, F.solo_st[kk], c) : 0;
+            F.solo_live[kk] = ok ? coef_row(n, kk, n * K + kk, agv, asv, F.solo_st[kk], c, std::false_type()) : 0;
             if (F.solo_live[kk]) F.solo_coef[kk] = c;
           }
         }

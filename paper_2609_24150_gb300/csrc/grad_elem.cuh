@@ -121,10 +121,22 @@ __device__ __forceinline__ RowStat load_row_stat(const LossWs& ws, int64_t r, bo
   return st;
 }
 
+// The row-local part of the coefficients: the offsets nC = -(M + Ls / s) of q~, p~ (at T) and of
+// q, p (at T = 1), from the row's own statistics (no window term), each rounding spelled out.
+template <bool GREEDY, bool SAMPLING, bool KL>
+__device__ __forceinline__ void row_coef_local(const BackwardArgs& a, const RowStat& st, RowCoef& c) {
+  c.sT = a.sT;
+  c.nCq = SAMPLING ? -__fadd_rn(st.Mq, __fdiv_rn(st.Lsq, a.sT)) : 0.f;
+  c.nCp = SAMPLING ? -__fadd_rn(st.Mp, __fdiv_rn(st.Lsp, a.sT)) : 0.f;
+  c.nCq1 = (GREEDY || KL) ? -__fadd_rn(st.Mq1, __fdiv_rn(st.Lsq1, kLog2e)) : 0.f;
+  c.nCp1 = KL ? -__fadd_rn(st.Mp1, __fdiv_rn(st.Lsp1, kLog2e)) : 0.f;
+}
+
 // The row's coefficients from its statistics, dE^g/da (unweighted), dE^s/da (weights folded),
 // the GRPO coefficient and whether the row is a valid position (the anchor's rows).  Returns
-// false when every term of the row is zero (the row's gradient is all zeros).
-template <bool GREEDY, bool SAMPLING, bool KL>
+// false when every term of the row is zero (the row's gradient is all zeros).  LOCAL_DONE: the
+// caller already formed the row-local part with row_coef_local (the same values).
+template <bool GREEDY, bool SAMPLING, bool KL, bool LOCAL_DONE = false>
 __device__ __forceinline__ bool row_coef(const BackwardArgs& a, float scale, float kscale, float dEg, float dEs,
                                          float cgr, bool pos_valid, const RowStat& st, RowCoef& c) {
   // every rounding spelled out (no contraction into fused multiply-adds), so that each kernel
@@ -134,11 +146,7 @@ __device__ __forceinline__ bool row_coef(const BackwardArgs& a, float scale, flo
   const float gs = SAMPLING ? __fmul_rn(__fmul_rn(scale, a.w_sampling), dEs) : 0.f;
   const float ck = (KL && pos_valid) ? kscale : 0.f;
   if (gg == 0.f && gs == 0.f && ck == 0.f && cg == 0.f) return false;
-  c.sT = a.sT;
-  c.nCq = SAMPLING ? -__fadd_rn(st.Mq, __fdiv_rn(st.Lsq, a.sT)) : 0.f;
-  c.nCp = SAMPLING ? -__fadd_rn(st.Mp, __fdiv_rn(st.Lsp, a.sT)) : 0.f;
-  c.nCq1 = (GREEDY || KL) ? -__fadd_rn(st.Mq1, __fdiv_rn(st.Lsq1, kLog2e)) : 0.f;
-  c.nCp1 = KL ? -__fadd_rn(st.Mp1, __fdiv_rn(st.Lsp1, kLog2e)) : 0.f;
+  if (!LOCAL_DONE) row_coef_local<GREEDY, SAMPLING, KL>(a, st, c);
   c.Ck = ck;
   const float qlt = SAMPLING ? st.qlt : 0.f;
   const float Bs = __fmul_rn(gs, a.invT);
@@ -248,20 +256,32 @@ __device__ __forceinline__ uint4 grad_vec(const RowCoef& c, const uint4& qw, con
 // is false (no window term) nothing is polled.  Returns, to every lane, whether the window's
 // words arrived; on lane 0, ag[j] and as[j] hold depth j's values (0 beyond K).  The abort flag
 // is read once for the warp (another warp may raise it meanwhile).
+struct NoPrePoll {
+  __device__ void operator()() const {}
+};
+
+// This row's mailbox word: (a^greedy, a^sample) as one 64-bit value, never the empty sentinel.
+__device__ __forceinline__ uint64_t mbox_word(float ag_r, float as_r) {
+  uint64_t word = ((uint64_t)__float_as_uint(as_r) << 32) | __float_as_uint(ag_r);
+  return word == kMboxEmpty ? 0 : word;  // (bit patterns no arithmetic yields; never sent)
+}
+
+// `publish`: lane 0 writes this row's word first (false when the caller has already written it);
+// `pre`: run by lane 0 before the window's words are polled, while the first poll is in flight.
+template <typename Pre = NoPrePoll>
 __device__ __forceinline__ bool window_exchange(uint64_t* mbox, int64_t r, int64_t r0, int K, int lane, float ag_r,
                                                 float as_r, bool need, volatile int* abort_flag, WsHeader* hdr,
-                                                uint64_t limit_ns, float* ag, float* as) {
-  if (lane == 0) {
-    uint64_t word = ((uint64_t)__float_as_uint(as_r) << 32) | __float_as_uint(ag_r);
-    if (word == kMboxEmpty) word = 0;  // (bit patterns no arithmetic yields; never sent)
-    ptx::st_relaxed(&mbox[r], word);
-  }
+                                                uint64_t limit_ns, float* ag, float* as, bool publish = true,
+                                                Pre pre = Pre()) {
+  if (lane == 0 && publish) ptx::st_relaxed(&mbox[r], mbox_word(ag_r, as_r));
   bool ok = __shfl_sync(0xffffffffu, *abort_flag == 0 ? 1 : 0, 0) != 0;
   uint64_t w = 0;
+  if (lane == 0 && !(ok && need)) pre();  // nothing to poll: the caller's work runs now
   if (ok && need) {
     const uint64_t t0 = ptx::now_ns();
     for (uint32_t it = 0;; ++it) {
       if (lane < K) w = ptx::ld_relaxed(&mbox[r0 + lane]);
+      if (it == 0 && lane == 0) pre();
       if (__all_sync(0xffffffffu, lane >= K || w != kMboxEmpty)) break;
       int quit = 0;  // lane 0 decides for the warp whether to give up
       if (lane == 0 && (*abort_flag || it >= kSpinLimit || ptx::now_ns() - t0 > limit_ns)) {
