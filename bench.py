@@ -552,8 +552,9 @@ def run_seq_grpo_phase(aal, dev, stream, rank, reps):
 
 def run_sequence_layout(aal, dev, stream, rank, reps):
     """The same loss over the sequence layout (Sec. 3.3): 4 sequences x 2048 positions, a window
-    of K=7 starting at every position, logits stored once per position; fwd + bwd timed with
-    events on the launching stream.  Unmasked, so every row is read (and written) once."""
+    of K=7 starting at every position, logits stored once per position; the one-call forward +
+    backward (aal_seq_loss_fwd_bwd) and the two calls, timed with events on the launching stream.
+    Unmasked, so every row is read (and written) once."""
     target, draft, _ = synth.make_seq_logits("seq_v128k", seed=rank, device=dev, masked=False)
     B, T, V = draft.shape
     K = synth.SEQUENCES["seq_v128k"].K
@@ -564,17 +565,22 @@ def run_sequence_layout(aal, dev, stream, rank, reps):
     fwd, bwd = _time_fwd_bwd(
         aal, lambda: aal.aal_seq_loss_fwd(prob, draft, target, None, ws, loss, None, stream),
         lambda: aal.aal_seq_loss_bwd(prob, draft, target, None, ws, 1.0, grad, stream), stream, reps)
+    fused = _time_call(lambda: aal.aal_seq_loss_fwd_bwd(prob, draft, target, None, ws, 1.0, loss, grad, None,
+                                                        stream), stream, reps)
     assert aal.aal_check_device_status(ws) == aal.AAL_OK
     R = B * T
     row = V * draft.element_size()
     fb, bb = 2 * R * row, 3 * R * row
     out = {"workload": f"seq_v128k: B={B} x T={T} positions, K={K}, V={V} bf16, unmasked; "
                        "EAL+WTV 0.5/0.5 at T=1 fwd+bwd",
-           "ms": round(fwd + bwd, 4), "fwd_ms": round(fwd, 4), "bwd_ms": round(bwd, 4),
-           "gbs": round((fb + bb) / ((fwd + bwd) * 1e-3) / 1e9, 1),
+           "call": "aal_seq_loss_fwd_bwd",
+           "ms": round(fused, 4), "gbs": round((fb + bb) / (fused * 1e-3) / 1e9, 1),
+           "min_traffic_gbs": round(3 * R * row / (fused * 1e-3) / 1e9, 1),
+           "positions_per_s": round(R / (fused * 1e-3), 1),
+           "windows_per_s": round(R / (fused * 1e-3), 1),
+           "two_call_ms": round(fwd + bwd, 4), "fwd_ms": round(fwd, 4), "bwd_ms": round(bwd, 4),
+           "two_call_gbs": round((fb + bb) / ((fwd + bwd) * 1e-3) / 1e9, 1),
            "fwd_gbs": round(fb / (fwd * 1e-3) / 1e9, 1), "bwd_gbs": round(bb / (bwd * 1e-3) / 1e9, 1),
-           "positions_per_s": round(R / ((fwd + bwd) * 1e-3), 1),
-           "windows_per_s": round(R / ((fwd + bwd) * 1e-3), 1),
            "loss": float(loss.item())}
     del target, draft, grad, ws
     return out

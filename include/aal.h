@@ -235,6 +235,22 @@ AAL_API aal_status aal_seq_loss_bwd(const aal_seq_problem* prob, const void* dra
                                     const uint8_t* mask, const void* workspace, size_t workspace_bytes,
                                     float dloss, void* grad_draft, void* stream);
 
+/* Forward and backward of the sequence loss in one call (Sec. 3.3: every position's row is read
+ * once for all K windows that contain it): the loss, eal and workspace of aal_seq_loss_fwd and
+ * the gradient of aal_seq_loss_bwd with the same dloss, bit for bit (same arguments, layouts and
+ * rules as those two calls).  With bf16 rows whose byte length is a multiple of 16, one
+ * cooperative launch streams the positions with one CTA per SM, consecutive positions on
+ * consecutive SMs at the same time, so that a position's gradient (which needs the acceptances
+ * of the K - 1 positions before and after it) is written while its rows are still in L2: 2 V b
+ * read and V b written per position, instead of 2 V b (forward) + 3 V b (backward).  Other
+ * problems (fp32, unaligned rows, token ids) run the two calls inside this one.  AAL_GRPO is
+ * rejected with AAL_ERR_UNSUPPORTED (its coefficients come from aal_seq_grpo_from_loss, between
+ * the forward and the backward).  A bounded device wait that ran out is reported by
+ * aal_check_device_status as AAL_ERR_TIMEOUT; the outputs are then not to be used. */
+AAL_API aal_status aal_seq_loss_fwd_bwd(const aal_seq_problem* prob, const void* draft, const void* target,
+                                        const uint8_t* mask, void* workspace, size_t workspace_bytes,
+                                        float dloss, float* loss, float* eal, void* grad_draft, void* stream);
+
 /* The GRPO surrogate of Sec. 3.4 over the windows of a completed aal_loss_fwd.
  *   N, K, V, dtype       must equal the loss problem's (windows of K depths, no mask: every
  *                        window is verified over all K depths).

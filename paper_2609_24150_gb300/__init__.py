@@ -51,6 +51,7 @@ from .aal import (  # noqa: F401
     aal_loss_fwd_bwd,
     aal_reward_workspace_size,
     aal_seq_loss_bwd,
+    aal_seq_loss_fwd_bwd,
     aal_seq_loss_fwd,
     aal_seq_workspace_size,
     aal_status_string,

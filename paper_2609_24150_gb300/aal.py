@@ -109,6 +109,7 @@ def library() -> ctypes.CDLL:
     lib.aal_seq_workspace_size.argtypes = [SP, ctypes.POINTER(sz)]
     lib.aal_seq_loss_fwd.argtypes = [SP, vp, vp, vp, vp, sz, vp, vp, vp]
     lib.aal_seq_loss_bwd.argtypes = [SP, vp, vp, vp, vp, sz, ctypes.c_float, vp, vp]
+    lib.aal_seq_loss_fwd_bwd.argtypes = [SP, vp, vp, vp, vp, sz, ctypes.c_float, vp, vp, vp, vp]
     GP = ctypes.POINTER(AalGrpoProblem)
     lib.aal_grpo_workspace_size.argtypes = [GP, ctypes.POINTER(sz)]
     lib.aal_grpo_from_loss.argtypes = [GP, P, vp, sz, vp, vp, sz, vp, vp, vp, vp, vp, vp]
@@ -379,6 +380,20 @@ def aal_seq_loss_bwd(problem: AalSeqProblem, draft, target, mask, workspace, dlo
         _ptr(mask, "mask", torch.uint8), _ptr(workspace, "workspace"), _nbytes(workspace),
         float(dloss), _ptr(grad, "grad"), _stream(stream))
     _check(code, "aal_seq_loss_bwd")
+
+
+def aal_seq_loss_fwd_bwd(problem: AalSeqProblem, draft, target, mask, workspace, dloss: float, loss, grad,
+                         eal=None, stream=None):
+    """Forward and backward of the sequence loss in one call: loss[0] (and eal[B*seq_len][2]) as
+    aal_seq_loss_fwd, grad as aal_seq_loss_bwd with the same dloss; each position's logits are
+    read from HBM once."""
+    R = problem.B * problem.seq_len
+    code = library().aal_seq_loss_fwd_bwd(
+        ctypes.byref(problem), _ptr(draft, "draft"), _ptr(target, "target"),
+        _ptr(mask, "mask", torch.uint8, R), _ptr(workspace, "workspace"), _nbytes(workspace),
+        float(dloss), _ptr(loss, "loss", torch.float32, 1), _ptr(eal, "eal", torch.float32, 2 * R),
+        _ptr(grad, "grad"), _stream(stream))
+    _check(code, "aal_seq_loss_fwd_bwd")
 
 
 def aal_accept_reward(problem: AalRewardProblem, draft, target, ref_draft, workspace, tau,

@@ -204,6 +204,36 @@ WindowArgs window_args(const aal_problem* prob, const uint8_t* mask, int cluster
   return wa;
 }
 
+// The window terms of a sequence problem.
+SeqWindowArgs seq_window_args(const aal_seq_problem* prob, const uint8_t* mask, int cluster, float* loss,
+                              float* eal, void* workspace, const SeqLayout& L) {
+  char* base = static_cast<char*>(workspace);
+  SeqWindowArgs wa;
+  wa.mask = mask;
+  wa.B = prob->B;
+  wa.T = prob->seq_len;
+  wa.K = (int32_t)prob->K;
+  wa.full_windows = prob->full_windows != 0;
+  wa.cluster = cluster;
+  wa.greedy = (prob->mode & AAL_GREEDY) != 0;
+  wa.sampling = (prob->mode & AAL_SAMPLING) != 0;
+  wa.kl = (prob->mode & AAL_KL) != 0;
+  wa.tv = (prob->mode & AAL_TV) != 0;
+  wa.w_greedy = prob->w_greedy;
+  wa.w_sampling = prob->w_sampling;
+  wa.w_kl = prob->w_kl;
+  wa.w_tv = prob->w_tv;
+  wa.loss = loss;
+  wa.eal = eal;
+  wa.pg = reinterpret_cast<float*>(base + L.pg);
+  wa.ps = reinterpret_cast<float*>(base + L.ps);
+  wa.ws = loss_ws(workspace, L.base);
+  wa.nwblk = L.base.nwblk;
+  wa.nvalid_g = prob->global_counts == 1 ? (int32_t)prob->n_windows_global : -1;
+  wa.npos_g = prob->global_counts == 1 ? (int32_t)prob->n_positions_global : -1;
+  return wa;
+}
+
 }  // namespace
 
 namespace aal {
@@ -213,7 +243,7 @@ int64_t debug_take_skip_chunk() { return g_skip_chunk.exchange(-1); }
 
 extern "C" {
 
-int32_t aal_abi_version(void) { return 10600; }
+int32_t aal_abi_version(void) { return 10700; }
 
 void aal_debug_fail_next_forward(int64_t chunk, uint64_t wait_limit_ns) {
   g_wait_limit_ns.store(wait_limit_ns);
@@ -405,31 +435,7 @@ aal_status aal_seq_loss_fwd(const aal_seq_problem* prob, const void* draft, cons
   e = launch_stats(draft, target, R, prob->V, prob->dtype, prob->mode, prob->temperature, ws, s, &cluster);
   if (e != cudaSuccess) return AAL_ERR_CUDA;
 
-  char* base = static_cast<char*>(workspace);
-  SeqWindowArgs wa;
-  wa.mask = mask;
-  wa.B = prob->B;
-  wa.T = prob->seq_len;
-  wa.K = (int32_t)prob->K;
-  wa.full_windows = prob->full_windows != 0;
-  wa.cluster = cluster;
-  wa.greedy = (prob->mode & AAL_GREEDY) != 0;
-  wa.sampling = (prob->mode & AAL_SAMPLING) != 0;
-  wa.kl = (prob->mode & AAL_KL) != 0;
-  wa.tv = (prob->mode & AAL_TV) != 0;
-  wa.w_greedy = prob->w_greedy;
-  wa.w_sampling = prob->w_sampling;
-  wa.w_kl = prob->w_kl;
-  wa.w_tv = prob->w_tv;
-  wa.loss = loss;
-  wa.eal = eal;
-  wa.pg = reinterpret_cast<float*>(base + L.pg);
-  wa.ps = reinterpret_cast<float*>(base + L.ps);
-  wa.ws = ws;
-  wa.nwblk = L.base.nwblk;
-  wa.nvalid_g = prob->global_counts == 1 ? (int32_t)prob->n_windows_global : -1;
-  wa.npos_g = prob->global_counts == 1 ? (int32_t)prob->n_positions_global : -1;
-  return cuda_status(launch_seq_window(wa, s));
+  return cuda_status(launch_seq_window(seq_window_args(prob, mask, cluster, loss, eal, workspace, L), s));
 }
 
 aal_status aal_seq_loss_bwd(const aal_seq_problem* prob, const void* draft, const void* target,
@@ -450,6 +456,67 @@ aal_status aal_seq_loss_bwd(const aal_seq_problem* prob, const void* draft, cons
                                  prob->temperature, prob->w_greedy, prob->w_sampling, prob->w_kl, dloss,
                                  loss_ws(const_cast<void*>(workspace), L.base), grad_draft,
                                  static_cast<cudaStream_t>(stream)));
+}
+
+aal_status aal_seq_loss_fwd_bwd(const aal_seq_problem* prob, const void* draft, const void* target,
+                                const uint8_t* mask, void* workspace, size_t workspace_bytes, float dloss,
+                                float* loss, float* eal, void* grad_draft, void* stream) {
+  aal_status st = check_seq(prob);
+  if (st != AAL_OK) return st;
+  if (prob->mode & AAL_GRPO) return AAL_ERR_UNSUPPORTED;  // its coefficients come between the two
+  if (!isfinite(dloss)) return AAL_ERR_INVALID_ARG;
+  if (loss == nullptr || !aligned(loss, 4) || (eal != nullptr && !aligned(eal, 4))) return AAL_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int64_t R = prob->B * prob->seq_len;
+  if (R == 0) return cuda_status(cudaMemsetAsync(loss, 0, sizeof(float), s));
+  if (draft == nullptr || target == nullptr || grad_draft == nullptr || !aligned(draft, 16) ||
+      !aligned(target, target_align(prob->mode)) || !aligned(grad_draft, 16))
+    return AAL_ERR_INVALID_ARG;
+  const SeqLayout L = seq_layout(prob->B, prob->seq_len, prob->K);
+  if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < L.total) return AAL_ERR_WORKSPACE;
+
+  // the fused kernel: bf16 rows of 16-byte multiples, both tensors as logits
+  const bool fusable = prob->dtype == AAL_BF16 && (prob->mode & AAL_IDS) == 0 && (prob->V * 2) % 16 == 0 &&
+                       prob->V * 2 >= g_fused_min_row_bytes.load();
+  if (fusable) {
+    LossWs ws = loss_ws(workspace, L.base);
+    if (cudaMemsetAsync(ws.hdr, 0, sizeof(WsHeader), s) != cudaSuccess) return AAL_ERR_CUDA;
+    if (cudaMemsetAsync(ws.mbox, 0xff, (size_t)R * 8, s) != cudaSuccess) return AAL_ERR_CUDA;  // kMboxEmpty
+    const SeqWindowArgs wa = seq_window_args(prob, mask, 1, loss, eal, workspace, L);
+    if (launch_seq_count_valid(mask, prob->B, prob->seq_len, (int32_t)prob->K, wa.full_windows, wa.nvalid_g,
+                               wa.npos_g, ws.hdr, s) != cudaSuccess)
+      return AAL_ERR_CUDA;
+    FusedArgs f;
+    f.st = stats_args(draft, target, R, prob->V, prob->mode, prob->temperature, ws);
+    f.bw = grad_args(draft, target, mask, R, prob->V, prob->mode, prob->temperature, prob->w_greedy, prob->w_kl,
+                     dloss, ws, grad_draft);
+    // the window flags and weights the exchange reads (win.N and win.mask are not used here)
+    f.win = WindowArgs{};
+    f.win.N = R;
+    f.win.K = (int32_t)prob->K;
+    f.win.greedy = wa.greedy;
+    f.win.sampling = wa.sampling;
+    f.win.kl = wa.kl;
+    f.win.tv = wa.tv;
+    f.win.w_greedy = wa.w_greedy;
+    f.win.w_sampling = wa.w_sampling;
+    f.win.w_kl = wa.w_kl;
+    f.win.w_tv = wa.w_tv;
+    f.groups = 0;
+    f.solos = 0;
+    f.n_group = 0;
+    f.seq_T = prob->seq_len;
+    f.seq_full = wa.full_windows ? 1 : 0;
+    f.seq_mask = mask;
+    const uint64_t limit = debug_wait_limit_ns();
+    bool launched = false;
+    if (launch_fused_seq(f, s, limit ? limit : kWaitLimitNs, &launched) != cudaSuccess) return AAL_ERR_CUDA;
+    // the loss from the statistics the fused kernel wrote, as aal_seq_loss_fwd forms it
+    if (launched) return cuda_status(launch_seq_window(wa, s));
+  }
+  st = aal_seq_loss_fwd(prob, draft, target, mask, workspace, workspace_bytes, loss, eal, stream);
+  if (st != AAL_OK) return st;
+  return aal_seq_loss_bwd(prob, draft, target, mask, workspace, workspace_bytes, dloss, grad_draft, stream);
 }
 
 aal_status aal_grpo_workspace_size(const aal_grpo_problem* prob, size_t* bytes) {

@@ -261,6 +261,11 @@ struct FusedArgs {
   int32_t groups;    // G
   int32_t solos;     // S solo CTAs after the groups' G K, each taking whole windows
   int64_t n_group;   // windows 0 .. n_group - 1 go to the groups, the rest to the solo CTAs
+  // the sequence layout (seq_T > 0): rows are the positions b*T + t of st.R = B*T, a window
+  // starts at every position; win.N and win.mask are unused there, seq_mask is the [B][T] mask
+  int64_t seq_T = 0;
+  int32_t seq_full = 0;  // W = windows with all K positions valid
+  const uint8_t* seq_mask = nullptr;
 };
 
 struct RewardRowArgs {
@@ -365,6 +370,11 @@ struct FusedIdsArgs {
   int32_t groups;    // G
   int32_t solos;     // S solo CTAs after the groups' G K, each taking whole windows
   int64_t n_group;   // windows 0 .. n_group - 1 go to the groups, the rest to the solo CTAs
+  // the sequence layout (seq_T > 0): rows are the positions b*T + t of st.R = B*T, a window
+  // starts at every position; win.N and win.mask are unused there, seq_mask is the [B][T] mask
+  int64_t seq_T = 0;
+  int32_t seq_full = 0;  // W = windows with all K positions valid
+  const uint8_t* seq_mask = nullptr;
 };
 
 // Windows per solo CTA for the fused kernels: G groups finish a window each in one row's time,
@@ -472,6 +482,12 @@ cudaError_t launch_count_valid(const uint8_t* mask, int64_t N, int32_t K, int32_
 cudaError_t launch_fused(const FusedArgs& f, cudaStream_t s, uint64_t limit_ns, bool* launched);
 // The same for token ids (then resolve_draft_argmax places the draft's greedy token).
 cudaError_t launch_fused_ids(const FusedIdsArgs& f, cudaStream_t s, uint64_t limit_ns, bool* launched);
+// The sequence layout's |W| and |positions| from the [B][T] mask, as the sequence window kernel
+// counts them.
+cudaError_t launch_seq_count_valid(const uint8_t* mask, int64_t B, int64_t T, int32_t K, bool full,
+                                   int32_t nvalid_g, int32_t npos_g, WsHeader* hdr, cudaStream_t s);
+// The fused forward + backward over the sequence layout (FusedArgs.seq_T > 0).
+cudaError_t launch_fused_seq(const FusedArgs& f, cudaStream_t s, uint64_t limit_ns, bool* launched);
 
 // ---------------------------------------------------------------------------
 // Device helpers.

@@ -29,6 +29,13 @@
 //   alone needs no window term and so no wait.
 // * The counts of valid windows and positions that scale the gradient are taken from the mask
 //   by count_valid before the launch (the separate forward gets them from its window kernel).
+// * Sequence layout (aal_seq_loss_fwd_bwd, SEQ): rows are positions and a window starts at every
+//   one, so a row's gradient needs the acceptances of the K - 1 positions on each side.  All CTAs
+//   walk the positions from the last one down, CTA c taking rows R-1-c, R-1-c-C, ...: a round of
+//   C consecutive positions is in flight at a time, a row's later neighbours are streamed beside
+//   it or have been, and warp 0 polls the 2K - 1 mailbox words around its row (seq_exchange)
+//   and forms the row's coefficients as the sequence window and gather kernels and the backward
+//   do, so that the result equals aal_seq_loss_fwd + aal_seq_loss_bwd bit for bit.
 // * Failure: every wait is bounded.  A CTA that gave up keeps walking its rows without waiting
 //   and still publishes a word for each, so its group does not wait on it for the whole limit;
 //   the workspace status word reports AAL_ERR_TIMEOUT and the outputs are not to be used.
@@ -57,7 +64,8 @@ constexpr size_t kFusedSmemBytes = (size_t)kSlots * kSlotBytes + sizeof(FusedSme
 
 // PASSES = 2 with the sampling (or TV) term, 1 without; NEED_Q1, KL, P1 as in rowstats_stream;
 // GREEDY and Q1_IS_QT as in the backward.  bf16 rows only (16-byte multiples).
-template <bool NEED_Q1, int PASSES, bool KL, bool GREEDY, bool Q1_IS_QT, bool P1 = false>
+// SEQ: the sequence layout (rows are positions; see fused_seq_rows below).
+template <bool NEED_Q1, int PASSES, bool KL, bool GREEDY, bool Q1_IS_QT, bool P1 = false, bool SEQ = false>
 __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, uint64_t limit_ns) {
   using T = uint16_t;
   constexpr bool SAMPLING = PASSES == 2;
@@ -77,7 +85,11 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
   const int64_t N = f.win.N;
   const int G = f.groups;
   const int64_t NG = f.n_group;        // windows 0 .. NG - 1 go to the groups, the rest to the solo CTAs
-  const bool solo = (int)blockIdx.x >= G * K;
+  const bool solo = !SEQ && (int)blockIdx.x >= G * K;
+  // sequence layout: CTA c takes rows R-1-c, R-1-c-C, ... (C = the grid), so that the rows in
+  // flight at a time are consecutive positions and a row's later neighbours, which its gradient
+  // waits on, are taken in the same round (by CTAs c-1 .. c-K+1) or an earlier one
+  const int C = gridDim.x;
   const int g = blockIdx.x / K, k = blockIdx.x % K;  // (a group's CTA)
   const int so = (int)blockIdx.x - G * K;            // (a solo CTA)
 
@@ -126,7 +138,9 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
           }
         }
       };
-      if (!solo) {
+      if (SEQ) {
+        for (int64_t p = a.R - 1 - blockIdx.x; p >= 0 && !*abort_flag; p -= C) issue(p, 0, PASSES + 1);
+      } else if (!solo) {
         for (int64_t n = g; n < NG && !*abort_flag; n += G) issue(n * K + k, 0, PASSES + 1);
       } else {
         // a whole window: the statistics of its K rows, then their gradients
@@ -396,7 +410,38 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
       }
     };
 
-    if (!solo) {
+    if (SEQ) {
+      // row r's gradient: warp 0 takes the acceptances of rows r - K + 1 .. r + K - 1 (those of
+      // its sequence) and forms the row's coefficients, as the sequence window and gather
+      // kernels and the backward do, then every consumer writes the row
+      const bool need = f.win.greedy || ov;
+      const bool with_greedy = GREEDY && f.bw.w_greedy != 0.f;
+      for (int64_t r = a.R - 1 - blockIdx.x; r >= 0; r -= C) {
+        RowStat st{};
+        float st_as = 0.f;
+        stats_row(r, st, st_as);
+        if (warp == 0) {
+          const int64_t lo = r - r % f.seq_T, hi = lo + f.seq_T - 1;
+          float dEg = 0.f, dEs = 0.f;
+          RowCoef c;
+          const bool ok = seq_exchange(a.ws.mbox, f.seq_mask, r, lo, hi, K, f.seq_full != 0, f.win.greedy,
+                                       f.win.sampling, f.win.tv, f.win.w_sampling, f.win.w_tv, need, lane,
+                                       abort_flag, hdr, limit_ns, &dEg, &dEs,
+                                       [&]() { row_coef_local<GREEDY, SAMPLING, KL>(f.bw, st, c); });
+          if (lane == 0) {
+            const bool pos_valid = f.bw.mask == nullptr || f.bw.mask[r] != 0;
+            F.live = ok && row_coef<GREEDY, SAMPLING, KL, true>(f.bw, scale, kscale, with_greedy ? dEg : 0.f,
+                                                                SAMPLING ? dEs : 0.f, 0.f, pos_valid, st, c)
+                         ? 1
+                         : 0;
+            if (F.live) F.coef = c;
+          }
+        }
+        named_barrier(kBarCoef, kConsumers);
+        const RowCoef c = F.coef;
+        grad_row(r, c, F.live);
+      }
+    } else if (!solo) {
       // one row of each of the group's windows: statistics, the window exchange, the gradient
       for (int64_t n = g; n < NG; n += G) {
         const int64_t r = n * K + k;
@@ -496,6 +541,67 @@ __global__ void __launch_bounds__(1024) count_valid(const uint8_t* mask, int64_t
   }
 }
 
+// The sequence layout's counts, as the sequence window kernel takes them: window n is in W when
+// its leading valid run K_n (stopping at the sequence's end or its first invalid position) is
+// >= 1, or = K with full windows; positions count when valid.
+__global__ void __launch_bounds__(1024) seq_count_valid(const uint8_t* mask, int64_t B, int64_t T, int32_t K,
+                                                        bool full, int32_t nvalid_g, int32_t npos_g, WsHeader* hdr) {
+  __shared__ unsigned long long sw, sp;
+  if (threadIdx.x == 0) {
+    sw = 0ull;
+    sp = 0ull;
+  }
+  __syncthreads();
+  unsigned long long w = 0, p = 0;
+  for (int64_t n = threadIdx.x; n < B * T; n += blockDim.x) {
+    const int64_t t = n % T;
+    int kn = 0;
+    while (kn < K && t + kn < T && (mask == nullptr || mask[n + kn] != 0)) ++kn;
+    if (full && kn < K) kn = 0;
+    w += kn >= 1;
+    p += mask == nullptr || mask[n] != 0;
+  }
+  atomicAdd(&sw, w);
+  atomicAdd(&sp, p);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    hdr->nvalid = nvalid_g >= 0 ? nvalid_g : (int32_t)sw;
+    hdr->npos = npos_g >= 0 ? npos_g : (int32_t)sp;
+  }
+}
+
+// The sequence layout: CTA c of C (one cooperative CTA per SM) takes rows R-1-c, R-1-c-C, ...:
+// the C rows in flight at a time are consecutive positions, and a row's gradient waits only on
+// rows after it, which are taken in the same round by the CTAs before it or in an earlier round.
+// Every wait so points to work that starts no later, and the launch cannot deadlock while all
+// its CTAs are resident (a cooperative launch).
+template <bool NQ1, int P, bool KL, bool GR, bool Q, bool P1 = false>
+cudaError_t go_fused_seq(const FusedArgs& f0, cudaStream_t s, uint64_t limit_ns, bool* launched) {
+  auto kern = fused_rows<NQ1, P, KL, GR, Q, P1, true>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFusedSmemBytes);
+  if (e != cudaSuccess) return e;
+  int dev = 0, sms = 0, per_sm = 0, coop = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev);
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, kFusedSmemBytes);
+  if (e != cudaSuccess) return e;
+  int64_t C = (int64_t)sms * per_sm;
+  if (C > f0.st.R) C = f0.st.R;
+  if (!coop || C < 1) return cudaSuccess;  // *launched stays false: the caller runs the two calls
+  const int elt = 2;
+  const int nch = (int)((f0.st.V + kHalfSlot / elt - 1) / (kHalfSlot / elt));
+  FusedArgs f = f0;
+  void* args[] = {&f, (void*)&nch, &limit_ns};
+  e = cudaLaunchCooperativeKernel((const void*)kern, dim3((unsigned)C), dim3(kThreads), args, kFusedSmemBytes, s);
+  if (e == cudaErrorCooperativeLaunchTooLarge) {
+    cudaGetLastError();
+    return cudaSuccess;
+  }
+  if (e == cudaSuccess) *launched = true;
+  return e;
+}
+
 template <bool NQ1, int P, bool KL, bool GR, bool Q, bool P1 = false>
 cudaError_t go_fused(const FusedArgs& f0, cudaStream_t s, uint64_t limit_ns, bool* launched) {
   auto kern = fused_rows<NQ1, P, KL, GR, Q, P1>;
@@ -540,32 +646,58 @@ cudaError_t launch_count_valid(const uint8_t* mask, int64_t N, int32_t K, int32_
   return cudaGetLastError();
 }
 
+cudaError_t launch_seq_count_valid(const uint8_t* mask, int64_t B, int64_t T, int32_t K, bool full,
+                                   int32_t nvalid_g, int32_t npos_g, WsHeader* hdr, cudaStream_t s) {
+  seq_count_valid<<<1, 1024, 0, s>>>(mask, B, T, K, full, nvalid_g, npos_g, hdr);
+  return cudaGetLastError();
+}
+
+namespace {
+template <bool SEQ, bool NQ1, int P, bool KL, bool GR, bool Q, bool P1 = false>
+cudaError_t go(const FusedArgs& f, cudaStream_t s, uint64_t limit_ns, bool* launched) {
+  if constexpr (SEQ)
+    return go_fused_seq<NQ1, P, KL, GR, Q, P1>(f, s, limit_ns, launched);
+  else
+    return go_fused<NQ1, P, KL, GR, Q, P1>(f, s, limit_ns, launched);
+}
+
 // The instantiation for the problem's flags, or none (launched = false) for a combination
 // this path does not take.
-cudaError_t launch_fused(const FusedArgs& f, cudaStream_t s, uint64_t limit_ns, bool* launched) {
+template <bool SEQ>
+cudaError_t dispatch_fused(const FusedArgs& f, cudaStream_t s, uint64_t limit_ns, bool* launched) {
   *launched = false;
   const bool two = f.st.overlap, kl = f.st.need_kl, nq1 = f.st.need_q1 && two;
   const bool greedy = f.bw.w_greedy != 0.f && !f.bw.grpo;
   const bool q = f.bw.q1_is_qT && two && (greedy || kl);
   if (!two) {
-    if (greedy && !kl) return go_fused<false, 1, false, true, false>(f, s, limit_ns, launched);
-    if (!greedy && kl) return go_fused<false, 1, true, false, false>(f, s, limit_ns, launched);
-    if (greedy && kl) return go_fused<false, 1, true, true, false>(f, s, limit_ns, launched);
+    if (greedy && !kl) return go<SEQ, false, 1, false, true, false>(f, s, limit_ns, launched);
+    if (!greedy && kl) return go<SEQ, false, 1, true, false, false>(f, s, limit_ns, launched);
+    if (greedy && kl) return go<SEQ, false, 1, true, true, false>(f, s, limit_ns, launched);
     return cudaSuccess;
   }
   if (kl) {  // at T = 1 q = q~ (one z_q state); else z_q and z_p both kept at T = 1 beside T
     if (q && !nq1)
-      return greedy ? go_fused<false, 2, true, true, true>(f, s, limit_ns, launched)
-                    : go_fused<false, 2, true, false, true>(f, s, limit_ns, launched);
+      return greedy ? go<SEQ, false, 2, true, true, true>(f, s, limit_ns, launched)
+                    : go<SEQ, false, 2, true, false, true>(f, s, limit_ns, launched);
     if (nq1 && !q)
-      return greedy ? go_fused<true, 2, true, true, false, true>(f, s, limit_ns, launched)
-                    : go_fused<true, 2, true, false, false, true>(f, s, limit_ns, launched);
+      return greedy ? go<SEQ, true, 2, true, true, false, true>(f, s, limit_ns, launched)
+                    : go<SEQ, true, 2, true, false, false, true>(f, s, limit_ns, launched);
     return cudaSuccess;
   }
-  if (!greedy && !nq1 && !q) return go_fused<false, 2, false, false, false>(f, s, limit_ns, launched);
-  if (greedy && !nq1 && q) return go_fused<false, 2, false, true, true>(f, s, limit_ns, launched);
-  if (greedy && nq1 && !q) return go_fused<true, 2, false, true, false>(f, s, limit_ns, launched);
+  if (!greedy && !nq1 && !q) return go<SEQ, false, 2, false, false, false>(f, s, limit_ns, launched);
+  if (greedy && !nq1 && q) return go<SEQ, false, 2, false, true, true>(f, s, limit_ns, launched);
+  if (greedy && nq1 && !q) return go<SEQ, true, 2, false, true, false>(f, s, limit_ns, launched);
   return cudaSuccess;
+}
+
+}  // namespace
+
+cudaError_t launch_fused(const FusedArgs& f, cudaStream_t s, uint64_t limit_ns, bool* launched) {
+  return dispatch_fused<false>(f, s, limit_ns, launched);
+}
+
+cudaError_t launch_fused_seq(const FusedArgs& f, cudaStream_t s, uint64_t limit_ns, bool* launched) {
+  return dispatch_fused<true>(f, s, limit_ns, launched);
 }
 
 }  // namespace aal

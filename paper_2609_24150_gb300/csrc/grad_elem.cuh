@@ -308,4 +308,99 @@ __device__ __forceinline__ bool window_exchange(uint64_t* mbox, int64_t r, int64
   return ok;
 }
 
+
+// dE/da_j of a window whose depth-i acceptance is held by lane (base + i) of the warp (each lane
+// names its own window and depth): the bits of window_term's dE[j], with the same roundings in
+// the same order, 0 for j >= kn; every lane of the warp must call it.
+__device__ __forceinline__ float window_partial(float a_l, int base, int j, int kn) {
+  float P = 1.f, S = 1.f;
+#pragma unroll
+  for (int i = 0; i < AAL_MAX_K; ++i) {  // P_j = a_0 ... a_{j-1}
+    const float v = __shfl_sync(0xffffffffu, a_l, (base + i) & 31);
+    if (i < j && i < kn) P = __fmul_rn(P, v);
+  }
+#pragma unroll
+  for (int i = AAL_MAX_K - 1; i >= 0; --i) {  // S_j = 1 + a_{j+1} (1 + a_{j+2} (...)) from the top
+    const float v = __shfl_sync(0xffffffffu, a_l, (base + i) & 31);
+    if (i > j && i < kn) S = __fmaf_rn(v, S, 1.f);
+  }
+  return j < kn ? __fmul_rn(P, S) : 0.f;
+}
+
+// The exchange of the fused sequence layout, run by one whole warp for row p (position p - lo of
+// the sequence whose rows are lo .. hi; every row's word is published with its statistics).
+// Lane l < 2K - 1 polls the word of row p - (K - 1) + l when that row is in the sequence,
+// bounded like window_exchange.  Lane j < K then forms the window that starts at row p - j (when
+// it starts inside the sequence) as the sequence window kernel does: its K_n leading valid
+// positions (stopping at the sequence's end or its first invalid position; 0 when full_windows
+// and K_n < K), dE/da by window_term, and the depth-j partials (greedy; sampling with w_s and
+// the TV term folded in).  Lane 0 adds them in increasing j, as the gather does, into dEg and
+// dEs.  Returns, to every lane, whether the words arrived.
+template <typename Pre = NoPrePoll>
+__device__ __forceinline__ bool seq_exchange(const uint64_t* mbox, const uint8_t* mask, int64_t p, int64_t lo,
+                                             int64_t hi, int K, bool full, bool greedy, bool sampling, bool tv,
+                                             float w_sampling, float w_tv, bool need, int lane,
+                                             volatile int* abort_flag, WsHeader* hdr, uint64_t limit_ns,
+                                             float* dEg, float* dEs, Pre pre = Pre()) {
+  bool ok = __shfl_sync(0xffffffffu, *abort_flag == 0 ? 1 : 0, 0) != 0;
+  // rows p - back .. p + fwd are the sequence's within K - 1 of p; lane l holds row p + l - (K - 1)
+  const int back = (int)min(p - lo, (int64_t)(K - 1)), fwd = (int)min(hi - p, (int64_t)(K - 1));
+  const int o = lane - (K - 1);
+  const bool mine = lane < 2 * K - 1 && o >= -back && o <= fwd;
+  const uint64_t* mrow = mbox + p;
+  uint64_t w = 0;
+  if (lane == 0 && !(ok && need)) pre();
+  if (ok && need) {
+    const uint64_t t0 = ptx::now_ns();
+    for (uint32_t it = 0;; ++it) {
+      if (mine) w = ptx::ld_relaxed(mrow + o);
+      if (it == 0 && lane == 0) pre();
+      if (__all_sync(0xffffffffu, !mine || w != kMboxEmpty)) break;
+      int quit = 0;
+      if (lane == 0 && (*abort_flag || it >= kSpinLimit || ptx::now_ns() - t0 > limit_ns)) {
+        if (!*abort_flag) {
+          *abort_flag = 1;
+          atomicExch(&hdr->status, kStatusTimeout);
+        }
+        quit = 1;
+      }
+      if (__shfl_sync(0xffffffffu, quit, 0)) {
+        ok = false;
+        break;
+      }
+      __nanosleep(64);
+    }
+  }
+  const float ag_l = __uint_as_float((uint32_t)w), as_l = __uint_as_float((uint32_t)(w >> 32));
+  // lane j: the window starting at row p - j, K_n positions long
+  int kn = 0;
+  if (need && lane < K && lane <= back) {
+    const uint8_t* mrow8 = mask != nullptr ? mask + (p - lane) : nullptr;
+    while (kn < K && kn - lane <= fwd && (mrow8 == nullptr || mrow8[kn] != 0)) ++kn;
+    if (full && kn < K) kn = 0;
+  }
+  // row p - j + i was polled by lane (K - 1) - j + i
+  const int base = (K - 1) - lane;
+  float pg = 0.f, ps = 0.f;
+  if (greedy) pg = window_partial(ag_l, base, lane, kn);
+  if (sampling || tv) {
+    const float d = sampling ? window_partial(as_l, base, lane, kn) : 0.f;
+    const float tvc = (tv && kn > 0) ? w_tv / (float)kn : 0.f;
+    ps = __fadd_rn(sampling ? __fmul_rn(w_sampling, d) : 0.f, lane < kn ? tvc : 0.f);
+  }
+  float g = 0.f, s = 0.f;
+#pragma unroll
+  for (int j = 0; j < AAL_MAX_K; ++j) {
+    const float pgj = __shfl_sync(0xffffffffu, pg, j);
+    const float psj = __shfl_sync(0xffffffffu, ps, j);
+    if (j < K && j <= back) {
+      if (greedy) g += pgj;
+      if (sampling || tv) s += psj;
+    }
+  }
+  *dEg = g;
+  *dEs = s;
+  return ok;
+}
+
 }  // namespace aal

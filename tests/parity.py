@@ -162,10 +162,11 @@ def loss_from_eal(run: LossRun, mode, wg, ws, nvalid):
 # -------------------------------------------------------------------------- sequence layout
 
 class SeqRun:
-    """Forward + backward of one sequence-layout problem through the C ABI."""
+    """Forward + backward of one sequence-layout problem through the C ABI (two calls, or the
+    one-call aal_seq_loss_fwd_bwd with ``fused``)."""
 
     def __init__(self, target, draft, mask, K, mode, T=1.0, wg=1.0, ws=1.0, dloss=1.0, full_windows=False,
-                 wkl=1.0, wtv=1.0):
+                 wkl=1.0, wtv=1.0, fused=False):
         self.prob = aal.seq_problem(draft, K, mode, T, wg, ws, full_windows, wkl, wtv)
         self.ws_buf = torch.empty(aal.aal_seq_workspace_size(self.prob), dtype=torch.uint8,
                                   device=draft.device)
@@ -173,9 +174,13 @@ class SeqRun:
         self.loss = torch.full((1,), float("nan"), dtype=torch.float32, device=draft.device)
         self.eal = torch.full((max(R, 1), 2), float("nan"), dtype=torch.float32, device=draft.device)
         self.grad = torch.full_like(draft, float("nan"))
-        aal.aal_seq_loss_fwd(self.prob, draft, target, mask, self.ws_buf, self.loss,
-                             self.eal if R > 0 else None)
-        aal.aal_seq_loss_bwd(self.prob, draft, target, mask, self.ws_buf, dloss, self.grad)
+        if fused:   # aal_seq_loss_fwd_bwd: one call
+            aal.aal_seq_loss_fwd_bwd(self.prob, draft, target, mask, self.ws_buf, dloss, self.loss, self.grad,
+                                     self.eal if R > 0 else None)
+        else:
+            aal.aal_seq_loss_fwd(self.prob, draft, target, mask, self.ws_buf, self.loss,
+                                 self.eal if R > 0 else None)
+            aal.aal_seq_loss_bwd(self.prob, draft, target, mask, self.ws_buf, dloss, self.grad)
         torch.cuda.synchronize()
         assert aal.aal_check_device_status(self.ws_buf) == aal.AAL_OK
 

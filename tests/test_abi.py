@@ -25,7 +25,8 @@ def _declared():
 
 def test_header_declares_the_entry_points():
     names = _declared()
-    assert {"aal_loss_fwd", "aal_loss_bwd", "aal_loss_fwd_bwd", "aal_accept_reward", "aal_workspace_size",
+    assert {"aal_loss_fwd", "aal_loss_bwd", "aal_loss_fwd_bwd", "aal_seq_loss_fwd", "aal_seq_loss_bwd",
+            "aal_seq_loss_fwd_bwd", "aal_accept_reward", "aal_workspace_size",
             "aal_reward_workspace_size", "aal_check_device_status", "aal_status_string",
             "aal_abi_version"} <= names
 
@@ -41,7 +42,7 @@ def test_library_exports_every_declared_symbol():
 
 
 def test_status_strings_and_version():
-    assert aal.aal_abi_version() == 10600
+    assert aal.aal_abi_version() == 10700
     for code in range(6):
         assert aal.aal_status_string(code).startswith("AAL_")
     assert aal.aal_status_string(99) == "unknown aal_status"
@@ -252,6 +253,14 @@ def test_seq_pointer_checks_before_launch():
     assert lib.aal_seq_loss_bwd(ctypes.byref(p), fake, fake, None, fake_ws, size, 1.0, None, None) == aal.AAL_ERR_INVALID_ARG
     assert lib.aal_seq_loss_bwd(ctypes.byref(p), fake, fake, None, fake_ws, size, float("inf"), fake, None) == aal.AAL_ERR_INVALID_ARG
     assert lib.aal_seq_loss_bwd(ctypes.byref(p), fake, fake, None, fake_ws + 128, size, 1.0, fake, None) == aal.AAL_ERR_WORKSPACE
+    fb = lib.aal_seq_loss_fwd_bwd
+    assert fb(ctypes.byref(p), fake, fake, None, fake_ws, size, 1.0, fake, None, None, None) == aal.AAL_ERR_INVALID_ARG
+    assert fb(ctypes.byref(p), fake, fake, None, fake_ws, size, 1.0, None, None, fake, None) == aal.AAL_ERR_INVALID_ARG
+    assert fb(ctypes.byref(p), fake, fake + 8, None, fake_ws, size, 1.0, fake, None, fake, None) == aal.AAL_ERR_INVALID_ARG
+    assert fb(ctypes.byref(p), fake, fake, None, fake_ws, size, float("nan"), fake, None, fake, None) == aal.AAL_ERR_INVALID_ARG
+    assert fb(ctypes.byref(p), fake, fake, None, fake_ws, size - 1, 1.0, fake, None, fake, None) == aal.AAL_ERR_WORKSPACE
+    g = _sprob(mode=aal.AAL_GREEDY | aal.AAL_GRPO)
+    assert fb(ctypes.byref(g), fake, fake, None, fake_ws, _seq_ws(g)[1], 1.0, fake, None, fake, None) == aal.AAL_ERR_UNSUPPORTED
 
 
 def _gprob(**kw):
