@@ -62,6 +62,8 @@ def parse():
                          "configs, rewardstream)")
     ap.add_argument("--windows", type=int, default=None,
                     help="run the first WINDOWS windows of the workload (profiling captures)")
+    ap.add_argument("--seq-len", type=int, default=None,
+                    help="positions per sequence of the sequence-layout line (profiling captures)")
     return ap.parse_args()
 
 
@@ -263,7 +265,7 @@ def run_ours(args, ws_count, rank, local):
     reps = max(5, args.steps // 2)
     greedy_obj = run_greedy_objective(aal, draft, target, grad, stream, reps) if "greedy" in lines else None
     greedy_ids = run_greedy_ids(aal, draft, target, grad, stream, reps) if "ids" in lines else None
-    seq = run_sequence_layout(aal, dev, stream, rank, reps) if "seq" in lines else None
+    seq = run_sequence_layout(aal, dev, stream, rank, reps, args.seq_len) if "seq" in lines else None
     grpo = run_grpo_phase(aal, dev, stream, rank, reps) if "grpo" in lines else None
     seq_grpo = run_seq_grpo_phase(aal, dev, stream, rank, reps) if "seqgrpo" in lines else None
     peak, peak_src = measured_peak()
@@ -550,12 +552,12 @@ def run_seq_grpo_phase(aal, dev, stream, rank, reps):
     return out
 
 
-def run_sequence_layout(aal, dev, stream, rank, reps):
+def run_sequence_layout(aal, dev, stream, rank, reps, seq_len=None):
     """The same loss over the sequence layout (Sec. 3.3): 4 sequences x 2048 positions, a window
     of K=7 starting at every position, logits stored once per position; the one-call forward +
     backward (aal_seq_loss_fwd_bwd) and the two calls, timed with events on the launching stream.
     Unmasked, so every row is read (and written) once."""
-    target, draft, _ = synth.make_seq_logits("seq_v128k", seed=rank, device=dev, masked=False)
+    target, draft, _ = synth.make_seq_logits("seq_v128k", seed=rank, device=dev, masked=False, seq_len=seq_len)
     B, T, V = draft.shape
     K = synth.SEQUENCES["seq_v128k"].K
     grad = torch.empty_like(draft)

@@ -511,7 +511,8 @@ aal_status aal_seq_loss_fwd_bwd(const aal_seq_problem* prob, const void* draft, 
     const uint64_t limit = debug_wait_limit_ns();
     bool launched = false;
     if (launch_fused_seq(f, s, limit ? limit : kWaitLimitNs, &launched) != cudaSuccess) return AAL_ERR_CUDA;
-    // the loss from the statistics the fused kernel wrote, as aal_seq_loss_fwd forms it
+    // the loss from the statistics the fused kernel wrote, and each position's dE/da, as
+    // aal_seq_loss_fwd forms them (the workspace then serves aal_seq_loss_bwd as well)
     if (launched) return cuda_status(launch_seq_window(wa, s));
   }
   st = aal_seq_loss_fwd(prob, draft, target, mask, workspace, workspace_bytes, loss, eal, stream);

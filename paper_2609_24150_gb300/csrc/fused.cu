@@ -543,30 +543,44 @@ __global__ void __launch_bounds__(1024) count_valid(const uint8_t* mask, int64_t
 
 // The sequence layout's counts, as the sequence window kernel takes them: window n is in W when
 // its leading valid run K_n (stopping at the sequence's end or its first invalid position) is
-// >= 1, or = K with full windows; positions count when valid.
+// >= 1, i.e. when position n is valid, or = K with full windows; positions count when valid.
+// Without a mask these are closed forms, and data-parallel counts given by the caller
+// (nvalid_g, npos_g >= 0) replace them; otherwise integer sums over the grid, added into the
+// header (zeroed by the caller), so the order does not matter.
 __global__ void __launch_bounds__(1024) seq_count_valid(const uint8_t* mask, int64_t B, int64_t T, int32_t K,
                                                         bool full, int32_t nvalid_g, int32_t npos_g, WsHeader* hdr) {
-  __shared__ unsigned long long sw, sp;
+  if (mask == nullptr || nvalid_g >= 0) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+      const int64_t per_seq = full ? (T >= K ? T - K + 1 : 0) : T;
+      hdr->nvalid = nvalid_g >= 0 ? nvalid_g : (int32_t)(B * per_seq);
+      hdr->npos = npos_g >= 0 ? npos_g : (int32_t)(B * T);
+    }
+    return;
+  }
+  __shared__ unsigned int sw, sp;
   if (threadIdx.x == 0) {
-    sw = 0ull;
-    sp = 0ull;
+    sw = 0u;
+    sp = 0u;
   }
   __syncthreads();
-  unsigned long long w = 0, p = 0;
-  for (int64_t n = threadIdx.x; n < B * T; n += blockDim.x) {
-    const int64_t t = n % T;
-    int kn = 0;
-    while (kn < K && t + kn < T && (mask == nullptr || mask[n + kn] != 0)) ++kn;
-    if (full && kn < K) kn = 0;
-    w += kn >= 1;
-    p += mask == nullptr || mask[n] != 0;
+  unsigned int w = 0, p = 0;
+  for (int64_t n = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; n < B * T; n += (int64_t)gridDim.x * blockDim.x) {
+    if (mask[n] == 0) continue;
+    ++p;
+    if (!full) {
+      ++w;
+    } else if (n % T + K <= T) {
+      int kk = 1;
+      while (kk < K && mask[n + kk] != 0) ++kk;
+      w += kk == K;
+    }
   }
   atomicAdd(&sw, w);
   atomicAdd(&sp, p);
   __syncthreads();
   if (threadIdx.x == 0) {
-    hdr->nvalid = nvalid_g >= 0 ? nvalid_g : (int32_t)sw;
-    hdr->npos = npos_g >= 0 ? npos_g : (int32_t)sp;
+    atomicAdd(reinterpret_cast<unsigned int*>(&hdr->nvalid), sw);
+    atomicAdd(reinterpret_cast<unsigned int*>(&hdr->npos), sp);
   }
 }
 
@@ -648,7 +662,13 @@ cudaError_t launch_count_valid(const uint8_t* mask, int64_t N, int32_t K, int32_
 
 cudaError_t launch_seq_count_valid(const uint8_t* mask, int64_t B, int64_t T, int32_t K, bool full,
                                    int32_t nvalid_g, int32_t npos_g, WsHeader* hdr, cudaStream_t s) {
-  seq_count_valid<<<1, 1024, 0, s>>>(mask, B, T, K, full, nvalid_g, npos_g, hdr);
+  int64_t blocks = 1;
+  if (mask != nullptr && nvalid_g < 0) {
+    blocks = (B * T + 1023) / 1024;
+    if (blocks > 152) blocks = 152;
+    if (blocks < 1) blocks = 1;
+  }
+  seq_count_valid<<<(unsigned)blocks, 1024, 0, s>>>(mask, B, T, K, full, nvalid_g, npos_g, hdr);
   return cudaGetLastError();
 }
 

@@ -97,6 +97,17 @@ def test_seq_fused_equals_two_calls(Bn, Tn, K, V, mode, T, wg, ws, wkl, wtv, mas
     assert_same(f, s)
 
 
+def test_seq_fused_workspace_serves_the_backward():
+    """The workspace after the one call is the forward's: aal_seq_loss_bwd with another dloss gives
+    the two calls' gradient for that dloss."""
+    t, d, m = _inputs(2, 200, 2000, seed=41, masked=True)
+    f = SeqRun(t, d, m, 7, B, 1.0, 0.5, 0.5, 1.0, fused=True)
+    g = torch.full_like(d, float("nan"))
+    aal.aal_seq_loss_bwd(f.prob, d, t, m, f.ws_buf, 3.0, g)
+    s = SeqRun(t, d, m, 7, B, 1.0, 0.5, 0.5, 3.0)
+    assert torch.equal(_bits(g), _bits(s.grad))
+
+
 def test_seq_fused_no_valid_window():
     t, d, _ = _inputs(2, 40, 4096, seed=5)
     m = torch.zeros((2, 40), dtype=torch.uint8, device=DEV)
