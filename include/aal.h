@@ -27,10 +27,10 @@
  *   Streams.  `stream` is a cudaStream_t (NULL = legacy default stream).  All
  *     calls are asynchronous on it; outputs are valid once the stream reaches
  *     the call.  Calls that share a workspace must be ordered on one stream.
- *     aal_loss_fwd, aal_loss_bwd, aal_loss_fwd_bwd (a cooperative launch among them) and
- *     aal_accept_reward_from_loss enqueue only kernels and asynchronous memsets on
- *     `stream`, so a step made of them can be captured in a CUDA graph and replayed; each
- *     replay gives the same bits as eager calls.
+ *     aal_loss_fwd, aal_loss_bwd, aal_loss_fwd_bwd, aal_seq_loss_fwd_bwd (cooperative
+ *     launches among them) and aal_accept_reward_from_loss enqueue only kernels and
+ *     asynchronous memsets on `stream`, so a step made of them can be captured in a CUDA
+ *     graph and replayed; each replay gives the same bits as eager calls.
  *   Errors.  Arguments are checked before anything is launched; a failed check
  *     returns AAL_ERR_INVALID_ARG / AAL_ERR_UNSUPPORTED / AAL_ERR_WORKSPACE and
  *     launches nothing.  A launch failure returns AAL_ERR_CUDA.  Device-side

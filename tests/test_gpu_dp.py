@@ -80,9 +80,22 @@ def test_windows_sharded_over_ranks(mode, T, wg, ws, fused, dtype, V):
     assert abs(sum(losses) - whole[0]) <= 1e-6 * abs(whole[0]) + 1e-7, (sum(losses), whole[0])
 
 
-def test_sequences_sharded_over_ranks():
-    """The sequence layout sharded by whole sequences (L_KL + 0.1 L_EAL and EAL + WTV)."""
-    target, draft, mask = synth.make_seq_logits("seq_tiny", seed=13)
+def _seq_fwd_bwd(p, d, t, m, w, loss, grad, dloss, fused):
+    if fused:
+        aal.aal_seq_loss_fwd_bwd(p, d, t, m, w, dloss, loss, grad)
+    else:
+        aal.aal_seq_loss_fwd(p, d, t, m, w, loss)
+        aal.aal_seq_loss_bwd(p, d, t, m, w, dloss, grad)
+
+
+@pytest.mark.parametrize("fused", [False, True])
+def test_sequences_sharded_over_ranks(fused):
+    """The sequence layout sharded by whole sequences (L_KL + 0.1 L_EAL and EAL + WTV), as two calls
+    (fp32 rows) and as the one-call form (bf16 rows, the fused kernel)."""
+    if fused:
+        target, draft, mask = synth.make_seq_logits("seq_tiny", seed=13, V=4104, dtype=torch.bfloat16)
+    else:
+        target, draft, mask = synth.make_seq_logits("seq_tiny", seed=13)
     t, d, m = target.to(DEV), draft.to(DEV), mask.to(DEV)
     Bn, Tn, V = d.shape
     K = 4
@@ -91,8 +104,7 @@ def test_sequences_sharded_over_ranks():
         wsb = torch.empty(aal.aal_seq_workspace_size(prob), dtype=torch.uint8, device=DEV)
         loss = torch.empty(1, device=DEV)
         grad = torch.empty_like(d)
-        aal.aal_seq_loss_fwd(prob, d, t, m, wsb, loss)
-        aal.aal_seq_loss_bwd(prob, d, t, m, wsb, 3.0, grad)
+        _seq_fwd_bwd(prob, d, t, m, wsb, loss, grad, 3.0, fused)
         torch.cuda.synchronize()
         nW = nP = int((m != 0).sum().item())       # every valid position starts a window in W
         parts, total = [], 0.0
@@ -102,8 +114,8 @@ def test_sequences_sharded_over_ranks():
             w2 = torch.empty(aal.aal_seq_workspace_size(p), dtype=torch.uint8, device=DEV)
             l2 = torch.empty(1, device=DEV)
             g2 = torch.empty_like(d[lo:hi])
-            aal.aal_seq_loss_fwd(p, d[lo:hi].contiguous(), t[lo:hi].contiguous(), m[lo:hi].contiguous(), w2, l2)
-            aal.aal_seq_loss_bwd(p, d[lo:hi].contiguous(), t[lo:hi].contiguous(), m[lo:hi].contiguous(), w2, 3.0, g2)
+            _seq_fwd_bwd(p, d[lo:hi].contiguous(), t[lo:hi].contiguous(), m[lo:hi].contiguous(), w2, l2, g2, 3.0,
+                         fused)
             torch.cuda.synchronize()
             assert aal.aal_check_device_status(w2) == aal.AAL_OK
             parts.append(g2)

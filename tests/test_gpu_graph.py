@@ -110,3 +110,43 @@ def test_fused_step_replays_bit_exactly(mode, T):
         assert aal.aal_check_device_status(ws) == aal.AAL_OK
         for a, b in zip((loss, eal, grad, tau, adv), ref):
             assert torch.equal(a, b)
+
+
+@pytest.mark.parametrize("masked", [False, True])
+def test_fused_sequence_step_replays_bit_exactly(masked):
+    """aal_seq_loss_fwd_bwd (async memsets, the count kernel, the cooperative fused launch, the
+    sequence window and gather kernels) captured once: replays equal eager calls bit for bit."""
+    target, draft, mask = synth.make_seq_logits("seq_tiny", seed=8, B=3, seq_len=120, V=4104,
+                                                dtype=torch.bfloat16, masked=masked)
+    t, d = target.to(DEV), draft.to(DEV)
+    m = None if mask is None else mask.to(DEV)
+    R = d.shape[0] * d.shape[1]
+    prob = aal.seq_problem(d, 6, aal.AAL_BOTH, 1.0, 0.4, 0.6)
+    ws = torch.empty(aal.aal_seq_workspace_size(prob), dtype=torch.uint8, device=DEV)
+    loss = torch.empty(1, device=DEV)
+    eal = torch.empty(R, 2, device=DEV)
+    grad = torch.empty_like(d)
+
+    def step():
+        aal.aal_seq_loss_fwd_bwd(prob, d, t, m, ws, 2.0, loss, grad, eal)
+
+    step()
+    torch.cuda.synchronize()
+    ref = [x.clone() for x in (loss, eal, grad)]
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        step()
+    torch.cuda.current_stream().wait_stream(s)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        step()
+    for x in (loss, eal, grad):
+        x.fill_(float("nan"))
+    for _ in range(2):
+        g.replay()
+        torch.cuda.synchronize()
+        assert aal.aal_check_device_status(ws) == aal.AAL_OK
+        for a, b in zip((loss, eal, grad), ref):
+            assert torch.equal(a, b)
