@@ -475,9 +475,13 @@ aal_status aal_seq_loss_fwd_bwd(const aal_seq_problem* prob, const void* draft, 
   const SeqLayout L = seq_layout(prob->B, prob->seq_len, prob->K);
   if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < L.total) return AAL_ERR_WORKSPACE;
 
-  // the fused kernel: bf16 rows of 16-byte multiples, both tensors as logits
+  // the fused kernel: bf16 rows of 16-byte multiples, both tensors as logits, and a round of
+  // rows (one per SM) that spans a window or holds every row (its order is deadlock-free then)
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return AAL_ERR_CUDA;
   const bool fusable = prob->dtype == AAL_BF16 && (prob->mode & AAL_IDS) == 0 && (prob->V * 2) % 16 == 0 &&
-                       prob->V * 2 >= g_fused_min_row_bytes.load();
+                       prob->V * 2 >= g_fused_min_row_bytes.load() && (sms >= prob->K || R <= sms);
   if (fusable) {
     LossWs ws = loss_ws(workspace, L.base);
     if (cudaMemsetAsync(ws.hdr, 0, sizeof(WsHeader), s) != cudaSuccess) return AAL_ERR_CUDA;

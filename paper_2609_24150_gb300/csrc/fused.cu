@@ -32,10 +32,11 @@
 // * Sequence layout (aal_seq_loss_fwd_bwd, SEQ): rows are positions and a window starts at every
 //   one, so a row's gradient needs the acceptances of the K - 1 positions on each side.  All CTAs
 //   walk the positions from the last one down, CTA c taking rows R-1-c, R-1-c-C, ...: a round of
-//   C consecutive positions is in flight at a time, a row's later neighbours are streamed beside
-//   it or have been, and warp 0 polls the 2K - 1 mailbox words around its row (seq_exchange)
-//   and forms the row's coefficients as the sequence window and gather kernels and the backward
-//   do, so that the result equals aal_seq_loss_fwd + aal_seq_loss_bwd bit for bit.
+//   C consecutive positions is in flight at a time, so a row's neighbours are streamed beside it
+//   (those of the last K - 1 CTAs' rows below them come with the next round), and warp 0 polls
+//   the 2K - 1 mailbox words around its row (seq_exchange) and forms the row's coefficients as
+//   the sequence window and gather kernels and the backward do, so that the result equals
+//   aal_seq_loss_fwd + aal_seq_loss_bwd bit for bit.  Deadlock-free for C >= K (go_fused_seq).
 // * Failure: every wait is bounded.  A CTA that gave up keeps walking its rows without waiting
 //   and still publishes a word for each, so its group does not wait on it for the whole limit;
 //   the workspace status word reports AAL_ERR_TIMEOUT and the outputs are not to be used.
@@ -87,8 +88,8 @@ __global__ void __launch_bounds__(kThreads, 1) fused_rows(FusedArgs f, int nch, 
   const int64_t NG = f.n_group;        // windows 0 .. NG - 1 go to the groups, the rest to the solo CTAs
   const bool solo = !SEQ && (int)blockIdx.x >= G * K;
   // sequence layout: CTA c takes rows R-1-c, R-1-c-C, ... (C = the grid), so that the rows in
-  // flight at a time are consecutive positions and a row's later neighbours, which its gradient
-  // waits on, are taken in the same round (by CTAs c-1 .. c-K+1) or an earlier one
+  // flight at a time are consecutive positions and a row's neighbours within K - 1 positions,
+  // whose statistics its gradient waits on, are taken in the same round or an adjacent one
   const int C = gridDim.x;
   const int g = blockIdx.x / K, k = blockIdx.x % K;  // (a group's CTA)
   const int so = (int)blockIdx.x - G * K;            // (a solo CTA)
@@ -584,11 +585,13 @@ __global__ void __launch_bounds__(1024) seq_count_valid(const uint8_t* mask, int
   }
 }
 
-// The sequence layout: CTA c of C (one cooperative CTA per SM) takes rows R-1-c, R-1-c-C, ...:
-// the C rows in flight at a time are consecutive positions, and a row's gradient waits only on
-// rows after it, which are taken in the same round by the CTAs before it or in an earlier round.
-// Every wait so points to work that starts no later, and the launch cannot deadlock while all
-// its CTAs are resident (a cooperative launch).
+// The sequence layout: CTA c of C (one cooperative CTA per SM) takes rows R-1-c, R-1-c-C, ...,
+// each row's statistics passes (S(p)) and then its gradient pass (G(p)), which waits on S(q) for
+// |q - p| <= K - 1.  Order the work by rank(S(q)) = R-1-q and rank(G(p)) = R-1-p + K - 1/2: a
+// gradient pass waits only on lower ranks, and a CTA's own sequence S(p), G(p), S(p - C), ...
+// rises in rank when C >= K.  So every wait points to lower-ranked work, no cycle of waits can
+// form, and the launch cannot deadlock while all its CTAs are resident (a cooperative launch).
+// The caller takes the fused path only when C >= K or one round holds every row.
 template <bool NQ1, int P, bool KL, bool GR, bool Q, bool P1 = false>
 cudaError_t go_fused_seq(const FusedArgs& f0, cudaStream_t s, uint64_t limit_ns, bool* launched) {
   auto kern = fused_rows<NQ1, P, KL, GR, Q, P1, true>;

@@ -6,7 +6,7 @@ gradient of aal_seq_loss_fwd followed by aal_seq_loss_bwd bit for bit: on the fu
 of 16-byte multiples; every flag combination it instantiates; masks with holes, prompts and padding;
 full_windows; sequences shorter than the window; fewer positions than SMs, exactly one round of
 rows, and several rounds, so that rows wait on neighbours taken in the same round and in the
-round before; full-size rows) and on the problems it hands to the two calls (fp32, unaligned rows,
+rounds before and after; full-size rows) and on the problems it hands to the two calls (fp32, unaligned rows,
 token ids).  Some cases are also checked against the oracle directly, and the bounded waits are
 driven to a timeout without a fault.
 """
@@ -153,7 +153,7 @@ def test_seq_grpo_is_refused():
                                                (KL | G, 1.0, 0.1, 0.0, False), (KL | TV, 1.0, 0.0, 0.0, False)])
 def test_seq_fused_against_the_oracle(mode, T, wg, ws, full):
     """B = 2 sequences of 200 positions, K = 7, V = 3000 (400 rows: three rounds on 152 SMs, rows
-    whose later neighbours were taken in the round before), masked: every output on every
+    whose neighbours are taken in the round before or after), masked: every output on every
     position against the oracle."""
     t, d, m = _inputs(2, 200, 3000, seed=29, masked=True)
     dloss = float(seq_window_counts(m, 2, 200))
