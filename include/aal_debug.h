@@ -37,12 +37,15 @@ AAL_API void aal_debug_fail_next_forward(int64_t chunk, uint64_t wait_limit_ns);
  * arithmetic: no GPU is touched. */
 AAL_API int64_t aal_debug_solo_windows(int64_t N, int32_t K, int32_t G, int32_t S);
 
-/* The shortest row (in bytes, V times the element size) for which aal_loss_fwd_bwd launches its
- * fused kernels; shorter rows run the two calls inside it, which are faster there (the fused
- * form pays a window exchange per row, and a short row has little streaming to hide it behind).
- * A negative value restores the default (AAL_FUSED_MIN_ROW_BYTES_DEFAULT); 0 fuses every row
- * the fused kernels take, so that a test can exercise them on short rows.  Either way the
- * results are those of the two calls, bit for bit. */
+/* The shortest row (in bytes, V times the element size) for which aal_loss_fwd_bwd and
+ * aal_seq_loss_fwd_bwd launch their fused kernels; shorter rows run the two calls inside them,
+ * which are faster there (the fused form pays a window exchange per row, and a short row has
+ * little streaming to hide it behind).  The same threshold picks the streamed forward's geometry
+ * for bf16 rows (shorter rows: 8 consumer warps and two CTAs an SM; also in the streamed sampling
+ * reward), so the forward inside the fused call and the separate forward agree.  A negative value
+ * restores the default (AAL_FUSED_MIN_ROW_BYTES_DEFAULT); 0 fuses every row the fused kernels
+ * take, so that a test can exercise them on short rows.  Either way the results of the one-call
+ * entry points are those of their two calls, bit for bit. */
 #define AAL_FUSED_MIN_ROW_BYTES_DEFAULT 131072
 AAL_API void aal_debug_fused_min_row_bytes(int64_t bytes);
 

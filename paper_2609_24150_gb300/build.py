@@ -17,9 +17,8 @@ PKG = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libaal.so")
-SOURCES = ["aal.cu", "rowstats.cu", "rowstats_stream.cu", "fused.cu", "window.cu", "backward.cu", "reward.cu",
-           "grpo.cu", "onetensor.cu",
-           "noalloc.cu"]
+SOURCES = ["aal.cu", "rowstats.cu", "rowstats_stream.cu", "rowstats_short.cu", "fused.cu", "window.cu",
+           "backward.cu", "reward.cu", "grpo.cu", "onetensor.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
          "-Xcompiler", "-fvisibility=hidden", "--extended-lambda"]

@@ -238,6 +238,7 @@ SeqWindowArgs seq_window_args(const aal_seq_problem* prob, const uint8_t* mask, 
 
 namespace aal {
 uint64_t debug_wait_limit_ns() { return g_wait_limit_ns.load(); }
+int64_t fused_min_row_bytes() { return g_fused_min_row_bytes.load(); }
 int64_t debug_take_skip_chunk() { return g_skip_chunk.exchange(-1); }
 }  // namespace aal
 
@@ -776,7 +777,9 @@ aal_status aal_accept_reward(const aal_reward_problem* prob, const void* draft, 
     sa.row_offset = prob->row_offset;
     sa.K = (int32_t)prob->K;
     const uint64_t limit = debug_wait_limit_ns();
-    e = launch_reward_stream(sa, s, limit ? limit : kWaitLimitNs);
+    // the geometry the loss forward takes for rows of this length (the same normalisers)
+    e = prob->V * 2 < fused_min_row_bytes() ? launch_reward_stream_short(sa, s, limit ? limit : kWaitLimitNs)
+                                            : launch_reward_stream(sa, s, limit ? limit : kWaitLimitNs);
   } else {
     e = launch_reward_rows(ra, prob->dtype == AAL_BF16, s);
   }

@@ -457,6 +457,12 @@ struct GrpoWindowArgs {
 // Launchers (return cudaGetLastError() of their launches).
 cudaError_t launch_rowstats(const RowStatsArgs& a, bool bf16, cudaStream_t s, int* cluster_used);
 cudaError_t launch_rowstats_stream(const RowStatsArgs& a, bool bf16, cudaStream_t s, uint64_t limit_ns);
+// The same kernels for short rows (rowstats_short.cu): 8 consumer warps, two CTAs an SM.
+cudaError_t launch_rowstats_stream_short(const RowStatsArgs& a, bool bf16, cudaStream_t s, uint64_t limit_ns);
+cudaError_t launch_reward_stream_short(const RowStatsArgs& a, cudaStream_t s, uint64_t limit_ns);
+// Rows shorter than this many bytes take the short-row geometry and the two calls inside
+// aal_loss_fwd_bwd / aal_seq_loss_fwd_bwd (128 KB unless the test hook changed it).
+int64_t fused_min_row_bytes();
 // The sampling reward's acceptance flags from one streamed pass over bf16 rows of 16-byte
 // multiples (a.sT = log2(e) / T, a.acc, a.seed, a.row_offset, a.K).
 cudaError_t launch_reward_stream(const RowStatsArgs& a, cudaStream_t s, uint64_t limit_ns);

@@ -246,8 +246,9 @@ cudaError_t launch_generic(const RowStatsArgs& a, cudaStream_t s) {
 }  // namespace
 
 // The TMA-streamed kernel (rowstats_stream.cu) serves rows whose byte length is a multiple
-// of 16: in two passes with the sampling term, in one pass without it.  Unaligned rows take
-// the generic kernel.
+// of 16: in two passes with the sampling term, in one pass without it; bf16 rows under the fused
+// call's threshold take its short-row geometry (rowstats_short.cu).  Unaligned rows take the
+// generic kernel.
 cudaError_t launch_rowstats(const RowStatsArgs& a, bool bf16, cudaStream_t s, int* cluster_used) {
   const int elt = bf16 ? 2 : 4;
   const bool aligned = ((a.V * elt) % 16 == 0) &&
@@ -255,6 +256,8 @@ cudaError_t launch_rowstats(const RowStatsArgs& a, bool bf16, cudaStream_t s, in
   if (aligned) {
     *cluster_used = 1;
     const uint64_t limit = debug_wait_limit_ns();
+    if (bf16 && a.V * 2 < fused_min_row_bytes())
+      return launch_rowstats_stream_short(a, bf16, s, limit ? limit : kWaitLimitNs);
     return launch_rowstats_stream(a, bf16, s, limit ? limit : kWaitLimitNs);
   }
   *cluster_used = 1;

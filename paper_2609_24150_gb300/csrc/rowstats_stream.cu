@@ -22,7 +22,8 @@
 //     sampling term at T != 1 that is a second z_p state, next to the one at T.  Its REWARD
 //     instance runs at the reward's T and decides the sampling acceptance at each row's end.
 //
-// There is no cross-CTA communication, so all 152 SMs run one CTA each.  Every wait is
+// There is no cross-CTA communication, so all 152 SMs run one CTA each (two with the short-row
+// geometry of rowstats_short.cu).  Every wait is
 // bounded (ptx::wait_phase); after a timeout every thread keeps walking the same loops
 // without waiting (a consumer still folds a chunk it finds landed, into results that are
 // never written), so all meet the same barriers, the producer drains its copies, and the
@@ -358,7 +359,7 @@ struct Smem2 {
 };
 
 template <typename T, bool NEED_Q1, bool KL, bool P1 = false>
-__global__ void __launch_bounds__(kThreads2, 1) rowstats_twopass(RowStatsArgs a, int nch, uint64_t limit_ns) {
+__global__ void __launch_bounds__(kThreads2, kCtasPerSm) rowstats_twopass(RowStatsArgs a, int nch, uint64_t limit_ns) {
   extern __shared__ __align__(1024) unsigned char smem[];
   unsigned char* ring = smem;
   Smem2& S = *reinterpret_cast<Smem2*>(smem + kSlots * kSlotBytes);
@@ -572,7 +573,7 @@ cudaError_t launch_twopass(const RowStatsArgs& a, cudaStream_t s, int nch, uint6
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  int64_t grid = sms;
+  int64_t grid = (int64_t)sms * kCtasPerSm;
   if (grid > a.R) grid = a.R;
   if (grid < 1) return cudaSuccess;
   kern<<<(unsigned)grid, kThreads2, kSmem2Bytes, s>>>(a, nch, limit_ns);
@@ -590,7 +591,14 @@ cudaError_t launch_two_pass(const RowStatsArgs& a, cudaStream_t s, int nch, uint
 
 }  // namespace
 
-cudaError_t launch_rowstats_stream(const RowStatsArgs& a, bool bf16, cudaStream_t s, uint64_t limit_ns) {
+// The exported launchers; rowstats_short.cu compiles this file again for short rows, under
+// other names and another ring geometry.
+#ifndef AAL_ROWSTATS_STREAM_NAME
+#define AAL_ROWSTATS_STREAM_NAME launch_rowstats_stream
+#define AAL_REWARD_STREAM_NAME launch_reward_stream
+#endif
+
+cudaError_t AAL_ROWSTATS_STREAM_NAME(const RowStatsArgs& a, bool bf16, cudaStream_t s, uint64_t limit_ns) {
   const int elt = bf16 ? 2 : 4;
   const int64_t CH = kHalfSlot / elt;
   const int nch = (int)((a.V + CH - 1) / CH);
@@ -598,7 +606,7 @@ cudaError_t launch_rowstats_stream(const RowStatsArgs& a, bool bf16, cudaStream_
   return bf16 ? launch_two_pass<uint16_t>(a, s, nch, limit_ns) : launch_two_pass<float>(a, s, nch, limit_ns);
 }
 
-cudaError_t launch_reward_stream(const RowStatsArgs& a, cudaStream_t s, uint64_t limit_ns) {
+cudaError_t AAL_REWARD_STREAM_NAME(const RowStatsArgs& a, cudaStream_t s, uint64_t limit_ns) {
   const int64_t CH = kHalfSlot / 2;
   const int nch = (int)((a.V + CH - 1) / CH);
   return launch_T<uint16_t, false, 1, false, false, true>(a, s, nch, limit_ns);
