@@ -584,7 +584,23 @@ def run_sequence_layout(aal, dev, stream, rank, reps, seq_len=None):
            "two_call_gbs": round((fb + bb) / ((fwd + bwd) * 1e-3) / 1e9, 1),
            "fwd_gbs": round(fb / (fwd * 1e-3) / 1e9, 1), "bwd_gbs": round(bb / (bwd * 1e-3) / 1e9, 1),
            "loss": float(loss.item())}
-    del target, draft, grad, ws
+    # x* as token ids (L_EAL): the draft alone read forward, draft read + gradient written backward
+    ids = target.argmax(-1).to(torch.int32).contiguous()
+    del target
+    iprob = aal.seq_problem(draft, K, aal.AAL_GREEDY | aal.AAL_IDS, 1.0, 1.0, 0.0)
+    iws = torch.empty(aal.aal_seq_workspace_size(iprob), dtype=torch.uint8, device=dev)
+    ifwd, ibwd = _time_fwd_bwd(
+        aal, lambda: aal.aal_seq_loss_fwd(iprob, draft, ids, None, iws, loss, None, stream),
+        lambda: aal.aal_seq_loss_bwd(iprob, draft, ids, None, iws, 1.0, grad, stream), stream, reps)
+    ifused = _time_call(lambda: aal.aal_seq_loss_fwd_bwd(iprob, draft, ids, None, iws, 1.0, loss, grad, None,
+                                                         stream), stream, reps)
+    assert aal.aal_check_device_status(iws) == aal.AAL_OK
+    ib = 3 * R * row
+    out["token_ids"] = {"mode": "L_EAL, x* as int32 ids", "call": "aal_seq_loss_fwd_bwd", "ms": round(ifused, 4),
+                        "gbs": round(ib / (ifused * 1e-3) / 1e9, 1), "two_call_ms": round(ifwd + ibwd, 4),
+                        "fwd_ms": round(ifwd, 4), "bwd_ms": round(ibwd, 4)}
+    del iws, ids
+    del draft, grad, ws
     return out
 
 

@@ -242,8 +242,9 @@ AAL_API aal_status aal_seq_loss_bwd(const aal_seq_problem* prob, const void* dra
  * cooperative launch streams the positions with one CTA per SM, consecutive positions on
  * consecutive SMs at the same time, so that a position's gradient (which needs the acceptances
  * of the K - 1 positions before and after it) is written while its rows are still in L2: 2 V b
- * read and V b written per position, instead of 2 V b (forward) + 3 V b (backward).  Other
- * problems (fp32, unaligned rows, token ids) run the two calls inside this one.  AAL_GRPO is
+ * read and V b written per position, instead of 2 V b (forward) + 3 V b (backward); with token
+ * ids (AAL_GREEDY | AAL_IDS) the draft alone is streamed the same way, V b read and V b written.
+ * Other problems (fp32, unaligned rows) run the two calls inside this one.  AAL_GRPO is
  * rejected with AAL_ERR_UNSUPPORTED (its coefficients come from aal_seq_grpo_from_loss, between
  * the forward and the backward).  A bounded device wait that ran out is reported by
  * aal_check_device_status as AAL_ERR_TIMEOUT; the outputs are then not to be used. */

@@ -476,13 +476,52 @@ aal_status aal_seq_loss_fwd_bwd(const aal_seq_problem* prob, const void* draft, 
   const SeqLayout L = seq_layout(prob->B, prob->seq_len, prob->K);
   if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < L.total) return AAL_ERR_WORKSPACE;
 
-  // the fused kernel: bf16 rows of 16-byte multiples, both tensors as logits, and a round of
-  // rows (one per SM) that spans a window or holds every row (its order is deadlock-free then)
+  // the fused kernels: bf16 rows of 16-byte multiples (both tensors as logits, or the draft with
+  // token ids), and a round of rows (one per SM) that spans a window or holds every row (their
+  // order is deadlock-free then)
   int dev = 0, sms = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
     return AAL_ERR_CUDA;
-  const bool fusable = prob->dtype == AAL_BF16 && (prob->mode & AAL_IDS) == 0 && (prob->V * 2) % 16 == 0 &&
-                       prob->V * 2 >= g_fused_min_row_bytes.load() && (sms >= prob->K || R <= sms);
+  const bool rows16 = prob->dtype == AAL_BF16 && (prob->V * 2) % 16 == 0 &&
+                      prob->V * 2 >= g_fused_min_row_bytes.load() && (sms >= prob->K || R <= sms);
+  const bool ids = (prob->mode & AAL_IDS) != 0;
+  if (rows16 && ids) {  // x* as token ids: the draft alone is streamed
+    LossWs ws = loss_ws(workspace, L.base);
+    if (cudaMemsetAsync(ws.hdr, 0, sizeof(WsHeader), s) != cudaSuccess) return AAL_ERR_CUDA;
+    if (cudaMemsetAsync(ws.mbox, 0xff, (size_t)R * 8, s) != cudaSuccess) return AAL_ERR_CUDA;  // kMboxEmpty
+    const SeqWindowArgs wa = seq_window_args(prob, mask, 1, loss, eal, workspace, L);
+    if (launch_seq_count_valid(mask, prob->B, prob->seq_len, (int32_t)prob->K, wa.full_windows, wa.nvalid_g,
+                               wa.npos_g, ws.hdr, s) != cudaSuccess)
+      return AAL_ERR_CUDA;
+    FusedIdsArgs f;
+    f.st.z = draft;
+    f.st.R = R;
+    f.st.V = prob->V;
+    f.st.lws = ws;
+    f.st.ids = static_cast<const int32_t*>(target);
+    f.st.acc = nullptr;
+    f.st.acc_ref = nullptr;
+    f.st.lpr = nullptr;
+    f.st.hdr = ws.hdr;
+    f.st.skip_chunk = debug_take_skip_chunk();
+    f.bw = grad_args(draft, target, mask, R, prob->V, prob->mode, prob->temperature, prob->w_greedy, prob->w_kl,
+                     dloss, ws, grad_draft);
+    f.win = WindowArgs{};
+    f.win.N = R;
+    f.win.K = (int32_t)prob->K;
+    f.win.greedy = wa.greedy;
+    f.groups = 0;
+    f.solos = 0;
+    f.n_group = 0;
+    f.seq_T = prob->seq_len;
+    f.seq_full = wa.full_windows ? 1 : 0;
+    f.seq_mask = mask;
+    const uint64_t limit = debug_wait_limit_ns();
+    bool launched = false;
+    if (launch_fused_ids_seq(f, s, limit ? limit : kWaitLimitNs, &launched) != cudaSuccess) return AAL_ERR_CUDA;
+    if (launched) return cuda_status(launch_seq_window(wa, s));
+  }
+  const bool fusable = rows16 && !ids;
   if (fusable) {
     LossWs ws = loss_ws(workspace, L.base);
     if (cudaMemsetAsync(ws.hdr, 0, sizeof(WsHeader), s) != cudaSuccess) return AAL_ERR_CUDA;

@@ -492,8 +492,9 @@ cudaError_t launch_fused_ids(const FusedIdsArgs& f, cudaStream_t s, uint64_t lim
 // counts them.
 cudaError_t launch_seq_count_valid(const uint8_t* mask, int64_t B, int64_t T, int32_t K, bool full,
                                    int32_t nvalid_g, int32_t npos_g, WsHeader* hdr, cudaStream_t s);
-// The fused forward + backward over the sequence layout (FusedArgs.seq_T > 0).
+// The fused forward + backward over the sequence layout (FusedArgs.seq_T > 0), and with token ids.
 cudaError_t launch_fused_seq(const FusedArgs& f, cudaStream_t s, uint64_t limit_ns, bool* launched);
+cudaError_t launch_fused_ids_seq(const FusedIdsArgs& f, cudaStream_t s, uint64_t limit_ns, bool* launched);
 
 // ---------------------------------------------------------------------------
 // Device helpers.

@@ -483,7 +483,10 @@ cudaError_t launch_T(const Stream1Args& a, bool ids, cudaStream_t s) {
 // for the gradient -dloss/|W| w_g dE/da a^g (delta_{u,x*} - q(u)).  Statistics, exchange and
 // coefficients reuse the IDS stream's and the backward's code, so the results are bitwise those
 // of aal_loss_fwd + aal_loss_bwd; resolve_draft_argmax and the window kernel run after it.
-// The SMs that G K leaves over take whole windows as solo CTAs, as in fused.cu.
+// The SMs that G K leaves over take whole windows as solo CTAs, as in fused.cu.  SEQ: the
+// sequence layout (aal_seq_loss_fwd_bwd with token ids), every CTA walking the positions from the
+// last one down and exchanging with the 2K - 1 positions around its row, as fused.cu's SEQ
+// instances do.
 constexpr int kRBarCoef = 3;
 
 struct FusedIdsSmem {
@@ -498,6 +501,7 @@ struct FusedIdsSmem {
 
 constexpr size_t kFIdsSmemBytes = (size_t)kRSlots * kRSlotBytes + sizeof(FusedIdsSmem);
 
+template <bool SEQ>
 __global__ void __launch_bounds__(kRThreads, 1) fused_ids_rows(FusedIdsArgs f, int nch, uint64_t limit_ns) {
   using T = uint16_t;
   constexpr int E = 8;
@@ -515,9 +519,10 @@ __global__ void __launch_bounds__(kRThreads, 1) fused_ids_rows(FusedIdsArgs f, i
   const int64_t N = f.win.N;
   const int G = f.groups;
   const int64_t NG = f.n_group;  // windows 0 .. NG - 1 go to the groups, the rest to the solo CTAs
-  const bool solo = (int)blockIdx.x >= G * K;
+  const bool solo = !SEQ && (int)blockIdx.x >= G * K;
   const int g = blockIdx.x / K, k = blockIdx.x % K;  // (a group's CTA)
   const int so = (int)blockIdx.x - G * K;            // (a solo CTA)
+  const int C = gridDim.x;                           // (the sequence layout: rows R-1-c, R-1-c-C, ...)
 
   if (threadIdx.x == 0) {
     for (int q = 0; q < kRSlots; ++q) {
@@ -556,7 +561,12 @@ __global__ void __launch_bounds__(kRThreads, 1) fused_ids_rows(FusedIdsArgs f, i
           }
         }
       };
-      if (!solo) {
+      if (SEQ) {
+        for (int64_t p = a.R - 1 - blockIdx.x; p >= 0 && !*abort_flag; p -= C) {
+          issue(p, 0);
+          issue(p, 1);
+        }
+      } else if (!solo) {
         for (int64_t n = g; n < NG && !*abort_flag; n += G) {
           issue(n * K + k, 0);
           issue(n * K + k, 1);
@@ -696,7 +706,33 @@ __global__ void __launch_bounds__(kRThreads, 1) fused_ids_rows(FusedIdsArgs f, i
       }
     };
 
-    if (!solo) {
+    if (SEQ) {
+      // each row: statistics, its mailbox word, the exchange with the positions around it (warp
+      // 0), the coefficients (thread 0), the gradient
+      for (int64_t r = a.R - 1 - blockIdx.x; r >= 0; r -= C) {
+        RowStat st{};
+        stats_row(r, st);
+        if (warp == 0) {
+          if (lane == 0) ptx::st_relaxed(&a.lws.mbox[r], mbox_word(st.ag, 0.f));
+          const int64_t lo = r - r % f.seq_T, hi = lo + f.seq_T - 1;
+          float dEg = 0.f, dEs = 0.f;
+          const bool ok = seq_exchange(a.lws.mbox, f.seq_mask, r, lo, hi, K, f.seq_full != 0, true, false, false,
+                                       0.f, 0.f, true, lane, abort_flag, hdr, limit_ns, &dEg, &dEs);
+          if (lane == 0) {
+            RowCoef c;
+            const bool pos_valid = f.bw.mask == nullptr || f.bw.mask[r] != 0;
+            F.live = ok && row_coef<true, false, false>(f.bw, scale, 0.f, f.bw.w_greedy != 0.f ? dEg : 0.f, 0.f, 0.f,
+                                                       pos_valid, st, c)
+                         ? 1
+                         : 0;
+            if (F.live) F.coef = c;
+          }
+        }
+        named_barrier(kRBarCoef, kRConsumers);
+        const RowCoef c = F.coef;
+        grad_row(r, c, F.live);
+      }
+    } else if (!solo) {
       // one row of each of the group's windows: statistics, the window exchange (warp 0: lane j
       // polls depth j), the coefficients (thread 0), the gradient
       for (int64_t n = g; n < NG; n += G) {
@@ -750,10 +786,12 @@ __global__ void __launch_bounds__(kRThreads, 1) fused_ids_rows(FusedIdsArgs f, i
 
 }  // namespace
 
-cudaError_t launch_fused_ids(const FusedIdsArgs& f0, cudaStream_t s, uint64_t limit_ns, bool* launched) {
+namespace {
+template <bool SEQ>
+cudaError_t go_fused_ids(const FusedIdsArgs& f0, cudaStream_t s, uint64_t limit_ns, bool* launched) {
   *launched = false;
   if (f0.bw.w_greedy == 0.f || f0.bw.grpo) return cudaSuccess;  // only the greedy term is fused here
-  auto kern = fused_ids_rows;
+  auto kern = fused_ids_rows<SEQ>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFIdsSmemBytes);
   if (e != cudaSuccess) return e;
   int dev = 0, sms = 0, per_sm = 0, coop = 0;
@@ -763,22 +801,31 @@ cudaError_t launch_fused_ids(const FusedIdsArgs& f0, cudaStream_t s, uint64_t li
   e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kRThreads, kFIdsSmemBytes);
   if (e != cudaSuccess) return e;
   const int64_t K = f0.win.K;
-  int64_t G = (int64_t)sms * per_sm / K;
-  if (G > f0.win.N) G = f0.win.N;
-  if (G > kMaxGroups) G = kMaxGroups;
-  if (!coop || G < 1) return cudaSuccess;
-  // the SMs left over by the groups take whole windows alone
-  const int64_t S = (int64_t)sms * per_sm - G * K;
-  const int64_t m = solo_windows_each(f0.win.N, K, G, S);
   FusedIdsArgs f = f0;
-  f.groups = (int32_t)G;
-  f.solos = m > 0 ? (int32_t)S : 0;
-  f.n_group = f0.win.N - m * f.solos;
+  int64_t grid = 0;
+  if (SEQ) {
+    // one CTA per SM walking the positions down; deadlock-free when a round spans a window or
+    // holds every row (fused.cu, go_fused_seq)
+    grid = (int64_t)sms * per_sm;
+    if (grid > f.st.R) grid = f.st.R;
+    if (!coop || grid < 1 || (grid < K && grid < f.st.R)) return cudaSuccess;
+  } else {
+    int64_t G = (int64_t)sms * per_sm / K;
+    if (G > f0.win.N) G = f0.win.N;
+    if (G > kMaxGroups) G = kMaxGroups;
+    if (!coop || G < 1) return cudaSuccess;
+    // the SMs left over by the groups take whole windows alone
+    const int64_t S = (int64_t)sms * per_sm - G * K;
+    const int64_t m = solo_windows_each(f0.win.N, K, G, S);
+    f.groups = (int32_t)G;
+    f.solos = m > 0 ? (int32_t)S : 0;
+    f.n_group = f0.win.N - m * f.solos;
+    grid = G * K + f.solos;
+  }
   const int CH = kRSlotBytes / 2;
   const int nch = (int)((f.st.V + CH - 1) / CH);
   void* args[] = {&f, (void*)&nch, &limit_ns};
-  e = cudaLaunchCooperativeKernel((const void*)kern, dim3((unsigned)(G * K + f.solos)), dim3(kRThreads), args,
-                                  kFIdsSmemBytes, s);
+  e = cudaLaunchCooperativeKernel((const void*)kern, dim3((unsigned)grid), dim3(kRThreads), args, kFIdsSmemBytes, s);
   if (e == cudaErrorCooperativeLaunchTooLarge) {  // fewer SMs available: the caller runs the two calls
     cudaGetLastError();
     return cudaSuccess;
@@ -787,6 +834,15 @@ cudaError_t launch_fused_ids(const FusedIdsArgs& f0, cudaStream_t s, uint64_t li
   *launched = true;
   resolve_draft_argmax<uint16_t><<<(unsigned)((f.st.R + 255) / 256), 256, 0, s>>>(f.st);
   return cudaGetLastError();
+}
+}  // namespace
+
+cudaError_t launch_fused_ids(const FusedIdsArgs& f, cudaStream_t s, uint64_t limit_ns, bool* launched) {
+  return go_fused_ids<false>(f, s, limit_ns, launched);
+}
+
+cudaError_t launch_fused_ids_seq(const FusedIdsArgs& f, cudaStream_t s, uint64_t limit_ns, bool* launched) {
+  return go_fused_ids<true>(f, s, limit_ns, launched);
 }
 
 cudaError_t launch_one_tensor(const Stream1Args& a, bool bf16, bool ids, cudaStream_t s) {

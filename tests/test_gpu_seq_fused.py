@@ -6,9 +6,9 @@ gradient of aal_seq_loss_fwd followed by aal_seq_loss_bwd bit for bit: on the fu
 of 16-byte multiples; every flag combination it instantiates; masks with holes, prompts and padding;
 full_windows; sequences shorter than the window; fewer positions than SMs, exactly one round of
 rows, and several rounds, so that rows wait on neighbours taken in the same round and in the
-rounds before and after; full-size rows) and on the problems it hands to the two calls (fp32, unaligned rows,
-token ids).  Some cases are also checked against the oracle directly, and the bounded waits are
-driven to a timeout without a fault.
+rounds before and after; full-size rows; token ids, with the draft alone streamed) and on the
+problems it hands to the two calls (fp32, unaligned rows).  Some cases are also checked against the
+oracle directly, and the bounded waits are driven to a timeout without a fault.
 """
 
 import numpy as np
@@ -17,7 +17,9 @@ import torch
 
 import paper_2609_24150_gb300 as aal
 import synth
-from tests.parity import SeqRun, assert_bands, check_seq_loss, check_seq_positions, seq_window_counts
+import oracle
+from tests.parity import (GRAD_ATOL, GRAD_RTOL, LOSS_ATOL, LOSS_RTOL, SeqRun, assert_bands, check_seq_loss,
+                          check_seq_positions, seq_window_counts)
 
 pytestmark = pytest.mark.gpu
 
@@ -136,10 +138,74 @@ def test_seq_problems_the_two_calls_take(mode, T, dtype, V):
     assert_same(f, s)
 
 
-def test_seq_token_ids_take_the_two_calls():
-    t, d, m = _inputs(2, 90, 4096, seed=31, masked=True)
+@pytest.mark.parametrize("Bn,Tn,K,V,masked,full", [
+    (2, 90, 4, 4096, True, False),      # fewer rows than SMs
+    (2, 200, 7, 2000, True, False),     # three rounds of rows
+    (2, 200, 7, 2000, True, True),      # ... full windows only
+    (1, 153, 8, 1000, False, False),    # one row in the second round, K = 8
+    (5, 64, 1, 4096, True, False),      # K = 1
+    (4, 3, 7, 4104, False, False),      # sequences shorter than the window
+    (30, 20, 3, 8, True, False),        # one 16-byte vector a row
+])
+@pytest.mark.parametrize("dloss_is_w", [False, True])
+def test_seq_token_ids_fused_equals_two_calls(Bn, Tn, K, V, masked, full, dloss_is_w):
+    """x* as token ids (AAL_GREEDY | AAL_IDS): the draft alone streamed, bitwise the two calls."""
+    t, d, m = _inputs(Bn, Tn, V, seed=Bn + Tn + K + V, masked=masked)
     ids = t.float().argmax(-1).to(torch.int32).contiguous()
-    f, s = _runs(ids, d, m, 4, G | IDS, 1.0, 1.0, 0.0, 1.0)
+    dloss = float(seq_window_counts(m, Bn, Tn)) if dloss_is_w else 1.0
+    f, s = _runs(ids, d, m, K, G | IDS, 1.0, 1.0, 0.0, dloss, full)
+    assert_same(f, s)
+
+
+def test_seq_token_ids_fused_against_the_oracle():
+    """400 rows (three rounds), masked, K = 7: every output on every position against the oracle."""
+    t, d, m = _inputs(2, 200, 3000, seed=37, masked=True)
+    ids = t.float().argmax(-1).to(torch.int32).contiguous()
+    dloss = float(seq_window_counts(m, 2, 200))
+    run = SeqRun(ids, d, m, 7, G | IDS, 1.0, 1.0, 0.0, dloss, fused=True)
+    ids_h, m_h = ids.cpu().numpy(), m.cpu().numpy()
+    fw = oracle.seq_loss_forward(None, d.cpu(), m_h, 7, oracle.MODE_GREEDY, xstar=ids_h)
+    np.testing.assert_allclose(run.eal.cpu().numpy()[:, 0], fw["eal_g"], rtol=LOSS_RTOL, atol=LOSS_ATOL)
+    assert abs(run.loss.item() - fw["loss"]) <= LOSS_RTOL * abs(fw["loss"]) + LOSS_ATOL
+    g_ref = oracle.seq_loss_backward(None, d.cpu(), m_h, 7, oracle.MODE_GREEDY, dloss=dloss, xstar=ids_h)
+    g = run.grad.double().cpu().numpy()
+    bad = np.abs(g - g_ref) > GRAD_ATOL + GRAD_RTOL * np.abs(g_ref)
+    assert not bad.any(), (int(bad.sum()), tuple(np.argwhere(bad)[0]))
+
+
+def test_seq_token_ids_out_of_range_reported():
+    t, d, _ = _inputs(2, 100, 4096, seed=43)
+    ids = t.float().argmax(-1).to(torch.int32).contiguous()
+    ids[1, 17] = 4096                                   # one id past the vocabulary
+    prob = aal.seq_problem(d, 5, G | IDS, 1.0, 1.0, 0.0)
+    ws = torch.empty(aal.aal_seq_workspace_size(prob), dtype=torch.uint8, device=DEV)
+    loss = torch.empty(1, device=DEV)
+    grad = torch.empty_like(d)
+    aal.aal_seq_loss_fwd_bwd(prob, d, ids, None, ws, 1.0, loss, grad)
+    assert aal.aal_check_device_status(ws) == aal.AAL_ERR_INVALID_ARG
+    ws2 = torch.empty_like(ws)
+    g2 = torch.empty_like(grad)
+    aal.aal_seq_loss_fwd(prob, d, ids, None, ws2, loss)
+    aal.aal_seq_loss_bwd(prob, d, ids, None, ws2, 1.0, g2)
+    assert aal.aal_check_device_status(ws2) == aal.AAL_ERR_INVALID_ARG
+    assert torch.equal(_bits(grad), _bits(g2))
+
+
+def test_seq_token_ids_ring_times_out_and_context_stays_usable():
+    t, d, _ = _inputs(2, 200, 40000, seed=12)
+    ids = t.float().argmax(-1).to(torch.int32).contiguous()
+    prob = aal.seq_problem(d, 7, G | IDS, 1.0, 1.0, 0.0)
+    ws = torch.empty(aal.aal_seq_workspace_size(prob), dtype=torch.uint8, device=DEV)
+    loss = torch.empty(1, device=DEV)
+    grad = torch.empty_like(d)
+    aal.aal_debug_fail_next_forward(2, 50_000_000)
+    try:
+        aal.aal_seq_loss_fwd_bwd(prob, d, ids, None, ws, 1.0, loss, grad)
+        assert aal.aal_check_device_status(ws) == aal.AAL_ERR_TIMEOUT
+        assert aal.aal_check_device_status(ws) == aal.AAL_OK
+    finally:
+        aal.aal_debug_fail_next_forward(-1, 0)
+    f, s = _runs(ids, d, None, 7, G | IDS, 1.0, 1.0, 0.0, 1.0)
     assert_same(f, s)
 
 
