@@ -260,6 +260,15 @@ def run_ours(args, ws_count, rank, local):
     r1.record(stream)
     torch.cuda.synchronize()
     ms_reward_sampled = r0.elapsed_time(r1) / reps
+    # the same draws with the normalisers the batch's loss forward left in ws: the draft alone read
+    aal.aal_accept_reward_sampled_from_loss(sprob, prob, draft, target, ws, rws, tau, rl, adv, stream)
+    r0.record(stream)
+    for _ in range(reps):
+        aal.aal_accept_reward_sampled_from_loss(sprob, prob, draft, target, ws, rws, tau, rl, adv, stream)
+    r1.record(stream)
+    torch.cuda.synchronize()
+    assert aal.aal_check_device_status(rws) == aal.AAL_OK
+    ms_reward_sampled_stats = r0.elapsed_time(r1) / reps
 
     lines = set() if args.no_seq else {x.strip() for x in args.lines.split(",") if x.strip()}
     reps = max(5, args.steps // 2)
@@ -312,7 +321,12 @@ def run_ours(args, ws_count, rank, local):
                           "bwd_gbs": round(b["bwd"] / (bwd2 * 1e-3) / 1e9, 1)},
         "reward_sampled_draft": {"ms": round(ms_reward_sampled, 4),
                                  "gbs": round(2 * R * V * 2 / (ms_reward_sampled * 1e-3) / 1e9, 1),
-                                 "note": "aal_accept_reward, AAL_SAMPLING | AAL_SAMPLED_DRAFT at T = 1"},
+                                 "note": "aal_accept_reward, AAL_SAMPLING | AAL_SAMPLED_DRAFT at T = 1",
+                                 "from_loss_ms": round(ms_reward_sampled_stats, 4),
+                                 "from_loss_gbs": round(R * V * 2 / (ms_reward_sampled_stats * 1e-3) / 1e9, 1),
+                                 "from_loss_note": "aal_accept_reward_sampled_from_loss after the step's forward: "
+                                                   "the same draws, the loss forward's normalisers, the draft "
+                                                   "alone streamed (V b a row)"},
         "reward_logit_pass": {"ms": round(ms_reward_pass, 4),
                               "gbs": round(2 * R * V * 2 / (ms_reward_pass * 1e-3) / 1e9, 1),
                               "note": "aal_accept_reward streaming draft + target itself"},

@@ -399,6 +399,26 @@ AAL_API aal_status aal_accept_reward_from_loss(const aal_reward_problem* rprob, 
                                                void* workspace, size_t workspace_bytes, int32_t* tau,
                                                float* rollout_len, float* advantage, void* stream);
 
+/* The sampled-draft reward (mode AAL_SAMPLING | AAL_SAMPLED_DRAFT, no reference draft) with the
+ * normalisers of p~ and q~ that aal_loss_fwd left in `loss_workspace`: the draws need every
+ * vocabulary entry of the draft, so the draft is streamed once (V b a row), but not the target,
+ * which is read at the drawn token only, and no log-sum-exp is formed.  The draws are those of
+ * aal_accept_reward; the acceptance uses the loss forward's normalisers instead of the reward's
+ * own, which may differ from them in the last bits, so a draw within rounding of its threshold
+ * may be decided the other way.
+ *   rprob     mode AAL_SAMPLING | AAL_SAMPLED_DRAFT; N, K, V, dtype must equal lprob's.
+ *   lprob, loss_workspace  a completed aal_loss_fwd (same stream) whose mode has the sampling
+ *             term at the reward's temperature (not token ids); otherwise AAL_ERR_INVALID_ARG.
+ *   draft, target  the [N][K][V] logits of that forward, 16-byte aligned.
+ *   workspace  at least aal_reward_workspace_size(rprob) bytes.
+ * Outputs as for aal_accept_reward (no reference draft).  Rows whose byte length is not a
+ * multiple of 16 run aal_accept_reward's own pass. */
+AAL_API aal_status aal_accept_reward_sampled_from_loss(const aal_reward_problem* rprob, const aal_problem* lprob,
+                                                       const void* draft, const void* target,
+                                                       const void* loss_workspace, size_t loss_workspace_bytes,
+                                                       void* workspace, size_t workspace_bytes, int32_t* tau,
+                                                       float* rollout_len, float* advantage, void* stream);
+
 /* aal_accept_reward without a workspace argument: the scratch lives in a fixed array inside
  * the library.  The paper has no counterpart; this exists for callers that cannot allocate
  * device memory -- e.g. a training loop whose device memory is all reserved up front by its

@@ -37,6 +37,7 @@ from .aal import (  # noqa: F401
     aal_abi_version,
     aal_accept_reward,
     aal_accept_reward_from_loss,
+    aal_accept_reward_sampled_from_loss,
     aal_accept_reward_noalloc,
     aal_check_device_status,
     aal_debug_fail_next_forward,

@@ -105,6 +105,7 @@ def library() -> ctypes.CDLL:
     lib.aal_accept_reward.argtypes = [RP, vp, vp, vp, vp, sz, vp, vp, vp, vp, vp]
     lib.aal_accept_reward_noalloc.argtypes = [RP, vp, vp, vp, vp, vp, vp, vp, vp]
     lib.aal_accept_reward_from_loss.argtypes = [RP, P, vp, sz, vp, sz, vp, vp, vp, vp]
+    lib.aal_accept_reward_sampled_from_loss.argtypes = [RP, P, vp, vp, vp, sz, vp, sz, vp, vp, vp, vp]
     SP = ctypes.POINTER(AalSeqProblem)
     lib.aal_seq_workspace_size.argtypes = [SP, ctypes.POINTER(sz)]
     lib.aal_seq_loss_fwd.argtypes = [SP, vp, vp, vp, vp, sz, vp, vp, vp]
@@ -128,7 +129,8 @@ def library() -> ctypes.CDLL:
     lib.aal_abi_version.restype = ctypes.c_int32
     for f in ("aal_workspace_size", "aal_reward_workspace_size", "aal_loss_fwd", "aal_loss_bwd", "aal_loss_fwd_bwd",
               "aal_accept_reward", "aal_accept_reward_noalloc", "aal_accept_reward_from_loss",
-              "aal_seq_workspace_size", "aal_seq_loss_fwd", "aal_seq_loss_bwd", "aal_check_device_status",
+              "aal_accept_reward_sampled_from_loss", "aal_seq_workspace_size", "aal_seq_loss_fwd",
+              "aal_seq_loss_bwd", "aal_seq_loss_fwd_bwd", "aal_check_device_status",
               "aal_grpo_workspace_size", "aal_grpo_from_loss", "aal_seq_grpo_workspace_size",
               "aal_seq_grpo_from_loss"):
         getattr(lib, f).restype = ctypes.c_int
@@ -421,6 +423,21 @@ def aal_accept_reward_from_loss(problem: AalRewardProblem, loss_problem_: AalPro
         _ptr(tau, "tau", torch.int32, N), _ptr(rollout_len, "rollout_len", torch.float32, nroll),
         _ptr(advantage, "advantage", torch.float32, nroll), _stream(stream))
     _check(code, "aal_accept_reward_from_loss")
+
+
+def aal_accept_reward_sampled_from_loss(problem: AalRewardProblem, loss_problem_: AalProblem, draft, target,
+                                        loss_workspace, workspace, tau, rollout_len, advantage, stream=None):
+    """The sampled-draft reward with the normalisers of a completed aal_loss_fwd: the draft
+    streamed once for the draws, the target read at the drawn tokens only."""
+    N = problem.N
+    nroll = N // max(1, problem.windows_per_rollout)
+    code = library().aal_accept_reward_sampled_from_loss(
+        ctypes.byref(problem), ctypes.byref(loss_problem_), _ptr(draft, "draft"), _ptr(target, "target"),
+        _ptr(loss_workspace, "loss_workspace"), _nbytes(loss_workspace), _ptr(workspace, "workspace"),
+        _nbytes(workspace), _ptr(tau, "tau", torch.int32, N),
+        _ptr(rollout_len, "rollout_len", torch.float32, nroll),
+        _ptr(advantage, "advantage", torch.float32, nroll), _stream(stream))
+    _check(code, "aal_accept_reward_sampled_from_loss")
 
 
 def aal_accept_reward_noalloc(problem: AalRewardProblem, draft, target, ref_draft, tau, tau_ref,

@@ -897,6 +897,73 @@ aal_status aal_accept_reward_from_loss(const aal_reward_problem* rprob, const aa
   return cuda_status(launch_reward_groups(ga, s));
 }
 
+aal_status aal_accept_reward_sampled_from_loss(const aal_reward_problem* rprob, const aal_problem* lprob,
+                                               const void* draft, const void* target, const void* loss_workspace,
+                                               size_t loss_workspace_bytes, void* workspace, size_t workspace_bytes,
+                                               int32_t* tau, float* rollout_len, float* advantage, void* stream) {
+  aal_status st = check_reward(rprob);
+  if (st != AAL_OK) return st;
+  st = check_problem(lprob);
+  if (st != AAL_OK) return st;
+  if (rprob->N != lprob->N || rprob->K != lprob->K || rprob->V != lprob->V || rprob->dtype != lprob->dtype)
+    return AAL_ERR_INVALID_ARG;
+  if (rprob->mode != (AAL_SAMPLING | AAL_SAMPLED_DRAFT)) return AAL_ERR_INVALID_ARG;
+  // the acceptance needs the loss's temperature-scaled normalisers at this T, from both logit tensors
+  if (!(lprob->mode & AAL_SAMPLING) || (lprob->mode & AAL_IDS) || lprob->temperature != rprob->temperature)
+    return AAL_ERR_INVALID_ARG;
+  if (rprob->N == 0) return AAL_OK;
+  if (draft == nullptr || target == nullptr || !aligned(draft, 16) || !aligned(target, 16)) return AAL_ERR_INVALID_ARG;
+  if (tau == nullptr || rollout_len == nullptr || advantage == nullptr || !aligned(tau, 4) ||
+      !aligned(rollout_len, 4) || !aligned(advantage, 4))
+    return AAL_ERR_INVALID_ARG;
+  const LossLayout LL = loss_layout(lprob->N, lprob->K);
+  if (loss_workspace == nullptr || !aligned(loss_workspace, 256) || loss_workspace_bytes < LL.total)
+    return AAL_ERR_WORKSPACE;
+  const RewardLayout L = reward_layout(rprob->N, rprob->K);
+  if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < L.total) return AAL_ERR_WORKSPACE;
+  const int64_t elt = rprob->dtype == AAL_BF16 ? 2 : 4;
+  if ((rprob->V * elt) % 16 != 0)  // rows that are not 16-byte multiples: the reward's own pass
+    return aal_accept_reward(rprob, draft, target, nullptr, workspace, workspace_bytes, tau, nullptr, rollout_len,
+                             advantage, stream);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  char* base = static_cast<char*>(workspace);
+  WsHeader* hdr = reinterpret_cast<WsHeader*>(base + L.hdr);
+  if (cudaMemsetAsync(hdr, 0, sizeof(WsHeader), s) != cudaSuccess) return AAL_ERR_CUDA;
+
+  RewardRowArgs ra;
+  ra.sampled_draft = true;
+  ra.zq = draft;
+  ra.zp = target;
+  ra.zr = nullptr;
+  ra.R = L.R;
+  ra.V = rprob->V;
+  ra.K = (int32_t)rprob->K;
+  ra.sampling = true;
+  ra.sT = kLog2e / rprob->temperature;
+  ra.seed = rprob->seed;
+  ra.row_offset = rprob->row_offset;
+  ra.acc = reinterpret_cast<uint8_t*>(base + L.acc);
+  ra.acc_ref = nullptr;
+  ra.hdr = hdr;
+  ra.lws = loss_ws(const_cast<void*>(loss_workspace), LL);
+  if (launch_reward_sampled_stats(ra, rprob->dtype == AAL_BF16, s) != cudaSuccess) return AAL_ERR_CUDA;
+
+  RewardGroupArgs ga;
+  ga.acc = ra.acc;
+  ga.acc_ref = nullptr;
+  ga.rbuf = reinterpret_cast<float*>(base + L.rbuf);
+  ga.N = rprob->N;
+  ga.K = (int32_t)rprob->K;
+  ga.wpr = rprob->windows_per_rollout;
+  ga.rpg = rprob->rollouts_per_group;
+  ga.adv_clip = rprob->adv_clip;
+  ga.tau = tau;
+  ga.tau_ref = nullptr;
+  ga.rollout_len = rollout_len;
+  ga.advantage = advantage;
+  return cuda_status(launch_reward_groups(ga, s));
+}
+
 aal_status aal_check_device_status(void* workspace, void* stream) {
   if (workspace == nullptr || !aligned(workspace, 256)) return AAL_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);

@@ -282,6 +282,7 @@ struct RewardRowArgs {
   uint8_t* acc;
   uint8_t* acc_ref;
   WsHeader* hdr;
+  LossWs lws;        // the sampled draft from a loss forward: its normalisers of z_p/T and z_q/T
 };
 
 // Acceptance flags from the statistics a loss forward left in its workspace.
@@ -477,6 +478,9 @@ cudaError_t launch_backward(const BackwardArgs& a, bool bf16, cudaStream_t s);
 cudaError_t launch_reward_rows(const RewardRowArgs& a, bool bf16, cudaStream_t s);
 cudaError_t launch_reward_groups(const RewardGroupArgs& a, cudaStream_t s);
 cudaError_t launch_reward_flags_from_stats(const RewardStatsArgs& a, cudaStream_t s);
+// The sampled-draft reward with the loss forward's normalisers (RewardRowArgs.lws): the draft alone
+// streamed for the draws, the target read at each drawn token; 16-byte rows.
+cudaError_t launch_reward_sampled_stats(const RewardRowArgs& a, bool bf16, cudaStream_t s);
 cudaError_t launch_one_tensor(const Stream1Args& a, bool bf16, bool ids, cudaStream_t s);
 cudaError_t launch_grpo_windows(const GrpoWindowArgs& a, cudaStream_t s);
 cudaError_t launch_seq_grpo_gather(const SeqGrpoArgs& a, cudaStream_t s);

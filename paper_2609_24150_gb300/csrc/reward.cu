@@ -359,7 +359,9 @@ __device__ __forceinline__ void lse_fold_bf16(Lse& L, const uint4& w, float s) {
 
 // Four blocks an SM for both instances: measured against five (without the reference draft,
 // 48 registers) and three (with it, 72 registers and no spill), both slower.
-template <typename T, bool REF>
+// STATS: the normalisers of z_p/T and z_q/T come from a loss forward's workspace (a.lws), so only
+// the draft is streamed (for the draws) and the target is read at the drawn token alone.
+template <typename T, bool REF, bool STATS = false>
 __global__ void __launch_bounds__(kRowThreads, 4) reward_sampled_rows(RewardRowArgs a) {
   __shared__ RowState red[kRowWarps];
   __shared__ Draw dred[2][kRowWarps];
@@ -383,11 +385,12 @@ __global__ void __launch_bounds__(kRowThreads, 4) reward_sampled_rows(RewardRowA
     const int64_t nv = a.V / E;
     for (int64_t i = threadIdx.x; i < nv; i += kRowThreads) {
       float qv[E], pv[E], rv[E], g[E], kq[E], kr[E];
-      const uint4 qw = ldg_stream(q4 + i), pw = ldg_stream(p4 + i);
+      const uint4 qw = ldg_stream(q4 + i);
+      const uint4 pw = STATS ? make_uint4(0, 0, 0, 0) : ldg_stream(p4 + i);
       uint4 rw = make_uint4(0, 0, 0, 0);
       if (REF) rw = ldg_stream(r4 + i);
       unpack_any<T>(qw, qv);
-      if (sizeof(T) != 2) unpack_any<T>(pw, pv);  // (the bf16 path folds z_p packed)
+      if (sizeof(T) != 2 && !STATS) unpack_any<T>(pw, pv);  // (the bf16 path folds z_p packed)
       if (REF) unpack_any<T>(rw, rv);
 #pragma unroll
       for (int h = 0; h < E / 4; ++h) {
@@ -404,7 +407,9 @@ __global__ void __launch_bounds__(kRowThreads, 4) reward_sampled_rows(RewardRowA
       }
       draw_fold<T, E>(dq, kq, qv, pw, i * E);
       if (REF) draw_fold<T, E>(dr, kr, rv, pw, i * E);
-      if (sizeof(T) == 2) {
+      if (STATS) {
+        // (the normalisers are the loss forward's)
+      } else if (sizeof(T) == 2) {
         lse_fold_bf16(st.lp, pw, a.sT);
         lse_fold_bf16(st.lq, qw, a.sT);
         if (REF) lse_fold_bf16(st.lr, rw, a.sT);
@@ -416,8 +421,10 @@ __global__ void __launch_bounds__(kRowThreads, 4) reward_sampled_rows(RewardRowA
     }
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) {
-      st.lp = lse_merge(st.lp, shfl_lse(st.lp, off), a.sT);
-      st.lq = lse_merge(st.lq, shfl_lse(st.lq, off), a.sT);
+      if (!STATS) {
+        st.lp = lse_merge(st.lp, shfl_lse(st.lp, off), a.sT);
+        st.lq = lse_merge(st.lq, shfl_lse(st.lq, off), a.sT);
+      }
       if (REF) st.lr = lse_merge(st.lr, shfl_lse(st.lr, off), a.sT);
       dq = draw_merge(dq, shfl_draw(dq, off));
       if (REF) dr = draw_merge(dr, shfl_draw(dr, off));
@@ -432,18 +439,30 @@ __global__ void __launch_bounds__(kRowThreads, 4) reward_sampled_rows(RewardRowA
       RowState t = red[0];
       Draw bq = dred[0][0], br = dred[1][0];
       for (int w = 1; w < kRowWarps; ++w) {
-        t.lp = lse_merge(t.lp, red[w].lp, a.sT);
-        t.lq = lse_merge(t.lq, red[w].lq, a.sT);
+        if (!STATS) {
+          t.lp = lse_merge(t.lp, red[w].lp, a.sT);
+          t.lq = lse_merge(t.lq, red[w].lq, a.sT);
+        }
         if (REF) t.lr = lse_merge(t.lr, red[w].lr, a.sT);
         bq = draw_merge(bq, dred[0][w]);
         if (REF) br = draw_merge(br, dred[1][w]);
       }
       const float u = philox_uniform(a.seed, (uint64_t)n_glob, k_depth);
-      const float Lsp = lse_ls(t.lp), Lsq = lse_ls(t.lq);
-      const float d = log2_prob(bq.zp, a.sT, t.lp.M, Lsp) - log2_prob(bq.z, a.sT, t.lq.M, Lsq);
+      float d;
+      if (STATS) {
+        // the target's logit at the drawn token (an all -inf draft row draws none: index 0)
+        const int64_t y = (bq.i >= 0 && bq.i < a.V) ? bq.i : 0;
+        const float zpy = sizeof(T) == 2
+                              ? __uint_as_float((uint32_t)static_cast<const uint16_t*>(a.zp)[r * a.V + y] << 16)
+                              : static_cast<const float*>(a.zp)[r * a.V + y];
+        d = log2_prob(zpy, a.sT, a.lws.Mp[r], a.lws.Lsp[r]) - log2_prob(bq.z, a.sT, a.lws.Mq[r], a.lws.Lsq[r]);
+      } else {
+        const float Lsp = lse_ls(t.lp), Lsq = lse_ls(t.lq);
+        d = log2_prob(bq.zp, a.sT, t.lp.M, Lsp) - log2_prob(bq.z, a.sT, t.lq.M, Lsq);
+      }
       a.acc[r] = (u < exp2f(fminf(d, 0.f))) ? 1 : 0;
       if (REF) {
-        const float Lsr = lse_ls(t.lr);
+        const float Lsp = lse_ls(t.lp), Lsr = lse_ls(t.lr);
         const float dd = log2_prob(br.zp, a.sT, t.lp.M, Lsp) - log2_prob(br.z, a.sT, t.lr.M, Lsr);
         a.acc_ref[r] = (u < exp2f(fminf(dd, 0.f))) ? 1 : 0;
       }
@@ -452,17 +471,17 @@ __global__ void __launch_bounds__(kRowThreads, 4) reward_sampled_rows(RewardRowA
   }
 }
 
-template <typename T, bool REF>
+template <typename T, bool REF, bool STATS = false>
 cudaError_t go_sampled(const RewardRowArgs& a, cudaStream_t s) {
   int dev = 0, sms = 0, per_sm = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, reward_sampled_rows<T, REF>, kRowThreads, 0);
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, reward_sampled_rows<T, REF, STATS>, kRowThreads, 0);
   if (per_sm < 1) per_sm = 1;
   int64_t grid = (int64_t)sms * per_sm;
   if (grid > a.R) grid = a.R;
   if (grid < 1) return cudaSuccess;
-  reward_sampled_rows<T, REF><<<(unsigned)grid, kRowThreads, 0, s>>>(a);
+  reward_sampled_rows<T, REF, STATS><<<(unsigned)grid, kRowThreads, 0, s>>>(a);
   return cudaGetLastError();
 }
 
@@ -586,6 +605,10 @@ cudaError_t launch_reward_flags_from_stats(const RewardStatsArgs& a, cudaStream_
 
 cudaError_t launch_reward_rows(const RewardRowArgs& a, bool bf16, cudaStream_t s) {
   return bf16 ? dispatch<uint16_t>(a, s) : dispatch<float>(a, s);
+}
+
+cudaError_t launch_reward_sampled_stats(const RewardRowArgs& a, bool bf16, cudaStream_t s) {
+  return bf16 ? go_sampled<uint16_t, false, true>(a, s) : go_sampled<float, false, true>(a, s);
 }
 
 cudaError_t launch_reward_groups(const RewardGroupArgs& a, cudaStream_t s) {

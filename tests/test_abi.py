@@ -197,6 +197,30 @@ def test_reward_from_loss_argument_checks():
     assert call(_rprob(N=8, K=4, V=100, mode=aal.AAL_SAMPLING, temperature=1.0), lps) == aal.AAL_ERR_INVALID_ARG
     # the loss workspace must be large enough
     assert call(rp, lp, fake, lsize - 1) == aal.AAL_ERR_WORKSPACE
+    # a sampled draft needs the logits: the other entry point
+    assert call(_rprob(N=8, K=4, V=100, mode=aal.AAL_SAMPLING | aal.AAL_SAMPLED_DRAFT), lps) == aal.AAL_ERR_INVALID_ARG
+
+
+def test_sampled_reward_from_loss_argument_checks():
+    lib = aal.library()
+    SD = aal.AAL_SAMPLING | aal.AAL_SAMPLED_DRAFT
+    lp = _prob(N=8, K=4, V=104, mode=aal.AAL_BOTH, temperature=0.8)
+    code, lsize = _ws_size(lp)
+    rp = _rprob(N=8, K=4, V=104, mode=SD, temperature=0.8)
+    fake = 1 << 24
+    out = ctypes.c_size_t(0)
+    assert lib.aal_reward_workspace_size(ctypes.byref(rp), ctypes.byref(out)) == 0
+    rsize = out.value
+    call = lambda r, l, d=fake, t=fake, lb=lsize, rb=rsize: lib.aal_accept_reward_sampled_from_loss(
+        ctypes.byref(r), ctypes.byref(l), d, t, fake, lb, fake, rb, fake, fake, fake, None)
+    assert call(_rprob(N=8, K=4, V=104, mode=aal.AAL_SAMPLING, temperature=0.8), lp) == aal.AAL_ERR_INVALID_ARG
+    assert call(_rprob(N=8, K=4, V=100, mode=SD, temperature=0.8), lp) == aal.AAL_ERR_INVALID_ARG
+    assert call(rp, _prob(N=8, K=4, V=104, mode=aal.AAL_GREEDY, temperature=0.8)) == aal.AAL_ERR_INVALID_ARG
+    assert call(rp, _prob(N=8, K=4, V=104, mode=aal.AAL_BOTH, temperature=1.0)) == aal.AAL_ERR_INVALID_ARG
+    assert call(rp, lp, d=None) == aal.AAL_ERR_INVALID_ARG
+    assert call(rp, lp, t=fake + 8) == aal.AAL_ERR_INVALID_ARG
+    assert call(rp, lp, lb=lsize - 1) == aal.AAL_ERR_WORKSPACE
+    assert call(rp, lp, rb=rsize - 1) == aal.AAL_ERR_WORKSPACE
 
 
 def _sprob(**kw):

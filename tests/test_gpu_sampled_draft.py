@@ -98,3 +98,70 @@ def test_full_prompt_group_mean_is_the_wtv_expected_length():
     taus, _, amb = oracle_windows(target, draft, None, T, 21, 0, sel)
     keep = ~amb
     np.testing.assert_array_equal(got["tau"][sel][keep], taus[keep])
+
+
+# ------------------------------------------------------------------ from a loss forward's normalisers
+
+def run_sampled_from_loss(target, draft, T, seed, row_offset, wpr, rpg, clip=5.0, loss_mode=aal.AAL_BOTH):
+    """aal_loss_fwd at T, then aal_accept_reward_sampled_from_loss over the same logits."""
+    lprob = aal.loss_problem(draft, loss_mode, T, 0.5, 0.5)
+    lws = torch.empty(aal.aal_workspace_size(lprob), dtype=torch.uint8, device=DEV)
+    loss = torch.empty(1, device=DEV)
+    aal.aal_loss_fwd(lprob, draft, target, None, lws, loss)
+    rprob = aal.reward_problem(draft, MODE, T, clip, seed, row_offset, wpr, rpg)
+    rws = torch.empty(aal.aal_reward_workspace_size(rprob), dtype=torch.uint8, device=DEV)
+    N = draft.shape[0]
+    tau = torch.full((N,), -1, dtype=torch.int32, device=DEV)
+    rl = torch.full((N // wpr,), float("nan"), device=DEV)
+    adv = torch.full((N // wpr,), float("nan"), device=DEV)
+    aal.aal_accept_reward_sampled_from_loss(rprob, lprob, draft, target, lws, rws, tau, rl, adv)
+    torch.cuda.synchronize()
+    assert aal.aal_check_device_status(rws) == aal.AAL_OK
+    return dict(tau=tau.cpu().numpy(), rollout_len=rl.cpu().numpy(), advantage=adv.cpu().numpy())
+
+
+@pytest.mark.parametrize("T", [1.0, 0.7])
+@pytest.mark.parametrize("dtype,V", [(torch.float32, 1000), (torch.bfloat16, 4104), (torch.bfloat16, 7),
+                                     (torch.bfloat16, 40000)])
+def test_sampled_reward_from_loss_normalisers(T, dtype, V):
+    """The draft streamed alone, the acceptance from the loss forward's normalisers: tau equals the
+    oracle's and the logit pass's on every window whose decisions are not within rounding (V = 7
+    rows are not 16-byte multiples and take the reward's own pass)."""
+    wpr, rpg, groups, K = 2, 4, 2, 4
+    target, draft, _ = synth.make_reward_logits(0, seed=5, windows_per_rollout=wpr, rollouts_per_group=rpg * groups,
+                                                K=K, V=V, dtype=dtype)
+    draft[::2] = target[::2]
+    t, d = target.to(DEV), draft.to(DEV)
+    got = run_sampled_from_loss(t, d, T, seed=13, row_offset=700, wpr=wpr, rpg=rpg, clip=3.0)
+    logit = run_reward(t, d, None, MODE, T, seed=13, row_offset=700, wpr=wpr, rpg=rpg, clip=3.0)
+    N = t.shape[0]
+    taus, _, amb = oracle_windows(t, d, None, T, 13, 700, range(N))
+    keep = ~amb
+    assert keep.sum() >= N - 2
+    np.testing.assert_array_equal(got["tau"][keep], taus[keep])
+    np.testing.assert_array_equal(got["tau"][keep], logit["tau"][keep])
+    if keep.all():
+        np.testing.assert_allclose(got["advantage"], logit["advantage"], rtol=0, atol=1e-6)
+    assert got["tau"].max() >= 1
+
+
+def test_sampled_reward_from_loss_full_group():
+    """One reward group (4096 windows, K = 8, V = 128256 bf16) after the WTV forward: tau equals the
+    logit pass's on all but the windows a rounding can tip (at most 1%), and sampled windows
+    match the oracle exactly."""
+    target, draft, _ = synth.make_reward_logits(0, seed=0, device=DEV)
+    N = draft.shape[0]
+    T = 1.0
+    got = run_sampled_from_loss(target, draft, T, seed=21, row_offset=0, wpr=256, rpg=16,
+                                loss_mode=aal.AAL_SAMPLING)
+    logit = run_reward(target, draft, None, MODE, T, seed=21, row_offset=0, wpr=256, rpg=16)
+    differ = got["tau"] != logit["tau"]
+    assert differ.mean() <= 0.01, differ.mean()
+    sel = [0, 1, 2049, N - 1] + [int(i) for i in np.flatnonzero(differ)[:4]]
+    taus, _, amb = oracle_windows(target, draft, None, T, 21, 0, sel)
+    keep = ~amb
+    np.testing.assert_array_equal(got["tau"][sel][keep], taus[keep])
+    # a window where the two paths differ must be one the oracle calls ambiguous
+    for j, n in enumerate(sel):
+        if differ[n]:
+            assert amb[j], n
