@@ -33,6 +33,22 @@
 namespace aal {
 namespace {
 
+// An L2 prefetch of global memory (no shared-memory destination, nothing to wait on).
+__device__ __forceinline__ void bulk_prefetch_l2(const void* src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
+}
+
+// Chunks of the next row that the two-pass producer prefetches into L2 when it starts a row's
+// L2 pass: its ring slots then hold that pass's chunks, so without the prefetch the next row's
+// first HBM copies would be issued only a few chunks before they are needed.
+constexpr int kPrefetchChunks = 2;
+
+}  // namespace
+}  // namespace aal
+
+namespace aal {
+namespace {
+
 using namespace ptx;
 
 // ---------------------------------------------------------------- whole-chunk steps
@@ -403,6 +419,12 @@ __global__ void __launch_bounds__(kThreads2, kCtasPerSm) rowstats_twopass(RowSta
         const char* qrow = static_cast<const char*>(a.zq) + r * a.V * ES;
         for (int pass = 0; pass < 2 && !*abort_flag; ++pass) {
           const uint64_t pol = pass == 0 ? keep : drop;
+          if (pass == 1 && i + 1 < m) {  // the next row's first chunks, into L2
+            const int64_t rn = row(i + 1);
+            const uint32_t pb = (uint32_t)(min((int64_t)kPrefetchChunks * CH, (int64_t)V) * ES);
+            bulk_prefetch_l2(static_cast<const char*>(a.zp) + rn * a.V * ES, pb);
+            bulk_prefetch_l2(static_cast<const char*>(a.zq) + rn * a.V * ES, pb);
+          }
           for (int c = 0; c < nch; ++c) {
             if (!wait_phase(&S.empty[pos.slot], pos.phase ^ 1u, abort_flag, limit_ns, hdr)) break;
             const int e0 = c * CH;
