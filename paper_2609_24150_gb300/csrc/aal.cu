@@ -119,24 +119,30 @@ RowStatsArgs stats_args(const void* draft, const void* target, int64_t R, int64_
   return ra;
 }
 
+// The draft's statistics pass with x* as token ids (`target` holds them; takes the test hook's
+// chunk).
+Stream1Args ids_args(const void* draft, const void* target, int64_t R, int64_t V, const LossWs& ws) {
+  Stream1Args a;
+  a.z = draft;
+  a.R = R;
+  a.V = V;
+  a.lws = ws;
+  a.ids = static_cast<const int32_t*>(target);
+  a.acc = nullptr;
+  a.acc_ref = nullptr;
+  a.lpr = nullptr;
+  a.hdr = ws.hdr;
+  a.skip_chunk = debug_take_skip_chunk();
+  return a;
+}
+
 // Per-row statistics of R logit rows (pass over z_p and z_q, or over z_q alone when `target`
 // holds token ids), shared by both layouts.
 cudaError_t launch_stats(const void* draft, const void* target, int64_t R, int64_t V, int32_t dtype,
                          int32_t mode, float temperature, const LossWs& ws, cudaStream_t s, int* cluster) {
   if (mode & AAL_IDS) {
-    Stream1Args a;
-    a.z = draft;
-    a.R = R;
-    a.V = V;
-    a.lws = ws;
-    a.ids = static_cast<const int32_t*>(target);
-    a.acc = nullptr;
-    a.acc_ref = nullptr;
-    a.lpr = nullptr;
-    a.hdr = ws.hdr;
-    a.skip_chunk = debug_take_skip_chunk();
     *cluster = 1;
-    return launch_one_tensor(a, dtype == AAL_BF16, true, s);
+    return launch_one_tensor(ids_args(draft, target, R, V, ws), dtype == AAL_BF16, true, s);
   }
   *cluster = 1;
   return launch_rowstats(stats_args(draft, target, R, V, mode, temperature, ws), dtype == AAL_BF16, s, cluster);
@@ -232,6 +238,23 @@ SeqWindowArgs seq_window_args(const aal_seq_problem* prob, const uint8_t* mask, 
   wa.nvalid_g = prob->global_counts == 1 ? (int32_t)prob->n_windows_global : -1;
   wa.npos_g = prob->global_counts == 1 ? (int32_t)prob->n_positions_global : -1;
   return wa;
+}
+
+// The window flags and weights the fused kernels' sequence exchange reads (win.N and win.mask
+// are not used in the sequence layout).
+WindowArgs seq_fused_win(const SeqWindowArgs& wa, int64_t R) {
+  WindowArgs w{};
+  w.N = R;
+  w.K = wa.K;
+  w.greedy = wa.greedy;
+  w.sampling = wa.sampling;
+  w.kl = wa.kl;
+  w.tv = wa.tv;
+  w.w_greedy = wa.w_greedy;
+  w.w_sampling = wa.w_sampling;
+  w.w_kl = wa.w_kl;
+  w.w_tv = wa.w_tv;
+  return w;
 }
 
 }  // namespace
@@ -362,16 +385,7 @@ aal_status aal_loss_fwd_bwd(const aal_problem* prob, const void* draft, const vo
     f.win = window_args(prob, mask, 1, loss, eal, ws, L.nwblk);
     if (launch_count_valid(mask, prob->N, (int32_t)prob->K, f.win.nvalid_g, f.win.npos_g, ws.hdr, s) != cudaSuccess)
       return AAL_ERR_CUDA;
-    f.st.z = draft;
-    f.st.R = L.R;
-    f.st.V = prob->V;
-    f.st.lws = ws;
-    f.st.ids = static_cast<const int32_t*>(target);
-    f.st.acc = nullptr;
-    f.st.acc_ref = nullptr;
-    f.st.lpr = nullptr;
-    f.st.hdr = ws.hdr;
-    f.st.skip_chunk = debug_take_skip_chunk();
+    f.st = ids_args(draft, target, L.R, prob->V, ws);
     f.bw = grad_args(draft, target, mask, L.R, prob->V, prob->mode, prob->temperature, prob->w_greedy,
                      prob->w_kl, dloss, ws, grad_draft);
     f.groups = 0;
@@ -494,22 +508,10 @@ aal_status aal_seq_loss_fwd_bwd(const aal_seq_problem* prob, const void* draft, 
                                wa.npos_g, ws.hdr, s) != cudaSuccess)
       return AAL_ERR_CUDA;
     FusedIdsArgs f;
-    f.st.z = draft;
-    f.st.R = R;
-    f.st.V = prob->V;
-    f.st.lws = ws;
-    f.st.ids = static_cast<const int32_t*>(target);
-    f.st.acc = nullptr;
-    f.st.acc_ref = nullptr;
-    f.st.lpr = nullptr;
-    f.st.hdr = ws.hdr;
-    f.st.skip_chunk = debug_take_skip_chunk();
+    f.st = ids_args(draft, target, R, prob->V, ws);
     f.bw = grad_args(draft, target, mask, R, prob->V, prob->mode, prob->temperature, prob->w_greedy, prob->w_kl,
                      dloss, ws, grad_draft);
-    f.win = WindowArgs{};
-    f.win.N = R;
-    f.win.K = (int32_t)prob->K;
-    f.win.greedy = wa.greedy;
+    f.win = seq_fused_win(wa, R);
     f.groups = 0;
     f.solos = 0;
     f.n_group = 0;
@@ -534,18 +536,7 @@ aal_status aal_seq_loss_fwd_bwd(const aal_seq_problem* prob, const void* draft, 
     f.st = stats_args(draft, target, R, prob->V, prob->mode, prob->temperature, ws);
     f.bw = grad_args(draft, target, mask, R, prob->V, prob->mode, prob->temperature, prob->w_greedy, prob->w_kl,
                      dloss, ws, grad_draft);
-    // the window flags and weights the exchange reads (win.N and win.mask are not used here)
-    f.win = WindowArgs{};
-    f.win.N = R;
-    f.win.K = (int32_t)prob->K;
-    f.win.greedy = wa.greedy;
-    f.win.sampling = wa.sampling;
-    f.win.kl = wa.kl;
-    f.win.tv = wa.tv;
-    f.win.w_greedy = wa.w_greedy;
-    f.win.w_sampling = wa.w_sampling;
-    f.win.w_kl = wa.w_kl;
-    f.win.w_tv = wa.w_tv;
+    f.win = seq_fused_win(wa, R);
     f.groups = 0;
     f.solos = 0;
     f.n_group = 0;
