@@ -87,6 +87,8 @@ CASES = [
     (4, 3, 7, 4104, B, 1.0, 0.5, 0.5, 1.0, 1.0, False, False),      # sequences shorter than the window
     (40, 5, 6, 256, B, 1.0, 0.5, 0.5, 1.0, 1.0, True, False),       # many short sequences, several rounds
     (30, 20, 3, 8, B, 1.0, 0.5, 0.5, 1.0, 1.0, True, False),        # one 16-byte vector a row
+    (1, 3, 7, 4104, B, 1.0, 0.5, 0.5, 1.0, 1.0, False, False),      # fewer rows than the window (one round)
+    (64, 1, 8, 2000, B, 1.0, 0.5, 0.5, 1.0, 1.0, True, False),      # sequences of one position
 ]
 
 
